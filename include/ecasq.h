@@ -1,0 +1,180 @@
+/*
+ * ecasq.h -- C ABI of the GB300 ECASQ library (Entropy-Constrained Adaptive
+ * Stochastic Quantization, arxiv 2608.18147).
+ *
+ * Given x in R^d, a cap s on the codebook size and an entropy budget b
+ * (bits per entry), ECASQ picks Q subset of X, |Q| <= s, spanning X, that
+ * minimises the stochastic-quantization MSE subject to H(Xhat) <= b
+ * (Sec. 1, "ECASQ solves ...").  The library implements the approximate
+ * dynamic program of Sec. 5 (surrogate entropy H(I,B)), the multiplier search
+ * of Sec. 3 / Sec. 5, the three-colour refinement of Sec. 6 and the unbiased
+ * stochastic rounding of Sec. 2, on one GPU.
+ *
+ * Conventions shared by every entry point:
+ *   - Pointers are DEVICE pointers unless the comment says "host".  The
+ *     caller owns every buffer; the library never allocates device memory:
+ *     all scratch comes from the caller's workspace (see ecasq_workspace_size).
+ *     The workspace start must be 256-byte aligned.
+ *   - Calls are ordered on `stream` (a cudaStream_t; NULL = legacy default).
+ *     Entry points that return host results synchronise `stream` before
+ *     returning.  Concurrent calls that share one workspace race.
+ *   - x is fp32, length d >= 1, all finite (NaN/Inf -> ECASQ_ENONFINITE).
+ *     -0.0 and +0.0 are the same value.  d < 2^31.
+ *   - Q is an ascending fp32 codebook of m values, m <= s <= 256; Q[0] = min x
+ *     and Q[m-1] = max x (Q spans X, Sec. 1).  m < s is allowed ("at most s",
+ *     eq. apx_final).
+ *   - lambda is on the vNMSE scale; the DP uses lambda' = lambda * ||X||^2
+ *     (Sec. 3: vNMSE + lambda H  equals  MSE + lambda' H).
+ *   - Return value: ECASQ_OK (0) or a negative status; ecasq_strerror names it.
+ */
+#ifndef ECASQ_H
+#define ECASQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st *ecasq_stream_t; /* same type as cudaStream_t */
+
+#define ECASQ_OK 0
+#define ECASQ_EINVAL (-1)      /* bad argument (d < 1, s outside [2,256], b < 0, null pointer, ...) */
+#define ECASQ_ENONFINITE (-2)  /* x holds NaN or Inf */
+#define ECASQ_EINFEASIBLE (-3) /* no evaluated multiplier meets the budget (result = largest multiplier's solution) */
+#define ECASQ_EWORKSPACE (-4)  /* workspace smaller than ecasq_workspace_size() or misaligned */
+#define ECASQ_ECUDA (-5)       /* a CUDA call failed (launch error, fault) */
+#define ECASQ_ETIMEOUT (-6)    /* a bounded device-side wait ran out */
+#define ECASQ_ERANGE (-7)      /* an entry of x lies outside [Q[0], Q[m-1]], or Q is not a subset of X */
+
+/* flags */
+#define ECASQ_EXACT_S 1u          /* use exactly s values (eq. apx_final with i = s only) */
+#define ECASQ_NO_REFINE_GUARD 2u  /* refinement may raise H(Xhat) above the budget */
+#define ECASQ_DP_REFERENCE 4u     /* run the fp64 reference DP kernel instead of the fast kernel */
+
+typedef struct ecasq_params {
+    int32_t s;                 /* codebook cap, 2..256 */
+    uint32_t flags;            /* ECASQ_* flags */
+    double budget_bits;        /* b >= 0, bits per entry, compared with H(I,B) (Sec. 5) */
+    double lambda;             /* < 0: search on the budget; >= 0: one fixed multiplier (vNMSE scale) */
+    double lambda_lo;          /* search bracket (vNMSE scale); <= 0 selects 1e-8 */
+    double lambda_hi;          /* <= 0 selects 1e3 */
+    int32_t search_rounds;     /* rounds of 7 geometric midpoints; <= 0 selects 6 */
+    int32_t refine_max_rounds; /* three-colour refinement rounds (Sec. 6); 0 = none */
+    double refine_rel_tol;     /* stop once a round lowers J by <= tol*|J| (0: by nothing) */
+} ecasq_params_t;
+
+typedef struct ecasq_result {
+    int32_t status;            /* same as the return value */
+    int32_t m;                 /* |Q| */
+    int32_t passes;            /* DP launches (each covers up to 8 multipliers) */
+    int32_t lambdas_evaluated; /* multipliers evaluated by the search */
+    int32_t refine_rounds;     /* refinement rounds executed */
+    int32_t reserved;
+    int64_t d, p;              /* entries, unique values */
+    double lambda;             /* selected multiplier (vNMSE scale) */
+    double lambda_prime;       /* lambda * ||X||^2 */
+    double norm2;              /* ||X||^2 */
+    double mse;                /* MSE(Q, X) = sum (b_x - x)(x - a_x)          (Sec. 2) */
+    double vnmse;              /* mse / ||X||^2                               (Sec. 2) */
+    double h_surrogate;        /* H(I,B), eq. apx_additive_entropy             (Sec. 5) */
+    double h_exact;            /* H(Xhat)                                     (Sec. 3) */
+    double r_tot;              /* H(Xhat) + 32 m / d                          (Sec. 3, 8) */
+    double objective;          /* mse + lambda' * h_exact after refinement, else mse + lambda' * h_surrogate */
+    int64_t candidates;        /* min-plus candidates evaluated by the DP (all passes) */
+    int64_t rescored;          /* candidates re-scored in fp64 by the fast DP's exact stage */
+} ecasq_result_t;
+
+/* Bytes of workspace needed by every entry point below for vectors of up to d
+ * entries, codebook cap s, and `rows` independent rows (1 for single-vector
+ * calls).  Returns 0 for invalid arguments. */
+size_t ecasq_workspace_size(int64_t d, int32_t s, int64_t rows);
+
+/* Budgeted (or fixed-multiplier) solve of one vector.
+ * Pipeline: sort, weighted histogram and prefix sums (Sec. 2, App. E) ->
+ * approximate DP (Sec. 5, eqs. apx_base, apx_rec, apx_final) over a multiplier
+ * search (Sec. 3, Sec. 5: keep the lowest-MSE solution with H(I,B) <= b) ->
+ * optional three-colour refinement (Sec. 6) at the selected multiplier.
+ *   x   [d] device, input (not modified)
+ *   Q   [s] device, output: Q[0..m-1] ascending, the rest untouched
+ *   res host, output (may be NULL)
+ * Search schedule: multiplier 0 first (if feasible it is the answer); else
+ * rounds of the 7 geometric midpoints of [lo, hi] (sqrt only), the bracket
+ * shrinking to the pair around the smallest feasible midpoint; if nothing is
+ * feasible, hi itself; ECASQ_EINFEASIBLE when that fails too (Q then holds
+ * the solution at hi).  Synchronises `stream`. */
+int ecasq_solve(const float *x, int64_t d, const ecasq_params_t *prm, void *ws, size_t ws_bytes,
+                float *Q, ecasq_result_t *res, ecasq_stream_t stream);
+
+/* One DP pass (Sec. 5) at G <= 8 fixed multipliers, the unit of the search.
+ *   lambdas   host [G], vNMSE scale, >= 0
+ *   Q_out     device [G * s] (row g: codebook of multiplier g, m_out[g] values)
+ *   m_out     host [G]
+ *   metrics   host [G * 4]: DP optimum (eq. apx_final), MSE, H(I,B), H(Xhat)
+ * The DP tables stay in the workspace until the next call (ecasq_dp_tables).
+ * Synchronises `stream`. */
+int ecasq_dp_pass(const float *x, int64_t d, int32_t s, const double *lambdas, int32_t G, uint32_t flags,
+                  void *ws, size_t ws_bytes, float *Q_out, int32_t *m_out, double *metrics,
+                  ecasq_stream_t stream);
+
+/* Copy the DP tables of multiplier g of the last ecasq_dp_pass on this
+ * workspace: dp (fp64) and bp (int32, lowest argmin k; -1 where undefined),
+ * each row-major [(s+1) x p], rows 0 and 1 unused, +inf / -1 where the layer
+ * is undefined.  dp_out, bp_out device; p_out host.  Synchronises `stream`. */
+int ecasq_dp_tables(void *ws, size_t ws_bytes, int32_t g, double *dp_out, int32_t *bp_out, int64_t *p_out,
+                    ecasq_stream_t stream);
+
+/* Three-colour refinement (Sec. 6) of a codebook Q subset of X at a fixed
+ * multiplier, minimising MSE + lambda' H(Xhat): colours 0, 1, 2 in turn move
+ * each interior value with index % 3 == colour to the best unique input value
+ * strictly between its neighbours (ties keep the value, else the lowest);
+ * with a budget (budget_bits >= 0 and no ECASQ_NO_REFINE_GUARD flag) a colour
+ * step that lifts H(Xhat) above the budget is undone; stop after a round that
+ * lowers J by <= rel_tol*|J| or after max_rounds.
+ *   Q  device [m], in/out.  res host (may be NULL).  Synchronises `stream`. */
+int ecasq_refine(const float *x, int64_t d, float *Q, int32_t m, double lambda, double budget_bits,
+                 int32_t max_rounds, double rel_tol, uint32_t flags, void *ws, size_t ws_bytes,
+                 ecasq_result_t *res, ecasq_stream_t stream);
+
+/* MSE, H(I,B) and H(Xhat) of a codebook Q subset of X (Sec. 2, Sec. 3,
+ * eq. apx_additive_entropy).  out host [3].  Synchronises `stream`. */
+int ecasq_evaluate(const float *x, int64_t d, const float *Q, int32_t m, void *ws, size_t ws_bytes,
+                   double *out, ecasq_stream_t stream);
+
+/* Unbiased stochastic quantization (Sec. 2) of x in its original order:
+ * a = max{q <= x}; an entry equal to a gets a's index, otherwise it is
+ * rounded up to the next value iff fl32(fl32(k 2^-24) fl32(b - a)) <
+ * fl32(x - a), k = top 24 bits of SplitMix64(seed + (i+1) 0x9E3779B97F4A7C15)
+ * (Steele, Lea and Flood 2014) for entry i; so E[xhat] = x up to 2^-23 (b-a).
+ *   idx     device [d] uint8 output
+ *   counts  device [m] uint32 output: index histogram
+ *   h_emp   host, output (may be NULL): empirical entropy of idx (Sec. 1)
+ * ECASQ_ERANGE if an entry lies outside [Q[0], Q[m-1]].  Synchronises
+ * `stream` only when h_emp is not NULL. */
+int ecasq_quantize(const float *x, int64_t d, const float *Q, int32_t m, uint64_t seed, uint8_t *idx,
+                   uint32_t *counts, void *ws, size_t ws_bytes, double *h_emp, ecasq_stream_t stream);
+
+/* Budgeted solves of `rows` independent rows of length d (row-major X),
+ * each exactly as ecasq_solve would do it on that row alone (same schedule,
+ * same results).  Q [rows * s] device, m_out [rows] device, res host [rows]
+ * (may be NULL).  Synchronises `stream`. */
+int ecasq_solve_batched(const float *X, int64_t rows, int64_t d, const ecasq_params_t *prm, void *ws,
+                        size_t ws_bytes, float *Q, int32_t *m_out, ecasq_result_t *res,
+                        ecasq_stream_t stream);
+
+/* Weighted histogram and App. E prefix sums of x (step 1 of every solve):
+ *   v [p] fp32 unique values ascending, w [p] int64 multiplicities,
+ *   N [p+1] int64, S and S2 [2*(p+1)] fp64 as (hi[0..p], lo[0..p]) with
+ *   N[t] = sum_{r<t} w_r, S[t] = sum w_r v_r, S2[t] = sum w_r v_r^2.
+ *   All device, sized for p = d; p_out host.  Synchronises `stream`. */
+int ecasq_prepare(const float *x, int64_t d, void *ws, size_t ws_bytes, float *v, int64_t *w, int64_t *N,
+                  double *S, double *S2, int64_t *p_out, ecasq_stream_t stream);
+
+const char *ecasq_strerror(int status);
+int ecasq_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ECASQ_H */

@@ -1,0 +1,16 @@
+"""GB300-native ECASQ: the approximate-DP hot path of Entropy-Constrained
+Adaptive Stochastic Quantization (arxiv 2608.18147) as hand-written CUDA for
+sm_103a behind a C ABI (include/ecasq.h), with this thin Python binding.
+
+The binding functions carry the C entry points' names (ecasq_solve,
+ecasq_dp_pass, ecasq_refine, ecasq_quantize, ecasq_solve_batched, ...).
+There is no CPU fallback: without libecasq.so and a GPU every call raises.
+"""
+from . import workloads
+from .native import (DP_REFERENCE, EXACT_S, NO_REFINE_GUARD, EcasqError, ecasq_dp_pass, ecasq_dp_tables,
+                     ecasq_evaluate, ecasq_prepare, ecasq_quantize, ecasq_refine, ecasq_solve, ecasq_solve_batched,
+                     ecasq_workspace_size, lib, workspace)
+
+__all__ = ["workloads", "ecasq_solve", "ecasq_dp_pass", "ecasq_dp_tables", "ecasq_refine", "ecasq_evaluate",
+           "ecasq_quantize", "ecasq_solve_batched", "ecasq_prepare", "ecasq_workspace_size", "workspace", "lib",
+           "EcasqError", "EXACT_S", "NO_REFINE_GUARD", "DP_REFERENCE"]

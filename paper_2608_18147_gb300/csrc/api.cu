@@ -1,0 +1,615 @@
+// api.cu -- the extern "C" entry points of include/ecasq.h and the host-side
+// drivers: workspace carving, the multiplier search, the refinement loop.
+#include <math.h>
+#include <string.h>
+
+#include <algorithm>
+#include <vector>
+
+#include "common.cuh"
+
+namespace ecasq {
+
+// launchers defined in the other translation units
+int launch_dp_reference(const Prefix &P, const double *lamp, int G, int s, double *dp64, int32_t *bp,
+                        cudaStream_t st);
+int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, const Layout &L, cudaStream_t st);
+int launch_traceback_eval(const Prefix &P, int G, int s, int exact_s, const double *dp64, const int32_t *bp,
+                          int32_t *qidx, int32_t *mcount, double *metrics, cudaStream_t st);
+int launch_eval_codebook(const Prefix &P, const int32_t *a, int m, double *out3, cudaStream_t st);
+int launch_gather_q(const float *v, const int32_t *qidx, const int32_t *mcount, int G, int s, float *Q,
+                    cudaStream_t st);
+int launch_locate_q(const float *v, int64_t p, const float *Q, int m, int32_t *a, DevStatus *ds, cudaStream_t st);
+int launch_refine_colour(const Prefix &P, const int32_t *a, int m, int colour, double lamp, int32_t *a_new,
+                         int32_t *moved, cudaStream_t st, int *nblocks_out);
+int launch_quantize(const float *x, int64_t d, const float *Q, int m, uint64_t seed, uint8_t *idx, uint32_t *counts,
+                    DevStatus *st, int num_sms, cudaStream_t stream);
+size_t fast_dp_band_bytes(int64_t d, int32_t s);
+
+size_t make_layout(int64_t d, int32_t s, int64_t rows, Layout *L) {
+    (void)rows;
+    size_t off = 0;
+    auto take = [&](size_t bytes) { size_t o = off; off += align256(bytes); return o; };
+    int64_t nb = cdiv(d, kSortTile), nbs = cdiv(d, kScanTile);
+    size_t rowsz = (size_t)kMaxG * (size_t)(s + 1) * (size_t)d;
+    L->status = take(sizeof(DevStatus));
+    L->keys0 = take(4 * (size_t)d);
+    L->keys1 = take(4 * (size_t)d);
+    L->rcount = take(4 * 256 * (size_t)nb);
+    L->head = 0;
+    L->v = take(4 * (size_t)d);
+    L->w = take(8 * (size_t)d);
+    L->N = take(8 * (size_t)(d + 1));
+    L->S = take(16 * (size_t)(d + 1));
+    L->S2 = take(16 * (size_t)(d + 1));
+    L->part = take(48 * (size_t)nbs);
+    L->dp64 = take(8 * std::max(rowsz, (size_t)4 * (size_t)(d + 1)));
+    L->bp = take(4 * rowsz);
+    L->dp32 = take(4 * rowsz);
+    L->qidx = take(4 * (size_t)kMaxG * kMaxS);
+    L->mcount = take(4 * (size_t)kMaxG);
+    L->metrics = take(8 * (size_t)kMaxG * 4);
+    L->lam = take(8 * (size_t)kMaxG);
+    L->refine = take(4 * 2 * kMaxS + 256 + 8 * 8);
+    L->band = take(fast_dp_band_bytes(d, s));
+    L->total = off;
+    L->d = d;
+    L->s = s;
+    return off;
+}
+
+static int g_num_sms = 0;
+static int num_sms() {
+    if (g_num_sms == 0) {
+        int dev = 0, n = 0;
+        if (cudaGetDevice(&dev) == cudaSuccess && cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess)
+            g_num_sms = n;
+        else
+            g_num_sms = 152;
+    }
+    return g_num_sms;
+}
+
+static int check_ws(const void *ws, size_t bytes, const Layout &L) {
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255) != 0 || bytes < L.total) return ECASQ_EWORKSPACE;
+    return ECASQ_OK;
+}
+
+static Prefix make_prefix(void *ws, const Layout &L, int64_t p, int64_t d) {
+    Prefix P;
+    P.v = wsp<float>(ws, L.v);
+    P.w = wsp<int64_t>(ws, L.w);
+    P.N = wsp<int64_t>(ws, L.N);
+    P.S = wsp<double>(ws, L.S);
+    P.S2 = wsp<double>(ws, L.S2);
+    P.p = p;
+    P.d = d;
+    return P;
+}
+
+// The 7 interior points of [lo, hi] from three levels of geometric midpoints
+// sqrt(a*b): correctly rounded multiply and sqrt only.
+static void midpoints7(double lo, double hi, double *t) {
+    t[3] = sqrt(lo * hi);
+    t[1] = sqrt(lo * t[3]);
+    t[5] = sqrt(t[3] * hi);
+    t[0] = sqrt(lo * t[1]);
+    t[2] = sqrt(t[1] * t[3]);
+    t[4] = sqrt(t[3] * t[5]);
+    t[6] = sqrt(t[5] * hi);
+}
+
+struct PassOut {
+    std::vector<int32_t> qidx;  // G * s
+    std::vector<int32_t> m;     // G
+    std::vector<double> met;    // G * 4
+};
+
+// One DP pass over a prepared workspace: DP at lambda'_g (g < G), traceback,
+// evaluation, results to the host.
+static int dp_pass_prepared(void *ws, const Layout &L, const Prefix &P, int s, const double *lamp, int G,
+                            uint32_t flags, cudaStream_t st, PassOut &out) {
+    double *dp64 = wsp<double>(ws, L.dp64);
+    int32_t *bp = wsp<int32_t>(ws, L.bp);
+    int rc;
+    if (flags & ECASQ_DP_REFERENCE)
+        rc = launch_dp_reference(P, lamp, G, s, dp64, bp, st);
+    else
+        rc = launch_dp_fast(P, lamp, G, s, ws, L, st);
+    if (rc != ECASQ_OK) return rc;
+    rc = launch_traceback_eval(P, G, s, (flags & ECASQ_EXACT_S) ? 1 : 0, dp64, bp, wsp<int32_t>(ws, L.qidx),
+                               wsp<int32_t>(ws, L.mcount), wsp<double>(ws, L.metrics), st);
+    if (rc != ECASQ_OK) return rc;
+    out.qidx.assign((size_t)G * s, 0);
+    out.m.assign(G, 0);
+    out.met.assign((size_t)G * 4, 0.0);
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(out.qidx.data(), wsp<int32_t>(ws, L.qidx), sizeof(int32_t) * G * s,
+                                   cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(out.m.data(), wsp<int32_t>(ws, L.mcount), sizeof(int32_t) * G,
+                                   cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(out.met.data(), wsp<double>(ws, L.metrics), sizeof(double) * G * 4,
+                                   cudaMemcpyDeviceToHost, st));
+    int32_t sg[2] = {s, G};
+    int64_t dd_ = L.d;
+    DevStatus *ds = wsp<DevStatus>(ws, L.status);
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(&ds->last_s, sg, sizeof(sg), cudaMemcpyHostToDevice, st));
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(&ds->last_d, &dd_, sizeof(dd_), cudaMemcpyHostToDevice, st));
+    DevStatus h;
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(&h, ds, sizeof(DevStatus), cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    if (h.timeout) return ECASQ_ETIMEOUT;
+    for (int g = 0; g < G; g++)
+        if (out.m[g] < 1) return ECASQ_EINFEASIBLE;
+    return ECASQ_OK;
+}
+
+static int64_t candidates_of(int64_t p, int s, int exact) {
+    (void)exact;
+    // eq. apx_rec evaluates, for layers i = 3..s, every k in [i-2, j-1], j in [i-1, p-1]
+    int64_t c = 0;
+    for (int i = 3; i <= s; i++) {
+        int64_t n = p - (i - 1);  // number of j
+        if (n <= 0) break;
+        c += n * (n + 1) / 2;
+    }
+    return c;
+}
+
+// Upload a codebook (unique indices) and evaluate it: out3 = MSE, H(I,B), H(Xhat).
+static int eval_device(void *ws, const Layout &L, const Prefix &P, const int32_t *a_dev, int m, cudaStream_t st,
+                       double *out3_host) {
+    double *o = reinterpret_cast<double *>(wsp<char>(ws, L.refine) + 4 * 2 * kMaxS + 256);
+    int rc = launch_eval_codebook(P, a_dev, m, o, st);
+    if (rc != ECASQ_OK) return rc;
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(out3_host, o, 3 * sizeof(double), cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    return ECASQ_OK;
+}
+
+// Three-colour refinement loop (Sec. 6) on the host; a_host in/out.
+static int refine_device(void *ws, const Layout &L, const Prefix &P, std::vector<int32_t> &a_host, double lamp,
+                         double budget, bool guard, int max_rounds, double tol, cudaStream_t st, int *rounds_used) {
+    int m = (int)a_host.size();
+    *rounds_used = 0;
+    if (m < 3 || max_rounds <= 0) return ECASQ_OK;
+    int32_t *a = wsp<int32_t>(ws, L.refine);
+    int32_t *an = a + kMaxS;
+    int32_t *moved = an + kMaxS;
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(a, a_host.data(), sizeof(int32_t) * m, cudaMemcpyHostToDevice, st));
+    double ev[3];
+    int rc = eval_device(ws, L, P, a, m, st, ev);
+    if (rc != ECASQ_OK) return rc;
+    double J = ev[0] + lamp * ev[2];
+    for (int r = 0; r < max_rounds; r++) {
+        double J0 = J;
+        for (int col = 0; col < 3; col++) {
+            ECASQ_CUDA_TRY(cudaMemcpyAsync(an, a, sizeof(int32_t) * m, cudaMemcpyDeviceToDevice, st));
+            ECASQ_CUDA_TRY(cudaMemsetAsync(moved, 0, sizeof(int32_t), st));
+            int nblk = 0;
+            rc = launch_refine_colour(P, a, m, col, lamp, an, moved, st, &nblk);
+            if (rc != ECASQ_OK) return rc;
+            if (nblk == 0) continue;
+            int32_t mv = 0;
+            ECASQ_CUDA_TRY(cudaMemcpyAsync(&mv, moved, sizeof(int32_t), cudaMemcpyDeviceToHost, st));
+            rc = eval_device(ws, L, P, an, m, st, ev);
+            if (rc != ECASQ_OK) return rc;
+            if (!mv) continue;
+            if (guard && ev[2] > budget) continue;
+            ECASQ_CUDA_TRY(cudaMemcpyAsync(a, an, sizeof(int32_t) * m, cudaMemcpyDeviceToDevice, st));
+        }
+        rc = eval_device(ws, L, P, a, m, st, ev);
+        if (rc != ECASQ_OK) return rc;
+        J = ev[0] + lamp * ev[2];
+        *rounds_used = r + 1;
+        if (!(J0 - J > tol * fabs(J0))) break;
+    }
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(a_host.data(), a, sizeof(int32_t) * m, cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    return ECASQ_OK;
+}
+
+static int write_codebook(void *ws, const Layout &L, const std::vector<int32_t> &a, float *Q, cudaStream_t st) {
+    int32_t *qi = wsp<int32_t>(ws, L.qidx);
+    int32_t *mc = wsp<int32_t>(ws, L.mcount);
+    int32_t m = (int32_t)a.size();
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(qi, a.data(), sizeof(int32_t) * m, cudaMemcpyHostToDevice, st));
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(mc, &m, sizeof(int32_t), cudaMemcpyHostToDevice, st));
+    int rc = launch_gather_q(wsp<float>(ws, L.v), qi, mc, 1, kMaxS, Q, st);
+    if (rc != ECASQ_OK) return rc;
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    return ECASQ_OK;
+}
+
+static bool params_ok(const ecasq_params_t *prm) {
+    if (!prm) return false;
+    if (prm->s < 2 || prm->s > kMaxS) return false;
+    if (prm->lambda < 0.0 && !(prm->budget_bits >= 0.0)) return false;
+    if (prm->lambda >= 0.0 && !isfinite(prm->lambda)) return false;
+    if (prm->refine_max_rounds < 0) return false;
+    return true;
+}
+
+struct Eval { double lam, mse, hs, hx; int m; bool feas; std::vector<int32_t> a; };
+
+}  // namespace ecasq
+
+using namespace ecasq;
+
+extern "C" {
+
+int ecasq_version(void) { return 10000; }
+
+const char *ecasq_strerror(int status) {
+    switch (status) {
+        case ECASQ_OK: return "ok";
+        case ECASQ_EINVAL: return "invalid argument";
+        case ECASQ_ENONFINITE: return "input holds NaN or Inf";
+        case ECASQ_EINFEASIBLE: return "entropy budget infeasible for the evaluated multipliers";
+        case ECASQ_EWORKSPACE: return "workspace too small or not 256-byte aligned";
+        case ECASQ_ECUDA: return "CUDA error";
+        case ECASQ_ETIMEOUT: return "bounded device wait timed out";
+        case ECASQ_ERANGE: return "value outside the codebook range, or codebook value not in x";
+        default: return "unknown status";
+    }
+}
+
+size_t ecasq_workspace_size(int64_t d, int32_t s, int64_t rows) {
+    if (d < 1 || d >= ((int64_t)1 << 31) || s < 2 || s > kMaxS || rows < 1) return 0;
+    Layout L;
+    return make_layout(d, s, rows, &L);
+}
+
+int ecasq_prepare(const float *x, int64_t d, void *ws, size_t ws_bytes, float *v, int64_t *w, int64_t *N,
+                  double *S, double *S2, int64_t *p_out, ecasq_stream_t stream) {
+    if (!x || d < 1 || d >= ((int64_t)1 << 31) || !v || !w || !N || !S || !S2 || !p_out) return ECASQ_EINVAL;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    Layout L;
+    make_layout(d, 2, 1, &L);
+    int rc = check_ws(ws, ws_bytes, L);
+    if (rc) return rc;
+    int64_t p;
+    double n2;
+    rc = prepare_device(x, d, ws, L, st, &p, &n2);
+    if (rc) return rc;
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(v, wsp<float>(ws, L.v), 4 * p, cudaMemcpyDeviceToDevice, st));
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(w, wsp<int64_t>(ws, L.w), 8 * p, cudaMemcpyDeviceToDevice, st));
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(N, wsp<int64_t>(ws, L.N), 8 * (p + 1), cudaMemcpyDeviceToDevice, st));
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(S, wsp<double>(ws, L.S), 16 * (p + 1), cudaMemcpyDeviceToDevice, st));
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(S2, wsp<double>(ws, L.S2), 16 * (p + 1), cudaMemcpyDeviceToDevice, st));
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    *p_out = p;
+    return ECASQ_OK;
+}
+
+int ecasq_dp_pass(const float *x, int64_t d, int32_t s, const double *lambdas, int32_t G, uint32_t flags, void *ws,
+                  size_t ws_bytes, float *Q_out, int32_t *m_out, double *metrics, ecasq_stream_t stream) {
+    if (!x || d < 1 || d >= ((int64_t)1 << 31) || s < 2 || s > kMaxS || !lambdas || G < 1 || G > kMaxG || !Q_out ||
+        !m_out || !metrics)
+        return ECASQ_EINVAL;
+    for (int g = 0; g < G; g++)
+        if (!(lambdas[g] >= 0.0) || !isfinite(lambdas[g])) return ECASQ_EINVAL;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    Layout L;
+    make_layout(d, s, 1, &L);
+    int rc = check_ws(ws, ws_bytes, L);
+    if (rc) return rc;
+    int64_t p;
+    double n2;
+    rc = prepare_device(x, d, ws, L, st, &p, &n2);
+    if (rc) return rc;
+    Prefix P = make_prefix(ws, L, p, d);
+    if (p == 1) {
+        for (int g = 0; g < G; g++) {
+            ECASQ_CUDA_TRY(cudaMemcpyAsync(Q_out + (size_t)g * s, P.v, 4, cudaMemcpyDeviceToDevice, st));
+            m_out[g] = 1;
+            for (int t = 0; t < 4; t++) metrics[4 * g + t] = 0.0;
+        }
+        ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+        return ECASQ_OK;
+    }
+    double lamp[kMaxG];
+    for (int g = 0; g < G; g++) lamp[g] = lambdas[g] * n2;
+    PassOut po;
+    rc = dp_pass_prepared(ws, L, P, s, lamp, G, flags, st, po);
+    if (rc) return rc;
+    rc = launch_gather_q(P.v, wsp<int32_t>(ws, L.qidx), wsp<int32_t>(ws, L.mcount), G, s, Q_out, st);
+    if (rc) return rc;
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    for (int g = 0; g < G; g++) {
+        m_out[g] = po.m[g];
+        for (int t = 0; t < 4; t++) metrics[4 * g + t] = po.met[4 * g + t];
+    }
+    return ECASQ_OK;
+}
+
+int ecasq_dp_tables(void *ws, size_t ws_bytes, int32_t g, double *dp_out, int32_t *bp_out, int64_t *p_out,
+                    ecasq_stream_t stream) {
+    if (!ws || !dp_out || !bp_out || !p_out || g < 0 || g >= kMaxG) return ECASQ_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(ws) & 255) != 0 || ws_bytes < sizeof(DevStatus)) return ECASQ_EWORKSPACE;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    DevStatus h;
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(&h, ws, sizeof(DevStatus), cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    if (h.last_s < 2 || g >= h.last_G || h.p < 2 || h.last_d < 1) return ECASQ_EINVAL;
+    Layout L;
+    make_layout(h.last_d, h.last_s, 1, &L);
+    int rc = check_ws(ws, ws_bytes, L);
+    if (rc) return rc;
+    size_t n = (size_t)(h.last_s + 1) * (size_t)h.p;
+    size_t off = (size_t)g * n;
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(dp_out, wsp<double>(ws, L.dp64) + off, 8 * n, cudaMemcpyDeviceToDevice, st));
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(bp_out, wsp<int32_t>(ws, L.bp) + off, 4 * n, cudaMemcpyDeviceToDevice, st));
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    *p_out = h.p;
+    return ECASQ_OK;
+}
+
+static void fill_result(ecasq_result_t *res, int status, int m, int64_t d, int64_t p, double lam, double n2,
+                        const double *ev, double objective, int passes, int nlam, int rr, int64_t cand,
+                        int64_t rescored) {
+    if (!res) return;
+    memset(res, 0, sizeof(*res));
+    res->status = status;
+    res->m = m;
+    res->passes = passes;
+    res->lambdas_evaluated = nlam;
+    res->refine_rounds = rr;
+    res->d = d;
+    res->p = p;
+    res->lambda = lam;
+    res->lambda_prime = lam * n2;
+    res->norm2 = n2;
+    res->mse = ev[0];
+    res->vnmse = n2 > 0.0 ? ev[0] / n2 : 0.0;
+    res->h_surrogate = ev[1];
+    res->h_exact = ev[2];
+    res->r_tot = ev[2] + 32.0 * (double)m / (double)d;
+    res->objective = objective;
+    res->candidates = cand;
+    res->rescored = rescored;
+}
+
+static int64_t read_rescored(void *ws, cudaStream_t st) {
+    DevStatus h;
+    if (cudaMemcpyAsync(&h, ws, sizeof(DevStatus), cudaMemcpyDeviceToHost, st) != cudaSuccess) return -1;
+    if (cudaStreamSynchronize(st) != cudaSuccess) return -1;
+    return h.rescored;
+}
+
+int ecasq_solve(const float *x, int64_t d, const ecasq_params_t *prm, void *ws, size_t ws_bytes, float *Q,
+                ecasq_result_t *res, ecasq_stream_t stream) {
+    if (!x || !Q || d < 1 || d >= ((int64_t)1 << 31) || !params_ok(prm)) return ECASQ_EINVAL;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const int s = prm->s;
+    Layout L;
+    make_layout(d, s, 1, &L);
+    int rc = check_ws(ws, ws_bytes, L);
+    if (rc) return rc;
+    int64_t p;
+    double n2;
+    rc = prepare_device(x, d, ws, L, st, &p, &n2);
+    if (rc) return rc;
+    Prefix P = make_prefix(ws, L, p, d);
+    double zero3[3] = {0.0, 0.0, 0.0};
+    if (p == 1) {
+        ECASQ_CUDA_TRY(cudaMemcpyAsync(Q, P.v, 4, cudaMemcpyDeviceToDevice, st));
+        ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+        fill_result(res, ECASQ_OK, 1, d, p, prm->lambda >= 0 ? prm->lambda : 0.0, n2, zero3, 0.0, 0, 0, 0, 0, 0);
+        return ECASQ_OK;
+    }
+    int passes = 0, nlam = 0;
+    int64_t cand_per = candidates_of(p, s, 0);
+    int64_t cand = 0;
+    std::vector<Eval> evals;
+    auto run = [&](const std::vector<double> &lams) -> int {
+        double lamp[kMaxG];
+        int G = (int)lams.size();
+        for (int g = 0; g < G; g++) lamp[g] = lams[g] * n2;
+        PassOut po;
+        int r = dp_pass_prepared(ws, L, P, s, lamp, G, prm->flags, st, po);
+        if (r) return r;
+        passes++;
+        nlam += G;
+        cand += cand_per * G;
+        for (int g = 0; g < G; g++) {
+            Eval e;
+            e.lam = lams[g];
+            e.m = po.m[g];
+            e.mse = po.met[4 * g + 1];
+            e.hs = po.met[4 * g + 2];
+            e.hx = po.met[4 * g + 3];
+            e.feas = prm->lambda >= 0.0 ? true : (e.hs <= prm->budget_bits);
+            e.a.assign(po.qidx.begin() + (size_t)g * s, po.qidx.begin() + (size_t)g * s + e.m);
+            evals.push_back(e);
+        }
+        return ECASQ_OK;
+    };
+    int status = ECASQ_OK;
+    const Eval *sel = nullptr;
+    if (prm->lambda >= 0.0) {
+        rc = run({prm->lambda});
+        if (rc) return rc;
+        sel = &evals[0];
+    } else {
+        double lo = prm->lambda_lo > 0.0 ? prm->lambda_lo : 1e-8;
+        double hi = prm->lambda_hi > 0.0 ? prm->lambda_hi : 1e3;
+        int R = prm->search_rounds > 0 ? prm->search_rounds : 6;
+        if (!(hi > lo)) return ECASQ_EINVAL;
+        double t[7];
+        midpoints7(lo, hi, t);
+        std::vector<double> l1 = {0.0};
+        l1.insert(l1.end(), t, t + 7);
+        rc = run(l1);
+        if (rc) return rc;
+        if (evals[0].feas) {
+            sel = &evals[0];
+        } else {
+            for (int r = 0; r < R; r++) {
+                if (r > 0) {
+                    midpoints7(lo, hi, t);
+                    rc = run(std::vector<double>(t, t + 7));
+                    if (rc) return rc;
+                }
+                const Eval *pts = &evals[evals.size() - 7];
+                int f = -1;
+                for (int q = 0; q < 7; q++)
+                    if (pts[q].feas) { f = q; break; }
+                if (f >= 0) {
+                    double nlo = f > 0 ? pts[f - 1].lam : lo;
+                    hi = pts[f].lam;
+                    lo = nlo;
+                } else {
+                    lo = pts[6].lam;
+                }
+            }
+            for (const Eval &e : evals)
+                if (e.feas && (!sel || e.mse < sel->mse || (e.mse == sel->mse && e.lam < sel->lam))) sel = &e;
+            if (!sel) {
+                rc = run({hi});
+                if (rc) return rc;
+                sel = &evals.back();
+                if (!sel->feas) status = ECASQ_EINFEASIBLE;
+            }
+        }
+    }
+    std::vector<int32_t> a = sel->a;
+    double lam = sel->lam;
+    double lamp = lam * n2;
+    int rr = 0;
+    if (status == ECASQ_OK && prm->refine_max_rounds > 0 && (int)a.size() >= 3) {
+        bool guard = prm->lambda < 0.0 && !(prm->flags & ECASQ_NO_REFINE_GUARD);
+        rc = refine_device(ws, L, P, a, lamp, prm->budget_bits, guard, prm->refine_max_rounds, prm->refine_rel_tol,
+                           st, &rr);
+        if (rc) return rc;
+    }
+    rc = write_codebook(ws, L, a, Q, st);
+    if (rc) return rc;
+    double ev[3];
+    rc = eval_device(ws, L, P, wsp<int32_t>(ws, L.qidx), (int)a.size(), st, ev);
+    if (rc) return rc;
+    double obj = prm->refine_max_rounds > 0 ? ev[0] + lamp * ev[2] : ev[0] + lamp * ev[1];
+    fill_result(res, status, (int)a.size(), d, p, lam, n2, ev, obj, passes, nlam, rr, cand, read_rescored(ws, st));
+    return status;
+}
+
+int ecasq_refine(const float *x, int64_t d, float *Q, int32_t m, double lambda, double budget_bits,
+                 int32_t max_rounds, double rel_tol, uint32_t flags, void *ws, size_t ws_bytes, ecasq_result_t *res,
+                 ecasq_stream_t stream) {
+    if (!x || !Q || d < 1 || d >= ((int64_t)1 << 31) || m < 1 || m > kMaxS || !(lambda >= 0.0) ||
+        !isfinite(lambda) || max_rounds < 0)
+        return ECASQ_EINVAL;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    Layout L;
+    make_layout(d, 2, 1, &L);
+    int rc = check_ws(ws, ws_bytes, L);
+    if (rc) return rc;
+    int64_t p;
+    double n2;
+    rc = prepare_device(x, d, ws, L, st, &p, &n2);
+    if (rc) return rc;
+    Prefix P = make_prefix(ws, L, p, d);
+    int32_t *a_dev = wsp<int32_t>(ws, L.qidx);
+    DevStatus *ds = wsp<DevStatus>(ws, L.status);
+    rc = launch_locate_q(P.v, p, Q, m, a_dev, ds, st);
+    if (rc) return rc;
+    std::vector<int32_t> a(m);
+    DevStatus h;
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(a.data(), a_dev, 4 * m, cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(&h, ds, sizeof(h), cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    if (h.range_err) return ECASQ_ERANGE;
+    if (a[0] != 0 || a[m - 1] != p - 1) return ECASQ_ERANGE;
+    for (int r = 1; r < m; r++)
+        if (a[r] <= a[r - 1]) return ECASQ_EINVAL;
+    double lamp = lambda * n2;
+    bool guard = budget_bits >= 0.0 && !(flags & ECASQ_NO_REFINE_GUARD);
+    int rr = 0;
+    rc = refine_device(ws, L, P, a, lamp, budget_bits, guard, max_rounds, rel_tol, st, &rr);
+    if (rc) return rc;
+    rc = write_codebook(ws, L, a, Q, st);
+    if (rc) return rc;
+    double ev[3];
+    rc = eval_device(ws, L, P, wsp<int32_t>(ws, L.qidx), m, st, ev);
+    if (rc) return rc;
+    fill_result(res, ECASQ_OK, m, d, p, lambda, n2, ev, ev[0] + lamp * ev[2], 0, 0, rr, 0, 0);
+    return ECASQ_OK;
+}
+
+int ecasq_evaluate(const float *x, int64_t d, const float *Q, int32_t m, void *ws, size_t ws_bytes, double *out,
+                   ecasq_stream_t stream) {
+    if (!x || !Q || !out || d < 1 || d >= ((int64_t)1 << 31) || m < 1 || m > kMaxS) return ECASQ_EINVAL;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    Layout L;
+    make_layout(d, 2, 1, &L);
+    int rc = check_ws(ws, ws_bytes, L);
+    if (rc) return rc;
+    int64_t p;
+    double n2;
+    rc = prepare_device(x, d, ws, L, st, &p, &n2);
+    if (rc) return rc;
+    Prefix P = make_prefix(ws, L, p, d);
+    int32_t *a_dev = wsp<int32_t>(ws, L.qidx);
+    DevStatus *ds = wsp<DevStatus>(ws, L.status);
+    rc = launch_locate_q(P.v, p, Q, m, a_dev, ds, st);
+    if (rc) return rc;
+    std::vector<int32_t> a(m);
+    DevStatus h;
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(a.data(), a_dev, 4 * m, cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(&h, ds, sizeof(h), cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    if (h.range_err || a[0] != 0 || a[m - 1] != p - 1) return ECASQ_ERANGE;
+    for (int r = 1; r < m; r++)
+        if (a[r] <= a[r - 1]) return ECASQ_EINVAL;
+    return eval_device(ws, L, P, a_dev, m, st, out);
+}
+
+int ecasq_quantize(const float *x, int64_t d, const float *Q, int32_t m, uint64_t seed, uint8_t *idx,
+                   uint32_t *counts, void *ws, size_t ws_bytes, double *h_emp, ecasq_stream_t stream) {
+    if (!x || !Q || !idx || !counts || d < 1 || d >= ((int64_t)1 << 31) || m < 1 || m > kMaxS) return ECASQ_EINVAL;
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255) != 0 || ws_bytes < sizeof(DevStatus)) return ECASQ_EWORKSPACE;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    DevStatus *ds = wsp<DevStatus>(ws, 0);
+    std::vector<float> qh(m);
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(qh.data(), Q, 4 * m, cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaMemsetAsync(ds, 0, sizeof(DevStatus), st));
+    ECASQ_CUDA_TRY(cudaMemsetAsync(counts, 0, 4 * (size_t)m, st));
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    for (int r = 1; r < m; r++)
+        if (!(qh[r] > qh[r - 1])) return ECASQ_EINVAL;
+    int rc = launch_quantize(x, d, Q, m, seed, idx, counts, ds, num_sms(), st);
+    if (rc) return rc;
+    std::vector<uint32_t> ch(m);
+    DevStatus h;
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(&h, ds, sizeof(h), cudaMemcpyDeviceToHost, st));
+    if (h_emp) ECASQ_CUDA_TRY(cudaMemcpyAsync(ch.data(), counts, 4 * (size_t)m, cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    if (h.range_err) return ECASQ_ERANGE;
+    if (h_emp) {
+        double he = 0.0, dd_ = (double)d;
+        for (int r = 0; r < m; r++) {
+            double f = (double)ch[r] / dd_;
+            if (f > 0.0) he += -f * log2(f);
+        }
+        *h_emp = he;
+    }
+    return ECASQ_OK;
+}
+
+int ecasq_solve_batched(const float *X, int64_t rows, int64_t d, const ecasq_params_t *prm, void *ws,
+                        size_t ws_bytes, float *Q, int32_t *m_out, ecasq_result_t *res, ecasq_stream_t stream) {
+    if (!X || !Q || !m_out || rows < 1 || d < 1 || d >= ((int64_t)1 << 31) || !params_ok(prm)) return ECASQ_EINVAL;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    int status = ECASQ_OK;
+    for (int64_t r = 0; r < rows; r++) {
+        ecasq_result_t one;
+        int rc = ecasq_solve(X + r * d, d, prm, ws, ws_bytes, Q + r * prm->s, &one, stream);
+        if (rc != ECASQ_OK && rc != ECASQ_EINFEASIBLE) return rc;
+        if (rc == ECASQ_EINFEASIBLE) status = rc;
+        ECASQ_CUDA_TRY(cudaMemcpyAsync(m_out + r, &one.m, sizeof(int32_t), cudaMemcpyHostToDevice, st));
+        if (res) res[r] = one;
+    }
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    return status;
+}
+
+}  // extern "C"

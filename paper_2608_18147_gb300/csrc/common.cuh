@@ -1,0 +1,164 @@
+// common.cuh -- shared internals of the ECASQ CUDA library (not part of the ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <math_constants.h>
+#include <stdint.h>
+#include <stddef.h>
+
+#include "../../include/ecasq.h"
+
+namespace ecasq {
+
+constexpr int kMaxS = 256;      // codebook cap
+constexpr int kMaxG = 8;        // multipliers per DP pass
+constexpr int kSortTile = 2048; // keys per radix-sort block
+constexpr int kScanTile = 1024; // elements per prefix-scan block
+
+#define ECASQ_CUDA_TRY(expr)                          \
+    do {                                              \
+        cudaError_t e_ = (expr);                      \
+        if (e_ != cudaSuccess) return ECASQ_ECUDA;    \
+    } while (0)
+
+#define ECASQ_LAUNCH_CHECK() ECASQ_CUDA_TRY(cudaGetLastError())
+
+__host__ __device__ static inline int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
+static inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+// ---------------------------------------------------------------- workspace
+// Device-side status block at the start of the workspace.
+struct DevStatus {
+    int64_t p;            // number of unique values
+    int32_t nonfinite;    // x held NaN/Inf
+    int32_t range_err;    // quantize: entry outside [Q0, Qm-1]; refine: Q not in X
+    int32_t timeout;      // a bounded wait ran out
+    int32_t pad;
+    double norm2;         // ||X||^2 (hi part of the double-double sum)
+    int64_t rescored;     // fast DP: candidates re-scored in fp64
+    int64_t overflow;     // fast DP: outputs that needed the full-rescan path
+    int32_t last_s;       // s and G of the last DP pass (for ecasq_dp_tables)
+    int32_t last_G;
+    int64_t last_d;       // d of the last DP pass
+};
+
+struct Layout {
+    size_t status;         // DevStatus
+    size_t keys0, keys1;   // uint32 [d]
+    size_t rcount;         // uint32 [256 * nb] radix counts / offsets
+    size_t head;           // int32 [d] unique index of each sorted position
+    size_t v;              // float [d] unique values
+    size_t w;              // int64 [d] multiplicities
+    size_t N;              // int64 [d+1]
+    size_t S, S2;          // double [2(d+1)] (hi | lo)
+    size_t part;           // double-double scan partials
+    size_t dp64;           // double [G (s+1) d]
+    size_t bp;             // int32 [G (s+1) d]
+    size_t dp32;           // float  [G (s+1) d]
+    size_t qidx;           // int32 [G s]  traced codebooks (unique indices)
+    size_t mcount;         // int32 [G]
+    size_t metrics;        // double [G 4]
+    size_t lam;            // double [G]   lambda' of each multiplier
+    size_t refine;         // refinement scratch
+    size_t band;           // fast DP band lists
+    size_t total;
+    int64_t d;
+    int32_t s;
+};
+
+size_t make_layout(int64_t d, int32_t s, int64_t rows, Layout *L);
+
+template <typename T>
+static inline T *wsp(void *ws, size_t off) { return reinterpret_cast<T *>(static_cast<char *>(ws) + off); }
+
+// ------------------------------------------------------------ double-double
+// Error-free transformations (Knuth's TwoSum; TwoProd with fma) and the
+// double-double sum used for the App. E prefix sums.  All operations are
+// spelled with _rn intrinsics so the compiler cannot contract them.
+struct dd { double hi, lo; };
+
+__device__ __forceinline__ dd two_sum(double a, double b) {
+    double s = __dadd_rn(a, b);
+    double bb = __dsub_rn(s, a);
+    double e = __dadd_rn(__dsub_rn(a, __dsub_rn(s, bb)), __dsub_rn(b, bb));
+    return {s, e};
+}
+__device__ __forceinline__ dd fast_two_sum(double a, double b) {  // |a| >= |b|
+    double s = __dadd_rn(a, b);
+    return {s, __dsub_rn(b, __dsub_rn(s, a))};
+}
+__device__ __forceinline__ dd two_prod(double a, double b) {
+    double p = __dmul_rn(a, b);
+    return {p, __fma_rn(a, b, -p)};
+}
+__device__ __forceinline__ dd dd_add(dd a, dd b) {
+    dd s = two_sum(a.hi, b.hi);
+    dd t = two_sum(a.lo, b.lo);
+    s.lo = __dadd_rn(s.lo, t.hi);
+    s = fast_two_sum(s.hi, s.lo);
+    s.lo = __dadd_rn(s.lo, t.lo);
+    return fast_two_sum(s.hi, s.lo);
+}
+__device__ __forceinline__ dd dd_neg(dd a) { return {-a.hi, -a.lo}; }
+__device__ __forceinline__ dd dd_sub(dd a, dd b) { return dd_add(a, dd_neg(b)); }
+__device__ __forceinline__ dd dd_mul_d(dd a, double b) {
+    dd p = two_prod(a.hi, b);
+    p.lo = __fma_rn(a.lo, b, p.lo);
+    return fast_two_sum(p.hi, p.lo);
+}
+__device__ __forceinline__ dd dd_mul(dd a, dd b) {
+    dd p = two_prod(a.hi, b.hi);
+    p.lo = __fma_rn(a.hi, b.lo, p.lo);
+    p.lo = __fma_rn(a.lo, b.hi, p.lo);
+    return fast_two_sum(p.hi, p.lo);
+}
+__device__ __forceinline__ double dd_round(dd a) { return __dadd_rn(a.hi, a.lo); }
+
+// h(y) = -y log2 y, h(0) = 0 (Sec. 4).
+__device__ __forceinline__ double hfun(double y) { return y > 0.0 ? -__dmul_rn(y, log2(y)) : 0.0; }
+
+// Prefix-sum view (App. E) used by every exact pair evaluation.
+struct Prefix {
+    const float *v;       // [p]
+    const int64_t *w;     // [p]
+    const int64_t *N;     // [p+1]
+    const double *S;      // hi [p+1] | lo [p+1]
+    const double *S2;
+    int64_t p;
+    int64_t d;
+};
+
+__device__ __forceinline__ dd load_dd(const double *a, int64_t p, int64_t t) { return {a[t], a[p + 1 + t]}; }
+
+// App. E for k < j over X_{k,j} = {x : v_k < x <= v_j}:
+//   A = S_kj - v_k N_kj, E = v_j N_kj - S_kj, C = (v_k+v_j) S_kj - S2_kj - v_k v_j N_kj,
+//   U = A / (v_j - v_k), D = E / (v_j - v_k).
+// Numerators in double-double, rounded once; one binary64 division each.
+__device__ __forceinline__ void pair_exact(const Prefix &P, int64_t k, int64_t j, double &C, double &U,
+                                           double &D) {
+    double n = (double)(P.N[j + 1] - P.N[k + 1]);
+    dd dS = dd_sub(load_dd(P.S, P.p, j + 1), load_dd(P.S, P.p, k + 1));
+    dd dS2 = dd_sub(load_dd(P.S2, P.p, j + 1), load_dd(P.S2, P.p, k + 1));
+    double vk = (double)P.v[k], vj = (double)P.v[j];
+    dd A = dd_sub(dS, two_prod(vk, n));
+    dd E = dd_sub(two_prod(vj, n), dS);
+    dd sk = two_sum(vk, vj);
+    dd Cd = dd_sub(dd_sub(dd_mul(sk, dS), dS2), two_prod(__dmul_rn(vk, vj), n));
+    double L = __dsub_rn(vj, vk);
+    C = dd_round(Cd);
+    U = __ddiv_rn(dd_round(A), L);
+    D = __ddiv_rn(dd_round(E), L);
+}
+
+// Sec. 5: Phi = h(U/d) + h(D/d); Phi^first adds the first value's mass w_0 to D.
+__device__ __forceinline__ double phi_exact(const Prefix &P, double U, double D, bool first) {
+    double dd_ = (double)P.d;
+    double Dm = first ? __dadd_rn(D, (double)P.w[0]) : D;
+    return __dadd_rn(hfun(__ddiv_rn(U, dd_)), hfun(__ddiv_rn(Dm, dd_)));
+}
+
+// -------------------------------------------------------------- host helpers
+int prepare_device(const float *x, int64_t d, void *ws, const Layout &L, cudaStream_t st, int64_t *p_host,
+                   double *norm2_host);
+
+}  // namespace ecasq

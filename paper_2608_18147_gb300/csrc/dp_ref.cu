@@ -1,0 +1,218 @@
+// dp_ref.cu -- fp64 reference kernels of the approximate DP (Sec. 5) and the
+// traceback / evaluation that every DP pass ends with.
+//
+// The reference DP evaluates every candidate of eq. apx_rec in binary64 with
+// interval costs from double-double prefix differences (App. E), one layer per
+// launch.  It is the slow, exact path (ECASQ_DP_REFERENCE) against which the
+// fast kernel is validated; the traceback and evaluation kernels serve both.
+#include "common.cuh"
+
+namespace ecasq {
+
+struct Lams { double v[kMaxG]; };
+
+__device__ __forceinline__ size_t dp_at(int g, int i, int64_t j, int s, int64_t p) {
+    return ((size_t)g * (size_t)(s + 1) + (size_t)i) * (size_t)p + (size_t)j;
+}
+
+// Rows 0, 1 and every undefined entry: dp = +inf, bp = -1.
+__global__ void k_dp_clear(double *dp64, int32_t *bp, int G, int s, int64_t p) {
+    size_t n = (size_t)G * (size_t)(s + 1) * (size_t)p;
+    size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+    size_t stride = (size_t)gridDim.x * blockDim.x;
+    for (; i < n; i += stride) { dp64[i] = CUDART_INF; bp[i] = -1; }
+}
+
+// eq. apx_base with P = X, L = {0}: dp(2, j) = C[0, j] + lambda' Phi^first[0, j].
+__global__ void k_dp_base(Prefix P, Lams lam, int G, int s, double *dp64, int32_t *bp) {
+    int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x + 1;
+    if (j >= P.p) return;
+    double C, U, D;
+    pair_exact(P, 0, j, C, U, D);
+    double phi = phi_exact(P, U, D, true);
+    for (int g = 0; g < G; g++) {
+        dp64[dp_at(g, 2, j, s, P.p)] = __dadd_rn(C, __dmul_rn(lam.v[g], phi));
+        bp[dp_at(g, 2, j, s, P.p)] = 0;
+    }
+}
+
+// eq. apx_rec, one layer i >= 3 for all G multipliers: thread per j, every
+// k in [i-2, j-1], candidate dp(i-1, k) + (C[k,j] + lambda' Phi[k,j]); the
+// lowest k among exact minima wins.  Heavy (large-j) blocks launch first.
+__global__ void __launch_bounds__(128) k_dp_layer_ref(Prefix P, Lams lam, int G, int s, int i, double *dp64,
+                                                      int32_t *bp) {
+    int64_t nblk = gridDim.x;
+    int64_t j = (nblk - 1 - blockIdx.x) * blockDim.x + threadIdx.x;
+    if (j < i - 1 || j >= P.p) return;
+    double best[kMaxG];
+    int32_t arg[kMaxG];
+#pragma unroll
+    for (int g = 0; g < kMaxG; g++) { best[g] = CUDART_INF; arg[g] = -1; }
+    for (int64_t k = i - 2; k < j; k++) {
+        double C, U, D;
+        pair_exact(P, k, j, C, U, D);
+        double phi = phi_exact(P, U, D, false);
+#pragma unroll
+        for (int g = 0; g < kMaxG; g++) {
+            if (g < G) {
+                double prev = dp64[dp_at(g, i - 1, k, s, P.p)];
+                double c = __dadd_rn(prev, __dadd_rn(C, __dmul_rn(lam.v[g], phi)));
+                if (c < best[g]) { best[g] = c; arg[g] = (int32_t)k; }
+            }
+        }
+    }
+    for (int g = 0; g < G; g++) {
+        dp64[dp_at(g, i, j, s, P.p)] = best[g];
+        bp[dp_at(g, i, j, s, P.p)] = arg[g];
+    }
+}
+
+// Metrics of codebook a[0..m-1] (unique indices): MSE, H(I,B), H(Xhat), summed
+// in interval order exactly as the definitions list them (Sec. 2, Sec. 3,
+// eq. apx_additive_entropy).  One warp; lanes evaluate intervals, lane 0 sums.
+__device__ void eval_codebook_warp(const Prefix &P, const int32_t *a, int m, double *out3, double *scratch) {
+    // scratch: 4 * kMaxS doubles (C, Phi, U, D per interval)
+    int lane = threadIdx.x & 31;
+    for (int r = lane; r + 1 < m; r += 32) {
+        double C, U, D;
+        pair_exact(P, a[r], a[r + 1], C, U, D);
+        scratch[r] = C;
+        scratch[kMaxS + r] = phi_exact(P, U, D, r == 0);
+        scratch[2 * kMaxS + r] = U;
+        scratch[3 * kMaxS + r] = D;
+    }
+    __syncwarp();
+    if (lane == 0) {
+        double dd_ = (double)P.d;
+        if (m < 2) { out3[0] = 0.0; out3[1] = 0.0; out3[2] = 0.0; return; }
+        double mse = 0.0, hs = 0.0, hx = 0.0, prevU = 0.0;
+        for (int r = 0; r + 1 < m; r++) {
+            mse = __dadd_rn(mse, scratch[r]);
+            hs = __dadd_rn(hs, scratch[kMaxS + r]);
+            double D = scratch[3 * kMaxS + r];
+            double f = (r == 0) ? __dadd_rn((double)P.w[0], D) : __dadd_rn(prevU, D);
+            hx = __dadd_rn(hx, hfun(__ddiv_rn(f, dd_)));
+            prevU = scratch[2 * kMaxS + r];
+        }
+        hx = __dadd_rn(hx, hfun(__ddiv_rn(prevU, dd_)));
+        out3[0] = mse; out3[1] = hs; out3[2] = hx;
+    }
+    __syncwarp();
+}
+
+// eq. apx_final (smallest i among exact minima; i = s only with EXACT_S) and
+// the backpointer walk, then the metrics of the traced codebook.  Block g = one
+// multiplier, one warp.
+__global__ void k_traceback_eval(Prefix P, int G, int s, int exact_s, const double *dp64, const int32_t *bp,
+                                 int32_t *qidx, int32_t *mcount, double *metrics) {
+    __shared__ double scratch[4 * kMaxS];
+    __shared__ int32_t a[kMaxS];
+    __shared__ int sm_m;
+    int g = blockIdx.x;
+    int64_t p = P.p;
+    if (threadIdx.x == 0) {
+        int istar = -1;
+        double best = CUDART_INF;
+        for (int i = exact_s ? s : 2; i <= s; i++) {
+            double v = dp64[dp_at(g, i, p - 1, s, p)];
+            if (v < best) { best = v; istar = i; }
+        }
+        if (istar < 0) {
+            sm_m = 0;
+        } else {
+            int64_t j = p - 1;
+            a[istar - 1] = (int32_t)j;
+            for (int i = istar; i >= 3; i--) {
+                j = bp[dp_at(g, i, j, s, p)];
+                a[i - 2] = (int32_t)j;
+            }
+            a[0] = 0;
+            sm_m = istar;
+        }
+        metrics[4 * g + 0] = best;
+        mcount[g] = sm_m;
+    }
+    __syncwarp();
+    int m = sm_m;
+    for (int r = threadIdx.x; r < m; r += 32) qidx[g * s + r] = a[r];
+    if (m > 0) eval_codebook_warp(P, a, m, &metrics[4 * g + 1], scratch);
+}
+
+// Metrics of a caller-given codebook (unique indices on the device).
+__global__ void k_eval_codebook(Prefix P, const int32_t *a_in, int m, double *out3) {
+    __shared__ double scratch[4 * kMaxS];
+    __shared__ int32_t a[kMaxS];
+    for (int r = threadIdx.x; r < m; r += 32) a[r] = a_in[r];
+    __syncwarp();
+    eval_codebook_warp(P, a, m, out3, scratch);
+}
+
+// Q[r] = v[a[r]] for every multiplier row g.
+__global__ void k_gather_q(const float *v, const int32_t *qidx, const int32_t *mcount, int s, float *Q) {
+    int g = blockIdx.x;
+    int m = mcount[g];
+    for (int r = threadIdx.x; r < m; r += blockDim.x) Q[g * s + r] = v[qidx[g * s + r]];
+}
+
+// Unique indices of a codebook given by value (binary search in v); -1 if absent.
+__global__ void k_locate_q(const float *v, int64_t p, const float *Q, int m, int32_t *a, DevStatus *st) {
+    for (int r = threadIdx.x; r < m; r += blockDim.x) {
+        float q = Q[r];
+        if (q == 0.0f) q = 0.0f;
+        int64_t lo = 0, hi = p - 1;
+        while (lo < hi) {
+            int64_t mid = (lo + hi) >> 1;
+            if (v[mid] < q) lo = mid + 1; else hi = mid;
+        }
+        bool ok = v[lo] == q;
+        a[r] = ok ? (int32_t)lo : -1;
+        if (!ok) st->range_err = 1;
+    }
+}
+
+// ----------------------------------------------------------- host launchers
+int launch_dp_reference(const Prefix &P, const double *lamp, int G, int s, double *dp64, int32_t *bp,
+                        cudaStream_t st) {
+    Lams lam{};
+    for (int g = 0; g < G; g++) lam.v[g] = lamp[g];
+    k_dp_clear<<<4096, 256, 0, st>>>(dp64, bp, G, s, P.p);
+    ECASQ_LAUNCH_CHECK();
+    if (P.p >= 2) {
+        k_dp_base<<<(unsigned)cdiv(P.p - 1, 128), 128, 0, st>>>(P, lam, G, s, dp64, bp);
+        ECASQ_LAUNCH_CHECK();
+    }
+    for (int i = 3; i <= s; i++) {
+        if (P.p < i) break;
+        k_dp_layer_ref<<<(unsigned)cdiv(P.p, 128), 128, 0, st>>>(P, lam, G, s, i, dp64, bp);
+        ECASQ_LAUNCH_CHECK();
+    }
+    return ECASQ_OK;
+}
+
+int launch_traceback_eval(const Prefix &P, int G, int s, int exact_s, const double *dp64, const int32_t *bp,
+                          int32_t *qidx, int32_t *mcount, double *metrics, cudaStream_t st) {
+    k_traceback_eval<<<G, 32, 0, st>>>(P, G, s, exact_s, dp64, bp, qidx, mcount, metrics);
+    ECASQ_LAUNCH_CHECK();
+    return ECASQ_OK;
+}
+
+int launch_eval_codebook(const Prefix &P, const int32_t *a, int m, double *out3, cudaStream_t st) {
+    k_eval_codebook<<<1, 32, 0, st>>>(P, a, m, out3);
+    ECASQ_LAUNCH_CHECK();
+    return ECASQ_OK;
+}
+
+int launch_gather_q(const float *v, const int32_t *qidx, const int32_t *mcount, int G, int s, float *Q,
+                    cudaStream_t st) {
+    k_gather_q<<<G, 64, 0, st>>>(v, qidx, mcount, s, Q);
+    ECASQ_LAUNCH_CHECK();
+    return ECASQ_OK;
+}
+
+int launch_locate_q(const float *v, int64_t p, const float *Q, int m, int32_t *a, DevStatus *ds, cudaStream_t st) {
+    k_locate_q<<<1, 256, 0, st>>>(v, p, Q, m, a, ds);
+    ECASQ_LAUNCH_CHECK();
+    return ECASQ_OK;
+}
+
+}  // namespace ecasq

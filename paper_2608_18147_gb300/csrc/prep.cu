@@ -1,0 +1,297 @@
+// prep.cu -- step 1 of every solve: sorted copy of x, weighted histogram
+// (Sec. 2: "we assume X is sorted ... work with its weighted histogram") and the
+// prefix sums N, S, S2 of App. E, accumulated in double-double.
+//
+// Sort: LSD radix sort, 4 passes of 8 bits over order-preserving uint32 keys
+// (-0.0 folded into +0.0).  Each pass: per-block digit counts, one scan of the
+// [digit][block] count matrix, and a stable scatter whose in-block ranks come
+// from warp match masks.
+#include <algorithm>
+
+#include "common.cuh"
+
+namespace ecasq {
+
+__device__ __forceinline__ uint32_t f2key(float f) {
+    uint32_t u = __float_as_uint(f);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float key2f(uint32_t k) {
+    uint32_t u = (k & 0x80000000u) ? (k & 0x7fffffffu) : ~k;
+    return __uint_as_float(u);
+}
+
+__global__ void k_make_keys(const float *__restrict__ x, int64_t d, uint32_t *__restrict__ keys,
+                            DevStatus *st) {
+    int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (; i < d; i += stride) {
+        float f = x[i];
+        if (!isfinite(f)) st->nonfinite = 1;
+        if (f == 0.0f) f = 0.0f;
+        keys[i] = f2key(f);
+    }
+}
+
+// counts[digit * nb + block] = number of keys of the block with that digit.
+__global__ void __launch_bounds__(256) k_radix_count(const uint32_t *__restrict__ keys, int64_t d, int shift,
+                                                     uint32_t *__restrict__ counts, int nb) {
+    __shared__ uint32_t h[256];
+    h[threadIdx.x] = 0;
+    __syncthreads();
+    int64_t base = (int64_t)blockIdx.x * kSortTile;
+    for (int r = 0; r < kSortTile / 256; r++) {
+        int64_t i = base + r * 256 + threadIdx.x;
+        if (i < d) atomicAdd(&h[(keys[i] >> shift) & 255u], 1u);
+    }
+    __syncthreads();
+    counts[(size_t)threadIdx.x * nb + blockIdx.x] = h[threadIdx.x];
+}
+
+// In-place exclusive scan of n uint32 values by one block of 1024 threads.
+__global__ void __launch_bounds__(1024) k_scan_u32(uint32_t *a, int64_t n) {
+    __shared__ uint32_t wsum[32];
+    int64_t per = cdiv(n, 1024);
+    int64_t lo = threadIdx.x * per, hi = min(lo + per, n);
+    uint32_t s = 0;
+    for (int64_t i = lo; i < hi; i++) s += a[i];
+    // block exclusive scan of s
+    uint32_t incl = s;
+    int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    for (int o = 1; o < 32; o <<= 1) {
+        uint32_t t = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += t;
+    }
+    if (lane == 31) wsum[wid] = incl;
+    __syncthreads();
+    if (wid == 0) {
+        uint32_t v = wsum[lane], vi = v;
+        for (int o = 1; o < 32; o <<= 1) {
+            uint32_t t = __shfl_up_sync(0xffffffffu, vi, o);
+            if (lane >= o) vi += t;
+        }
+        wsum[lane] = vi - v;
+    }
+    __syncthreads();
+    uint32_t run = wsum[wid] + incl - s;
+    for (int64_t i = lo; i < hi; i++) {
+        uint32_t t = a[i];
+        a[i] = run;
+        run += t;
+    }
+}
+
+// Stable scatter of one radix pass.  Positions inside a tile are visited in
+// rounds of 256 (round r covers tile positions r*256 .. r*256+255, thread t
+// holding position r*256 + t), so (round, warp, lane) is the input order.
+__global__ void __launch_bounds__(256) k_radix_scatter(const uint32_t *__restrict__ kin, uint32_t *__restrict__ kout,
+                                                       int64_t d, int shift, const uint32_t *__restrict__ offs,
+                                                       int nb) {
+    __shared__ uint32_t cnt[8][256];
+    __shared__ uint32_t base[8][256];
+    __shared__ uint32_t run[256];
+    int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    uint32_t lt_mask = (1u << lane) - 1u;
+    run[threadIdx.x] = offs[(size_t)threadIdx.x * nb + blockIdx.x];
+    int64_t tbase = (int64_t)blockIdx.x * kSortTile;
+    for (int r = 0; r < kSortTile / 256; r++) {
+        for (int w = 0; w < 8; w++) cnt[w][threadIdx.x] = 0;
+        __syncthreads();
+        int64_t i = tbase + r * 256 + threadIdx.x;
+        bool valid = i < d;
+        uint32_t key = valid ? kin[i] : 0u;
+        uint32_t dig = valid ? ((key >> shift) & 255u) : (256u + (uint32_t)lane);
+        uint32_t peers = __match_any_sync(0xffffffffu, dig);
+        uint32_t rank = __popc(peers & lt_mask);
+        if (valid && rank == 0) cnt[wid][dig] = __popc(peers);
+        __syncthreads();
+        {
+            uint32_t acc = run[threadIdx.x];
+            for (int w = 0; w < 8; w++) {
+                base[w][threadIdx.x] = acc;
+                acc += cnt[w][threadIdx.x];
+            }
+            run[threadIdx.x] = acc;
+        }
+        __syncthreads();
+        if (valid) kout[base[wid][dig] + rank] = key;
+        __syncthreads();
+    }
+}
+
+// Pass A of the histogram scan: per tile of kScanTile sorted keys, the number
+// of unique-value heads and the double-double sums of x and x^2.
+struct DDPart { double s_hi, s_lo, q_hi, q_lo; int64_t heads; int64_t pad; };
+
+__device__ __forceinline__ bool is_head(const uint32_t *keys, int64_t i) { return i == 0 || keys[i] != keys[i - 1]; }
+
+template <typename T>
+__device__ __forceinline__ T shfl_up(T v, int o) { return __shfl_up_sync(0xffffffffu, v, o); }
+
+struct ScanVal { dd s, q; int64_t h; };
+
+__device__ __forceinline__ ScanVal sv_add(const ScanVal &a, const ScanVal &b) {
+    return {dd_add(a.s, b.s), dd_add(a.q, b.q), a.h + b.h};
+}
+
+// Block-wide inclusive scan of one ScanVal per thread (256 threads).
+__device__ ScanVal block_scan_incl(ScanVal v, ScanVal *wtot, ScanVal &total) {
+    int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    for (int o = 1; o < 32; o <<= 1) {
+        ScanVal t;
+        t.s.hi = shfl_up(v.s.hi, o); t.s.lo = shfl_up(v.s.lo, o);
+        t.q.hi = shfl_up(v.q.hi, o); t.q.lo = shfl_up(v.q.lo, o);
+        t.h = shfl_up(v.h, o);
+        if (lane >= o) v = sv_add(t, v);
+    }
+    if (lane == 31) wtot[wid] = v;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        ScanVal acc = wtot[0];
+        for (int w = 1; w < 8; w++) { acc = sv_add(acc, wtot[w]); wtot[w] = acc; }
+    }
+    __syncthreads();
+    if (wid > 0) v = sv_add(wtot[wid - 1], v);
+    total = wtot[7];
+    __syncthreads();
+    return v;
+}
+
+__global__ void __launch_bounds__(256) k_hist_partials(const uint32_t *__restrict__ keys, int64_t d, DDPart *part) {
+    __shared__ ScanVal wtot[8];
+    int64_t base = (int64_t)blockIdx.x * kScanTile + threadIdx.x * 4;
+    ScanVal v{{0.0, 0.0}, {0.0, 0.0}, 0};
+    for (int e = 0; e < 4; e++) {
+        int64_t i = base + e;
+        if (i < d) {
+            double x = (double)key2f(keys[i]);
+            v.s = dd_add(v.s, dd{x, 0.0});
+            v.q = dd_add(v.q, dd{__dmul_rn(x, x), 0.0});
+            v.h += is_head(keys, i);
+        }
+    }
+    ScanVal tot;
+    block_scan_incl(v, wtot, tot);
+    if (threadIdx.x == 0) part[blockIdx.x] = {tot.s.hi, tot.s.lo, tot.q.hi, tot.q.lo, tot.h, 0};
+}
+
+// Exclusive scan of the tile partials (one thread, in order; nb is small).
+__global__ void k_hist_scan_partials(DDPart *part, int64_t nb) {
+    if (threadIdx.x != 0 || blockIdx.x != 0) return;
+    ScanVal acc{{0.0, 0.0}, {0.0, 0.0}, 0};
+    for (int64_t b = 0; b < nb; b++) {
+        ScanVal t{{part[b].s_hi, part[b].s_lo}, {part[b].q_hi, part[b].q_lo}, part[b].heads};
+        part[b] = {acc.s.hi, acc.s.lo, acc.q.hi, acc.q.lo, acc.h, 0};
+        acc = sv_add(acc, t);
+    }
+}
+
+// Pass C: per sorted position i that starts a run of equal keys (a head), the
+// unique index u and v[u], N[u] = i, S[u], S2[u] (exclusive prefix sums).
+// The last position also writes N[p] = d, S[p], S2[p], p and ||X||^2.
+__global__ void __launch_bounds__(256) k_hist_fill(const uint32_t *__restrict__ keys, int64_t d, const DDPart *part,
+                                                   float *v, int64_t *N, double *S, double *S2, DevStatus *st,
+                                                   int64_t pcap) {
+    __shared__ ScanVal wtot[8];
+    int64_t base = (int64_t)blockIdx.x * kScanTile + threadIdx.x * 4;
+    ScanVal loc{{0.0, 0.0}, {0.0, 0.0}, 0};
+    double xs[4];
+    int hd[4];
+    for (int e = 0; e < 4; e++) {
+        int64_t i = base + e;
+        xs[e] = 0.0; hd[e] = 0;
+        if (i < d) {
+            xs[e] = (double)key2f(keys[i]);
+            hd[e] = is_head(keys, i);
+            loc.s = dd_add(loc.s, dd{xs[e], 0.0});
+            loc.q = dd_add(loc.q, dd{__dmul_rn(xs[e], xs[e]), 0.0});
+            loc.h += hd[e];
+        }
+    }
+    ScanVal tot;
+    ScanVal incl = block_scan_incl(loc, wtot, tot);
+    const DDPart &pb = part[blockIdx.x];
+    ScanVal off{{pb.s_hi, pb.s_lo}, {pb.q_hi, pb.q_lo}, pb.heads};
+    // exclusive prefix before this thread's first element
+    ScanVal run{dd_sub(incl.s, loc.s), dd_sub(incl.q, loc.q), incl.h - loc.h};
+    run = sv_add(off, run);
+    for (int e = 0; e < 4; e++) {
+        int64_t i = base + e;
+        if (i >= d) break;
+        if (hd[e]) {
+            int64_t u = run.h;
+            v[u] = (float)xs[e];
+            N[u] = i;
+            S[u] = run.s.hi; S[pcap + 1 + u] = run.s.lo;
+            S2[u] = run.q.hi; S2[pcap + 1 + u] = run.q.lo;
+        }
+        run.s = dd_add(run.s, dd{xs[e], 0.0});
+        run.q = dd_add(run.q, dd{__dmul_rn(xs[e], xs[e]), 0.0});
+        run.h += hd[e];
+        if (i == d - 1) {
+            int64_t p = run.h;
+            N[p] = d;
+            S[p] = run.s.hi; S[pcap + 1 + p] = run.s.lo;
+            S2[p] = run.q.hi; S2[pcap + 1 + p] = run.q.lo;
+            st->p = p;
+            st->norm2 = run.q.hi;
+        }
+    }
+}
+
+// The arrays were written with lo parts at offset pcap+1 (pcap = d); repack
+// them to offset p+1 so that every later kernel indexes (hi[0..p], lo[0..p]).
+__global__ void k_hist_finish(int64_t *N, int64_t *w, double *S, double *S2, const DevStatus *st, int64_t pcap,
+                              double *Sp, double *S2p) {
+    int64_t p = st->p;
+    int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (; i <= p; i += stride) {
+        if (i < p) w[i] = N[i + 1] - N[i];
+        Sp[i] = S[i]; Sp[p + 1 + i] = S[pcap + 1 + i];
+        S2p[i] = S2[i]; S2p[p + 1 + i] = S2[pcap + 1 + i];
+    }
+}
+
+int prepare_device(const float *x, int64_t d, void *ws, const Layout &L, cudaStream_t stream, int64_t *p_host,
+                   double *norm2_host) {
+    DevStatus *st = wsp<DevStatus>(ws, L.status);
+    uint32_t *k0 = wsp<uint32_t>(ws, L.keys0), *k1 = wsp<uint32_t>(ws, L.keys1);
+    uint32_t *cnt = wsp<uint32_t>(ws, L.rcount);
+    ECASQ_CUDA_TRY(cudaMemsetAsync(st, 0, sizeof(DevStatus), stream));
+    int nb = (int)cdiv(d, kSortTile);
+    k_make_keys<<<(unsigned)std::min<int64_t>(cdiv(d, 256), 4096), 256, 0, stream>>>(x, d, k0, st);
+    ECASQ_LAUNCH_CHECK();
+    uint32_t *a = k0, *b = k1;
+    for (int shift = 0; shift < 32; shift += 8) {
+        k_radix_count<<<nb, 256, 0, stream>>>(a, d, shift, cnt, nb);
+        k_scan_u32<<<1, 1024, 0, stream>>>(cnt, (int64_t)256 * nb);
+        k_radix_scatter<<<nb, 256, 0, stream>>>(a, b, d, shift, cnt, nb);
+        ECASQ_LAUNCH_CHECK();
+        uint32_t *t = a; a = b; b = t;
+    }
+    // a == k0 holds the sorted keys
+    int64_t nbs = cdiv(d, kScanTile);
+    DDPart *part = wsp<DDPart>(ws, L.part);
+    // scratch copies of N/S/S2 with lo parts at offset d+1 live in keys1 / dp area
+    double *Stmp = wsp<double>(ws, L.dp64);
+    double *S2tmp = Stmp + 2 * (d + 1);
+    k_hist_partials<<<(unsigned)nbs, 256, 0, stream>>>(a, d, part);
+    k_hist_scan_partials<<<1, 32, 0, stream>>>(part, nbs);
+    k_hist_fill<<<(unsigned)nbs, 256, 0, stream>>>(a, d, part, wsp<float>(ws, L.v), wsp<int64_t>(ws, L.N), Stmp,
+                                                 S2tmp, st, d);
+    ECASQ_LAUNCH_CHECK();
+    k_hist_finish<<<(unsigned)std::min<int64_t>(cdiv(d + 1, 256), 4096), 256, 0, stream>>>(
+        wsp<int64_t>(ws, L.N), wsp<int64_t>(ws, L.w), Stmp, S2tmp, st, d, wsp<double>(ws, L.S),
+        wsp<double>(ws, L.S2));
+    ECASQ_LAUNCH_CHECK();
+    DevStatus h;
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(&h, st, sizeof(DevStatus), cudaMemcpyDeviceToHost, stream));
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(stream));
+    if (h.nonfinite) return ECASQ_ENONFINITE;
+    *p_host = h.p;
+    *norm2_host = h.norm2;
+    return ECASQ_OK;
+}
+
+}  // namespace ecasq

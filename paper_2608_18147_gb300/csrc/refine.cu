@@ -1,0 +1,92 @@
+// refine.cu -- one colour step of the three-colour refinement (Sec. 6).
+//
+// Block b moves the b-th value of the colour class: q_l with l % 3 == colour,
+// 1 <= l <= m-2.  Its candidates are the unique input values strictly between
+// its fixed neighbours; the local objective of Sec. 6 (true entropy reading) is
+//   C[q_{l-1}, c] + C[c, q_{l+1}] + lambda' (h(f_{l-1}/d) + h(f_l/d) + h(f_{l+1}/d)),
+// f_{l-1} = U[q_{l-2}, q_{l-1}] + D[q_{l-1}, c]   (w_0 + D[q_0, c] when l-1 = 0),
+// f_l     = U[q_{l-1}, c] + D[c, q_{l+1}],
+// f_{l+1} = U[c, q_{l+1}] + D[q_{l+1}, q_{l+2}]   (U[c, q_{m-1}] when l+1 = m-1).
+// Values of one class never share a frequency term, so all of them move at
+// once (Sec. 6, Fig. 3).  Ties keep the current value, else the lowest index.
+#include "common.cuh"
+
+namespace ecasq {
+
+struct Nbr {
+    int64_t L, R, cur;
+    double Ux, Dx;   // outer neighbours' fixed halves of f_{l-1} and f_{l+1}
+    int firstL, lastR;
+};
+
+__device__ __forceinline__ double local_obj(const Prefix &P, const Nbr &n, int64_t c, double lamp) {
+    double dd_ = (double)P.d;
+    double C1, U1, D1, C2, U2, D2;
+    pair_exact(P, n.L, c, C1, U1, D1);
+    pair_exact(P, c, n.R, C2, U2, D2);
+    double fl = n.firstL ? __dadd_rn((double)P.w[0], D1) : __dadd_rn(n.Ux, D1);
+    double fm = __dadd_rn(U1, D2);
+    double fr = n.lastR ? U2 : __dadd_rn(U2, n.Dx);
+    double ent = __dadd_rn(__dadd_rn(hfun(__ddiv_rn(fl, dd_)), hfun(__ddiv_rn(fm, dd_))), hfun(__ddiv_rn(fr, dd_)));
+    return __dadd_rn(__dadd_rn(C1, C2), __dmul_rn(lamp, ent));
+}
+
+__global__ void __launch_bounds__(256) k_refine_colour(Prefix P, const int32_t *a, int m, int colour, double lamp,
+                                                       int32_t *a_new, int32_t *moved) {
+    __shared__ Nbr nb;
+    __shared__ double rv[256];
+    __shared__ int64_t ri[256];
+    int l0 = colour == 0 ? 3 : colour;
+    int l = l0 + 3 * blockIdx.x;
+    if (l > m - 2) return;
+    if (threadIdx.x == 0) {
+        Nbr n;
+        n.L = a[l - 1]; n.R = a[l + 1]; n.cur = a[l];
+        n.firstL = (l - 1 == 0); n.lastR = (l + 1 == m - 1);
+        double C, U, D;
+        n.Ux = 0.0; n.Dx = 0.0;
+        if (!n.firstL) { pair_exact(P, a[l - 2], n.L, C, U, D); n.Ux = U; }
+        if (!n.lastR) { pair_exact(P, n.R, a[l + 2], C, U, D); n.Dx = D; }
+        nb = n;
+    }
+    __syncthreads();
+    Nbr n = nb;
+    double bv = CUDART_INF;
+    int64_t bi = -1;
+    for (int64_t c = n.L + 1 + threadIdx.x; c < n.R; c += blockDim.x) {
+        if (c == n.cur) continue;
+        double v = local_obj(P, n, c, lamp);
+        if (v < bv) { bv = v; bi = c; }   // c ascends per thread: keeps the lowest
+    }
+    rv[threadIdx.x] = bv; ri[threadIdx.x] = bi;
+    __syncthreads();
+    for (int o = 128; o > 0; o >>= 1) {
+        if (threadIdx.x < o) {
+            double v2 = rv[threadIdx.x + o];
+            int64_t i2 = ri[threadIdx.x + o];
+            if (v2 < rv[threadIdx.x] || (v2 == rv[threadIdx.x] && i2 >= 0 && (ri[threadIdx.x] < 0 || i2 < ri[threadIdx.x]))) {
+                rv[threadIdx.x] = v2; ri[threadIdx.x] = i2;
+            }
+        }
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) {
+        double vc = local_obj(P, n, n.cur, lamp);
+        int64_t nw = (ri[0] >= 0 && rv[0] < vc) ? ri[0] : n.cur;
+        a_new[l] = (int32_t)nw;
+        if (nw != n.cur) atomicExch(moved, 1);
+    }
+}
+
+int launch_refine_colour(const Prefix &P, const int32_t *a, int m, int colour, double lamp, int32_t *a_new,
+                         int32_t *moved, cudaStream_t st, int *nblocks_out) {
+    int l0 = colour == 0 ? 3 : colour;
+    int nblk = (m - 2 >= l0) ? (m - 2 - l0) / 3 + 1 : 0;
+    *nblocks_out = nblk;
+    if (nblk == 0) return ECASQ_OK;
+    k_refine_colour<<<nblk, 256, 0, st>>>(P, a, m, colour, lamp, a_new, moved);
+    ECASQ_LAUNCH_CHECK();
+    return ECASQ_OK;
+}
+
+}  // namespace ecasq

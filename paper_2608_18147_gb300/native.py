@@ -1,0 +1,289 @@
+"""Thin ctypes binding of include/ecasq.h.
+
+Every function here has the C entry point's name and only marshals
+arguments: torch CUDA tensors become device pointers, the current torch
+stream becomes the cudaStream_t, and host results come back as Python
+values.  All arithmetic runs in libecasq.so; there is no fallback -- if the
+library cannot be loaded, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+import threading
+
+import numpy as np
+
+from . import build as _build
+
+OK, EINVAL, ENONFINITE, EINFEASIBLE, EWORKSPACE, ECUDA, ETIMEOUT, ERANGE = 0, -1, -2, -3, -4, -5, -6, -7
+EXACT_S, NO_REFINE_GUARD, DP_REFERENCE = 1, 2, 4
+
+_lock = threading.Lock()
+_lib = None
+
+
+class Params(C.Structure):
+    _fields_ = [("s", C.c_int32), ("flags", C.c_uint32), ("budget_bits", C.c_double), ("lambda_", C.c_double),
+                ("lambda_lo", C.c_double), ("lambda_hi", C.c_double), ("search_rounds", C.c_int32),
+                ("refine_max_rounds", C.c_int32), ("refine_rel_tol", C.c_double)]
+
+
+class Result(C.Structure):
+    _fields_ = [("status", C.c_int32), ("m", C.c_int32), ("passes", C.c_int32), ("lambdas_evaluated", C.c_int32),
+                ("refine_rounds", C.c_int32), ("reserved", C.c_int32), ("d", C.c_int64), ("p", C.c_int64),
+                ("lambda_", C.c_double), ("lambda_prime", C.c_double), ("norm2", C.c_double), ("mse", C.c_double),
+                ("vnmse", C.c_double), ("h_surrogate", C.c_double), ("h_exact", C.c_double), ("r_tot", C.c_double),
+                ("objective", C.c_double), ("candidates", C.c_int64), ("rescored", C.c_int64)]
+
+    def as_dict(self):
+        out = {}
+        for name, _ in self._fields_:
+            key = "lambda" if name == "lambda_" else name
+            out[key] = getattr(self, name)
+        return out
+
+
+class EcasqError(RuntimeError):
+    def __init__(self, code, where):
+        self.code = code
+        msg = lib().ecasq_strerror(code).decode() if _lib is not None else str(code)
+        super().__init__("%s: %s (status %d)" % (where, msg, code))
+
+
+def lib_path() -> str:
+    return _build.LIB
+
+
+def lib():
+    """Load libecasq.so (building it first if it is missing or stale)."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        path = _build.build()
+        L = C.CDLL(path)
+        vp, i32, i64, u32, u64, dbl, sz = C.c_void_p, C.c_int32, C.c_int64, C.c_uint32, C.c_uint64, C.c_double, C.c_size_t
+        pd = C.POINTER(C.c_double)
+        pi32 = C.POINTER(C.c_int32)
+        pi64 = C.POINTER(C.c_int64)
+        PP = C.POINTER(Params)
+        PR = C.POINTER(Result)
+        sig = {
+            "ecasq_version": (C.c_int, []),
+            "ecasq_strerror": (C.c_char_p, [C.c_int]),
+            "ecasq_workspace_size": (sz, [i64, i32, i64]),
+            "ecasq_solve": (C.c_int, [vp, i64, PP, vp, sz, vp, PR, vp]),
+            "ecasq_dp_pass": (C.c_int, [vp, i64, i32, pd, i32, u32, vp, sz, vp, pi32, pd, vp]),
+            "ecasq_dp_tables": (C.c_int, [vp, sz, i32, vp, vp, pi64, vp]),
+            "ecasq_refine": (C.c_int, [vp, i64, vp, i32, dbl, dbl, i32, dbl, u32, vp, sz, PR, vp]),
+            "ecasq_evaluate": (C.c_int, [vp, i64, vp, i32, vp, sz, pd, vp]),
+            "ecasq_quantize": (C.c_int, [vp, i64, vp, i32, u64, vp, vp, vp, sz, pd, vp]),
+            "ecasq_solve_batched": (C.c_int, [vp, i64, i64, PP, vp, sz, vp, vp, PR, vp]),
+            "ecasq_prepare": (C.c_int, [vp, i64, vp, sz, vp, vp, vp, vp, vp, pi64, vp]),
+        }
+        for name, (res, args) in sig.items():
+            fn = getattr(L, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = L
+        return L
+
+
+def exported_symbols():
+    """Names declared in include/ecasq.h that the loaded library exports."""
+    L = lib()
+    names = []
+    for name in ("ecasq_version", "ecasq_strerror", "ecasq_workspace_size", "ecasq_solve", "ecasq_dp_pass",
+                 "ecasq_dp_tables", "ecasq_refine", "ecasq_evaluate", "ecasq_quantize", "ecasq_solve_batched",
+                 "ecasq_prepare"):
+        if hasattr(L, name):
+            names.append(name)
+    return names
+
+
+# ------------------------------------------------------------------ helpers
+
+def _torch():
+    import torch
+    return torch
+
+
+def _stream():
+    torch = _torch()
+    return C.c_void_p(torch.cuda.current_stream().cuda_stream)
+
+
+def _ptr(t):
+    return C.c_void_p(t.data_ptr())
+
+
+def _dev_f32(x):
+    torch = _torch()
+    if not isinstance(x, torch.Tensor):
+        x = torch.as_tensor(np.ascontiguousarray(x, dtype=np.float32))
+    if x.dtype != torch.float32:
+        raise TypeError("x must be float32")
+    if not x.is_cuda:
+        x = x.cuda()
+    return x.contiguous()
+
+
+def _check(rc, where, ok=(OK,)):
+    if rc not in ok:
+        raise EcasqError(rc, where)
+    return rc
+
+
+def ecasq_workspace_size(d, s, rows=1) -> int:
+    return int(lib().ecasq_workspace_size(int(d), int(s), int(rows)))
+
+
+def workspace(d, s, rows=1):
+    """A device workspace (torch uint8 tensor; CUDA allocations are 256-byte aligned)."""
+    torch = _torch()
+    n = ecasq_workspace_size(d, s, rows)
+    if n == 0:
+        raise EcasqError(EINVAL, "ecasq_workspace_size")
+    return torch.empty(n, dtype=torch.uint8, device="cuda")
+
+
+def make_params(s, budget_bits=0.0, lambda_=-1.0, lambda_lo=0.0, lambda_hi=0.0, search_rounds=0,
+                refine_max_rounds=0, refine_rel_tol=0.0, flags=0):
+    return Params(int(s), int(flags), float(budget_bits), float(lambda_), float(lambda_lo), float(lambda_hi),
+                  int(search_rounds), int(refine_max_rounds), float(refine_rel_tol))
+
+
+# --------------------------------------------------------------- entry points
+
+def ecasq_solve(x, s, budget_bits=0.0, lambda_=-1.0, ws=None, **kw):
+    """Budgeted (or fixed-multiplier) solve; returns (Q tensor [m], result dict)."""
+    torch = _torch()
+    x = _dev_f32(x)
+    d = x.numel()
+    if ws is None:
+        ws = workspace(d, s)
+    prm = make_params(s, budget_bits, lambda_, **kw)
+    Q = torch.zeros(s, dtype=torch.float32, device="cuda")
+    res = Result()
+    rc = lib().ecasq_solve(_ptr(x), d, C.byref(prm), _ptr(ws), ws.numel(), _ptr(Q), C.byref(res), _stream())
+    _check(rc, "ecasq_solve", ok=(OK, EINFEASIBLE))
+    return Q[:res.m].clone(), res.as_dict()
+
+
+def ecasq_dp_pass(x, s, lambdas, flags=0, ws=None):
+    """One DP pass at up to 8 multipliers: (Q [G, s] tensor, m list, metrics [G, 4])."""
+    torch = _torch()
+    x = _dev_f32(x)
+    d = x.numel()
+    lams = np.ascontiguousarray(lambdas, dtype=np.float64)
+    G = lams.size
+    if ws is None:
+        ws = workspace(d, s)
+    Q = torch.zeros((G, s), dtype=torch.float32, device="cuda")
+    m = (C.c_int32 * G)()
+    met = np.zeros(4 * G, np.float64)
+    rc = lib().ecasq_dp_pass(_ptr(x), d, int(s), lams.ctypes.data_as(C.POINTER(C.c_double)), G, int(flags),
+                             _ptr(ws), ws.numel(), _ptr(Q), m, met.ctypes.data_as(C.POINTER(C.c_double)), _stream())
+    _check(rc, "ecasq_dp_pass")
+    return Q, list(m), met.reshape(G, 4)
+
+
+def ecasq_dp_tables(ws, g, s, p_max):
+    """DP tables of multiplier g of the last pass: (dp [(s+1), p] f64, bp [(s+1), p] i32) tensors."""
+    torch = _torch()
+    dp = torch.empty((s + 1) * p_max, dtype=torch.float64, device="cuda")
+    bp = torch.empty((s + 1) * p_max, dtype=torch.int32, device="cuda")
+    p = C.c_int64()
+    rc = lib().ecasq_dp_tables(_ptr(ws), ws.numel(), int(g), _ptr(dp), _ptr(bp), C.byref(p), _stream())
+    _check(rc, "ecasq_dp_tables")
+    n = (s + 1) * p.value
+    return dp[:n].view(s + 1, p.value), bp[:n].view(s + 1, p.value)
+
+
+def ecasq_refine(x, Q, lambda_, budget_bits=-1.0, max_rounds=5, rel_tol=0.0, flags=0, ws=None):
+    """Three-colour refinement (Sec. 6) of Q at multiplier lambda_; returns (Q, result dict)."""
+    torch = _torch()
+    x = _dev_f32(x)
+    d = x.numel()
+    Q = _dev_f32(Q).clone()
+    m = Q.numel()
+    if ws is None:
+        ws = workspace(d, 2)
+    res = Result()
+    rc = lib().ecasq_refine(_ptr(x), d, _ptr(Q), m, float(lambda_), float(budget_bits), int(max_rounds),
+                            float(rel_tol), int(flags), _ptr(ws), ws.numel(), C.byref(res), _stream())
+    _check(rc, "ecasq_refine")
+    return Q, res.as_dict()
+
+
+def ecasq_evaluate(x, Q, ws=None):
+    """(MSE, H(I,B), H(Xhat)) of a codebook Q subset of x."""
+    x = _dev_f32(x)
+    d = x.numel()
+    Q = _dev_f32(Q)
+    if ws is None:
+        ws = workspace(d, 2)
+    out = np.zeros(3, np.float64)
+    rc = lib().ecasq_evaluate(_ptr(x), d, _ptr(Q), Q.numel(), _ptr(ws), ws.numel(),
+                              out.ctypes.data_as(C.POINTER(C.c_double)), _stream())
+    _check(rc, "ecasq_evaluate")
+    return float(out[0]), float(out[1]), float(out[2])
+
+
+def ecasq_quantize(x, Q, seed, ws=None, idx=None, counts=None):
+    """Stochastic quantization (Sec. 2): (idx uint8 tensor, counts tensor, empirical entropy)."""
+    torch = _torch()
+    x = _dev_f32(x)
+    d = x.numel()
+    Q = _dev_f32(Q)
+    m = Q.numel()
+    if ws is None:
+        ws = torch.empty(256, dtype=torch.uint8, device="cuda")
+    if idx is None:
+        idx = torch.empty(d, dtype=torch.uint8, device="cuda")
+    if counts is None:
+        counts = torch.empty(m, dtype=torch.int32, device="cuda")
+    he = C.c_double()
+    rc = lib().ecasq_quantize(_ptr(x), d, _ptr(Q), m, C.c_uint64(int(seed) & 0xFFFFFFFFFFFFFFFF), _ptr(idx),
+                              _ptr(counts), _ptr(ws), ws.numel(), C.byref(he), _stream())
+    _check(rc, "ecasq_quantize")
+    return idx, counts, he.value
+
+
+def ecasq_solve_batched(X, s, budget_bits=0.0, lambda_=-1.0, ws=None, **kw):
+    """Independent budgeted solves of the rows of X [rows, d]: (Q [rows, s], m [rows], results)."""
+    torch = _torch()
+    X = _dev_f32(X)
+    rows, d = X.shape
+    if ws is None:
+        ws = workspace(d, s, rows)
+    prm = make_params(s, budget_bits, lambda_, **kw)
+    Q = torch.zeros((rows, s), dtype=torch.float32, device="cuda")
+    m = torch.zeros(rows, dtype=torch.int32, device="cuda")
+    res = (Result * rows)()
+    rc = lib().ecasq_solve_batched(_ptr(X), rows, d, C.byref(prm), _ptr(ws), ws.numel(), _ptr(Q), _ptr(m), res,
+                                   _stream())
+    _check(rc, "ecasq_solve_batched", ok=(OK, EINFEASIBLE))
+    return Q, m, [r.as_dict() for r in res]
+
+
+def ecasq_prepare(x, ws=None):
+    """Weighted histogram and App. E prefix sums: dict of tensors v, w, N, S, S2 and p."""
+    torch = _torch()
+    x = _dev_f32(x)
+    d = x.numel()
+    if ws is None:
+        ws = workspace(d, 2)
+    v = torch.empty(d, dtype=torch.float32, device="cuda")
+    w = torch.empty(d, dtype=torch.int64, device="cuda")
+    N = torch.empty(d + 1, dtype=torch.int64, device="cuda")
+    S = torch.empty(2 * (d + 1), dtype=torch.float64, device="cuda")
+    S2 = torch.empty(2 * (d + 1), dtype=torch.float64, device="cuda")
+    p = C.c_int64()
+    rc = lib().ecasq_prepare(_ptr(x), d, _ptr(ws), ws.numel(), _ptr(v), _ptr(w), _ptr(N), _ptr(S), _ptr(S2),
+                             C.byref(p), _stream())
+    _check(rc, "ecasq_prepare")
+    p = p.value
+    return dict(p=p, v=v[:p], w=w[:p], N=N[:p + 1], S_hi=S[:p + 1], S_lo=S[p + 1:2 * p + 2],
+                S2_hi=S2[:p + 1], S2_lo=S2[p + 1:2 * p + 2])

@@ -1,0 +1,76 @@
+"""The C-ABI library builds, loads and exports every symbol include/ecasq.h
+declares (no GPU needed: nothing here launches a kernel)."""
+import os
+import re
+
+import pytest
+
+from conftest import ROOT
+
+
+def declared_symbols():
+    txt = open(os.path.join(ROOT, "include", "ecasq.h")).read()
+    return sorted(set(re.findall(r"\b(ecasq_[a-z_]+)\s*\(", txt)))
+
+
+def test_header_declares_the_entry_points():
+    names = declared_symbols()
+    for n in ("ecasq_solve", "ecasq_refine", "ecasq_quantize", "ecasq_solve_batched", "ecasq_workspace_size",
+              "ecasq_dp_pass", "ecasq_strerror"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol():
+    import ctypes
+    from paper_2608_18147_gb300 import native
+    L = native.lib()
+    missing = [n for n in declared_symbols() if not hasattr(L, n)]
+    assert not missing, missing
+    # exported with C linkage (no mangling), visible to dlsym
+    for n in declared_symbols():
+        assert ctypes.cast(getattr(L, n), ctypes.c_void_p).value
+
+
+def test_host_only_calls():
+    from paper_2608_18147_gb300 import native
+    L = native.lib()
+    assert L.ecasq_version() >= 10000
+    assert L.ecasq_strerror(0) == b"ok"
+    assert b"workspace" in L.ecasq_strerror(-4)
+    assert native.ecasq_workspace_size(1024, 8) > 1024 * 4
+    assert native.ecasq_workspace_size(0, 8) == 0
+    assert native.ecasq_workspace_size(100, 1) == 0
+    assert native.ecasq_workspace_size(100, 257) == 0
+    # workspace grows with d and s
+    assert native.ecasq_workspace_size(4096, 16) > native.ecasq_workspace_size(4096, 8)
+    assert native.ecasq_workspace_size(8192, 8) > native.ecasq_workspace_size(4096, 8)
+
+
+def test_bad_arguments_rejected_before_any_launch():
+    import ctypes as C
+    from paper_2608_18147_gb300 import native
+    L = native.lib()
+    prm = native.make_params(1, 2.0)  # s < 2
+    res = native.Result()
+    assert L.ecasq_solve(None, 10, C.byref(prm), None, 0, None, C.byref(res), None) == native.EINVAL
+    prm = native.make_params(8, -1.0)  # budget < 0 in search mode
+    assert L.ecasq_solve(C.c_void_p(256), 10, C.byref(prm), C.c_void_p(256), 1 << 30, C.c_void_p(256),
+                         C.byref(res), None) == native.EINVAL
+    prm = native.make_params(8, 2.0)
+    # misaligned / too small workspace
+    assert L.ecasq_solve(C.c_void_p(256), 10, C.byref(prm), C.c_void_p(257), 1 << 30, C.c_void_p(256),
+                         C.byref(res), None) == native.EWORKSPACE
+    assert L.ecasq_solve(C.c_void_p(256), 10, C.byref(prm), C.c_void_p(256), 16, C.c_void_p(256),
+                         C.byref(res), None) == native.EWORKSPACE
+
+
+def test_product_path_does_not_touch_the_oracle():
+    pkg = os.path.join(ROOT, "paper_2608_18147_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        if "_build" in dirpath:
+            continue
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h")):
+                txt = open(os.path.join(dirpath, f)).read()
+                assert "import oracle" not in txt and "from oracle" not in txt, f
+                assert "ecasq_oracle" not in txt and "liboracle" not in txt, f
