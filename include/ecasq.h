@@ -52,6 +52,7 @@ typedef struct CUstream_st *ecasq_stream_t; /* same type as cudaStream_t */
 #define ECASQ_EXACT_S 1u          /* use exactly s values (eq. apx_final with i = s only) */
 #define ECASQ_NO_REFINE_GUARD 2u  /* refinement may raise H(Xhat) above the budget */
 #define ECASQ_DP_REFERENCE 4u     /* run the fp64 reference DP kernel instead of the fast kernel */
+#define ECASQ_TIME_KERNELS 8u     /* time the DP kernels with CUDA events (ecasq_result_t.dp_kernel_ms) */
 
 typedef struct ecasq_params {
     int32_t s;                 /* codebook cap, 2..256 */
@@ -84,6 +85,9 @@ typedef struct ecasq_result {
     double objective;          /* mse + lambda' * h_exact after refinement, else mse + lambda' * h_surrogate */
     int64_t candidates;        /* min-plus candidates evaluated by the DP (all passes) */
     int64_t rescored;          /* candidates re-scored in fp64 by the fast DP's exact stage */
+    double dp_kernel_ms;       /* with ECASQ_TIME_KERNELS: summed duration of the min-plus kernel launches */
+    int32_t dp_kernel_launches;/* with ECASQ_TIME_KERNELS: number of those launches */
+    int32_t reserved2;
 } ecasq_result_t;
 
 /* Bytes of workspace needed by every entry point below for vectors of up to d
@@ -170,6 +174,10 @@ int ecasq_solve_batched(const float *X, int64_t rows, int64_t d, const ecasq_par
  *   All device, sized for p = d; p_out host.  Synchronises `stream`. */
 int ecasq_prepare(const float *x, int64_t d, void *ws, size_t ws_bytes, float *v, int64_t *w, int64_t *N,
                   double *S, double *S2, int64_t *p_out, ecasq_stream_t stream);
+
+/* Kernels this library has launched in the calling process so far (all
+ * threads, all entry points): a monotone counter for launch accounting. */
+int64_t ecasq_kernel_launches(void);
 
 const char *ecasq_strerror(int status);
 int ecasq_version(void);

@@ -4,6 +4,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <atomic>
 #include <vector>
 
 #include "common.cuh"
@@ -26,12 +27,41 @@ int launch_quantize(const float *x, int64_t d, const float *Q, int m, uint64_t s
                     DevStatus *st, int num_sms, cudaStream_t stream);
 size_t fast_dp_band_bytes(int64_t d, int32_t s);
 
+static std::atomic<long long> g_launches{0};
+void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+
+// CUDA events around the min-plus kernel when ECASQ_TIME_KERNELS is set.
+struct KernelTimer {
+    bool on = false;
+    cudaEvent_t e0 = nullptr, e1 = nullptr;
+    double ms = 0.0;
+    int launches = 0;
+};
+static thread_local KernelTimer g_timer;
+void timer_begin(cudaStream_t st) {
+    if (!g_timer.on) return;
+    if (!g_timer.e0) { cudaEventCreate(&g_timer.e0); cudaEventCreate(&g_timer.e1); }
+    cudaEventRecord(g_timer.e0, st);
+}
+void timer_end(cudaStream_t st) {
+    if (!g_timer.on) return;
+    cudaEventRecord(g_timer.e1, st);
+}
+static void timer_collect() {
+    if (!g_timer.on || !g_timer.e0) return;
+    float ms = 0.f;
+    if (cudaEventSynchronize(g_timer.e1) == cudaSuccess && cudaEventElapsedTime(&ms, g_timer.e0, g_timer.e1) == cudaSuccess) {
+        g_timer.ms += ms;
+        g_timer.launches += 1;
+    }
+}
+
 size_t make_layout(int64_t d, int32_t s, int64_t rows, Layout *L) {
     (void)rows;
     size_t off = 0;
     auto take = [&](size_t bytes) { size_t o = off; off += align256(bytes); return o; };
     int64_t nb = cdiv(d, kSortTile), nbs = cdiv(d, kScanTile);
-    size_t rowsz = (size_t)kMaxG * (size_t)(s + 1) * (size_t)d;
+    size_t rowsz = (size_t)kMaxG * (size_t)(s + 1) * (size_t)table_stride(d);
     L->status = take(sizeof(DevStatus));
     L->keys0 = take(4 * (size_t)d);
     L->keys1 = take(4 * (size_t)d);
@@ -84,6 +114,7 @@ static Prefix make_prefix(void *ws, const Layout &L, int64_t p, int64_t d) {
     P.S2 = wsp<double>(ws, L.S2);
     P.p = p;
     P.d = d;
+    P.ps = table_stride(p);
     return P;
 }
 
@@ -117,6 +148,7 @@ static int dp_pass_prepared(void *ws, const Layout &L, const Prefix &P, int s, c
     else
         rc = launch_dp_fast(P, lamp, G, s, ws, L, st);
     if (rc != ECASQ_OK) return rc;
+    timer_collect();
     rc = launch_traceback_eval(P, G, s, (flags & ECASQ_EXACT_S) ? 1 : 0, dp64, bp, wsp<int32_t>(ws, L.qidx),
                                wsp<int32_t>(ws, L.mcount), wsp<double>(ws, L.metrics), st);
     if (rc != ECASQ_OK) return rc;
@@ -239,6 +271,8 @@ extern "C" {
 
 int ecasq_version(void) { return 10000; }
 
+int64_t ecasq_kernel_launches(void) { return (int64_t)g_launches.load(); }
+
 const char *ecasq_strerror(int status) {
     switch (status) {
         case ECASQ_OK: return "ok";
@@ -335,10 +369,12 @@ int ecasq_dp_tables(void *ws, size_t ws_bytes, int32_t g, double *dp_out, int32_
     make_layout(h.last_d, h.last_s, 1, &L);
     int rc = check_ws(ws, ws_bytes, L);
     if (rc) return rc;
-    size_t n = (size_t)(h.last_s + 1) * (size_t)h.p;
-    size_t off = (size_t)g * n;
-    ECASQ_CUDA_TRY(cudaMemcpyAsync(dp_out, wsp<double>(ws, L.dp64) + off, 8 * n, cudaMemcpyDeviceToDevice, st));
-    ECASQ_CUDA_TRY(cudaMemcpyAsync(bp_out, wsp<int32_t>(ws, L.bp) + off, 4 * n, cudaMemcpyDeviceToDevice, st));
+    size_t ps = (size_t)table_stride(h.p), rowsn = (size_t)(h.last_s + 1);
+    size_t off = (size_t)g * rowsn * ps;
+    ECASQ_CUDA_TRY(cudaMemcpy2DAsync(dp_out, 8 * (size_t)h.p, wsp<double>(ws, L.dp64) + off, 8 * ps, 8 * (size_t)h.p,
+                                     rowsn, cudaMemcpyDeviceToDevice, st));
+    ECASQ_CUDA_TRY(cudaMemcpy2DAsync(bp_out, 4 * (size_t)h.p, wsp<int32_t>(ws, L.bp) + off, 4 * ps, 4 * (size_t)h.p,
+                                     rowsn, cudaMemcpyDeviceToDevice, st));
     ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
     *p_out = h.p;
     return ECASQ_OK;
@@ -381,6 +417,9 @@ int ecasq_solve(const float *x, int64_t d, const ecasq_params_t *prm, void *ws, 
     if (!x || !Q || d < 1 || d >= ((int64_t)1 << 31) || !params_ok(prm)) return ECASQ_EINVAL;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     const int s = prm->s;
+    g_timer.on = (prm->flags & ECASQ_TIME_KERNELS) != 0;
+    g_timer.ms = 0.0;
+    g_timer.launches = 0;
     Layout L;
     make_layout(d, s, 1, &L);
     int rc = check_ws(ws, ws_bytes, L);
@@ -489,6 +528,8 @@ int ecasq_solve(const float *x, int64_t d, const ecasq_params_t *prm, void *ws, 
     if (rc) return rc;
     double obj = prm->refine_max_rounds > 0 ? ev[0] + lamp * ev[2] : ev[0] + lamp * ev[1];
     fill_result(res, status, (int)a.size(), d, p, lam, n2, ev, obj, passes, nlam, rr, cand, read_rescored(ws, st));
+    if (res) { res->dp_kernel_ms = g_timer.ms; res->dp_kernel_launches = g_timer.launches; }
+    g_timer.on = false;
     return status;
 }
 

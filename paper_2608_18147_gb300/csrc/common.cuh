@@ -24,6 +24,9 @@ constexpr int kScanTile = 1024; // elements per prefix-scan block
 #define ECASQ_LAUNCH_CHECK() ECASQ_CUDA_TRY(cudaGetLastError())
 
 __host__ __device__ static inline int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
+// Row stride of every DP table: p rounded up to 64 entries, so each row starts
+// 256-byte aligned (the fast kernel copies rows with 16-byte cp.async).
+__host__ __device__ static inline int64_t table_stride(int64_t p) { return (p + 63) & ~(int64_t)63; }
 static inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 // ---------------------------------------------------------------- workspace
@@ -33,13 +36,15 @@ struct DevStatus {
     int32_t nonfinite;    // x held NaN/Inf
     int32_t range_err;    // quantize: entry outside [Q0, Qm-1]; refine: Q not in X
     int32_t timeout;      // a bounded wait ran out
-    int32_t pad;
+    int32_t bound_viol;   // fast DP: fp32 minima outside their certified error bound
     double norm2;         // ||X||^2 (hi part of the double-double sum)
     int64_t rescored;     // fast DP: candidates re-scored in fp64
     int64_t overflow;     // fast DP: outputs that needed the full-rescan path
     int32_t last_s;       // s and G of the last DP pass (for ecasq_dp_tables)
     int32_t last_G;
     int64_t last_d;       // d of the last DP pass
+    int64_t members;      // fast DP: band members found (all outputs)
+    int64_t big_bands;    // fast DP: outputs with more members than the inline list holds
 };
 
 struct Layout {
@@ -126,6 +131,7 @@ struct Prefix {
     const double *S2;
     int64_t p;
     int64_t d;
+    int64_t ps;           // DP-table row stride, table_stride(p)
 };
 
 __device__ __forceinline__ dd load_dd(const double *a, int64_t p, int64_t t) { return {a[t], a[p + 1 + t]}; }
@@ -158,6 +164,9 @@ __device__ __forceinline__ double phi_exact(const Prefix &P, double U, double D,
 }
 
 // -------------------------------------------------------------- host helpers
+// Kernels launched by this library in this process (all threads).
+void note_launch();
+
 int prepare_device(const float *x, int64_t d, void *ws, const Layout &L, cudaStream_t st, int64_t *p_host,
                    double *norm2_host);
 

@@ -1,19 +1,779 @@
-// dp_fast.cu -- fast approximate-DP kernel (Sec. 5).  Placeholder that routes
-// to the fp64 reference kernel until the fp32-filter kernel lands.
+// dp_fast.cu -- fast approximate DP (Sec. 5, eqs. apx_base / apx_rec / apx_final).
+//
+// Three stages per DP pass, for up to 8 multipliers at once:
+//
+// 1. k_wavefront: an fp32 filter over the whole (k, j) triangle with every
+//    layer i = 3..s fused.  A persistent CTA owns a block of 64 columns j and
+//    sweeps 64-wide tiles of k in increasing order; the tile k-block K may be
+//    used as soon as column block K has published all its layers (a flag with
+//    release/acquire order, bounded waits).  Two producer warps turn each tile
+//    into interval costs C[k,j] and Phi[k,j] (App. E quantities rebuilt with
+//    compensated fp32 recurrences that add one point at a time, all terms
+//    non-negative, from a double-double anchor per tile and column); the
+//    consumer warps evaluate dp(i-1,k) + C + lambda' Phi for their (layer,
+//    column, multiplier) outputs with packed f32x2 adds and 3-input mins.
+//    Per output the kernel keeps the fp32 minimum and up to two runs of
+//    consecutive tiles whose minimum came within the certified error band of it.
+// 2. k_extract: for every output, re-evaluate the listed tiles bit-identically
+//    and keep the members k whose fp32 value lies within the band (up to 8
+//    inline; the count is kept either way).
+// 3. k_exact_layer (one launch per layer): re-score the members in binary64
+//    with double-double interval costs (the reference formulas) and take the
+//    lowest k among exact minima: dp64, bp.  Outputs with more members, or
+//    whose tile runs overflowed, re-scan their tiles in fp32 and re-score the
+//    members they meet on the fly -- never a full binary64 scan.
+//
+// The fp32 band: with u = 2^-24, each fp32 candidate value carries a relative
+// error of at most eps_i = max(eps_{i-1}, 20u) + 1.0001u (eps_2 = 1.0001u), so
+// the exact argmin k* satisfies val32(k*) <= m32 (1 + eps_i)/(1 - eps_i).  The
+// 20u budget for one interval cost: compensated sums (~1u), point terms
+// (<= 3.5u for C), correctly rounded reciprocal and products (~3u), and the
+// documented error of __log2f (2^-22 absolute on [0.5,2), 2 ulp elsewhere),
+// amplified at most 2.44x through h(y) = -y log2 y for y <= 1/2; values
+// y > 1/2 are evaluated through 1 - y computed from the complementary mass.
+// The exact stage re-checks |m32 - dp64| <= eps_i dp64 for every output and
+// counts violations.
+#include <algorithm>
+
 #include "common.cuh"
 
 namespace ecasq {
 
 int launch_dp_reference(const Prefix &P, const double *lamp, int G, int s, double *dp64, int32_t *bp,
                         cudaStream_t st);
+void timer_begin(cudaStream_t st);
+void timer_end(cudaStream_t st);
 
-size_t fast_dp_band_bytes(int64_t d, int32_t s) {
-    (void)d; (void)s;
-    return 256;
+constexpr int BJ = 64;         // columns per block
+constexpr int BK = 64;         // k per tile
+constexpr int LPT = 7;         // layers per consumer thread
+constexpr int JPT = 4;         // columns per consumer thread (stride 16)
+constexpr int NJQ = BJ / JPT;  // 16 column groups
+constexpr int NPROD = 64;      // producer threads: one per column of the block
+constexpr int PSTR = BK + 4;   // padded row stride (floats) of the interval-cost buffers
+constexpr int MAXCONS = 256;
+constexpr int NMEM = 8;        // members kept inline per output
+constexpr int64_t kMaxFastP = (int64_t)1 << 20;
+constexpr uint32_t kSpinLimit = 1u << 26;
+
+// Band word (64 bits): bits 0-1 number of tile runs (0..2), bit 2 overflow; run r
+// (r = 0, 1) at bit 3 + 19 r: first tile (14 bits) and length - 1 (5 bits, <= 32 tiles).
+// Tiles arrive in increasing order of K (the diagonal block, K = J, last).
+__device__ __forceinline__ uint64_t band_reset(uint32_t K) { return 1ull | ((uint64_t)K << 3); }
+__device__ __forceinline__ uint64_t band_append(uint64_t w, uint32_t K) {
+    uint32_t c = (uint32_t)(w & 3u);
+    if (w & 4u) return w;
+    if (c == 0) return band_reset(K);
+    int sh = 3 + 19 * (int)(c - 1);
+    uint32_t st = (uint32_t)(w >> sh) & 0x3FFFu, len = ((uint32_t)(w >> (sh + 14)) & 31u) + 1u;
+    if (K == st + len && len < 32u) return w + (1ull << (sh + 14));  // extend the last run
+    if (c == 1) return (w & ~3ull) | 2ull | ((uint64_t)K << 22);     // open the second run
+    return w | 4ull;
+}
+__device__ __forceinline__ void band_run(uint64_t w, int r, uint32_t &st, uint32_t &len) {
+    int sh = 3 + 19 * r;
+    st = (uint32_t)(w >> sh) & 0x3FFFu;
+    len = ((uint32_t)(w >> (sh + 14)) & 31u) + 1u;
 }
 
-int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, const Layout &L, cudaStream_t st) {
-    return launch_dp_reference(P, lamp, G, s, wsp<double>(ws, L.dp64), wsp<int32_t>(ws, L.bp), st);
+// Per-pass constants, copied once to device memory (kernels index them at run time).
+struct FastParams {
+    float tau[kMaxS + 1];  // per layer: band factor 2 eps_i / (1 - eps_i), with margin
+    float eps[kMaxS + 1];  // per layer: eps_i
+    float lam32[kMaxG];    // lambda'_g rounded to fp32
+    double lam64[kMaxG];
+};
+
+struct FastArgs {
+    const float *v;
+    const float *wf;       // multiplicities as fp32 (exact below 2^24)
+    const int64_t *N;
+    const double *S, *S2;  // hi [p+1] | lo [p+1]
+    int64_t p, d;
+    int64_t ps;            // table row stride (multiple of 64)
+    float invd;            // correctly rounded 1/d
+    int G, s, lgc, Gc, nsplit, nJ, ncons;
+    const FastParams *prm;
+    float *dp32;           // [G][s+1][p]
+    uint64_t *band;        // [G][s+1][ps] tile runs per output
+    int32_t *mcnt;         // [G][s+1][ps] band members (-1: runs overflowed)
+    int32_t *members;      // [G][s+1][ps][NMEM]
+    int *done;             // [nsplit][nJ]
+    int *ticket;
+    int *abort_flag;
+    DevStatus *st;
+};
+
+__device__ __forceinline__ size_t oidx(const FastArgs &a, int g, int i, int64_t j) {
+    return ((size_t)g * (size_t)(a.s + 1) + (size_t)i) * (size_t)a.ps + (size_t)j;
+}
+
+// ------------------------------------------------------------ fp32 numerics
+
+// Sum2 step (Ogita, Rump, Oishi 2005): x + c carries the running sum of
+// non-negative terms; TwoSum keeps the rounding error of each addition.
+__device__ __forceinline__ void comp_add(float &x, float &c, float t) {
+    float s = __fadd_rn(x, t);
+    float bb = __fsub_rn(s, x);
+    float e = __fadd_rn(__fsub_rn(x, __fsub_rn(s, bb)), __fsub_rn(t, bb));
+    x = s;
+    c = __fadd_rn(c, e);
+}
+
+// -log2(1 - z) for z in [0, 1/2], from log(1 - z) = -2 atanh(z / (2 - z)).
+__device__ __forceinline__ float neg_log2_1m(float z) {
+    float t = __fdiv_rn(z, __fsub_rn(2.0f, z));  // t in [0, 1/3]
+    float t2 = __fmul_rn(t, t);
+    // 2 (t + t^3/3 + ... + t^15/15) / ln 2; the next term is below 2^-26 t
+    float q = 1.0f / 15.0f;
+    q = __fmaf_rn(q, t2, 1.0f / 13.0f);
+    q = __fmaf_rn(q, t2, 1.0f / 11.0f);
+    q = __fmaf_rn(q, t2, 1.0f / 9.0f);
+    q = __fmaf_rn(q, t2, 1.0f / 7.0f);
+    q = __fmaf_rn(q, t2, 1.0f / 5.0f);
+    q = __fmaf_rn(q, t2, 1.0f / 3.0f);
+    q = __fmaf_rn(q, t2, 1.0f);
+    return __fmul_rn(__fmul_rn(t, q), 2.8853900817779268f);  // 2 / ln 2
+}
+
+// h(y) = -y log2 y with y = m / d; `comp` = (d - m) / d computed from the
+// complementary mass, used when y > 1/2.
+__device__ __forceinline__ float h32(float y, float comp) {
+    if (!(y > 0.0f)) return 0.0f;
+    if (y <= 0.5f) return fmaxf(__fmul_rn(y, -__log2f(y)), 0.0f);
+    return fmaxf(__fmul_rn(y, neg_log2_1m(fminf(comp, 0.5f))), 0.0f);
+}
+
+// Recurrence state of one column j while k descends: N = sum w, E = sum w (v_j - v_t),
+// A = sum w (v_t - v_k), C = sum w (v_j - v_t)(v_t - v_k) over t in (k, j].
+struct Rec {
+    float N, E, Ec, A, Ac, C, Cc;
+};
+
+// Interval cost of (k, j) from the state: C and Phi = h(U/d) + h(D/d) (Sec. 5).
+__device__ __forceinline__ void rec_emit(const Rec &r, float vj, float vk, float d_f, float invd, float &Cout,
+                                         float &Phi) {
+    float Eu = __fadd_rn(r.E, r.Ec), Au = __fadd_rn(r.A, r.Ac);
+    Cout = __fadd_rn(fmaxf(__fadd_rn(r.C, r.Cc), 0.0f), 0.0f);  // >= +0 (no -0)
+    float L = __fsub_rn(vj, vk);
+    float rL = __frcp_rn(L);
+    float D = __fmul_rn(Eu, rL), U = __fmul_rn(Au, rL);
+    float yU = __fmul_rn(U, invd), yD = __fmul_rn(D, invd);
+    float out = __fsub_rn(d_f, r.N);  // mass outside the interval (exact)
+    float cU = __fmul_rn(__fadd_rn(out, D), invd), cD = __fmul_rn(__fadd_rn(out, U), invd);
+    Phi = __fadd_rn(__fadd_rn(h32(yU, cU), h32(yD, cD)), 0.0f);  // >= +0 (no -0)
+}
+
+// Add point t = k+1 (moving from k+1 to k): vt = v_{k+1}, wt = w_{k+1}, dk = v_{k+1} - v_k.
+__device__ __forceinline__ void rec_step(Rec &r, float vj, float vt, float wt, float dk) {
+    r.N = __fadd_rn(r.N, wt);
+    comp_add(r.E, r.Ec, __fmul_rn(wt, __fsub_rn(vj, vt)));
+    float Eu = __fadd_rn(r.E, r.Ec);
+    comp_add(r.A, r.Ac, __fmul_rn(dk, r.N));
+    comp_add(r.C, r.Cc, __fmul_rn(dk, Eu));
+}
+
+// Anchor of a tile: the state of pair (k, j) from double-double prefix sums.
+__device__ __forceinline__ void split_f(dd x, float &hi, float &lo) {
+    double t = dd_round(x);
+    hi = __double2float_rn(t);
+    lo = __double2float_rn(__dadd_rn(__dsub_rn(x.hi, (double)hi), x.lo));
+}
+
+__device__ void rec_anchor(const FastArgs &a, int64_t k, int64_t j, Rec &r) {
+    int64_t n = a.N[j + 1] - a.N[k + 1];
+    double nd = (double)n;
+    dd dS = dd_sub(load_dd(a.S, a.p, j + 1), load_dd(a.S, a.p, k + 1));
+    dd dS2 = dd_sub(load_dd(a.S2, a.p, j + 1), load_dd(a.S2, a.p, k + 1));
+    double vk = (double)a.v[k], vj = (double)a.v[j];
+    dd A = dd_sub(dS, two_prod(vk, nd));
+    dd E = dd_sub(two_prod(vj, nd), dS);
+    dd Cd = dd_sub(dd_sub(dd_mul(two_sum(vk, vj), dS), dS2), two_prod(__dmul_rn(vk, vj), nd));
+    r.N = (float)n;
+    split_f(E, r.E, r.Ec);
+    split_f(A, r.A, r.Ac);
+    split_f(Cd, r.C, r.Cc);
+}
+
+__device__ __forceinline__ Rec rec_empty() { return {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f}; }
+
+// ------------------------------------------------------------ named barriers
+__device__ __forceinline__ void bar_sync(int id, int n) { asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory"); }
+__device__ __forceinline__ void bar_arrive(int id, int n) { asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(n) : "memory"); }
+enum { BAR_FULL = 1, BAR_EMPTY = 3, BAR_CONS = 5, BAR_PROD = 6 };
+
+__device__ __forceinline__ int ld_acquire(const int *p) {
+    int v;
+    asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ void st_release(int *p, int v) {
+    asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// packed fp32 pair arithmetic (sm_100+)
+__device__ __forceinline__ float2 add2(float2 a, float2 b) {
+    float2 d;
+    asm("{\n\t.reg .b64 ra, rb, rd;\n\tmov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+        "add.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(d.x), "=f"(d.y) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return d;
+}
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
+    float2 d;
+    asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\tmov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+        "mov.b64 rc, {%6, %7};\n\tfma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(d.x), "=f"(d.y) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+    return d;
+}
+__device__ __forceinline__ float min3(float a, float b, float c) {
+    float d;
+    asm("min.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
+// ------------------------------------------------------------ shared memory
+struct TileMeta {
+    int J, K, split, kind;  // kind: 0 off-diagonal, 1 diagonal, 2 stop
+};
+
+struct __align__(16) Smem {
+    float C[2][BJ][PSTR];
+    float Phi[2][BJ][PSTR];
+    float diag[2][kMaxG][BJ];             // dp32 of the previous / current layer inside the column
+    float kv[BK], kw[BK], kd[BK];         // v_k (k0..k0+63), w_{k+1}, v_{k+1} - v_k
+    TileMeta meta[2];
+    int ticket;
+    int pad[3];
+    // followed by dp32 slices [2][Gc * (s-2)][BK] (dynamic)
+};
+
+// ------------------------------------------------------------------ kernel
+__global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    Smem &S = *reinterpret_cast<Smem *>(smem_raw);
+    float *sDP = reinterpret_cast<float *>(smem_raw + sizeof(Smem));
+    const int L = a.s - 2;                // layers 3..s
+    const int rowsDP = a.Gc * L;          // staged dp32 rows per tile (layers 2..s-1)
+    const int tid = threadIdx.x;
+    const int nall = NPROD + a.ncons;
+
+    if (tid < NPROD) {
+        // =========================== producer warps ===========================
+        const int jl = tid;  // column within the block
+        uint32_t n = 0;      // tile sequence number
+        const float d_f = (float)a.d;
+        for (;;) {
+            if (tid == 0) S.ticket = atomicAdd(a.ticket, 1);
+            bar_sync(BAR_PROD, NPROD);
+            int t = S.ticket;
+            bar_sync(BAR_PROD, NPROD);
+            bool stop = t >= a.nJ * a.nsplit;
+            int J = stop ? 0 : t / a.nsplit, split = stop ? 0 : t % a.nsplit;
+            int ntiles = stop ? 1 : J + 1;
+            for (int K = 0; K < ntiles; K++) {
+                int b = n & 1;
+                if (n >= 2) bar_sync(BAR_EMPTY + b, nall);
+                if (stop) {
+                    if (tid == 0) S.meta[b] = {0, 0, 0, 2};
+                    bar_arrive(BAR_FULL + b, nall);
+                    n++;
+                    break;
+                }
+                bool diag = (K == J);
+                int64_t k0 = (int64_t)K * BK, j0 = (int64_t)J * BJ;
+                int64_t j = j0 + jl;
+                // wait for column block K (bounded); the diagonal needs nothing
+                if (!diag && tid == 0) {
+                    const int *flag = a.done + (size_t)split * a.nJ + K;
+                    uint32_t spins = 0;
+                    while (ld_acquire(flag) == 0) {
+                        if (*(volatile int *)a.abort_flag) break;
+                        if (++spins > kSpinLimit) {
+                            a.st->timeout = 1;
+                            atomicExch(a.abort_flag, 1);
+                            break;
+                        }
+                        __nanosleep(64);
+                    }
+                }
+                bar_sync(BAR_PROD, NPROD);
+                // per-k constants of the tile
+                {
+                    int64_t k = k0 + jl;
+                    S.kv[jl] = k < a.p ? a.v[k] : 0.f;
+                    S.kw[jl] = (k + 1 < a.p) ? a.wf[k + 1] : 0.f;
+                    S.kd[jl] = (k + 1 < a.p) ? __fsub_rn(a.v[k + 1], a.v[k]) : 0.f;
+                }
+                // dp32 slice of rows (g, layer 2..s-1) for k in the tile (cp.async, L2 only)
+                if (!diag) {
+                    int gbase = split * a.Gc;
+                    int n16 = rowsDP * (BK / 4);
+                    float *dst = sDP + (size_t)b * rowsDP * BK;
+                    for (int q = tid; q < n16; q += NPROD) {
+                        int row = q / (BK / 4), c4 = q % (BK / 4);
+                        int gl = row / L, li = row % L;  // layer index li -> dp row i = 2 + li
+                        int g = gbase + gl;
+                        float *sp = dst + (size_t)row * BK + c4 * 4;
+                        if (g < a.G) {
+                            const float *gp = a.dp32 + oidx(a, g, 2 + li, k0 + c4 * 4);
+                            unsigned sa = (unsigned)__cvta_generic_to_shared(sp);
+                            asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(sa), "l"(gp) : "memory");
+                        } else {
+                            *reinterpret_cast<float4 *>(sp) = make_float4(CUDART_INF_F, CUDART_INF_F, CUDART_INF_F,
+                                                                          CUDART_INF_F);
+                        }
+                    }
+                    asm volatile("cp.async.commit_group;" ::: "memory");
+                }
+                bar_sync(BAR_PROD, NPROD);
+                // interval costs of column j for k in the tile (descending k)
+                float (*Cr)[PSTR] = S.C[b];
+                float (*Pr)[PSTR] = S.Phi[b];
+                if (j < a.p) {
+                    float vj = a.v[j];
+                    Rec r;
+                    int kl_hi;
+                    if (diag) {
+                        r = rec_empty();
+                        kl_hi = (int)(j - j0) - 1;  // k = j-1 first
+                        // state for k = j: empty; step to k = j-1 adds t = j
+                        for (int kl = BK - 1; kl > kl_hi; kl--) { Cr[jl][kl] = CUDART_INF_F; Pr[jl][kl] = 0.f; }
+                        for (int kl = kl_hi; kl >= 0; kl--) {
+                            rec_step(r, vj, S.kv[kl + 1], S.kw[kl], S.kd[kl]);  // kl + 1 <= 63
+                            float c, ph;
+                            rec_emit(r, vj, S.kv[kl], d_f, a.invd, c, ph);
+                            Cr[jl][kl] = c; Pr[jl][kl] = ph;
+                        }
+                    } else {
+                        rec_anchor(a, k0 + BK - 1, j, r);
+                        float c, ph;
+                        rec_emit(r, vj, S.kv[BK - 1], d_f, a.invd, c, ph);
+                        Cr[jl][BK - 1] = c; Pr[jl][BK - 1] = ph;
+                        for (int kl = BK - 2; kl >= 0; kl--) {
+                            rec_step(r, vj, S.kv[kl + 1], S.kw[kl], S.kd[kl]);
+                            rec_emit(r, vj, S.kv[kl], d_f, a.invd, c, ph);
+                            Cr[jl][kl] = c; Pr[jl][kl] = ph;
+                        }
+                    }
+                } else {
+                    for (int kl = 0; kl < BK; kl++) { Cr[jl][kl] = CUDART_INF_F; Pr[jl][kl] = 0.f; }
+                }
+                if (!diag) asm volatile("cp.async.wait_all;" ::: "memory");
+                if (tid == 0) S.meta[b] = {J, K, split, diag ? 1 : 0};
+                bar_arrive(BAR_FULL + b, nall);
+                n++;
+            }
+            if (stop) break;
+        }
+        // drain: wait until the consumers released the last two buffers
+        for (uint32_t q = (n >= 2 ? n - 2 : 0); q < n; q++) bar_sync(BAR_EMPTY + (q & 1), nall);
+        return;
+    }
+
+    // ============================= consumer warps =============================
+    const int ct = tid - NPROD;
+    const int jq = ct % NJQ;
+    const int rest = ct / NJQ;
+    const int lg = rest % a.lgc;
+    const int gl = rest / a.lgc;
+    const bool active = ct < a.Gc * a.lgc * NJQ;
+    uint32_t n = 0;
+    float best[LPT][JPT];
+    uint64_t word[LPT][JPT];
+    for (;;) {
+        int b = n & 1;
+        bar_sync(BAR_FULL + b, nall);
+        TileMeta m = S.meta[b];
+        if (m.kind == 2) { bar_arrive(BAR_EMPTY + b, nall); break; }
+        const int g = m.split * a.Gc + gl;
+        const bool own = active && g < a.G;
+        const int64_t j0 = (int64_t)m.J * BJ;
+        const float lam = own ? a.prm->lam32[g] : 0.f;
+        if (m.K == 0) {
+#pragma unroll
+            for (int l = 0; l < LPT; l++)
+#pragma unroll
+                for (int q = 0; q < JPT; q++) { best[l][q] = CUDART_INF_F; word[l][q] = 0ull; }
+        }
+        if (m.kind == 0) {
+            // Candidate values are >= +0, so their bit patterns order like the
+            // floats: the running minimum is kept as int bits and updated with
+            // integer min (ALU pipe) next to the packed adds (FMA pipe).
+            int cm[LPT][JPT];
+#pragma unroll
+            for (int l = 0; l < LPT; l++)
+#pragma unroll
+                for (int q = 0; q < JPT; q++) cm[l][q] = 0x7f800000;  // +inf
+            if (own) {
+                const float *dpb = sDP + (size_t)b * rowsDP * BK + (size_t)gl * L * BK;
+                float2 lam2 = make_float2(lam, lam);
+#pragma unroll 1
+                for (int kk = 0; kk < BK; kk += 4) {
+                    float2 W[JPT][2];
+#pragma unroll
+                    for (int q = 0; q < JPT; q++) {
+                        float4 c4 = *reinterpret_cast<const float4 *>(&S.C[b][jq + NJQ * q][kk]);
+                        float4 f4 = *reinterpret_cast<const float4 *>(&S.Phi[b][jq + NJQ * q][kk]);
+                        W[q][0] = fma2(lam2, make_float2(f4.x, f4.y), make_float2(c4.x, c4.y));
+                        W[q][1] = fma2(lam2, make_float2(f4.z, f4.w), make_float2(c4.z, c4.w));
+                    }
+#pragma unroll
+                    for (int l = 0; l < LPT; l++) {
+                        int li = lg * LPT + l;  // layer i = 3 + li uses dp row 2 + li
+                        if (li < L) {
+                            float4 d4 = *reinterpret_cast<const float4 *>(dpb + (size_t)li * BK + kk);
+                            float2 da = make_float2(d4.x, d4.y), db = make_float2(d4.z, d4.w);
+#pragma unroll
+                            for (int q = 0; q < JPT; q++) {
+                                float2 t0 = add2(da, W[q][0]);
+                                float2 t1 = add2(db, W[q][1]);
+                                int c = min(min(cm[l][q], __float_as_int(t0.x)), __float_as_int(t0.y));
+                                cm[l][q] = min(min(c, __float_as_int(t1.x)), __float_as_int(t1.y));
+                            }
+                        }
+                    }
+                }
+                // band bookkeeping for this tile
+#pragma unroll
+                for (int l = 0; l < LPT; l++) {
+                    int li = lg * LPT + l;
+                    if (li < L) {
+                        float tau = a.prm->tau[3 + li];
+#pragma unroll
+                        for (int q = 0; q < JPT; q++) {
+                            float c = __int_as_float(cm[l][q]), bb = best[l][q];
+                            if (c < CUDART_INF_F) {
+                                float T = __fmul_rn(bb, tau);
+                                if (c < __fsub_rn(bb, T)) { word[l][q] = band_reset((uint32_t)m.K); best[l][q] = c; }
+                                else if (c <= __fadd_rn(bb, T)) { word[l][q] = band_append(word[l][q], (uint32_t)m.K); best[l][q] = fminf(bb, c); }
+                            }
+                        }
+                    }
+                }
+            }
+            bar_arrive(BAR_EMPTY + b, nall);
+        } else {
+            // ---------------- diagonal block: layers in order ----------------
+            // previous-layer values inside the column: layer 2 from the base kernel
+            for (int q = ct; q < a.Gc * BJ; q += a.ncons) {
+                int gg = q / BJ, jj = q % BJ;
+                int g2 = m.split * a.Gc + gg;
+                int64_t jx = j0 + jj;
+                S.diag[0][gg][jj] = (g2 < a.G && jx < a.p) ? a.dp32[oidx(a, g2, 2, jx)] : CUDART_INF_F;
+            }
+            bar_sync(BAR_CONS, a.ncons);
+            int cur = 0;
+            for (int li = 0; li < L; li++) {
+                const int i = 3 + li;
+                const int l = li - lg * LPT;
+                if (own && l >= 0 && l < LPT) {
+#pragma unroll
+                    for (int lx = 0; lx < LPT; lx++) {
+                        if (lx != l) continue;
+#pragma unroll
+                        for (int q = 0; q < JPT; q++) {
+                            int jl = jq + NJQ * q;
+                            int64_t j = j0 + jl;
+                            float c = CUDART_INF_F;
+                            for (int kl = 0; kl < jl; kl++) {
+                                float W = __fmaf_rn(lam, S.Phi[b][jl][kl], S.C[b][jl][kl]);
+                                c = fminf(c, __fadd_rn(S.diag[cur][gl][kl], W));
+                            }
+                            float bb = best[lx][q];
+                            if (c < CUDART_INF_F) {
+                                float T = __fmul_rn(bb, a.prm->tau[i]);
+                                if (c < __fsub_rn(bb, T)) { word[lx][q] = band_reset((uint32_t)m.J); bb = c; }
+                                else if (c <= __fadd_rn(bb, T)) { word[lx][q] = band_append(word[lx][q], (uint32_t)m.J); bb = fminf(bb, c); }
+                            }
+                            best[lx][q] = bb;
+                            S.diag[cur ^ 1][gl][jl] = bb;
+                            if (j < a.p) {
+                                a.dp32[oidx(a, g, i, j)] = bb;
+                                a.band[oidx(a, g, i, j)] = word[lx][q];
+                            }
+                        }
+                    }
+                }
+                bar_sync(BAR_CONS, a.ncons);
+                cur ^= 1;
+            }
+            // publish the column block (all layers, all multipliers of this split)
+            if (ct == 0) {
+                __threadfence();
+                st_release(a.done + (size_t)m.split * a.nJ + m.J, 1);
+            }
+            bar_arrive(BAR_EMPTY + b, nall);
+        }
+        n++;
+    }
+}
+
+// ------------------------------------------------------------ base layer
+// eq. apx_base for every multiplier: exact dp64, bp and the fp32 copy; all
+// other rows cleared (dp64 = +inf, bp = -1, dp32 = +inf).
+__global__ void k_fast_clear(double *dp64, int32_t *bp, float *dp32, size_t n) {
+    size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+    size_t stride = (size_t)gridDim.x * blockDim.x;
+    for (; i < n; i += stride) { dp64[i] = CUDART_INF; bp[i] = -1; dp32[i] = CUDART_INF_F; }
+}
+
+__global__ void k_fast_base(Prefix P, FastArgs a, double *dp64, int32_t *bp) {
+    int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x + 1;
+    if (j >= P.p) return;
+    double C, U, D;
+    pair_exact(P, 0, j, C, U, D);
+    double phi = phi_exact(P, U, D, true);
+    for (int g = 0; g < a.G; g++) {
+        double v = __dadd_rn(C, __dmul_rn(a.prm->lam64[g], phi));
+        dp64[oidx(a, g, 2, j)] = v;
+        bp[oidx(a, g, 2, j)] = 0;
+        a.dp32[oidx(a, g, 2, j)] = __fadd_rn(__double2float_rn(v), 0.0f);  // >= +0 (no -0)
+    }
+}
+
+// ------------------------------------------------------------- extraction
+// fp32 value of candidate k for output (g, i, j), bit-identical to the wavefront.
+__device__ __forceinline__ float cand32(float dprev, float lam, float C, float Phi) {
+    return __fadd_rn(dprev, __fmaf_rn(lam, Phi, C));
+}
+
+// Visit the candidates k of tile K for output (g, i, j) in the wavefront's fp32
+// arithmetic (k descending) and call f(k) for every k with value <= thr.
+template <typename F>
+__device__ void visit_tile(const FastArgs &a, int g, int i, int64_t j, int64_t K, float thr, F &&f) {
+    int64_t J = j / BJ, j0 = J * BJ, k0 = K * BK;
+    float vj = a.v[j];
+    float lam = a.prm->lam32[g];
+    const float d_f = (float)a.d;
+    const float *prev = a.dp32 + oidx(a, g, i - 1, 0);
+    Rec r;
+    int64_t khi;
+    float c, ph;
+    if (K == J) {
+        r = rec_empty();
+        khi = j;  // state of the empty interval (j, j]
+    } else {
+        khi = k0 + BK - 1;
+        rec_anchor(a, khi, j, r);
+        rec_emit(r, vj, a.v[khi], d_f, a.invd, c, ph);
+        if (cand32(prev[khi], lam, c, ph) <= thr) f(khi);
+    }
+    for (int64_t k = khi - 1; k >= k0; k--) {
+        rec_step(r, vj, a.v[k + 1], a.wf[k + 1], __fsub_rn(a.v[k + 1], a.v[k]));
+        rec_emit(r, vj, a.v[k], d_f, a.invd, c, ph);
+        if (cand32(prev[k], lam, c, ph) <= thr) f(k);
+    }
+}
+
+// Tiles listed by a band word (in increasing order), or all tiles 0..J when it overflowed.
+template <typename F>
+__device__ void visit_band(const FastArgs &a, int g, int i, int64_t j, uint64_t w, float thr, F &&f) {
+    int64_t J = j / BJ;
+    if (w & 4u) {
+        for (int64_t K = 0; K <= J; K++) visit_tile(a, g, i, j, K, thr, f);
+        return;
+    }
+    int nr = (int)(w & 3u);
+    for (int r = 0; r < nr; r++) {
+        uint32_t st, len;
+        band_run(w, r, st, len);
+        for (uint32_t K = st; K < st + len; K++) visit_tile(a, g, i, j, (int64_t)K, thr, f);
+    }
+}
+
+__device__ __forceinline__ float band_threshold(const FastArgs &a, int i, float m32) {
+    return __fadd_rn(m32, __fmul_rn(m32, a.prm->tau[i]));
+}
+
+__global__ void k_extract(FastArgs a) {
+    int64_t tot = (int64_t)a.G * (a.s - 2) * a.p;
+    int64_t id = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    unsigned long long nmem = 0, nbig = 0, nover = 0;
+    for (; id < tot; id += stride) {
+        int64_t j = id % a.p;
+        int64_t r = id / a.p;
+        int i = 3 + (int)(r % (a.s - 2));
+        int g = (int)(r / (a.s - 2));
+        if (j < i - 1) continue;
+        size_t o = oidx(a, g, i, j);
+        float m32 = a.dp32[o];
+        if (!(m32 < CUDART_INF_F)) { a.mcnt[o] = 0; continue; }
+        uint64_t w = a.band[o];
+        if (w & 4u) { a.mcnt[o] = -1; nover++; continue; }
+        int32_t *mem = a.members + o * NMEM;
+        int cnt = 0;
+        visit_band(a, g, i, j, w, band_threshold(a, i, m32), [&](int64_t k) {
+            if (cnt < NMEM) mem[cnt] = (int32_t)k;
+            cnt++;
+        });
+        a.mcnt[o] = cnt;
+        nmem += cnt;
+        nbig += cnt > NMEM;
+    }
+    if (nmem) atomicAdd((unsigned long long *)&a.st->members, nmem);
+    if (nbig) atomicAdd((unsigned long long *)&a.st->big_bands, nbig);
+    if (nover) atomicAdd((unsigned long long *)&a.st->overflow, nover);
+}
+
+// ----------------------------------------------------------- exact layer
+__device__ __forceinline__ void exact_candidate(const Prefix &P, const double *prev, int64_t k, int64_t j,
+                                                double lam, double &best, int32_t &arg) {
+    double C, U, D;
+    pair_exact(P, k, j, C, U, D);
+    double c = __dadd_rn(prev[k], __dadd_rn(C, __dmul_rn(lam, phi_exact(P, U, D, false))));
+    if (c < best || (c == best && k < arg)) { best = c; arg = (int32_t)k; }
+}
+
+__global__ void k_exact_layer(Prefix P, FastArgs a, int i, double *dp64, int32_t *bp) {
+    int64_t tot = (int64_t)a.G * a.p;
+    int64_t id = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (id >= tot) return;
+    int64_t j = id % a.p;
+    int g = (int)(id / a.p);
+    if (j < i - 1) return;
+    size_t o = oidx(a, g, i, j);
+    float m32 = a.dp32[o];
+    if (!(m32 < CUDART_INF_F)) return;
+    int cnt = a.mcnt[o];
+    double lam = a.prm->lam64[g];
+    const double *prev = dp64 + oidx(a, g, i - 1, 0);
+    double best = CUDART_INF;
+    int32_t arg = INT32_MAX;
+    long long nres = 0;
+    if (cnt >= 0 && cnt <= NMEM) {
+        const int32_t *mem = a.members + o * NMEM;
+        for (int q = 0; q < cnt; q++) exact_candidate(P, prev, mem[q], j, lam, best, arg);
+        nres = cnt;
+    } else {
+        // many members or overflowed runs: re-scan the tiles in fp32, re-score members on the fly
+        visit_band(a, g, i, j, a.band[o], band_threshold(a, i, m32), [&](int64_t k) {
+            exact_candidate(P, prev, k, j, lam, best, arg);
+            nres++;
+        });
+    }
+    if (arg == INT32_MAX) arg = -1;
+    dp64[o] = best;
+    bp[o] = arg;
+    // certificate check: the fp32 minimum must lie within eps_i of the exact one
+    double e = (double)a.prm->eps[i];
+    if (!(fabs((double)m32 - best) <= e * best * 1.0001)) atomicAdd(&a.st->bound_viol, 1);
+    atomicAdd((unsigned long long *)&a.st->rescored, (unsigned long long)nres);
+}
+
+// ------------------------------------------------------------------ host
+__global__ void k_weights_f32(const int64_t *w, float *wf, int64_t p) {
+    int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < p) wf[i] = (float)w[i];
+}
+
+__global__ void k_store_params(FastParams prm, FastParams *dst) {
+    if (threadIdx.x == 0 && blockIdx.x == 0) *dst = prm;
+}
+
+size_t fast_dp_band_bytes(int64_t d, int32_t s) {
+    size_t rows = (size_t)kMaxG * (size_t)(s + 1) * (size_t)table_stride(d);
+    size_t nJ = (size_t)cdiv(d, BJ);
+    return align256(8 * rows) + align256(4 * rows) + align256(4 * NMEM * rows) +
+           align256(4 * (size_t)kMaxG * nJ + 64) + align256(sizeof(FastParams));
+}
+
+static size_t smem_bytes(int Gc, int s) { return sizeof(Smem) + (size_t)2 * Gc * (s - 2) * BK * sizeof(float); }
+
+// Certified band factors (see the file header): eps_2 = 1.0001u, eps_i = max(eps_{i-1}, 20u) + 1.0001u.
+static void band_factors(int s, FastParams &fp) {
+    const double u = 1.0 / 16777216.0;
+    for (int i = 0; i <= kMaxS; i++) { fp.tau[i] = 0.f; fp.eps[i] = 0.f; }
+    double eps = 1.0001 * u;
+    fp.eps[2] = (float)eps;
+    for (int i = 3; i <= s; i++) {
+        eps = std::max(eps, 20.0 * u) + 1.0001 * u;
+        fp.eps[i] = (float)eps;
+        fp.tau[i] = (float)(2.0 * eps / (1.0 - eps) * 1.001 + 2.0 * u);
+    }
+}
+
+int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, const Layout &Lw, cudaStream_t st) {
+    double *dp64 = wsp<double>(ws, Lw.dp64);
+    int32_t *bp = wsp<int32_t>(ws, Lw.bp);
+    // small inputs, very large ones and huge counts take the reference kernel
+    if (P.p < 2 * BJ || P.p > kMaxFastP || P.d >= (1 << 24) || s < 3 || cdiv(s - 2, LPT) * NJQ > MAXCONS)
+        return launch_dp_reference(P, lamp, G, s, dp64, bp, st);
+    FastArgs a{};
+    a.v = P.v;
+    a.N = P.N;
+    a.S = P.S;
+    a.S2 = P.S2;
+    a.p = P.p;
+    a.d = P.d;
+    a.ps = P.ps;
+    a.invd = 1.0f / (float)P.d;  // IEEE division on the host: correctly rounded
+    a.G = G;
+    a.s = s;
+    a.lgc = (int)cdiv(s - 2, LPT);
+    a.Gc = std::max(1, std::min(G, MAXCONS / (a.lgc * NJQ)));
+    a.nsplit = (int)cdiv(G, a.Gc);
+    a.nJ = (int)cdiv(P.p, BJ);
+    a.ncons = (int)cdiv((int64_t)a.Gc * a.lgc * NJQ, 32) * 32;
+    FastParams fp;
+    band_factors(s, fp);
+    for (int g = 0; g < kMaxG; g++) {
+        fp.lam64[g] = g < G ? lamp[g] : 0.0;
+        fp.lam32[g] = (float)fp.lam64[g];
+    }
+    size_t rows = (size_t)kMaxG * (size_t)(s + 1) * (size_t)table_stride(Lw.d);
+    char *base = wsp<char>(ws, Lw.band);
+    a.dp32 = wsp<float>(ws, Lw.dp32);
+    a.band = reinterpret_cast<uint64_t *>(base);
+    base += align256(8 * rows);
+    a.mcnt = reinterpret_cast<int32_t *>(base);
+    base += align256(4 * rows);
+    a.members = reinterpret_cast<int32_t *>(base);
+    base += align256(4 * NMEM * rows);
+    int *flags = reinterpret_cast<int *>(base);
+    base += align256(4 * (size_t)kMaxG * (size_t)cdiv(Lw.d, BJ) + 64);
+    FastParams *dprm = reinterpret_cast<FastParams *>(base);
+    a.prm = dprm;
+    a.done = flags;
+    a.ticket = flags + (size_t)kMaxG * a.nJ;
+    a.abort_flag = a.ticket + 1;
+    a.st = wsp<DevStatus>(ws, Lw.status);
+    float *wf = wsp<float>(ws, Lw.keys1);  // the sort's ping-pong buffer is free now
+    a.wf = wf;
+    size_t n = (size_t)G * (size_t)(s + 1) * (size_t)P.ps;
+    note_launch();
+    k_store_params<<<1, 32, 0, st>>>(fp, dprm);
+    note_launch();
+    k_fast_clear<<<4096, 256, 0, st>>>(dp64, bp, a.dp32, n);
+    note_launch();
+    k_weights_f32<<<(unsigned)cdiv(P.p, 256), 256, 0, st>>>(P.w, wf, P.p);
+    ECASQ_LAUNCH_CHECK();
+    ECASQ_CUDA_TRY(cudaMemsetAsync(flags, 0, sizeof(int) * ((size_t)kMaxG * a.nJ + 2), st));
+    note_launch();
+    k_fast_base<<<(unsigned)cdiv(P.p - 1, 128), 128, 0, st>>>(P, a, dp64, bp);
+    ECASQ_LAUNCH_CHECK();
+    size_t smem = smem_bytes(a.Gc, s);
+    ECASQ_CUDA_TRY(cudaFuncSetAttribute(k_wavefront, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    int dev = 0, nsm = 0;
+    ECASQ_CUDA_TRY(cudaGetDevice(&dev));
+    ECASQ_CUDA_TRY(cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev));
+    int grid = std::min(nsm, a.nJ * a.nsplit);
+    timer_begin(st);
+    note_launch();
+    k_wavefront<<<grid, NPROD + a.ncons, smem, st>>>(a);
+    timer_end(st);
+    ECASQ_LAUNCH_CHECK();
+    int64_t tot = (int64_t)G * (s - 2) * P.p;
+    note_launch();
+    k_extract<<<(unsigned)std::min<int64_t>(cdiv(tot, 128), (int64_t)nsm * 64), 128, 0, st>>>(a);
+    ECASQ_LAUNCH_CHECK();
+    for (int i = 3; i <= s; i++) {
+        note_launch();
+        k_exact_layer<<<(unsigned)cdiv((int64_t)G * P.p, 128), 128, 0, st>>>(P, a, i, dp64, bp);
+        ECASQ_LAUNCH_CHECK();
+    }
+    return ECASQ_OK;
 }
 
 }  // namespace ecasq

@@ -9,6 +9,9 @@
 
 namespace ecasq {
 
+void timer_begin(cudaStream_t st);
+void timer_end(cudaStream_t st);
+
 struct Lams { double v[kMaxG]; };
 
 __device__ __forceinline__ size_t dp_at(int g, int i, int64_t j, int s, int64_t p) {
@@ -31,8 +34,8 @@ __global__ void k_dp_base(Prefix P, Lams lam, int G, int s, double *dp64, int32_
     pair_exact(P, 0, j, C, U, D);
     double phi = phi_exact(P, U, D, true);
     for (int g = 0; g < G; g++) {
-        dp64[dp_at(g, 2, j, s, P.p)] = __dadd_rn(C, __dmul_rn(lam.v[g], phi));
-        bp[dp_at(g, 2, j, s, P.p)] = 0;
+        dp64[dp_at(g, 2, j, s, P.ps)] = __dadd_rn(C, __dmul_rn(lam.v[g], phi));
+        bp[dp_at(g, 2, j, s, P.ps)] = 0;
     }
 }
 
@@ -55,15 +58,15 @@ __global__ void __launch_bounds__(128) k_dp_layer_ref(Prefix P, Lams lam, int G,
 #pragma unroll
         for (int g = 0; g < kMaxG; g++) {
             if (g < G) {
-                double prev = dp64[dp_at(g, i - 1, k, s, P.p)];
+                double prev = dp64[dp_at(g, i - 1, k, s, P.ps)];
                 double c = __dadd_rn(prev, __dadd_rn(C, __dmul_rn(lam.v[g], phi)));
                 if (c < best[g]) { best[g] = c; arg[g] = (int32_t)k; }
             }
         }
     }
     for (int g = 0; g < G; g++) {
-        dp64[dp_at(g, i, j, s, P.p)] = best[g];
-        bp[dp_at(g, i, j, s, P.p)] = arg[g];
+        dp64[dp_at(g, i, j, s, P.ps)] = best[g];
+        bp[dp_at(g, i, j, s, P.ps)] = arg[g];
     }
 }
 
@@ -114,7 +117,7 @@ __global__ void k_traceback_eval(Prefix P, int G, int s, int exact_s, const doub
         int istar = -1;
         double best = CUDART_INF;
         for (int i = exact_s ? s : 2; i <= s; i++) {
-            double v = dp64[dp_at(g, i, p - 1, s, p)];
+            double v = dp64[dp_at(g, i, p - 1, s, P.ps)];
             if (v < best) { best = v; istar = i; }
         }
         if (istar < 0) {
@@ -123,7 +126,7 @@ __global__ void k_traceback_eval(Prefix P, int G, int s, int exact_s, const doub
             int64_t j = p - 1;
             a[istar - 1] = (int32_t)j;
             for (int i = istar; i >= 3; i--) {
-                j = bp[dp_at(g, i, j, s, p)];
+                j = bp[dp_at(g, i, j, s, P.ps)];
                 a[i - 2] = (int32_t)j;
             }
             a[0] = 0;
@@ -175,28 +178,35 @@ int launch_dp_reference(const Prefix &P, const double *lamp, int G, int s, doubl
                         cudaStream_t st) {
     Lams lam{};
     for (int g = 0; g < G; g++) lam.v[g] = lamp[g];
-    k_dp_clear<<<4096, 256, 0, st>>>(dp64, bp, G, s, P.p);
+    note_launch();
+    k_dp_clear<<<4096, 256, 0, st>>>(dp64, bp, G, s, P.ps);
     ECASQ_LAUNCH_CHECK();
     if (P.p >= 2) {
+        note_launch();
         k_dp_base<<<(unsigned)cdiv(P.p - 1, 128), 128, 0, st>>>(P, lam, G, s, dp64, bp);
         ECASQ_LAUNCH_CHECK();
     }
+    timer_begin(st);
     for (int i = 3; i <= s; i++) {
         if (P.p < i) break;
+        note_launch();
         k_dp_layer_ref<<<(unsigned)cdiv(P.p, 128), 128, 0, st>>>(P, lam, G, s, i, dp64, bp);
         ECASQ_LAUNCH_CHECK();
     }
+    timer_end(st);
     return ECASQ_OK;
 }
 
 int launch_traceback_eval(const Prefix &P, int G, int s, int exact_s, const double *dp64, const int32_t *bp,
                           int32_t *qidx, int32_t *mcount, double *metrics, cudaStream_t st) {
+    note_launch();
     k_traceback_eval<<<G, 32, 0, st>>>(P, G, s, exact_s, dp64, bp, qidx, mcount, metrics);
     ECASQ_LAUNCH_CHECK();
     return ECASQ_OK;
 }
 
 int launch_eval_codebook(const Prefix &P, const int32_t *a, int m, double *out3, cudaStream_t st) {
+    note_launch();
     k_eval_codebook<<<1, 32, 0, st>>>(P, a, m, out3);
     ECASQ_LAUNCH_CHECK();
     return ECASQ_OK;
@@ -204,12 +214,14 @@ int launch_eval_codebook(const Prefix &P, const int32_t *a, int m, double *out3,
 
 int launch_gather_q(const float *v, const int32_t *qidx, const int32_t *mcount, int G, int s, float *Q,
                     cudaStream_t st) {
+    note_launch();
     k_gather_q<<<G, 64, 0, st>>>(v, qidx, mcount, s, Q);
     ECASQ_LAUNCH_CHECK();
     return ECASQ_OK;
 }
 
 int launch_locate_q(const float *v, int64_t p, const float *Q, int m, int32_t *a, DevStatus *ds, cudaStream_t st) {
+    note_launch();
     k_locate_q<<<1, 256, 0, st>>>(v, p, Q, m, a, ds);
     ECASQ_LAUNCH_CHECK();
     return ECASQ_OK;

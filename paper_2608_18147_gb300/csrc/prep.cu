@@ -260,12 +260,16 @@ int prepare_device(const float *x, int64_t d, void *ws, const Layout &L, cudaStr
     uint32_t *cnt = wsp<uint32_t>(ws, L.rcount);
     ECASQ_CUDA_TRY(cudaMemsetAsync(st, 0, sizeof(DevStatus), stream));
     int nb = (int)cdiv(d, kSortTile);
+    note_launch();
     k_make_keys<<<(unsigned)std::min<int64_t>(cdiv(d, 256), 4096), 256, 0, stream>>>(x, d, k0, st);
     ECASQ_LAUNCH_CHECK();
     uint32_t *a = k0, *b = k1;
     for (int shift = 0; shift < 32; shift += 8) {
+        note_launch();
         k_radix_count<<<nb, 256, 0, stream>>>(a, d, shift, cnt, nb);
+        note_launch();
         k_scan_u32<<<1, 1024, 0, stream>>>(cnt, (int64_t)256 * nb);
+        note_launch();
         k_radix_scatter<<<nb, 256, 0, stream>>>(a, b, d, shift, cnt, nb);
         ECASQ_LAUNCH_CHECK();
         uint32_t *t = a; a = b; b = t;
@@ -276,11 +280,15 @@ int prepare_device(const float *x, int64_t d, void *ws, const Layout &L, cudaStr
     // scratch copies of N/S/S2 with lo parts at offset d+1 live in keys1 / dp area
     double *Stmp = wsp<double>(ws, L.dp64);
     double *S2tmp = Stmp + 2 * (d + 1);
+    note_launch();
     k_hist_partials<<<(unsigned)nbs, 256, 0, stream>>>(a, d, part);
+    note_launch();
     k_hist_scan_partials<<<1, 32, 0, stream>>>(part, nbs);
+    note_launch();
     k_hist_fill<<<(unsigned)nbs, 256, 0, stream>>>(a, d, part, wsp<float>(ws, L.v), wsp<int64_t>(ws, L.N), Stmp,
                                                  S2tmp, st, d);
     ECASQ_LAUNCH_CHECK();
+    note_launch();
     k_hist_finish<<<(unsigned)std::min<int64_t>(cdiv(d + 1, 256), 4096), 256, 0, stream>>>(
         wsp<int64_t>(ws, L.N), wsp<int64_t>(ws, L.w), Stmp, S2tmp, st, d, wsp<double>(ws, L.S),
         wsp<double>(ws, L.S2));

@@ -82,6 +82,7 @@ int launch_quantize(const float *x, int64_t d, const float *Q, int m, uint64_t s
     int64_t groups = cdiv(d, 4);
     int64_t blocks = std::min<int64_t>(cdiv(groups, 256), (int64_t)num_sms * 8);
     if (blocks < 1) blocks = 1;
+    note_launch();
     k_quantize<<<(unsigned)blocks, 256, 0, stream>>>(x, d, Q, m, seed, idx, counts, st);
     ECASQ_LAUNCH_CHECK();
     return ECASQ_OK;

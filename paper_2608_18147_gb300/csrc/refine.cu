@@ -84,6 +84,7 @@ int launch_refine_colour(const Prefix &P, const int32_t *a, int m, int colour, d
     int nblk = (m - 2 >= l0) ? (m - 2 - l0) / 3 + 1 : 0;
     *nblocks_out = nblk;
     if (nblk == 0) return ECASQ_OK;
+    note_launch();
     k_refine_colour<<<nblk, 256, 0, st>>>(P, a, m, colour, lamp, a_new, moved);
     ECASQ_LAUNCH_CHECK();
     return ECASQ_OK;

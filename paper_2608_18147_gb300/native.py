@@ -17,7 +17,7 @@ import numpy as np
 from . import build as _build
 
 OK, EINVAL, ENONFINITE, EINFEASIBLE, EWORKSPACE, ECUDA, ETIMEOUT, ERANGE = 0, -1, -2, -3, -4, -5, -6, -7
-EXACT_S, NO_REFINE_GUARD, DP_REFERENCE = 1, 2, 4
+EXACT_S, NO_REFINE_GUARD, DP_REFERENCE, TIME_KERNELS = 1, 2, 4, 8
 
 _lock = threading.Lock()
 _lib = None
@@ -34,7 +34,8 @@ class Result(C.Structure):
                 ("refine_rounds", C.c_int32), ("reserved", C.c_int32), ("d", C.c_int64), ("p", C.c_int64),
                 ("lambda_", C.c_double), ("lambda_prime", C.c_double), ("norm2", C.c_double), ("mse", C.c_double),
                 ("vnmse", C.c_double), ("h_surrogate", C.c_double), ("h_exact", C.c_double), ("r_tot", C.c_double),
-                ("objective", C.c_double), ("candidates", C.c_int64), ("rescored", C.c_int64)]
+                ("objective", C.c_double), ("candidates", C.c_int64), ("rescored", C.c_int64),
+                ("dp_kernel_ms", C.c_double), ("dp_kernel_launches", C.c_int32), ("reserved2", C.c_int32)]
 
     def as_dict(self):
         out = {}
@@ -81,6 +82,7 @@ def lib():
             "ecasq_quantize": (C.c_int, [vp, i64, vp, i32, u64, vp, vp, vp, sz, pd, vp]),
             "ecasq_solve_batched": (C.c_int, [vp, i64, i64, PP, vp, sz, vp, vp, PR, vp]),
             "ecasq_prepare": (C.c_int, [vp, i64, vp, sz, vp, vp, vp, vp, vp, pi64, vp]),
+            "ecasq_kernel_launches": (i64, []),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -96,7 +98,7 @@ def exported_symbols():
     names = []
     for name in ("ecasq_version", "ecasq_strerror", "ecasq_workspace_size", "ecasq_solve", "ecasq_dp_pass",
                  "ecasq_dp_tables", "ecasq_refine", "ecasq_evaluate", "ecasq_quantize", "ecasq_solve_batched",
-                 "ecasq_prepare"):
+                 "ecasq_prepare", "ecasq_kernel_launches"):
         if hasattr(L, name):
             names.append(name)
     return names
@@ -133,6 +135,17 @@ def _check(rc, where, ok=(OK,)):
     if rc not in ok:
         raise EcasqError(rc, where)
     return rc
+
+
+def ws_status(ws):
+    """Counters the library leaves at the start of a workspace after a call
+    (unique values, device-side flags, fast-DP statistics)."""
+    raw = ws[:80].cpu().numpy().tobytes()
+    (p, nonfinite, range_err, timeout, bound_viol, norm2, rescored, overflow, last_s, last_G, last_d, members,
+     big_bands) = __import__("struct").unpack("<qiiiidqqiiqqq", raw)
+    return dict(p=p, nonfinite=nonfinite, range_err=range_err, timeout=timeout, bound_viol=bound_viol, norm2=norm2,
+                rescored=rescored, overflow=overflow, last_s=last_s, last_G=last_G, last_d=last_d, members=members,
+                big_bands=big_bands)
 
 
 def ecasq_workspace_size(d, s, rows=1) -> int:
@@ -287,3 +300,8 @@ def ecasq_prepare(x, ws=None):
     p = p.value
     return dict(p=p, v=v[:p], w=w[:p], N=N[:p + 1], S_hi=S[:p + 1], S_lo=S[p + 1:2 * p + 2],
                 S2_hi=S2[:p + 1], S2_lo=S2[p + 1:2 * p + 2])
+
+
+def ecasq_kernel_launches() -> int:
+    """Kernels the library has launched in this process so far."""
+    return int(lib().ecasq_kernel_launches())

@@ -96,9 +96,61 @@ def _dp_parity(E, oracle_mod, x, s, lams, flags, exact_s=False):
 
 
 @pytest.mark.parametrize("lams", [[0.0], [0.0, 1e-4, 0.01, 0.05, 0.2, 0.6, 2.0, 40.0]])
-def test_dp_reference_parity_normal1024(E, oracle_mod, lams):
+@pytest.mark.parametrize("flags_name", ["DP_REFERENCE", "FAST"])
+def test_dp_parity_normal1024(E, oracle_mod, lams, flags_name):
     x = workloads.normal(1024, 0)
-    _dp_parity(E, oracle_mod, x, 8, lams, E.DP_REFERENCE)
+    _dp_parity(E, oracle_mod, x, 8, lams, getattr(E, flags_name, 0))
+
+
+@pytest.mark.parametrize("name,s,lams", [
+    ("ragged2049", 6, [0.0, 0.03, 0.4]),
+    ("ragged2049", 16, [0.0, 1e-3, 0.05, 0.4, 3.0]),
+    ("dups", 8, [0.0, 0.1]),
+    ("tiny_offset", 9, [0.0, 0.02, 0.5]),
+    ("normal1024", 3, [0.0, 0.3]),
+    ("normal1024", 23, [0.0, 0.01, 0.2, 1.0, 5.0, 20.0, 100.0]),
+])
+def test_dp_fast_parity(E, oracle_mod, name, s, lams):
+    """The fast kernel (fp32 filter + certified band + exact re-scoring) against the oracle."""
+    x = inputs_small()[name]
+    _dp_parity(E, oracle_mod, x, s, lams, 0)
+
+
+def test_dp_fast_matches_reference_16k(E, oracle_mod):
+    """d = 16384 (signed LogNormal), s = 16, 8 multipliers: fast vs reference DP tables, and
+    sampled decisions against the oracle given the GPU's previous layer."""
+    x = workloads.signed_lognormal(16384, 0)
+    s = 16
+    lams = [0.0, 1e-5, 1e-3, 0.01, 0.05, 0.2, 1.0, 10.0]
+    wsf, wsr = E.workspace(x.size, s), E.workspace(x.size, s)
+    Qf, mf, metf = E.ecasq_dp_pass(x, s, lams, flags=0, ws=wsf)
+    stf = E.native.ws_status(wsf)
+    Qr, mr, metr = E.ecasq_dp_pass(x, s, lams, flags=E.DP_REFERENCE, ws=wsr)
+    assert stf["bound_viol"] == 0 and stf["timeout"] == 0
+    H = oracle_mod.Hist(x)
+    rng = np.random.default_rng(5)
+    for g in range(len(lams)):
+        dpf, bpf = [t.cpu().numpy() for t in E.ecasq_dp_tables(wsf, g, s, x.size)]
+        dpr, bpr = [t.cpu().numpy() for t in E.ecasq_dp_tables(wsr, g, s, x.size)]
+        np.testing.assert_array_equal(np.isfinite(dpf), np.isfinite(dpr))
+        fin = np.isfinite(dpr)
+        np.testing.assert_allclose(dpf[fin], dpr[fin], rtol=DP_RTOL)
+        mism = np.argwhere((bpf != bpr) & (bpr >= 0))
+        lp = lams[g] * H.norm2
+        for i, j in mism[:50]:  # any disagreement must be a near-tie for the oracle
+            best, arg, second = H.dp_decision(dpr[i - 1], int(i), int(j), lp)
+            vf = H.dp_candidate(dpr[i - 1][bpf[i, j]], bpf[i, j], j, lp)
+            assert vf <= best * (1 + TIE)
+        assert mism.shape[0] <= 1e-6 * bpr.size + 5
+        for _ in range(6):  # sampled decisions straight from the oracle's formulas
+            i = int(rng.integers(3, s + 1))
+            j = int(rng.integers(i - 1, x.size if H.p == x.size else H.p))
+            best, arg, second = H.dp_decision(dpf[i - 1], i, j, lp)
+            assert dpf[i, j] == pytest.approx(best, rel=DP_RTOL)
+            if second > best * (1 + TIE):
+                assert bpf[i, j] == arg
+        assert mf[g] == mr[g]
+        np.testing.assert_array_equal(Qf[g].cpu().numpy(), Qr[g].cpu().numpy())
 
 
 @pytest.mark.parametrize("name", ["dups", "ragged2049", "tiny_offset", "two_values"])
@@ -122,9 +174,9 @@ def test_dp_reference_parity_s_exceeds_p(E, oracle_mod):
 
 # --------------------------------------------------------------- the search
 
-@pytest.mark.parametrize("flags_name", ["DP_REFERENCE"])
+@pytest.mark.parametrize("flags_name", ["DP_REFERENCE", "FAST"])
 def test_solve_parity_normal1024(E, oracle_mod, flags_name):
-    flags = getattr(E, flags_name)
+    flags = getattr(E, flags_name, 0)
     x = workloads.normal(1024, 0)
     Q, res = E.ecasq_solve(x, 8, budget_bits=2.0, flags=flags)
     o = oracle_mod.solve_budget(x, 8, 2.0)
@@ -138,7 +190,7 @@ def test_solve_parity_normal1024(E, oracle_mod, flags_name):
 
 def test_solve_with_refinement_parity(E, oracle_mod):
     x = workloads.normal(1024, 0)
-    Q, res = E.ecasq_solve(x, 8, budget_bits=2.0, refine_max_rounds=5, refine_rel_tol=1e-9, flags=E.DP_REFERENCE)
+    Q, res = E.ecasq_solve(x, 8, budget_bits=2.0, refine_max_rounds=5, refine_rel_tol=1e-9)
     o = oracle_mod.solve_budget(x, 8, 2.0, refine_rounds=5, refine_tol=1e-9)
     np.testing.assert_array_equal(Q.cpu().numpy(), o["Q"])
     assert res["refine_rounds"] == o.get("refine_rounds", 0)
