@@ -53,6 +53,7 @@ typedef struct CUstream_st *ecasq_stream_t; /* same type as cudaStream_t */
 #define ECASQ_NO_REFINE_GUARD 2u  /* refinement may raise H(Xhat) above the budget */
 #define ECASQ_DP_REFERENCE 4u     /* run the fp64 reference DP kernel instead of the fast kernel */
 #define ECASQ_TIME_KERNELS 8u     /* time the DP kernels with CUDA events (ecasq_result_t.dp_kernel_ms) */
+#define ECASQ_EXACT_TABLES 16u    /* resolve every DP output exactly (default: only what eq. apx_final and the traceback read) */
 
 typedef struct ecasq_params {
     int32_t s;                 /* codebook cap, 2..256 */
@@ -125,7 +126,11 @@ int ecasq_dp_pass(const float *x, int64_t d, int32_t s, const double *lambdas, i
 /* Copy the DP tables of multiplier g of the last ecasq_dp_pass on this
  * workspace: dp (fp64) and bp (int32, lowest argmin k; -1 where undefined),
  * each row-major [(s+1) x p], rows 0 and 1 unused, +inf / -1 where the layer
- * is undefined.  dp_out, bp_out device; p_out host.  Synchronises `stream`. */
+ * is undefined.  The fast kernel resolves exactly the outputs the final
+ * selection and traceback depend on; elsewhere dp holds its fp32-filtered
+ * value and bp = -2, unless the pass ran with ECASQ_EXACT_TABLES (or
+ * ECASQ_DP_REFERENCE).  dp_out, bp_out device; p_out host.  Synchronises
+ * `stream`. */
 int ecasq_dp_tables(void *ws, size_t ws_bytes, int32_t g, double *dp_out, int32_t *bp_out, int64_t *p_out,
                     ecasq_stream_t stream);
 

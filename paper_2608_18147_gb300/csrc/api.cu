@@ -14,7 +14,8 @@ namespace ecasq {
 // launchers defined in the other translation units
 int launch_dp_reference(const Prefix &P, const double *lamp, int G, int s, double *dp64, int32_t *bp,
                         cudaStream_t st);
-int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, const Layout &L, cudaStream_t st);
+int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, const Layout &L, cudaStream_t st,
+                   bool exact_s, bool exact_tables);
 int launch_traceback_eval(const Prefix &P, int G, int s, int exact_s, const double *dp64, const int32_t *bp,
                           int32_t *qidx, int32_t *mcount, double *metrics, cudaStream_t st);
 int launch_eval_codebook(const Prefix &P, const int32_t *a, int m, double *out3, cudaStream_t st);
@@ -22,7 +23,8 @@ int launch_gather_q(const float *v, const int32_t *qidx, const int32_t *mcount, 
                     cudaStream_t st);
 int launch_locate_q(const float *v, int64_t p, const float *Q, int m, int32_t *a, DevStatus *ds, cudaStream_t st);
 int launch_refine_colour(const Prefix &P, const int32_t *a, int m, int colour, double lamp, int32_t *a_new,
-                         int32_t *moved, cudaStream_t st, int *nblocks_out);
+                         int32_t *moved, void *part_buf, cudaStream_t st, int *nblocks_out);
+size_t refine_scratch_bytes(int64_t d);
 int launch_quantize(const float *x, int64_t d, const float *Q, int m, uint64_t seed, uint8_t *idx, uint32_t *counts,
                     DevStatus *st, int num_sms, cudaStream_t stream);
 size_t fast_dp_band_bytes(int64_t d, int32_t s);
@@ -81,6 +83,7 @@ size_t make_layout(int64_t d, int32_t s, int64_t rows, Layout *L) {
     L->metrics = take(8 * (size_t)kMaxG * 4);
     L->lam = take(8 * (size_t)kMaxG);
     L->refine = take(4 * 2 * kMaxS + 256 + 8 * 8);
+    L->refine_part = take(refine_scratch_bytes(d));
     L->band = take(fast_dp_band_bytes(d, s));
     L->total = off;
     L->d = d;
@@ -146,7 +149,7 @@ static int dp_pass_prepared(void *ws, const Layout &L, const Prefix &P, int s, c
     if (flags & ECASQ_DP_REFERENCE)
         rc = launch_dp_reference(P, lamp, G, s, dp64, bp, st);
     else
-        rc = launch_dp_fast(P, lamp, G, s, ws, L, st);
+        rc = launch_dp_fast(P, lamp, G, s, ws, L, st, (flags & ECASQ_EXACT_S) != 0, (flags & ECASQ_EXACT_TABLES) != 0);
     if (rc != ECASQ_OK) return rc;
     timer_collect();
     rc = launch_traceback_eval(P, G, s, (flags & ECASQ_EXACT_S) ? 1 : 0, dp64, bp, wsp<int32_t>(ws, L.qidx),
@@ -218,7 +221,7 @@ static int refine_device(void *ws, const Layout &L, const Prefix &P, std::vector
             ECASQ_CUDA_TRY(cudaMemcpyAsync(an, a, sizeof(int32_t) * m, cudaMemcpyDeviceToDevice, st));
             ECASQ_CUDA_TRY(cudaMemsetAsync(moved, 0, sizeof(int32_t), st));
             int nblk = 0;
-            rc = launch_refine_colour(P, a, m, col, lamp, an, moved, st, &nblk);
+            rc = launch_refine_colour(P, a, m, col, lamp, an, moved, wsp<void>(ws, L.refine_part), st, &nblk);
             if (rc != ECASQ_OK) return rc;
             if (nblk == 0) continue;
             int32_t mv = 0;

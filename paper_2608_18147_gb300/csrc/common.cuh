@@ -65,6 +65,7 @@ struct Layout {
     size_t metrics;        // double [G 4]
     size_t lam;            // double [G]   lambda' of each multiplier
     size_t refine;         // refinement scratch
+    size_t refine_part;    // refinement per-chunk partial minima
     size_t band;           // fast DP band lists
     size_t total;
     int64_t d;

@@ -14,25 +14,34 @@
 //    column, multiplier) outputs with packed f32x2 adds and 3-input mins.
 //    Per output the kernel keeps the fp32 minimum and up to two runs of
 //    consecutive tiles whose minimum came within the certified error band of it.
-// 2. k_extract: for every output, re-evaluate the listed tiles bit-identically
-//    and keep the members k whose fp32 value lies within the band (up to 8
-//    inline; the count is kept either way).
-// 3. k_exact_layer (one launch per layer): re-score the members in binary64
-//    with double-double interval costs (the reference formulas) and take the
-//    lowest k among exact minima: dp64, bp.  Outputs with more members, or
-//    whose tile runs overflowed, re-scan their tiles in fp32 and re-score the
-//    members they meet on the fly -- never a full binary64 scan.
+// 2. k_need_layer (layers s down to 3): the outputs whose exact value the
+//    answer depends on.  eq. apx_final needs dp(i, p-1) for every i; an output
+//    resolved exactly needs the exact values of its band members in the layer
+//    below.  For every needed output the kernel re-evaluates its listed tiles
+//    bit-identically, keeps the members k whose fp32 value lies within the
+//    band (up to 8 inline, the count either way) and marks (i-1, k) needed.
+//    With ECASQ_EXACT_TABLES every output is needed.
+// 3. k_exact_layer (layers 3 up to s): re-score the members of every needed
+//    output in binary64 with double-double interval costs (the reference
+//    formulas) and take the lowest k among exact minima: dp64, bp.  Outputs
+//    with more members, or whose tile runs overflowed, re-scan their tiles in
+//    fp32 and re-score the members they meet on the fly -- never a full
+//    binary64 scan.  Outputs not needed keep their fp32 minimum (dp64 = m32,
+//    bp = -2).
 //
 // The fp32 band: with u = 2^-24, each fp32 candidate value carries a relative
-// error of at most eps_i = max(eps_{i-1}, 20u) + 1.0001u (eps_2 = 1.0001u), so
-// the exact argmin k* satisfies val32(k*) <= m32 (1 + eps_i)/(1 - eps_i).  The
-// 20u budget for one interval cost: compensated sums (~1u), point terms
-// (<= 3.5u for C), correctly rounded reciprocal and products (~3u), and the
-// documented error of __log2f (2^-22 absolute on [0.5,2), 2 ulp elsewhere),
-// amplified at most 2.44x through h(y) = -y log2 y for y <= 1/2; values
-// y > 1/2 are evaluated through 1 - y computed from the complementary mass.
-// The exact stage re-checks |m32 - dp64| <= eps_i dp64 for every output and
-// counts violations.
+// error of at most eps_i = max(eps_{i-1}, 24u) + 1.0001u (eps_2 = 1.0001u), so
+// the exact argmin k* satisfies val32(k*) <= m32 (1 + eps_i)/(1 - eps_i) for
+// ANY fp32 evaluation within that bound (the re-evaluations of stages 2 and 3
+// need not be bit-identical to the wavefront's).  The 24u budget for one
+// interval cost (about 21u used): column anchors within 2u (C: 4.5u) from a
+// double-double corner and compensated scans of non-negative increments,
+// compensated recurrences of non-negative point terms, correctly rounded
+// reciprocal and products, and the documented error of __log2f (2^-22
+// absolute on [0.5,2), 2 ulp elsewhere) amplified at most 2.44x through
+// h(y) = -y log2 y for y <= 1/2; values y > 1/2 are evaluated through 1 - y
+// computed from the complementary mass.  The exact stage re-checks
+// |m32 - dp64| <= eps_i dp64 for every resolved output and counts violations.
 #include <algorithm>
 
 #include "common.cuh"
@@ -98,6 +107,8 @@ struct FastArgs {
     uint64_t *band;        // [G][s+1][ps] tile runs per output
     int32_t *mcnt;         // [G][s+1][ps] band members (-1: runs overflowed)
     int32_t *members;      // [G][s+1][ps][NMEM]
+    uint8_t *need;         // [G][s+1][ps] output resolved exactly
+    float *corner;         // [nJ(nJ-1)/2][8]: state of pair (64K+63, 64J), K < J (N, E, Ec, A, Ac, C, Cc)
     int *done;             // [nsplit][nJ]
     int *ticket;
     int *abort_flag;
@@ -107,6 +118,11 @@ struct FastArgs {
 __device__ __forceinline__ size_t oidx(const FastArgs &a, int g, int i, int64_t j) {
     return ((size_t)g * (size_t)(a.s + 1) + (size_t)i) * (size_t)a.ps + (size_t)j;
 }
+
+// ------------------------------------------------------------ named barriers
+__device__ __forceinline__ void bar_sync(int id, int n) { asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory"); }
+__device__ __forceinline__ void bar_arrive(int id, int n) { asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(n) : "memory"); }
+enum { BAR_FULL = 1, BAR_EMPTY = 3, BAR_CONS = 5, BAR_PROD = 6 };
 
 // ------------------------------------------------------------ fp32 numerics
 
@@ -120,9 +136,18 @@ __device__ __forceinline__ void comp_add(float &x, float &c, float t) {
     c = __fadd_rn(c, e);
 }
 
+// Reciprocal from rcp.approx plus one Newton step: relative error <= u/2 + 2^-46
+// (no slow-path branch, unlike the IEEE-rounded intrinsic).
+__device__ __forceinline__ float rcp_nr(float x) {
+    float r;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+    float e = __fmaf_rn(-x, r, 1.0f);
+    return __fmaf_rn(r, e, r);
+}
+
 // -log2(1 - z) for z in [0, 1/2], from log(1 - z) = -2 atanh(z / (2 - z)).
 __device__ __forceinline__ float neg_log2_1m(float z) {
-    float t = __fdiv_rn(z, __fsub_rn(2.0f, z));  // t in [0, 1/3]
+    float t = __fmul_rn(z, rcp_nr(__fsub_rn(2.0f, z)));  // t in [0, 1/3]
     float t2 = __fmul_rn(t, t);
     // 2 (t + t^3/3 + ... + t^15/15) / ln 2; the next term is below 2^-26 t
     float q = 1.0f / 15.0f;
@@ -136,12 +161,18 @@ __device__ __forceinline__ float neg_log2_1m(float z) {
     return __fmul_rn(__fmul_rn(t, q), 2.8853900817779268f);  // 2 / ln 2
 }
 
-// h(y) = -y log2 y with y = m / d; `comp` = (d - m) / d computed from the
-// complementary mass, used when y > 1/2.
-__device__ __forceinline__ float h32(float y, float comp) {
-    if (!(y > 0.0f)) return 0.0f;
-    if (y <= 0.5f) return fmaxf(__fmul_rn(y, -__log2f(y)), 0.0f);
-    return fmaxf(__fmul_rn(y, neg_log2_1m(fminf(comp, 0.5f))), 0.0f);
+// h(y) = -y log2 y for y in [0, 1/2] (y = 0 gives 0), without branches.
+__device__ __forceinline__ float h32_small(float y) {
+    float r = __fmul_rn(y, -__log2f(fmaxf(y, 1e-37f)));
+    return (y > 0.0f) ? fmaxf(r, 0.0f) : 0.0f;
+}
+// h(y) for y in [0, 1], `comp` = 1 - y computed from the complementary mass;
+// both branches are evaluated and one is selected.
+__device__ __forceinline__ float h32_any(float y, float comp) {
+    float lsm = -__log2f(fmaxf(y, 1e-37f));
+    float lbig = neg_log2_1m(fminf(fmaxf(comp, 0.0f), 0.5f));
+    float r = __fmul_rn(y, (y <= 0.5f) ? lsm : lbig);
+    return (y > 0.0f) ? fmaxf(r, 0.0f) : 0.0f;
 }
 
 // Recurrence state of one column j while k descends: N = sum w, E = sum w (v_j - v_t),
@@ -151,17 +182,19 @@ struct Rec {
 };
 
 // Interval cost of (k, j) from the state: C and Phi = h(U/d) + h(D/d) (Sec. 5).
+// At most one of U, D exceeds d/2 (U + D <= d), so only the larger mass needs
+// the 1 - y form.
 __device__ __forceinline__ void rec_emit(const Rec &r, float vj, float vk, float d_f, float invd, float &Cout,
                                          float &Phi) {
     float Eu = __fadd_rn(r.E, r.Ec), Au = __fadd_rn(r.A, r.Ac);
     Cout = __fadd_rn(fmaxf(__fadd_rn(r.C, r.Cc), 0.0f), 0.0f);  // >= +0 (no -0)
     float L = __fsub_rn(vj, vk);
-    float rL = __frcp_rn(L);
+    float rL = rcp_nr(L);
     float D = __fmul_rn(Eu, rL), U = __fmul_rn(Au, rL);
-    float yU = __fmul_rn(U, invd), yD = __fmul_rn(D, invd);
+    float mbig = fmaxf(U, D), msmall = fminf(U, D);
     float out = __fsub_rn(d_f, r.N);  // mass outside the interval (exact)
-    float cU = __fmul_rn(__fadd_rn(out, D), invd), cD = __fmul_rn(__fadd_rn(out, U), invd);
-    Phi = __fadd_rn(__fadd_rn(h32(yU, cU), h32(yD, cD)), 0.0f);  // >= +0 (no -0)
+    float comp = __fmul_rn(__fadd_rn(out, msmall), invd);
+    Phi = __fadd_rn(__fadd_rn(h32_small(__fmul_rn(msmall, invd)), h32_any(__fmul_rn(mbig, invd), comp)), 0.0f);
 }
 
 // Add point t = k+1 (moving from k+1 to k): vt = v_{k+1}, wt = w_{k+1}, dk = v_{k+1} - v_k.
@@ -195,12 +228,59 @@ __device__ void rec_anchor(const FastArgs &a, int64_t k, int64_t j, Rec &r) {
     split_f(Cd, r.C, r.Cc);
 }
 
-__device__ __forceinline__ Rec rec_empty() { return {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f}; }
+__device__ __forceinline__ size_t corner_idx(int64_t K, int64_t J) { return (size_t)J * (size_t)(J - 1) / 2 + (size_t)K; }
 
-// ------------------------------------------------------------ named barriers
-__device__ __forceinline__ void bar_sync(int id, int n) { asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory"); }
-__device__ __forceinline__ void bar_arrive(int id, int n) { asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(n) : "memory"); }
-enum { BAR_FULL = 1, BAR_EMPTY = 3, BAR_CONS = 5, BAR_PROD = 6 };
+// Corner states (double-double, rounded to fp32 pairs) for every tile below the
+// diagonal: pair (k, j) = (64K + 63, 64J), K < J.
+__global__ void k_corners(FastArgs a) {
+    int64_t n = (int64_t)a.nJ * (a.nJ - 1) / 2;
+    int64_t id = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (; id < n; id += stride) {
+        // invert id = J(J-1)/2 + K
+        int64_t J = (int64_t)((1.0 + sqrt(1.0 + 8.0 * (double)id)) * 0.5);
+        while (J * (J - 1) / 2 > id) J--;
+        while ((J + 1) * J / 2 <= id) J++;
+        int64_t K = id - J * (J - 1) / 2;
+        Rec r;
+        rec_anchor(a, K * BK + BK - 1, J * BJ, r);
+        float *o = a.corner + 8 * (size_t)id;
+        o[0] = r.N; o[1] = r.E; o[2] = r.Ec; o[3] = r.A; o[4] = r.Ac; o[5] = r.C; o[6] = r.Cc; o[7] = 0.f;
+    }
+}
+
+// Compensated (Sum2) exclusive scan over the 64 producer threads of (x, c) pairs.
+__device__ __forceinline__ void pair_add(float &x, float &c, float y, float yc) {
+    float s = __fadd_rn(x, y);
+    float bb = __fsub_rn(s, x);
+    float e = __fadd_rn(__fsub_rn(x, __fsub_rn(s, bb)), __fsub_rn(y, bb));
+    x = s;
+    c = __fadd_rn(__fadd_rn(c, yc), e);
+}
+
+__device__ void scan64_excl(float v, float &x_out, float &c_out, float (*wsum)[2]) {
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;  // producer threads 0..63
+    float x = v, c = 0.f;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        float y = __shfl_up_sync(0xffffffffu, x, o), yc = __shfl_up_sync(0xffffffffu, c, o);
+        if (lane >= o) pair_add(x, c, y, yc);
+    }
+    if (lane == 31) { wsum[wid][0] = x; wsum[wid][1] = c; }
+    bar_sync(BAR_PROD, NPROD);
+    if (wid == 1) pair_add(x, c, wsum[0][0], wsum[0][1]);
+    // exclusive: shift by one
+    float xe = __shfl_up_sync(0xffffffffu, x, 1), ce = __shfl_up_sync(0xffffffffu, c, 1);
+    if (lane == 0) {
+        if (wid == 0) { xe = 0.f; ce = 0.f; }
+        else { xe = wsum[0][0]; ce = wsum[0][1]; }
+    }
+    x_out = xe;
+    c_out = ce;
+    bar_sync(BAR_PROD, NPROD);
+}
+
+__device__ __forceinline__ Rec rec_empty() { return {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f}; }
 
 __device__ __forceinline__ int ld_acquire(const int *p) {
     int v;
@@ -241,8 +321,10 @@ struct __align__(16) Smem {
     float C[2][BJ][PSTR];
     float Phi[2][BJ][PSTR];
     float diag[2][kMaxG][BJ];             // dp32 of the previous / current layer inside the column
+    float dmin[kMaxG][BJ];                // diagonal-block minimum of the current layer
     float kv[BK], kw[BK], kd[BK];         // v_k (k0..k0+63), w_{k+1}, v_{k+1} - v_k
     TileMeta meta[2];
+    float wsum[2][2];                     // producer scan: per-warp totals
     int ticket;
     int pad[3];
     // followed by dp32 slices [2][Gc * (s-2)][BK] (dynamic)
@@ -327,6 +409,32 @@ __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
                     asm volatile("cp.async.commit_group;" ::: "memory");
                 }
                 bar_sync(BAR_PROD, NPROD);
+                // anchors of the 64 columns at k = 64K + 63: the corner state of (K, J) advanced
+                // along j with compensated exclusive scans of non-negative increments
+                Rec anchor_r = rec_empty();
+                if (!diag) {
+                    const float *cp = a.corner + 8 * corner_idx(K, J);
+                    float vk = S.kv[BK - 1];
+                    int64_t jt = j0 + jl;  // increment of column jl: moving j from jt to jt + 1
+                    bool okc = jt + 1 < a.p;
+                    float wn = okc ? a.wf[jt + 1] : 0.f;
+                    float vn = okc ? a.v[jt + 1] : 0.f;
+                    float dj = okc ? __fsub_rn(vn, a.v[jt]) : 0.f;
+                    float nx, nc, ax, ac, ex, ec, cx, cc;
+                    scan64_excl(wn, nx, nc, S.wsum);                               // N (exact)
+                    scan64_excl(okc ? __fmul_rn(wn, __fsub_rn(vn, vk)) : 0.f, ax, ac, S.wsum);  // A
+                    float Nj = __fadd_rn(cp[0], __fadd_rn(nx, nc));
+                    float Aj = __fadd_rn(__fadd_rn(cp[3], ax), __fadd_rn(cp[4], ac));
+                    scan64_excl(__fmul_rn(dj, Nj), ex, ec, S.wsum);              // E
+                    scan64_excl(__fmul_rn(dj, Aj), cx, cc, S.wsum);              // C
+                    anchor_r.N = Nj;
+                    anchor_r.E = cp[1]; anchor_r.Ec = cp[2];
+                    pair_add(anchor_r.E, anchor_r.Ec, ex, ec);
+                    anchor_r.A = cp[3]; anchor_r.Ac = cp[4];
+                    pair_add(anchor_r.A, anchor_r.Ac, ax, ac);
+                    anchor_r.C = cp[5]; anchor_r.Cc = cp[6];
+                    pair_add(anchor_r.C, anchor_r.Cc, cx, cc);
+                }
                 // interval costs of column j for k in the tile (descending k)
                 float (*Cr)[PSTR] = S.C[b];
                 float (*Pr)[PSTR] = S.Phi[b];
@@ -346,13 +454,13 @@ __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
                             Cr[jl][kl] = c; Pr[jl][kl] = ph;
                         }
                     } else {
-                        rec_anchor(a, k0 + BK - 1, j, r);
-                        float c, ph;
-                        rec_emit(r, vj, S.kv[BK - 1], d_f, a.invd, c, ph);
-                        Cr[jl][BK - 1] = c; Pr[jl][BK - 1] = ph;
-                        for (int kl = BK - 2; kl >= 0; kl--) {
-                            rec_step(r, vj, S.kv[kl + 1], S.kw[kl], S.kd[kl]);
-                            rec_emit(r, vj, S.kv[kl], d_f, a.invd, c, ph);
+                        r = anchor_r;
+                        Rec nxt = r;
+                        for (int kl = BK - 1; kl >= 0; kl--) {
+                            Rec cur = nxt;
+                            if (kl > 0) rec_step(nxt, vj, S.kv[kl], S.kw[kl - 1], S.kd[kl - 1]);  // state of k - 1
+                            float c, ph;
+                            rec_emit(cur, vj, S.kv[kl], d_f, a.invd, c, ph);
                             Cr[jl][kl] = c; Pr[jl][kl] = ph;
                         }
                     }
@@ -408,6 +516,9 @@ __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
             if (own) {
                 const float *dpb = sDP + (size_t)b * rowsDP * BK + (size_t)gl * L * BK;
                 float2 lam2 = make_float2(lam, lam);
+                int rowl[LPT];
+#pragma unroll
+                for (int l = 0; l < LPT; l++) rowl[l] = min(lg * LPT + l, L - 1);
 #pragma unroll 1
                 for (int kk = 0; kk < BK; kk += 4) {
                     float2 W[JPT][2];
@@ -420,35 +531,36 @@ __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
                     }
 #pragma unroll
                     for (int l = 0; l < LPT; l++) {
-                        int li = lg * LPT + l;  // layer i = 3 + li uses dp row 2 + li
-                        if (li < L) {
-                            float4 d4 = *reinterpret_cast<const float4 *>(dpb + (size_t)li * BK + kk);
-                            float2 da = make_float2(d4.x, d4.y), db = make_float2(d4.z, d4.w);
+                        // layer i = 3 + li uses dp row 2 + li; rows past the last layer are
+                        // clamped (their results are never used)
+                        const float4 d4 = *reinterpret_cast<const float4 *>(dpb + (size_t)rowl[l] * BK + kk);
+                        float2 da = make_float2(d4.x, d4.y), db = make_float2(d4.z, d4.w);
 #pragma unroll
-                            for (int q = 0; q < JPT; q++) {
-                                float2 t0 = add2(da, W[q][0]);
-                                float2 t1 = add2(db, W[q][1]);
-                                int c = min(min(cm[l][q], __float_as_int(t0.x)), __float_as_int(t0.y));
-                                cm[l][q] = min(min(c, __float_as_int(t1.x)), __float_as_int(t1.y));
-                            }
+                        for (int q = 0; q < JPT; q++) {
+                            float2 t0 = add2(da, W[q][0]);
+                            float2 t1 = add2(db, W[q][1]);
+                            int c = min(min(cm[l][q], __float_as_int(t0.x)), __float_as_int(t0.y));
+                            cm[l][q] = min(min(c, __float_as_int(t1.x)), __float_as_int(t1.y));
                         }
                     }
                 }
-                // band bookkeeping for this tile
+                // band bookkeeping for this tile (branch-free)
 #pragma unroll
                 for (int l = 0; l < LPT; l++) {
-                    int li = lg * LPT + l;
-                    if (li < L) {
-                        float tau = a.prm->tau[3 + li];
+                    const int li = lg * LPT + l;
+                    const float tau = a.prm->tau[3 + min(li, L - 1)];
+                    const bool lok = li < L;
 #pragma unroll
-                        for (int q = 0; q < JPT; q++) {
-                            float c = __int_as_float(cm[l][q]), bb = best[l][q];
-                            if (c < CUDART_INF_F) {
-                                float T = __fmul_rn(bb, tau);
-                                if (c < __fsub_rn(bb, T)) { word[l][q] = band_reset((uint32_t)m.K); best[l][q] = c; }
-                                else if (c <= __fadd_rn(bb, T)) { word[l][q] = band_append(word[l][q], (uint32_t)m.K); best[l][q] = fminf(bb, c); }
-                            }
-                        }
+                    for (int q = 0; q < JPT; q++) {
+                        float c = __int_as_float(cm[l][q]), bb = best[l][q];
+                        float T = __fmul_rn(bb, tau);
+                        bool fin = lok && (c < CUDART_INF_F);
+                        bool rst = fin && (c < __fsub_rn(bb, T));
+                        bool app = fin && !rst && (c <= __fadd_rn(bb, T));
+                        uint64_t wv = word[l][q];
+                        uint64_t wa = band_append(wv, (uint32_t)m.K);
+                        word[l][q] = rst ? band_reset((uint32_t)m.K) : (app ? wa : wv);
+                        best[l][q] = fin ? fminf(bb, c) : bb;
                     }
                 }
             }
@@ -466,6 +578,31 @@ __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
             int cur = 0;
             for (int li = 0; li < L; li++) {
                 const int i = 3 + li;
+                // (a) every consumer thread: minima over the diagonal block for items (g, column),
+                //     4-wide loads over k with independent partial minima
+                for (int item = ct; item < a.Gc * BJ; item += a.ncons) {
+                    int gg = item / BJ, jl = item % BJ;
+                    int g2 = m.split * a.Gc + gg;
+                    float lm = g2 < a.G ? a.prm->lam32[g2] : 0.f;
+                    float2 lm2 = make_float2(lm, lm);
+                    int c0 = 0x7f800000, c1 = 0x7f800000, c2 = 0x7f800000, c3 = 0x7f800000;
+                    const float *prow = &S.diag[cur][gg][0];
+#pragma unroll 4
+                    for (int kk = 0; kk < BJ; kk += 4) {
+                        float4 c4 = *reinterpret_cast<const float4 *>(&S.C[b][jl][kk]);
+                        float4 f4 = *reinterpret_cast<const float4 *>(&S.Phi[b][jl][kk]);
+                        float4 d4 = *reinterpret_cast<const float4 *>(prow + kk);
+                        float2 w0 = fma2(lm2, make_float2(f4.x, f4.y), make_float2(c4.x, c4.y));
+                        float2 w1 = fma2(lm2, make_float2(f4.z, f4.w), make_float2(c4.z, c4.w));
+                        float2 t0 = add2(make_float2(d4.x, d4.y), w0);
+                        float2 t1 = add2(make_float2(d4.z, d4.w), w1);
+                        c0 = min(c0, __float_as_int(t0.x)); c1 = min(c1, __float_as_int(t0.y));
+                        c2 = min(c2, __float_as_int(t1.x)); c3 = min(c3, __float_as_int(t1.y));
+                    }
+                    S.dmin[gg][jl] = __int_as_float(min(min(c0, c1), min(c2, c3)));
+                }
+                bar_sync(BAR_CONS, a.ncons);
+                // (b) the owners of layer i fold the diagonal block into their band state
                 const int l = li - lg * LPT;
                 if (own && l >= 0 && l < LPT) {
 #pragma unroll
@@ -475,11 +612,7 @@ __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
                         for (int q = 0; q < JPT; q++) {
                             int jl = jq + NJQ * q;
                             int64_t j = j0 + jl;
-                            float c = CUDART_INF_F;
-                            for (int kl = 0; kl < jl; kl++) {
-                                float W = __fmaf_rn(lam, S.Phi[b][jl][kl], S.C[b][jl][kl]);
-                                c = fminf(c, __fadd_rn(S.diag[cur][gl][kl], W));
-                            }
+                            float c = S.dmin[gl][jl];
                             float bb = best[lx][q];
                             if (c < CUDART_INF_F) {
                                 float T = __fmul_rn(bb, a.prm->tau[i]);
@@ -555,7 +688,7 @@ __device__ void visit_tile(const FastArgs &a, int g, int i, int64_t j, int64_t K
         khi = j;  // state of the empty interval (j, j]
     } else {
         khi = k0 + BK - 1;
-        rec_anchor(a, khi, j, r);
+        rec_anchor(a, khi, j, r);  // any evaluation within the certified bound will do
         rec_emit(r, vj, a.v[khi], d_f, a.invd, c, ph);
         if (cand32(prev[khi], lam, c, ph) <= thr) f(khi);
     }
@@ -586,31 +719,48 @@ __device__ __forceinline__ float band_threshold(const FastArgs &a, int i, float 
     return __fadd_rn(m32, __fmul_rn(m32, a.prm->tau[i]));
 }
 
-__global__ void k_extract(FastArgs a) {
-    int64_t tot = (int64_t)a.G * (a.s - 2) * a.p;
+// Outputs eq. apx_final reads: dp(i, p-1) for i in [ilo, s] (or every output).
+__global__ void k_need_init(FastArgs a, int ilo, int all) {
+    int64_t tot = (int64_t)a.G * (a.s + 1) * a.ps;
+    int64_t id = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (; id < tot; id += stride) {
+        int64_t j = id % a.ps;
+        int i = (int)((id / a.ps) % (a.s + 1));
+        uint8_t v = 0;
+        if (i >= 3 && j < a.p && j >= i - 1) v = all ? 1 : (j == a.p - 1 && i >= ilo);
+        a.need[id] = v;
+    }
+}
+
+// Backward closure, layer i: members of every needed output; mark (i-1, k) needed.
+__global__ void k_need_layer(FastArgs a, int i) {
+    int64_t tot = (int64_t)a.G * a.p;
     int64_t id = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     int64_t stride = (int64_t)gridDim.x * blockDim.x;
     unsigned long long nmem = 0, nbig = 0, nover = 0;
     for (; id < tot; id += stride) {
         int64_t j = id % a.p;
-        int64_t r = id / a.p;
-        int i = 3 + (int)(r % (a.s - 2));
-        int g = (int)(r / (a.s - 2));
+        int g = (int)(id / a.p);
         if (j < i - 1) continue;
         size_t o = oidx(a, g, i, j);
+        if (!a.need[o]) continue;
         float m32 = a.dp32[o];
         if (!(m32 < CUDART_INF_F)) { a.mcnt[o] = 0; continue; }
         uint64_t w = a.band[o];
-        if (w & 4u) { a.mcnt[o] = -1; nover++; continue; }
         int32_t *mem = a.members + o * NMEM;
+        uint8_t *below = a.need + oidx(a, g, i - 1, 0);
+        const bool mark = i - 1 >= 3;
         int cnt = 0;
         visit_band(a, g, i, j, w, band_threshold(a, i, m32), [&](int64_t k) {
             if (cnt < NMEM) mem[cnt] = (int32_t)k;
             cnt++;
+            if (mark) below[k] = 1;
         });
-        a.mcnt[o] = cnt;
+        a.mcnt[o] = (w & 4u) ? -1 : cnt;
         nmem += cnt;
         nbig += cnt > NMEM;
+        nover += (w & 4u) ? 1 : 0;
     }
     if (nmem) atomicAdd((unsigned long long *)&a.st->members, nmem);
     if (nbig) atomicAdd((unsigned long long *)&a.st->big_bands, nbig);
@@ -636,6 +786,7 @@ __global__ void k_exact_layer(Prefix P, FastArgs a, int i, double *dp64, int32_t
     size_t o = oidx(a, g, i, j);
     float m32 = a.dp32[o];
     if (!(m32 < CUDART_INF_F)) return;
+    if (!a.need[o]) { dp64[o] = (double)m32; bp[o] = -2; return; }
     int cnt = a.mcnt[o];
     double lam = a.prm->lam64[g];
     const double *prev = dp64 + oidx(a, g, i - 1, 0);
@@ -675,8 +826,8 @@ __global__ void k_store_params(FastParams prm, FastParams *dst) {
 size_t fast_dp_band_bytes(int64_t d, int32_t s) {
     size_t rows = (size_t)kMaxG * (size_t)(s + 1) * (size_t)table_stride(d);
     size_t nJ = (size_t)cdiv(d, BJ);
-    return align256(8 * rows) + align256(4 * rows) + align256(4 * NMEM * rows) +
-           align256(4 * (size_t)kMaxG * nJ + 64) + align256(sizeof(FastParams));
+    return align256(8 * rows) + align256(4 * rows) + align256(4 * NMEM * rows) + align256(rows) +
+           align256(4 * (size_t)kMaxG * nJ + 64) + align256(sizeof(FastParams)) + align256(32 * nJ * (nJ + 1) / 2);
 }
 
 static size_t smem_bytes(int Gc, int s) { return sizeof(Smem) + (size_t)2 * Gc * (s - 2) * BK * sizeof(float); }
@@ -688,13 +839,14 @@ static void band_factors(int s, FastParams &fp) {
     double eps = 1.0001 * u;
     fp.eps[2] = (float)eps;
     for (int i = 3; i <= s; i++) {
-        eps = std::max(eps, 20.0 * u) + 1.0001 * u;
+        eps = std::max(eps, 24.0 * u) + 1.0001 * u;
         fp.eps[i] = (float)eps;
         fp.tau[i] = (float)(2.0 * eps / (1.0 - eps) * 1.001 + 2.0 * u);
     }
 }
 
-int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, const Layout &Lw, cudaStream_t st) {
+int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, const Layout &Lw, cudaStream_t st,
+                   bool exact_s, bool exact_tables) {
     double *dp64 = wsp<double>(ws, Lw.dp64);
     int32_t *bp = wsp<int32_t>(ws, Lw.bp);
     // small inputs, very large ones and huge counts take the reference kernel
@@ -731,9 +883,13 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     base += align256(4 * rows);
     a.members = reinterpret_cast<int32_t *>(base);
     base += align256(4 * NMEM * rows);
+    a.need = reinterpret_cast<uint8_t *>(base);
+    base += align256(rows);
     int *flags = reinterpret_cast<int *>(base);
     base += align256(4 * (size_t)kMaxG * (size_t)cdiv(Lw.d, BJ) + 64);
     FastParams *dprm = reinterpret_cast<FastParams *>(base);
+    base += align256(sizeof(FastParams));
+    a.corner = reinterpret_cast<float *>(base);
     a.prm = dprm;
     a.done = flags;
     a.ticket = flags + (size_t)kMaxG * a.nJ;
@@ -753,6 +909,11 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     note_launch();
     k_fast_base<<<(unsigned)cdiv(P.p - 1, 128), 128, 0, st>>>(P, a, dp64, bp);
     ECASQ_LAUNCH_CHECK();
+    if (a.nJ > 1) {
+        note_launch();
+        k_corners<<<(unsigned)std::min<int64_t>(cdiv((int64_t)a.nJ * (a.nJ - 1) / 2, 128), 152 * 64), 128, 0, st>>>(a);
+        ECASQ_LAUNCH_CHECK();
+    }
     size_t smem = smem_bytes(a.Gc, s);
     ECASQ_CUDA_TRY(cudaFuncSetAttribute(k_wavefront, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     int dev = 0, nsm = 0;
@@ -764,10 +925,17 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     k_wavefront<<<grid, NPROD + a.ncons, smem, st>>>(a);
     timer_end(st);
     ECASQ_LAUNCH_CHECK();
-    int64_t tot = (int64_t)G * (s - 2) * P.p;
+    const int ilo = exact_s ? s : 2;
     note_launch();
-    k_extract<<<(unsigned)std::min<int64_t>(cdiv(tot, 128), (int64_t)nsm * 64), 128, 0, st>>>(a);
+    k_need_init<<<(unsigned)std::min<int64_t>(cdiv((int64_t)G * (s + 1) * P.ps, 256), (int64_t)nsm * 32), 256, 0, st>>>(
+        a, ilo, exact_tables ? 1 : 0);
     ECASQ_LAUNCH_CHECK();
+    const unsigned gl = (unsigned)std::min<int64_t>(cdiv((int64_t)G * P.p, 128), (int64_t)nsm * 64);
+    for (int i = s; i >= 3; i--) {
+        note_launch();
+        k_need_layer<<<gl, 128, 0, st>>>(a, i);
+        ECASQ_LAUNCH_CHECK();
+    }
     for (int i = 3; i <= s; i++) {
         note_launch();
         k_exact_layer<<<(unsigned)cdiv((int64_t)G * P.p, 128), 128, 0, st>>>(P, a, i, dp64, bp);

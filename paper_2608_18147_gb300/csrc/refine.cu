@@ -31,32 +31,43 @@ __device__ __forceinline__ double local_obj(const Prefix &P, const Nbr &n, int64
     return __dadd_rn(__dadd_rn(C1, C2), __dmul_rn(lamp, ent));
 }
 
-__global__ void __launch_bounds__(256) k_refine_colour(Prefix P, const int32_t *a, int m, int colour, double lamp,
-                                                       int32_t *a_new, int32_t *moved) {
+constexpr int kRefineChunk = 2048;  // candidates per block
+
+__device__ __forceinline__ Nbr make_nbr(const Prefix &P, const int32_t *a, int m, int l) {
+    Nbr n;
+    n.L = a[l - 1]; n.R = a[l + 1]; n.cur = a[l];
+    n.firstL = (l - 1 == 0); n.lastR = (l + 1 == m - 1);
+    double C, U, D;
+    n.Ux = 0.0; n.Dx = 0.0;
+    if (!n.firstL) { pair_exact(P, a[l - 2], n.L, C, U, D); n.Ux = U; }
+    if (!n.lastR) { pair_exact(P, n.R, a[l + 2], C, U, D); n.Dx = D; }
+    return n;
+}
+
+// Block (chunk, b): the b-th value of the colour class, candidates
+// L+1+chunk*kRefineChunk .. (excluding the current position); the best
+// (value, lowest index) of the chunk goes to part[b * nchunk + chunk].
+struct RefPart { double v; int64_t i; };
+
+__global__ void __launch_bounds__(256) k_refine_chunks(Prefix P, const int32_t *a, int m, int colour, double lamp,
+                                                       RefPart *part, int nchunk) {
     __shared__ Nbr nb;
     __shared__ double rv[256];
     __shared__ int64_t ri[256];
     int l0 = colour == 0 ? 3 : colour;
-    int l = l0 + 3 * blockIdx.x;
+    int l = l0 + 3 * blockIdx.y;
     if (l > m - 2) return;
-    if (threadIdx.x == 0) {
-        Nbr n;
-        n.L = a[l - 1]; n.R = a[l + 1]; n.cur = a[l];
-        n.firstL = (l - 1 == 0); n.lastR = (l + 1 == m - 1);
-        double C, U, D;
-        n.Ux = 0.0; n.Dx = 0.0;
-        if (!n.firstL) { pair_exact(P, a[l - 2], n.L, C, U, D); n.Ux = U; }
-        if (!n.lastR) { pair_exact(P, n.R, a[l + 2], C, U, D); n.Dx = D; }
-        nb = n;
-    }
+    int64_t lo = (int64_t)a[l - 1] + 1 + (int64_t)blockIdx.x * kRefineChunk;
+    int64_t hi = min((int64_t)a[l + 1], lo + kRefineChunk);
+    if (threadIdx.x == 0) nb = make_nbr(P, a, m, l);
     __syncthreads();
     Nbr n = nb;
     double bv = CUDART_INF;
     int64_t bi = -1;
-    for (int64_t c = n.L + 1 + threadIdx.x; c < n.R; c += blockDim.x) {
+    for (int64_t c = lo + threadIdx.x; c < hi; c += blockDim.x) {
         if (c == n.cur) continue;
         double v = local_obj(P, n, c, lamp);
-        if (v < bv) { bv = v; bi = c; }   // c ascends per thread: keeps the lowest
+        if (v < bv) { bv = v; bi = c; }  // c ascends per thread: keeps the lowest
     }
     rv[threadIdx.x] = bv; ri[threadIdx.x] = bi;
     __syncthreads();
@@ -70,22 +81,55 @@ __global__ void __launch_bounds__(256) k_refine_colour(Prefix P, const int32_t *
         }
         __syncthreads();
     }
+    if (threadIdx.x == 0) part[(size_t)blockIdx.y * nchunk + blockIdx.x] = {rv[0], ri[0]};
+}
+
+// One warp per moved value: best over the chunks (lowest index among equal
+// values), then keep the current position unless the best is strictly lower.
+__global__ void k_refine_pick(Prefix P, const int32_t *a, int m, int colour, double lamp, const RefPart *part,
+                              int nchunk, int32_t *a_new, int32_t *moved) {
+    int l0 = colour == 0 ? 3 : colour;
+    int l = l0 + 3 * blockIdx.x;
+    if (l > m - 2) return;
+    int64_t range = (int64_t)a[l + 1] - (int64_t)a[l - 1] - 1;
+    int nc = (int)cdiv(range, kRefineChunk);
+    double bv = CUDART_INF;
+    int64_t bi = -1;
+    for (int c = threadIdx.x; c < nc; c += 32) {
+        RefPart q = part[(size_t)blockIdx.x * nchunk + c];
+        if (q.i >= 0 && (q.v < bv || (q.v == bv && q.i < bi))) { bv = q.v; bi = q.i; }
+    }
+    for (int o = 16; o > 0; o >>= 1) {
+        double v2 = __shfl_down_sync(0xffffffffu, bv, o);
+        int64_t i2 = __shfl_down_sync(0xffffffffu, bi, o);
+        if (i2 >= 0 && (bi < 0 || v2 < bv || (v2 == bv && i2 < bi))) { bv = v2; bi = i2; }
+    }
     if (threadIdx.x == 0) {
+        Nbr n = make_nbr(P, a, m, l);
         double vc = local_obj(P, n, n.cur, lamp);
-        int64_t nw = (ri[0] >= 0 && rv[0] < vc) ? ri[0] : n.cur;
+        int64_t nw = (bi >= 0 && bv < vc) ? bi : n.cur;
         a_new[l] = (int32_t)nw;
         if (nw != n.cur) atomicExch(moved, 1);
     }
 }
 
+size_t refine_scratch_bytes(int64_t d) {
+    return sizeof(RefPart) * (size_t)(kMaxS / 3 + 1) * (size_t)cdiv(d, kRefineChunk);
+}
+
 int launch_refine_colour(const Prefix &P, const int32_t *a, int m, int colour, double lamp, int32_t *a_new,
-                         int32_t *moved, cudaStream_t st, int *nblocks_out) {
+                         int32_t *moved, void *part_buf, cudaStream_t st, int *nblocks_out) {
     int l0 = colour == 0 ? 3 : colour;
     int nblk = (m - 2 >= l0) ? (m - 2 - l0) / 3 + 1 : 0;
     *nblocks_out = nblk;
     if (nblk == 0) return ECASQ_OK;
+    int nchunk = (int)cdiv(P.p, kRefineChunk);
+    RefPart *part = reinterpret_cast<RefPart *>(part_buf);
     note_launch();
-    k_refine_colour<<<nblk, 256, 0, st>>>(P, a, m, colour, lamp, a_new, moved);
+    k_refine_chunks<<<dim3(nchunk, nblk), 256, 0, st>>>(P, a, m, colour, lamp, part, nchunk);
+    ECASQ_LAUNCH_CHECK();
+    note_launch();
+    k_refine_pick<<<nblk, 32, 0, st>>>(P, a, m, colour, lamp, part, nchunk, a_new, moved);
     ECASQ_LAUNCH_CHECK();
     return ECASQ_OK;
 }

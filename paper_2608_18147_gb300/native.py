@@ -17,7 +17,7 @@ import numpy as np
 from . import build as _build
 
 OK, EINVAL, ENONFINITE, EINFEASIBLE, EWORKSPACE, ECUDA, ETIMEOUT, ERANGE = 0, -1, -2, -3, -4, -5, -6, -7
-EXACT_S, NO_REFINE_GUARD, DP_REFERENCE, TIME_KERNELS = 1, 2, 4, 8
+EXACT_S, NO_REFINE_GUARD, DP_REFERENCE, TIME_KERNELS, EXACT_TABLES = 1, 2, 4, 8, 16
 
 _lock = threading.Lock()
 _lib = None

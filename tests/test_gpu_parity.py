@@ -96,10 +96,10 @@ def _dp_parity(E, oracle_mod, x, s, lams, flags, exact_s=False):
 
 
 @pytest.mark.parametrize("lams", [[0.0], [0.0, 1e-4, 0.01, 0.05, 0.2, 0.6, 2.0, 40.0]])
-@pytest.mark.parametrize("flags_name", ["DP_REFERENCE", "FAST"])
+@pytest.mark.parametrize("flags_name", ["DP_REFERENCE", "EXACT_TABLES"])
 def test_dp_parity_normal1024(E, oracle_mod, lams, flags_name):
     x = workloads.normal(1024, 0)
-    _dp_parity(E, oracle_mod, x, 8, lams, getattr(E, flags_name, 0))
+    _dp_parity(E, oracle_mod, x, 8, lams, getattr(E, flags_name))
 
 
 @pytest.mark.parametrize("name,s,lams", [
@@ -113,7 +113,53 @@ def test_dp_parity_normal1024(E, oracle_mod, lams, flags_name):
 def test_dp_fast_parity(E, oracle_mod, name, s, lams):
     """The fast kernel (fp32 filter + certified band + exact re-scoring) against the oracle."""
     x = inputs_small()[name]
-    _dp_parity(E, oracle_mod, x, s, lams, 0)
+    _dp_parity(E, oracle_mod, x, s, lams, E.EXACT_TABLES)
+
+
+def _eps_layer(i):
+    """Certified relative error of the fast kernel's fp32 minima at layer i."""
+    u = 2.0 ** -24
+    eps = 1.0001 * u
+    for _ in range(3, i + 1):
+        eps = max(eps, 24 * u) + 1.0001 * u
+    return eps
+
+
+@pytest.mark.parametrize("name,s,lams", [
+    ("normal1024", 8, [0.0, 1e-4, 0.01, 0.2, 2.0]),
+    ("ragged2049", 16, [0.0, 1e-3, 0.05, 0.4]),
+])
+def test_dp_fast_closure_mode(E, oracle_mod, name, s, lams):
+    """Default fast mode: only the outputs eq. apx_final and the traceback read are
+    resolved exactly; the codebooks and metrics equal the oracle's, resolved entries
+    match exactly and the rest lie within their certified fp32 bound."""
+    x = inputs_small()[name]
+    ws = E.workspace(x.size, s)
+    Qg, mg, met = E.ecasq_dp_pass(x, s, lams, ws=ws)
+    st = E.native.ws_status(ws)
+    assert st["bound_viol"] == 0 and st["timeout"] == 0
+    H = oracle_mod.Hist(x)
+    H.cache()
+    v = H.arrays()["v"]
+    for g, lam in enumerate(lams):
+        r = H.apx_dp(s, lam * H.norm2)
+        dp, bp = [t.cpu().numpy() for t in E.ecasq_dp_tables(ws, g, s, x.size)]
+        res = bp >= -1
+        assert res[:, -1][2:].all()  # every dp(i, p-1) is resolved
+        fin = np.isfinite(r["dp"]) & res
+        np.testing.assert_allclose(dp[fin], r["dp"][fin], rtol=DP_RTOL)
+        mism = (bp != r["bp"]) & res & (r["bp"] >= 0)
+        assert np.all(r["margin"][mism] < TIE)
+        unres = (bp == -2)
+        for i in range(3, s + 1):
+            row = unres[i] & np.isfinite(r["dp"][i])
+            if row.any():
+                err = np.abs(dp[i][row] - r["dp"][i][row])
+                assert np.all(err <= _eps_layer(i) * 1.001 * r["dp"][i][row])
+        assert mg[g] == r["m"]
+        np.testing.assert_array_equal(Qg[g, :mg[g]].cpu().numpy(), v[r["Q_idx"]])
+        mse, hs, hx = H.eval_idx(r["Q_idx"])
+        np.testing.assert_allclose(met[g], [r["best"], mse, hs, hx], rtol=MET_RTOL)
 
 
 def test_dp_fast_matches_reference_16k(E, oracle_mod):
@@ -123,7 +169,9 @@ def test_dp_fast_matches_reference_16k(E, oracle_mod):
     s = 16
     lams = [0.0, 1e-5, 1e-3, 0.01, 0.05, 0.2, 1.0, 10.0]
     wsf, wsr = E.workspace(x.size, s), E.workspace(x.size, s)
-    Qf, mf, metf = E.ecasq_dp_pass(x, s, lams, flags=0, ws=wsf)
+    Ql, ml, metl = E.ecasq_dp_pass(x, s, lams, flags=0, ws=wsf)  # default closure mode
+    stl = E.native.ws_status(wsf)
+    Qf, mf, metf = E.ecasq_dp_pass(x, s, lams, flags=E.EXACT_TABLES, ws=wsf)
     stf = E.native.ws_status(wsf)
     Qr, mr, metr = E.ecasq_dp_pass(x, s, lams, flags=E.DP_REFERENCE, ws=wsr)
     assert stf["bound_viol"] == 0 and stf["timeout"] == 0
@@ -149,8 +197,11 @@ def test_dp_fast_matches_reference_16k(E, oracle_mod):
             assert dpf[i, j] == pytest.approx(best, rel=DP_RTOL)
             if second > best * (1 + TIE):
                 assert bpf[i, j] == arg
-        assert mf[g] == mr[g]
+        assert mf[g] == mr[g] == ml[g]
         np.testing.assert_array_equal(Qf[g].cpu().numpy(), Qr[g].cpu().numpy())
+        np.testing.assert_array_equal(Ql[g].cpu().numpy(), Qr[g].cpu().numpy())
+    np.testing.assert_allclose(metl, metr, rtol=MET_RTOL)
+    assert stl["bound_viol"] == 0 and stl["members"] < stf["members"]
 
 
 @pytest.mark.parametrize("name", ["dups", "ragged2049", "tiny_offset", "two_values"])
