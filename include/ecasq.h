@@ -164,6 +164,37 @@ int ecasq_evaluate(const float *x, int64_t d, const float *Q, int32_t m, void *w
 int ecasq_quantize(const float *x, int64_t d, const float *Q, int32_t m, uint64_t seed, uint8_t *idx,
                    uint32_t *counts, void *ws, size_t ws_bytes, double *h_emp, ecasq_stream_t stream);
 
+/* ecasq_quantize without a workspace: same arguments minus (ws, ws_bytes),
+ * same kernel, same results (idx, counts and h_emp equal to ecasq_quantize's
+ * for the same inputs and seed).  The paper has no counterpart: this is an
+ * interface convenience around the quantizer of Sec. 2.
+ *
+ * Who needs it: callers that cannot hand the library device memory at the
+ * point where they quantize -- a hook inside a training or serving framework
+ * that runs where the framework forbids allocation (its caching allocator
+ * may not be re-entered there), a latency-critical path that cannot afford an
+ * allocation's synchronisation, or a process already at its memory limit.
+ * The function itself calls no device allocator (no cudaMalloc/cudaFree, no
+ * allocating library routine); idx and counts are the caller's buffers.
+ *
+ * Scratch: a fixed 256-byte block of device memory inside this library, one
+ * per device, holding one status record.  Its range-error flag must be zero
+ * when the kernel starts; every call zeroes it on `stream` before its launch.
+ * Limits: m <= 256 (the codebook cap) and d < 2^31, as for ecasq_quantize;
+ * larger sizes return ECASQ_EINVAL.  The scratch does not grow with d.
+ *
+ * Set-up: the first call on each device looks up the scratch's device address
+ * (cudaGetSymbolAddress, which may load this library's device code) and keeps
+ * it; an error there returns ECASQ_ECUDA.  Make that first call on each device
+ * before any stream capture begins.
+ *
+ * Concurrency: all calls on one device share the one scratch block.  Calls
+ * that overlap in time on the same device -- from several host threads, or on
+ * streams not ordered with each other -- race on it (one call's reset can
+ * erase another's error flag); serialise them.  Synchronises `stream`. */
+int ecasq_quantize_noalloc(const float *x, int64_t d, const float *Q, int32_t m, uint64_t seed, uint8_t *idx,
+                           uint32_t *counts, double *h_emp, ecasq_stream_t stream);
+
 /* Budgeted solves of `rows` independent rows of length d (row-major X),
  * each exactly as ecasq_solve would do it on that row alone (same schedule,
  * same results).  Q [rows * s] device, m_out [rows] device, res host [rows]

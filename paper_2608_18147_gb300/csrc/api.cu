@@ -5,6 +5,7 @@
 
 #include <algorithm>
 #include <atomic>
+#include <mutex>
 #include <vector>
 
 #include "common.cuh"
@@ -101,6 +102,31 @@ static int num_sms() {
             g_num_sms = 152;
     }
     return g_num_sms;
+}
+
+// Scratch of ecasq_quantize_noalloc: one status record in a fixed block of
+// this library's device memory (no allocation at call time).  The record's
+// range-error flag must read zero when the kernel starts.
+constexpr size_t kNoAllocScratchBytes = 256;
+static_assert(sizeof(DevStatus) <= kNoAllocScratchBytes, "status record larger than the fixed scratch block");
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+constexpr int kNoAllocMaxDevices = 64;
+static std::mutex g_noalloc_mu;
+static void *g_noalloc_addr[kNoAllocMaxDevices];
+
+// Device address of the scratch block on the current device, looked up once
+// per device (cudaGetSymbolAddress) and kept.
+static int noalloc_scratch(void **out) {
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kNoAllocMaxDevices) return ECASQ_ECUDA;
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!g_noalloc_addr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return ECASQ_ECUDA;
+        g_noalloc_addr[dev] = p;
+    }
+    *out = g_noalloc_addr[dev];
+    return ECASQ_OK;
 }
 
 static int check_ws(const void *ws, size_t bytes, const Layout &L) {
@@ -626,6 +652,42 @@ int ecasq_quantize(const float *x, int64_t d, const float *Q, int32_t m, uint64_
     DevStatus h;
     ECASQ_CUDA_TRY(cudaMemcpyAsync(&h, ds, sizeof(h), cudaMemcpyDeviceToHost, st));
     if (h_emp) ECASQ_CUDA_TRY(cudaMemcpyAsync(ch.data(), counts, 4 * (size_t)m, cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    if (h.range_err) return ECASQ_ERANGE;
+    if (h_emp) {
+        double he = 0.0, dd_ = (double)d;
+        for (int r = 0; r < m; r++) {
+            double f = (double)ch[r] / dd_;
+            if (f > 0.0) he += -f * log2(f);
+        }
+        *h_emp = he;
+    }
+    return ECASQ_OK;
+}
+
+// Same checks, kernel and host arithmetic as ecasq_quantize; the status record
+// lives in the fixed scratch block and host copies in fixed-size arrays.
+int ecasq_quantize_noalloc(const float *x, int64_t d, const float *Q, int32_t m, uint64_t seed, uint8_t *idx,
+                           uint32_t *counts, double *h_emp, ecasq_stream_t stream) {
+    if (!x || !Q || !idx || !counts || d < 1 || d >= ((int64_t)1 << 31) || m < 1 || m > kMaxS) return ECASQ_EINVAL;
+    void *scratch = nullptr;
+    int rc = noalloc_scratch(&scratch);
+    if (rc) return rc;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    DevStatus *ds = reinterpret_cast<DevStatus *>(scratch);
+    float qh[kMaxS];
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(qh, Q, 4 * (size_t)m, cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaMemsetAsync(ds, 0, sizeof(DevStatus), st));
+    ECASQ_CUDA_TRY(cudaMemsetAsync(counts, 0, 4 * (size_t)m, st));
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    for (int r = 1; r < m; r++)
+        if (!(qh[r] > qh[r - 1])) return ECASQ_EINVAL;
+    rc = launch_quantize(x, d, Q, m, seed, idx, counts, ds, num_sms(), st);
+    if (rc) return rc;
+    uint32_t ch[kMaxS];
+    DevStatus h;
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(&h, ds, sizeof(h), cudaMemcpyDeviceToHost, st));
+    if (h_emp) ECASQ_CUDA_TRY(cudaMemcpyAsync(ch, counts, 4 * (size_t)m, cudaMemcpyDeviceToHost, st));
     ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
     if (h.range_err) return ECASQ_ERANGE;
     if (h_emp) {

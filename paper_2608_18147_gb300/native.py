@@ -80,6 +80,7 @@ def lib():
             "ecasq_refine": (C.c_int, [vp, i64, vp, i32, dbl, dbl, i32, dbl, u32, vp, sz, PR, vp]),
             "ecasq_evaluate": (C.c_int, [vp, i64, vp, i32, vp, sz, pd, vp]),
             "ecasq_quantize": (C.c_int, [vp, i64, vp, i32, u64, vp, vp, vp, sz, pd, vp]),
+            "ecasq_quantize_noalloc": (C.c_int, [vp, i64, vp, i32, u64, vp, vp, pd, vp]),
             "ecasq_solve_batched": (C.c_int, [vp, i64, i64, PP, vp, sz, vp, vp, PR, vp]),
             "ecasq_prepare": (C.c_int, [vp, i64, vp, sz, vp, vp, vp, vp, vp, pi64, vp]),
             "ecasq_kernel_launches": (i64, []),
@@ -97,7 +98,8 @@ def exported_symbols():
     L = lib()
     names = []
     for name in ("ecasq_version", "ecasq_strerror", "ecasq_workspace_size", "ecasq_solve", "ecasq_dp_pass",
-                 "ecasq_dp_tables", "ecasq_refine", "ecasq_evaluate", "ecasq_quantize", "ecasq_solve_batched",
+                 "ecasq_dp_tables", "ecasq_refine", "ecasq_evaluate", "ecasq_quantize", "ecasq_quantize_noalloc",
+                 "ecasq_solve_batched",
                  "ecasq_prepare", "ecasq_kernel_launches"):
         if hasattr(L, name):
             names.append(name)
@@ -262,6 +264,19 @@ def ecasq_quantize(x, Q, seed, ws=None, idx=None, counts=None):
                               _ptr(counts), _ptr(ws), ws.numel(), C.byref(he), _stream())
     _check(rc, "ecasq_quantize")
     return idx, counts, he.value
+
+
+def ecasq_quantize_noalloc(x, Q, seed, idx, counts):
+    """ecasq_quantize without a workspace; idx (uint8 [d]) and counts (int32 [m])
+    are the caller's device tensors.  Returns the empirical entropy."""
+    x = _dev_f32(x)
+    Q = _dev_f32(Q)
+    he = C.c_double()
+    rc = lib().ecasq_quantize_noalloc(_ptr(x), x.numel(), _ptr(Q), Q.numel(),
+                                      C.c_uint64(int(seed) & 0xFFFFFFFFFFFFFFFF), _ptr(idx), _ptr(counts),
+                                      C.byref(he), _stream())
+    _check(rc, "ecasq_quantize_noalloc")
+    return he.value
 
 
 def ecasq_solve_batched(X, s, budget_bits=0.0, lambda_=-1.0, ws=None, **kw):
