@@ -16,7 +16,8 @@ namespace ecasq {
 int launch_dp_reference(const Prefix &P, const double *lamp, int G, int s, double *dp64, int32_t *bp,
                         cudaStream_t st);
 int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, const Layout &L, cudaStream_t st,
-                   bool exact_s, bool exact_tables);
+                   bool exact_s, bool exact_tables, float *costs, bool build_costs);
+size_t resident_costs_bytes(int64_t d);
 int launch_traceback_eval(const Prefix &P, int G, int s, int exact_s, const double *dp64, const int32_t *bp,
                           int32_t *qidx, int32_t *mcount, double *metrics, cudaStream_t st);
 int launch_eval_codebook(const Prefix &P, const int32_t *a, int m, double *out3, cudaStream_t st);
@@ -86,6 +87,8 @@ size_t make_layout(int64_t d, int32_t s, int64_t rows, Layout *L) {
     L->refine = take(4 * 2 * kMaxS + 256 + 8 * 8);
     L->refine_part = take(refine_scratch_bytes(d));
     L->band = take(fast_dp_band_bytes(d, s));
+    L->costs = 0;
+    L->costs_bytes = 0;
     L->total = off;
     L->d = d;
     L->s = s;
@@ -129,6 +132,17 @@ static int noalloc_scratch(void **out) {
     return ECASQ_OK;
 }
 
+// ECASQ_RESIDENT_COSTS: the interval-cost tiles follow the common layout.
+static int add_resident_costs(uint32_t flags, Layout *L) {
+    if (!(flags & ECASQ_RESIDENT_COSTS)) return ECASQ_OK;
+    size_t cb = resident_costs_bytes(L->d);
+    if (!cb || L->total > SIZE_MAX - align256(cb)) return ECASQ_EINVAL;
+    L->costs = L->total;
+    L->costs_bytes = cb;
+    L->total += align256(cb);
+    return ECASQ_OK;
+}
+
 static int check_ws(const void *ws, size_t bytes, const Layout &L) {
     if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255) != 0 || bytes < L.total) return ECASQ_EWORKSPACE;
     return ECASQ_OK;
@@ -167,15 +181,21 @@ struct PassOut {
 
 // One DP pass over a prepared workspace: DP at lambda'_g (g < G), traceback,
 // evaluation, results to the host.
+// costs_built: in/out, whether the resident interval costs (if the layout has
+// them) already hold this call's prefix data.
 static int dp_pass_prepared(void *ws, const Layout &L, const Prefix &P, int s, const double *lamp, int G,
-                            uint32_t flags, cudaStream_t st, PassOut &out) {
+                            uint32_t flags, cudaStream_t st, PassOut &out, bool *costs_built) {
     double *dp64 = wsp<double>(ws, L.dp64);
     int32_t *bp = wsp<int32_t>(ws, L.bp);
     int rc;
-    if (flags & ECASQ_DP_REFERENCE)
+    if (flags & ECASQ_DP_REFERENCE) {
         rc = launch_dp_reference(P, lamp, G, s, dp64, bp, st);
-    else
-        rc = launch_dp_fast(P, lamp, G, s, ws, L, st, (flags & ECASQ_EXACT_S) != 0, (flags & ECASQ_EXACT_TABLES) != 0);
+    } else {
+        float *costs = L.costs_bytes ? wsp<float>(ws, L.costs) : nullptr;
+        rc = launch_dp_fast(P, lamp, G, s, ws, L, st, (flags & ECASQ_EXACT_S) != 0, (flags & ECASQ_EXACT_TABLES) != 0,
+                            costs, costs && !*costs_built);
+        if (costs && rc == ECASQ_OK) *costs_built = true;
+    }
     if (rc != ECASQ_OK) return rc;
     timer_collect();
     rc = launch_traceback_eval(P, G, s, (flags & ECASQ_EXACT_S) ? 1 : 0, dp64, bp, wsp<int32_t>(ws, L.qidx),
@@ -322,6 +342,14 @@ size_t ecasq_workspace_size(int64_t d, int32_t s, int64_t rows) {
     return make_layout(d, s, rows, &L);
 }
 
+size_t ecasq_workspace_size_flags(int64_t d, int32_t s, int64_t rows, uint32_t flags) {
+    size_t base = ecasq_workspace_size(d, s, rows);
+    if (!base || !(flags & ECASQ_RESIDENT_COSTS)) return base;
+    size_t cb = resident_costs_bytes(d);
+    if (!cb || base > SIZE_MAX - align256(cb)) return 0;
+    return base + align256(cb);
+}
+
 int ecasq_prepare(const float *x, int64_t d, void *ws, size_t ws_bytes, float *v, int64_t *w, int64_t *N,
                   double *S, double *S2, int64_t *p_out, ecasq_stream_t stream) {
     if (!x || d < 1 || d >= ((int64_t)1 << 31) || !v || !w || !N || !S || !S2 || !p_out) return ECASQ_EINVAL;
@@ -354,7 +382,9 @@ int ecasq_dp_pass(const float *x, int64_t d, int32_t s, const double *lambdas, i
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     Layout L;
     make_layout(d, s, 1, &L);
-    int rc = check_ws(ws, ws_bytes, L);
+    int rc = add_resident_costs(flags, &L);
+    if (rc) return rc;
+    rc = check_ws(ws, ws_bytes, L);
     if (rc) return rc;
     int64_t p;
     double n2;
@@ -373,7 +403,8 @@ int ecasq_dp_pass(const float *x, int64_t d, int32_t s, const double *lambdas, i
     double lamp[kMaxG];
     for (int g = 0; g < G; g++) lamp[g] = lambdas[g] * n2;
     PassOut po;
-    rc = dp_pass_prepared(ws, L, P, s, lamp, G, flags, st, po);
+    bool costs_built = false;
+    rc = dp_pass_prepared(ws, L, P, s, lamp, G, flags, st, po, &costs_built);
     if (rc) return rc;
     rc = launch_gather_q(P.v, wsp<int32_t>(ws, L.qidx), wsp<int32_t>(ws, L.mcount), G, s, Q_out, st);
     if (rc) return rc;
@@ -451,7 +482,9 @@ int ecasq_solve(const float *x, int64_t d, const ecasq_params_t *prm, void *ws, 
     g_timer.launches = 0;
     Layout L;
     make_layout(d, s, 1, &L);
-    int rc = check_ws(ws, ws_bytes, L);
+    int rc = add_resident_costs(prm->flags, &L);
+    if (rc) return rc;
+    rc = check_ws(ws, ws_bytes, L);
     if (rc) return rc;
     int64_t p;
     double n2;
@@ -459,6 +492,7 @@ int ecasq_solve(const float *x, int64_t d, const ecasq_params_t *prm, void *ws, 
     if (rc) return rc;
     Prefix P = make_prefix(ws, L, p, d);
     double zero3[3] = {0.0, 0.0, 0.0};
+    bool costs_built = false;
     if (p == 1) {
         ECASQ_CUDA_TRY(cudaMemcpyAsync(Q, P.v, 4, cudaMemcpyDeviceToDevice, st));
         ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
@@ -474,7 +508,7 @@ int ecasq_solve(const float *x, int64_t d, const ecasq_params_t *prm, void *ws, 
         int G = (int)lams.size();
         for (int g = 0; g < G; g++) lamp[g] = lams[g] * n2;
         PassOut po;
-        int r = dp_pass_prepared(ws, L, P, s, lamp, G, prm->flags, st, po);
+        int r = dp_pass_prepared(ws, L, P, s, lamp, G, prm->flags, st, po, &costs_built);
         if (r) return r;
         passes++;
         nlam += G;

@@ -67,6 +67,8 @@ struct Layout {
     size_t refine;         // refinement scratch
     size_t refine_part;    // refinement per-chunk partial minima
     size_t band;           // fast DP band lists
+    size_t costs;          // resident interval-cost tiles (ECASQ_RESIDENT_COSTS), after everything else
+    size_t costs_bytes;    // 0 when absent
     size_t total;
     int64_t d;
     int32_t s;

@@ -64,6 +64,11 @@ constexpr int MAXCONS = 256;
 constexpr int NMEM = 8;        // members kept inline per output
 constexpr int64_t kMaxFastP = (int64_t)1 << 20;
 constexpr uint32_t kSpinLimit = 1u << 26;
+constexpr uint32_t kCopySpinLimit = 1u << 22;  // waits on bulk copies (microseconds when healthy)
+// Resident interval costs: per tile, C[64][PSTR] then Phi[64][PSTR] (the shared-memory layout).
+constexpr int kCostHalfFloats = BJ * PSTR;
+constexpr uint32_t kCostHalfBytes = (uint32_t)(kCostHalfFloats * sizeof(float));  // 17408, a multiple of 16
+constexpr size_t kCostTileFloats = 2 * (size_t)kCostHalfFloats;
 
 // Band word (64 bits): bits 0-1 number of tile runs (0..2), bit 2 overflow; run r
 // (r = 0, 1) at bit 3 + 19 r: first tile (14 bits) and length - 1 (5 bits, <= 32 tiles).
@@ -109,6 +114,7 @@ struct FastArgs {
     int32_t *members;      // [G][s+1][ps][NMEM]
     uint8_t *need;         // [G][s+1][ps] output resolved exactly
     float *corner;         // [nJ(nJ-1)/2][8]: state of pair (64K+63, 64J), K < J (N, E, Ec, A, Ac, C, Cc)
+    const float *costs;    // resident interval costs (tile (K, J) at J(J+1)/2 + K), or null: computed per tile
     int *done;             // [nsplit][nJ]
     int *ticket;
     int *abort_flag;
@@ -312,6 +318,66 @@ __device__ __forceinline__ float min3(float a, float b, float c) {
     return d;
 }
 
+// ------------------------------------------- bulk copies (TMA engine) and mbarriers
+__device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+__device__ __forceinline__ void mbar_init(unsigned long long *bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_fence_init() { asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory"); }
+// arrive once and raise the phase's expected transaction count by `bytes`
+__device__ __forceinline__ void mbar_expect_tx(unsigned long long *bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_test(unsigned long long *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tmbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Bounded wait for phase `parity` of `bar`: on expiry record a timeout, raise the abort flag and return.
+__device__ __forceinline__ void mbar_wait_bounded(unsigned long long *bar, uint32_t parity, DevStatus *st, int *abort_flag) {
+    uint32_t spins = 0;
+    while (!mbar_test(bar, parity)) {
+        if (++spins > kCopySpinLimit) {
+            st->timeout = 1;
+            atomicExch(abort_flag, 1);
+            return;
+        }
+        __nanosleep(32);
+    }
+}
+__device__ __forceinline__ uint64_t policy_evict_first() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+// global -> shared, completion counted on `bar` (bytes and both addresses multiples of 16)
+__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, unsigned long long *bar,
+                                         uint64_t policy) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(
+            smem_u32(dst)),
+        "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
+        : "memory");
+}
+// shared -> global, bulk-group completion
+__device__ __forceinline__ void bulk_s2g(void *dst, const void *src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst), "r"(smem_u32(src)), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read_all() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// generic-proxy writes to shared memory -> visible to later bulk copies
+__device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+__host__ __device__ __forceinline__ size_t cost_tile_idx(int64_t K, int64_t J) {
+    return (size_t)J * (size_t)(J + 1) / 2 + (size_t)K;
+}
+
 // ------------------------------------------------------------ shared memory
 struct TileMeta {
     int J, K, split, kind;  // kind: 0 off-diagonal, 1 diagonal, 2 stop
@@ -327,10 +393,129 @@ struct __align__(16) Smem {
     float wsum[2][2];                     // producer scan: per-warp totals
     int ticket;
     int pad[3];
+    unsigned long long mbar[2];           // resident costs: bulk-copy completion of buffer b
+    unsigned long long pad2[2];
     // followed by dp32 slices [2][Gc * (s-2)][BK] (dynamic)
 };
 
+// ------------------------------------------------------- one tile of interval costs
+// Per-k constants of the tile starting at k0 (k = k0 + jl): v_k, w_{k+1}, v_{k+1} - v_k.
+__device__ __forceinline__ void tile_consts(const FastArgs &a, int64_t k0, int jl, float *kv, float *kw, float *kd) {
+    int64_t k = k0 + jl;
+    kv[jl] = k < a.p ? a.v[k] : 0.f;
+    kw[jl] = (k + 1 < a.p) ? a.wf[k + 1] : 0.f;
+    kd[jl] = (k + 1 < a.p) ? __fsub_rn(a.v[k + 1], a.v[k]) : 0.f;
+}
+
+// Interval costs C[k, j] and Phi[k, j] of column j = 64J + jl for the 64 k of tile K
+// (k descending) into Cr[jl][.] and Pr[jl][.]; +inf / 0 where k >= j or j >= p.
+// Threads 0..63 of the block all call it (the anchors' scans synchronise them on
+// BAR_PROD); kv, kw, kd hold tile_consts of tile K, visible to all 64.
+__device__ void tile_columns(const FastArgs &a, int64_t K, int64_t J, int jl, const float *kv, const float *kw,
+                             const float *kd, float (*wsum)[2], float (*Cr)[PSTR], float (*Pr)[PSTR]) {
+    const bool diag = (K == J);
+    const int64_t j0 = J * BJ;
+    const int64_t j = j0 + jl;
+    const float d_f = (float)a.d;
+        // anchors of the 64 columns at k = 64K + 63: the corner state of (K, J) advanced
+        // along j with compensated exclusive scans of non-negative increments
+        Rec anchor_r = rec_empty();
+        if (!diag) {
+            const float *cp = a.corner + 8 * corner_idx(K, J);
+            float vk = kv[BK - 1];
+            int64_t jt = j0 + jl;  // increment of column jl: moving j from jt to jt + 1
+            bool okc = jt + 1 < a.p;
+            float wn = okc ? a.wf[jt + 1] : 0.f;
+            float vn = okc ? a.v[jt + 1] : 0.f;
+            float dj = okc ? __fsub_rn(vn, a.v[jt]) : 0.f;
+            float nx, nc, ax, ac, ex, ec, cx, cc;
+            scan64_excl(wn, nx, nc, wsum);                               // N (exact)
+            scan64_excl(okc ? __fmul_rn(wn, __fsub_rn(vn, vk)) : 0.f, ax, ac, wsum);  // A
+            float Nj = __fadd_rn(cp[0], __fadd_rn(nx, nc));
+            float Aj = __fadd_rn(__fadd_rn(cp[3], ax), __fadd_rn(cp[4], ac));
+            scan64_excl(__fmul_rn(dj, Nj), ex, ec, wsum);              // E
+            scan64_excl(__fmul_rn(dj, Aj), cx, cc, wsum);              // C
+            anchor_r.N = Nj;
+            anchor_r.E = cp[1]; anchor_r.Ec = cp[2];
+            pair_add(anchor_r.E, anchor_r.Ec, ex, ec);
+            anchor_r.A = cp[3]; anchor_r.Ac = cp[4];
+            pair_add(anchor_r.A, anchor_r.Ac, ax, ac);
+            anchor_r.C = cp[5]; anchor_r.Cc = cp[6];
+            pair_add(anchor_r.C, anchor_r.Cc, cx, cc);
+        }
+        // interval costs of column j for k in the tile (descending k)
+        if (j < a.p) {
+            float vj = a.v[j];
+            Rec r;
+            int kl_hi;
+            if (diag) {
+                r = rec_empty();
+                kl_hi = (int)(j - j0) - 1;  // k = j-1 first
+                // state for k = j: empty; step to k = j-1 adds t = j
+                for (int kl = BK - 1; kl > kl_hi; kl--) { Cr[jl][kl] = CUDART_INF_F; Pr[jl][kl] = 0.f; }
+                for (int kl = kl_hi; kl >= 0; kl--) {
+                    rec_step(r, vj, kv[kl + 1], kw[kl], kd[kl]);  // kl + 1 <= 63
+                    float c, ph;
+                    rec_emit(r, vj, kv[kl], d_f, a.invd, c, ph);
+                    Cr[jl][kl] = c; Pr[jl][kl] = ph;
+                }
+            } else {
+                r = anchor_r;
+                Rec nxt = r;
+                for (int kl = BK - 1; kl >= 0; kl--) {
+                    Rec cur = nxt;
+                    if (kl > 0) rec_step(nxt, vj, kv[kl], kw[kl - 1], kd[kl - 1]);  // state of k - 1
+                    float c, ph;
+                    rec_emit(cur, vj, kv[kl], d_f, a.invd, c, ph);
+                    Cr[jl][kl] = c; Pr[jl][kl] = ph;
+                }
+            }
+        } else {
+            for (int kl = 0; kl < BK; kl++) { Cr[jl][kl] = CUDART_INF_F; Pr[jl][kl] = 0.f; }
+        }
+}
+
+// Resident interval costs: every tile (K <= J) computed once, exactly as the
+// wavefront's own producer computes it, staged in shared memory and written out
+// by a bulk copy.  64 threads per block; blocks stride over the tiles.
+struct __align__(16) BuildSmem {
+    float C[BJ][PSTR];
+    float Phi[BJ][PSTR];
+    float kv[BK], kw[BK], kd[BK];
+    float wsum[2][2];
+};
+
+__global__ void __launch_bounds__(NPROD) k_build_costs(FastArgs a, float *costs) {
+    __shared__ BuildSmem S;
+    const int jl = threadIdx.x;
+    const int64_t ntiles = (int64_t)a.nJ * (a.nJ + 1) / 2;
+    for (int64_t t = blockIdx.x; t < ntiles; t += gridDim.x) {
+        // invert t = J(J+1)/2 + K, K <= J
+        int64_t J = (int64_t)((sqrt(8.0 * (double)t + 1.0) - 1.0) * 0.5);
+        while (J * (J + 1) / 2 > t) J--;
+        while ((J + 1) * (J + 2) / 2 <= t) J++;
+        int64_t K = t - J * (J + 1) / 2;
+        tile_consts(a, K * BK, jl, S.kv, S.kw, S.kd);
+        bar_sync(BAR_PROD, NPROD);
+        tile_columns(a, K, J, jl, S.kv, S.kw, S.kd, S.wsum, S.C, S.Phi);
+        fence_proxy_async_smem();
+        bar_sync(BAR_PROD, NPROD);
+        if (jl == 0) {
+            float *dst = costs + (size_t)t * kCostTileFloats;
+            bulk_s2g(dst, &S.C[0][0], kCostHalfBytes);
+            bulk_s2g(dst + kCostHalfFloats, &S.Phi[0][0], kCostHalfBytes);
+            bulk_commit();
+            bulk_wait_read_all();  // shared buffers free again
+        }
+        bar_sync(BAR_PROD, NPROD);
+    }
+    if (jl == 0) bulk_wait_all();
+}
+
 // ------------------------------------------------------------------ kernel
+// kCosts: the interval-cost tiles come from the resident table (one bulk copy per
+// half tile); otherwise the producer warps compute them (tile_columns).
+template <bool kCosts>
 __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     Smem &S = *reinterpret_cast<Smem *>(smem_raw);
@@ -339,12 +524,20 @@ __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
     const int rowsDP = a.Gc * L;          // staged dp32 rows per tile (layers 2..s-1)
     const int tid = threadIdx.x;
     const int nall = NPROD + a.ncons;
+    if (kCosts) {
+        if (tid == 0) {
+            mbar_init(&S.mbar[0], 1);
+            mbar_init(&S.mbar[1], 1);
+            mbar_fence_init();
+        }
+        __syncthreads();
+    }
 
     if (tid < NPROD) {
         // =========================== producer warps ===========================
         const int jl = tid;  // column within the block
         uint32_t n = 0;      // tile sequence number
-        const float d_f = (float)a.d;
+        const uint64_t policy = kCosts ? policy_evict_first() : 0ull;
         for (;;) {
             if (tid == 0) S.ticket = atomicAdd(a.ticket, 1);
             bar_sync(BAR_PROD, NPROD);
@@ -363,8 +556,7 @@ __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
                     break;
                 }
                 bool diag = (K == J);
-                int64_t k0 = (int64_t)K * BK, j0 = (int64_t)J * BJ;
-                int64_t j = j0 + jl;
+                int64_t k0 = (int64_t)K * BK;
                 // wait for column block K (bounded); the diagonal needs nothing
                 if (!diag && tid == 0) {
                     const int *flag = a.done + (size_t)split * a.nJ + K;
@@ -380,12 +572,15 @@ __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
                     }
                 }
                 bar_sync(BAR_PROD, NPROD);
-                // per-k constants of the tile
-                {
-                    int64_t k = k0 + jl;
-                    S.kv[jl] = k < a.p ? a.v[k] : 0.f;
-                    S.kw[jl] = (k + 1 < a.p) ? a.wf[k + 1] : 0.f;
-                    S.kd[jl] = (k + 1 < a.p) ? __fsub_rn(a.v[k + 1], a.v[k]) : 0.f;
+                if (kCosts) {
+                    if (tid == 0) {
+                        const float *src = a.costs + cost_tile_idx(K, J) * kCostTileFloats;
+                        mbar_expect_tx(&S.mbar[b], 2 * kCostHalfBytes);
+                        bulk_g2s(&S.C[b][0][0], src, kCostHalfBytes, &S.mbar[b], policy);
+                        bulk_g2s(&S.Phi[b][0][0], src + kCostHalfFloats, kCostHalfBytes, &S.mbar[b], policy);
+                    }
+                } else {
+                    tile_consts(a, k0, jl, S.kv, S.kw, S.kd);
                 }
                 // dp32 slice of rows (g, layer 2..s-1) for k in the tile (cp.async, L2 only)
                 if (!diag) {
@@ -408,64 +603,11 @@ __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
                     }
                     asm volatile("cp.async.commit_group;" ::: "memory");
                 }
-                bar_sync(BAR_PROD, NPROD);
-                // anchors of the 64 columns at k = 64K + 63: the corner state of (K, J) advanced
-                // along j with compensated exclusive scans of non-negative increments
-                Rec anchor_r = rec_empty();
-                if (!diag) {
-                    const float *cp = a.corner + 8 * corner_idx(K, J);
-                    float vk = S.kv[BK - 1];
-                    int64_t jt = j0 + jl;  // increment of column jl: moving j from jt to jt + 1
-                    bool okc = jt + 1 < a.p;
-                    float wn = okc ? a.wf[jt + 1] : 0.f;
-                    float vn = okc ? a.v[jt + 1] : 0.f;
-                    float dj = okc ? __fsub_rn(vn, a.v[jt]) : 0.f;
-                    float nx, nc, ax, ac, ex, ec, cx, cc;
-                    scan64_excl(wn, nx, nc, S.wsum);                               // N (exact)
-                    scan64_excl(okc ? __fmul_rn(wn, __fsub_rn(vn, vk)) : 0.f, ax, ac, S.wsum);  // A
-                    float Nj = __fadd_rn(cp[0], __fadd_rn(nx, nc));
-                    float Aj = __fadd_rn(__fadd_rn(cp[3], ax), __fadd_rn(cp[4], ac));
-                    scan64_excl(__fmul_rn(dj, Nj), ex, ec, S.wsum);              // E
-                    scan64_excl(__fmul_rn(dj, Aj), cx, cc, S.wsum);              // C
-                    anchor_r.N = Nj;
-                    anchor_r.E = cp[1]; anchor_r.Ec = cp[2];
-                    pair_add(anchor_r.E, anchor_r.Ec, ex, ec);
-                    anchor_r.A = cp[3]; anchor_r.Ac = cp[4];
-                    pair_add(anchor_r.A, anchor_r.Ac, ax, ac);
-                    anchor_r.C = cp[5]; anchor_r.Cc = cp[6];
-                    pair_add(anchor_r.C, anchor_r.Cc, cx, cc);
-                }
-                // interval costs of column j for k in the tile (descending k)
-                float (*Cr)[PSTR] = S.C[b];
-                float (*Pr)[PSTR] = S.Phi[b];
-                if (j < a.p) {
-                    float vj = a.v[j];
-                    Rec r;
-                    int kl_hi;
-                    if (diag) {
-                        r = rec_empty();
-                        kl_hi = (int)(j - j0) - 1;  // k = j-1 first
-                        // state for k = j: empty; step to k = j-1 adds t = j
-                        for (int kl = BK - 1; kl > kl_hi; kl--) { Cr[jl][kl] = CUDART_INF_F; Pr[jl][kl] = 0.f; }
-                        for (int kl = kl_hi; kl >= 0; kl--) {
-                            rec_step(r, vj, S.kv[kl + 1], S.kw[kl], S.kd[kl]);  // kl + 1 <= 63
-                            float c, ph;
-                            rec_emit(r, vj, S.kv[kl], d_f, a.invd, c, ph);
-                            Cr[jl][kl] = c; Pr[jl][kl] = ph;
-                        }
-                    } else {
-                        r = anchor_r;
-                        Rec nxt = r;
-                        for (int kl = BK - 1; kl >= 0; kl--) {
-                            Rec cur = nxt;
-                            if (kl > 0) rec_step(nxt, vj, S.kv[kl], S.kw[kl - 1], S.kd[kl - 1]);  // state of k - 1
-                            float c, ph;
-                            rec_emit(cur, vj, S.kv[kl], d_f, a.invd, c, ph);
-                            Cr[jl][kl] = c; Pr[jl][kl] = ph;
-                        }
-                    }
+                if (kCosts) {
+                    mbar_wait_bounded(&S.mbar[b], (n >> 1) & 1u, a.st, a.abort_flag);
                 } else {
-                    for (int kl = 0; kl < BK; kl++) { Cr[jl][kl] = CUDART_INF_F; Pr[jl][kl] = 0.f; }
+                    bar_sync(BAR_PROD, NPROD);
+                    tile_columns(a, K, J, jl, S.kv, S.kw, S.kd, S.wsum, S.C[b], S.Phi[b]);
                 }
                 if (!diag) asm volatile("cp.async.wait_all;" ::: "memory");
                 if (tid == 0) S.meta[b] = {J, K, split, diag ? 1 : 0};
@@ -494,6 +636,7 @@ __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
         bar_sync(BAR_FULL + b, nall);
         TileMeta m = S.meta[b];
         if (m.kind == 2) { bar_arrive(BAR_EMPTY + b, nall); break; }
+        if (kCosts) mbar_wait_bounded(&S.mbar[b], (n >> 1) & 1u, a.st, a.abort_flag);  // bulk copies landed
         const int g = m.split * a.Gc + gl;
         const bool own = active && g < a.G;
         const int64_t j0 = (int64_t)m.J * BJ;
@@ -676,10 +819,19 @@ __device__ __forceinline__ float cand32(float dprev, float lam, float C, float P
 template <typename F>
 __device__ void visit_tile(const FastArgs &a, int g, int i, int64_t j, int64_t K, float thr, F &&f) {
     int64_t J = j / BJ, j0 = J * BJ, k0 = K * BK;
-    float vj = a.v[j];
     float lam = a.prm->lam32[g];
-    const float d_f = (float)a.d;
     const float *prev = a.dp32 + oidx(a, g, i - 1, 0);
+    if (a.costs) {
+        // the wavefront's own interval costs, read back from the resident table
+        const float *cr = a.costs + cost_tile_idx(K, J) * kCostTileFloats + (size_t)(j - j0) * PSTR;
+        const float *pr = cr + kCostHalfFloats;
+        int64_t khi = (K == J) ? j - 1 : k0 + BK - 1;
+        for (int64_t k = khi; k >= k0; k--)
+            if (cand32(prev[k], lam, cr[k - k0], pr[k - k0]) <= thr) f(k);
+        return;
+    }
+    float vj = a.v[j];
+    const float d_f = (float)a.d;
     Rec r;
     int64_t khi;
     float c, ph;
@@ -845,8 +997,17 @@ static void band_factors(int s, FastParams &fp) {
     }
 }
 
+size_t resident_costs_bytes(int64_t d) {
+    if (d < 1) return 0;
+    double nJ = (double)cdiv(d, BJ);
+    double bytes = nJ * (nJ + 1.0) * 0.5 * (double)kCostTileFloats * sizeof(float);
+    if (!(bytes < 9.0e18)) return 0;
+    size_t n = (size_t)cdiv(d, BJ);
+    return n * (n + 1) / 2 * kCostTileFloats * sizeof(float);
+}
+
 int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, const Layout &Lw, cudaStream_t st,
-                   bool exact_s, bool exact_tables) {
+                   bool exact_s, bool exact_tables, float *costs, bool build_costs) {
     double *dp64 = wsp<double>(ws, Lw.dp64);
     int32_t *bp = wsp<int32_t>(ws, Lw.bp);
     // small inputs, very large ones and huge counts take the reference kernel
@@ -890,6 +1051,7 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     FastParams *dprm = reinterpret_cast<FastParams *>(base);
     base += align256(sizeof(FastParams));
     a.corner = reinterpret_cast<float *>(base);
+    a.costs = costs;
     a.prm = dprm;
     a.done = flags;
     a.ticket = flags + (size_t)kMaxG * a.nJ;
@@ -909,20 +1071,30 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     note_launch();
     k_fast_base<<<(unsigned)cdiv(P.p - 1, 128), 128, 0, st>>>(P, a, dp64, bp);
     ECASQ_LAUNCH_CHECK();
-    if (a.nJ > 1) {
+    int dev = 0, nsm = 0;
+    ECASQ_CUDA_TRY(cudaGetDevice(&dev));
+    ECASQ_CUDA_TRY(cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev));
+    // corner states: needed by every tile the producer computes (per pass, or once into the table)
+    if (a.nJ > 1 && (!costs || build_costs)) {
         note_launch();
         k_corners<<<(unsigned)std::min<int64_t>(cdiv((int64_t)a.nJ * (a.nJ - 1) / 2, 128), 152 * 64), 128, 0, st>>>(a);
         ECASQ_LAUNCH_CHECK();
     }
+    if (costs && build_costs) {
+        int per_sm = 0;
+        ECASQ_CUDA_TRY(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_build_costs, NPROD, 0));
+        int64_t ntiles = (int64_t)a.nJ * (a.nJ + 1) / 2;
+        note_launch();
+        k_build_costs<<<(unsigned)std::min<int64_t>(ntiles, (int64_t)nsm * std::max(per_sm, 1)), NPROD, 0, st>>>(a, costs);
+        ECASQ_LAUNCH_CHECK();
+    }
     size_t smem = smem_bytes(a.Gc, s);
-    ECASQ_CUDA_TRY(cudaFuncSetAttribute(k_wavefront, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-    int dev = 0, nsm = 0;
-    ECASQ_CUDA_TRY(cudaGetDevice(&dev));
-    ECASQ_CUDA_TRY(cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev));
+    auto wave = costs ? k_wavefront<true> : k_wavefront<false>;
+    ECASQ_CUDA_TRY(cudaFuncSetAttribute(wave, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     int grid = std::min(nsm, a.nJ * a.nsplit);
     timer_begin(st);
     note_launch();
-    k_wavefront<<<grid, NPROD + a.ncons, smem, st>>>(a);
+    wave<<<grid, NPROD + a.ncons, smem, st>>>(a);
     timer_end(st);
     ECASQ_LAUNCH_CHECK();
     const int ilo = exact_s ? s : 2;

@@ -17,7 +17,7 @@ import numpy as np
 from . import build as _build
 
 OK, EINVAL, ENONFINITE, EINFEASIBLE, EWORKSPACE, ECUDA, ETIMEOUT, ERANGE = 0, -1, -2, -3, -4, -5, -6, -7
-EXACT_S, NO_REFINE_GUARD, DP_REFERENCE, TIME_KERNELS, EXACT_TABLES = 1, 2, 4, 8, 16
+EXACT_S, NO_REFINE_GUARD, DP_REFERENCE, TIME_KERNELS, EXACT_TABLES, RESIDENT_COSTS = 1, 2, 4, 8, 16, 32
 
 _lock = threading.Lock()
 _lib = None
@@ -74,6 +74,7 @@ def lib():
             "ecasq_version": (C.c_int, []),
             "ecasq_strerror": (C.c_char_p, [C.c_int]),
             "ecasq_workspace_size": (sz, [i64, i32, i64]),
+            "ecasq_workspace_size_flags": (sz, [i64, i32, i64, u32]),
             "ecasq_solve": (C.c_int, [vp, i64, PP, vp, sz, vp, PR, vp]),
             "ecasq_dp_pass": (C.c_int, [vp, i64, i32, pd, i32, u32, vp, sz, vp, pi32, pd, vp]),
             "ecasq_dp_tables": (C.c_int, [vp, sz, i32, vp, vp, pi64, vp]),
@@ -97,7 +98,8 @@ def exported_symbols():
     """Names declared in include/ecasq.h that the loaded library exports."""
     L = lib()
     names = []
-    for name in ("ecasq_version", "ecasq_strerror", "ecasq_workspace_size", "ecasq_solve", "ecasq_dp_pass",
+    for name in ("ecasq_version", "ecasq_strerror", "ecasq_workspace_size", "ecasq_workspace_size_flags",
+                 "ecasq_solve", "ecasq_dp_pass",
                  "ecasq_dp_tables", "ecasq_refine", "ecasq_evaluate", "ecasq_quantize", "ecasq_quantize_noalloc",
                  "ecasq_solve_batched",
                  "ecasq_prepare", "ecasq_kernel_launches"):
@@ -154,10 +156,14 @@ def ecasq_workspace_size(d, s, rows=1) -> int:
     return int(lib().ecasq_workspace_size(int(d), int(s), int(rows)))
 
 
-def workspace(d, s, rows=1):
+def ecasq_workspace_size_flags(d, s, rows=1, flags=0) -> int:
+    return int(lib().ecasq_workspace_size_flags(int(d), int(s), int(rows), int(flags)))
+
+
+def workspace(d, s, rows=1, flags=0):
     """A device workspace (torch uint8 tensor; CUDA allocations are 256-byte aligned)."""
     torch = _torch()
-    n = ecasq_workspace_size(d, s, rows)
+    n = ecasq_workspace_size_flags(d, s, rows, flags)
     if n == 0:
         raise EcasqError(EINVAL, "ecasq_workspace_size")
     return torch.empty(n, dtype=torch.uint8, device="cuda")
@@ -177,7 +183,7 @@ def ecasq_solve(x, s, budget_bits=0.0, lambda_=-1.0, ws=None, **kw):
     x = _dev_f32(x)
     d = x.numel()
     if ws is None:
-        ws = workspace(d, s)
+        ws = workspace(d, s, flags=kw.get("flags", 0))
     prm = make_params(s, budget_bits, lambda_, **kw)
     Q = torch.zeros(s, dtype=torch.float32, device="cuda")
     res = Result()
@@ -194,7 +200,7 @@ def ecasq_dp_pass(x, s, lambdas, flags=0, ws=None):
     lams = np.ascontiguousarray(lambdas, dtype=np.float64)
     G = lams.size
     if ws is None:
-        ws = workspace(d, s)
+        ws = workspace(d, s, flags=flags)
     Q = torch.zeros((G, s), dtype=torch.float32, device="cuda")
     m = (C.c_int32 * G)()
     met = np.zeros(4 * G, np.float64)
@@ -285,7 +291,7 @@ def ecasq_solve_batched(X, s, budget_bits=0.0, lambda_=-1.0, ws=None, **kw):
     X = _dev_f32(X)
     rows, d = X.shape
     if ws is None:
-        ws = workspace(d, s, rows)
+        ws = workspace(d, s, rows, flags=kw.get("flags", 0))
     prm = make_params(s, budget_bits, lambda_, **kw)
     Q = torch.zeros((rows, s), dtype=torch.float32, device="cuda")
     m = torch.zeros(rows, dtype=torch.int32, device="cuda")

@@ -41,6 +41,12 @@ def test_host_only_calls():
     assert native.ecasq_workspace_size(0, 8) == 0
     assert native.ecasq_workspace_size(100, 1) == 0
     assert native.ecasq_workspace_size(100, 257) == 0
+    # resident interval costs: 34816 bytes per 64 x 64 tile on top of the base size
+    base = native.ecasq_workspace_size(4096, 8)
+    assert native.ecasq_workspace_size_flags(4096, 8, 1, 0) == base
+    assert native.ecasq_workspace_size_flags(4096, 8, 1, native.RESIDENT_COSTS) == base + 64 * 65 // 2 * 34816
+    assert native.ecasq_workspace_size_flags(2 ** 31 - 1, 8, 1, native.RESIDENT_COSTS) == 0  # beyond size_t
+    assert native.ecasq_workspace_size_flags(0, 8, 1, native.RESIDENT_COSTS) == 0
     # workspace grows with d and s
     assert native.ecasq_workspace_size(4096, 16) > native.ecasq_workspace_size(4096, 8)
     assert native.ecasq_workspace_size(8192, 8) > native.ecasq_workspace_size(4096, 8)
