@@ -39,7 +39,7 @@ struct DevStatus {
     int32_t bound_viol;   // fast DP: fp32 minima outside their certified error bound
     double norm2;         // ||X||^2 (hi part of the double-double sum)
     int64_t rescored;     // fast DP: candidates re-scored in fp64
-    int64_t overflow;     // fast DP: outputs that needed the full-rescan path
+    int64_t overflow;     // fast DP: needed outputs whose band spans more than 32 tiles
     int32_t last_s;       // s and G of the last DP pass (for ecasq_dp_tables)
     int32_t last_G;
     int64_t last_d;       // d of the last DP pass

@@ -2,32 +2,34 @@
 //
 // Three stages per DP pass, for up to 8 multipliers at once:
 //
-// 1. k_wavefront: an fp32 filter over the whole (k, j) triangle with every
-//    layer i = 3..s fused.  A persistent CTA owns a block of 64 columns j and
-//    sweeps 64-wide tiles of k in increasing order; the tile k-block K may be
-//    used as soon as column block K has published all its layers (a flag with
-//    release/acquire order, bounded waits).  Two producer warps turn each tile
-//    into interval costs C[k,j] and Phi[k,j] (App. E quantities rebuilt with
+// 1. k_wavefront / k_wavefront_res: an fp32 filter over the whole (k, j)
+//    triangle with every layer i = 3..s fused.  A persistent CTA owns a block of
+//    64 columns j and sweeps 64-wide tiles of k in increasing order; the tile
+//    k-block K may be used as soon as column block K has published all its
+//    layers (a flag with release/acquire order, bounded waits).  The interval
+//    costs C[k,j] and Phi[k,j] of a tile (App. E quantities rebuilt with
 //    compensated fp32 recurrences that add one point at a time, all terms
-//    non-negative, from a double-double anchor per tile and column); the
-//    consumer warps evaluate dp(i-1,k) + C + lambda' Phi for their (layer,
-//    column, multiplier) outputs with packed f32x2 adds and 3-input mins.
-//    Per output the kernel keeps the fp32 minimum and up to two runs of
-//    consecutive tiles whose minimum came within the certified error band of it.
+//    non-negative, from a double-double anchor per tile and column) are either
+//    computed by two producer warps next to the consumers (k_wavefront), or
+//    computed once per call into a resident table (k_build_costs) and streamed
+//    in with bulk copies (k_wavefront_res, ECASQ_RESIDENT_COSTS); the values are
+//    bit-identical.  The consumer threads evaluate dp(i-1,k) + C + lambda' Phi
+//    for their (layer, column, multiplier) outputs with packed f32x2 adds and
+//    integer mins.  Per output the kernel keeps the fp32 minimum and up to two
+//    runs of tiles whose minimum came within the certified error band of it.
 // 2. k_need_layer (layers s down to 3): the outputs whose exact value the
 //    answer depends on.  eq. apx_final needs dp(i, p-1) for every i; an output
 //    resolved exactly needs the exact values of its band members in the layer
 //    below.  For every needed output the kernel re-evaluates its listed tiles
-//    bit-identically, keeps the members k whose fp32 value lies within the
+//    (within the certified bound; bit-identically from the resident table), keeps the members k whose fp32 value lies within the
 //    band (up to 8 inline, the count either way) and marks (i-1, k) needed.
 //    With ECASQ_EXACT_TABLES every output is needed.
 // 3. k_exact_layer (layers 3 up to s): re-score the members of every needed
 //    output in binary64 with double-double interval costs (the reference
 //    formulas) and take the lowest k among exact minima: dp64, bp.  Outputs
-//    with more members, or whose tile runs overflowed, re-scan their tiles in
-//    fp32 and re-score the members they meet on the fly -- never a full
-//    binary64 scan.  Outputs not needed keep their fp32 minimum (dp64 = m32,
-//    bp = -2).
+//    with more members re-scan their band's tiles in fp32 and re-score the
+//    members they meet on the fly -- never a full binary64 scan.  Outputs not
+//    needed keep their fp32 minimum (dp64 = m32, bp = -2).
 //
 // The fp32 band: with u = 2^-24, each fp32 candidate value carries a relative
 // error of at most eps_i = max(eps_{i-1}, 24u) + 1.0001u (eps_2 = 1.0001u), so
@@ -70,25 +72,23 @@ constexpr int kCostHalfFloats = BJ * PSTR;
 constexpr uint32_t kCostHalfBytes = (uint32_t)(kCostHalfFloats * sizeof(float));  // 17408, a multiple of 16
 constexpr size_t kCostTileFloats = 2 * (size_t)kCostHalfFloats;
 
-// Band word (64 bits): bits 0-1 number of tile runs (0..2), bit 2 overflow; run r
-// (r = 0, 1) at bit 3 + 19 r: first tile (14 bits) and length - 1 (5 bits, <= 32 tiles).
-// Tiles arrive in increasing order of K (the diagonal block, K = J, last).
-__device__ __forceinline__ uint64_t band_reset(uint32_t K) { return 1ull | ((uint64_t)K << 3); }
-__device__ __forceinline__ uint64_t band_append(uint64_t w, uint32_t K) {
-    uint32_t c = (uint32_t)(w & 3u);
-    if (w & 4u) return w;
-    if (c == 0) return band_reset(K);
-    int sh = 3 + 19 * (int)(c - 1);
-    uint32_t st = (uint32_t)(w >> sh) & 0x3FFFu, len = ((uint32_t)(w >> (sh + 14)) & 31u) + 1u;
-    if (K == st + len && len < 32u) return w + (1ull << (sh + 14));  // extend the last run
-    if (c == 1) return (w & ~3ull) | 2ull | ((uint64_t)K << 22);     // open the second run
-    return w | 4ull;
+// Band of an output: up to two runs of tile indices K (< 2^14), tiles arriving in
+// increasing K (the diagonal block, K = J, last).  Low word: run 1 as
+// first << 16 | last; high word: run 2 the same way, 0 when absent (a second run
+// starts at a tile >= 2).  A tile within the band extends run 1 when it follows
+// run 1 directly and there is no run 2, else opens run 2, else extends run 2 to
+// itself (the gap is then scanned too: a superset, never a miss).  A tile below
+// the band restarts it: run 1 = [K, K], no run 2.
+__device__ __forceinline__ void band_update(uint32_t &w1, uint32_t &w2, bool rst, bool app, uint32_t K,
+                                            uint32_t KK) {
+    const bool has2 = w2 != 0u;
+    const bool ext1 = app && !has2 && ((w1 & 0xFFFFu) + 1u == K);
+    const uint32_t n1 = ext1 ? ((w1 & 0xFFFF0000u) | K) : w1;
+    const uint32_t n2 = (app && !ext1) ? (has2 ? ((w2 & 0xFFFF0000u) | K) : KK) : w2;
+    w1 = rst ? KK : n1;
+    w2 = rst ? 0u : n2;
 }
-__device__ __forceinline__ void band_run(uint64_t w, int r, uint32_t &st, uint32_t &len) {
-    int sh = 3 + 19 * r;
-    st = (uint32_t)(w >> sh) & 0x3FFFu;
-    len = ((uint32_t)(w >> (sh + 14)) & 31u) + 1u;
-}
+__device__ __forceinline__ uint64_t band_pack(uint32_t w1, uint32_t w2) { return ((uint64_t)w2 << 32) | w1; }
 
 // Per-pass constants, copied once to device memory (kernels index them at run time).
 struct FastParams {
@@ -108,9 +108,9 @@ struct FastArgs {
     float invd;            // correctly rounded 1/d
     int G, s, lgc, Gc, nsplit, nJ, ncons;
     const FastParams *prm;
-    float *dp32;           // [G][s+1][p]
+    float *dp32;           // tile-major fp32 copy of dp: see d32()
     uint64_t *band;        // [G][s+1][ps] tile runs per output
-    int32_t *mcnt;         // [G][s+1][ps] band members (-1: runs overflowed)
+    int32_t *mcnt;         // [G][s+1][ps] band members
     int32_t *members;      // [G][s+1][ps][NMEM]
     uint8_t *need;         // [G][s+1][ps] output resolved exactly
     float *corner;         // [nJ(nJ-1)/2][8]: state of pair (64K+63, 64J), K < J (N, E, Ec, A, Ac, C, Cc)
@@ -120,6 +120,12 @@ struct FastArgs {
     int *abort_flag;
     DevStatus *st;
 };
+
+// The fp32 copy of dp is stored tile-major, [column block][g][i][64], so that the
+// rows (g, i = 2..s-1) one tile of k needs are one contiguous run per multiplier.
+__device__ __forceinline__ size_t d32(const FastArgs &a, int g, int i, int64_t j) {
+    return (((size_t)(j >> 6) * (size_t)a.G + (size_t)g) * (size_t)(a.s + 1) + (size_t)i) * BJ + (size_t)(j & 63);
+}
 
 __device__ __forceinline__ size_t oidx(const FastArgs &a, int g, int i, int64_t j) {
     return ((size_t)g * (size_t)(a.s + 1) + (size_t)i) * (size_t)a.ps + (size_t)j;
@@ -368,6 +374,15 @@ __device__ __forceinline__ void bulk_s2g(void *dst, const void *src, uint32_t by
     asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst), "r"(smem_u32(src)), "r"(bytes)
                  : "memory");
 }
+// global -> shared without a cache hint (rows every later block reads again)
+__device__ __forceinline__ void bulk_g2s_nohint(void *dst, const void *src, uint32_t bytes, unsigned long long *bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     smem_u32(dst)),
+                 "l"(src), "r"(bytes), "r"(smem_u32(bar))
+                 : "memory");
+}
+// global writes seen through generic loads/acquire -> ordered before later bulk copies
+__device__ __forceinline__ void fence_proxy_async_global() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_read_all() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
@@ -395,6 +410,8 @@ struct __align__(16) Smem {
     int pad[3];
     unsigned long long mbar[2];           // resident costs: bulk-copy completion of buffer b
     unsigned long long pad2[2];
+    float tau[kMaxS + 1];                 // FastParams::tau and lam32, read on every tile
+    float lam32[kMaxG];
     // followed by dp32 slices [2][Gc * (s-2)][BK] (dynamic)
 };
 
@@ -512,10 +529,200 @@ __global__ void __launch_bounds__(NPROD) k_build_costs(FastArgs a, float *costs)
     if (jl == 0) bulk_wait_all();
 }
 
-// ------------------------------------------------------------------ kernel
-// kCosts: the interval-cost tiles come from the resident table (one bulk copy per
-// half tile); otherwise the producer warps compute them (tile_columns).
-template <bool kCosts>
+// ------------------------------------------------------------ consumer side
+// A consumer thread owns the outputs (g = split * Gc + gl, layers 3 + lg * LPT + l,
+// columns jq + 16 q of the block) and keeps their band state in registers.
+struct ConsId {
+    int ct, jq, lg, gl;
+    bool active;
+};
+__device__ __forceinline__ ConsId cons_id(const FastArgs &a, int ct) {
+    ConsId id;
+    id.ct = ct;
+    id.jq = ct % NJQ;
+    const int rest = ct / NJQ;
+    id.lg = rest % a.lgc;
+    id.gl = rest / a.lgc;
+    id.active = ct < a.Gc * a.lgc * NJQ;
+    return id;
+}
+
+struct ConsState {
+    float best[LPT][JPT];
+    uint32_t w1[LPT][JPT], w2[LPT][JPT];  // band runs (band_update)
+};
+__device__ __forceinline__ void cons_reset(ConsState &cs) {
+#pragma unroll
+    for (int l = 0; l < LPT; l++)
+#pragma unroll
+        for (int q = 0; q < JPT; q++) { cs.best[l][q] = CUDART_INF_F; cs.w1[l][q] = 0u; cs.w2[l][q] = 0u; }
+}
+
+// Off-diagonal tile K: the fp32 minimum over the tile's 64 k of every output the
+// thread owns (g must be a real multiplier), folded into its band state.
+// Candidate values are >= +0, so their bit patterns order like the floats: the
+// running minimum is kept as int bits and updated with integer min (ALU pipe)
+// next to the packed adds (FMA pipe).
+__device__ __forceinline__ void cons_offdiag(const FastArgs &a, const Smem &S, const float *sDPb, int b, uint32_t K,
+                                             int g, const ConsId &id, ConsState &cs) {
+    const int L = a.s - 2;
+    int cm[LPT][JPT];
+#pragma unroll
+    for (int l = 0; l < LPT; l++)
+#pragma unroll
+        for (int q = 0; q < JPT; q++) cm[l][q] = 0x7f800000;  // +inf
+    const float *dpb = sDPb + (size_t)id.gl * L * BK;
+    const float lam = S.lam32[g];
+    const float2 lam2 = make_float2(lam, lam);
+    int rowl[LPT];
+#pragma unroll
+    for (int l = 0; l < LPT; l++) rowl[l] = min(id.lg * LPT + l, L - 1);
+#pragma unroll 1
+    for (int kk = 0; kk < BK; kk += 4) {
+        float2 W[JPT][2];
+#pragma unroll
+        for (int q = 0; q < JPT; q++) {
+            float4 c4 = *reinterpret_cast<const float4 *>(&S.C[b][id.jq + NJQ * q][kk]);
+            float4 f4 = *reinterpret_cast<const float4 *>(&S.Phi[b][id.jq + NJQ * q][kk]);
+            W[q][0] = fma2(lam2, make_float2(f4.x, f4.y), make_float2(c4.x, c4.y));
+            W[q][1] = fma2(lam2, make_float2(f4.z, f4.w), make_float2(c4.z, c4.w));
+        }
+#pragma unroll
+        for (int l = 0; l < LPT; l++) {
+            // layer i = 3 + li uses dp row 2 + li; rows past the last layer are
+            // clamped (their results are never used)
+            const float4 d4 = *reinterpret_cast<const float4 *>(dpb + (size_t)rowl[l] * BK + kk);
+            float2 da = make_float2(d4.x, d4.y), db = make_float2(d4.z, d4.w);
+#pragma unroll
+            for (int q = 0; q < JPT; q++) {
+                float2 t0 = add2(da, W[q][0]);
+                float2 t1 = add2(db, W[q][1]);
+                int c = min(min(cm[l][q], __float_as_int(t0.x)), __float_as_int(t0.y));
+                cm[l][q] = min(min(c, __float_as_int(t1.x)), __float_as_int(t1.y));
+            }
+        }
+    }
+    // band bookkeeping (branch-free; layers past the last one carry state that is never read)
+    const uint32_t KK = (K << 16) | K;
+#pragma unroll
+    for (int l = 0; l < LPT; l++) {
+        const float tau = S.tau[3 + rowl[l]];
+#pragma unroll
+        for (int q = 0; q < JPT; q++) {
+            float c = __int_as_float(cm[l][q]), bb = cs.best[l][q];
+            float T = __fmul_rn(bb, tau);
+            bool fin = c < CUDART_INF_F;
+            bool rst = fin && !(c >= __fsub_rn(bb, T));  // also the first finite tile (bb = +inf)
+            bool app = fin && !rst && (c <= __fadd_rn(bb, T));
+            band_update(cs.w1[l][q], cs.w2[l][q], rst, app, K, KK);
+            cs.best[l][q] = fminf(bb, c);
+        }
+    }
+}
+
+// Diagonal block J (its tile in buffer b): layers in order, each needing the
+// previous layer's values inside the block; then dp32 and the band words of the
+// block go to global memory.  All `a.ncons` consumer threads take part (BAR_CONS).
+__device__ __forceinline__ void cons_diag(const FastArgs &a, Smem &S, int b, int J, int split, const ConsId &id,
+                                          ConsState &cs) {
+    const int L = a.s - 2;
+    const int ct = id.ct;
+    const int g = split * a.Gc + id.gl;
+    const bool own = id.active && g < a.G;
+    const int64_t j0 = (int64_t)J * BJ;
+    // previous-layer values inside the column: layer 2 from the base kernel
+    for (int q = ct; q < a.Gc * BJ; q += a.ncons) {
+        int gg = q / BJ, jj = q % BJ;
+        int g2 = split * a.Gc + gg;
+        int64_t jx = j0 + jj;
+        S.diag[0][gg][jj] = (g2 < a.G && jx < a.p) ? a.dp32[d32(a, g2, 2, jx)] : CUDART_INF_F;
+    }
+    bar_sync(BAR_CONS, a.ncons);
+    int cur = 0;
+    const uint32_t K = (uint32_t)J, KK = (K << 16) | K;
+    for (int li = 0; li < L; li++) {
+        const int i = 3 + li;
+        // (a) every consumer thread: minima over the diagonal block for items (g, column),
+        //     4-wide loads over k with independent partial minima
+        for (int item = ct; item < a.Gc * BJ; item += a.ncons) {
+            int gg = item / BJ, jl = item % BJ;
+            int g2 = split * a.Gc + gg;
+            float lm = g2 < a.G ? S.lam32[g2] : 0.f;
+            float2 lm2 = make_float2(lm, lm);
+            int c0 = 0x7f800000, c1 = 0x7f800000, c2 = 0x7f800000, c3 = 0x7f800000;
+            const float *prow = &S.diag[cur][gg][0];
+#pragma unroll 4
+            for (int kk = 0; kk < BJ; kk += 4) {
+                float4 c4 = *reinterpret_cast<const float4 *>(&S.C[b][jl][kk]);
+                float4 f4 = *reinterpret_cast<const float4 *>(&S.Phi[b][jl][kk]);
+                float4 d4 = *reinterpret_cast<const float4 *>(prow + kk);
+                float2 v0 = fma2(lm2, make_float2(f4.x, f4.y), make_float2(c4.x, c4.y));
+                float2 v1 = fma2(lm2, make_float2(f4.z, f4.w), make_float2(c4.z, c4.w));
+                float2 t0 = add2(make_float2(d4.x, d4.y), v0);
+                float2 t1 = add2(make_float2(d4.z, d4.w), v1);
+                c0 = min(c0, __float_as_int(t0.x)); c1 = min(c1, __float_as_int(t0.y));
+                c2 = min(c2, __float_as_int(t1.x)); c3 = min(c3, __float_as_int(t1.y));
+            }
+            S.dmin[gg][jl] = __int_as_float(min(min(c0, c1), min(c2, c3)));
+        }
+        bar_sync(BAR_CONS, a.ncons);
+        // (b) the owners of layer i fold the diagonal block into their band state
+        const int l = li - id.lg * LPT;
+        if (own && l >= 0 && l < LPT) {
+#pragma unroll
+            for (int lx = 0; lx < LPT; lx++) {
+                if (lx != l) continue;
+#pragma unroll
+                for (int q = 0; q < JPT; q++) {
+                    int jl = id.jq + NJQ * q;
+                    int64_t j = j0 + jl;
+                    float c = S.dmin[id.gl][jl];
+                    float bb = cs.best[lx][q];
+                    float T = __fmul_rn(bb, S.tau[i]);
+                    bool fin = c < CUDART_INF_F;
+                    bool rst = fin && !(c >= __fsub_rn(bb, T));
+                    bool app = fin && !rst && (c <= __fadd_rn(bb, T));
+                    band_update(cs.w1[lx][q], cs.w2[lx][q], rst, app, K, KK);
+                    bb = fminf(bb, c);
+                    cs.best[lx][q] = bb;
+                    S.diag[cur ^ 1][id.gl][jl] = bb;
+                    if (j < a.p) {
+                        a.dp32[d32(a, g, i, j)] = bb;
+                        a.band[oidx(a, g, i, j)] = band_pack(cs.w1[lx][q], cs.w2[lx][q]);
+                    }
+                }
+            }
+        }
+        bar_sync(BAR_CONS, a.ncons);
+        cur ^= 1;
+    }
+}
+
+// Bounded wait (one thread) until column block K of `split` is published.
+__device__ __forceinline__ void wait_block(const FastArgs &a, int split, int K) {
+    const int *flag = a.done + (size_t)split * a.nJ + K;
+    uint32_t spins = 0;
+    while (ld_acquire(flag) == 0) {
+        if (*(volatile int *)a.abort_flag) break;
+        if (++spins > kSpinLimit) {
+            a.st->timeout = 1;
+            atomicExch(a.abort_flag, 1);
+            break;
+        }
+        __nanosleep(64);
+    }
+}
+
+// Publish column block J of `split` (after every thread's stores of the block).
+__device__ __forceinline__ void publish_block(const FastArgs &a, int split, int J) {
+    __threadfence();
+    st_release(a.done + (size_t)split * a.nJ + J, 1);
+}
+
+// ------------------------------------------------------------------ kernels
+// Fused producer: two producer warps compute each tile's interval costs
+// (tile_columns) and stage the dp32 rows with cp.async while the consumer warps
+// evaluate the previous tile (named barriers FULL / EMPTY per buffer).
 __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     Smem &S = *reinterpret_cast<Smem *>(smem_raw);
@@ -524,20 +731,14 @@ __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
     const int rowsDP = a.Gc * L;          // staged dp32 rows per tile (layers 2..s-1)
     const int tid = threadIdx.x;
     const int nall = NPROD + a.ncons;
-    if (kCosts) {
-        if (tid == 0) {
-            mbar_init(&S.mbar[0], 1);
-            mbar_init(&S.mbar[1], 1);
-            mbar_fence_init();
-        }
-        __syncthreads();
-    }
+    for (int q = tid; q <= kMaxS; q += blockDim.x) S.tau[q] = a.prm->tau[q];
+    if (tid < kMaxG) S.lam32[tid] = a.prm->lam32[tid];
+    __syncthreads();
 
     if (tid < NPROD) {
         // =========================== producer warps ===========================
         const int jl = tid;  // column within the block
         uint32_t n = 0;      // tile sequence number
-        const uint64_t policy = kCosts ? policy_evict_first() : 0ull;
         for (;;) {
             if (tid == 0) S.ticket = atomicAdd(a.ticket, 1);
             bar_sync(BAR_PROD, NPROD);
@@ -558,30 +759,9 @@ __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
                 bool diag = (K == J);
                 int64_t k0 = (int64_t)K * BK;
                 // wait for column block K (bounded); the diagonal needs nothing
-                if (!diag && tid == 0) {
-                    const int *flag = a.done + (size_t)split * a.nJ + K;
-                    uint32_t spins = 0;
-                    while (ld_acquire(flag) == 0) {
-                        if (*(volatile int *)a.abort_flag) break;
-                        if (++spins > kSpinLimit) {
-                            a.st->timeout = 1;
-                            atomicExch(a.abort_flag, 1);
-                            break;
-                        }
-                        __nanosleep(64);
-                    }
-                }
+                if (!diag && tid == 0) wait_block(a, split, K);
                 bar_sync(BAR_PROD, NPROD);
-                if (kCosts) {
-                    if (tid == 0) {
-                        const float *src = a.costs + cost_tile_idx(K, J) * kCostTileFloats;
-                        mbar_expect_tx(&S.mbar[b], 2 * kCostHalfBytes);
-                        bulk_g2s(&S.C[b][0][0], src, kCostHalfBytes, &S.mbar[b], policy);
-                        bulk_g2s(&S.Phi[b][0][0], src + kCostHalfFloats, kCostHalfBytes, &S.mbar[b], policy);
-                    }
-                } else {
-                    tile_consts(a, k0, jl, S.kv, S.kw, S.kd);
-                }
+                tile_consts(a, k0, jl, S.kv, S.kw, S.kd);
                 // dp32 slice of rows (g, layer 2..s-1) for k in the tile (cp.async, L2 only)
                 if (!diag) {
                     int gbase = split * a.Gc;
@@ -593,7 +773,7 @@ __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
                         int g = gbase + gl;
                         float *sp = dst + (size_t)row * BK + c4 * 4;
                         if (g < a.G) {
-                            const float *gp = a.dp32 + oidx(a, g, 2 + li, k0 + c4 * 4);
+                            const float *gp = a.dp32 + d32(a, g, 2 + li, k0 + c4 * 4);
                             unsigned sa = (unsigned)__cvta_generic_to_shared(sp);
                             asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(sa), "l"(gp) : "memory");
                         } else {
@@ -603,12 +783,8 @@ __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
                     }
                     asm volatile("cp.async.commit_group;" ::: "memory");
                 }
-                if (kCosts) {
-                    mbar_wait_bounded(&S.mbar[b], (n >> 1) & 1u, a.st, a.abort_flag);
-                } else {
-                    bar_sync(BAR_PROD, NPROD);
-                    tile_columns(a, K, J, jl, S.kv, S.kw, S.kd, S.wsum, S.C[b], S.Phi[b]);
-                }
+                bar_sync(BAR_PROD, NPROD);
+                tile_columns(a, K, J, jl, S.kv, S.kw, S.kd, S.wsum, S.C[b], S.Phi[b]);
                 if (!diag) asm volatile("cp.async.wait_all;" ::: "memory");
                 if (tid == 0) S.meta[b] = {J, K, split, diag ? 1 : 0};
                 bar_arrive(BAR_FULL + b, nall);
@@ -622,166 +798,114 @@ __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
     }
 
     // ============================= consumer warps =============================
-    const int ct = tid - NPROD;
-    const int jq = ct % NJQ;
-    const int rest = ct / NJQ;
-    const int lg = rest % a.lgc;
-    const int gl = rest / a.lgc;
-    const bool active = ct < a.Gc * a.lgc * NJQ;
+    const ConsId id = cons_id(a, tid - NPROD);
+    ConsState cs;
     uint32_t n = 0;
-    float best[LPT][JPT];
-    uint64_t word[LPT][JPT];
     for (;;) {
         int b = n & 1;
         bar_sync(BAR_FULL + b, nall);
         TileMeta m = S.meta[b];
         if (m.kind == 2) { bar_arrive(BAR_EMPTY + b, nall); break; }
-        if (kCosts) mbar_wait_bounded(&S.mbar[b], (n >> 1) & 1u, a.st, a.abort_flag);  // bulk copies landed
-        const int g = m.split * a.Gc + gl;
-        const bool own = active && g < a.G;
-        const int64_t j0 = (int64_t)m.J * BJ;
-        const float lam = own ? a.prm->lam32[g] : 0.f;
-        if (m.K == 0) {
-#pragma unroll
-            for (int l = 0; l < LPT; l++)
-#pragma unroll
-                for (int q = 0; q < JPT; q++) { best[l][q] = CUDART_INF_F; word[l][q] = 0ull; }
-        }
+        const int g = m.split * a.Gc + id.gl;
+        if (m.K == 0) cons_reset(cs);
         if (m.kind == 0) {
-            // Candidate values are >= +0, so their bit patterns order like the
-            // floats: the running minimum is kept as int bits and updated with
-            // integer min (ALU pipe) next to the packed adds (FMA pipe).
-            int cm[LPT][JPT];
-#pragma unroll
-            for (int l = 0; l < LPT; l++)
-#pragma unroll
-                for (int q = 0; q < JPT; q++) cm[l][q] = 0x7f800000;  // +inf
-            if (own) {
-                const float *dpb = sDP + (size_t)b * rowsDP * BK + (size_t)gl * L * BK;
-                float2 lam2 = make_float2(lam, lam);
-                int rowl[LPT];
-#pragma unroll
-                for (int l = 0; l < LPT; l++) rowl[l] = min(lg * LPT + l, L - 1);
-#pragma unroll 1
-                for (int kk = 0; kk < BK; kk += 4) {
-                    float2 W[JPT][2];
-#pragma unroll
-                    for (int q = 0; q < JPT; q++) {
-                        float4 c4 = *reinterpret_cast<const float4 *>(&S.C[b][jq + NJQ * q][kk]);
-                        float4 f4 = *reinterpret_cast<const float4 *>(&S.Phi[b][jq + NJQ * q][kk]);
-                        W[q][0] = fma2(lam2, make_float2(f4.x, f4.y), make_float2(c4.x, c4.y));
-                        W[q][1] = fma2(lam2, make_float2(f4.z, f4.w), make_float2(c4.z, c4.w));
-                    }
-#pragma unroll
-                    for (int l = 0; l < LPT; l++) {
-                        // layer i = 3 + li uses dp row 2 + li; rows past the last layer are
-                        // clamped (their results are never used)
-                        const float4 d4 = *reinterpret_cast<const float4 *>(dpb + (size_t)rowl[l] * BK + kk);
-                        float2 da = make_float2(d4.x, d4.y), db = make_float2(d4.z, d4.w);
-#pragma unroll
-                        for (int q = 0; q < JPT; q++) {
-                            float2 t0 = add2(da, W[q][0]);
-                            float2 t1 = add2(db, W[q][1]);
-                            int c = min(min(cm[l][q], __float_as_int(t0.x)), __float_as_int(t0.y));
-                            cm[l][q] = min(min(c, __float_as_int(t1.x)), __float_as_int(t1.y));
-                        }
-                    }
-                }
-                // band bookkeeping for this tile (branch-free)
-#pragma unroll
-                for (int l = 0; l < LPT; l++) {
-                    const int li = lg * LPT + l;
-                    const float tau = a.prm->tau[3 + min(li, L - 1)];
-                    const bool lok = li < L;
-#pragma unroll
-                    for (int q = 0; q < JPT; q++) {
-                        float c = __int_as_float(cm[l][q]), bb = best[l][q];
-                        float T = __fmul_rn(bb, tau);
-                        bool fin = lok && (c < CUDART_INF_F);
-                        bool rst = fin && (c < __fsub_rn(bb, T));
-                        bool app = fin && !rst && (c <= __fadd_rn(bb, T));
-                        uint64_t wv = word[l][q];
-                        uint64_t wa = band_append(wv, (uint32_t)m.K);
-                        word[l][q] = rst ? band_reset((uint32_t)m.K) : (app ? wa : wv);
-                        best[l][q] = fin ? fminf(bb, c) : bb;
-                    }
-                }
-            }
+            if (id.active && g < a.G) cons_offdiag(a, S, sDP + (size_t)b * rowsDP * BK, b, (uint32_t)m.K, g, id, cs);
             bar_arrive(BAR_EMPTY + b, nall);
         } else {
-            // ---------------- diagonal block: layers in order ----------------
-            // previous-layer values inside the column: layer 2 from the base kernel
-            for (int q = ct; q < a.Gc * BJ; q += a.ncons) {
-                int gg = q / BJ, jj = q % BJ;
-                int g2 = m.split * a.Gc + gg;
-                int64_t jx = j0 + jj;
-                S.diag[0][gg][jj] = (g2 < a.G && jx < a.p) ? a.dp32[oidx(a, g2, 2, jx)] : CUDART_INF_F;
-            }
-            bar_sync(BAR_CONS, a.ncons);
-            int cur = 0;
-            for (int li = 0; li < L; li++) {
-                const int i = 3 + li;
-                // (a) every consumer thread: minima over the diagonal block for items (g, column),
-                //     4-wide loads over k with independent partial minima
-                for (int item = ct; item < a.Gc * BJ; item += a.ncons) {
-                    int gg = item / BJ, jl = item % BJ;
-                    int g2 = m.split * a.Gc + gg;
-                    float lm = g2 < a.G ? a.prm->lam32[g2] : 0.f;
-                    float2 lm2 = make_float2(lm, lm);
-                    int c0 = 0x7f800000, c1 = 0x7f800000, c2 = 0x7f800000, c3 = 0x7f800000;
-                    const float *prow = &S.diag[cur][gg][0];
-#pragma unroll 4
-                    for (int kk = 0; kk < BJ; kk += 4) {
-                        float4 c4 = *reinterpret_cast<const float4 *>(&S.C[b][jl][kk]);
-                        float4 f4 = *reinterpret_cast<const float4 *>(&S.Phi[b][jl][kk]);
-                        float4 d4 = *reinterpret_cast<const float4 *>(prow + kk);
-                        float2 w0 = fma2(lm2, make_float2(f4.x, f4.y), make_float2(c4.x, c4.y));
-                        float2 w1 = fma2(lm2, make_float2(f4.z, f4.w), make_float2(c4.z, c4.w));
-                        float2 t0 = add2(make_float2(d4.x, d4.y), w0);
-                        float2 t1 = add2(make_float2(d4.z, d4.w), w1);
-                        c0 = min(c0, __float_as_int(t0.x)); c1 = min(c1, __float_as_int(t0.y));
-                        c2 = min(c2, __float_as_int(t1.x)); c3 = min(c3, __float_as_int(t1.y));
-                    }
-                    S.dmin[gg][jl] = __int_as_float(min(min(c0, c1), min(c2, c3)));
-                }
-                bar_sync(BAR_CONS, a.ncons);
-                // (b) the owners of layer i fold the diagonal block into their band state
-                const int l = li - lg * LPT;
-                if (own && l >= 0 && l < LPT) {
-#pragma unroll
-                    for (int lx = 0; lx < LPT; lx++) {
-                        if (lx != l) continue;
-#pragma unroll
-                        for (int q = 0; q < JPT; q++) {
-                            int jl = jq + NJQ * q;
-                            int64_t j = j0 + jl;
-                            float c = S.dmin[gl][jl];
-                            float bb = best[lx][q];
-                            if (c < CUDART_INF_F) {
-                                float T = __fmul_rn(bb, a.prm->tau[i]);
-                                if (c < __fsub_rn(bb, T)) { word[lx][q] = band_reset((uint32_t)m.J); bb = c; }
-                                else if (c <= __fadd_rn(bb, T)) { word[lx][q] = band_append(word[lx][q], (uint32_t)m.J); bb = fminf(bb, c); }
-                            }
-                            best[lx][q] = bb;
-                            S.diag[cur ^ 1][gl][jl] = bb;
-                            if (j < a.p) {
-                                a.dp32[oidx(a, g, i, j)] = bb;
-                                a.band[oidx(a, g, i, j)] = word[lx][q];
-                            }
-                        }
-                    }
-                }
-                bar_sync(BAR_CONS, a.ncons);
-                cur ^= 1;
-            }
-            // publish the column block (all layers, all multipliers of this split)
-            if (ct == 0) {
-                __threadfence();
-                st_release(a.done + (size_t)m.split * a.nJ + m.J, 1);
-            }
+            cons_diag(a, S, b, m.J, m.split, id, cs);
+            if (id.ct == 0) publish_block(a, m.split, m.J);
             bar_arrive(BAR_EMPTY + b, nall);
         }
         n++;
+    }
+}
+
+// Warp 0 of the resident-cost kernel: expect the bytes of tile (K, J) on mbar[b]
+// and issue its bulk copies into buffer b -- the interval costs from the resident
+// table and, off the diagonal, the dp32 rows (g, layers 2..s-1) of the split's
+// real multipliers (rows of other slots are never read).
+__device__ __forceinline__ void res_issue(const FastArgs &a, Smem &S, float *sDP, int b, int K, int J, int split,
+                                          uint64_t policy, int lane) {
+    const int L = a.s - 2, rowsDP = a.Gc * L;
+    const int gbase = split * a.Gc;
+    const int ngv = (K == J) ? 0 : std::min(a.G - gbase, a.Gc);  // real multipliers of the split
+    const uint32_t rows_bytes = (uint32_t)(L * BK * sizeof(float));   // rows 2..s-1 of one multiplier
+    if (lane == 0) {
+        const float *src = a.costs + cost_tile_idx(K, J) * kCostTileFloats;
+        mbar_expect_tx(&S.mbar[b], 2 * kCostHalfBytes + (uint32_t)ngv * rows_bytes);
+        bulk_g2s(&S.C[b][0][0], src, kCostHalfBytes, &S.mbar[b], policy);
+        bulk_g2s(&S.Phi[b][0][0], src + kCostHalfFloats, kCostHalfBytes, &S.mbar[b], policy);
+    }
+    __syncwarp();
+    if (lane < ngv) {
+        fence_proxy_async_global();  // rows other blocks wrote with generic stores
+        float *dst = sDP + (size_t)b * rowsDP * BK + (size_t)lane * L * BK;
+        bulk_g2s_nohint(dst, a.dp32 + d32(a, gbase + lane, 2, (int64_t)K * BK), rows_bytes, &S.mbar[b]);
+    }
+}
+
+// Resident interval costs: no producer warps.  Warp 0 claims the column blocks,
+// waits for the flags and issues the bulk copies of tile K+1 while tile K is
+// evaluated (two buffers, one mbarrier each); all MAXCONS threads are consumers.
+__global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    Smem &S = *reinterpret_cast<Smem *>(smem_raw);
+    float *sDP = reinterpret_cast<float *>(smem_raw + sizeof(Smem));
+    const int L = a.s - 2;
+    const int rowsDP = a.Gc * L;
+    const int ct = threadIdx.x;
+    const int lane = ct & 31;
+    for (int q = ct; q <= kMaxS; q += blockDim.x) S.tau[q] = a.prm->tau[q];
+    if (ct < kMaxG) S.lam32[ct] = a.prm->lam32[ct];
+    if (ct == 0) {
+        mbar_init(&S.mbar[0], 1);
+        mbar_init(&S.mbar[1], 1);
+        mbar_fence_init();
+    }
+    __syncthreads();
+    const ConsId id = cons_id(a, ct);
+    ConsState cs;
+    const uint64_t policy = policy_evict_first();
+    uint32_t n = 0;  // tile sequence number: buffer n & 1, its fill number n >> 1
+    for (;;) {
+        if (ct == 0) S.ticket = atomicAdd(a.ticket, 1);
+        __syncthreads();
+        const int t = S.ticket;
+        if (t >= a.nJ * a.nsplit) break;
+        const int J = t / a.nsplit, split = t % a.nsplit;
+        const int g = split * a.Gc + id.gl;
+        const bool own = id.active && g < a.G;
+        cons_reset(cs);
+        if (ct < 32) {
+            if (lane == 0 && J > 0) wait_block(a, split, 0);
+            __syncwarp();
+            res_issue(a, S, sDP, n & 1, 0, J, split, policy, lane);
+        }
+        for (int K = 0; K <= J; K++) {
+            const int b = n & 1;
+            bool pending = false;  // warp 0: tile K+1 still to be issued
+            if (ct < 32 && K < J) {
+                int ready = 1;
+                if (lane == 0 && K + 1 < J) ready = ld_acquire(a.done + (size_t)split * a.nJ + K + 1) != 0;
+                ready = __shfl_sync(0xffffffffu, ready, 0);
+                if (ready) res_issue(a, S, sDP, b ^ 1, K + 1, J, split, policy, lane);
+                pending = !ready;
+            }
+            mbar_wait_bounded(&S.mbar[b], (n >> 1) & 1u, a.st, a.abort_flag);
+            if (K < J) {
+                if (own) cons_offdiag(a, S, sDP + (size_t)b * rowsDP * BK, b, (uint32_t)K, g, id, cs);
+            } else {
+                cons_diag(a, S, b, J, split, id, cs);
+                if (ct == 0) publish_block(a, split, J);
+            }
+            __syncthreads();  // buffer b free for tile K+2
+            if (ct < 32 && pending) {
+                if (lane == 0) wait_block(a, split, K + 1);
+                __syncwarp();
+                res_issue(a, S, sDP, b ^ 1, K + 1, J, split, policy, lane);
+            }
+            n++;
+        }
     }
 }
 
@@ -804,7 +928,7 @@ __global__ void k_fast_base(Prefix P, FastArgs a, double *dp64, int32_t *bp) {
         double v = __dadd_rn(C, __dmul_rn(a.prm->lam64[g], phi));
         dp64[oidx(a, g, 2, j)] = v;
         bp[oidx(a, g, 2, j)] = 0;
-        a.dp32[oidx(a, g, 2, j)] = __fadd_rn(__double2float_rn(v), 0.0f);  // >= +0 (no -0)
+        a.dp32[d32(a, g, 2, j)] = __fadd_rn(__double2float_rn(v), 0.0f);  // >= +0 (no -0)
     }
 }
 
@@ -820,7 +944,7 @@ template <typename F>
 __device__ void visit_tile(const FastArgs &a, int g, int i, int64_t j, int64_t K, float thr, F &&f) {
     int64_t J = j / BJ, j0 = J * BJ, k0 = K * BK;
     float lam = a.prm->lam32[g];
-    const float *prev = a.dp32 + oidx(a, g, i - 1, 0);
+    const float *prev = a.dp32 + d32(a, g, i - 1, k0) - k0;  // prev[k] for k in tile K
     if (a.costs) {
         // the wavefront's own interval costs, read back from the resident table
         const float *cr = a.costs + cost_tile_idx(K, J) * kCostTileFloats + (size_t)(j - j0) * PSTR;
@@ -851,20 +975,19 @@ __device__ void visit_tile(const FastArgs &a, int g, int i, int64_t j, int64_t K
     }
 }
 
-// Tiles listed by a band word (in increasing order), or all tiles 0..J when it overflowed.
+// Tiles listed by a band word (band_update), in increasing order.
 template <typename F>
 __device__ void visit_band(const FastArgs &a, int g, int i, int64_t j, uint64_t w, float thr, F &&f) {
-    int64_t J = j / BJ;
-    if (w & 4u) {
-        for (int64_t K = 0; K <= J; K++) visit_tile(a, g, i, j, K, thr, f);
-        return;
-    }
-    int nr = (int)(w & 3u);
-    for (int r = 0; r < nr; r++) {
-        uint32_t st, len;
-        band_run(w, r, st, len);
-        for (uint32_t K = st; K < st + len; K++) visit_tile(a, g, i, j, (int64_t)K, thr, f);
-    }
+    const uint32_t w1 = (uint32_t)w, w2 = (uint32_t)(w >> 32);
+    for (uint32_t K = w1 >> 16; K <= (w1 & 0xFFFFu); K++) visit_tile(a, g, i, j, (int64_t)K, thr, f);
+    if (w2)
+        for (uint32_t K = w2 >> 16; K <= (w2 & 0xFFFFu); K++) visit_tile(a, g, i, j, (int64_t)K, thr, f);
+}
+
+// Tiles a band word spans (both runs).
+__device__ __forceinline__ uint32_t band_tiles(uint64_t w) {
+    const uint32_t w1 = (uint32_t)w, w2 = (uint32_t)(w >> 32);
+    return (w1 & 0xFFFFu) - (w1 >> 16) + 1u + (w2 ? (w2 & 0xFFFFu) - (w2 >> 16) + 1u : 0u);
 }
 
 __device__ __forceinline__ float band_threshold(const FastArgs &a, int i, float m32) {
@@ -897,7 +1020,7 @@ __global__ void k_need_layer(FastArgs a, int i) {
         if (j < i - 1) continue;
         size_t o = oidx(a, g, i, j);
         if (!a.need[o]) continue;
-        float m32 = a.dp32[o];
+        float m32 = a.dp32[d32(a, g, i, j)];
         if (!(m32 < CUDART_INF_F)) { a.mcnt[o] = 0; continue; }
         uint64_t w = a.band[o];
         int32_t *mem = a.members + o * NMEM;
@@ -909,10 +1032,10 @@ __global__ void k_need_layer(FastArgs a, int i) {
             cnt++;
             if (mark) below[k] = 1;
         });
-        a.mcnt[o] = (w & 4u) ? -1 : cnt;
+        a.mcnt[o] = cnt;
         nmem += cnt;
         nbig += cnt > NMEM;
-        nover += (w & 4u) ? 1 : 0;
+        nover += band_tiles(w) > 32u ? 1 : 0;  // wide bands (diagnostic)
     }
     if (nmem) atomicAdd((unsigned long long *)&a.st->members, nmem);
     if (nbig) atomicAdd((unsigned long long *)&a.st->big_bands, nbig);
@@ -936,7 +1059,7 @@ __global__ void k_exact_layer(Prefix P, FastArgs a, int i, double *dp64, int32_t
     int g = (int)(id / a.p);
     if (j < i - 1) return;
     size_t o = oidx(a, g, i, j);
-    float m32 = a.dp32[o];
+    float m32 = a.dp32[d32(a, g, i, j)];
     if (!(m32 < CUDART_INF_F)) return;
     if (!a.need[o]) { dp64[o] = (double)m32; bp[o] = -2; return; }
     int cnt = a.mcnt[o];
@@ -1089,12 +1212,12 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
         ECASQ_LAUNCH_CHECK();
     }
     size_t smem = smem_bytes(a.Gc, s);
-    auto wave = costs ? k_wavefront<true> : k_wavefront<false>;
+    auto wave = costs ? k_wavefront_res : k_wavefront;
     ECASQ_CUDA_TRY(cudaFuncSetAttribute(wave, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     int grid = std::min(nsm, a.nJ * a.nsplit);
     timer_begin(st);
     note_launch();
-    wave<<<grid, NPROD + a.ncons, smem, st>>>(a);
+    wave<<<grid, (costs ? 0 : NPROD) + a.ncons, smem, st>>>(a);
     timer_end(st);
     ECASQ_LAUNCH_CHECK();
     const int ilo = exact_s ? s : 2;
