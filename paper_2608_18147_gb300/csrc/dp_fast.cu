@@ -90,6 +90,22 @@ __device__ __forceinline__ void band_update(uint32_t &w1, uint32_t &w2, bool rst
 }
 __device__ __forceinline__ uint64_t band_pack(uint32_t w1, uint32_t w2) { return ((uint64_t)w2 << 32) | w1; }
 
+// Fold the minimum c of tile K (>= +0, or +inf) into an output's running minimum
+// bb and band: below bb - bb tau restarts the band, up to bb + bb tau joins it.
+// Non-negative floats order like their bit patterns, so the tests are unsigned
+// integer compares; bb = +inf makes bb - T a NaN, whose bits lie above every
+// value, so the first tile restarts the band (an all-+inf tile too, harmlessly:
+// outputs whose minimum stays +inf are never resolved).
+__device__ __forceinline__ void band_fold(float c, float &bb, float tau, uint32_t &w1, uint32_t &w2, uint32_t K,
+                                          uint32_t KK) {
+    const float T = __fmul_rn(bb, tau);
+    const uint32_t ci = __float_as_uint(c);
+    const bool rst = ci < __float_as_uint(__fsub_rn(bb, T));
+    const bool app = !rst && ci <= __float_as_uint(__fadd_rn(bb, T));
+    band_update(w1, w2, rst, app, K, KK);
+    bb = fminf(bb, c);
+}
+
 // Per-pass constants, copied once to device memory (kernels index them at run time).
 struct FastParams {
     float tau[kMaxS + 1];  // per layer: band factor 2 eps_i / (1 - eps_i), with margin
@@ -608,15 +624,7 @@ __device__ __forceinline__ void cons_offdiag(const FastArgs &a, const Smem &S, c
     for (int l = 0; l < LPT; l++) {
         const float tau = S.tau[3 + rowl[l]];
 #pragma unroll
-        for (int q = 0; q < JPT; q++) {
-            float c = __int_as_float(cm[l][q]), bb = cs.best[l][q];
-            float T = __fmul_rn(bb, tau);
-            bool fin = c < CUDART_INF_F;
-            bool rst = fin && !(c >= __fsub_rn(bb, T));  // also the first finite tile (bb = +inf)
-            bool app = fin && !rst && (c <= __fadd_rn(bb, T));
-            band_update(cs.w1[l][q], cs.w2[l][q], rst, app, K, KK);
-            cs.best[l][q] = fminf(bb, c);
-        }
+        for (int q = 0; q < JPT; q++) band_fold(__int_as_float(cm[l][q]), cs.best[l][q], tau, cs.w1[l][q], cs.w2[l][q], K, KK);
     }
 }
 
@@ -676,15 +684,8 @@ __device__ __forceinline__ void cons_diag(const FastArgs &a, Smem &S, int b, int
                 for (int q = 0; q < JPT; q++) {
                     int jl = id.jq + NJQ * q;
                     int64_t j = j0 + jl;
-                    float c = S.dmin[id.gl][jl];
-                    float bb = cs.best[lx][q];
-                    float T = __fmul_rn(bb, S.tau[i]);
-                    bool fin = c < CUDART_INF_F;
-                    bool rst = fin && !(c >= __fsub_rn(bb, T));
-                    bool app = fin && !rst && (c <= __fadd_rn(bb, T));
-                    band_update(cs.w1[lx][q], cs.w2[lx][q], rst, app, K, KK);
-                    bb = fminf(bb, c);
-                    cs.best[lx][q] = bb;
+                    band_fold(S.dmin[id.gl][jl], cs.best[lx][q], S.tau[i], cs.w1[lx][q], cs.w2[lx][q], K, KK);
+                    const float bb = cs.best[lx][q];
                     S.diag[cur ^ 1][id.gl][jl] = bb;
                     if (j < a.p) {
                         a.dp32[d32(a, g, i, j)] = bb;
