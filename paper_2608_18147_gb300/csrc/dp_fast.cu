@@ -418,7 +418,6 @@ struct __align__(16) Smem {
     float C[2][BJ][PSTR];
     float Phi[2][BJ][PSTR];
     float diag[2][kMaxG][BJ];             // dp32 of the previous / current layer inside the column
-    float dmin[kMaxG][BJ];                // diagonal-block minimum of the current layer
     float kv[BK], kw[BK], kd[BK];         // v_k (k0..k0+63), w_{k+1}, v_{k+1} - v_k
     TileMeta meta[2];
     float wsum[2][2];                     // producer scan: per-warp totals
@@ -629,62 +628,76 @@ __device__ __forceinline__ void cons_offdiag(const FastArgs &a, const Smem &S, c
 }
 
 // Diagonal block J (its tile in buffer b): layers in order, each needing the
-// previous layer's values inside the block; then dp32 and the band words of the
-// block go to global memory.  All `a.ncons` consumer threads take part (BAR_CONS).
+// previous layer's values inside the block; dp32 and the band words of the block
+// go to global memory.  The owner of an output computes its minimum over the
+// block's 64 k; when a.lgc == 2 the partner lane (lane ^ 16: same multiplier and
+// columns, the other layer group) takes half of the k range and the halves meet
+// by a shuffle.  All `a.ncons` consumer threads take part (BAR_CONS).
+// staged: S.diag[0] already holds layer 2 of the block (bulk copy), else it is
+// loaded here.
 __device__ __forceinline__ void cons_diag(const FastArgs &a, Smem &S, int b, int J, int split, const ConsId &id,
-                                          ConsState &cs) {
+                                          ConsState &cs, bool staged) {
     const int L = a.s - 2;
     const int ct = id.ct;
     const int g = split * a.Gc + id.gl;
     const bool own = id.active && g < a.G;
     const int64_t j0 = (int64_t)J * BJ;
-    // previous-layer values inside the column: layer 2 from the base kernel
-    for (int q = ct; q < a.Gc * BJ; q += a.ncons) {
-        int gg = q / BJ, jj = q % BJ;
-        int g2 = split * a.Gc + gg;
-        int64_t jx = j0 + jj;
-        S.diag[0][gg][jj] = (g2 < a.G && jx < a.p) ? a.dp32[d32(a, g2, 2, jx)] : CUDART_INF_F;
-    }
-    bar_sync(BAR_CONS, a.ncons);
-    int cur = 0;
-    const uint32_t K = (uint32_t)J, KK = (K << 16) | K;
-    for (int li = 0; li < L; li++) {
-        const int i = 3 + li;
-        // (a) every consumer thread: minima over the diagonal block for items (g, column),
-        //     4-wide loads over k with independent partial minima
-        for (int item = ct; item < a.Gc * BJ; item += a.ncons) {
-            int gg = item / BJ, jl = item % BJ;
+    if (!staged) {
+        for (int q = ct; q < a.Gc * BJ; q += a.ncons) {
+            int gg = q / BJ, jj = q % BJ;
             int g2 = split * a.Gc + gg;
-            float lm = g2 < a.G ? S.lam32[g2] : 0.f;
-            float2 lm2 = make_float2(lm, lm);
-            int c0 = 0x7f800000, c1 = 0x7f800000, c2 = 0x7f800000, c3 = 0x7f800000;
-            const float *prow = &S.diag[cur][gg][0];
-#pragma unroll 4
-            for (int kk = 0; kk < BJ; kk += 4) {
-                float4 c4 = *reinterpret_cast<const float4 *>(&S.C[b][jl][kk]);
-                float4 f4 = *reinterpret_cast<const float4 *>(&S.Phi[b][jl][kk]);
-                float4 d4 = *reinterpret_cast<const float4 *>(prow + kk);
-                float2 v0 = fma2(lm2, make_float2(f4.x, f4.y), make_float2(c4.x, c4.y));
-                float2 v1 = fma2(lm2, make_float2(f4.z, f4.w), make_float2(c4.z, c4.w));
-                float2 t0 = add2(make_float2(d4.x, d4.y), v0);
-                float2 t1 = add2(make_float2(d4.z, d4.w), v1);
-                c0 = min(c0, __float_as_int(t0.x)); c1 = min(c1, __float_as_int(t0.y));
-                c2 = min(c2, __float_as_int(t1.x)); c3 = min(c3, __float_as_int(t1.y));
-            }
-            S.dmin[gg][jl] = __int_as_float(min(min(c0, c1), min(c2, c3)));
+            int64_t jx = j0 + jj;
+            S.diag[0][gg][jj] = (g2 < a.G && jx < a.p) ? a.dp32[d32(a, g2, 2, jx)] : CUDART_INF_F;
         }
         bar_sync(BAR_CONS, a.ncons);
-        // (b) the owners of layer i fold the diagonal block into their band state
-        const int l = li - id.lg * LPT;
-        if (own && l >= 0 && l < LPT) {
+    }
+    const bool pair = a.lgc == 2;  // warp-uniform
+    const float lam = own ? S.lam32[g] : 0.f;
+    const float2 lam2 = make_float2(lam, lam);
+    const uint32_t K = (uint32_t)J, KK = (K << 16) | K;
+    int cur = 0;
+    for (int li = 0; li < L; li++) {
+        const int i = 3 + li;
+        const int olg = li / LPT, l = li - olg * LPT;
+        const bool owner = own && id.lg == olg;
+        const int kbeg = (pair && !owner) ? BJ / 2 : 0;
+        const int kend = (pair && owner) ? BJ / 2 : BJ;
+        int m0[JPT], m1[JPT];
+#pragma unroll
+        for (int q = 0; q < JPT; q++) { m0[q] = 0x7f800000; m1[q] = 0x7f800000; }
+        if (own && (owner || pair)) {
+            const float *prow = &S.diag[cur][id.gl][0];
+#pragma unroll 2
+            for (int kk = kbeg; kk < kend; kk += 4) {
+                const float4 d4 = *reinterpret_cast<const float4 *>(prow + kk);
+#pragma unroll
+                for (int q = 0; q < JPT; q++) {
+                    const int jl = id.jq + NJQ * q;
+                    float4 c4 = *reinterpret_cast<const float4 *>(&S.C[b][jl][kk]);
+                    float4 f4 = *reinterpret_cast<const float4 *>(&S.Phi[b][jl][kk]);
+                    float2 v0 = fma2(lam2, make_float2(f4.x, f4.y), make_float2(c4.x, c4.y));
+                    float2 v1 = fma2(lam2, make_float2(f4.z, f4.w), make_float2(c4.z, c4.w));
+                    float2 t0 = add2(make_float2(d4.x, d4.y), v0);
+                    float2 t1 = add2(make_float2(d4.z, d4.w), v1);
+                    m0[q] = min(min(m0[q], __float_as_int(t0.x)), __float_as_int(t0.y));
+                    m1[q] = min(min(m1[q], __float_as_int(t1.x)), __float_as_int(t1.y));
+                }
+            }
+        }
+#pragma unroll
+        for (int q = 0; q < JPT; q++) {
+            m0[q] = min(m0[q], m1[q]);
+            if (pair) m0[q] = min(m0[q], __shfl_xor_sync(0xffffffffu, m0[q], 16));
+        }
+        if (owner) {
 #pragma unroll
             for (int lx = 0; lx < LPT; lx++) {
                 if (lx != l) continue;
 #pragma unroll
                 for (int q = 0; q < JPT; q++) {
-                    int jl = id.jq + NJQ * q;
-                    int64_t j = j0 + jl;
-                    band_fold(S.dmin[id.gl][jl], cs.best[lx][q], S.tau[i], cs.w1[lx][q], cs.w2[lx][q], K, KK);
+                    const int jl = id.jq + NJQ * q;
+                    const int64_t j = j0 + jl;
+                    band_fold(__int_as_float(m0[q]), cs.best[lx][q], S.tau[i], cs.w1[lx][q], cs.w2[lx][q], K, KK);
                     const float bb = cs.best[lx][q];
                     S.diag[cur ^ 1][id.gl][jl] = bb;
                     if (j < a.p) {
@@ -696,6 +709,113 @@ __device__ __forceinline__ void cons_diag(const FastArgs &a, Smem &S, int b, int
         }
         bar_sync(BAR_CONS, a.ncons);
         cur ^= 1;
+    }
+}
+
+// Diagonal block when a.lgc == 2 (the usual s <= 16): lanes 0-15 of a warp take
+// k in [0, 32) of the block and lanes 16-31 k in [32, 64), for the same
+// multiplier and columns; the costs W = C + lambda' Phi of a lane's 4 x 32 pairs
+// stay in registers for all layers, so each layer reads only the previous
+// layer's 64 values from shared memory.  The band state is parked in `park`
+// ([3][LPT][JPT][ncons] words: best, run 1, run 2) and folded there; the block
+// ends with its diagonal, so the registers are not restored.
+__device__ __forceinline__ void cons_diag_pair(const FastArgs &a, Smem &S, uint32_t *park, int b, int J, int split,
+                                               const ConsId &id, ConsState &cs) {
+    const int L = a.s - 2;
+    const int ct = id.ct, nc = a.ncons;
+    const int g = split * a.Gc + id.gl;
+    const bool own = id.active && g < a.G;  // uniform over a warp (one multiplier per warp)
+    const int64_t j0 = (int64_t)J * BJ;
+    const int kh = (ct & 16) ? BJ / 2 : 0;
+    constexpr int NS = LPT * JPT;
+#pragma unroll
+    for (int l = 0; l < LPT; l++)
+#pragma unroll
+        for (int q = 0; q < JPT; q++) {
+            const int x = (l * JPT + q) * nc + ct;
+            park[x] = __float_as_uint(cs.best[l][q]);
+            park[NS * nc + x] = cs.w1[l][q];
+            park[2 * NS * nc + x] = cs.w2[l][q];
+        }
+    asm volatile("" ::: "memory");  // the state leaves the registers before W is built
+    float2 W[JPT][BJ / 4];  // W[q][p] = costs of k = kh + 2p, kh + 2p + 1 for column jq + 16 q
+    {
+        const float lam = own ? S.lam32[g] : 0.f;
+        const float2 lam2 = make_float2(lam, lam);
+#pragma unroll
+        for (int q = 0; q < JPT; q++) {
+            const int jl = id.jq + NJQ * q;
+#pragma unroll
+            for (int kk = 0; kk < BJ / 2; kk += 4) {
+                float4 c4 = *reinterpret_cast<const float4 *>(&S.C[b][jl][kh + kk]);
+                float4 f4 = *reinterpret_cast<const float4 *>(&S.Phi[b][jl][kh + kk]);
+                W[q][kk / 2] = fma2(lam2, make_float2(f4.x, f4.y), make_float2(c4.x, c4.y));
+                W[q][kk / 2 + 1] = fma2(lam2, make_float2(f4.z, f4.w), make_float2(c4.z, c4.w));
+            }
+            asm volatile("" ::: "memory");  // one column's loads in flight at a time (register pressure)
+        }
+    }
+    const uint32_t K = (uint32_t)J, KK = (K << 16) | K;
+    int cur = 0;
+    for (int li = 0; li < L; li++) {
+        const int i = 3 + li;
+        const int olg = li / LPT, l = li - olg * LPT;
+        const bool owner = own && id.lg == olg;
+        int m0[JPT], m1[JPT];
+#pragma unroll
+        for (int q = 0; q < JPT; q++) { m0[q] = 0x7f800000; m1[q] = 0x7f800000; }
+        if (own) {
+            const float *prow = &S.diag[cur][id.gl][kh];
+#pragma unroll
+            for (int kk = 0; kk < BJ / 2; kk += 4) {
+                const float4 d4 = *reinterpret_cast<const float4 *>(prow + kk);
+                const float2 da = make_float2(d4.x, d4.y), db = make_float2(d4.z, d4.w);
+#pragma unroll
+                for (int q = 0; q < JPT; q++) {
+                    float2 t0 = add2(da, W[q][kk / 2]);
+                    float2 t1 = add2(db, W[q][kk / 2 + 1]);
+                    m0[q] = min(min(m0[q], __float_as_int(t0.x)), __float_as_int(t0.y));
+                    m1[q] = min(min(m1[q], __float_as_int(t1.x)), __float_as_int(t1.y));
+                }
+            }
+        }
+#pragma unroll
+        for (int q = 0; q < JPT; q++) {
+            m0[q] = min(m0[q], m1[q]);
+            m0[q] = min(m0[q], __shfl_xor_sync(0xffffffffu, m0[q], 16));
+        }
+        if (owner) {
+#pragma unroll
+            for (int q = 0; q < JPT; q++) {
+                const int jl = id.jq + NJQ * q;
+                const int x = (l * JPT + q) * nc + ct;
+                float bb = __uint_as_float(park[x]);
+                uint32_t w1 = park[NS * nc + x], w2 = park[2 * NS * nc + x];
+                band_fold(__int_as_float(m0[q]), bb, S.tau[i], w1, w2, K, KK);
+                park[x] = __float_as_uint(bb);
+                park[NS * nc + x] = w1;
+                park[2 * NS * nc + x] = w2;
+                S.diag[cur ^ 1][id.gl][jl] = bb;
+            }
+        }
+        bar_sync(BAR_CONS, nc);
+        cur ^= 1;
+    }
+    // the block's final values and bands, from the parked state
+    if (own) {
+#pragma unroll
+        for (int l = 0; l < LPT; l++) {
+            const int i = 3 + id.lg * LPT + l;
+            if (i > a.s) break;
+#pragma unroll
+            for (int q = 0; q < JPT; q++) {
+                const int64_t j = j0 + id.jq + NJQ * q;
+                if (j >= a.p) continue;
+                const int x = (l * JPT + q) * nc + ct;
+                a.dp32[d32(a, g, i, j)] = __uint_as_float(park[x]);
+                a.band[oidx(a, g, i, j)] = band_pack(park[NS * nc + x], park[2 * NS * nc + x]);
+            }
+        }
     }
 }
 
@@ -813,7 +933,7 @@ __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
             if (id.active && g < a.G) cons_offdiag(a, S, sDP + (size_t)b * rowsDP * BK, b, (uint32_t)m.K, g, id, cs);
             bar_arrive(BAR_EMPTY + b, nall);
         } else {
-            cons_diag(a, S, b, m.J, m.split, id, cs);
+            cons_diag(a, S, b, m.J, m.split, id, cs, false);
             if (id.ct == 0) publish_block(a, m.split, m.J);
             bar_arrive(BAR_EMPTY + b, nall);
         }
@@ -829,8 +949,10 @@ __device__ __forceinline__ void res_issue(const FastArgs &a, Smem &S, float *sDP
                                           uint64_t policy, int lane) {
     const int L = a.s - 2, rowsDP = a.Gc * L;
     const int gbase = split * a.Gc;
-    const int ngv = (K == J) ? 0 : std::min(a.G - gbase, a.Gc);  // real multipliers of the split
-    const uint32_t rows_bytes = (uint32_t)(L * BK * sizeof(float));   // rows 2..s-1 of one multiplier
+    const bool diag = K == J;
+    const int ngv = std::min(a.G - gbase, a.Gc);  // real multipliers of the split
+    // off the diagonal: rows 2..s-1 of tile K; on it: row 2 of the block (S.diag[0])
+    const uint32_t rows_bytes = (uint32_t)((diag ? 1 : L) * BK * sizeof(float));
     if (lane == 0) {
         const float *src = a.costs + cost_tile_idx(K, J) * kCostTileFloats;
         mbar_expect_tx(&S.mbar[b], 2 * kCostHalfBytes + (uint32_t)ngv * rows_bytes);
@@ -840,7 +962,7 @@ __device__ __forceinline__ void res_issue(const FastArgs &a, Smem &S, float *sDP
     __syncwarp();
     if (lane < ngv) {
         fence_proxy_async_global();  // rows other blocks wrote with generic stores
-        float *dst = sDP + (size_t)b * rowsDP * BK + (size_t)lane * L * BK;
+        float *dst = diag ? &S.diag[0][lane][0] : sDP + (size_t)b * rowsDP * BK + (size_t)lane * L * BK;
         bulk_g2s_nohint(dst, a.dp32 + d32(a, gbase + lane, 2, (int64_t)K * BK), rows_bytes, &S.mbar[b]);
     }
 }
@@ -882,10 +1004,10 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
             __syncwarp();
             res_issue(a, S, sDP, n & 1, 0, J, split, policy, lane);
         }
-        for (int K = 0; K <= J; K++) {
+        for (int K = 0; K < J; K++) {  // off-diagonal tiles
             const int b = n & 1;
             bool pending = false;  // warp 0: tile K+1 still to be issued
-            if (ct < 32 && K < J) {
+            if (ct < 32) {
                 int ready = 1;
                 if (lane == 0 && K + 1 < J) ready = ld_acquire(a.done + (size_t)split * a.nJ + K + 1) != 0;
                 ready = __shfl_sync(0xffffffffu, ready, 0);
@@ -893,18 +1015,24 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
                 pending = !ready;
             }
             mbar_wait_bounded(&S.mbar[b], (n >> 1) & 1u, a.st, a.abort_flag);
-            if (K < J) {
-                if (own) cons_offdiag(a, S, sDP + (size_t)b * rowsDP * BK, b, (uint32_t)K, g, id, cs);
-            } else {
-                cons_diag(a, S, b, J, split, id, cs);
-                if (ct == 0) publish_block(a, split, J);
-            }
+            if (own) cons_offdiag(a, S, sDP + (size_t)b * rowsDP * BK, b, (uint32_t)K, g, id, cs);
             __syncthreads();  // buffer b free for tile K+2
             if (ct < 32 && pending) {
                 if (lane == 0) wait_block(a, split, K + 1);
                 __syncwarp();
                 res_issue(a, S, sDP, b ^ 1, K + 1, J, split, policy, lane);
             }
+            n++;
+        }
+        {  // the diagonal tile (issued with tile J-1, or at the block start when J = 0)
+            const int b = n & 1;
+            mbar_wait_bounded(&S.mbar[b], (n >> 1) & 1u, a.st, a.abort_flag);
+            if (a.lgc == 2)
+                cons_diag_pair(a, S, reinterpret_cast<uint32_t *>(sDP + (size_t)2 * rowsDP * BK), b, J, split, id, cs);
+            else
+                cons_diag(a, S, b, J, split, id, cs, true);
+            if (ct == 0) publish_block(a, split, J);
+            __syncthreads();
             n++;
         }
     }
@@ -1213,6 +1341,7 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
         ECASQ_LAUNCH_CHECK();
     }
     size_t smem = smem_bytes(a.Gc, s);
+    if (costs && a.lgc == 2) smem += (size_t)3 * LPT * JPT * a.ncons * sizeof(uint32_t);  // parked band state
     auto wave = costs ? k_wavefront_res : k_wavefront;
     ECASQ_CUDA_TRY(cudaFuncSetAttribute(wave, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     int grid = std::min(nsm, a.nJ * a.nsplit);
