@@ -131,6 +131,9 @@ struct FastArgs {
     uint8_t *need;         // [G][s+1][ps] output resolved exactly
     float *corner;         // [nJ(nJ-1)/2][8]: state of pair (64K+63, 64J), K < J (N, E, Ec, A, Ac, C, Cc)
     const float *costs;    // resident interval costs (tile (K, J) at J(J+1)/2 + K), or null: computed per tile
+    float *mdp;            // [nJ][G][mdp_stride]: min over the block's 64 columns of dp32(g, i, .)
+    int mdp_stride;        // s + 1 rounded up to a multiple of 4 (16-byte rows)
+    int prune;             // skip tiles by the lower bound (resident costs, two layer groups)
     int *done;             // [nsplit][nJ]
     int *ticket;
     int *abort_flag;
@@ -427,6 +430,7 @@ struct __align__(16) Smem {
     unsigned long long pad2[2];
     float tau[kMaxS + 1];                 // FastParams::tau and lam32, read on every tile
     float lam32[kMaxG];
+    __align__(16) float mdp[2][kMaxG][20];  // staged dp32 block minima (tile skipping, s <= 19)
     // followed by dp32 slices [2][Gc * (s-2)][BK] (dynamic)
 };
 
@@ -475,7 +479,9 @@ __device__ void tile_columns(const FastArgs &a, int64_t K, int64_t J, int jl, co
             anchor_r.C = cp[5]; anchor_r.Cc = cp[6];
             pair_add(anchor_r.C, anchor_r.Cc, cx, cc);
         }
-        // interval costs of column j for k in the tile (descending k)
+        // interval costs of column j for k in the tile (descending k); the row's
+        // padding slot BK receives min_k C and min_k Phi (lower bounds for tile skipping)
+        float mc = CUDART_INF_F, mp = CUDART_INF_F;
         if (j < a.p) {
             float vj = a.v[j];
             Rec r;
@@ -485,11 +491,13 @@ __device__ void tile_columns(const FastArgs &a, int64_t K, int64_t J, int jl, co
                 kl_hi = (int)(j - j0) - 1;  // k = j-1 first
                 // state for k = j: empty; step to k = j-1 adds t = j
                 for (int kl = BK - 1; kl > kl_hi; kl--) { Cr[jl][kl] = CUDART_INF_F; Pr[jl][kl] = 0.f; }
+                if (kl_hi < BK - 1) mp = 0.f;
                 for (int kl = kl_hi; kl >= 0; kl--) {
                     rec_step(r, vj, kv[kl + 1], kw[kl], kd[kl]);  // kl + 1 <= 63
                     float c, ph;
                     rec_emit(r, vj, kv[kl], d_f, a.invd, c, ph);
                     Cr[jl][kl] = c; Pr[jl][kl] = ph;
+                    mc = fminf(mc, c); mp = fminf(mp, ph);
                 }
             } else {
                 r = anchor_r;
@@ -500,11 +508,15 @@ __device__ void tile_columns(const FastArgs &a, int64_t K, int64_t J, int jl, co
                     float c, ph;
                     rec_emit(cur, vj, kv[kl], d_f, a.invd, c, ph);
                     Cr[jl][kl] = c; Pr[jl][kl] = ph;
+                    mc = fminf(mc, c); mp = fminf(mp, ph);
                 }
             }
         } else {
             for (int kl = 0; kl < BK; kl++) { Cr[jl][kl] = CUDART_INF_F; Pr[jl][kl] = 0.f; }
+            mp = 0.f;
         }
+        Cr[jl][BK] = mc;
+        Pr[jl][BK] = mp;
 }
 
 // Resident interval costs: every tile (K <= J) computed once, exactly as the
@@ -592,6 +604,30 @@ __device__ __forceinline__ void cons_offdiag(const FastArgs &a, const Smem &S, c
     int rowl[LPT];
 #pragma unroll
     for (int l = 0; l < LPT; l++) rowl[l] = min(id.lg * LPT + l, L - 1);
+    if (a.prune) {
+        // Exact tile skipping.  Every candidate of the tile for output (l, q) is
+        // >= lb = fl(min dp(i-1, .) + fl(fma(lam, min Phi, min C))) (rounding is monotone);
+        // when lb exceeds the output's band limit bb + bb tau, the tile changes neither
+        // its minimum nor its band.  The warp skips when that holds for all its outputs.
+        const float *md = &S.mdp[b][0][0] + (size_t)id.gl * a.mdp_stride + 2;
+        float lbq[JPT];
+#pragma unroll
+        for (int q = 0; q < JPT; q++) {
+            const int jl = id.jq + NJQ * q;
+            lbq[q] = __fmaf_rn(lam, S.Phi[b][jl][BK], S.C[b][jl][BK]);
+        }
+        bool need = false;
+#pragma unroll
+        for (int l = 0; l < LPT; l++) {
+            const float m = md[rowl[l]], tau = S.tau[3 + rowl[l]];
+#pragma unroll
+            for (int q = 0; q < JPT; q++) {
+                const float bb = cs.best[l][q];
+                need |= __fadd_rn(m, lbq[q]) <= __fadd_rn(bb, __fmul_rn(bb, tau));
+            }
+        }
+        if (!__any_sync(__activemask(), need)) return;
+    }
 #pragma unroll 1
     for (int kk = 0; kk < BK; kk += 4) {
         float2 W[JPT][2];
@@ -738,6 +774,13 @@ __device__ __forceinline__ void cons_diag_pair(const FastArgs &a, Smem &S, uint3
             park[2 * NS * nc + x] = cs.w2[l][q];
         }
     asm volatile("" ::: "memory");  // the state leaves the registers before W is built
+    const int lane = ct & 31;
+    if (a.prune && own) {  // block minimum of layer 2 (values are >= +0: integer min on the bits)
+        int v = min(__float_as_int(S.diag[0][id.gl][lane]), __float_as_int(S.diag[0][id.gl][lane + 32]));
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) v = min(v, __shfl_xor_sync(0xffffffffu, v, o));
+        if (lane == 0) a.mdp[((size_t)J * a.G + g) * a.mdp_stride + 2] = __int_as_float(v);
+    }
     float2 W[JPT][BJ / 4];  // W[q][p] = costs of k = kh + 2p, kh + 2p + 1 for column jq + 16 q
     {
         const float lam = own ? S.lam32[g] : 0.f;
@@ -801,19 +844,28 @@ __device__ __forceinline__ void cons_diag_pair(const FastArgs &a, Smem &S, uint3
         bar_sync(BAR_CONS, nc);
         cur ^= 1;
     }
-    // the block's final values and bands, from the parked state
+    // the block's final values and bands, from the parked state, and the block
+    // minimum of every layer (over the 64 columns a half-warp holds)
     if (own) {
 #pragma unroll
         for (int l = 0; l < LPT; l++) {
             const int i = 3 + id.lg * LPT + l;
-            if (i > a.s) break;
+            const bool real = i <= a.s;
+            int v = 0x7f800000;
 #pragma unroll
             for (int q = 0; q < JPT; q++) {
                 const int64_t j = j0 + id.jq + NJQ * q;
-                if (j >= a.p) continue;
                 const int x = (l * JPT + q) * nc + ct;
-                a.dp32[d32(a, g, i, j)] = __uint_as_float(park[x]);
-                a.band[oidx(a, g, i, j)] = band_pack(park[NS * nc + x], park[2 * NS * nc + x]);
+                v = min(v, (int)park[x]);
+                if (real && j < a.p) {
+                    a.dp32[d32(a, g, i, j)] = __uint_as_float(park[x]);
+                    a.band[oidx(a, g, i, j)] = band_pack(park[NS * nc + x], park[2 * NS * nc + x]);
+                }
+            }
+            if (a.prune) {
+#pragma unroll
+                for (int o = 8; o > 0; o >>= 1) v = min(v, __shfl_xor_sync(0xffffffffu, v, o));
+                if (real && id.jq == 0) a.mdp[((size_t)J * a.G + g) * a.mdp_stride + i] = __int_as_float(v);
             }
         }
     }
@@ -955,9 +1007,14 @@ __device__ __forceinline__ void res_issue(const FastArgs &a, Smem &S, float *sDP
     const uint32_t rows_bytes = (uint32_t)((diag ? 1 : L) * BK * sizeof(float));
     if (lane == 0) {
         const float *src = a.costs + cost_tile_idx(K, J) * kCostTileFloats;
-        mbar_expect_tx(&S.mbar[b], 2 * kCostHalfBytes + (uint32_t)ngv * rows_bytes);
+        const uint32_t mdp_bytes = (a.prune && !diag) ? (uint32_t)(ngv * a.mdp_stride * sizeof(float)) : 0u;
+        mbar_expect_tx(&S.mbar[b], 2 * kCostHalfBytes + (uint32_t)ngv * rows_bytes + mdp_bytes);
         bulk_g2s(&S.C[b][0][0], src, kCostHalfBytes, &S.mbar[b], policy);
         bulk_g2s(&S.Phi[b][0][0], src + kCostHalfFloats, kCostHalfBytes, &S.mbar[b], policy);
+        if (mdp_bytes) {
+            fence_proxy_async_global();
+            bulk_g2s_nohint(&S.mdp[b][0][0], a.mdp + ((size_t)K * a.G + gbase) * a.mdp_stride, mdp_bytes, &S.mbar[b]);
+        }
     }
     __syncwarp();
     if (lane < ngv) {
@@ -1227,11 +1284,14 @@ __global__ void k_store_params(FastParams prm, FastParams *dst) {
     if (threadIdx.x == 0 && blockIdx.x == 0) *dst = prm;
 }
 
+static int mdp_stride(int s) { return (s + 1 + 3) & ~3; }
+
 size_t fast_dp_band_bytes(int64_t d, int32_t s) {
     size_t rows = (size_t)kMaxG * (size_t)(s + 1) * (size_t)table_stride(d);
     size_t nJ = (size_t)cdiv(d, BJ);
     return align256(8 * rows) + align256(4 * rows) + align256(4 * NMEM * rows) + align256(rows) +
-           align256(4 * (size_t)kMaxG * nJ + 64) + align256(sizeof(FastParams)) + align256(32 * nJ * (nJ + 1) / 2);
+           align256(4 * (size_t)kMaxG * nJ + 64) + align256(sizeof(FastParams)) + align256(32 * nJ * (nJ + 1) / 2) +
+           align256(4 * (size_t)kMaxG * (size_t)mdp_stride(s) * nJ);
 }
 
 static size_t smem_bytes(int Gc, int s) { return sizeof(Smem) + (size_t)2 * Gc * (s - 2) * BK * sizeof(float); }
@@ -1303,6 +1363,12 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     FastParams *dprm = reinterpret_cast<FastParams *>(base);
     base += align256(sizeof(FastParams));
     a.corner = reinterpret_cast<float *>(base);
+    {
+        size_t nJd = (size_t)cdiv(Lw.d, BJ);
+        a.mdp = reinterpret_cast<float *>(base + align256(32 * nJd * (nJd + 1) / 2));
+    }
+    a.mdp_stride = mdp_stride(s);
+    a.prune = (costs && a.lgc == 2 && a.mdp_stride <= 20) ? 1 : 0;
     a.costs = costs;
     a.prm = dprm;
     a.done = flags;
