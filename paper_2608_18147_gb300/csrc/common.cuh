@@ -45,6 +45,8 @@ struct DevStatus {
     int64_t last_d;       // d of the last DP pass
     int64_t members;      // fast DP: band members found (all outputs)
     int64_t big_bands;    // fast DP: outputs with more members than the inline list holds
+    int64_t tiles_run;    // fast DP, resident costs: (warp, tile) units evaluated
+    int64_t tiles_skipped; // ... and skipped by the lower bound
 };
 
 struct Layout {

@@ -24,7 +24,8 @@
 //    (within the certified bound; bit-identically from the resident table), keeps the members k whose fp32 value lies within the
 //    band (up to 8 inline, the count either way) and marks (i-1, k) needed.
 //    With ECASQ_EXACT_TABLES every output is needed.
-// 3. k_exact_layer (layers 3 up to s): re-score the members of every needed
+// 3. k_exact_small / k_exact_big (layers 3 up to s, over the lists the need
+//    stage wrote; k_fill_unneeded first): re-score the members of every needed
 //    output in binary64 with double-double interval costs (the reference
 //    formulas) and take the lowest k among exact minima: dp64, bp.  Outputs
 //    with more members re-scan their band's tiles in fp32 and re-score the
@@ -131,6 +132,8 @@ struct FastArgs {
     uint8_t *need;         // [G][s+1][ps] output resolved exactly
     float *corner;         // [nJ(nJ-1)/2][8]: state of pair (64K+63, 64J), K < J (N, E, Ec, A, Ac, C, Cc)
     const float *costs;    // resident interval costs (tile (K, J) at J(J+1)/2 + K), or null: computed per tile
+    int32_t *lists;        // [s+1][2][G ps]: needed outputs of layer i (g << 24 | j); 0: <= NMEM members, 1: more
+    int *list_cnt;         // [s+1][2]
     float *mdp;            // [nJ][G][mdp_stride]: min over the block's 64 columns of dp32(g, i, .)
     int mdp_stride;        // s + 1 rounded up to a multiple of 4 (16-byte rows)
     int prune;             // skip tiles by the lower bound (resident costs, two layer groups)
@@ -590,7 +593,8 @@ __device__ __forceinline__ void cons_reset(ConsState &cs) {
 // Candidate values are >= +0, so their bit patterns order like the floats: the
 // running minimum is kept as int bits and updated with integer min (ALU pipe)
 // next to the packed adds (FMA pipe).
-__device__ __forceinline__ void cons_offdiag(const FastArgs &a, const Smem &S, const float *sDPb, int b, uint32_t K,
+// Returns false when the warp skipped the tile (see below).
+__device__ __forceinline__ bool cons_offdiag(const FastArgs &a, const Smem &S, const float *sDPb, int b, uint32_t K,
                                              int g, const ConsId &id, ConsState &cs) {
     const int L = a.s - 2;
     int cm[LPT][JPT];
@@ -626,7 +630,7 @@ __device__ __forceinline__ void cons_offdiag(const FastArgs &a, const Smem &S, c
                 need |= __fadd_rn(m, lbq[q]) <= __fadd_rn(bb, __fmul_rn(bb, tau));
             }
         }
-        if (!__any_sync(__activemask(), need)) return;
+        if (!__any_sync(__activemask(), need)) return false;
     }
 #pragma unroll 1
     for (int kk = 0; kk < BK; kk += 4) {
@@ -661,6 +665,7 @@ __device__ __forceinline__ void cons_offdiag(const FastArgs &a, const Smem &S, c
 #pragma unroll
         for (int q = 0; q < JPT; q++) band_fold(__int_as_float(cm[l][q]), cs.best[l][q], tau, cs.w1[l][q], cs.w2[l][q], K, KK);
     }
+    return true;
 }
 
 // Diagonal block J (its tile in buffer b): layers in order, each needing the
@@ -1047,6 +1052,7 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
     ConsState cs;
     const uint64_t policy = policy_evict_first();
     uint32_t n = 0;  // tile sequence number: buffer n & 1, its fill number n >> 1
+    unsigned long long n_run = 0, n_skip = 0;  // lane 0 of each warp: its (warp, tile) units
     for (;;) {
         if (ct == 0) S.ticket = atomicAdd(a.ticket, 1);
         __syncthreads();
@@ -1072,7 +1078,11 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
                 pending = !ready;
             }
             mbar_wait_bounded(&S.mbar[b], (n >> 1) & 1u, a.st, a.abort_flag);
-            if (own) cons_offdiag(a, S, sDP + (size_t)b * rowsDP * BK, b, (uint32_t)K, g, id, cs);
+            if (own) {
+                const bool ran = cons_offdiag(a, S, sDP + (size_t)b * rowsDP * BK, b, (uint32_t)K, g, id, cs);
+                n_run += ran ? 1 : 0;
+                n_skip += ran ? 0 : 1;
+            }
             __syncthreads();  // buffer b free for tile K+2
             if (ct < 32 && pending) {
                 if (lane == 0) wait_block(a, split, K + 1);
@@ -1092,6 +1102,10 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
             __syncthreads();
             n++;
         }
+    }
+    if (lane == 0 && (n_run | n_skip)) {
+        atomicAdd((unsigned long long *)&a.st->tiles_run, n_run);
+        atomicAdd((unsigned long long *)&a.st->tiles_skipped, n_skip);
     }
 }
 
@@ -1194,38 +1208,82 @@ __global__ void k_need_init(FastArgs a, int ilo, int all) {
     }
 }
 
-// Backward closure, layer i: members of every needed output; mark (i-1, k) needed.
+// Warp-aggregated append of `v` to list[*cnt] by the lanes of `mask` that want it.
+__device__ __forceinline__ void warp_append(unsigned mask, bool want, int32_t v, int32_t *list, int *cnt) {
+    const unsigned m = __ballot_sync(mask, want);
+    if (!m) return;
+    const int lane = threadIdx.x & 31;
+    const int leader = __ffs(m) - 1;
+    int base = 0;
+    if (lane == leader) base = atomicAdd(cnt, __popc(m));
+    base = __shfl_sync(mask, base, leader);
+    if (want) list[base + __popc(m & ((1u << lane) - 1u))] = v;
+}
+
+__device__ __forceinline__ int32_t *layer_list(const FastArgs &a, int i, int kind) {
+    return a.lists + ((size_t)i * 2 + kind) * (size_t)a.G * (size_t)a.ps;
+}
+
+// Backward closure, layer i: members of every needed output; mark (i-1, k) needed;
+// list the needed outputs for the exact stage (inline members / big bands).
 __global__ void k_need_layer(FastArgs a, int i) {
-    int64_t tot = (int64_t)a.G * a.p;
-    int64_t id = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    const int64_t tot = (int64_t)a.G * a.p;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     unsigned long long nmem = 0, nbig = 0, nover = 0;
-    for (; id < tot; id += stride) {
-        int64_t j = id % a.p;
-        int g = (int)(id / a.p);
-        if (j < i - 1) continue;
-        size_t o = oidx(a, g, i, j);
-        if (!a.need[o]) continue;
-        float m32 = a.dp32[d32(a, g, i, j)];
-        if (!(m32 < CUDART_INF_F)) { a.mcnt[o] = 0; continue; }
-        uint64_t w = a.band[o];
-        int32_t *mem = a.members + o * NMEM;
-        uint8_t *below = a.need + oidx(a, g, i - 1, 0);
-        const bool mark = i - 1 >= 3;
+    int32_t *lsmall = layer_list(a, i, 0), *lbig = layer_list(a, i, 1);
+    int *csmall = a.list_cnt + 2 * i, *cbig = csmall + 1;
+    for (int64_t base = (int64_t)blockIdx.x * blockDim.x; base < tot; base += stride) {  // warp-uniform trip count
+        const int64_t id = base + threadIdx.x;
+        bool listed = false;
         int cnt = 0;
-        visit_band(a, g, i, j, w, band_threshold(a, i, m32), [&](int64_t k) {
-            if (cnt < NMEM) mem[cnt] = (int32_t)k;
-            cnt++;
-            if (mark) below[k] = 1;
-        });
-        a.mcnt[o] = cnt;
-        nmem += cnt;
-        nbig += cnt > NMEM;
-        nover += band_tiles(w) > 32u ? 1 : 0;  // wide bands (diagnostic)
+        int32_t packed = 0;
+        if (id < tot) {
+            const int64_t j = id % a.p;
+            const int g = (int)(id / a.p);
+            const size_t o = oidx(a, g, i, j);
+            if (j >= i - 1 && a.need[o]) {
+                const float m32 = a.dp32[d32(a, g, i, j)];
+                if (!(m32 < CUDART_INF_F)) {
+                    a.mcnt[o] = 0;
+                } else {
+                    const uint64_t w = a.band[o];
+                    int32_t *mem = a.members + o * NMEM;
+                    uint8_t *below = a.need + oidx(a, g, i - 1, 0);
+                    const bool mark = i - 1 >= 3;
+                    visit_band(a, g, i, j, w, band_threshold(a, i, m32), [&](int64_t k) {
+                        if (cnt < NMEM) mem[cnt] = (int32_t)k;
+                        cnt++;
+                        if (mark) below[k] = 1;
+                    });
+                    a.mcnt[o] = cnt;
+                    nmem += cnt;
+                    nbig += cnt > NMEM;
+                    nover += band_tiles(w) > 32u ? 1 : 0;  // wide bands (diagnostic)
+                    listed = true;
+                    packed = (int32_t)((g << 24) | (int32_t)j);
+                }
+            }
+        }
+        warp_append(0xffffffffu, listed && cnt <= NMEM, packed, lsmall, csmall);
+        warp_append(0xffffffffu, listed && cnt > NMEM, packed, lbig, cbig);
     }
     if (nmem) atomicAdd((unsigned long long *)&a.st->members, nmem);
     if (nbig) atomicAdd((unsigned long long *)&a.st->big_bands, nbig);
     if (nover) atomicAdd((unsigned long long *)&a.st->overflow, nover);
+}
+
+// Outputs the answer does not read keep their fp32 minimum: dp64 = m32, bp = -2.
+__global__ void k_fill_unneeded(FastArgs a, double *dp64, int32_t *bp) {
+    const int64_t tot = (int64_t)a.G * (a.s + 1) * a.ps;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t o = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; o < tot; o += stride) {
+        const int64_t j = o % a.ps;
+        const int i = (int)((o / a.ps) % (a.s + 1));
+        const int g = (int)(o / (a.ps * (a.s + 1)));
+        if (i < 3 || j >= a.p || j < i - 1 || a.need[o]) continue;
+        const float m32 = a.dp32[d32(a, g, i, j)];
+        if (m32 < CUDART_INF_F) { dp64[o] = (double)m32; bp[o] = -2; }
+    }
 }
 
 // ----------------------------------------------------------- exact layer
@@ -1237,41 +1295,121 @@ __device__ __forceinline__ void exact_candidate(const Prefix &P, const double *p
     if (c < best || (c == best && k < arg)) { best = c; arg = (int32_t)k; }
 }
 
-__global__ void k_exact_layer(Prefix P, FastArgs a, int i, double *dp64, int32_t *bp) {
-    int64_t tot = (int64_t)a.G * a.p;
-    int64_t id = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (id >= tot) return;
-    int64_t j = id % a.p;
-    int g = (int)(id / a.p);
-    if (j < i - 1) return;
-    size_t o = oidx(a, g, i, j);
-    float m32 = a.dp32[d32(a, g, i, j)];
-    if (!(m32 < CUDART_INF_F)) return;
-    if (!a.need[o]) { dp64[o] = (double)m32; bp[o] = -2; return; }
-    int cnt = a.mcnt[o];
-    double lam = a.prm->lam64[g];
-    const double *prev = dp64 + oidx(a, g, i - 1, 0);
-    double best = CUDART_INF;
-    int32_t arg = INT32_MAX;
-    long long nres = 0;
-    if (cnt >= 0 && cnt <= NMEM) {
-        const int32_t *mem = a.members + o * NMEM;
-        for (int q = 0; q < cnt; q++) exact_candidate(P, prev, mem[q], j, lam, best, arg);
-        nres = cnt;
-    } else {
-        // many members or overflowed runs: re-scan the tiles in fp32, re-score members on the fly
-        visit_band(a, g, i, j, a.band[o], band_threshold(a, i, m32), [&](int64_t k) {
-            exact_candidate(P, prev, k, j, lam, best, arg);
-            nres++;
-        });
-    }
-    if (arg == INT32_MAX) arg = -1;
+// Result of a resolved output and its certificate check: the fp32 minimum must lie
+// within eps_i of the exact one.
+__device__ __forceinline__ bool exact_store(const FastArgs &a, int g, int i, int64_t j, double best, int32_t arg,
+                                            double *dp64, int32_t *bp) {
+    const size_t o = oidx(a, g, i, j);
     dp64[o] = best;
-    bp[o] = arg;
-    // certificate check: the fp32 minimum must lie within eps_i of the exact one
-    double e = (double)a.prm->eps[i];
-    if (!(fabs((double)m32 - best) <= e * best * 1.0001)) atomicAdd(&a.st->bound_viol, 1);
-    atomicAdd((unsigned long long *)&a.st->rescored, (unsigned long long)nres);
+    bp[o] = arg == INT32_MAX ? -1 : arg;
+    const float m32 = a.dp32[d32(a, g, i, j)];
+    const double e = (double)a.prm->eps[i];
+    return fabs((double)m32 - best) <= e * best * 1.0001;
+}
+
+__device__ __forceinline__ void count_exact(const FastArgs &a, unsigned long long nres, int nviol) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        nres += __shfl_xor_sync(0xffffffffu, nres, o);
+        nviol += __shfl_xor_sync(0xffffffffu, nviol, o);
+    }
+    if ((threadIdx.x & 31) == 0) {
+        if (nres) atomicAdd((unsigned long long *)&a.st->rescored, nres);
+        if (nviol) atomicAdd(&a.st->bound_viol, nviol);
+    }
+}
+
+// Layer i, outputs with at most NMEM members: one thread each, binary64 re-scoring
+// with double-double interval costs; the lowest k among exact minima wins.
+__global__ void k_exact_small(Prefix P, FastArgs a, int i, double *dp64, int32_t *bp) {
+    const int n = a.list_cnt[2 * i];
+    const int32_t *list = layer_list(a, i, 0);
+    unsigned long long nres = 0;
+    int nviol = 0;
+    const int stride = gridDim.x * blockDim.x;
+    for (int base = blockIdx.x * blockDim.x; base < n; base += stride) {  // warp-uniform trip count
+        const int e = base + threadIdx.x;
+        if (e < n) {
+            const int32_t v = list[e];
+            const int g = v >> 24;
+            const int64_t j = v & 0xFFFFFF;
+            const size_t o = oidx(a, g, i, j);
+            const int cnt = a.mcnt[o];
+            const double lam = a.prm->lam64[g];
+            const double *prev = dp64 + oidx(a, g, i - 1, 0);
+            const int32_t *mem = a.members + o * NMEM;
+            double best = CUDART_INF;
+            int32_t arg = INT32_MAX;
+            for (int q = 0; q < cnt; q++) exact_candidate(P, prev, mem[q], j, lam, best, arg);
+            nres += cnt;
+            nviol += exact_store(a, g, i, j, best, arg, dp64, bp) ? 0 : 1;
+        }
+    }
+    count_exact(a, nres, nviol);
+}
+
+// Layer i, outputs with more members: one warp each (fp32 re-evaluation within the
+// band, exact re-scoring of the members met), then the lanes' results meet (value,
+// then lowest k).  With resident costs the lanes split every tile's k (the table
+// gives any pair directly); otherwise they take whole tiles (the recurrence of
+// visit_tile runs along k).
+__global__ void k_exact_big(Prefix P, FastArgs a, int i, double *dp64, int32_t *bp) {
+    const int n = a.list_cnt[2 * i + 1];
+    const int32_t *list = layer_list(a, i, 1);
+    const int lane = threadIdx.x & 31;
+    const int warps = gridDim.x * (blockDim.x >> 5);
+    unsigned long long nres = 0;
+    int nviol = 0;
+    for (int e = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); e < n; e += warps) {
+        const int32_t v = list[e];
+        const int g = v >> 24;
+        const int64_t j = v & 0xFFFFFF;
+        const size_t o = oidx(a, g, i, j);
+        const float m32 = a.dp32[d32(a, g, i, j)];
+        const float thr = band_threshold(a, i, m32);
+        const uint64_t w = a.band[o];
+        const uint32_t w1 = (uint32_t)w, w2 = (uint32_t)(w >> 32);
+        const uint32_t n1 = (w1 & 0xFFFFu) - (w1 >> 16) + 1u;
+        const uint32_t ntile = n1 + (w2 ? (w2 & 0xFFFFu) - (w2 >> 16) + 1u : 0u);
+        const double lam = a.prm->lam64[g];
+        const double *prev = dp64 + oidx(a, g, i - 1, 0);
+        double best = CUDART_INF;
+        int32_t arg = INT32_MAX;
+        if (a.costs) {
+            const float lam32 = a.prm->lam32[g];
+            const int64_t J = j / BJ, j0 = J * BJ;
+            for (uint32_t t = 0; t < ntile; t++) {
+                const int64_t K = t < n1 ? (w1 >> 16) + t : (w2 >> 16) + (t - n1);
+                const int64_t k0 = K * BK;
+                const float *cr = a.costs + cost_tile_idx(K, J) * kCostTileFloats + (size_t)(j - j0) * PSTR;
+                const float *pr = cr + kCostHalfFloats;
+                const float *prev32 = a.dp32 + d32(a, g, i - 1, k0) - k0;
+                const int64_t khi = (K == J) ? j - 1 : k0 + BK - 1;
+                for (int64_t k = k0 + lane; k <= khi; k += 32) {
+                    if (cand32(prev32[k], lam32, cr[k - k0], pr[k - k0]) <= thr) {
+                        exact_candidate(P, prev, k, j, lam, best, arg);
+                        nres++;
+                    }
+                }
+            }
+        } else {
+            for (uint32_t t = lane; t < ntile; t += 32) {
+                const uint32_t K = t < n1 ? (w1 >> 16) + t : (w2 >> 16) + (t - n1);
+                visit_tile(a, g, i, j, (int64_t)K, thr, [&](int64_t k) {
+                    exact_candidate(P, prev, k, j, lam, best, arg);
+                    nres++;
+                });
+            }
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+            const double b2 = __shfl_xor_sync(0xffffffffu, best, off);
+            const int32_t a2 = __shfl_xor_sync(0xffffffffu, arg, off);
+            if (b2 < best || (b2 == best && a2 < arg)) { best = b2; arg = a2; }
+        }
+        if (lane == 0) nviol += exact_store(a, g, i, j, best, arg, dp64, bp) ? 0 : 1;
+    }
+    count_exact(a, nres, nviol);
 }
 
 // ------------------------------------------------------------------ host
@@ -1291,7 +1429,9 @@ size_t fast_dp_band_bytes(int64_t d, int32_t s) {
     size_t nJ = (size_t)cdiv(d, BJ);
     return align256(8 * rows) + align256(4 * rows) + align256(4 * NMEM * rows) + align256(rows) +
            align256(4 * (size_t)kMaxG * nJ + 64) + align256(sizeof(FastParams)) + align256(32 * nJ * (nJ + 1) / 2) +
-           align256(4 * (size_t)kMaxG * (size_t)mdp_stride(s) * nJ);
+           align256(4 * (size_t)kMaxG * (size_t)mdp_stride(s) * nJ) +
+           align256(2 * 4 * (size_t)kMaxG * (size_t)(s + 1) * (size_t)table_stride(d)) +
+           align256(4 * 2 * (size_t)(s + 1));
 }
 
 static size_t smem_bytes(int Gc, int s) { return sizeof(Smem) + (size_t)2 * Gc * (s - 2) * BK * sizeof(float); }
@@ -1365,7 +1505,12 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     a.corner = reinterpret_cast<float *>(base);
     {
         size_t nJd = (size_t)cdiv(Lw.d, BJ);
-        a.mdp = reinterpret_cast<float *>(base + align256(32 * nJd * (nJd + 1) / 2));
+        char *q = base + align256(32 * nJd * (nJd + 1) / 2);
+        a.mdp = reinterpret_cast<float *>(q);
+        q += align256(4 * (size_t)kMaxG * (size_t)mdp_stride(s) * nJd);
+        a.lists = reinterpret_cast<int32_t *>(q);
+        q += align256(2 * 4 * (size_t)kMaxG * (size_t)(s + 1) * (size_t)table_stride(Lw.d));
+        a.list_cnt = reinterpret_cast<int *>(q);
     }
     a.mdp_stride = mdp_stride(s);
     a.prune = (costs && a.lgc == 2 && a.mdp_stride <= 20) ? 1 : 0;
@@ -1421,15 +1566,23 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     k_need_init<<<(unsigned)std::min<int64_t>(cdiv((int64_t)G * (s + 1) * P.ps, 256), (int64_t)nsm * 32), 256, 0, st>>>(
         a, ilo, exact_tables ? 1 : 0);
     ECASQ_LAUNCH_CHECK();
+    ECASQ_CUDA_TRY(cudaMemsetAsync(a.list_cnt, 0, sizeof(int) * 2 * (size_t)(s + 1), st));
     const unsigned gl = (unsigned)std::min<int64_t>(cdiv((int64_t)G * P.p, 128), (int64_t)nsm * 64);
     for (int i = s; i >= 3; i--) {
         note_launch();
         k_need_layer<<<gl, 128, 0, st>>>(a, i);
         ECASQ_LAUNCH_CHECK();
     }
+    note_launch();
+    k_fill_unneeded<<<(unsigned)std::min<int64_t>(cdiv((int64_t)G * (s + 1) * P.ps, 256), (int64_t)nsm * 32), 256, 0,
+                      st>>>(a, dp64, bp);
+    ECASQ_LAUNCH_CHECK();
     for (int i = 3; i <= s; i++) {
         note_launch();
-        k_exact_layer<<<(unsigned)cdiv((int64_t)G * P.p, 128), 128, 0, st>>>(P, a, i, dp64, bp);
+        k_exact_small<<<(unsigned)nsm * 8, 128, 0, st>>>(P, a, i, dp64, bp);
+        ECASQ_LAUNCH_CHECK();
+        note_launch();
+        k_exact_big<<<(unsigned)nsm * 16, 128, 0, st>>>(P, a, i, dp64, bp);
         ECASQ_LAUNCH_CHECK();
     }
     return ECASQ_OK;

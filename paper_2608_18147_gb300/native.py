@@ -144,12 +144,12 @@ def _check(rc, where, ok=(OK,)):
 def ws_status(ws):
     """Counters the library leaves at the start of a workspace after a call
     (unique values, device-side flags, fast-DP statistics)."""
-    raw = ws[:80].cpu().numpy().tobytes()
+    raw = ws[:96].cpu().numpy().tobytes()
     (p, nonfinite, range_err, timeout, bound_viol, norm2, rescored, overflow, last_s, last_G, last_d, members,
-     big_bands) = __import__("struct").unpack("<qiiiidqqiiqqq", raw)
+     big_bands, tiles_run, tiles_skipped) = __import__("struct").unpack("<qiiiidqqiiqqqqq", raw)
     return dict(p=p, nonfinite=nonfinite, range_err=range_err, timeout=timeout, bound_viol=bound_viol, norm2=norm2,
                 rescored=rescored, overflow=overflow, last_s=last_s, last_G=last_G, last_d=last_d, members=members,
-                big_bands=big_bands)
+                big_bands=big_bands, tiles_run=tiles_run, tiles_skipped=tiles_skipped)
 
 
 def ecasq_workspace_size(d, s, rows=1) -> int:
