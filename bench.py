@@ -31,6 +31,10 @@ SM_COUNT = 152
 FP32_LANES = 128          # FP32-pipe lanes per SM (adds and min/max share them)
 SM_MAX_MHZ = 2070.0
 OPS_PER_CANDIDATE = 2     # one add and one min per min-plus candidate
+# DRAM bytes of one k_wavefront_res launch per 64 x 64 tile, from the ncu capture in
+# profiles/k_wavefront_res_lognormal_d16384_s16.md (read 1.146458 GB + write 7.4 MB over
+# 32896 tiles); the benchmark launch is scaled by its own tile count.
+TRAFFIC_PER_TILE = (1.146458e9 + 7.448576e6) / 32896
 ORACLE_SAMPLE = 16384     # entries of the CPU baseline's bounded sample
 
 
@@ -228,15 +232,19 @@ def main():
     cand_total = sum(r["candidates"] for r in results)
     clocks = clk.summary()
     st = E.native.ws_status(ws)  # counters of the last solve
+    last_p = results[-1]["p"]
     units = st["tiles_run"] + st["tiles_skipped"]
     run_frac = st["tiles_run"] / units if units else 1.0
 
     # roofline of the min-plus kernel: FP32-pipe ops (one add + one min per candidate)
     achieved = OPS_PER_CANDIDATE * cand_total / (dp_ms / 1000.0) / 1e12 if dp_ms > 0 else None
     peak = SM_COUNT * FP32_LANES * SM_MAX_MHZ * 1e6 / 1e12
+    nJ = (last_p + 63) // 64
+    traffic = TRAFFIC_PER_TILE * nJ * (nJ + 1) // 2 if (flags & E.RESIDENT_COSTS) else None
     roofline = {"bound": "alu", "achieved": achieved, "peak": peak, "unit": "TOP/s",
-                "frac": (achieved / peak) if achieved else None, "traffic": None,
-                "kernel": "k_wavefront",
+                "frac": (achieved / peak) if achieved else None, "traffic": traffic,
+                "traffic_note": "DRAM bytes per launch, scaled from an ncu capture at d = 16384 by tiles",
+                "kernel": "k_wavefront_res" if (flags & E.RESIDENT_COSTS) else "k_wavefront",
                 "peak_basis": "152 SMs x 128 FP32-pipe lanes (adds and mins share them) x 2070 MHz max clock",
                 "avg_launch_ms": dp_ms / max(dp_launches, 1), "launches": dp_launches,
                 "ops_basis": "algorithmic: 2 ops for every candidate of eq. apx_rec (all layers, multipliers, k < j)",
