@@ -18,6 +18,10 @@ int launch_dp_reference(const Prefix &P, const double *lamp, int G, int s, doubl
 int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, const Layout &L, cudaStream_t st,
                    bool exact_s, bool exact_tables, float *costs, bool build_costs);
 size_t resident_costs_bytes(int64_t d);
+int launch_rows_prepare(const float *X, int64_t rows, const RowsData &R, cudaStream_t st);
+int launch_rows_pass(const RowsPass &A, int nact, int pmax, cudaStream_t st);
+int launch_rows_gather(const RowsData &R, const int32_t *a, const int32_t *m, int64_t rows, int s, float *Q,
+                       cudaStream_t st);
 int launch_traceback_eval(const Prefix &P, int G, int s, int exact_s, const double *dp64, const int32_t *bp,
                           int32_t *qidx, int32_t *mcount, double *metrics, cudaStream_t st);
 int launch_eval_codebook(const Prefix &P, const int32_t *a, int m, double *out3, cudaStream_t st);
@@ -130,6 +134,41 @@ static int noalloc_scratch(void **out) {
     }
     *out = g_noalloc_addr[dev];
     return ECASQ_OK;
+}
+
+// Batched short rows (d <= kScanTile): per-row prefix data, pass scratch and
+// results, placed after the single-row layout (which the rows that cannot take the
+// batched path still use).
+struct RowsLayout {
+    size_t v, w, N, S, S2, p, norm2, nonfinite, bp, lam, act, mcount, metrics, qidx, sel, m, total;
+};
+static size_t rows_layout(int64_t d, int32_t s, int64_t rows, RowsLayout *R) {
+    size_t off = 0;
+    auto take = [&](size_t bytes) { size_t o = off; off += align256(bytes); return o; };
+    const size_t n = (size_t)rows, dc = (size_t)d;
+    R->v = take(4 * n * dc);
+    R->w = take(8 * n * dc);
+    R->N = take(8 * n * (dc + 1));
+    R->S = take(16 * n * (dc + 1));
+    R->S2 = take(16 * n * (dc + 1));
+    R->p = take(8 * n);
+    R->norm2 = take(8 * n);
+    R->nonfinite = take(4 * n);
+    R->bp = take(4 * n * kMaxG * (size_t)(s + 1) * dc);
+    R->lam = take(8 * n * kMaxG);
+    R->act = take(4 * n);
+    R->mcount = take(4 * n * kMaxG);
+    R->metrics = take(32 * n * kMaxG);
+    R->qidx = take(4 * n * kMaxG * (size_t)s);
+    R->sel = take(4 * n * (size_t)s);
+    R->m = take(4 * n);
+    R->total = off;
+    return off;
+}
+static size_t rows_region_bytes(int64_t d, int32_t s, int64_t rows) {
+    if (d > kScanTile) return 0;
+    RowsLayout R;
+    return rows_layout(d, s, rows, &R);
 }
 
 // ECASQ_RESIDENT_COSTS: the interval-cost tiles follow the common layout.
@@ -339,7 +378,7 @@ const char *ecasq_strerror(int status) {
 size_t ecasq_workspace_size(int64_t d, int32_t s, int64_t rows) {
     if (d < 1 || d >= ((int64_t)1 << 31) || s < 2 || s > kMaxS || rows < 1) return 0;
     Layout L;
-    return make_layout(d, s, rows, &L);
+    return make_layout(d, s, rows, &L) + rows_region_bytes(d, s, rows);
 }
 
 size_t ecasq_workspace_size_flags(int64_t d, int32_t s, int64_t rows, uint32_t flags) {
@@ -735,10 +774,257 @@ int ecasq_quantize_noalloc(const float *x, int64_t d, const float *Q, int32_t m,
     return ECASQ_OK;
 }
 
+// Short rows (d <= kScanTile, no refinement): every row runs the multiplier search
+// of ecasq_solve in lockstep with the others -- one k_rows_pass launch per round
+// for all rows still searching -- with the per-row arithmetic of the reference DP,
+// so each row's result equals ecasq_solve on that row alone.  Rows with more than
+// kRowsMaxP unique values, longer rows and refinement take ecasq_solve row by row.
+static int solve_rows_batched(const float *X, int64_t rows, int64_t d, const ecasq_params_t *prm, void *ws,
+                              size_t ws_bytes, float *Q, int32_t *m_out, ecasq_result_t *res, cudaStream_t st) {
+    const int s = prm->s;
+    Layout L1;
+    make_layout(d, s, 1, &L1);
+    int rc = add_resident_costs(prm->flags, &L1);
+    if (rc) return rc;
+    RowsLayout RL;
+    rows_layout(d, s, rows, &RL);
+    const size_t roff = align256(L1.total);
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255) != 0 || ws_bytes < roff + RL.total) return ECASQ_EWORKSPACE;
+    char *rb = static_cast<char *>(ws) + roff;
+    RowsData R;
+    R.v = reinterpret_cast<float *>(rb + RL.v);
+    R.w = reinterpret_cast<int64_t *>(rb + RL.w);
+    R.N = reinterpret_cast<int64_t *>(rb + RL.N);
+    R.S = reinterpret_cast<double *>(rb + RL.S);
+    R.S2 = reinterpret_cast<double *>(rb + RL.S2);
+    R.p = reinterpret_cast<int64_t *>(rb + RL.p);
+    R.norm2 = reinterpret_cast<double *>(rb + RL.norm2);
+    R.nonfinite = reinterpret_cast<int32_t *>(rb + RL.nonfinite);
+    R.d = d;
+    R.dcap = d;
+    rc = launch_rows_prepare(X, rows, R, st);
+    if (rc) return rc;
+    std::vector<int64_t> ph(rows);
+    std::vector<double> n2h(rows);
+    std::vector<int32_t> nfh(rows);
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(ph.data(), R.p, 8 * (size_t)rows, cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(n2h.data(), R.norm2, 8 * (size_t)rows, cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(nfh.data(), R.nonfinite, 4 * (size_t)rows, cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    for (int64_t r = 0; r < rows; r++)
+        if (nfh[r]) return ECASQ_ENONFINITE;
+
+    // per-row search state (the schedule of ecasq_solve)
+    struct Row {
+        std::vector<Eval> evals;
+        double lo, hi;
+        bool done = false, failed = false;
+        int sel = -1, status = ECASQ_OK, passes = 0, nlam = 0;
+    };
+    std::vector<Row> st_rows(rows);
+    const bool fixed = prm->lambda >= 0.0;
+    double lo0 = prm->lambda_lo > 0.0 ? prm->lambda_lo : 1e-8;
+    double hi0 = prm->lambda_hi > 0.0 ? prm->lambda_hi : 1e3;
+    const int Rn = prm->search_rounds > 0 ? prm->search_rounds : 6;
+    if (!fixed && !(hi0 > lo0)) return ECASQ_EINVAL;
+    std::vector<int64_t> slow;  // rows that take ecasq_solve
+    for (int64_t r = 0; r < rows; r++) {
+        st_rows[r].lo = lo0;
+        st_rows[r].hi = hi0;
+        if (ph[r] > kRowsMaxP) { slow.push_back(r); st_rows[r].done = true; }
+        else if (ph[r] == 1) st_rows[r].done = true;
+    }
+    int32_t *actd = reinterpret_cast<int32_t *>(rb + RL.act);
+    double *lamd = reinterpret_cast<double *>(rb + RL.lam);
+    int32_t *mcd = reinterpret_cast<int32_t *>(rb + RL.mcount);
+    double *metd = reinterpret_cast<double *>(rb + RL.metrics);
+    int32_t *qid = reinterpret_cast<int32_t *>(rb + RL.qidx);
+    // one pass over `act` rows, G multipliers each (lams: row-major [nact][G], vNMSE scale)
+    auto pass = [&](const std::vector<int32_t> &act, const std::vector<double> &lams, int G) -> int {
+        const int nact = (int)act.size();
+        if (!nact) return ECASQ_OK;
+        std::vector<double> lamp((size_t)nact * G);
+        int pmax = 2;
+        for (int b = 0; b < nact; b++) {
+            for (int g = 0; g < G; g++) lamp[(size_t)b * G + g] = lams[(size_t)b * G + g] * n2h[act[b]];
+            pmax = std::max<int>(pmax, (int)ph[act[b]]);
+        }
+        ECASQ_CUDA_TRY(cudaMemcpyAsync(actd, act.data(), 4 * (size_t)nact, cudaMemcpyHostToDevice, st));
+        ECASQ_CUDA_TRY(cudaMemcpyAsync(lamd, lamp.data(), 8 * lamp.size(), cudaMemcpyHostToDevice, st));
+        RowsPass A;
+        A.R = R;
+        A.rows = actd;
+        A.lam = lamd;
+        A.G = G;
+        A.s = s;
+        A.exact_s = (prm->flags & ECASQ_EXACT_S) ? 1 : 0;
+        A.bp = reinterpret_cast<int32_t *>(rb + RL.bp);
+        A.qidx = qid;
+        A.mcount = mcd;
+        A.metrics = metd;
+        int r2 = launch_rows_pass(A, nact, pmax, st);
+        if (r2) return r2;
+        std::vector<int32_t> mh((size_t)nact * G), qh((size_t)nact * G * s);
+        std::vector<double> meth((size_t)nact * G * 4);
+        ECASQ_CUDA_TRY(cudaMemcpyAsync(mh.data(), mcd, 4 * mh.size(), cudaMemcpyDeviceToHost, st));
+        ECASQ_CUDA_TRY(cudaMemcpyAsync(qh.data(), qid, 4 * qh.size(), cudaMemcpyDeviceToHost, st));
+        ECASQ_CUDA_TRY(cudaMemcpyAsync(meth.data(), metd, 8 * meth.size(), cudaMemcpyDeviceToHost, st));
+        ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+        for (int b = 0; b < nact; b++) {
+            Row &w = st_rows[act[b]];
+            w.passes++;
+            w.nlam += G;
+            bool bad = false;
+            for (int g = 0; g < G; g++) {
+                const size_t q = (size_t)b * G + g;
+                Eval e;
+                e.lam = lams[q];
+                e.m = mh[q];
+                e.mse = meth[4 * q + 1];
+                e.hs = meth[4 * q + 2];
+                e.hx = meth[4 * q + 3];
+                e.feas = fixed ? true : (e.hs <= prm->budget_bits);
+                e.a.assign(qh.begin() + q * s, qh.begin() + q * s + std::max(e.m, 0));
+                w.evals.push_back(e);
+                if (e.m < 1) bad = true;
+            }
+            if (bad) { w.failed = true; w.done = true; w.status = ECASQ_EINFEASIBLE; }
+        }
+        return ECASQ_OK;
+    };
+    auto active = [&]() {
+        std::vector<int32_t> act;
+        for (int64_t r = 0; r < rows; r++)
+            if (!st_rows[r].done) act.push_back((int32_t)r);
+        return act;
+    };
+    if (fixed) {
+        std::vector<int32_t> act = active();
+        rc = pass(act, std::vector<double>(act.size(), prm->lambda), 1);
+        if (rc) return rc;
+        for (int32_t r : act)
+            if (!st_rows[r].failed) st_rows[r].sel = 0;
+    } else {
+        double t[7];
+        {  // multiplier 0 and the first round together
+            std::vector<int32_t> act = active();
+            midpoints7(lo0, hi0, t);
+            std::vector<double> lams;
+            for (size_t b = 0; b < act.size(); b++) {
+                lams.push_back(0.0);
+                lams.insert(lams.end(), t, t + 7);
+            }
+            rc = pass(act, lams, 8);
+            if (rc) return rc;
+            for (int32_t r : act) {
+                Row &w = st_rows[r];
+                if (w.failed) continue;
+                if (w.evals[0].feas) { w.sel = 0; w.done = true; }
+            }
+        }
+        for (int rr = 0; rr < Rn; rr++) {
+            std::vector<int32_t> act = active();
+            if (rr > 0) {
+                std::vector<double> lams;
+                for (int32_t r : act) {
+                    midpoints7(st_rows[r].lo, st_rows[r].hi, t);
+                    lams.insert(lams.end(), t, t + 7);
+                }
+                rc = pass(act, lams, 7);
+                if (rc) return rc;
+            }
+            for (int32_t r : act) {
+                Row &w = st_rows[r];
+                if (w.failed) continue;
+                const Eval *pts = &w.evals[w.evals.size() - 7];
+                int f = -1;
+                for (int q = 0; q < 7; q++)
+                    if (pts[q].feas) { f = q; break; }
+                if (f >= 0) {
+                    double nlo = f > 0 ? pts[f - 1].lam : w.lo;
+                    w.hi = pts[f].lam;
+                    w.lo = nlo;
+                } else {
+                    w.lo = pts[6].lam;
+                }
+            }
+        }
+        std::vector<int32_t> need_hi;
+        std::vector<double> his;
+        for (int32_t r : active()) {
+            Row &w = st_rows[r];
+            for (size_t q = 0; q < w.evals.size(); q++) {
+                const Eval &e = w.evals[q];
+                if (e.feas && (w.sel < 0 || e.mse < w.evals[w.sel].mse ||
+                               (e.mse == w.evals[w.sel].mse && e.lam < w.evals[w.sel].lam)))
+                    w.sel = (int)q;
+            }
+            if (w.sel < 0) { need_hi.push_back(r); his.push_back(w.hi); }
+        }
+        rc = pass(need_hi, his, 1);
+        if (rc) return rc;
+        for (int32_t r : need_hi) {
+            Row &w = st_rows[r];
+            if (w.failed) continue;
+            w.sel = (int)w.evals.size() - 1;
+            if (!w.evals[w.sel].feas) w.status = ECASQ_EINFEASIBLE;
+        }
+    }
+    // selected codebooks -> Q, m; results
+    std::vector<int32_t> selh((size_t)rows * s, 0), mh(rows, 0);
+    int status = ECASQ_OK;
+    for (int64_t r = 0; r < rows; r++) {
+        Row &w = st_rows[r];
+        if (std::find(slow.begin(), slow.end(), r) != slow.end()) continue;
+        double zero3[3] = {0.0, 0.0, 0.0};
+        if (ph[r] == 1) {
+            mh[r] = 1;
+            selh[(size_t)r * s] = 0;
+            fill_result(res ? &res[r] : nullptr, ECASQ_OK, 1, d, 1, fixed ? prm->lambda : 0.0, n2h[r], zero3, 0.0, 0, 0,
+                        0, 0, 0);
+            continue;
+        }
+        if (w.failed || w.sel < 0) {
+            status = ECASQ_EINFEASIBLE;
+            if (res) { memset(&res[r], 0, sizeof(res[r])); res[r].status = ECASQ_EINFEASIBLE; res[r].d = d; res[r].p = ph[r]; }
+            continue;
+        }
+        const Eval &e = w.evals[w.sel];
+        mh[r] = e.m;
+        for (int q = 0; q < e.m; q++) selh[(size_t)r * s + q] = e.a[q];
+        const double ev[3] = {e.mse, e.hs, e.hx};
+        const double lamp = e.lam * n2h[r];
+        if (w.status != ECASQ_OK) status = w.status;
+        fill_result(res ? &res[r] : nullptr, w.status, e.m, d, ph[r], e.lam, n2h[r], ev, ev[0] + lamp * ev[1], w.passes,
+                    w.nlam, 0, candidates_of(ph[r], s, 0) * w.nlam, 0);
+    }
+    int32_t *seld = reinterpret_cast<int32_t *>(rb + RL.sel);
+    int32_t *md = reinterpret_cast<int32_t *>(rb + RL.m);
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(seld, selh.data(), 4 * selh.size(), cudaMemcpyHostToDevice, st));
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(md, mh.data(), 4 * mh.size(), cudaMemcpyHostToDevice, st));
+    rc = launch_rows_gather(R, seld, md, rows, s, Q, st);
+    if (rc) return rc;
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(m_out, md, 4 * (size_t)rows, cudaMemcpyDeviceToDevice, st));
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    // rows with many unique values: the single-row path (its layout sits before the row data)
+    for (int64_t r : slow) {
+        ecasq_result_t one;
+        rc = ecasq_solve(X + r * d, d, prm, ws, roff, Q + r * s, &one, reinterpret_cast<ecasq_stream_t>(st));
+        if (rc != ECASQ_OK && rc != ECASQ_EINFEASIBLE) return rc;
+        if (rc == ECASQ_EINFEASIBLE) status = rc;
+        ECASQ_CUDA_TRY(cudaMemcpyAsync(m_out + r, &one.m, sizeof(int32_t), cudaMemcpyHostToDevice, st));
+        if (res) res[r] = one;
+    }
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    return status;
+}
+
 int ecasq_solve_batched(const float *X, int64_t rows, int64_t d, const ecasq_params_t *prm, void *ws,
                         size_t ws_bytes, float *Q, int32_t *m_out, ecasq_result_t *res, ecasq_stream_t stream) {
     if (!X || !Q || !m_out || rows < 1 || d < 1 || d >= ((int64_t)1 << 31) || !params_ok(prm)) return ECASQ_EINVAL;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (d <= kScanTile && prm->refine_max_rounds == 0)
+        return solve_rows_batched(X, rows, d, prm, ws, ws_bytes, Q, m_out, res, st);
     int status = ECASQ_OK;
     for (int64_t r = 0; r < rows; r++) {
         ecasq_result_t one;

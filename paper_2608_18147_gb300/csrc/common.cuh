@@ -127,6 +127,31 @@ __device__ __forceinline__ double dd_round(dd a) { return __dadd_rn(a.hi, a.lo);
 // h(y) = -y log2 y, h(0) = 0 (Sec. 4).
 __device__ __forceinline__ double hfun(double y) { return y > 0.0 ? -__dmul_rn(y, log2(y)) : 0.0; }
 
+// Per-row prefix data of the batched path (rows of length d <= kScanTile): row r
+// holds v[dcap], w[dcap], N[dcap+1], S and S2 [2(dcap+1)] packed as (hi[0..p], lo[0..p]).
+struct RowsData {
+    float *v;
+    int64_t *w, *N;
+    double *S, *S2;
+    int64_t *p;       // [rows]
+    double *norm2;    // [rows]
+    int32_t *nonfinite;  // [rows]
+    int64_t d, dcap;
+};
+
+// One search round of the batched path: block b runs row rows[b] at G multipliers.
+constexpr int kRowsMaxP = 128;  // unique values per row the batched path holds in shared memory
+struct RowsPass {
+    RowsData R;
+    const int32_t *rows;  // [nact] row of each block
+    const double *lam;    // [nact][G] lambda' of the row
+    int G, s, exact_s;
+    int32_t *bp;          // [nact][G][s+1][dcap]
+    int32_t *qidx;        // [nact][G][s]
+    int32_t *mcount;      // [nact][G]
+    double *metrics;      // [nact][G][4]
+};
+
 // Prefix-sum view (App. E) used by every exact pair evaluation.
 struct Prefix {
     const float *v;       // [p]

@@ -173,6 +173,155 @@ __global__ void k_locate_q(const float *v, int64_t p, const float *Q, int m, int
     }
 }
 
+// ------------------------------------------------------------ short rows
+// One DP pass of the search for many independent rows (p <= kRowsMaxP), one block
+// per row: the interval costs of every pair k < j of the row are computed once into
+// shared memory (pair_exact / phi_exact, the reference formulas), then eq. apx_base
+// and apx_rec run for the row's G multipliers with two layers in shared memory
+// (candidates, lowest k and smallest i exactly as k_dp_base, k_dp_layer_ref and
+// k_traceback_eval), and each multiplier's codebook is traced and evaluated by
+// eval_codebook_warp.  Backpointers go to the caller's scratch.
+__host__ __device__ __forceinline__ int tri(int k, int j) { return j * (j - 1) / 2 + k; }
+
+__global__ void __launch_bounds__(256) k_rows_pass(RowsPass A) {
+    extern __shared__ __align__(16) double rsm[];
+    const int b = blockIdx.x;
+    const int64_t row = A.rows[b];
+    const RowsData &R = A.R;
+    const int64_t dcap = R.dcap;
+    const int p = (int)R.p[row];
+    const int G = A.G, s = A.s;
+    Prefix P;
+    P.v = R.v + row * dcap;
+    P.w = R.w + row * dcap;
+    P.N = R.N + row * (dcap + 1);
+    P.S = R.S + row * 2 * (dcap + 1);
+    P.S2 = R.S2 + row * 2 * (dcap + 1);
+    P.p = p;
+    P.d = R.d;
+    P.ps = p;
+    const int npair = p * (p - 1) / 2;
+    double *Cs = rsm;                    // [npair]
+    double *Ph = Cs + npair;             // [npair]
+    double *PhF = Ph + npair;            // [p]   Phi^first[0, j]
+    double *dpb = PhF + p;               // [2][G][p]
+    double *last = dpb + 2 * G * p;      // [G][s+1] dp(i, p-1)
+    double *scratch = last + G * (s + 1);  // [4 kMaxS] evaluation scratch
+    __shared__ int32_t a_sm[kMaxS];
+    __shared__ int sm_m;
+    double lam[kMaxG];
+#pragma unroll
+    for (int g = 0; g < kMaxG; g++) lam[g] = g < G ? A.lam[(size_t)b * G + g] : 0.0;
+    for (int t = threadIdx.x; t < npair; t += blockDim.x) {
+        int j = (int)((1.0 + sqrt(1.0 + 8.0 * (double)t)) * 0.5);
+        while (j * (j - 1) / 2 > t) j--;
+        while ((j + 1) * j / 2 <= t) j++;
+        int k = t - j * (j - 1) / 2;
+        double C, U, D;
+        pair_exact(P, k, j, C, U, D);
+        Cs[t] = C;
+        Ph[t] = phi_exact(P, U, D, false);
+        if (k == 0) PhF[j] = phi_exact(P, U, D, true);
+    }
+    for (int q = threadIdx.x; q < G * (s + 1); q += blockDim.x) last[q] = CUDART_INF;
+    int32_t *bp = A.bp + (size_t)b * G * (s + 1) * dcap;
+    __syncthreads();
+    // eq. apx_base: dp(2, j) = C[0, j] + lambda' Phi^first[0, j]
+    for (int q = threadIdx.x; q < G * p; q += blockDim.x) {
+        int g = q / p, j = q % p;
+        double v = CUDART_INF;
+        int32_t arg = -1;
+        if (j >= 1) { v = __dadd_rn(Cs[tri(0, j)], __dmul_rn(lam[g], PhF[j])); arg = 0; }
+        dpb[g * p + j] = v;
+        bp[((size_t)g * (s + 1) + 2) * dcap + j] = arg;
+        if (j == p - 1) last[g * (s + 1) + 2] = v;
+    }
+    __syncthreads();
+    // eq. apx_rec, layers 3..s
+    int cur = 0;
+    for (int i = 3; i <= s; i++) {
+        const double *prev = dpb + (size_t)cur * G * p;
+        double *nxt = dpb + (size_t)(cur ^ 1) * G * p;
+        for (int q = threadIdx.x; q < G * p; q += blockDim.x) {
+            int g = q / p, j = q % p;
+            double best = CUDART_INF;
+            int32_t arg = -1;
+            for (int k = i - 2; k < j; k++) {
+                double c = __dadd_rn(prev[g * p + k], __dadd_rn(Cs[tri(k, j)], __dmul_rn(lam[g], Ph[tri(k, j)])));
+                if (c < best) { best = c; arg = k; }
+            }
+            nxt[g * p + j] = best;
+            bp[((size_t)g * (s + 1) + i) * dcap + j] = arg;
+            if (j == p - 1) last[g * (s + 1) + i] = best;
+        }
+        __syncthreads();
+        cur ^= 1;
+    }
+    // eq. apx_final and the traceback, then the metrics (one warp, multiplier by multiplier)
+    if (threadIdx.x < 32) {
+        for (int g = 0; g < G; g++) {
+            if (threadIdx.x == 0) {
+                int istar = -1;
+                double best = CUDART_INF;
+                for (int i = A.exact_s ? s : 2; i <= s; i++) {
+                    double v = last[g * (s + 1) + i];
+                    if (v < best) { best = v; istar = i; }
+                }
+                if (istar < 0) {
+                    sm_m = 0;
+                } else {
+                    int64_t j = p - 1;
+                    a_sm[istar - 1] = (int32_t)j;
+                    for (int i = istar; i >= 3; i--) {
+                        j = bp[((size_t)g * (s + 1) + i) * dcap + j];
+                        a_sm[i - 2] = (int32_t)j;
+                    }
+                    a_sm[0] = 0;
+                    sm_m = istar;
+                }
+                A.metrics[((size_t)b * G + g) * 4 + 0] = best;
+                A.mcount[(size_t)b * G + g] = sm_m;
+            }
+            __syncwarp();
+            const int m = sm_m;
+            for (int r = threadIdx.x; r < m; r += 32) A.qidx[((size_t)b * G + g) * s + r] = a_sm[r];
+            if (m > 0) eval_codebook_warp(P, a_sm, m, &A.metrics[((size_t)b * G + g) * 4 + 1], scratch);
+            __syncwarp();
+        }
+    }
+}
+
+size_t rows_pass_smem(int p, int G, int s) {
+    size_t npair = (size_t)p * (p - 1) / 2;
+    return sizeof(double) * (2 * npair + (size_t)p + 2 * (size_t)G * p + (size_t)G * (s + 1) + 4 * (size_t)kMaxS);
+}
+
+int launch_rows_pass(const RowsPass &A, int nact, int pmax, cudaStream_t st) {
+    if (nact == 0) return ECASQ_OK;
+    if (pmax > kRowsMaxP) return ECASQ_EINVAL;
+    size_t smem = rows_pass_smem(pmax, A.G, A.s);
+    ECASQ_CUDA_TRY(cudaFuncSetAttribute(k_rows_pass, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    note_launch();
+    k_rows_pass<<<(unsigned)nact, 256, smem, st>>>(A);
+    ECASQ_LAUNCH_CHECK();
+    return ECASQ_OK;
+}
+
+// Q[row][r] = v_row[a[row][r]] for the selected codebooks.
+__global__ void k_rows_gather(RowsData R, const int32_t *a, const int32_t *m, int s, float *Q) {
+    const int64_t row = blockIdx.x;
+    const float *v = R.v + row * R.dcap;
+    for (int r = threadIdx.x; r < m[row]; r += blockDim.x) Q[row * s + r] = v[a[row * s + r]];
+}
+
+int launch_rows_gather(const RowsData &R, const int32_t *a, const int32_t *m, int64_t rows, int s, float *Q,
+                       cudaStream_t st) {
+    note_launch();
+    k_rows_gather<<<(unsigned)rows, 32, 0, st>>>(R, a, m, s, Q);
+    ECASQ_LAUNCH_CHECK();
+    return ECASQ_OK;
+}
+
 // ----------------------------------------------------------- host launchers
 int launch_dp_reference(const Prefix &P, const double *lamp, int G, int s, double *dp64, int32_t *bp,
                         cudaStream_t st) {

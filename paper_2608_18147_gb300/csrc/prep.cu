@@ -253,6 +253,107 @@ __global__ void k_hist_finish(int64_t *N, int64_t *w, double *S, double *S2, con
     }
 }
 
+// ------------------------------------------------------------ short rows
+// One block per row of length d <= kScanTile: the sorted keys (bitonic sort in
+// shared memory; the order is unique, so any exact sort gives the same keys) and
+// then the arithmetic of k_hist_fill for a single tile (zero tile offset), so that
+// v, w, N, S, S2, p and ||X||^2 of every row equal what prepare_device gives for
+// that row alone.
+__global__ void __launch_bounds__(256) k_rows_prepare(const float *__restrict__ X, RowsData R) {
+    __shared__ uint32_t keys[kScanTile];
+    __shared__ ScanVal wtot[8];
+    __shared__ int nonfin;
+    const int64_t row = blockIdx.x;
+    const int d = (int)R.d;
+    const float *x = X + row * R.d;
+    if (threadIdx.x == 0) nonfin = 0;
+    __syncthreads();
+    for (int i = threadIdx.x; i < kScanTile; i += blockDim.x) {
+        uint32_t k = 0xFFFFFFFFu;  // above every finite key: padding sorts last
+        if (i < d) {
+            float f = x[i];
+            if (!isfinite(f)) nonfin = 1;
+            if (f == 0.0f) f = 0.0f;
+            k = f2key(f);
+        }
+        keys[i] = k;
+    }
+    __syncthreads();
+    int n2 = 1;
+    while (n2 < d) n2 <<= 1;
+    for (int kk = 2; kk <= n2; kk <<= 1) {
+        for (int jj = kk >> 1; jj > 0; jj >>= 1) {
+            for (int i = threadIdx.x; i < n2; i += blockDim.x) {
+                int l = i ^ jj;
+                if (l > i) {
+                    uint32_t a = keys[i], b = keys[l];
+                    bool up = (i & kk) == 0;
+                    if ((a > b) == up) { keys[i] = b; keys[l] = a; }
+                }
+            }
+            __syncthreads();
+        }
+    }
+    const int64_t dcap = R.dcap;
+    float *v = R.v + row * dcap;
+    int64_t *N = R.N + row * (dcap + 1), *w = R.w + row * dcap;
+    double *S = R.S + row * 2 * (dcap + 1), *S2 = R.S2 + row * 2 * (dcap + 1);
+    // k_hist_fill, one tile
+    const int base = threadIdx.x * 4;
+    ScanVal loc{{0.0, 0.0}, {0.0, 0.0}, 0};
+    double xs[4];
+    int hd[4];
+    for (int e = 0; e < 4; e++) {
+        int i = base + e;
+        xs[e] = 0.0; hd[e] = 0;
+        if (i < d) {
+            xs[e] = (double)key2f(keys[i]);
+            hd[e] = (i == 0 || keys[i] != keys[i - 1]);
+            loc.s = dd_add(loc.s, dd{xs[e], 0.0});
+            loc.q = dd_add(loc.q, dd{__dmul_rn(xs[e], xs[e]), 0.0});
+            loc.h += hd[e];
+        }
+    }
+    ScanVal tot;
+    ScanVal incl = block_scan_incl(loc, wtot, tot);
+    const int64_t p = tot.h;
+    ScanVal off{{0.0, 0.0}, {0.0, 0.0}, 0};
+    ScanVal run{dd_sub(incl.s, loc.s), dd_sub(incl.q, loc.q), incl.h - loc.h};
+    run = sv_add(off, run);
+    for (int e = 0; e < 4; e++) {
+        int i = base + e;
+        if (i >= d) break;
+        if (hd[e]) {
+            int64_t u = run.h;
+            v[u] = (float)xs[e];
+            N[u] = i;
+            S[u] = run.s.hi; S[p + 1 + u] = run.s.lo;
+            S2[u] = run.q.hi; S2[p + 1 + u] = run.q.lo;
+        }
+        run.s = dd_add(run.s, dd{xs[e], 0.0});
+        run.q = dd_add(run.q, dd{__dmul_rn(xs[e], xs[e]), 0.0});
+        run.h += hd[e];
+        if (i == d - 1) {
+            N[p] = d;
+            S[p] = run.s.hi; S[p + 1 + p] = run.s.lo;
+            S2[p] = run.q.hi; S2[p + 1 + p] = run.q.lo;
+            R.p[row] = p;
+            R.norm2[row] = run.q.hi;
+        }
+    }
+    __syncthreads();
+    for (int u = threadIdx.x; u < p; u += blockDim.x) w[u] = N[u + 1] - N[u];
+    if (threadIdx.x == 0) R.nonfinite[row] = nonfin;
+}
+
+int launch_rows_prepare(const float *X, int64_t rows, const RowsData &R, cudaStream_t st) {
+    if (R.d < 1 || R.d > kScanTile) return ECASQ_EINVAL;
+    note_launch();
+    k_rows_prepare<<<(unsigned)rows, 256, 0, st>>>(X, R);
+    ECASQ_LAUNCH_CHECK();
+    return ECASQ_OK;
+}
+
 int prepare_device(const float *x, int64_t d, void *ws, const Layout &L, cudaStream_t stream, int64_t *p_host,
                    double *norm2_host) {
     DevStatus *st = wsp<DevStatus>(ws, L.status);
