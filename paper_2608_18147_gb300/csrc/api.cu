@@ -140,7 +140,8 @@ static int noalloc_scratch(void **out) {
 // results, placed after the single-row layout (which the rows that cannot take the
 // batched path still use).
 struct RowsLayout {
-    size_t v, w, N, S, S2, p, norm2, nonfinite, bp, lam, act, mcount, metrics, qidx, sel, m, total;
+    size_t v, w, N, S, S2, p, norm2, nonfinite, bp, lam, act, mcount, metrics, qidx, sel, m, pairs, total;
+    int64_t pstride;
 };
 static size_t rows_layout(int64_t d, int32_t s, int64_t rows, RowsLayout *R) {
     size_t off = 0;
@@ -162,6 +163,9 @@ static size_t rows_layout(int64_t d, int32_t s, int64_t rows, RowsLayout *R) {
     R->qidx = take(4 * n * kMaxG * (size_t)s);
     R->sel = take(4 * n * (size_t)s);
     R->m = take(4 * n);
+    const int64_t pm = std::min<int64_t>(d, kRowsMaxP);
+    R->pstride = pm * (pm - 1) + pm;
+    R->pairs = take(8 * n * (size_t)R->pstride);
     R->total = off;
     return off;
 }
@@ -839,6 +843,7 @@ static int solve_rows_batched(const float *X, int64_t rows, int64_t d, const eca
     int32_t *mcd = reinterpret_cast<int32_t *>(rb + RL.mcount);
     double *metd = reinterpret_cast<double *>(rb + RL.metrics);
     int32_t *qid = reinterpret_cast<int32_t *>(rb + RL.qidx);
+    bool pairs_ready = false;
     // one pass over `act` rows, G multipliers each (lams: row-major [nact][G], vNMSE scale)
     auto pass = [&](const std::vector<int32_t> &act, const std::vector<double> &lams, int G) -> int {
         const int nact = (int)act.size();
@@ -862,7 +867,11 @@ static int solve_rows_batched(const float *X, int64_t rows, int64_t d, const eca
         A.qidx = qid;
         A.mcount = mcd;
         A.metrics = metd;
+        A.pairs = reinterpret_cast<double *>(rb + RL.pairs);
+        A.pstride = RL.pstride;
+        A.pairs_ready = pairs_ready ? 1 : 0;
         int r2 = launch_rows_pass(A, nact, pmax, st);
+        pairs_ready = true;  // every active row of a later round was active in this one
         if (r2) return r2;
         std::vector<int32_t> mh((size_t)nact * G), qh((size_t)nact * G * s);
         std::vector<double> meth((size_t)nact * G * 4);

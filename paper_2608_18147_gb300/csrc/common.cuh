@@ -150,6 +150,9 @@ struct RowsPass {
     int32_t *qidx;        // [nact][G][s]
     int32_t *mcount;      // [nact][G]
     double *metrics;      // [nact][G][4]
+    double *pairs;        // [rows][pstride]: the row's C, Phi (pair order) and Phi^first, kept across rounds
+    int64_t pstride;      // doubles per row: 2 npair(pmax) + pmax
+    int pairs_ready;      // the rows' interval costs are already in `pairs`
 };
 
 // Prefix-sum view (App. E) used by every exact pair evaluation.

@@ -212,16 +212,23 @@ __global__ void __launch_bounds__(256) k_rows_pass(RowsPass A) {
     double lam[kMaxG];
 #pragma unroll
     for (int g = 0; g < kMaxG; g++) lam[g] = g < G ? A.lam[(size_t)b * G + g] : 0.0;
-    for (int t = threadIdx.x; t < npair; t += blockDim.x) {
-        int j = (int)((1.0 + sqrt(1.0 + 8.0 * (double)t)) * 0.5);
-        while (j * (j - 1) / 2 > t) j--;
-        while ((j + 1) * j / 2 <= t) j++;
-        int k = t - j * (j - 1) / 2;
-        double C, U, D;
-        pair_exact(P, k, j, C, U, D);
-        Cs[t] = C;
-        Ph[t] = phi_exact(P, U, D, false);
-        if (k == 0) PhF[j] = phi_exact(P, U, D, true);
+    double *gp = A.pairs + row * A.pstride;  // the same three arrays, kept across rounds
+    if (A.pairs_ready) {
+        for (int t = threadIdx.x; t < 2 * npair + p; t += blockDim.x) Cs[t] = gp[t];
+    } else {
+        for (int t = threadIdx.x; t < npair; t += blockDim.x) {
+            int j = (int)((1.0 + sqrt(1.0 + 8.0 * (double)t)) * 0.5);
+            while (j * (j - 1) / 2 > t) j--;
+            while ((j + 1) * j / 2 <= t) j++;
+            int k = t - j * (j - 1) / 2;
+            double C, U, D;
+            pair_exact(P, k, j, C, U, D);
+            Cs[t] = C;
+            Ph[t] = phi_exact(P, U, D, false);
+            if (k == 0) PhF[j] = phi_exact(P, U, D, true);
+        }
+        __syncthreads();
+        for (int t = threadIdx.x; t < 2 * npair + p; t += blockDim.x) gp[t] = Cs[t];
     }
     for (int q = threadIdx.x; q < G * (s + 1); q += blockDim.x) last[q] = CUDART_INF;
     int32_t *bp = A.bp + (size_t)b * G * (s + 1) * dcap;
