@@ -31,7 +31,7 @@ __device__ __forceinline__ double local_obj(const Prefix &P, const Nbr &n, int64
     return __dadd_rn(__dadd_rn(C1, C2), __dmul_rn(lamp, ent));
 }
 
-constexpr int kRefineChunk = 2048;  // candidates per block
+constexpr int kRefineChunk = 256;   // candidates per block: one per thread, so a value's range spreads over many SMs
 
 __device__ __forceinline__ Nbr make_nbr(const Prefix &P, const int32_t *a, int m, int l) {
     Nbr n;
