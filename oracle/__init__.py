@@ -55,6 +55,7 @@ def _load():
         pi64 = C.POINTER(C.c_int64)
         sig = {
             "or_hist_new": (P, [pf, i64, pi32]),
+            "or_hist_new_grid": (P, [pf, i64, pf, i64, pi32]),
             "or_hist_free": (None, [P]),
             "or_hist_info": (None, [P, pi64, pi64, pd]),
             "or_hist_arrays": (None, [P, pf, pi64, pi64, pd, pd, pd, pd]),
@@ -106,13 +107,20 @@ def num_threads() -> int:
 class Hist:
     """Sorted weighted histogram of x with App. E prefix sums (Sec. 2, App. E)."""
 
-    def __init__(self, x):
+    def __init__(self, x, grid=None):
+        """grid: optional candidate set P (ascending fp32, first = min x, last = max x);
+        by default P = the unique values of x."""
         lib = _load()
         self._x = _f32(x)
         st = C.c_int32(0)
-        self._h = lib.or_hist_new(_ptr(self._x, C.c_float), self._x.size, C.byref(st))
+        if grid is None:
+            self._h = lib.or_hist_new(_ptr(self._x, C.c_float), self._x.size, C.byref(st))
+        else:
+            self._grid = _f32(grid)
+            self._h = lib.or_hist_new_grid(_ptr(self._x, C.c_float), self._x.size, _ptr(self._grid, C.c_float),
+                                           self._grid.size, C.byref(st))
         if not self._h:
-            raise OracleError(st.value, "or_hist_new")
+            raise OracleError(st.value, "or_hist_new" if grid is None else "or_hist_new_grid")
         d, p, n2 = C.c_int64(), C.c_int64(), C.c_double()
         lib.or_hist_info(self._h, C.byref(d), C.byref(p), C.byref(n2))
         self.d, self.p, self.norm2 = d.value, p.value, n2.value
@@ -292,9 +300,10 @@ def quantize(x, Q, seed):
 
 
 def solve_budget(x, s, budget, lo=1e-8, hi=1e3, rounds=6, refine_rounds=0, refine_tol=0.0,
-                 guard=True, exact_s=False):
-    """Full budgeted pipeline: search, then optional refinement at the chosen lambda."""
-    H = Hist(x)
+                 guard=True, exact_s=False, grid=None):
+    """Full budgeted pipeline: search, then optional refinement at the chosen lambda
+    (codebook drawn from `grid` when given, else from the unique values of x)."""
+    H = Hist(x, grid)
     if H.p <= 20000:
         H.cache()
     r = H.search(s, budget, lo, hi, rounds, exact_s)

@@ -17,6 +17,8 @@
  *
  * Functions and the passages they follow:
  *   or_hist_new      Sec. 2 (sorted copy, weighted histogram), App. E (prefix sums)
+ *   or_hist_new_grid Sec. 5 / App. E for a general permissible set P: the same
+ *                    histogram view with P as the candidate values
  *   pair_q           App. E: U_P, D_P, C_P from prefix differences
  *   h, or_phi        Sec. 4 (h), Sec. 5 (Phi, Phi^first)
  *   or_apx_dp        Sec. 5, eqs. apx_base / apx_rec / apx_final
@@ -131,6 +133,58 @@ or_hist *or_hist_new(const float *x, int64_t d, int32_t *status) {
         H->S2[t + 1] = H->S2[t] + ww * vv * vv;
     }
     H->norm2 = (double)H->S2[p];
+    return H;
+}
+
+/* General permissible set P (Sec. 5, App. E): candidate values p_0 < ... < p_{n-1}
+ * with p_0 = min x and p_{n-1} = max x, so that L = {0} and R = {n-1} (eqs.
+ * apx_base, apx_final).  The histogram view takes v = P and, for every t,
+ * w_t = |{x : p_{t-1} < x <= p_t}| (w_0 = |{x : x <= p_0}| = n_0, the first
+ * value's own mass of Phi^first) and the prefix sums of App. E,
+ *   N[t+1] = |{x <= p_t}|,  S[t+1] = sum_{x <= p_t} x,  S2[t+1] = sum_{x <= p_t} x^2,
+ * accumulated entry by entry in binary128.  Every later function then reads
+ * X_{a,b} = {x : p_a < x <= p_b} for a < b, as App. E defines it for P. */
+or_hist *or_hist_new_grid(const float *x, int64_t d, const float *P, int64_t n, int32_t *status) {
+    *status = OR_OK;
+    if (!x || d < 1 || !P || n < 1) { *status = OR_EINVAL; return NULL; }
+    for (int64_t i = 0; i < d; i++)
+        if (!isfinite(x[i])) { *status = OR_ENONFINITE; return NULL; }
+    for (int64_t t = 0; t < n; t++)
+        if (!isfinite(P[t]) || (t > 0 && !(P[t] > P[t - 1]))) { *status = OR_EINVAL; return NULL; }
+    float *xs = (float *)malloc(sizeof(float) * (size_t)d);
+    or_hist *H = (or_hist *)calloc(1, sizeof(or_hist));
+    if (!xs || !H) { free(xs); free(H); *status = OR_ENOMEM; return NULL; }
+    for (int64_t i = 0; i < d; i++) xs[i] = (x[i] == 0.0f) ? 0.0f : x[i];
+    qsort(xs, (size_t)d, sizeof(float), cmp_f32);
+    float p0 = P[0] == 0.0f ? 0.0f : P[0], pl = P[n - 1] == 0.0f ? 0.0f : P[n - 1];
+    if (p0 != xs[0] || pl != xs[d - 1]) { free(xs); free(H); *status = OR_EINVAL; return NULL; }
+    H->d = d; H->p = n;
+    H->v = (float *)malloc(sizeof(float) * (size_t)n);
+    H->w = (int64_t *)malloc(sizeof(int64_t) * (size_t)n);
+    H->N = (int64_t *)malloc(sizeof(int64_t) * (size_t)(n + 1));
+    H->S = (q128 *)malloc(sizeof(q128) * (size_t)(n + 1));
+    H->S2 = (q128 *)malloc(sizeof(q128) * (size_t)(n + 1));
+    if (!H->v || !H->w || !H->N || !H->S || !H->S2) { free(xs); or_hist_free(H); *status = OR_ENOMEM; return NULL; }
+    H->N[0] = 0; H->S[0] = 0; H->S2[0] = 0;
+    int64_t i = 0;
+    q128 sacc = 0, qacc = 0;
+    for (int64_t t = 0; t < n; t++) {
+        float pt = P[t] == 0.0f ? 0.0f : P[t];
+        H->v[t] = pt;
+        int64_t i0 = i;
+        while (i < d && xs[i] <= pt) {
+            q128 xv = (q128)xs[i];
+            sacc += xv;
+            qacc += xv * xv;
+            i++;
+        }
+        H->w[t] = i - i0;
+        H->N[t + 1] = i;
+        H->S[t + 1] = sacc;
+        H->S2[t + 1] = qacc;
+    }
+    free(xs);
+    H->norm2 = (double)H->S2[n];
     return H;
 }
 
