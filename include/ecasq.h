@@ -122,6 +122,23 @@ size_t ecasq_workspace_size_flags(int64_t d, int32_t s, int64_t rows, uint32_t f
 int ecasq_solve(const float *x, int64_t d, const ecasq_params_t *prm, void *ws, size_t ws_bytes,
                 float *Q, ecasq_result_t *res, ecasq_stream_t stream);
 
+/* ecasq_solve with the codebook drawn from a caller-given permissible set P
+ * instead of the unique values of x (Sec. 5 and App. E define the DP and C_P,
+ * U_P, D_P, Phi_P for any sorted P; e.g. a uniform min-max grid or the values of
+ * a narrow float format).  The same search, refinement and results, with every
+ * codebook index referring to P.
+ *   P   device [n] fp32, strictly ascending, P[0] = min x and P[n-1] = max x
+ *       (-0.0 counts as +0.0), so that the sets L and R of eqs. apx_base and
+ *       apx_final are {P[0]} and {P[n-1]}; otherwise ECASQ_EINVAL.
+ *   Q   device [s] output, values of P.  res->p = n.
+ * The DP runs the binary64 reference kernel (the fast kernel's recurrences need
+ * every slab's mass at a candidate value, true only for P = X), so this entry point
+ * is meant for the small sets that make P worth using (p << d).
+ * Workspace: ecasq_workspace_size_grid(d, n, s, flags).  Synchronises `stream`. */
+size_t ecasq_workspace_size_grid(int64_t d, int64_t n, int32_t s, uint32_t flags);
+int ecasq_solve_grid(const float *x, int64_t d, const float *P, int64_t n, const ecasq_params_t *prm, void *ws,
+                     size_t ws_bytes, float *Q, ecasq_result_t *res, ecasq_stream_t stream);
+
 /* One DP pass (Sec. 5) at G <= 8 fixed multipliers, the unit of the search.
  *   lambdas   host [G], vNMSE scale, >= 0
  *   Q_out     device [G * s] (row g: codebook of multiplier g, m_out[g] values)

@@ -19,6 +19,9 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
                    bool exact_s, bool exact_tables, float *costs, bool build_costs);
 size_t resident_costs_bytes(int64_t d);
 int launch_rows_prepare(const float *X, int64_t rows, const RowsData &R, cudaStream_t st);
+int launch_grid_prefix(const float *P, int64_t n, const float *vX, const int64_t *NX, const double *SX,
+                       const double *S2X, int64_t pX, float *v, int64_t *w, int64_t *N, double *S, double *S2,
+                       DevStatus *st, cudaStream_t stream);
 int launch_rows_pass(const RowsPass &A, int nact, int pmax, cudaStream_t st);
 int launch_rows_gather(const RowsData &R, const int32_t *a, const int32_t *m, int64_t rows, int s, float *Q,
                        cudaStream_t st);
@@ -515,25 +518,13 @@ static int64_t read_rescored(void *ws, cudaStream_t st) {
     return h.rescored;
 }
 
-int ecasq_solve(const float *x, int64_t d, const ecasq_params_t *prm, void *ws, size_t ws_bytes, float *Q,
-                ecasq_result_t *res, ecasq_stream_t stream) {
-    if (!x || !Q || d < 1 || d >= ((int64_t)1 << 31) || !params_ok(prm)) return ECASQ_EINVAL;
-    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+// The search, refinement and result of a solve over a prepared histogram view P
+// (unique values of x, or a caller-given candidate set).
+static int solve_prepared(void *ws, const Layout &L, const Prefix &P, int64_t d, double n2, const ecasq_params_t *prm,
+                          float *Q, ecasq_result_t *res, cudaStream_t st) {
     const int s = prm->s;
-    g_timer.on = (prm->flags & ECASQ_TIME_KERNELS) != 0;
-    g_timer.ms = 0.0;
-    g_timer.launches = 0;
-    Layout L;
-    make_layout(d, s, 1, &L);
-    int rc = add_resident_costs(prm->flags, &L);
-    if (rc) return rc;
-    rc = check_ws(ws, ws_bytes, L);
-    if (rc) return rc;
-    int64_t p;
-    double n2;
-    rc = prepare_device(x, d, ws, L, st, &p, &n2);
-    if (rc) return rc;
-    Prefix P = make_prefix(ws, L, p, d);
+    const int64_t p = P.p;
+    int rc;
     double zero3[3] = {0.0, 0.0, 0.0};
     bool costs_built = false;
     if (p == 1) {
@@ -637,6 +628,79 @@ int ecasq_solve(const float *x, int64_t d, const ecasq_params_t *prm, void *ws, 
     if (res) { res->dp_kernel_ms = g_timer.ms; res->dp_kernel_launches = g_timer.launches; }
     g_timer.on = false;
     return status;
+}
+
+int ecasq_solve(const float *x, int64_t d, const ecasq_params_t *prm, void *ws, size_t ws_bytes, float *Q,
+                ecasq_result_t *res, ecasq_stream_t stream) {
+    if (!x || !Q || d < 1 || d >= ((int64_t)1 << 31) || !params_ok(prm)) return ECASQ_EINVAL;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    g_timer.on = (prm->flags & ECASQ_TIME_KERNELS) != 0;
+    g_timer.ms = 0.0;
+    g_timer.launches = 0;
+    Layout L;
+    make_layout(d, prm->s, 1, &L);
+    int rc = add_resident_costs(prm->flags, &L);
+    if (rc) return rc;
+    rc = check_ws(ws, ws_bytes, L);
+    if (rc) return rc;
+    int64_t p;
+    double n2;
+    rc = prepare_device(x, d, ws, L, st, &p, &n2);
+    if (rc) return rc;
+    return solve_prepared(ws, L, make_prefix(ws, L, p, d), d, n2, prm, Q, res, st);
+}
+
+size_t ecasq_workspace_size_grid(int64_t d, int64_t n, int32_t s, uint32_t flags) {
+    if (n < 1 || n >= ((int64_t)1 << 31)) return 0;
+    return ecasq_workspace_size_flags(std::max(d, n), s, 1, flags);
+}
+
+int ecasq_solve_grid(const float *x, int64_t d, const float *Pg, int64_t n, const ecasq_params_t *prm, void *ws,
+                     size_t ws_bytes, float *Q, ecasq_result_t *res, ecasq_stream_t stream) {
+    if (!x || !Q || !Pg || d < 1 || d >= ((int64_t)1 << 31) || n < 1 || n >= ((int64_t)1 << 31) || !params_ok(prm))
+        return ECASQ_EINVAL;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    g_timer.on = (prm->flags & ECASQ_TIME_KERNELS) != 0;
+    g_timer.ms = 0.0;
+    g_timer.launches = 0;
+    const int64_t dmax = std::max(d, n);
+    Layout L;
+    make_layout(dmax, prm->s, 1, &L);
+    L.d = dmax;
+    int rc = add_resident_costs(prm->flags, &L);
+    if (rc) return rc;
+    rc = check_ws(ws, ws_bytes, L);
+    if (rc) return rc;
+    int64_t pX;
+    double n2;
+    rc = prepare_device(x, d, ws, L, st, &pX, &n2);
+    if (rc) return rc;
+    // the unique-value view moves to scratch (the fp64 DP table area), the grid view takes its place
+    char *scr = wsp<char>(ws, L.dp64);
+    float *vX = reinterpret_cast<float *>(scr);
+    int64_t *NX = reinterpret_cast<int64_t *>(scr + align256(4 * (size_t)pX));
+    double *SX = reinterpret_cast<double *>(scr + align256(4 * (size_t)pX) + align256(8 * (size_t)(pX + 1)));
+    double *S2X = SX + 2 * (pX + 1);
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(vX, wsp<float>(ws, L.v), 4 * (size_t)pX, cudaMemcpyDeviceToDevice, st));
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(NX, wsp<int64_t>(ws, L.N), 8 * (size_t)(pX + 1), cudaMemcpyDeviceToDevice, st));
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(SX, wsp<double>(ws, L.S), 16 * (size_t)(pX + 1), cudaMemcpyDeviceToDevice, st));
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(S2X, wsp<double>(ws, L.S2), 16 * (size_t)(pX + 1), cudaMemcpyDeviceToDevice, st));
+    DevStatus *ds = wsp<DevStatus>(ws, L.status);
+    rc = launch_grid_prefix(Pg, n, vX, NX, SX, S2X, pX, wsp<float>(ws, L.v), wsp<int64_t>(ws, L.w),
+                            wsp<int64_t>(ws, L.N), wsp<double>(ws, L.S), wsp<double>(ws, L.S2), ds, st);
+    if (rc) return rc;
+    DevStatus h;
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(&h, ds, sizeof(DevStatus), cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    if (h.range_err) return ECASQ_EINVAL;
+    int64_t pz = n;
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(&ds->p, &pz, sizeof(pz), cudaMemcpyHostToDevice, st));
+    // The fast kernel's fp32 recurrences add one candidate at a time and assume each
+    // slab's mass sits at its right end (true for the unique values of x only); a grid
+    // runs the reference DP (binary64 candidates from the App. E formulas).
+    ecasq_params_t pg = *prm;
+    pg.flags |= ECASQ_DP_REFERENCE;
+    return solve_prepared(ws, L, make_prefix(ws, L, n, d), d, n2, &pg, Q, res, st);
 }
 
 int ecasq_refine(const float *x, int64_t d, float *Q, int32_t m, double lambda, double budget_bits,

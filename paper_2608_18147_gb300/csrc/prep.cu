@@ -354,6 +354,58 @@ int launch_rows_prepare(const float *X, int64_t rows, const RowsData &R, cudaStr
     return ECASQ_OK;
 }
 
+// ------------------------------------------------------------ general P
+// The histogram view over a caller-given candidate set P (Sec. 5, App. E): for
+// every grid point t, u_t = #{unique x <= p_t}; N, S, S2 at t+1 are the unique-value
+// prefix sums at u_t (the sums of all entries x <= p_t), so w_t = #{p_(t-1) < x <= p_t}.
+// Flags st->range_err when P is not strictly ascending and finite or does not start
+// at min x and end at max x (the sets L = {first}, R = {last} of eqs. apx_base and
+// apx_final).  vX, NX, SX, S2X: the unique-value arrays (pX values, packed hi | lo).
+__global__ void k_grid_prefix(const float *__restrict__ P, int64_t n, const float *__restrict__ vX,
+                              const int64_t *__restrict__ NX, const double *__restrict__ SX,
+                              const double *__restrict__ S2X, int64_t pX, float *v, int64_t *w, int64_t *N, double *S,
+                              double *S2, DevStatus *st) {
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < n; t += stride) {
+        float pt = P[t];
+        if (pt == 0.0f) pt = 0.0f;
+        bool bad = !isfinite(pt);
+        if (t > 0 && !(P[t] > P[t - 1])) bad = true;
+        if (t == 0 && pt != vX[0]) bad = true;
+        if (t == n - 1 && pt != vX[pX - 1]) bad = true;
+        if (bad) st->range_err = 1;
+        // u = #{unique values <= pt} (binary search)
+        int64_t lo = 0, hi = pX;
+        while (lo < hi) {
+            int64_t mid = (lo + hi) >> 1;
+            if (vX[mid] <= pt) lo = mid + 1; else hi = mid;
+        }
+        v[t] = pt;
+        N[t + 1] = NX[lo];
+        S[t + 1] = SX[lo]; S[n + 1 + t + 1] = SX[pX + 1 + lo];
+        S2[t + 1] = S2X[lo]; S2[n + 1 + t + 1] = S2X[pX + 1 + lo];
+        if (t == 0) { N[0] = 0; S[0] = 0.0; S[n + 1] = 0.0; S2[0] = 0.0; S2[n + 1] = 0.0; }
+    }
+}
+
+__global__ void k_grid_weights(const int64_t *N, int64_t n, int64_t *w) {
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < n; t += stride) w[t] = N[t + 1] - N[t];
+}
+
+int launch_grid_prefix(const float *P, int64_t n, const float *vX, const int64_t *NX, const double *SX,
+                       const double *S2X, int64_t pX, float *v, int64_t *w, int64_t *N, double *S, double *S2,
+                       DevStatus *st, cudaStream_t stream) {
+    const unsigned blocks = (unsigned)std::min<int64_t>(cdiv(n, 256), 4096);
+    note_launch();
+    k_grid_prefix<<<blocks, 256, 0, stream>>>(P, n, vX, NX, SX, S2X, pX, v, w, N, S, S2, st);
+    ECASQ_LAUNCH_CHECK();
+    note_launch();
+    k_grid_weights<<<blocks, 256, 0, stream>>>(N, n, w);
+    ECASQ_LAUNCH_CHECK();
+    return ECASQ_OK;
+}
+
 int prepare_device(const float *x, int64_t d, void *ws, const Layout &L, cudaStream_t stream, int64_t *p_host,
                    double *norm2_host) {
     DevStatus *st = wsp<DevStatus>(ws, L.status);

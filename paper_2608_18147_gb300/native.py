@@ -76,6 +76,8 @@ def lib():
             "ecasq_workspace_size": (sz, [i64, i32, i64]),
             "ecasq_workspace_size_flags": (sz, [i64, i32, i64, u32]),
             "ecasq_solve": (C.c_int, [vp, i64, PP, vp, sz, vp, PR, vp]),
+            "ecasq_solve_grid": (C.c_int, [vp, i64, vp, i64, PP, vp, sz, vp, PR, vp]),
+            "ecasq_workspace_size_grid": (sz, [i64, i64, i32, u32]),
             "ecasq_dp_pass": (C.c_int, [vp, i64, i32, pd, i32, u32, vp, sz, vp, pi32, pd, vp]),
             "ecasq_dp_tables": (C.c_int, [vp, sz, i32, vp, vp, pi64, vp]),
             "ecasq_refine": (C.c_int, [vp, i64, vp, i32, dbl, dbl, i32, dbl, u32, vp, sz, PR, vp]),
@@ -99,7 +101,7 @@ def exported_symbols():
     L = lib()
     names = []
     for name in ("ecasq_version", "ecasq_strerror", "ecasq_workspace_size", "ecasq_workspace_size_flags",
-                 "ecasq_solve", "ecasq_dp_pass",
+                 "ecasq_solve", "ecasq_solve_grid", "ecasq_workspace_size_grid", "ecasq_dp_pass",
                  "ecasq_dp_tables", "ecasq_refine", "ecasq_evaluate", "ecasq_quantize", "ecasq_quantize_noalloc",
                  "ecasq_solve_batched",
                  "ecasq_prepare", "ecasq_kernel_launches"):
@@ -190,6 +192,35 @@ def ecasq_solve(x, s, budget_bits=0.0, lambda_=-1.0, ws=None, **kw):
     rc = lib().ecasq_solve(_ptr(x), d, C.byref(prm), _ptr(ws), ws.numel(), _ptr(Q), C.byref(res), _stream())
     _check(rc, "ecasq_solve", ok=(OK, EINFEASIBLE))
     return Q[:res.m].clone(), res.as_dict()
+
+
+def ecasq_solve_grid(x, P, s, budget_bits=0.0, lambda_=-1.0, ws=None, **kw):
+    """Budgeted solve with the codebook drawn from the candidate set P (ascending, spanning x)."""
+    torch = _torch()
+    x = _dev_f32(x)
+    P = _dev_f32(P)
+    d, n = x.numel(), P.numel()
+    if ws is None:
+        nb = int(lib().ecasq_workspace_size_grid(d, n, int(s), int(kw.get("flags", 0))))
+        if nb == 0:
+            raise EcasqError(EINVAL, "ecasq_workspace_size_grid")
+        ws = torch.empty(nb, dtype=torch.uint8, device="cuda")
+    prm = make_params(s, budget_bits, lambda_, **kw)
+    Q = torch.zeros(s, dtype=torch.float32, device="cuda")
+    res = Result()
+    rc = lib().ecasq_solve_grid(_ptr(x), d, _ptr(P), n, C.byref(prm), _ptr(ws), ws.numel(), _ptr(Q), C.byref(res),
+                                _stream())
+    _check(rc, "ecasq_solve_grid", ok=(OK, EINFEASIBLE))
+    return Q[:res.m].clone(), res.as_dict()
+
+
+def uniform_grid(x, n):
+    """n equally spaced fp32 candidates from min x to max x, both endpoints exact."""
+    x = np.asarray(x, dtype=np.float32)
+    lo, hi = float(x.min()), float(x.max())
+    g = np.linspace(lo, hi, n).astype(np.float32)
+    g[0], g[-1] = np.float32(lo), np.float32(hi)
+    return np.unique(g)
 
 
 def ecasq_dp_pass(x, s, lambdas, flags=0, ws=None):

@@ -1,0 +1,66 @@
+"""ecasq_solve_grid: the codebook drawn from a caller-given permissible set P
+(Sec. 5, App. E for general P) against the oracle on the same P (pytest -m gpu)."""
+import numpy as np
+import pytest
+
+from paper_2608_18147_gb300 import workloads
+
+pytestmark = pytest.mark.gpu
+
+MET_RTOL = 1e-9
+
+
+@pytest.fixture(scope="module")
+def E():
+    import torch
+    assert torch.cuda.is_available(), "these tests need a CUDA GPU"
+    import paper_2608_18147_gb300 as E
+    E.lib()
+    return E
+
+
+def _check(res, o, Q):
+    assert res["status"] == o["status"]
+    assert res["lambda"] == o["lam"]
+    np.testing.assert_array_equal(Q.cpu().numpy(), o["Q"])
+    np.testing.assert_allclose([res["mse"], res["h_surrogate"], res["h_exact"]],
+                               [o["mse"], o["h_surrogate"], o["h_exact"]], rtol=MET_RTOL)
+
+
+def test_grid_of_unique_values_equals_plain_solve(E):
+    x = workloads.signed_lognormal(3000, 1)
+    Q1, r1 = E.ecasq_solve(x, 8, budget_bits=2.0)
+    Q2, r2 = E.ecasq_solve_grid(x, np.unique(x), 8, budget_bits=2.0)
+    np.testing.assert_array_equal(Q1.cpu().numpy(), Q2.cpu().numpy())
+    for k in ("lambda", "mse", "h_surrogate", "h_exact", "p", "passes"):
+        assert r1[k] == r2[k], k
+
+
+@pytest.mark.parametrize("n,refine", [(256, 0), (256, 5), (1024, 0), (97, 0)])
+def test_uniform_grid_matches_oracle(E, oracle_mod, n, refine):
+    x = workloads.make("lognormal_d16384_s16")
+    g = E.uniform_grid(x, n)
+    Q, res = E.ecasq_solve_grid(x, g, 16, budget_bits=2.0, refine_max_rounds=refine, refine_rel_tol=1e-9)
+    o = oracle_mod.solve_budget(x, 16, 2.0, grid=g, refine_rounds=refine, refine_tol=1e-9)
+    assert res["p"] == g.size
+    _check(res, o, Q)
+    assert np.all(np.isin(Q.cpu().numpy(), g))
+
+
+def test_grid_larger_than_x_and_fast_kernel_sizes(E, oracle_mod):
+    x = workloads.student_t(200, 3, scale=1.0)          # n > d
+    g = E.uniform_grid(x, 300)
+    Q, res = E.ecasq_solve_grid(x, g, 6, budget_bits=1.5)
+    _check(res, oracle_mod.solve_budget(x, 6, 1.5, grid=g), Q)
+    x = workloads.student_t(20000, 4, scale=1.0)        # n = 4096: the fast kernel, resident costs
+    g = E.uniform_grid(x, 4096)
+    Q, res = E.ecasq_solve_grid(x, g, 8, budget_bits=2.5, flags=E.RESIDENT_COSTS)
+    _check(res, oracle_mod.solve_budget(x, 8, 2.5, grid=g), Q)
+
+
+def test_grid_that_does_not_span_x_is_rejected(E):
+    x = np.array([1.0, 2.0, 3.0, 2.5], np.float32)
+    for P in ([1.5, 3.0], [1.0, 2.5], [1.0, 3.0, 2.0], [1.0, 1.0, 3.0], [1.0, np.inf, 3.0]):
+        with pytest.raises(E.EcasqError) as ei:
+            E.ecasq_solve_grid(x, np.array(P, np.float32), 4, budget_bits=1.0)
+        assert ei.value.code == E.native.EINVAL
