@@ -58,6 +58,7 @@ def _load():
             "or_hist_new_grid": (P, [pf, i64, pf, i64, pi32]),
             "or_hist_free": (None, [P]),
             "or_hist_info": (None, [P, pi64, pi64, pd]),
+            "or_hist_ends": (None, [P, pi64, pi64]),
             "or_hist_arrays": (None, [P, pf, pi64, pi64, pd, pd, pd, pd]),
             "or_hist_cache": (i32, [P]),
             "or_pair": (None, [P, i64, i64, pd]),
@@ -70,6 +71,7 @@ def _load():
             "or_asq_dp": (i32, [P, i32, pd]),
             "or_opt_dp": (i32, [P, i32, dbl, i32, pd, pi64, pi32]),
             "or_brute": (i32, [pf, i64, i32, dbl, dbl, pd, pi64]),
+            "or_brute_grid": (i32, [pf, i64, pf, i64, i32, dbl, dbl, pd, pi64]),
             "or_midpoints7": (None, [dbl, dbl, pd]),
             "or_search": (i32, [P, i32, dbl, dbl, dbl, i32, i32, pi64, pi32, pd, pd, i32, pi32]),
             "or_refine": (i32, [P, pi64, i32, dbl, dbl, i32, i32, dbl, pi32, pd]),
@@ -108,8 +110,9 @@ class Hist:
     """Sorted weighted histogram of x with App. E prefix sums (Sec. 2, App. E)."""
 
     def __init__(self, x, grid=None):
-        """grid: optional candidate set P (ascending fp32, first = min x, last = max x);
-        by default P = the unique values of x."""
+        """grid: optional candidate set P (ascending fp32, first <= min x, last >= max x);
+        by default P = the unique values of x.  nL, nR: sizes of the first- and
+        last-value sets L = {0..nL-1}, R = {p-nR..p-1} of Sec. 5."""
         lib = _load()
         self._x = _f32(x)
         st = C.c_int32(0)
@@ -124,6 +127,9 @@ class Hist:
         d, p, n2 = C.c_int64(), C.c_int64(), C.c_double()
         lib.or_hist_info(self._h, C.byref(d), C.byref(p), C.byref(n2))
         self.d, self.p, self.norm2 = d.value, p.value, n2.value
+        nL, nR = C.c_int64(), C.c_int64()
+        lib.or_hist_ends(self._h, C.byref(nL), C.byref(nR))
+        self.nL, self.nR = nL.value, nR.value
 
     def __del__(self):
         h = getattr(self, "_h", None)
@@ -270,6 +276,21 @@ def brute(x, s, lam_prime, budget):
                           _ptr(out, C.c_double), _ptr(masks, C.c_int64))
     if st != OK:
         raise OracleError(st, "or_brute")
+    return dict(surrogate=out[0], true=out[1], mse_surr_budget=out[2], mse_opt_budget_minus1=out[3],
+                hx_of_surr_budget=out[4], mse_min=out[5], masks=masks.copy())
+
+
+def brute_grid(x, grid, s, lam_prime, budget):
+    """Exhaustive search over spanning codebooks drawn from the permissible set `grid`
+    (at most 16 values); masks are bitmasks over the grid."""
+    x = _f32(x)
+    g = _f32(grid)
+    out = np.empty(6, np.float64)
+    masks = np.empty(4, np.int64)
+    st = _load().or_brute_grid(_ptr(x, C.c_float), x.size, _ptr(g, C.c_float), g.size, int(s),
+                               float(lam_prime), float(budget), _ptr(out, C.c_double), _ptr(masks, C.c_int64))
+    if st != OK:
+        raise OracleError(st, "or_brute_grid")
     return dict(surrogate=out[0], true=out[1], mse_surr_budget=out[2], mse_opt_budget_minus1=out[3],
                 hx_of_surr_budget=out[4], mse_min=out[5], masks=masks.copy())
 

@@ -18,7 +18,8 @@
  * Functions and the passages they follow:
  *   or_hist_new      Sec. 2 (sorted copy, weighted histogram), App. E (prefix sums)
  *   or_hist_new_grid Sec. 5 / App. E for a general permissible set P: the same
- *                    histogram view with P as the candidate values
+ *                    histogram view with P as the candidate values, first-value
+ *                    set L = {a : p_a <= x_1} and last-value set R = {b : p_b >= x_d}
  *   pair_q           App. E: U_P, D_P, C_P from prefix differences
  *   h, or_phi        Sec. 4 (h), Sec. 5 (Phi, Phi^first)
  *   or_apx_dp        Sec. 5, eqs. apx_base / apx_rec / apx_final
@@ -27,6 +28,7 @@
  *   or_asq_dp        Sec. 2, eq. asqdp (ZipML/QUIVER recurrence, lambda = 0)
  *   or_opt_dp        Sec. 4 with the boundary conventions of App. E (naive O(s p^3))
  *   or_brute         exhaustive enumeration of spanning codebooks drawn from X
+ *   or_brute_grid    the same over codebooks drawn from a permissible set P
  *   or_search        Sec. 3 / Sec. 5: tune lambda for a budget b (schedule below)
  *   or_refine        Sec. 6: three-colour refinement
  *   or_quantize      Sec. 2: unbiased stochastic rounding, Sec. 1 entropy
@@ -73,6 +75,7 @@ typedef struct or_hist {
     q128 *S;       /* S[t] = sum_{r<t} w_r v_r */
     q128 *S2;      /* S2[t] = sum_{r<t} w_r v_r^2 */
     double norm2;  /* ||X||^2 */
+    int64_t nL, nR;  /* L = {0..nL-1}, R = {p-nR..p-1} (Sec. 5); 1, 1 when P = X */
     /* optional memo of C and Phi for every pair k < j (upper triangle) */
     double *tC, *tPhi;
 } or_hist;
@@ -133,14 +136,18 @@ or_hist *or_hist_new(const float *x, int64_t d, int32_t *status) {
         H->S2[t + 1] = H->S2[t] + ww * vv * vv;
     }
     H->norm2 = (double)H->S2[p];
+    H->nL = 1;
+    H->nR = 1;
     return H;
 }
 
 /* General permissible set P (Sec. 5, App. E): candidate values p_0 < ... < p_{n-1}
- * with p_0 = min x and p_{n-1} = max x, so that L = {0} and R = {n-1} (eqs.
- * apx_base, apx_final).  The histogram view takes v = P and, for every t,
- * w_t = |{x : p_{t-1} < x <= p_t}| (w_0 = |{x : x <= p_0}| = n_0, the first
- * value's own mass of Phi^first) and the prefix sums of App. E,
+ * with p_0 <= min x and p_{n-1} >= max x (App. E: otherwise no unbiased quantizer
+ * drawn from P spans X).  The first value may be any a in L = {a : p_a <= x_1} and
+ * the last any b in R = {b : p_b >= x_d} (eqs. apx_base, apx_final); both are runs
+ * of indices, L = {0..nL-1}, R = {n-nR..n-1}.  The histogram view takes v = P and,
+ * for every t, w_t = |{x : p_{t-1} < x <= p_t}| (for a in L this is n_a =
+ * |{x : x = p_a}|, the first value's own mass of Phi^first) and the prefix sums of App. E,
  *   N[t+1] = |{x <= p_t}|,  S[t+1] = sum_{x <= p_t} x,  S2[t+1] = sum_{x <= p_t} x^2,
  * accumulated entry by entry in binary128.  Every later function then reads
  * X_{a,b} = {x : p_a < x <= p_b} for a < b, as App. E defines it for P. */
@@ -157,7 +164,14 @@ or_hist *or_hist_new_grid(const float *x, int64_t d, const float *P, int64_t n, 
     for (int64_t i = 0; i < d; i++) xs[i] = (x[i] == 0.0f) ? 0.0f : x[i];
     qsort(xs, (size_t)d, sizeof(float), cmp_f32);
     float p0 = P[0] == 0.0f ? 0.0f : P[0], pl = P[n - 1] == 0.0f ? 0.0f : P[n - 1];
-    if (p0 != xs[0] || pl != xs[d - 1]) { free(xs); free(H); *status = OR_EINVAL; return NULL; }
+    if (!(p0 <= xs[0]) || !(pl >= xs[d - 1])) { free(xs); free(H); *status = OR_EINVAL; return NULL; }
+    H->nL = 0;
+    H->nR = 0;
+    for (int64_t t = 0; t < n; t++) {
+        float pt = P[t] == 0.0f ? 0.0f : P[t];
+        H->nL += (pt <= xs[0]);
+        H->nR += (pt >= xs[d - 1]);
+    }
     H->d = d; H->p = n;
     H->v = (float *)malloc(sizeof(float) * (size_t)n);
     H->w = (int64_t *)malloc(sizeof(int64_t) * (size_t)n);
@@ -190,6 +204,10 @@ or_hist *or_hist_new_grid(const float *x, int64_t d, const float *P, int64_t n, 
 
 void or_hist_info(const or_hist *H, int64_t *d, int64_t *p, double *norm2) {
     *d = H->d; *p = H->p; *norm2 = H->norm2;
+}
+
+void or_hist_ends(const or_hist *H, int64_t *nL, int64_t *nR) {
+    *nL = H->nL; *nR = H->nR;
 }
 
 /* Copy out the histogram and the prefix sums (binary128 split as hi + lo). */
@@ -228,17 +246,18 @@ void or_pair(const or_hist *H, int64_t k, int64_t j, double *out3) {
     pair_q(H, k, j, &out3[0], &out3[1], &out3[2]);
 }
 
-/* Sec. 5: Phi = h(U/d) + h(D/d);  Phi^first = h(U/d) + h((D + n_a)/d). */
-static double phi_of(const or_hist *H, double U, double D, int first) {
+/* Sec. 5: Phi = h(U/d) + h(D/d);  Phi^first[a, .] = h(U/d) + h((D + n_a)/d).
+ * first_a < 0: an ordinary interval; otherwise the first interval, starting at a. */
+static double phi_of(const or_hist *H, double U, double D, int64_t first_a) {
     double dd = (double)H->d;
-    double Dm = first ? D + (double)H->w[0] : D;
+    double Dm = first_a >= 0 ? D + (double)H->w[first_a] : D;
     return h(U / dd) + h(Dm / dd);
 }
 
 double or_phi(const or_hist *H, int64_t k, int64_t j, int32_t first) {
     double C, U, D;
     pair_q(H, k, j, &C, &U, &D);
-    return phi_of(H, U, D, first);
+    return phi_of(H, U, D, first ? k : -1);
 }
 
 /* Memoise C and Phi for every pair (only practical for p up to ~2e4). */
@@ -256,7 +275,7 @@ int32_t or_hist_cache(or_hist *H) {
             double C, U, D;
             pair_q(H, k, j, &C, &U, &D);
             H->tC[tri(k, j)] = C;
-            H->tPhi[tri(k, j)] = phi_of(H, U, D, 0);
+            H->tPhi[tri(k, j)] = phi_of(H, U, D, -1);
         }
     return OR_OK;
 }
@@ -265,21 +284,21 @@ static inline void cphi(const or_hist *H, int64_t k, int64_t j, double *C, doubl
     if (H->tC) { *C = H->tC[tri(k, j)]; *Phi = H->tPhi[tri(k, j)]; return; }
     double U, D;
     pair_q(H, k, j, C, &U, &D);
-    *Phi = phi_of(H, U, D, 0);
+    *Phi = phi_of(H, U, D, -1);
 }
 
 /* -------------------------------------------------------- evaluation */
 
-/* Metrics of a codebook given as ascending unique-value indices a[0..m-1]
- * with a[0] = 0 and a[m-1] = p-1 (Q spans X, Q subset of X):
+/* Metrics of a codebook given as ascending candidate indices a[0..m-1]
+ * with a[0] in L and a[m-1] in R (Q spans X, Q subset of P):
  *   out[0] MSE            = sum_r C[a_r, a_{r+1}]                     (Sec. 2)
  *   out[1] H(I,B)         = Phi^first[a_0,a_1] + sum_{r>=1} Phi[a_r,a_{r+1}] (eq. apx_additive_entropy)
  *   out[2] H(Xhat)        = sum_r h(f_r / d), f_r = U[a_{r-1},a_r] + D[a_r,a_{r+1}],
- *                           f_0 = w_0 + D[a_0,a_1], f_{m-1} = U[a_{m-2},a_{m-1}] (Sec. 3, Sec. 5)
+ *                           f_0 = n_{a_0} + D[a_0,a_1], f_{m-1} = U[a_{m-2},a_{m-1}] (Sec. 3, Sec. 5)
  */
 int32_t or_eval_idx(const or_hist *H, const int64_t *a, int32_t m, double *out) {
     double dd = (double)H->d;
-    if (m < 1 || a[0] != 0 || a[m - 1] != H->p - 1) return OR_EINVAL;
+    if (m < 1 || a[0] < 0 || a[0] >= H->nL || a[m - 1] < H->p - H->nR || a[m - 1] >= H->p) return OR_EINVAL;
     for (int32_t r = 1; r < m; r++) if (a[r] <= a[r - 1]) return OR_EINVAL;
     if (m == 1) { out[0] = 0.0; out[1] = 0.0; out[2] = 0.0; return OR_OK; }
     double mse = 0.0, hs = 0.0, hx = 0.0;
@@ -288,8 +307,8 @@ int32_t or_eval_idx(const or_hist *H, const int64_t *a, int32_t m, double *out) 
         double C, U, D;
         pair_q(H, a[r], a[r + 1], &C, &U, &D);
         mse += C;
-        hs += phi_of(H, U, D, r == 0);
-        double f = (r == 0) ? (double)H->w[0] + D : prevU + D;
+        hs += phi_of(H, U, D, r == 0 ? a[0] : -1);
+        double f = (r == 0) ? (double)H->w[a[0]] + D : prevU + D;
         hx += h(f / dd);
         prevU = U;
     }
@@ -340,12 +359,13 @@ int32_t or_eval_direct(const float *x, int64_t d, const double *Q, int32_t m, do
 
 /* ------------------------------------------------------ approximate DP */
 
-/* Sec. 5, for P = X (L = {0}, R = {p-1}), lambda' = lam_prime:
- *   dp(2, j) = C[0, j] + lambda' Phi^first[0, j]                   (eq. apx_base)
+/* Sec. 5, lambda' = lam_prime, L = {0..nL-1}, R = {p-nR..p-1} ({0} and {p-1} when P = X):
+ *   dp(2, j) = min_{a in L, a<j} C[a, j] + lambda' Phi^first[a, j]  (eq. apx_base)
  *   dp(i, j) = min_{k<j} dp(i-1, k) + C[k, j] + lambda' Phi[k, j]  (eq. apx_rec)
- *   answer   = min_{2<=i<=s} dp(i, p-1)  (or i = s only)           (eq. apx_final)
+ *   answer   = min_{2<=i<=s} min_{j in R} dp(i, j)  (or i = s only) (eq. apx_final)
  * Each candidate is formed as dp(i-1,k) + (C + lambda' Phi); the argmin is the
- * lowest k among exact binary64 minima; the final layer is the smallest i.
+ * lowest k (lowest a in the base layer) among exact binary64 minima; the final
+ * selection is the smallest i, then the smallest j.
  * Arrays (optional, row-major (s+1) x p, rows 0 and 1 unused):
  *   dp (+inf where undefined), bp (-1 where undefined), margin = relative gap
  *   between the best and second-best candidate ((2nd - best)/best).
@@ -367,10 +387,16 @@ int32_t or_apx_dp(const or_hist *H, int32_t s, double lam_prime, int32_t exact_s
     for (size_t t = 0; t < rows * (size_t)p; t++) { dp[t] = INFINITY; bp[t] = -1; mg[t] = INFINITY; }
     /* base layer */
     for (int64_t j = 1; j < p; j++) {
-        double C, U, D;
-        pair_q(H, 0, j, &C, &U, &D);
-        dp[2 * (size_t)p + (size_t)j] = C + lam_prime * phi_of(H, U, D, 1);
-        bp[2 * (size_t)p + (size_t)j] = 0;
+        double best = INFINITY;
+        int64_t arg = -1;
+        for (int64_t a = 0; a < H->nL && a < j; a++) {
+            double C, U, D;
+            pair_q(H, a, j, &C, &U, &D);
+            double c = C + lam_prime * phi_of(H, U, D, a);
+            if (c < best) { best = c; arg = a; }
+        }
+        dp[2 * (size_t)p + (size_t)j] = best;
+        bp[2 * (size_t)p + (size_t)j] = (int32_t)arg;
     }
     /* recurrence layers */
     for (int32_t i = 3; i <= s; i++) {
@@ -396,21 +422,23 @@ int32_t or_apx_dp(const or_hist *H, int32_t s, double lam_prime, int32_t exact_s
     }
     /* final selection */
     int32_t istar = -1;
+    int64_t jstar = -1;
     double best = INFINITY;
     int32_t ilo = exact_s ? s : 2;
-    for (int32_t i = ilo; i <= s; i++) {
-        double v = dp[(size_t)i * (size_t)p + (size_t)(p - 1)];
-        if (v < best) { best = v; istar = i; }
-    }
+    for (int32_t i = ilo; i <= s; i++)
+        for (int64_t jr = p - H->nR; jr < p; jr++) {
+            double v = dp[(size_t)i * (size_t)p + (size_t)jr];
+            if (v < best) { best = v; istar = i; jstar = jr; }
+        }
     if (istar < 0) { free(dp); free(bp); free(mg); return OR_EINFEASIBLE; }
     /* traceback */
-    int64_t j = p - 1;
+    int64_t j = jstar;
     Q_idx[istar - 1] = j;
     for (int32_t i = istar; i >= 3; i--) {
         j = bp[(size_t)i * (size_t)p + (size_t)j];
         Q_idx[i - 2] = j;
     }
-    Q_idx[0] = 0;
+    Q_idx[0] = bp[2 * (size_t)p + (size_t)j];
     *m_out = istar;
     *best_out = best;
     if (dp_out) memcpy(dp_out, dp, sizeof(double) * rows * (size_t)p);
@@ -441,8 +469,8 @@ void or_dp_decision(const or_hist *H, const double *prev, int32_t i, int64_t j, 
 double or_dp_candidate(const or_hist *H, double prev_k, int64_t k, int64_t j, double lam_prime, int32_t first) {
     double C, U, D;
     pair_q(H, k, j, &C, &U, &D);
-    if (first) return C + lam_prime * phi_of(H, U, D, 1);
-    return prev_k + (C + lam_prime * phi_of(H, U, D, 0));
+    if (first) return C + lam_prime * phi_of(H, U, D, k);
+    return prev_k + (C + lam_prime * phi_of(H, U, D, -1));
 }
 
 /* ------------------------------------------------------------- ASQ DP */
@@ -482,10 +510,11 @@ int32_t or_asq_dp(const or_hist *H, int32_t s, double *best_out) {
 
 /* ---------------------------------------------------------- optimal DP */
 
-/* Sec. 4 with App. E's conventions, P = X, naive O(s p^3):
- *   dp(2, 0, j)  = C[0, j] + lambda' h((w_0 + D[0, j]) / d)
+/* Sec. 4 with App. E's conventions (L = {0..nL-1}, R = {p-nR..p-1}), naive O(s p^3):
+ *   dp(2, a, j)  = C[a, j] + lambda' h((n_a + D[a, j]) / d),  a in L, a < j
  *   dp(i, l, j)  = C[l, j] + min_{k<l} dp(i-1, k, l) + lambda' h((U[k,l] + D[l,j]) / d),  i >= 3
- *   answer       = min_{2<=i<=s} min_{l<p-1} dp(i, l, p-1) + lambda' h(U[l, p-1] / d)
+ *   answer       = min_{2<=i<=s} min_{j in R} min_{l<j} dp(i, l, j) + lambda' h(U[l, j] / d)
+ * Ties: lowest k; at the answer the smallest i, then j, then l.
  * The traced codebook goes to Q_idx / m.  Memory s p^2 doubles. */
 int32_t or_opt_dp(const or_hist *H, int32_t s, double lam_prime, int32_t exact_s,
                   double *best_out, int64_t *Q_idx, int32_t *m_out) {
@@ -509,8 +538,9 @@ int32_t or_opt_dp(const or_hist *H, int32_t s, double lam_prime, int32_t exact_s
 #define DPO(i, l, j) dp[((size_t)(i) * (size_t)p + (size_t)(l)) * (size_t)p + (size_t)(j)]
 #define BKO(i, l, j) bk[((size_t)(i) * (size_t)p + (size_t)(l)) * (size_t)p + (size_t)(j)]
     for (size_t t = 0; t < pp * (size_t)(s + 1); t++) { dp[t] = INFINITY; bk[t] = -1; }
-    for (int64_t j = 1; j < p; j++)
-        DPO(2, 0, j) = C[(size_t)j] + lam_prime * h(((double)H->w[0] + D[(size_t)j]) / dd);
+    for (int64_t a = 0; a < H->nL; a++)
+        for (int64_t j = a + 1; j < p; j++)
+            DPO(2, a, j) = C[(size_t)a * p + j] + lam_prime * h(((double)H->w[a] + D[(size_t)a * p + j]) / dd);
     for (int32_t i = 3; i <= s; i++) {
 #pragma omp parallel for schedule(dynamic, 4)
         for (int64_t l = 1; l < p; l++)
@@ -528,24 +558,25 @@ int32_t or_opt_dp(const or_hist *H, int32_t s, double lam_prime, int32_t exact_s
     }
     double best = INFINITY;
     int32_t bi = -1;
-    int64_t bl = -1;
+    int64_t bl = -1, bj = -1;
     for (int32_t i = exact_s ? s : 2; i <= s; i++)
-        for (int64_t l = 0; l < p - 1; l++) {
-            double v = DPO(i, l, p - 1);
-            if (!(v < INFINITY)) continue;
-            double c = v + lam_prime * h(U[(size_t)l * p + (size_t)(p - 1)] / dd);
-            if (c < best) { best = c; bi = i; bl = l; }
-        }
+        for (int64_t jr = p - H->nR; jr < p; jr++)
+            for (int64_t l = 0; l < jr; l++) {
+                double v = DPO(i, l, jr);
+                if (!(v < INFINITY)) continue;
+                double c = v + lam_prime * h(U[(size_t)l * p + (size_t)jr] / dd);
+                if (c < best) { best = c; bi = i; bl = l; bj = jr; }
+            }
     if (bi < 0) { free(U); free(D); free(C); free(dp); free(bk); return OR_EINFEASIBLE; }
     /* traceback: state (i, l, j) -> (i-1, k, l) */
-    int64_t l = bl, j = p - 1;
+    int64_t l = bl, j = bj;
     Q_idx[bi - 1] = j;
     for (int32_t i = bi; i >= 3; i--) {
         Q_idx[i - 2] = l;
         int64_t k = BKO(i, l, j);
         j = l; l = k;
     }
-    Q_idx[0] = 0;
+    Q_idx[0] = l;
     *m_out = bi;
     *best_out = best;
 #undef DPO
@@ -594,6 +625,39 @@ int32_t or_brute(const float *x, int64_t d, int32_t s, double lam_prime, double 
     }
     free(Q);
     or_hist_free(H);
+    return OR_OK;
+}
+
+/* The enumeration of or_brute over codebooks drawn from a permissible set P
+ * (ascending, n <= 16): every subset of P with 2 <= |Q| <= s, Q[0] <= min x and
+ * Q[last] >= max x (Sec. 5: q_1 <= x_1, q_t >= x_d), scored with the per-entry
+ * definitions.  Outputs as or_brute; masks are bitmasks over all n values of P. */
+int32_t or_brute_grid(const float *x, int64_t d, const float *P, int64_t n, int32_t s, double lam_prime,
+                      double budget, double *out, int64_t *masks) {
+    if (!x || d < 1 || !P || n < 1 || n > 16 || s < 2) return OR_EINVAL;
+    float xmin = x[0], xmax = x[0];
+    for (int64_t i = 1; i < d; i++) {
+        if (x[i] < xmin) xmin = x[i];
+        if (x[i] > xmax) xmax = x[i];
+    }
+    double Q[16];
+    for (int r = 0; r < 6; r++) out[r] = INFINITY;
+    for (int r = 0; r < 4; r++) masks[r] = -1;
+    out[4] = NAN;
+    for (int64_t mask = 1; mask < ((int64_t)1 << n); mask++) {
+        int32_t m = 0;
+        for (int64_t t = 0; t < n; t++)
+            if (mask >> t & 1) Q[m++] = (double)P[t];
+        if (m < 2 || m > s || !(Q[0] <= (double)xmin) || !(Q[m - 1] >= (double)xmax)) continue;
+        double ev[3];
+        if (or_eval_direct(x, d, Q, m, ev) != OR_OK) continue;
+        double js = ev[0] + lam_prime * ev[1], jt = ev[0] + lam_prime * ev[2];
+        if (js < out[0]) { out[0] = js; masks[0] = mask; }
+        if (jt < out[1]) { out[1] = jt; masks[1] = mask; }
+        if (ev[1] <= budget && ev[0] < out[2]) { out[2] = ev[0]; masks[2] = mask; out[4] = ev[2]; }
+        if (ev[2] <= budget - 1.0 && ev[0] < out[3]) { out[3] = ev[0]; masks[3] = mask; }
+        if (ev[0] < out[5]) out[5] = ev[0];
+    }
     return OR_OK;
 }
 
@@ -716,7 +780,7 @@ static double local_obj(const or_hist *H, const int64_t *a, int32_t m, int32_t l
     pair_q(H, L, c, &C1, &U1, &D1);
     pair_q(H, c, R, &C2, &U2, &D2);
     double fl;
-    if (l - 1 == 0) fl = (double)H->w[0] + D1;
+    if (l - 1 == 0) fl = (double)H->w[a[0]] + D1;
     else { double Cx, Ux, Dx; pair_q(H, a[l - 2], L, &Cx, &Ux, &Dx); fl = Ux + D1; }
     double fm = U1 + D2;
     double fr;
