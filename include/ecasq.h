@@ -127,10 +127,14 @@ int ecasq_solve(const float *x, int64_t d, const ecasq_params_t *prm, void *ws, 
  * U_P, D_P, Phi_P for any sorted P; e.g. a uniform min-max grid or the values of
  * a narrow float format).  The same search, refinement and results, with every
  * codebook index referring to P.
- *   P   device [n] fp32, strictly ascending, P[0] = min x and P[n-1] = max x
- *       (-0.0 counts as +0.0), so that the sets L and R of eqs. apx_base and
- *       apx_final are {P[0]} and {P[n-1]}; otherwise ECASQ_EINVAL.
+ *   P   device [n] fp32, finite, strictly ascending, P[0] <= min x and
+ *       P[n-1] >= max x (-0.0 counts as +0.0); otherwise ECASQ_EINVAL.  The first
+ *       codebook value ranges over L = {P[a] <= min x} (eq. apx_base) and the last
+ *       over R = {P[b] >= max x} (eq. apx_final); ties go to the smallest size,
+ *       then the smallest last index, then the lowest first index.
  *   Q   device [s] output, values of P.  res->p = n.
+ * Refinement moves interior values only; the first and last stay where the DP
+ * put them.
  * The DP runs the binary64 reference kernel (the fast kernel's recurrences need
  * every slab's mass at a candidate value, true only for P = X), so this entry point
  * is meant for the small sets that make P worth using (p << d).

@@ -692,15 +692,18 @@ int ecasq_solve_grid(const float *x, int64_t d, const float *Pg, int64_t n, cons
     DevStatus h;
     ECASQ_CUDA_TRY(cudaMemcpyAsync(&h, ds, sizeof(DevStatus), cudaMemcpyDeviceToHost, st));
     ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
-    if (h.range_err) return ECASQ_EINVAL;
+    if (h.range_err || h.grid_nL < 1 || h.grid_nR < 1) return ECASQ_EINVAL;
     int64_t pz = n;
     ECASQ_CUDA_TRY(cudaMemcpyAsync(&ds->p, &pz, sizeof(pz), cudaMemcpyHostToDevice, st));
+    Prefix P = make_prefix(ws, L, n, d);
+    P.nL = h.grid_nL;
+    P.nR = h.grid_nR;
     // The fast kernel's fp32 recurrences add one candidate at a time and assume each
     // slab's mass sits at its right end (true for the unique values of x only); a grid
     // runs the reference DP (binary64 candidates from the App. E formulas).
     ecasq_params_t pg = *prm;
     pg.flags |= ECASQ_DP_REFERENCE;
-    return solve_prepared(ws, L, make_prefix(ws, L, n, d), d, n2, &pg, Q, res, st);
+    return solve_prepared(ws, L, P, d, n2, &pg, Q, res, st);
 }
 
 int ecasq_refine(const float *x, int64_t d, float *Q, int32_t m, double lambda, double budget_bits,

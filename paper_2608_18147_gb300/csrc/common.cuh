@@ -47,6 +47,8 @@ struct DevStatus {
     int64_t big_bands;    // fast DP: outputs with more members than the inline list holds
     int64_t tiles_run;    // fast DP, resident costs: (warp, tile) units evaluated
     int64_t tiles_skipped; // ... and skipped by the lower bound
+    int64_t grid_nL;      // permissible set: |L| = #{p_a <= min x}, |R| = #{p_b >= max x} (Sec. 5)
+    int64_t grid_nR;
 };
 
 struct Layout {
@@ -165,6 +167,8 @@ struct Prefix {
     int64_t p;
     int64_t d;
     int64_t ps;           // DP-table row stride, table_stride(p)
+    int64_t nL = 1;       // first-value set L = {0..nL-1}, last-value set R = {p-nR..p-1}
+    int64_t nR = 1;       // (Sec. 5); both 1 when the candidates are the unique values of x
 };
 
 __device__ __forceinline__ dd load_dd(const double *a, int64_t p, int64_t t) { return {a[t], a[p + 1 + t]}; }
@@ -194,6 +198,12 @@ __device__ __forceinline__ double phi_exact(const Prefix &P, double U, double D,
     double dd_ = (double)P.d;
     double Dm = first ? __dadd_rn(D, (double)P.w[0]) : D;
     return __dadd_rn(hfun(__ddiv_rn(U, dd_)), hfun(__ddiv_rn(Dm, dd_)));
+}
+
+// Phi^first[a, .] for a first value a in L: the down symbol also holds n_a = w_a.
+__device__ __forceinline__ double phi_first_at(const Prefix &P, int64_t a, double U, double D) {
+    double dd_ = (double)P.d;
+    return __dadd_rn(hfun(__ddiv_rn(U, dd_)), hfun(__ddiv_rn(__dadd_rn(D, (double)P.w[a]), dd_)));
 }
 
 // -------------------------------------------------------------- host helpers

@@ -26,16 +26,30 @@ __global__ void k_dp_clear(double *dp64, int32_t *bp, int G, int s, int64_t p) {
     for (; i < n; i += stride) { dp64[i] = CUDART_INF; bp[i] = -1; }
 }
 
-// eq. apx_base with P = X, L = {0}: dp(2, j) = C[0, j] + lambda' Phi^first[0, j].
+// eq. apx_base: dp(2, j) = min over a in L, a < j, of C[a, j] + lambda' Phi^first[a, j]
+// (lowest a among exact minima; L = {0} when P = X).
 __global__ void k_dp_base(Prefix P, Lams lam, int G, int s, double *dp64, int32_t *bp) {
     int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x + 1;
     if (j >= P.p) return;
-    double C, U, D;
-    pair_exact(P, 0, j, C, U, D);
-    double phi = phi_exact(P, U, D, true);
+    double best[kMaxG];
+    int32_t arg[kMaxG];
+#pragma unroll
+    for (int g = 0; g < kMaxG; g++) { best[g] = CUDART_INF; arg[g] = -1; }
+    for (int64_t a = 0; a < P.nL && a < j; a++) {
+        double C, U, D;
+        pair_exact(P, a, j, C, U, D);
+        double phi = phi_first_at(P, a, U, D);
+#pragma unroll
+        for (int g = 0; g < kMaxG; g++) {
+            if (g < G) {
+                double c = __dadd_rn(C, __dmul_rn(lam.v[g], phi));
+                if (c < best[g]) { best[g] = c; arg[g] = (int32_t)a; }
+            }
+        }
+    }
     for (int g = 0; g < G; g++) {
-        dp64[dp_at(g, 2, j, s, P.ps)] = __dadd_rn(C, __dmul_rn(lam.v[g], phi));
-        bp[dp_at(g, 2, j, s, P.ps)] = 0;
+        dp64[dp_at(g, 2, j, s, P.ps)] = best[g];
+        bp[dp_at(g, 2, j, s, P.ps)] = arg[g];
     }
 }
 
@@ -80,7 +94,7 @@ __device__ void eval_codebook_warp(const Prefix &P, const int32_t *a, int m, dou
         double C, U, D;
         pair_exact(P, a[r], a[r + 1], C, U, D);
         scratch[r] = C;
-        scratch[kMaxS + r] = phi_exact(P, U, D, r == 0);
+        scratch[kMaxS + r] = r == 0 ? phi_first_at(P, a[0], U, D) : phi_exact(P, U, D, false);
         scratch[2 * kMaxS + r] = U;
         scratch[3 * kMaxS + r] = D;
     }
@@ -93,7 +107,7 @@ __device__ void eval_codebook_warp(const Prefix &P, const int32_t *a, int m, dou
             mse = __dadd_rn(mse, scratch[r]);
             hs = __dadd_rn(hs, scratch[kMaxS + r]);
             double D = scratch[3 * kMaxS + r];
-            double f = (r == 0) ? __dadd_rn((double)P.w[0], D) : __dadd_rn(prevU, D);
+            double f = (r == 0) ? __dadd_rn((double)P.w[a[0]], D) : __dadd_rn(prevU, D);
             hx = __dadd_rn(hx, hfun(__ddiv_rn(f, dd_)));
             prevU = scratch[2 * kMaxS + r];
         }
@@ -103,9 +117,10 @@ __device__ void eval_codebook_warp(const Prefix &P, const int32_t *a, int m, dou
     __syncwarp();
 }
 
-// eq. apx_final (smallest i among exact minima; i = s only with EXACT_S) and
-// the backpointer walk, then the metrics of the traced codebook.  Block g = one
-// multiplier, one warp.
+// eq. apx_final over i and j in R (smallest i, then smallest j, among exact minima;
+// i = s only with EXACT_S) and the backpointer walk down to the first value
+// a = bp(2, .), then the metrics of the traced codebook.  Block g = one multiplier,
+// one warp.
 __global__ void k_traceback_eval(Prefix P, int G, int s, int exact_s, const double *dp64, const int32_t *bp,
                                  int32_t *qidx, int32_t *mcount, double *metrics) {
     __shared__ double scratch[4 * kMaxS];
@@ -115,21 +130,23 @@ __global__ void k_traceback_eval(Prefix P, int G, int s, int exact_s, const doub
     int64_t p = P.p;
     if (threadIdx.x == 0) {
         int istar = -1;
+        int64_t jstar = -1;
         double best = CUDART_INF;
-        for (int i = exact_s ? s : 2; i <= s; i++) {
-            double v = dp64[dp_at(g, i, p - 1, s, P.ps)];
-            if (v < best) { best = v; istar = i; }
-        }
+        for (int i = exact_s ? s : 2; i <= s; i++)
+            for (int64_t jr = p - P.nR; jr < p; jr++) {
+                double v = dp64[dp_at(g, i, jr, s, P.ps)];
+                if (v < best) { best = v; istar = i; jstar = jr; }
+            }
         if (istar < 0) {
             sm_m = 0;
         } else {
-            int64_t j = p - 1;
+            int64_t j = jstar;
             a[istar - 1] = (int32_t)j;
             for (int i = istar; i >= 3; i--) {
                 j = bp[dp_at(g, i, j, s, P.ps)];
                 a[i - 2] = (int32_t)j;
             }
-            a[0] = 0;
+            a[0] = bp[dp_at(g, 2, j, s, P.ps)];
             sm_m = istar;
         }
         metrics[4 * g + 0] = best;

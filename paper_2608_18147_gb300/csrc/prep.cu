@@ -358,9 +358,11 @@ int launch_rows_prepare(const float *X, int64_t rows, const RowsData &R, cudaStr
 // The histogram view over a caller-given candidate set P (Sec. 5, App. E): for
 // every grid point t, u_t = #{unique x <= p_t}; N, S, S2 at t+1 are the unique-value
 // prefix sums at u_t (the sums of all entries x <= p_t), so w_t = #{p_(t-1) < x <= p_t}.
-// Flags st->range_err when P is not strictly ascending and finite or does not start
-// at min x and end at max x (the sets L = {first}, R = {last} of eqs. apx_base and
-// apx_final).  vX, NX, SX, S2X: the unique-value arrays (pX values, packed hi | lo).
+// Flags st->range_err when P is not strictly ascending and finite, starts above min x
+// or ends below max x (App. E: then no quantizer drawn from P spans X), and records
+// the sizes of the first- and last-value sets L = {a : p_a <= min x} and
+// R = {b : p_b >= max x} of eqs. apx_base and apx_final in st->grid_nL, grid_nR.
+// vX, NX, SX, S2X: the unique-value arrays (pX values, packed hi | lo).
 __global__ void k_grid_prefix(const float *__restrict__ P, int64_t n, const float *__restrict__ vX,
                               const int64_t *__restrict__ NX, const double *__restrict__ SX,
                               const double *__restrict__ S2X, int64_t pX, float *v, int64_t *w, int64_t *N, double *S,
@@ -371,9 +373,13 @@ __global__ void k_grid_prefix(const float *__restrict__ P, int64_t n, const floa
         if (pt == 0.0f) pt = 0.0f;
         bool bad = !isfinite(pt);
         if (t > 0 && !(P[t] > P[t - 1])) bad = true;
-        if (t == 0 && pt != vX[0]) bad = true;
-        if (t == n - 1 && pt != vX[pX - 1]) bad = true;
+        if (t == 0 && !(pt <= vX[0])) bad = true;
+        if (t == n - 1 && !(pt >= vX[pX - 1])) bad = true;
         if (bad) st->range_err = 1;
+        // L = {a : p_a <= min x} and R = {b : p_b >= max x} are runs at the two ends
+        // (P ascending): the last member of L and the first of R record the sizes
+        if (pt <= vX[0] && (t == n - 1 || !(P[t + 1] <= vX[0]))) st->grid_nL = t + 1;
+        if (pt >= vX[pX - 1] && (t == 0 || !(P[t - 1] >= vX[pX - 1]))) st->grid_nR = n - t;
         // u = #{unique values <= pt} (binary search)
         int64_t lo = 0, hi = pX;
         while (lo < hi) {

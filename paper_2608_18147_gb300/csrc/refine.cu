@@ -4,7 +4,7 @@
 // 1 <= l <= m-2.  Its candidates are the unique input values strictly between
 // its fixed neighbours; the local objective of Sec. 6 (true entropy reading) is
 //   C[q_{l-1}, c] + C[c, q_{l+1}] + lambda' (h(f_{l-1}/d) + h(f_l/d) + h(f_{l+1}/d)),
-// f_{l-1} = U[q_{l-2}, q_{l-1}] + D[q_{l-1}, c]   (w_0 + D[q_0, c] when l-1 = 0),
+// f_{l-1} = U[q_{l-2}, q_{l-1}] + D[q_{l-1}, c]   (n_{q_0} + D[q_0, c] when l-1 = 0),
 // f_l     = U[q_{l-1}, c] + D[c, q_{l+1}],
 // f_{l+1} = U[c, q_{l+1}] + D[q_{l+1}, q_{l+2}]   (U[c, q_{m-1}] when l+1 = m-1).
 // Values of one class never share a frequency term, so all of them move at
@@ -14,7 +14,7 @@
 namespace ecasq {
 
 struct Nbr {
-    int64_t L, R, cur;
+    int64_t L, R, cur, a0;
     double Ux, Dx;   // outer neighbours' fixed halves of f_{l-1} and f_{l+1}
     int firstL, lastR;
 };
@@ -24,7 +24,7 @@ __device__ __forceinline__ double local_obj(const Prefix &P, const Nbr &n, int64
     double C1, U1, D1, C2, U2, D2;
     pair_exact(P, n.L, c, C1, U1, D1);
     pair_exact(P, c, n.R, C2, U2, D2);
-    double fl = n.firstL ? __dadd_rn((double)P.w[0], D1) : __dadd_rn(n.Ux, D1);
+    double fl = n.firstL ? __dadd_rn((double)P.w[n.a0], D1) : __dadd_rn(n.Ux, D1);
     double fm = __dadd_rn(U1, D2);
     double fr = n.lastR ? U2 : __dadd_rn(U2, n.Dx);
     double ent = __dadd_rn(__dadd_rn(hfun(__ddiv_rn(fl, dd_)), hfun(__ddiv_rn(fm, dd_))), hfun(__ddiv_rn(fr, dd_)));
@@ -35,7 +35,7 @@ constexpr int kRefineChunk = 256;   // candidates per block: one per thread, so 
 
 __device__ __forceinline__ Nbr make_nbr(const Prefix &P, const int32_t *a, int m, int l) {
     Nbr n;
-    n.L = a[l - 1]; n.R = a[l + 1]; n.cur = a[l];
+    n.L = a[l - 1]; n.R = a[l + 1]; n.cur = a[l]; n.a0 = a[0];
     n.firstL = (l - 1 == 0); n.lastR = (l + 1 == m - 1);
     double C, U, D;
     n.Ux = 0.0; n.Dx = 0.0;

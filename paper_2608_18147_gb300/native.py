@@ -146,12 +146,13 @@ def _check(rc, where, ok=(OK,)):
 def ws_status(ws):
     """Counters the library leaves at the start of a workspace after a call
     (unique values, device-side flags, fast-DP statistics)."""
-    raw = ws[:96].cpu().numpy().tobytes()
+    raw = ws[:112].cpu().numpy().tobytes()
     (p, nonfinite, range_err, timeout, bound_viol, norm2, rescored, overflow, last_s, last_G, last_d, members,
-     big_bands, tiles_run, tiles_skipped) = __import__("struct").unpack("<qiiiidqqiiqqqqq", raw)
+     big_bands, tiles_run, tiles_skipped, grid_nL, grid_nR) = __import__("struct").unpack("<qiiiidqqiiqqqqqqq", raw)
     return dict(p=p, nonfinite=nonfinite, range_err=range_err, timeout=timeout, bound_viol=bound_viol, norm2=norm2,
                 rescored=rescored, overflow=overflow, last_s=last_s, last_G=last_G, last_d=last_d, members=members,
-                big_bands=big_bands, tiles_run=tiles_run, tiles_skipped=tiles_skipped)
+                big_bands=big_bands, tiles_run=tiles_run, tiles_skipped=tiles_skipped, grid_nL=grid_nL,
+                grid_nR=grid_nR)
 
 
 def ecasq_workspace_size(d, s, rows=1) -> int:
@@ -195,7 +196,8 @@ def ecasq_solve(x, s, budget_bits=0.0, lambda_=-1.0, ws=None, **kw):
 
 
 def ecasq_solve_grid(x, P, s, budget_bits=0.0, lambda_=-1.0, ws=None, **kw):
-    """Budgeted solve with the codebook drawn from the candidate set P (ascending, spanning x)."""
+    """Budgeted solve with the codebook drawn from the candidate set P (strictly ascending,
+    P[0] <= min x, P[-1] >= max x)."""
     torch = _torch()
     x = _dev_f32(x)
     P = _dev_f32(P)

@@ -64,3 +64,44 @@ def test_grid_that_does_not_span_x_is_rejected(E):
         with pytest.raises(E.EcasqError) as ei:
             E.ecasq_solve_grid(x, np.array(P, np.float32), 4, budget_bits=1.0)
         assert ei.value.code == E.native.EINVAL
+
+
+def wide_grid(x, n, below, above):
+    lo, hi = float(x.min()), float(x.max())
+    g = np.linspace(lo - below, hi + above, n).astype(np.float32)
+    return np.unique(np.concatenate([g, np.array([lo, hi], np.float32)]))
+
+
+@pytest.mark.parametrize("refine", [0, 3])
+def test_grid_with_several_first_and_last_candidates(E, oracle_mod, refine):
+    """L = {p_a <= min x} and R = {p_b >= max x} with several members each (eqs. apx_base,
+    apx_final): the base layer minimises over a in L, the final selection over j in R."""
+    x = workloads.signed_lognormal(5000, 11)
+    span = float(x.max() - x.min())
+    g = wide_grid(x, 300, 0.05 * span, 0.08 * span)
+    import torch
+    ws = torch.empty(int(E.lib().ecasq_workspace_size_grid(x.size, g.size, 8, 0)), dtype=torch.uint8,
+                     device="cuda")
+    Q, res = E.ecasq_solve_grid(x, g, 8, budget_bits=2.0, ws=ws, refine_max_rounds=refine, refine_rel_tol=1e-9)
+    H = oracle_mod.Hist(x, g)
+    st = E.native.ws_status(ws)
+    assert (st["grid_nL"], st["grid_nR"]) == (H.nL, H.nR)
+    assert H.nL > 1 and H.nR > 1
+    _check(res, oracle_mod.solve_budget(x, 8, 2.0, grid=g, refine_rounds=refine, refine_tol=1e-9), Q)
+
+
+def test_appF1_example_on_the_gpu(E, oracle_mod):
+    """App. F.1: X = half 0s, half 2s; P = (0,1,2,3,4); s = 2.  At every multiplier the
+    GPU returns the oracle's codebook ({0,2} or {0,4}, never {0,3}); the budgeted solve
+    at b = 0.95 returns {0, 4}, the best Lagrangian point under the budget."""
+    x = np.array([0.0] * 32 + [2.0] * 32, np.float32)
+    P = np.arange(5, dtype=np.float32)
+    H = oracle_mod.Hist(x, P)
+    for lam in (0.01, 1.0, 4.0, 5.5, 6.5, 20.0):
+        Q, res = E.ecasq_solve_grid(x, P, 2, lambda_=lam)
+        o = H.apx_dp(2, lam * H.norm2, tables=False)
+        np.testing.assert_array_equal(Q.cpu().numpy(), P[o["Q_idx"]])
+        assert Q.cpu().numpy().tolist() in ([0.0, 2.0], [0.0, 4.0])
+    Q, res = E.ecasq_solve_grid(x, P, 2, budget_bits=0.95)
+    _check(res, oracle_mod.solve_budget(x, 2, 0.95, grid=P), Q)
+    assert Q.cpu().numpy().tolist() == [0.0, 4.0]
