@@ -75,6 +75,9 @@ def _load():
             "or_midpoints7": (None, [dbl, dbl, pd]),
             "or_search": (i32, [P, i32, dbl, dbl, dbl, i32, i32, pi64, pi32, pd, pd, i32, pi32]),
             "or_refine": (i32, [P, pi64, i32, dbl, dbl, i32, i32, dbl, pi32, pd]),
+            "or_timeshare": (i32, [P, i32, dbl, dbl, dbl, i32, i32, pi64, pi32, pi64, pi32, pd, pd, pd]),
+            "or_quantize_timeshare": (i32, [pf, i64, pf, i32, pf, i32, dbl, u64, u64, C.POINTER(C.c_uint8),
+                                            C.POINTER(C.c_uint8), C.POINTER(C.c_uint32), pd]),
             "or_splitmix64": (u64, [u64]),
             "or_quantize": (i32, [pf, i64, pf, i32, u64, C.POINTER(C.c_uint8),
                                   C.POINTER(C.c_uint32), pd]),
@@ -242,6 +245,24 @@ class Hist:
                     h_surrogate=res[2], h_exact=res[3], trace=trace[:6 * n].reshape(n, 6).copy(),
                     n_evaluated=nt.value)
 
+    def timeshare(self, s, budget, lo=1e-8, hi=1e3, rounds=6, exact_s=False):
+        """Two-way time-sharing of Sec. 7 around the budget (reading in the C file)."""
+        Qm = np.empty(s + 1, np.int64)
+        Qp = np.empty(s + 1, np.int64)
+        mm, mp = C.c_int32(), C.c_int32()
+        mmet, pmet = np.empty(3), np.empty(3)
+        out = np.empty(6)
+        st = _load().or_timeshare(self._h, int(s), float(budget), float(lo), float(hi), int(rounds),
+                                  int(bool(exact_s)), _ptr(Qm, C.c_int64), C.byref(mm), _ptr(Qp, C.c_int64),
+                                  C.byref(mp), _ptr(mmet, C.c_double), _ptr(pmet, C.c_double),
+                                  _ptr(out, C.c_double))
+        if st != OK:
+            raise OracleError(st, "or_timeshare")
+        return dict(beta=out[0], lam_minus=out[1], lam_plus=out[2], mse=out[3], h_surrogate=out[4],
+                    h_exact=out[5], minus_idx=Qm[:mm.value].copy(), plus_idx=Qp[:mp.value].copy(),
+                    minus=dict(mse=mmet[0], h_surrogate=mmet[1], h_exact=mmet[2]),
+                    plus=dict(mse=pmet[0], h_surrogate=pmet[1], h_exact=pmet[2]))
+
     def refine(self, a, lam_prime, budget=np.inf, guard=False, max_rounds=5, tol=0.0):
         """Three-colour refinement of Sec. 6 (true Lagrangian, reading in the C file)."""
         a = np.array(a, dtype=np.int64)
@@ -318,6 +339,29 @@ def quantize(x, Q, seed):
     if st != OK:
         raise OracleError(st, "or_quantize")
     return idx, counts, he.value
+
+
+def quantize_timeshare(x, Qm, Qp, beta, seed, seed_ts):
+    """Time-shared stochastic quantization (Sec. 7): (idx, sel, counts, rate)."""
+    x = _f32(x)
+    Qm = _f32(Qm)
+    if Qp is None or len(Qp) == 0:
+        Qp, mp = np.zeros(1, np.float32), 0
+    else:
+        Qp = _f32(Qp)
+        mp = Qp.size
+    idx = np.empty(x.size, np.uint8)
+    sel = np.empty(x.size, np.uint8)
+    counts = np.empty(Qm.size + mp, np.uint32)
+    rate = C.c_double()
+    st = _load().or_quantize_timeshare(_ptr(x, C.c_float), x.size, _ptr(Qm, C.c_float), Qm.size,
+                                       _ptr(Qp, C.c_float), mp, float(beta),
+                                       C.c_uint64(seed & 0xFFFFFFFFFFFFFFFF), C.c_uint64(seed_ts & 0xFFFFFFFFFFFFFFFF),
+                                       _ptr(idx, C.c_uint8), _ptr(sel, C.c_uint8), _ptr(counts, C.c_uint32),
+                                       C.byref(rate))
+    if st != OK:
+        raise OracleError(st, "or_quantize_timeshare")
+    return idx, sel, counts, rate.value
 
 
 def solve_budget(x, s, budget, lo=1e-8, hi=1e3, rounds=6, refine_rounds=0, refine_tol=0.0,

@@ -30,6 +30,8 @@
  *   or_brute         exhaustive enumeration of spanning codebooks drawn from X
  *   or_brute_grid    the same over codebooks drawn from a permissible set P
  *   or_search        Sec. 3 / Sec. 5: tune lambda for a budget b (schedule below)
+ *   or_timeshare     Sec. 7: two-way time-sharing between the evaluated points
+ *                    around b; or_quantize_timeshare encodes with it
  *   or_refine        Sec. 6: three-colour refinement
  *   or_quantize      Sec. 2: unbiased stochastic rounding, Sec. 1 entropy
  *
@@ -701,9 +703,13 @@ static int32_t eval_lambda(const or_hist *H, int32_t s, double lam, int32_t exac
  *   answer: minimum MSE over the feasible evaluated points, ties to the smaller lambda.
  * trace (cap rows of 6 doubles): lam, mse, H(I,B), H(Xhat), m, feasible.
  * res: lam, mse, H(I,B), H(Xhat). */
-int32_t or_search(const or_hist *H, int32_t s, double budget, double lo, double hi, int32_t rounds,
-                  int32_t exact_s, int64_t *Q_idx, int32_t *m_out, double *res,
-                  double *trace, int32_t trace_cap, int32_t *n_trace) {
+/* plus: when not NULL, also the evaluated infeasible point of least H(I,B)
+ * (ties: less MSE, then the smaller lambda) and its codebook (Sec. 7's Q+). */
+typedef struct { or_point pt; int64_t *Q; int have; } or_plus;
+
+static int32_t search_core(const or_hist *H, int32_t s, double budget, double lo, double hi, int32_t rounds,
+                           int32_t exact_s, int64_t *Q_idx, int32_t *m_out, double *res,
+                           double *trace, int32_t trace_cap, int32_t *n_trace, or_plus *plus) {
     if (!(budget >= 0.0) || !(lo > 0.0) || !(hi > lo) || rounds < 1 || s < 2) return OR_EINVAL;
     int64_t *Qb = (int64_t *)malloc(sizeof(int64_t) * (size_t)(s + 1));
     int64_t *Qbest = (int64_t *)malloc(sizeof(int64_t) * (size_t)(s + 1));
@@ -721,6 +727,13 @@ int32_t or_search(const or_hist *H, int32_t s, double budget, double lo, double 
         if ((pt).feasible && (!have || (pt).mse < best.mse ||                        \
                               ((pt).mse == best.mse && (pt).lam < best.lam))) {      \
             best = (pt); have = 1; memcpy(Qbest, Qb, sizeof(int64_t) * (size_t)(pt).m); \
+        }                                                                            \
+        if (plus && !(pt).feasible &&                                                \
+            (!plus->have || (pt).hs < plus->pt.hs ||                                 \
+             ((pt).hs == plus->pt.hs && ((pt).mse < plus->pt.mse ||                  \
+                                         ((pt).mse == plus->pt.mse && (pt).lam < plus->pt.lam))))) { \
+            plus->pt = (pt); plus->have = 1;                                         \
+            memcpy(plus->Q, Qb, sizeof(int64_t) * (size_t)(pt).m);                   \
         }                                                                            \
     } while (0)
     or_point pt;
@@ -760,6 +773,51 @@ done:
     *n_trace = nt;
     free(Qb); free(Qbest);
     return st;
+}
+
+int32_t or_search(const or_hist *H, int32_t s, double budget, double lo, double hi, int32_t rounds,
+                  int32_t exact_s, int64_t *Q_idx, int32_t *m_out, double *res,
+                  double *trace, int32_t trace_cap, int32_t *n_trace) {
+    return search_core(H, s, budget, lo, hi, rounds, exact_s, Q_idx, m_out, res, trace, trace_cap, n_trace, NULL);
+}
+
+/* Two-way time-sharing (Sec. 7).  Q- is the budgeted solve's answer (least MSE with
+ * H(I,B) = b- <= b); Q+ is the evaluated point of least rate b+ > b.  Each entry
+ * uses Q+ with probability beta = (b - b-)/(b+ - b-), so the expected MSE and rate
+ * are the beta-mixtures of the two.  Readings: the rate is H(I,B), the quantity the
+ * budget constrains; beta = 0 (no Q+) when every evaluated point is feasible, when
+ * b- = b, or when Q+ does not have less MSE than Q- (time-sharing cannot help).
+ * out: beta, lam-, lam+, and the mixture's MSE, H(I,B), H(Xhat); m_plus = 0 without Q+.
+ * The search runs as or_search; status as or_search. */
+int32_t or_timeshare(const or_hist *H, int32_t s, double budget, double lo, double hi, int32_t rounds,
+                     int32_t exact_s, int64_t *Qm_idx, int32_t *m_minus, int64_t *Qp_idx, int32_t *m_plus,
+                     double *minus_met, double *plus_met, double *out) {
+    double res[4];
+    double trace[6];
+    int32_t nt;
+    or_plus plus;
+    plus.have = 0;
+    plus.Q = Qp_idx;
+    int32_t st = search_core(H, s, budget, lo, hi, rounds, exact_s, Qm_idx, m_minus, res, trace, 0, &nt, &plus);
+    if (st != OR_OK) return st;
+    minus_met[0] = res[1]; minus_met[1] = res[2]; minus_met[2] = res[3];
+    double beta = 0.0;
+    if (plus.have && plus.pt.mse < res[1] && res[2] < budget)
+        beta = (budget - res[2]) / (plus.pt.hs - res[2]);
+    if (beta > 0.0) {
+        *m_plus = plus.pt.m;
+        plus_met[0] = plus.pt.mse; plus_met[1] = plus.pt.hs; plus_met[2] = plus.pt.hx;
+        out[2] = plus.pt.lam;
+    } else {
+        *m_plus = 0;
+        plus_met[0] = plus_met[1] = plus_met[2] = NAN;
+        out[2] = NAN;
+    }
+    out[0] = beta;
+    out[1] = res[0];
+    for (int r = 0; r < 3; r++)
+        out[3 + r] = beta > 0.0 ? (1.0 - beta) * minus_met[r] + beta * plus_met[r] : minus_met[r];
+    return OR_OK;
 }
 
 /* ----------------------------------------------------------- refinement */
@@ -878,6 +936,52 @@ int32_t or_quantize(const float *x, int64_t d, const float *Q, int32_t m, uint64
     double he = 0.0, dd = (double)d;
     for (int32_t r = 0; r < m; r++) he += h((double)counts[r] / dd);
     *h_emp = he;
+    return OR_OK;
+}
+
+/* Time-shared stochastic quantization (Sec. 7 with Sec. 2): entry i (original order)
+ * uses Q+ iff k_s * 2^-24 < beta, k_s the top 24 bits of SplitMix64(seed_ts +
+ * (i+1)*0x9E3779B97F4A7C15) (binary64 compare, exact), then rounds within the chosen
+ * codebook with the rule of or_quantize (seed, same counter i).  sel[i] = 1 for Q+.
+ * counts: [mm] for Q-, then [mp] for Q+.  rate: the bits per entry of coding each
+ * part with its own empirical law, -(1/d) sum_parts sum_r c_r log2(c_r / n_part). */
+int32_t or_quantize_timeshare(const float *x, int64_t d, const float *Qm, int32_t mm, const float *Qp,
+                              int32_t mp, double beta, uint64_t seed, uint64_t seed_ts, uint8_t *idx,
+                              uint8_t *sel, uint32_t *counts, double *rate) {
+    if (d < 1 || mm < 1 || mm > 256 || mp < 0 || mp > 256 || !(beta >= 0.0 && beta <= 1.0)) return OR_EINVAL;
+    if (beta > 0.0 && mp < 1) return OR_EINVAL;
+    for (int32_t r = 0; r < mm + mp; r++) counts[r] = 0;
+    for (int64_t i = 0; i < d; i++) {
+        uint64_t zs = or_splitmix64(seed_ts + (uint64_t)(i + 1) * 0x9E3779B97F4A7C15ULL);
+        int use_plus = (double)(uint32_t)(zs >> 40) * 0x1p-24 < beta;
+        const float *Q = use_plus ? Qp : Qm;
+        int32_t m = use_plus ? mp : mm;
+        float xv = x[i];
+        if (!(xv >= Q[0] && xv <= Q[m - 1])) return OR_ERANGE;
+        int32_t lo = 0, hi = m - 1;
+        while (lo < hi) {
+            int32_t mid = (lo + hi + 1) / 2;
+            if (Q[mid] <= xv) lo = mid; else hi = mid - 1;
+        }
+        int32_t t = lo;
+        if (Q[t] != xv) {
+            uint64_t z = or_splitmix64(seed + (uint64_t)(i + 1) * 0x9E3779B97F4A7C15ULL);
+            float k = (float)(uint32_t)(z >> 40) * 0x1p-24f;
+            if (k * (Q[t + 1] - Q[t]) < xv - Q[t]) t += 1;
+        }
+        idx[i] = (uint8_t)t;
+        if (sel) sel[i] = (uint8_t)use_plus;
+        counts[(use_plus ? mm : 0) + t]++;
+    }
+    double bits = 0.0;
+    for (int part = 0; part < 2; part++) {
+        int32_t off = part ? mm : 0, m = part ? mp : mm;
+        double n = 0.0;
+        for (int32_t r = 0; r < m; r++) n += (double)counts[off + r];
+        for (int32_t r = 0; r < m; r++)
+            if (counts[off + r]) bits -= (double)counts[off + r] * log2((double)counts[off + r] / n);
+    }
+    *rate = bits / (double)d;
     return OR_OK;
 }
 
