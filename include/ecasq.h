@@ -94,6 +94,21 @@ typedef struct ecasq_result {
     int32_t reserved2;
 } ecasq_result_t;
 
+/* Two-way time-sharing (Sec. 7): the mixture of the budgeted solution Q- (rate
+ * b- <= b) and the evaluated point Q+ of least rate b+ > b, each entry using Q+
+ * with probability beta = (b - b-)/(b+ - b-).  Rates are H(I,B), the quantity the
+ * budget constrains; MSE and rates of the mixture are linear in beta. */
+typedef struct ecasq_timeshare {
+    double beta;               /* probability of Q+; 0 = Q- alone (no Q+, b- = b, or Q+ not better) */
+    double lambda_plus;        /* multiplier of Q+ (vNMSE scale); NaN without Q+ */
+    double mse, vnmse;         /* of the mixture */
+    double h_surrogate;        /* H(I,B) of the mixture (= b when beta > 0) */
+    double h_exact;            /* H(Xhat) of the mixture */
+    double plus_mse, plus_h_surrogate, plus_h_exact;  /* of Q+; NaN without Q+ */
+    int32_t m_plus;            /* |Q+|, 0 without Q+ */
+    int32_t reserved;
+} ecasq_timeshare_t;
+
 /* Bytes of workspace needed by every entry point below for vectors of up to d
  * entries, codebook cap s, and `rows` independent rows (1 for single-vector
  * calls).  Returns 0 for invalid arguments. */
@@ -142,6 +157,44 @@ int ecasq_solve(const float *x, int64_t d, const ecasq_params_t *prm, void *ws, 
 size_t ecasq_workspace_size_grid(int64_t d, int64_t n, int32_t s, uint32_t flags);
 int ecasq_solve_grid(const float *x, int64_t d, const float *P, int64_t n, const ecasq_params_t *prm, void *ws,
                      size_t ws_bytes, float *Q, ecasq_result_t *res, ecasq_stream_t stream);
+
+/* Budgeted solve with two-way time-sharing (Sec. 7): the multiplier search of
+ * ecasq_solve (or of ecasq_solve_grid when P is not NULL), then Q+ = the evaluated
+ * point with the least H(I,B) above the budget (ties: less MSE, then the smaller
+ * multiplier) and beta as in ecasq_timeshare_t.  Every evaluated point is a
+ * minimiser of the surrogate Lagrangian, so the mixture reaches the budget exactly
+ * with an MSE linear in beta.  prm->lambda must be < 0 (a budget) and
+ * prm->refine_max_rounds 0, else ECASQ_EINVAL.
+ *   P, n  as ecasq_solve_grid, or P = NULL for the unique values of x
+ *   Qm    device [s] output: Q- (as ecasq_solve's Q)
+ *   Qp    device [s] output: Q+ when ts->m_plus > 0, else untouched
+ *   res   host (may be NULL): ecasq_solve's result for Q-
+ *   ts    host output
+ * Workspace: ecasq_workspace_size_flags(d, s, 1, flags), or with P
+ * ecasq_workspace_size_grid(d, n, s, flags).  Synchronises `stream`. */
+int ecasq_solve_timeshare(const float *x, int64_t d, const float *P, int64_t n, const ecasq_params_t *prm, void *ws,
+                          size_t ws_bytes, float *Qm, float *Qp, ecasq_result_t *res, ecasq_timeshare_t *ts,
+                          ecasq_stream_t stream);
+
+/* Time-shared stochastic quantization (Sec. 7 with Sec. 2): entry i (original
+ * order) uses Qp iff k_s 2^-24 < beta in binary64, k_s = top 24 bits of
+ * SplitMix64(seed_ts + (i+1) 0x9E3779B97F4A7C15), then rounds within its codebook
+ * exactly as ecasq_quantize with `seed` (same counter i).  A decoder that knows
+ * seed_ts regenerates the partition; `sel` is a convenience copy of it.
+ *   Qm [mm], Qp [mp]  device, ascending; mp may be 0 (and Qp NULL) when beta = 0
+ *   idx     device [d] uint8 output: index into the entry's codebook
+ *   sel     device [d] uint8 output (may be NULL): 1 where Qp was used
+ *   counts  device [mm + mp] uint32 output: index histograms of Qm, then Qp
+ *   ws      device, >= 256 bytes, 256-byte aligned (status record)
+ *   rate    host (may be NULL): bits per entry of coding each part with its own
+ *           empirical law, -(1/d) sum_parts sum_r c_r log2(c_r / n_part)
+ * ECASQ_EINVAL for beta outside [0, 1], non-ascending codebooks or mp = 0 with
+ * beta > 0; ECASQ_ERANGE if an entry lies outside its codebook's range.
+ * Synchronises `stream`. */
+int ecasq_quantize_timeshare(const float *x, int64_t d, const float *Qm, int32_t mm, const float *Qp, int32_t mp,
+                             double beta, uint64_t seed, uint64_t seed_ts, uint8_t *idx, uint8_t *sel,
+                             uint32_t *counts, void *ws, size_t ws_bytes, double *rate, ecasq_stream_t stream);
+
 
 /* One DP pass (Sec. 5) at G <= 8 fixed multipliers, the unit of the search.
  *   lambdas   host [G], vNMSE scale, >= 0

@@ -36,6 +36,9 @@ int launch_refine_colour(const Prefix &P, const int32_t *a, int m, int colour, d
 size_t refine_scratch_bytes(int64_t d);
 int launch_quantize(const float *x, int64_t d, const float *Q, int m, uint64_t seed, uint8_t *idx, uint32_t *counts,
                     DevStatus *st, int num_sms, cudaStream_t stream);
+int launch_quantize_timeshare(const float *x, int64_t d, const float *Qm, int mm, const float *Qp, int mp,
+                              double beta, uint64_t seed, uint64_t seed_ts, uint8_t *idx, uint8_t *sel,
+                              uint32_t *counts, DevStatus *st, int num_sms, cudaStream_t stream);
 size_t fast_dp_band_bytes(int64_t d, int32_t s);
 
 static std::atomic<long long> g_launches{0};
@@ -520,8 +523,12 @@ static int64_t read_rescored(void *ws, cudaStream_t st) {
 
 // The search, refinement and result of a solve over a prepared histogram view P
 // (unique values of x, or a caller-given candidate set).
+// Sec. 7: the evaluated infeasible point of least H(I,B) (ties: less MSE, then the
+// smaller multiplier), the Q+ of two-way time-sharing.
+struct PlusPoint { bool have = false; double lam = 0.0, mse = 0.0, hs = 0.0, hx = 0.0; std::vector<int32_t> a; };
+
 static int solve_prepared(void *ws, const Layout &L, const Prefix &P, int64_t d, double n2, const ecasq_params_t *prm,
-                          float *Q, ecasq_result_t *res, cudaStream_t st) {
+                          float *Q, ecasq_result_t *res, cudaStream_t st, PlusPoint *plus = nullptr) {
     const int s = prm->s;
     const int64_t p = P.p;
     int rc;
@@ -608,6 +615,17 @@ static int solve_prepared(void *ws, const Layout &L, const Prefix &P, int64_t d,
             }
         }
     }
+    if (plus) {
+        for (const Eval &e : evals) {
+            if (e.feas) continue;
+            if (!plus->have || e.hs < plus->hs ||
+                (e.hs == plus->hs && (e.mse < plus->mse || (e.mse == plus->mse && e.lam < plus->lam)))) {
+                plus->have = true;
+                plus->lam = e.lam; plus->mse = e.mse; plus->hs = e.hs; plus->hx = e.hx;
+                plus->a = e.a;
+            }
+        }
+    }
     std::vector<int32_t> a = sel->a;
     double lam = sel->lam;
     double lamp = lam * n2;
@@ -630,24 +648,38 @@ static int solve_prepared(void *ws, const Layout &L, const Prefix &P, int64_t d,
     return status;
 }
 
+// Layout, workspace check, sort / histogram / prefix sums of x (Sec. 2, App. E).
+static int prepare_plain(const float *x, int64_t d, const ecasq_params_t *prm, void *ws, size_t ws_bytes, Layout *L,
+                         Prefix *P, double *n2, cudaStream_t st) {
+    make_layout(d, prm->s, 1, L);
+    int rc = add_resident_costs(prm->flags, L);
+    if (rc) return rc;
+    rc = check_ws(ws, ws_bytes, *L);
+    if (rc) return rc;
+    int64_t p;
+    rc = prepare_device(x, d, ws, *L, st, &p, n2);
+    if (rc) return rc;
+    *P = make_prefix(ws, *L, p, d);
+    return ECASQ_OK;
+}
+
+static void timer_reset(const ecasq_params_t *prm) {
+    g_timer.on = (prm->flags & ECASQ_TIME_KERNELS) != 0;
+    g_timer.ms = 0.0;
+    g_timer.launches = 0;
+}
+
 int ecasq_solve(const float *x, int64_t d, const ecasq_params_t *prm, void *ws, size_t ws_bytes, float *Q,
                 ecasq_result_t *res, ecasq_stream_t stream) {
     if (!x || !Q || d < 1 || d >= ((int64_t)1 << 31) || !params_ok(prm)) return ECASQ_EINVAL;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    g_timer.on = (prm->flags & ECASQ_TIME_KERNELS) != 0;
-    g_timer.ms = 0.0;
-    g_timer.launches = 0;
+    timer_reset(prm);
     Layout L;
-    make_layout(d, prm->s, 1, &L);
-    int rc = add_resident_costs(prm->flags, &L);
-    if (rc) return rc;
-    rc = check_ws(ws, ws_bytes, L);
-    if (rc) return rc;
-    int64_t p;
+    Prefix P;
     double n2;
-    rc = prepare_device(x, d, ws, L, st, &p, &n2);
+    int rc = prepare_plain(x, d, prm, ws, ws_bytes, &L, &P, &n2, st);
     if (rc) return rc;
-    return solve_prepared(ws, L, make_prefix(ws, L, p, d), d, n2, prm, Q, res, st);
+    return solve_prepared(ws, L, P, d, n2, prm, Q, res, st);
 }
 
 size_t ecasq_workspace_size_grid(int64_t d, int64_t n, int32_t s, uint32_t flags) {
@@ -655,16 +687,12 @@ size_t ecasq_workspace_size_grid(int64_t d, int64_t n, int32_t s, uint32_t flags
     return ecasq_workspace_size_flags(std::max(d, n), s, 1, flags);
 }
 
-int ecasq_solve_grid(const float *x, int64_t d, const float *Pg, int64_t n, const ecasq_params_t *prm, void *ws,
-                     size_t ws_bytes, float *Q, ecasq_result_t *res, ecasq_stream_t stream) {
-    if (!x || !Q || !Pg || d < 1 || d >= ((int64_t)1 << 31) || n < 1 || n >= ((int64_t)1 << 31) || !params_ok(prm))
-        return ECASQ_EINVAL;
-    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    g_timer.on = (prm->flags & ECASQ_TIME_KERNELS) != 0;
-    g_timer.ms = 0.0;
-    g_timer.launches = 0;
+// The histogram view over a permissible set P (Sec. 5, App. E): prepare x, then
+// gather the prefix sums at the points of P; P->nL, P->nR receive |L|, |R|.
+static int prepare_grid(const float *x, int64_t d, const float *Pg, int64_t n, const ecasq_params_t *prm, void *ws,
+                        size_t ws_bytes, Layout *Lo, Prefix *Po, double *n2o, cudaStream_t st) {
     const int64_t dmax = std::max(d, n);
-    Layout L;
+    Layout &L = *Lo;
     make_layout(dmax, prm->s, 1, &L);
     L.d = dmax;
     int rc = add_resident_costs(prm->flags, &L);
@@ -695,15 +723,84 @@ int ecasq_solve_grid(const float *x, int64_t d, const float *Pg, int64_t n, cons
     if (h.range_err || h.grid_nL < 1 || h.grid_nR < 1) return ECASQ_EINVAL;
     int64_t pz = n;
     ECASQ_CUDA_TRY(cudaMemcpyAsync(&ds->p, &pz, sizeof(pz), cudaMemcpyHostToDevice, st));
-    Prefix P = make_prefix(ws, L, n, d);
-    P.nL = h.grid_nL;
-    P.nR = h.grid_nR;
+    *Po = make_prefix(ws, L, n, d);
+    Po->nL = h.grid_nL;
+    Po->nR = h.grid_nR;
+    *n2o = n2;
+    return ECASQ_OK;
+}
+
+int ecasq_solve_grid(const float *x, int64_t d, const float *Pg, int64_t n, const ecasq_params_t *prm, void *ws,
+                     size_t ws_bytes, float *Q, ecasq_result_t *res, ecasq_stream_t stream) {
+    if (!x || !Q || !Pg || d < 1 || d >= ((int64_t)1 << 31) || n < 1 || n >= ((int64_t)1 << 31) || !params_ok(prm))
+        return ECASQ_EINVAL;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    timer_reset(prm);
+    Layout L;
+    Prefix P;
+    double n2;
+    int rc = prepare_grid(x, d, Pg, n, prm, ws, ws_bytes, &L, &P, &n2, st);
+    if (rc) return rc;
     // The fast kernel's fp32 recurrences add one candidate at a time and assume each
     // slab's mass sits at its right end (true for the unique values of x only); a grid
     // runs the reference DP (binary64 candidates from the App. E formulas).
     ecasq_params_t pg = *prm;
     pg.flags |= ECASQ_DP_REFERENCE;
     return solve_prepared(ws, L, P, d, n2, &pg, Q, res, st);
+}
+
+int ecasq_solve_timeshare(const float *x, int64_t d, const float *Pg, int64_t n, const ecasq_params_t *prm, void *ws,
+                          size_t ws_bytes, float *Qm, float *Qp, ecasq_result_t *res, ecasq_timeshare_t *ts,
+                          ecasq_stream_t stream) {
+    if (!x || !Qm || !Qp || !ts || d < 1 || d >= ((int64_t)1 << 31) || !params_ok(prm) || !(prm->lambda < 0.0) ||
+        prm->refine_max_rounds != 0)
+        return ECASQ_EINVAL;
+    if (Pg && (n < 1 || n >= ((int64_t)1 << 31))) return ECASQ_EINVAL;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    timer_reset(prm);
+    Layout L;
+    Prefix P;
+    double n2;
+    ecasq_params_t pg = *prm;
+    int rc;
+    if (Pg) {
+        rc = prepare_grid(x, d, Pg, n, prm, ws, ws_bytes, &L, &P, &n2, st);
+        pg.flags |= ECASQ_DP_REFERENCE;
+    } else {
+        rc = prepare_plain(x, d, prm, ws, ws_bytes, &L, &P, &n2, st);
+    }
+    if (rc) return rc;
+    PlusPoint plus;
+    ecasq_result_t rm;
+    int status = solve_prepared(ws, L, P, d, n2, &pg, Qm, &rm, st, &plus);
+    if (res) *res = rm;
+    memset(ts, 0, sizeof(*ts));
+    ts->lambda_plus = NAN;
+    ts->plus_mse = ts->plus_h_surrogate = ts->plus_h_exact = NAN;
+    if (status != ECASQ_OK) return status;
+    // Sec. 7: beta = (b - b-)/(b+ - b-) when Q+ exists, has less MSE and b- < b
+    double beta = 0.0;
+    if (plus.have && plus.mse < rm.mse && rm.h_surrogate < prm->budget_bits)
+        beta = (prm->budget_bits - rm.h_surrogate) / (plus.hs - rm.h_surrogate);
+    double mm[3] = {rm.mse, rm.h_surrogate, rm.h_exact};
+    double mx[3] = {rm.mse, rm.h_surrogate, rm.h_exact};
+    if (beta > 0.0) {
+        rc = write_codebook(ws, L, plus.a, Qp, st);
+        if (rc) return rc;
+        double pm[3] = {plus.mse, plus.hs, plus.hx};
+        for (int r = 0; r < 3; r++) mx[r] = (1.0 - beta) * mm[r] + beta * pm[r];
+        ts->m_plus = (int32_t)plus.a.size();
+        ts->lambda_plus = plus.lam;
+        ts->plus_mse = plus.mse;
+        ts->plus_h_surrogate = plus.hs;
+        ts->plus_h_exact = plus.hx;
+    }
+    ts->beta = beta;
+    ts->mse = mx[0];
+    ts->vnmse = n2 > 0.0 ? mx[0] / n2 : 0.0;
+    ts->h_surrogate = mx[1];
+    ts->h_exact = mx[2];
+    return ECASQ_OK;
 }
 
 int ecasq_refine(const float *x, int64_t d, float *Q, int32_t m, double lambda, double budget_bits,
@@ -841,6 +938,49 @@ int ecasq_quantize_noalloc(const float *x, int64_t d, const float *Q, int32_t m,
             if (f > 0.0) he += -f * log2(f);
         }
         *h_emp = he;
+    }
+    return ECASQ_OK;
+}
+
+int ecasq_quantize_timeshare(const float *x, int64_t d, const float *Qm, int32_t mm, const float *Qp, int32_t mp,
+                             double beta, uint64_t seed, uint64_t seed_ts, uint8_t *idx, uint8_t *sel,
+                             uint32_t *counts, void *ws, size_t ws_bytes, double *rate, ecasq_stream_t stream) {
+    if (!x || !Qm || !idx || !counts || d < 1 || d >= ((int64_t)1 << 31) || mm < 1 || mm > kMaxS || mp < 0 ||
+        mp > kMaxS || !(beta >= 0.0 && beta <= 1.0) || (beta > 0.0 && (mp < 1 || !Qp)))
+        return ECASQ_EINVAL;
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255) != 0 || ws_bytes < sizeof(DevStatus)) return ECASQ_EWORKSPACE;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    DevStatus *ds = wsp<DevStatus>(ws, 0);
+    float qh[2 * kMaxS];
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(qh, Qm, 4 * (size_t)mm, cudaMemcpyDeviceToHost, st));
+    if (mp > 0) ECASQ_CUDA_TRY(cudaMemcpyAsync(qh + kMaxS, Qp, 4 * (size_t)mp, cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaMemsetAsync(ds, 0, sizeof(DevStatus), st));
+    ECASQ_CUDA_TRY(cudaMemsetAsync(counts, 0, 4 * (size_t)(mm + mp), st));
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    for (int r = 1; r < mm; r++)
+        if (!(qh[r] > qh[r - 1])) return ECASQ_EINVAL;
+    for (int r = 1; r < mp; r++)
+        if (!(qh[kMaxS + r] > qh[kMaxS + r - 1])) return ECASQ_EINVAL;
+    int rc = launch_quantize_timeshare(x, d, Qm, mm, mp > 0 ? Qp : Qm, mp, beta, seed, seed_ts, idx, sel, counts, ds,
+                                       num_sms(), st);
+    if (rc) return rc;
+    uint32_t ch[2 * kMaxS];
+    DevStatus h;
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(&h, ds, sizeof(h), cudaMemcpyDeviceToHost, st));
+    if (rate) ECASQ_CUDA_TRY(cudaMemcpyAsync(ch, counts, 4 * (size_t)(mm + mp), cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    if (h.range_err) return ECASQ_ERANGE;
+    if (rate) {
+        // each part coded with its own empirical law: -(1/d) sum_parts sum_r c_r log2(c_r / n_part)
+        double bits = 0.0;
+        for (int part = 0; part < 2; part++) {
+            int off = part ? mm : 0, m = part ? mp : mm;
+            double np_ = 0.0;
+            for (int r = 0; r < m; r++) np_ += (double)ch[off + r];
+            for (int r = 0; r < m; r++)
+                if (ch[off + r]) bits -= (double)ch[off + r] * log2((double)ch[off + r] / np_);
+        }
+        *rate = bits / (double)d;
     }
     return ECASQ_OK;
 }

@@ -88,4 +88,53 @@ int launch_quantize(const float *x, int64_t d, const float *Q, int m, uint64_t s
     return ECASQ_OK;
 }
 
+// Two-way time-sharing (Sec. 7): entry i uses Q+ iff k_s * 2^-24 < beta (binary64,
+// exact), k_s = top 24 bits of SplitMix64(seed_ts + (i+1) * 0x9E3779B97F4A7C15),
+// then rounds within its codebook exactly as k_quantize (seed, same counter i).
+// counts: [mm] for Q-, then [mp] for Q+; sel (may be null): 1 where Q+ was used.
+__global__ void __launch_bounds__(256) k_quantize_timeshare(const float *__restrict__ x, int64_t d,
+                                                            const float *__restrict__ Qm, int mm,
+                                                            const float *__restrict__ Qp, int mp, double beta,
+                                                            uint64_t seed, uint64_t seed_ts, uint8_t *__restrict__ idx,
+                                                            uint8_t *__restrict__ sel, uint32_t *__restrict__ counts,
+                                                            DevStatus *st) {
+    __shared__ float q[2][kMaxS];
+    __shared__ uint32_t hcount[2 * kMaxS];
+    for (int r = threadIdx.x; r < kMaxS; r += blockDim.x) {
+        q[0][r] = r < mm ? Qm[r] : 0.0f;
+        q[1][r] = r < mp ? Qp[r] : 0.0f;
+        hcount[r] = 0;
+        hcount[kMaxS + r] = 0;
+    }
+    __syncthreads();
+    bool bad = false;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < d; i += stride) {
+        uint64_t zs = splitmix64(seed_ts + (uint64_t)(i + 1) * 0x9E3779B97F4A7C15ull);
+        int part = __dmul_rn((double)(uint32_t)(zs >> 40), 0x1p-24) < beta ? 1 : 0;
+        int t = quant_one(x[i], i, q[part], part ? mp : mm, seed, bad);
+        idx[i] = (uint8_t)t;
+        if (sel) sel[i] = (uint8_t)part;
+        atomicAdd(&hcount[part * kMaxS + t], 1u);
+    }
+    if (bad) st->range_err = 1;
+    __syncthreads();
+    for (int r = threadIdx.x; r < mm; r += blockDim.x)
+        if (hcount[r]) atomicAdd(&counts[r], hcount[r]);
+    for (int r = threadIdx.x; r < mp; r += blockDim.x)
+        if (hcount[kMaxS + r]) atomicAdd(&counts[mm + r], hcount[kMaxS + r]);
+}
+
+int launch_quantize_timeshare(const float *x, int64_t d, const float *Qm, int mm, const float *Qp, int mp,
+                              double beta, uint64_t seed, uint64_t seed_ts, uint8_t *idx, uint8_t *sel,
+                              uint32_t *counts, DevStatus *st, int num_sms, cudaStream_t stream) {
+    int64_t blocks = std::min<int64_t>(cdiv(d, 256), (int64_t)num_sms * 8);
+    if (blocks < 1) blocks = 1;
+    note_launch();
+    k_quantize_timeshare<<<(unsigned)blocks, 256, 0, stream>>>(x, d, Qm, mm, Qp, mp, beta, seed, seed_ts, idx, sel,
+                                                               counts, st);
+    ECASQ_LAUNCH_CHECK();
+    return ECASQ_OK;
+}
+
 }  // namespace ecasq

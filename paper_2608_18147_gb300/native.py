@@ -45,6 +45,16 @@ class Result(C.Structure):
         return out
 
 
+class Timeshare(C.Structure):
+    _fields_ = [("beta", C.c_double), ("lambda_plus", C.c_double), ("mse", C.c_double), ("vnmse", C.c_double),
+                ("h_surrogate", C.c_double), ("h_exact", C.c_double), ("plus_mse", C.c_double),
+                ("plus_h_surrogate", C.c_double), ("plus_h_exact", C.c_double), ("m_plus", C.c_int32),
+                ("reserved", C.c_int32)]
+
+    def as_dict(self):
+        return {name: getattr(self, name) for name, _ in self._fields_}
+
+
 class EcasqError(RuntimeError):
     def __init__(self, code, where):
         self.code = code
@@ -78,6 +88,9 @@ def lib():
             "ecasq_solve": (C.c_int, [vp, i64, PP, vp, sz, vp, PR, vp]),
             "ecasq_solve_grid": (C.c_int, [vp, i64, vp, i64, PP, vp, sz, vp, PR, vp]),
             "ecasq_workspace_size_grid": (sz, [i64, i64, i32, u32]),
+            "ecasq_solve_timeshare": (C.c_int, [vp, i64, vp, i64, PP, vp, sz, vp, vp, PR, C.POINTER(Timeshare), vp]),
+            "ecasq_quantize_timeshare": (C.c_int, [vp, i64, vp, i32, vp, i32, dbl, u64, u64, vp, vp, vp, vp, sz, pd,
+                                                   vp]),
             "ecasq_dp_pass": (C.c_int, [vp, i64, i32, pd, i32, u32, vp, sz, vp, pi32, pd, vp]),
             "ecasq_dp_tables": (C.c_int, [vp, sz, i32, vp, vp, pi64, vp]),
             "ecasq_refine": (C.c_int, [vp, i64, vp, i32, dbl, dbl, i32, dbl, u32, vp, sz, PR, vp]),
@@ -101,7 +114,8 @@ def exported_symbols():
     L = lib()
     names = []
     for name in ("ecasq_version", "ecasq_strerror", "ecasq_workspace_size", "ecasq_workspace_size_flags",
-                 "ecasq_solve", "ecasq_solve_grid", "ecasq_workspace_size_grid", "ecasq_dp_pass",
+                 "ecasq_solve", "ecasq_solve_grid", "ecasq_workspace_size_grid", "ecasq_solve_timeshare",
+                 "ecasq_quantize_timeshare", "ecasq_dp_pass",
                  "ecasq_dp_tables", "ecasq_refine", "ecasq_evaluate", "ecasq_quantize", "ecasq_quantize_noalloc",
                  "ecasq_solve_batched",
                  "ecasq_prepare", "ecasq_kernel_launches"):
@@ -214,6 +228,58 @@ def ecasq_solve_grid(x, P, s, budget_bits=0.0, lambda_=-1.0, ws=None, **kw):
                                 _stream())
     _check(rc, "ecasq_solve_grid", ok=(OK, EINFEASIBLE))
     return Q[:res.m].clone(), res.as_dict()
+
+
+def ecasq_solve_timeshare(x, s, budget_bits, P=None, ws=None, **kw):
+    """Budgeted solve with two-way time-sharing (Sec. 7): (Q- tensor, Q+ tensor or empty,
+    result dict of Q-, time-sharing dict).  P: optional permissible set as in ecasq_solve_grid."""
+    torch = _torch()
+    x = _dev_f32(x)
+    d = x.numel()
+    flags = int(kw.get("flags", 0))
+    if P is not None:
+        P = _dev_f32(P)
+        n = P.numel()
+        nb = int(lib().ecasq_workspace_size_grid(d, n, int(s), flags))
+    else:
+        n = 0
+        nb = int(lib().ecasq_workspace_size_flags(d, int(s), 1, flags))
+    if ws is None:
+        if nb == 0:
+            raise EcasqError(EINVAL, "workspace size")
+        ws = torch.empty(nb, dtype=torch.uint8, device="cuda")
+    prm = make_params(s, budget_bits, -1.0, **kw)
+    Qm = torch.zeros(s, dtype=torch.float32, device="cuda")
+    Qp = torch.zeros(s, dtype=torch.float32, device="cuda")
+    res = Result()
+    ts = Timeshare()
+    rc = lib().ecasq_solve_timeshare(_ptr(x), d, _ptr(P) if P is not None else None, n, C.byref(prm), _ptr(ws),
+                                     ws.numel(), _ptr(Qm), _ptr(Qp), C.byref(res), C.byref(ts), _stream())
+    _check(rc, "ecasq_solve_timeshare", ok=(OK, EINFEASIBLE))
+    return Qm[:res.m].clone(), Qp[:ts.m_plus].clone(), res.as_dict(), ts.as_dict()
+
+
+def ecasq_quantize_timeshare(x, Qm, Qp, beta, seed, seed_ts, ws=None, with_sel=True):
+    """Time-shared stochastic quantization (Sec. 7): (idx, sel or None, counts [mm + mp], rate)."""
+    torch = _torch()
+    x = _dev_f32(x)
+    d = x.numel()
+    Qm = _dev_f32(Qm)
+    Qp = _dev_f32(Qp) if Qp is not None and len(Qp) else None
+    mm, mp = Qm.numel(), (Qp.numel() if Qp is not None else 0)
+    if ws is None:
+        ws = torch.empty(256, dtype=torch.uint8, device="cuda")
+    idx = torch.empty(d, dtype=torch.uint8, device="cuda")
+    sel = torch.empty(d, dtype=torch.uint8, device="cuda") if with_sel else None
+    counts = torch.empty(mm + mp, dtype=torch.int32, device="cuda")
+    rate = C.c_double()
+    rc = lib().ecasq_quantize_timeshare(_ptr(x), d, _ptr(Qm), mm, _ptr(Qp) if Qp is not None else None, mp,
+                                        float(beta), C.c_uint64(int(seed) & 0xFFFFFFFFFFFFFFFF),
+                                        C.c_uint64(int(seed_ts) & 0xFFFFFFFFFFFFFFFF), _ptr(idx),
+                                        _ptr(sel) if sel is not None else None, _ptr(counts), _ptr(ws), ws.numel(),
+                                        C.byref(rate), _stream())
+    _check(rc, "ecasq_quantize_timeshare")
+    return idx, sel, counts, rate.value
 
 
 def uniform_grid(x, n):

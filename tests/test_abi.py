@@ -68,6 +68,18 @@ def test_bad_arguments_rejected_before_any_launch():
                          C.byref(res), None) == native.EWORKSPACE
     assert L.ecasq_solve(C.c_void_p(256), 10, C.byref(prm), C.c_void_p(256), 16, C.c_void_p(256),
                          C.byref(res), None) == native.EWORKSPACE
+    # time-sharing needs a budget search without refinement (Sec. 7)
+    ts = native.Timeshare()
+    v = C.c_void_p(256)
+    for bad in (native.make_params(8, 2.0, 0.5), native.make_params(8, 2.0, refine_max_rounds=2)):
+        assert L.ecasq_solve_timeshare(v, 10, None, 0, C.byref(bad), v, 1 << 30, v, v, C.byref(res), C.byref(ts),
+                                       None) == native.EINVAL
+    assert L.ecasq_solve_timeshare(v, 10, None, 0, C.byref(prm), v, 1 << 30, v, v, C.byref(res), None,
+                                   None) == native.EINVAL
+    rate = C.c_double()
+    for beta, mp in ((1.5, 2), (-0.1, 2), (0.5, 0)):
+        assert L.ecasq_quantize_timeshare(v, 10, v, 2, v, mp, beta, 1, 2, v, None, v, v, 256, C.byref(rate),
+                                          None) == native.EINVAL
 
 
 def test_product_path_does_not_touch_the_oracle():
