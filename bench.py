@@ -11,6 +11,12 @@ Prints one JSON line (rank 0).  `value` is min-plus candidate evaluations per
 second over the whole job (inputs resident in HBM); `e2e` is the same metric
 through the C ABI with host buffers; `roofline` relates the min-plus kernel to
 the FP32-pipe issue peak; `cpu_baseline` is the CPU oracle on a bounded sample.
+
+Other rows of the path, each timed the same way on the chosen --config:
+  --mode grid       the codebook drawn from a uniform min-max grid of --grid values
+                    (Sec. 5 / App. E general P); metric: solves/s
+  --mode timeshare  the budgeted solve with two-way time-sharing (Sec. 7) and the
+                    time-shared encode; metric: solves/s
 """
 import argparse
 import json
@@ -47,6 +53,8 @@ def parse():
     ap.add_argument("--config", default="studentt_d131072_s16")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--mode", default="solve", choices=["solve", "grid", "timeshare"])
+    ap.add_argument("--grid", type=int, default=256, help="grid size for --mode grid")
     return ap.parse_args()
 
 
@@ -155,6 +163,71 @@ def run_reference(args, cfg, x):
     print(json.dumps(out), flush=True)
 
 
+def run_other_mode(args, cfg, x_np):
+    """--mode grid / timeshare: solves per second of that entry point on one GPU,
+    timed with CUDA events around `steps` solves (+ encodes), inputs in HBM."""
+    import torch
+    import paper_2608_18147_gb300 as E
+    s, budget = cfg["s"], cfg["budgets"][0]
+    d = x_np.size
+    x = torch.as_tensor(x_np).cuda()
+    idx = torch.empty(d, dtype=torch.uint8, device="cuda")
+    counts = torch.empty(2 * s, dtype=torch.int32, device="cuda")
+    qws = torch.empty(256, dtype=torch.uint8, device="cuda")
+    flags = E.TIME_KERNELS
+    if args.mode == "grid":
+        g = torch.as_tensor(E.uniform_grid(x_np, args.grid)).cuda()
+        ws = torch.empty(int(E.lib().ecasq_workspace_size_grid(d, g.numel(), s, flags)), dtype=torch.uint8,
+                         device="cuda")
+
+        def step():
+            Q, res = E.ecasq_solve_grid(x, g, s, budget_bits=budget, ws=ws, flags=flags)
+            _, _, he = E.ecasq_quantize(x, Q, seed=12345, ws=qws, idx=idx, counts=counts[:Q.numel()])
+            return res, {}
+    else:
+        need = E.ecasq_workspace_size_flags(d, s, 1, E.RESIDENT_COSTS)
+        if 0 < need <= 0.6 * torch.cuda.mem_get_info()[0]:
+            flags |= E.RESIDENT_COSTS
+        ws = E.workspace(d, s, flags=flags)
+
+        def step():
+            Qm, Qp, res, ts = E.ecasq_solve_timeshare(x, s, budget, ws=ws, flags=flags)
+            _, _, _, rate = E.ecasq_quantize_timeshare(x, Qm, Qp, ts["beta"], 12345, 678, ws=qws)
+            ts["rate_emp"] = rate
+            return res, ts
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    launches0 = E.ecasq_kernel_launches()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    out_res = []
+    with ClockSampler(int(os.environ.get("LOCAL_RANK", "0"))) as clk:
+        ev0.record(stream)
+        for _ in range(args.steps):
+            out_res.append(step())
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    ms = ev0.elapsed_time(ev1)
+    res, ts = out_res[-1]
+    dp_ms = sum(r["dp_kernel_ms"] for r, _ in out_res)
+    dp_launches = sum(r["dp_kernel_launches"] for r, _ in out_res)
+    out = {"metric": "ECASQ %s solve: solves/s" % args.mode, "value": args.steps / (ms / 1000.0),
+           "unit": "solves/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": ms / args.steps, "higher_is_better": True, "vs_baseline": None,
+           "dtype": "f64" if args.mode == "grid" else "f32 (fp64 exact stage)", "data": "synthetic",
+           "config": {"workload": args.config, "mode": args.mode, "d": d, "s": s, "budget_bits": budget,
+                      "grid": args.grid if args.mode == "grid" else None,
+                      "resident_costs": bool(flags & E.RESIDENT_COSTS)},
+           "solve": {"m": res["m"], "p": res["p"], "lambda": res["lambda"], "vnmse": res["vnmse"],
+                     "h_surrogate": res["h_surrogate"], "h_exact": res["h_exact"], "passes": res["passes"],
+                     "candidates_per_solve": res["candidates"], "dp_ms_per_solve": dp_ms / args.steps,
+                     "dp_launches_per_solve": dp_launches / args.steps},
+           "timeshare": ts or None, "gpu_launches": E.ecasq_kernel_launches() - launches0,
+           "clocks": clk.summary()}
+    print(json.dumps(out), flush=True)
+
+
 def main():
     args = parse()
     from paper_2608_18147_gb300 import workloads
@@ -167,6 +240,9 @@ def main():
     import numpy as np
     import torch
     import paper_2608_18147_gb300 as E
+    if args.mode != "solve":
+        run_other_mode(args, cfg, x_np)
+        return
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))

@@ -150,9 +150,13 @@ int ecasq_solve(const float *x, int64_t d, const ecasq_params_t *prm, void *ws, 
  *   Q   device [s] output, values of P.  res->p = n.
  * Refinement moves interior values only; the first and last stay where the DP
  * put them.
- * The DP runs the binary64 reference kernel (the fast kernel's recurrences need
- * every slab's mass at a candidate value, true only for P = X), so this entry point
- * is meant for the small sets that make P worth using (p << d).
+ * DP: the interval costs of every pair of P are evaluated once per call in binary64
+ * (24 bytes per pair, n <= 32768) and each layer is filtered in fp32 with a certified
+ * band whose members are re-scored in binary64, so the result equals the binary64
+ * reference kernel's (ECASQ_DP_REFERENCE forces that kernel; sets above 32768
+ * values use it).  The fast kernel of ecasq_solve is not used: its recurrences need
+ * every slab's mass at a candidate value, true only for P = X.  ECASQ_RESIDENT_COSTS
+ * is ignored.
  * Workspace: ecasq_workspace_size_grid(d, n, s, flags).  Synchronises `stream`. */
 size_t ecasq_workspace_size_grid(int64_t d, int64_t n, int32_t s, uint32_t flags);
 int ecasq_solve_grid(const float *x, int64_t d, const float *P, int64_t n, const ecasq_params_t *prm, void *ws,

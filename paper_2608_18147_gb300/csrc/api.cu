@@ -40,6 +40,9 @@ int launch_quantize_timeshare(const float *x, int64_t d, const float *Qm, int mm
                               double beta, uint64_t seed, uint64_t seed_ts, uint8_t *idx, uint8_t *sel,
                               uint32_t *counts, DevStatus *st, int num_sms, cudaStream_t stream);
 size_t fast_dp_band_bytes(int64_t d, int32_t s);
+size_t grid_pairs_bytes(int64_t n);
+int launch_dp_grid(const Prefix &P, const double *lamp, int G, int s, double *dp64, int32_t *bp, float *dp32,
+                   void *pairs, bool build_pairs, int num_sms, cudaStream_t st);
 
 static std::atomic<long long> g_launches{0};
 void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
@@ -99,6 +102,8 @@ size_t make_layout(int64_t d, int32_t s, int64_t rows, Layout *L) {
     L->band = take(fast_dp_band_bytes(d, s));
     L->costs = 0;
     L->costs_bytes = 0;
+    L->gpairs = 0;
+    L->gpairs_bytes = 0;
     L->total = off;
     L->d = d;
     L->s = s;
@@ -239,6 +244,10 @@ static int dp_pass_prepared(void *ws, const Layout &L, const Prefix &P, int s, c
     int rc;
     if (flags & ECASQ_DP_REFERENCE) {
         rc = launch_dp_reference(P, lamp, G, s, dp64, bp, st);
+    } else if (L.gpairs_bytes) {
+        rc = launch_dp_grid(P, lamp, G, s, dp64, bp, wsp<float>(ws, L.dp32), wsp<void>(ws, L.gpairs), !*costs_built,
+                            num_sms(), st);
+        if (rc == ECASQ_OK) *costs_built = true;
     } else {
         float *costs = L.costs_bytes ? wsp<float>(ws, L.costs) : nullptr;
         rc = launch_dp_fast(P, lamp, G, s, ws, L, st, (flags & ECASQ_EXACT_S) != 0, (flags & ECASQ_EXACT_TABLES) != 0,
@@ -683,8 +692,11 @@ int ecasq_solve(const float *x, int64_t d, const ecasq_params_t *prm, void *ws, 
 }
 
 size_t ecasq_workspace_size_grid(int64_t d, int64_t n, int32_t s, uint32_t flags) {
-    if (n < 1 || n >= ((int64_t)1 << 31)) return 0;
-    return ecasq_workspace_size_flags(std::max(d, n), s, 1, flags);
+    (void)flags;  // the grid DP keeps its own pair cache; resident tiles are not used
+    if (d < 1 || d >= ((int64_t)1 << 31) || n < 1 || n >= ((int64_t)1 << 31) || s < 2 || s > kMaxS) return 0;
+    Layout L;
+    make_layout(std::max(d, n), s, 1, &L);
+    return L.total + align256(grid_pairs_bytes(n));
 }
 
 // The histogram view over a permissible set P (Sec. 5, App. E): prepare x, then
@@ -695,9 +707,13 @@ static int prepare_grid(const float *x, int64_t d, const float *Pg, int64_t n, c
     Layout &L = *Lo;
     make_layout(dmax, prm->s, 1, &L);
     L.d = dmax;
-    int rc = add_resident_costs(prm->flags, &L);
-    if (rc) return rc;
-    rc = check_ws(ws, ws_bytes, L);
+    size_t gb = grid_pairs_bytes(n);
+    if (gb) {
+        L.gpairs = L.total;
+        L.gpairs_bytes = gb;
+        L.total += align256(gb);
+    }
+    int rc = check_ws(ws, ws_bytes, L);
     if (rc) return rc;
     int64_t pX;
     double n2;
@@ -726,6 +742,7 @@ static int prepare_grid(const float *x, int64_t d, const float *Pg, int64_t n, c
     *Po = make_prefix(ws, L, n, d);
     Po->nL = h.grid_nL;
     Po->nR = h.grid_nR;
+    Po->scale32 = (n2 > 0.0 && std::isfinite(n2)) ? std::ldexp(1.0, -std::ilogb(n2)) : 1.0;
     *n2o = n2;
     return ECASQ_OK;
 }
@@ -743,9 +760,9 @@ int ecasq_solve_grid(const float *x, int64_t d, const float *Pg, int64_t n, cons
     if (rc) return rc;
     // The fast kernel's fp32 recurrences add one candidate at a time and assume each
     // slab's mass sits at its right end (true for the unique values of x only); a grid
-    // runs the reference DP (binary64 candidates from the App. E formulas).
+    // runs the grid DP (cached pair costs), or beyond kGridPairsMax the reference DP.
     ecasq_params_t pg = *prm;
-    pg.flags |= ECASQ_DP_REFERENCE;
+    if (!L.gpairs_bytes) pg.flags |= ECASQ_DP_REFERENCE;
     return solve_prepared(ws, L, P, d, n2, &pg, Q, res, st);
 }
 
@@ -765,7 +782,7 @@ int ecasq_solve_timeshare(const float *x, int64_t d, const float *Pg, int64_t n,
     int rc;
     if (Pg) {
         rc = prepare_grid(x, d, Pg, n, prm, ws, ws_bytes, &L, &P, &n2, st);
-        pg.flags |= ECASQ_DP_REFERENCE;
+        if (rc == ECASQ_OK && !L.gpairs_bytes) pg.flags |= ECASQ_DP_REFERENCE;
     } else {
         rc = prepare_plain(x, d, prm, ws, ws_bytes, &L, &P, &n2, st);
     }

@@ -73,6 +73,8 @@ struct Layout {
     size_t band;           // fast DP band lists
     size_t costs;          // resident interval-cost tiles (ECASQ_RESIDENT_COSTS), after everything else
     size_t costs_bytes;    // 0 when absent
+    size_t gpairs;         // grid DP pair cache (permissible sets up to kGridPairsMax values)
+    size_t gpairs_bytes;   // 0 when absent
     size_t total;
     int64_t d;
     int32_t s;
@@ -169,7 +171,11 @@ struct Prefix {
     int64_t ps;           // DP-table row stride, table_stride(p)
     int64_t nL = 1;       // first-value set L = {0..nL-1}, last-value set R = {p-nR..p-1}
     int64_t nR = 1;       // (Sec. 5); both 1 when the candidates are the unique values of x
+    double scale32 = 1.0; // grid DP: power of two that brings ||X||^2 into [1, 2) for fp32 copies
 };
+
+// Largest permissible set whose pair costs the grid DP caches (24 bytes per pair).
+constexpr int64_t kGridPairsMax = 32768;
 
 __device__ __forceinline__ dd load_dd(const double *a, int64_t p, int64_t t) { return {a[t], a[p + 1 + t]}; }
 

@@ -347,8 +347,9 @@ int launch_rows_gather(const RowsData &R, const int32_t *a, const int32_t *m, in
 }
 
 // ----------------------------------------------------------- host launchers
-int launch_dp_reference(const Prefix &P, const double *lamp, int G, int s, double *dp64, int32_t *bp,
-                        cudaStream_t st) {
+// Tables cleared (dp = +inf, bp = -1) and layer 2 (eq. apx_base) filled.
+int launch_dp_clear_base(const Prefix &P, const double *lamp, int G, int s, double *dp64, int32_t *bp,
+                         cudaStream_t st) {
     Lams lam{};
     for (int g = 0; g < G; g++) lam.v[g] = lamp[g];
     note_launch();
@@ -359,6 +360,15 @@ int launch_dp_reference(const Prefix &P, const double *lamp, int G, int s, doubl
         k_dp_base<<<(unsigned)cdiv(P.p - 1, 128), 128, 0, st>>>(P, lam, G, s, dp64, bp);
         ECASQ_LAUNCH_CHECK();
     }
+    return ECASQ_OK;
+}
+
+int launch_dp_reference(const Prefix &P, const double *lamp, int G, int s, double *dp64, int32_t *bp,
+                        cudaStream_t st) {
+    Lams lam{};
+    for (int g = 0; g < G; g++) lam.v[g] = lamp[g];
+    int rc = launch_dp_clear_base(P, lamp, G, s, dp64, bp, st);
+    if (rc != ECASQ_OK) return rc;
     timer_begin(st);
     for (int i = 3; i <= s; i++) {
         if (P.p < i) break;

@@ -105,3 +105,28 @@ def test_appF1_example_on_the_gpu(E, oracle_mod):
     Q, res = E.ecasq_solve_grid(x, P, 2, budget_bits=0.95)
     _check(res, oracle_mod.solve_budget(x, 2, 0.95, grid=P), Q)
     assert Q.cpu().numpy().tolist() == [0.0, 4.0]
+
+
+@pytest.mark.parametrize("case", ["uniform", "wide", "dynamic_range", "ties"])
+def test_grid_dp_equals_reference_kernel(E, case):
+    """The grid DP (cached pair costs, fp32 band, binary64 re-scoring) returns what the
+    binary64 reference kernel returns, bit for bit, at every evaluated multiplier."""
+    rng = np.random.default_rng(5)
+    if case == "uniform":
+        x = workloads.student_t(30000, 8, scale=1.0)
+        g = E.uniform_grid(x, 2000)
+    elif case == "wide":
+        x = workloads.signed_lognormal(8000, 12)
+        g = wide_grid(x, 700, 1.0, 3.0)
+    elif case == "dynamic_range":    # fp32 copies of tiny intervals underflow after scaling
+        x = np.concatenate([rng.standard_normal(3000) * 1e-25, rng.standard_normal(40) * 1e15]).astype(np.float32)
+        g = np.unique(np.concatenate([np.sort(x)[::7], [x.min(), x.max()]]).astype(np.float32))
+    else:                            # many zero-mass intervals: exact ties between candidates
+        x = np.repeat(np.arange(12, dtype=np.float32), 50)
+        g = np.linspace(0, 11, 400).astype(np.float32)
+    for b in (1.0, 2.5):
+        Q1, r1 = E.ecasq_solve_grid(x, g, 8, budget_bits=b)
+        Q2, r2 = E.ecasq_solve_grid(x, g, 8, budget_bits=b, flags=E.DP_REFERENCE)
+        np.testing.assert_array_equal(Q1.cpu().numpy(), Q2.cpu().numpy())
+        for k in ("status", "lambda", "mse", "h_surrogate", "h_exact", "passes", "lambdas_evaluated"):
+            assert r1[k] == r2[k], k
