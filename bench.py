@@ -17,6 +17,8 @@ Other rows of the path, each timed the same way on the chosen --config:
                     (Sec. 5 / App. E general P); metric: solves/s
   --mode timeshare  the budgeted solve with two-way time-sharing (Sec. 7) and the
                     time-shared encode; metric: solves/s
+  --mode opt        one pass of the optimal DP (Sec. 4) at 8 multipliers over a uniform
+                    grid of --grid values; metric: candidate evaluations/s
 """
 import argparse
 import json
@@ -53,7 +55,7 @@ def parse():
     ap.add_argument("--config", default="studentt_d131072_s16")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--mode", default="solve", choices=["solve", "grid", "timeshare"])
+    ap.add_argument("--mode", default="solve", choices=["solve", "grid", "timeshare", "opt"])
     ap.add_argument("--grid", type=int, default=256, help="grid size for --mode grid")
     return ap.parse_args()
 
@@ -175,6 +177,9 @@ def run_other_mode(args, cfg, x_np):
     counts = torch.empty(2 * s, dtype=torch.int32, device="cuda")
     qws = torch.empty(256, dtype=torch.uint8, device="cuda")
     flags = E.TIME_KERNELS
+    if args.mode == "opt":
+        run_opt_mode(args, cfg, x_np)
+        return
     if args.mode == "grid":
         g = torch.as_tensor(E.uniform_grid(x_np, args.grid)).cuda()
         ws = torch.empty(int(E.lib().ecasq_workspace_size_grid(d, g.numel(), s, flags)), dtype=torch.uint8,
@@ -225,6 +230,55 @@ def run_other_mode(args, cfg, x_np):
                      "dp_launches_per_solve": dp_launches / args.steps},
            "timeshare": ts or None, "gpu_launches": E.ecasq_kernel_launches() - launches0,
            "clocks": clk.summary()}
+    print(json.dumps(out), flush=True)
+
+
+def opt_candidates(n, s, G, nL=1):
+    """Candidates of the optimal DP's layers 3..s (Sec. 4): for each l, the finite
+    predecessors k (k < nL at i = 3, i - 3 <= k < l above) times the outputs j > l, x G."""
+    import numpy as np
+    l = np.arange(n - 1, dtype=np.int64)
+    c = 0
+    for i in range(3, s + 1):
+        nk = np.minimum(nL, l) if i == 3 else np.maximum(l - (i - 3), 0)
+        c += int(np.sum(nk * (n - 1 - l)))
+    return c * G
+
+
+def run_opt_mode(args, cfg, x_np):
+    import numpy as np
+    import torch
+    import paper_2608_18147_gb300 as E
+    s = cfg["s"]
+    d = x_np.size
+    g = E.uniform_grid(x_np, args.grid)
+    n = g.size
+    lams = [0.0] + list(np.geomspace(1e-6, 1e2, 7))
+    x = torch.as_tensor(x_np).cuda()
+    gd = torch.as_tensor(g).cuda()
+    ws = torch.empty(int(E.lib().ecasq_workspace_size_opt(d, n, s, len(lams))), dtype=torch.uint8, device="cuda")
+    for _ in range(args.warmup):
+        E.ecasq_opt_dp(x, s, lams, P=gd, ws=ws)
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    launches0 = E.ecasq_kernel_launches()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(int(os.environ.get("LOCAL_RANK", "0"))) as clk:
+        ev0.record(stream)
+        for _ in range(args.steps):
+            Q, m, met = E.ecasq_opt_dp(x, s, lams, P=gd, ws=ws)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    ms = ev0.elapsed_time(ev1) / args.steps
+    cand = opt_candidates(n, s, len(lams))
+    out = {"metric": "ECASQ optimal DP pass (Sec. 4): candidate evals/s", "value": cand / (ms / 1000.0),
+           "unit": "candidate evals/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": ms, "higher_is_better": True, "vs_baseline": None,
+           "dtype": "f32 (fp64 band re-scoring)", "data": "synthetic",
+           "config": {"workload": args.config, "mode": "opt", "d": d, "s": s, "grid": n, "multipliers": len(lams)},
+           "pass": {"candidates": cand, "m": list(m), "optimum": met[:, 0].tolist(), "vnmse": (met[:, 1] / float(
+               np.sum(x_np.astype(np.float64) ** 2))).tolist()},
+           "gpu_launches": E.ecasq_kernel_launches() - launches0, "clocks": clk.summary()}
     print(json.dumps(out), flush=True)
 
 

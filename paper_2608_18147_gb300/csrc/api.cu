@@ -43,6 +43,10 @@ size_t fast_dp_band_bytes(int64_t d, int32_t s);
 size_t grid_pairs_bytes(int64_t n);
 int launch_dp_grid(const Prefix &P, const double *lamp, int G, int s, double *dp64, int32_t *bp, float *dp32,
                    void *pairs, bool build_pairs, int num_sms, cudaStream_t st);
+size_t opt_pairs_bytes(int64_t n);
+size_t opt_tables_bytes(int64_t n, int s, int G);
+int launch_opt_dp(const Prefix &P, const double *lamp, int G, int s, int exact_s, void *pairs, bool build_pairs,
+                  void *tables, int32_t *qidx, int32_t *mcount, double *metrics, int num_sms, cudaStream_t st);
 
 static std::atomic<long long> g_launches{0};
 void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
@@ -699,6 +703,10 @@ size_t ecasq_workspace_size_grid(int64_t d, int64_t n, int32_t s, uint32_t flags
     return L.total + align256(grid_pairs_bytes(n));
 }
 
+static int grid_view(const float *x, int64_t d, const float *Pg, int64_t n, void *ws, const Layout &L, Prefix *Po,
+                     double *n2o, cudaStream_t st);
+static double scale32_of(double n2);
+
 // The histogram view over a permissible set P (Sec. 5, App. E): prepare x, then
 // gather the prefix sums at the points of P; P->nL, P->nR receive |L|, |R|.
 static int prepare_grid(const float *x, int64_t d, const float *Pg, int64_t n, const ecasq_params_t *prm, void *ws,
@@ -715,9 +723,20 @@ static int prepare_grid(const float *x, int64_t d, const float *Pg, int64_t n, c
     }
     int rc = check_ws(ws, ws_bytes, L);
     if (rc) return rc;
+    return grid_view(x, d, Pg, n, ws, L, Po, n2o, st);
+}
+
+static double scale32_of(double n2) {
+    return (n2 > 0.0 && std::isfinite(n2)) ? std::ldexp(1.0, -std::ilogb(n2)) : 1.0;
+}
+
+// Sort / histogram / prefix sums of x, then the grid view of P in place of the
+// unique values (needs L.dp64 as scratch for the unique-value arrays).
+static int grid_view(const float *x, int64_t d, const float *Pg, int64_t n, void *ws, const Layout &L, Prefix *Po,
+                     double *n2o, cudaStream_t st) {
     int64_t pX;
     double n2;
-    rc = prepare_device(x, d, ws, L, st, &pX, &n2);
+    int rc = prepare_device(x, d, ws, L, st, &pX, &n2);
     if (rc) return rc;
     // the unique-value view moves to scratch (the fp64 DP table area), the grid view takes its place
     char *scr = wsp<char>(ws, L.dp64);
@@ -742,7 +761,7 @@ static int prepare_grid(const float *x, int64_t d, const float *Pg, int64_t n, c
     *Po = make_prefix(ws, L, n, d);
     Po->nL = h.grid_nL;
     Po->nR = h.grid_nR;
-    Po->scale32 = (n2 > 0.0 && std::isfinite(n2)) ? std::ldexp(1.0, -std::ilogb(n2)) : 1.0;
+    Po->scale32 = scale32_of(n2);
     *n2o = n2;
     return ECASQ_OK;
 }
@@ -956,6 +975,81 @@ int ecasq_quantize_noalloc(const float *x, int64_t d, const float *Q, int32_t m,
         }
         *h_emp = he;
     }
+    return ECASQ_OK;
+}
+
+// Optimal DP (Sec. 4): base layout, then the pair quantities C, U, D and the
+// tables dp, bk of G multipliers.
+static bool opt_layout(int64_t d, int64_t n, int32_t s, int32_t G, Layout *L, size_t *pairs_off, size_t *tables_off) {
+    if (d < 1 || d >= ((int64_t)1 << 31) || n < 1 || n > kOptMax || s < 2 || s > kMaxS || G < 1 || G > kMaxG)
+        return false;
+    make_layout(std::max(d, n), s, 1, L);
+    L->d = std::max(d, n);
+    *pairs_off = L->total;
+    *tables_off = *pairs_off + align256(opt_pairs_bytes(n));
+    L->total = *tables_off + align256(opt_tables_bytes(n, s, G));
+    return true;
+}
+
+size_t ecasq_workspace_size_opt(int64_t d, int64_t n, int32_t s, int32_t G) {
+    Layout L;
+    size_t po, to;
+    return opt_layout(d, n, s, G, &L, &po, &to) ? L.total : 0;
+}
+
+int ecasq_opt_dp(const float *x, int64_t d, const float *Pg, int64_t n, int32_t s, const double *lambdas, int32_t G,
+                 uint32_t flags, void *ws, size_t ws_bytes, float *Q_out, int32_t *m_out, double *metrics,
+                 ecasq_stream_t stream) {
+    if (!x || !lambdas || !Q_out || !m_out || !metrics || d < 1 || d >= ((int64_t)1 << 31) || G < 1 || G > kMaxG ||
+        s < 2 || s > kMaxS)
+        return ECASQ_EINVAL;
+    for (int g = 0; g < G; g++)
+        if (!(lambdas[g] >= 0.0) || !std::isfinite(lambdas[g])) return ECASQ_EINVAL;
+    if (Pg && (n < 1 || n > kOptMax)) return ECASQ_EINVAL;
+    if (!Pg && d > kOptMax) return ECASQ_EINVAL;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const int64_t nmax = Pg ? n : d;
+    Layout L;
+    size_t pairs_off, tables_off;
+    if (!opt_layout(d, nmax, s, G, &L, &pairs_off, &tables_off)) return ECASQ_EINVAL;
+    int rc = check_ws(ws, ws_bytes, L);
+    if (rc) return rc;
+    Prefix P;
+    double n2;
+    if (Pg) {
+        rc = grid_view(x, d, Pg, n, ws, L, &P, &n2, st);
+        if (rc) return rc;
+    } else {
+        int64_t p;
+        rc = prepare_device(x, d, ws, L, st, &p, &n2);
+        if (rc) return rc;
+        P = make_prefix(ws, L, p, d);
+        P.scale32 = scale32_of(n2);
+    }
+    int32_t *qidx = wsp<int32_t>(ws, L.qidx);
+    int32_t *mc = wsp<int32_t>(ws, L.mcount);
+    double *met = wsp<double>(ws, L.metrics);
+    if (P.p == 1) {
+        ECASQ_CUDA_TRY(cudaMemcpyAsync(Q_out, P.v, 4, cudaMemcpyDeviceToDevice, st));
+        ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+        for (int g = 0; g < G; g++) {
+            m_out[g] = 1;
+            for (int r = 0; r < 4; r++) metrics[4 * g + r] = 0.0;
+        }
+        return ECASQ_OK;
+    }
+    double lamp[kMaxG];
+    for (int g = 0; g < G; g++) lamp[g] = lambdas[g] * n2;
+    rc = launch_opt_dp(P, lamp, G, s, (flags & ECASQ_EXACT_S) ? 1 : 0, wsp<void>(ws, pairs_off), true,
+                       wsp<void>(ws, tables_off), qidx, mc, met, num_sms(), st);
+    if (rc) return rc;
+    rc = launch_gather_q(P.v, qidx, mc, G, s, Q_out, st);
+    if (rc) return rc;
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(m_out, mc, sizeof(int32_t) * G, cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(metrics, met, sizeof(double) * 4 * G, cudaMemcpyDeviceToHost, st));
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    for (int g = 0; g < G; g++)
+        if (m_out[g] < 1) return ECASQ_EINFEASIBLE;
     return ECASQ_OK;
 }
 

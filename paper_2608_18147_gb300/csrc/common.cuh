@@ -176,6 +176,8 @@ struct Prefix {
 
 // Largest permissible set whose pair costs the grid DP caches (24 bytes per pair).
 constexpr int64_t kGridPairsMax = 32768;
+// Largest candidate set of the optimal DP (Sec. 4): one block row per l in a launch.
+constexpr int64_t kOptMax = 16384;
 
 __device__ __forceinline__ dd load_dd(const double *a, int64_t p, int64_t t) { return {a[t], a[p + 1 + t]}; }
 
@@ -210,6 +212,39 @@ __device__ __forceinline__ double phi_exact(const Prefix &P, double U, double D,
 __device__ __forceinline__ double phi_first_at(const Prefix &P, int64_t a, double U, double D) {
     double dd_ = (double)P.d;
     return __dadd_rn(hfun(__ddiv_rn(U, dd_)), hfun(__ddiv_rn(__dadd_rn(D, (double)P.w[a]), dd_)));
+}
+
+// Metrics of codebook a[0..m-1] (unique indices): MSE, H(I,B), H(Xhat), summed
+// in interval order exactly as the definitions list them (Sec. 2, Sec. 3,
+// eq. apx_additive_entropy).  One warp; lanes evaluate intervals, lane 0 sums.
+static __device__ __noinline__ void eval_codebook_warp(const Prefix &P, const int32_t *a, int m, double *out3, double *scratch) {
+    // scratch: 4 * kMaxS doubles (C, Phi, U, D per interval)
+    int lane = threadIdx.x & 31;
+    for (int r = lane; r + 1 < m; r += 32) {
+        double C, U, D;
+        pair_exact(P, a[r], a[r + 1], C, U, D);
+        scratch[r] = C;
+        scratch[kMaxS + r] = r == 0 ? phi_first_at(P, a[0], U, D) : phi_exact(P, U, D, false);
+        scratch[2 * kMaxS + r] = U;
+        scratch[3 * kMaxS + r] = D;
+    }
+    __syncwarp();
+    if (lane == 0) {
+        double dd_ = (double)P.d;
+        if (m < 2) { out3[0] = 0.0; out3[1] = 0.0; out3[2] = 0.0; return; }
+        double mse = 0.0, hs = 0.0, hx = 0.0, prevU = 0.0;
+        for (int r = 0; r + 1 < m; r++) {
+            mse = __dadd_rn(mse, scratch[r]);
+            hs = __dadd_rn(hs, scratch[kMaxS + r]);
+            double D = scratch[3 * kMaxS + r];
+            double f = (r == 0) ? __dadd_rn((double)P.w[a[0]], D) : __dadd_rn(prevU, D);
+            hx = __dadd_rn(hx, hfun(__ddiv_rn(f, dd_)));
+            prevU = scratch[2 * kMaxS + r];
+        }
+        hx = __dadd_rn(hx, hfun(__ddiv_rn(prevU, dd_)));
+        out3[0] = mse; out3[1] = hs; out3[2] = hx;
+    }
+    __syncwarp();
 }
 
 // -------------------------------------------------------------- host helpers

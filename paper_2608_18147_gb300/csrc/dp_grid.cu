@@ -89,12 +89,12 @@ __global__ void __launch_bounds__(256) k_grid_layer(GridArgs A, int i) {
         for (int g = 0; g < kMaxG; g++)
             if (g < G) m[g] = fminf(m[g], __fadd_rn(A.dp32[g_at(A, g, i - 1, k)], __fmaf_rn(A.lam32[g], cf.y, cf.x)));
     }
-    double T[kMaxG];
+    float T[kMaxG];  // rounded down to fp32: for an fp32 candidate c, c <= T32 exactly when c <= T
 #pragma unroll
     for (int g = 0; g < kMaxG; g++) {
         float v = m[g];
         for (int o = 16; o > 0; o >>= 1) v = fminf(v, __shfl_xor_sync(0xffffffffu, v, o));
-        T[g] = __dadd_rn(__dmul_rn((double)v, 1.0 + 10.0 * 0x1p-24), A.slack[g]);
+        T[g] = __double2float_rd(__dadd_rn(__dmul_rn((double)v, 1.0 + 10.0 * 0x1p-24), A.slack[g]));
     }
     double best[kMaxG];
     int32_t arg[kMaxG];
@@ -106,7 +106,7 @@ __global__ void __launch_bounds__(256) k_grid_layer(GridArgs A, int i) {
         for (int g = 0; g < kMaxG; g++) {
             if (g < G) {
                 float v = __fadd_rn(A.dp32[g_at(A, g, i - 1, k)], __fmaf_rn(A.lam32[g], cf.y, cf.x));
-                if ((double)v <= T[g]) {
+                if (v <= T[g]) {
                     double2 e = A.pc64[tb + k];
                     double c = __dadd_rn(A.dp64[g_at(A, g, i - 1, k)], __dadd_rn(e.x, __dmul_rn(A.lam64[g], e.y)));
                     if (c < best[g]) { best[g] = c; arg[g] = (int32_t)k; }  // k ascends per lane

@@ -84,39 +84,6 @@ __global__ void __launch_bounds__(128) k_dp_layer_ref(Prefix P, Lams lam, int G,
     }
 }
 
-// Metrics of codebook a[0..m-1] (unique indices): MSE, H(I,B), H(Xhat), summed
-// in interval order exactly as the definitions list them (Sec. 2, Sec. 3,
-// eq. apx_additive_entropy).  One warp; lanes evaluate intervals, lane 0 sums.
-__device__ void eval_codebook_warp(const Prefix &P, const int32_t *a, int m, double *out3, double *scratch) {
-    // scratch: 4 * kMaxS doubles (C, Phi, U, D per interval)
-    int lane = threadIdx.x & 31;
-    for (int r = lane; r + 1 < m; r += 32) {
-        double C, U, D;
-        pair_exact(P, a[r], a[r + 1], C, U, D);
-        scratch[r] = C;
-        scratch[kMaxS + r] = r == 0 ? phi_first_at(P, a[0], U, D) : phi_exact(P, U, D, false);
-        scratch[2 * kMaxS + r] = U;
-        scratch[3 * kMaxS + r] = D;
-    }
-    __syncwarp();
-    if (lane == 0) {
-        double dd_ = (double)P.d;
-        if (m < 2) { out3[0] = 0.0; out3[1] = 0.0; out3[2] = 0.0; return; }
-        double mse = 0.0, hs = 0.0, hx = 0.0, prevU = 0.0;
-        for (int r = 0; r + 1 < m; r++) {
-            mse = __dadd_rn(mse, scratch[r]);
-            hs = __dadd_rn(hs, scratch[kMaxS + r]);
-            double D = scratch[3 * kMaxS + r];
-            double f = (r == 0) ? __dadd_rn((double)P.w[a[0]], D) : __dadd_rn(prevU, D);
-            hx = __dadd_rn(hx, hfun(__ddiv_rn(f, dd_)));
-            prevU = scratch[2 * kMaxS + r];
-        }
-        hx = __dadd_rn(hx, hfun(__ddiv_rn(prevU, dd_)));
-        out3[0] = mse; out3[1] = hs; out3[2] = hx;
-    }
-    __syncwarp();
-}
-
 // eq. apx_final over i and j in R (smallest i, then smallest j, among exact minima;
 // i = s only with EXACT_S) and the backpointer walk down to the first value
 // a = bp(2, .), then the metrics of the traced codebook.  Block g = one multiplier,

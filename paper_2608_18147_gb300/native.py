@@ -88,6 +88,8 @@ def lib():
             "ecasq_solve": (C.c_int, [vp, i64, PP, vp, sz, vp, PR, vp]),
             "ecasq_solve_grid": (C.c_int, [vp, i64, vp, i64, PP, vp, sz, vp, PR, vp]),
             "ecasq_workspace_size_grid": (sz, [i64, i64, i32, u32]),
+            "ecasq_workspace_size_opt": (sz, [i64, i64, i32, i32]),
+            "ecasq_opt_dp": (C.c_int, [vp, i64, vp, i64, i32, pd, i32, u32, vp, sz, vp, pi32, pd, vp]),
             "ecasq_solve_timeshare": (C.c_int, [vp, i64, vp, i64, PP, vp, sz, vp, vp, PR, C.POINTER(Timeshare), vp]),
             "ecasq_quantize_timeshare": (C.c_int, [vp, i64, vp, i32, vp, i32, dbl, u64, u64, vp, vp, vp, vp, sz, pd,
                                                    vp]),
@@ -115,7 +117,7 @@ def exported_symbols():
     names = []
     for name in ("ecasq_version", "ecasq_strerror", "ecasq_workspace_size", "ecasq_workspace_size_flags",
                  "ecasq_solve", "ecasq_solve_grid", "ecasq_workspace_size_grid", "ecasq_solve_timeshare",
-                 "ecasq_quantize_timeshare", "ecasq_dp_pass",
+                 "ecasq_quantize_timeshare", "ecasq_workspace_size_opt", "ecasq_opt_dp", "ecasq_dp_pass",
                  "ecasq_dp_tables", "ecasq_refine", "ecasq_evaluate", "ecasq_quantize", "ecasq_quantize_noalloc",
                  "ecasq_solve_batched",
                  "ecasq_prepare", "ecasq_kernel_launches"):
@@ -280,6 +282,33 @@ def ecasq_quantize_timeshare(x, Qm, Qp, beta, seed, seed_ts, ws=None, with_sel=T
                                         C.byref(rate), _stream())
     _check(rc, "ecasq_quantize_timeshare")
     return idx, sel, counts, rate.value
+
+
+def ecasq_opt_dp(x, s, lambdas, P=None, flags=0, ws=None):
+    """Optimal DP of Sec. 4 at up to 8 fixed multipliers (vNMSE scale): (Q [G, s] tensor,
+    m list, metrics [G, 4] = optimum, MSE, H(I,B), H(Xhat)).  P: optional permissible set."""
+    torch = _torch()
+    x = _dev_f32(x)
+    d = x.numel()
+    lams = np.ascontiguousarray(np.atleast_1d(lambdas), dtype=np.float64)
+    G = lams.size
+    n = 0
+    if P is not None:
+        P = _dev_f32(P)
+        n = P.numel()
+    if ws is None:
+        nb = int(lib().ecasq_workspace_size_opt(d, n if P is not None else d, int(s), G))
+        if nb == 0:
+            raise EcasqError(EINVAL, "ecasq_workspace_size_opt")
+        ws = torch.empty(nb, dtype=torch.uint8, device="cuda")
+    Q = torch.zeros((G, s), dtype=torch.float32, device="cuda")
+    m = (C.c_int32 * G)()
+    met = np.zeros(4 * G, np.float64)
+    rc = lib().ecasq_opt_dp(_ptr(x), d, _ptr(P) if P is not None else None, n, int(s),
+                            lams.ctypes.data_as(C.POINTER(C.c_double)), G, int(flags), _ptr(ws), ws.numel(), _ptr(Q),
+                            m, met.ctypes.data_as(C.POINTER(C.c_double)), _stream())
+    _check(rc, "ecasq_opt_dp")
+    return Q, list(m), met.reshape(G, 4)
 
 
 def uniform_grid(x, n):
