@@ -200,6 +200,31 @@ int ecasq_quantize_timeshare(const float *x, int64_t d, const float *Qm, int32_t
                              uint32_t *counts, void *ws, size_t ws_bytes, double *rate, ecasq_stream_t stream);
 
 
+/* The optimal DP of Sec. 4 (App. E for a permissible set) at G <= 8 fixed
+ * multipliers: the least MSE + lambda' H(Xhat) over codebooks drawn from P (or from
+ * the unique values of x when P is NULL) with at most s values (exactly s with
+ * ECASQ_EXACT_S), first value in L and last in R as in eq. apx_base / apx_final.
+ * State (i, l, j) with the entropy of p_l charged once both neighbours are known:
+ *   dp(2, a, j) = C[a, j] + lambda' h((n_a + D[a, j]) / d)                     (a in L)
+ *   dp(i, l, j) = C[l, j] + min_{k<l} dp(i-1, k, l) + lambda' h((U[k, l] + D[l, j]) / d)
+ *   optimum     = min_{i, j in R, l<j} dp(i, l, j) + lambda' h(U[l, j] / d)
+ * Ties: lowest k; at the optimum the smallest i, then j, then l.  Every candidate is
+ * filtered in fp32 and every one within a certified band is re-scored in binary64
+ * with the formula above, so values and decisions are those of a binary64 evaluation.
+ * O(p^3 s / 6) candidates and O(p^2 s G) table cells: meant for p up to a few
+ * thousand (the candidate set is capped at 16384 values).
+ *   lambdas   host [G], vNMSE scale (lambda' = lambda ||X||^2), >= 0 and finite
+ *   P, n      device [n] permissible set (as ecasq_solve_grid) or NULL (n ignored)
+ *   Q_out     device [G * s] (row g: codebook of multiplier g, m_out[g] values)
+ *   m_out     host [G]
+ *   metrics   host [G * 4]: optimum, MSE, H(I,B), H(Xhat) of the traced codebook
+ * Workspace: ecasq_workspace_size_opt(d, n or d, s, G) (about 12 G s p^2 / 2 bytes of
+ * tables plus 12 p^2 bytes of pair quantities).  Synchronises `stream`. */
+size_t ecasq_workspace_size_opt(int64_t d, int64_t n, int32_t s, int32_t G);
+int ecasq_opt_dp(const float *x, int64_t d, const float *P, int64_t n, int32_t s, const double *lambdas, int32_t G,
+                 uint32_t flags, void *ws, size_t ws_bytes, float *Q_out, int32_t *m_out, double *metrics,
+                 ecasq_stream_t stream);
+
 /* One DP pass (Sec. 5) at G <= 8 fixed multipliers, the unit of the search.
  *   lambdas   host [G], vNMSE scale, >= 0
  *   Q_out     device [G * s] (row g: codebook of multiplier g, m_out[g] values)
