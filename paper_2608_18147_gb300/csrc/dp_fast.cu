@@ -832,14 +832,21 @@ __device__ __forceinline__ void cons_diag_pair(const FastArgs &a, Smem &S, uint3
             m0[q] = min(m0[q], m1[q]);
             m0[q] = min(m0[q], __shfl_xor_sync(0xffffffffu, m0[q], 16));
         }
-        if (owner) {
+        if (own) {
+            // both halves of the warp fold: the owner half (layer group olg) columns
+            // q = 0, 1 into its own slots, the other half q = 2, 3 into the owner's
+            // slots (lane ^ 16 holds the same columns); m0 is complete in both halves
+            const bool mine = id.lg == olg;
+            const int cto = mine ? ct : (ct ^ 16);
 #pragma unroll
-            for (int q = 0; q < JPT; q++) {
+            for (int qq = 0; qq < JPT / 2; qq++) {
+                const int q = mine ? qq : qq + JPT / 2;
+                const int mq = mine ? m0[qq] : m0[qq + JPT / 2];
                 const int jl = id.jq + NJQ * q;
-                const int x = (l * JPT + q) * nc + ct;
+                const int x = (l * JPT + q) * nc + cto;
                 float bb = __uint_as_float(park[x]);
                 uint32_t w1 = park[NS * nc + x], w2 = park[2 * NS * nc + x];
-                band_fold(__int_as_float(m0[q]), bb, S.tau[i], w1, w2, K, KK);
+                band_fold(__int_as_float(mq), bb, S.tau[i], w1, w2, K, KK);
                 park[x] = __float_as_uint(bb);
                 park[NS * nc + x] = w1;
                 park[2 * NS * nc + x] = w2;
@@ -849,8 +856,9 @@ __device__ __forceinline__ void cons_diag_pair(const FastArgs &a, Smem &S, uint3
         bar_sync(BAR_CONS, nc);
         cur ^= 1;
     }
-    // the block's final values and bands, from the parked state, and the block
-    // minimum of every layer (over the 64 columns a half-warp holds)
+    // the block's final values from the parked state, and the block minimum of
+    // every layer (over the 64 columns a half-warp holds); the band words follow
+    // after the block is published (diag_pair_bands: only the exact stage reads them)
     if (own) {
 #pragma unroll
         for (int l = 0; l < LPT; l++) {
@@ -862,16 +870,33 @@ __device__ __forceinline__ void cons_diag_pair(const FastArgs &a, Smem &S, uint3
                 const int64_t j = j0 + id.jq + NJQ * q;
                 const int x = (l * JPT + q) * nc + ct;
                 v = min(v, (int)park[x]);
-                if (real && j < a.p) {
-                    a.dp32[d32(a, g, i, j)] = __uint_as_float(park[x]);
-                    a.band[oidx(a, g, i, j)] = band_pack(park[NS * nc + x], park[2 * NS * nc + x]);
-                }
+                if (real && j < a.p) a.dp32[d32(a, g, i, j)] = __uint_as_float(park[x]);
             }
             if (a.prune) {
 #pragma unroll
                 for (int o = 8; o > 0; o >>= 1) v = min(v, __shfl_xor_sync(0xffffffffu, v, o));
                 if (real && id.jq == 0) a.mdp[((size_t)J * a.G + g) * a.mdp_stride + i] = __int_as_float(v);
             }
+        }
+    }
+}
+
+// Band words of the diagonal block from the parked state (after cons_diag_pair).
+__device__ __forceinline__ void diag_pair_bands(const FastArgs &a, const uint32_t *park, int J, int split,
+                                                const ConsId &id) {
+    const int ct = id.ct, nc = a.ncons;
+    const int g = split * a.Gc + id.gl;
+    if (!(id.active && g < a.G)) return;
+    constexpr int NS = LPT * JPT;
+    const int64_t j0 = (int64_t)J * BJ;
+#pragma unroll
+    for (int l = 0; l < LPT; l++) {
+        const int i = 3 + id.lg * LPT + l;
+#pragma unroll
+        for (int q = 0; q < JPT; q++) {
+            const int64_t j = j0 + id.jq + NJQ * q;
+            const int x = (l * JPT + q) * nc + ct;
+            if (i <= a.s && j < a.p) a.band[oidx(a, g, i, j)] = band_pack(park[NS * nc + x], park[2 * NS * nc + x]);
         }
     }
 }
@@ -1094,12 +1119,14 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
         {  // the diagonal tile (issued with tile J-1, or at the block start when J = 0)
             const int b = n & 1;
             mbar_wait_bounded(&S.mbar[b], (n >> 1) & 1u, a.st, a.abort_flag);
+            uint32_t *park = reinterpret_cast<uint32_t *>(sDP + (size_t)2 * rowsDP * BK);
             if (a.lgc == 2)
-                cons_diag_pair(a, S, reinterpret_cast<uint32_t *>(sDP + (size_t)2 * rowsDP * BK), b, J, split, id, cs);
+                cons_diag_pair(a, S, park, b, J, split, id, cs);
             else
                 cons_diag(a, S, b, J, split, id, cs, true);
+            __syncthreads();  // every thread's dp32 and layer minima of block J are stored
             if (ct == 0) publish_block(a, split, J);
-            __syncthreads();
+            if (a.lgc == 2) diag_pair_bands(a, park, J, split, id);
             n++;
         }
     }
