@@ -40,9 +40,9 @@ FP32_LANES = 128          # FP32-pipe lanes per SM (adds and min/max share them)
 SM_MAX_MHZ = 2070.0
 OPS_PER_CANDIDATE = 2     # one add and one min per min-plus candidate
 # DRAM bytes of one k_wavefront_res launch per 64 x 64 tile, from the ncu capture in
-# profiles/k_wavefront_res_lognormal_d16384_s16.md (read 1.146458 GB + write 7.4 MB over
+# profiles/k_wavefront_res_lognormal_d16384_s16.md (read 1.146089 GB + write 7.2 MB over
 # 32896 tiles); the benchmark launch is scaled by its own tile count.
-TRAFFIC_PER_TILE = (1.146458e9 + 7.448576e6) / 32896
+TRAFFIC_PER_TILE = (1.146089e9 + 7.165184e6) / 32896
 ORACLE_SAMPLE = 16384     # entries of the CPU baseline's bounded sample
 
 
