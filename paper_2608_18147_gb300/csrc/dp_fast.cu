@@ -808,7 +808,6 @@ __device__ __forceinline__ void cons_diag_pair(const FastArgs &a, Smem &S, uint3
     for (int li = 0; li < L; li++) {
         const int i = 3 + li;
         const int olg = li / LPT, l = li - olg * LPT;
-        const bool owner = own && id.lg == olg;
         int m0[JPT], m1[JPT];
 #pragma unroll
         for (int q = 0; q < JPT; q++) { m0[q] = 0x7f800000; m1[q] = 0x7f800000; }
