@@ -60,6 +60,22 @@ def parse():
     return ap.parse_args()
 
 
+def max_over_ranks(x, dist, device):
+    """The largest x over all ranks (the job's time is its slowest replica's)."""
+    if dist is None:
+        return float(x)
+    import torch
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(world, units_per_rank, ms):
+    """Units per second of the whole job: every replica processes units_per_rank in ms
+    (the max over ranks), so the aggregate is world * units / time (weak scaling)."""
+    return world * units_per_rank / (ms / 1000.0)
+
+
 def candidates_per_multiplier(p, s):
     """Candidates of eq. apx_rec for one multiplier: layers 3..s, j in [i-1, p-1], k in [i-2, j-1]."""
     c = 0
@@ -350,13 +366,9 @@ def main():
         ev1.record(stream)
         barrier()
     launches = E.ecasq_kernel_launches() - launches0
-    ms = ev0.elapsed_time(ev1)
-    if dist is not None:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ev0.elapsed_time(ev1), dist, "cuda")
     cand_step = statistics.mean(r["candidates"] for r in results)
-    value = world * args.steps * cand_step / (ms / 1000.0)
+    value = whole_job_rate(world, args.steps * cand_step, ms)
     dp_ms = sum(r["dp_kernel_ms"] for r in results)
     dp_launches = sum(r["dp_kernel_launches"] for r in results)
     cand_total = sum(r["candidates"] for r in results)
@@ -401,12 +413,8 @@ def main():
             cand_e += res["candidates"]
         e1.record(stream)
         barrier()
-        ms_e = e0.elapsed_time(e1)
-        if dist is not None:
-            t = torch.tensor([ms_e], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ms_e = float(t.item())
-        e2e = {"value": world * cand_e / (ms_e / 1000.0), "unit": UNIT, "h2d_bytes_per_step": 4 * d,
+        ms_e = max_over_ranks(e0.elapsed_time(e1), dist, "cuda")
+        e2e = {"value": whole_job_rate(world, cand_e, ms_e), "unit": UNIT, "h2d_bytes_per_step": 4 * d,
                "d2h_bytes_per_step": d + 4 * int(qh.numel()), "ms_per_step": ms_e / args.steps}
 
     cb = None
