@@ -19,6 +19,9 @@ Other rows of the path, each timed the same way on the chosen --config:
                     time-shared encode; metric: solves/s
   --mode opt        one pass of the optimal DP (Sec. 4) at 8 multipliers over a uniform
                     grid of --grid values; metric: candidate evaluations/s
+  --mode hbm        the HBM-bound rows on vectors far larger than L2: the encode (A10,
+                    2^28 entries) and the sort + histogram + prefix sums (A1-A3, 2^26
+                    entries); metric: GB/s of algorithmic traffic
 """
 import argparse
 import json
@@ -55,7 +58,7 @@ def parse():
     ap.add_argument("--config", default="studentt_d131072_s16")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--mode", default="solve", choices=["solve", "grid", "timeshare", "opt"])
+    ap.add_argument("--mode", default="solve", choices=["solve", "grid", "timeshare", "opt", "hbm"])
     ap.add_argument("--grid", type=int, default=256, help="grid size for --mode grid")
     return ap.parse_args()
 
@@ -196,6 +199,9 @@ def run_other_mode(args, cfg, x_np):
     if args.mode == "opt":
         run_opt_mode(args, cfg, x_np)
         return
+    if args.mode == "hbm":
+        run_hbm_mode(args)
+        return
     if args.mode == "grid":
         g = torch.as_tensor(E.uniform_grid(x_np, args.grid)).cuda()
         ws = torch.empty(int(E.lib().ecasq_workspace_size_grid(d, g.numel(), s, flags)), dtype=torch.uint8,
@@ -246,6 +252,68 @@ def run_other_mode(args, cfg, x_np):
                      "dp_launches_per_solve": dp_launches / args.steps},
            "timeshare": ts or None, "gpu_launches": E.ecasq_kernel_launches() - launches0,
            "clocks": clk.summary()}
+    print(json.dumps(out), flush=True)
+
+
+def run_hbm_mode(args):
+    """Encode (4 B read + 1 B written per entry) and preparation (four 8-bit LSD radix
+    passes, 8 B per entry each, then the histogram and prefix sums) on seeded normal
+    vectors generated on the device.  Each call synchronises its stream, so the CUDA-event
+    time of a call includes the host's part of it: the GB/s are lower bounds."""
+    import torch
+    import paper_2608_18147_gb300 as E
+    peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))) if os.path.exists(
+        os.path.join(ROOT, "MEASURED_PEAKS.json")) else {"hbm_gbs": 6800.0}
+    gen = torch.Generator(device="cuda").manual_seed(0)
+    out = {"metric": "ECASQ HBM-bound rows: GB/s of algorithmic traffic", "unit": "GB/s", "n_gpus": 1,
+           "steps": args.steps, "warmup": args.warmup, "higher_is_better": True, "vs_baseline": None,
+           "data": "synthetic (seeded normal, generated on the device)", "dtype": "f32 in, u8 out"}
+    stream = torch.cuda.current_stream()
+
+    def timed(fn):
+        for _ in range(args.warmup):
+            fn()
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ts = []
+        for _ in range(args.steps):
+            torch.cuda.synchronize()
+            ev0.record(stream)
+            fn()
+            ev1.record(stream)
+            torch.cuda.synchronize()
+            ts.append(ev0.elapsed_time(ev1))
+        return statistics.median(ts)
+
+    d = 1 << 28
+    x = torch.randn(d, generator=gen, device="cuda", dtype=torch.float32)
+    Q = torch.quantile(x[: 1 << 20], torch.linspace(0, 1, 16, device="cuda")).contiguous()
+    Q[0], Q[-1] = x.min(), x.max()
+    Q = torch.unique(Q)
+    idx = torch.empty(d, dtype=torch.uint8, device="cuda")
+    counts = torch.empty(Q.numel(), dtype=torch.int32, device="cuda")
+    qws = torch.empty(256, dtype=torch.uint8, device="cuda")
+    ms_q = timed(lambda: E.ecasq_quantize(x, Q, seed=1, ws=qws, idx=idx, counts=counts))
+    gbs_q = 5.0 * d / (ms_q / 1000.0) / 1e9
+    ms_t = timed(lambda: E.ecasq_quantize_timeshare(x, Q, Q, 0.5, 1, 2, ws=qws))
+    gbs_t = 6.0 * d / (ms_t / 1000.0) / 1e9
+    del x, idx
+    torch.cuda.empty_cache()
+    d2 = 1 << 26
+    x2 = torch.randn(d2, generator=gen, device="cuda", dtype=torch.float32)
+    ws2 = torch.empty(int(E.lib().ecasq_workspace_size_prep(d2)), dtype=torch.uint8, device="cuda")
+    ms_p = timed(lambda: E.ecasq_prepare(x2, ws=ws2))
+    gbs_p = 32.0 * d2 / (ms_p / 1000.0) / 1e9
+    peak = peaks["hbm_gbs"]
+    out.update(value=gbs_q, ms_per_step=ms_q,
+               config={"workload": "normal, 2^28 entries (encode), 2^26 (prepare)", "mode": "hbm",
+                       "codebook": int(Q.numel()), "l2": "vectors of 1 GiB and 256 MiB, far above the 129 MB L2"},
+               roofline={"bound": "hbm", "achieved": gbs_q, "peak": peak, "unit": "GB/s", "frac": gbs_q / peak,
+                         "traffic": None, "kernel": "k_quantize", "peak_basis": "MEASURED_PEAKS.json hbm_gbs"},
+               rows={"encode": {"ms": ms_q, "bytes_per_entry": 5, "GBs": gbs_q, "frac": gbs_q / peak},
+                     "encode_timeshare": {"ms": ms_t, "bytes_per_entry": 6, "GBs": gbs_t, "frac": gbs_t / peak},
+                     "prepare": {"ms": ms_p, "bytes_per_entry": 32, "GBs": gbs_p, "frac": gbs_p / peak,
+                                 "basis": "4 LSD radix passes x (4 B read + 4 B written); the histogram, "
+                                          "prefix sums and count passes are extra"}})
     print(json.dumps(out), flush=True)
 
 

@@ -320,7 +320,10 @@ int ecasq_solve_batched(const float *X, int64_t rows, int64_t d, const ecasq_par
  *   v [p] fp32 unique values ascending, w [p] int64 multiplicities,
  *   N [p+1] int64, S and S2 [2*(p+1)] fp64 as (hi[0..p], lo[0..p]) with
  *   N[t] = sum_{r<t} w_r, S[t] = sum w_r v_r, S2[t] = sum w_r v_r^2.
- *   All device, sized for p = d; p_out host.  Synchronises `stream`. */
+ *   All device, sized for p = d; p_out host.  Workspace: ecasq_workspace_size_prep(d)
+ *   (about 92 d bytes: the sort's keys, the histogram and the sums; the solves'
+ *   workspace holds far more).  Synchronises `stream`. */
+size_t ecasq_workspace_size_prep(int64_t d);
 int ecasq_prepare(const float *x, int64_t d, void *ws, size_t ws_bytes, float *v, int64_t *w, int64_t *N,
                   double *S, double *S2, int64_t *p_out, ecasq_stream_t stream);
 

@@ -114,6 +114,31 @@ size_t make_layout(int64_t d, int32_t s, int64_t rows, Layout *L) {
     return off;
 }
 
+// Only what the sort, histogram and prefix sums use (ecasq_prepare): the regions of
+// make_layout up to the scan partials, then a 32 (d+1)-byte scratch in place of the
+// DP tables (the fp64 sums before their double-double split).
+static size_t make_prep_layout(int64_t d, Layout *L) {
+    memset(L, 0, sizeof(*L));
+    size_t off = 0;
+    auto take = [&](size_t bytes) { size_t o = off; off += align256(bytes); return o; };
+    int64_t nb = cdiv(d, kSortTile), nbs = cdiv(d, kScanTile);
+    L->status = take(sizeof(DevStatus));
+    L->keys0 = take(4 * (size_t)d);
+    L->keys1 = take(4 * (size_t)d);
+    L->rcount = take(4 * 256 * (size_t)nb);
+    L->v = take(4 * (size_t)d);
+    L->w = take(8 * (size_t)d);
+    L->N = take(8 * (size_t)(d + 1));
+    L->S = take(16 * (size_t)(d + 1));
+    L->S2 = take(16 * (size_t)(d + 1));
+    L->part = take(48 * (size_t)nbs);
+    L->dp64 = take(8 * 4 * (size_t)(d + 1));
+    L->total = off;
+    L->d = d;
+    L->s = 2;
+    return off;
+}
+
 static int g_num_sms = 0;
 static int num_sms() {
     if (g_num_sms == 0) {
@@ -412,12 +437,18 @@ size_t ecasq_workspace_size_flags(int64_t d, int32_t s, int64_t rows, uint32_t f
     return base + align256(cb);
 }
 
+size_t ecasq_workspace_size_prep(int64_t d) {
+    if (d < 1 || d >= ((int64_t)1 << 31)) return 0;
+    Layout L;
+    return make_prep_layout(d, &L);
+}
+
 int ecasq_prepare(const float *x, int64_t d, void *ws, size_t ws_bytes, float *v, int64_t *w, int64_t *N,
                   double *S, double *S2, int64_t *p_out, ecasq_stream_t stream) {
     if (!x || d < 1 || d >= ((int64_t)1 << 31) || !v || !w || !N || !S || !S2 || !p_out) return ECASQ_EINVAL;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     Layout L;
-    make_layout(d, 2, 1, &L);
+    make_prep_layout(d, &L);
     int rc = check_ws(ws, ws_bytes, L);
     if (rc) return rc;
     int64_t p;

@@ -48,36 +48,45 @@ __global__ void __launch_bounds__(256) k_radix_count(const uint32_t *__restrict_
     counts[(size_t)threadIdx.x * nb + blockIdx.x] = h[threadIdx.x];
 }
 
-// In-place exclusive scan of n uint32 values by one block of 1024 threads.
+// In-place exclusive scan of n uint32 values by one block of 1024 threads, in
+// coalesced tiles of 4096 (four consecutive values per thread) with a running carry.
 __global__ void __launch_bounds__(1024) k_scan_u32(uint32_t *a, int64_t n) {
     __shared__ uint32_t wsum[32];
-    int64_t per = cdiv(n, 1024);
-    int64_t lo = threadIdx.x * per, hi = min(lo + per, n);
-    uint32_t s = 0;
-    for (int64_t i = lo; i < hi; i++) s += a[i];
-    // block exclusive scan of s
-    uint32_t incl = s;
-    int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-    for (int o = 1; o < 32; o <<= 1) {
-        uint32_t t = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += t;
-    }
-    if (lane == 31) wsum[wid] = incl;
+    __shared__ uint32_t carry;
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    if (threadIdx.x == 0) carry = 0;
     __syncthreads();
-    if (wid == 0) {
-        uint32_t v = wsum[lane], vi = v;
+    for (int64_t base = 0; base < n; base += 4 * 1024) {
+        const int64_t i0 = base + 4 * (int64_t)threadIdx.x;
+        uint32_t v[4];
+#pragma unroll
+        for (int e = 0; e < 4; e++) v[e] = i0 + e < n ? a[i0 + e] : 0u;
+        const uint32_t s = v[0] + v[1] + v[2] + v[3];
+        uint32_t incl = s;
         for (int o = 1; o < 32; o <<= 1) {
-            uint32_t t = __shfl_up_sync(0xffffffffu, vi, o);
-            if (lane >= o) vi += t;
+            uint32_t t = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += t;
         }
-        wsum[lane] = vi - v;
-    }
-    __syncthreads();
-    uint32_t run = wsum[wid] + incl - s;
-    for (int64_t i = lo; i < hi; i++) {
-        uint32_t t = a[i];
-        a[i] = run;
-        run += t;
+        if (lane == 31) wsum[wid] = incl;
+        __syncthreads();
+        if (wid == 0) {
+            uint32_t w = wsum[lane], wi = w;
+            for (int o = 1; o < 32; o <<= 1) {
+                uint32_t t = __shfl_up_sync(0xffffffffu, wi, o);
+                if (lane >= o) wi += t;
+            }
+            wsum[lane] = wi - w;
+        }
+        __syncthreads();
+        uint32_t run = carry + wsum[wid] + incl - s;
+#pragma unroll
+        for (int e = 0; e < 4; e++) {
+            if (i0 + e < n) a[i0 + e] = run;
+            run += v[e];
+        }
+        __syncthreads();  // every thread has read carry and wsum
+        if (threadIdx.x == blockDim.x - 1) carry = run;  // the old carry plus this tile's total
+        __syncthreads();
     }
 }
 
@@ -176,10 +185,24 @@ __global__ void __launch_bounds__(256) k_hist_partials(const uint32_t *__restric
 }
 
 // Exclusive scan of the tile partials (one thread, in order; nb is small).
-__global__ void k_hist_scan_partials(DDPart *part, int64_t nb) {
-    if (threadIdx.x != 0 || blockIdx.x != 0) return;
-    ScanVal acc{{0.0, 0.0}, {0.0, 0.0}, 0};
-    for (int64_t b = 0; b < nb; b++) {
+// Exclusive scan of the tiles' partials by one block of 256 threads: each thread sums a
+// contiguous run of tiles in order, the runs' totals are scanned across the block
+// (block_scan_incl), and each thread then writes its run's exclusive prefixes.
+__global__ void __launch_bounds__(256) k_hist_scan_partials(DDPart *part, int64_t nb) {
+    __shared__ ScanVal wtot[8];
+    __shared__ ScanVal incl_all[256];
+    const int64_t per = cdiv(nb, (int64_t)blockDim.x);
+    const int64_t lo = min((int64_t)threadIdx.x * per, nb), hi = min(lo + per, nb);
+    ScanVal s{{0.0, 0.0}, {0.0, 0.0}, 0};
+    for (int64_t b = lo; b < hi; b++) {
+        ScanVal t{{part[b].s_hi, part[b].s_lo}, {part[b].q_hi, part[b].q_lo}, part[b].heads};
+        s = sv_add(s, t);
+    }
+    ScanVal total;
+    incl_all[threadIdx.x] = block_scan_incl(s, wtot, total);
+    __syncthreads();
+    ScanVal acc = threadIdx.x > 0 ? incl_all[threadIdx.x - 1] : ScanVal{{0.0, 0.0}, {0.0, 0.0}, 0};
+    for (int64_t b = lo; b < hi; b++) {
         ScanVal t{{part[b].s_hi, part[b].s_lo}, {part[b].q_hi, part[b].q_lo}, part[b].heads};
         part[b] = {acc.s.hi, acc.s.lo, acc.q.hi, acc.q.lo, acc.h, 0};
         acc = sv_add(acc, t);
@@ -442,7 +465,7 @@ int prepare_device(const float *x, int64_t d, void *ws, const Layout &L, cudaStr
     note_launch();
     k_hist_partials<<<(unsigned)nbs, 256, 0, stream>>>(a, d, part);
     note_launch();
-    k_hist_scan_partials<<<1, 32, 0, stream>>>(part, nbs);
+    k_hist_scan_partials<<<1, 256, 0, stream>>>(part, nbs);
     note_launch();
     k_hist_fill<<<(unsigned)nbs, 256, 0, stream>>>(a, d, part, wsp<float>(ws, L.v), wsp<int64_t>(ws, L.N), Stmp,
                                                  S2tmp, st, d);

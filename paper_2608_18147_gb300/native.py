@@ -89,6 +89,7 @@ def lib():
             "ecasq_solve_grid": (C.c_int, [vp, i64, vp, i64, PP, vp, sz, vp, PR, vp]),
             "ecasq_workspace_size_grid": (sz, [i64, i64, i32, u32]),
             "ecasq_workspace_size_opt": (sz, [i64, i64, i32, i32]),
+            "ecasq_workspace_size_prep": (sz, [i64]),
             "ecasq_opt_dp": (C.c_int, [vp, i64, vp, i64, i32, pd, i32, u32, vp, sz, vp, pi32, pd, vp]),
             "ecasq_solve_timeshare": (C.c_int, [vp, i64, vp, i64, PP, vp, sz, vp, vp, PR, C.POINTER(Timeshare), vp]),
             "ecasq_quantize_timeshare": (C.c_int, [vp, i64, vp, i32, vp, i32, dbl, u64, u64, vp, vp, vp, vp, sz, pd,
@@ -117,7 +118,8 @@ def exported_symbols():
     names = []
     for name in ("ecasq_version", "ecasq_strerror", "ecasq_workspace_size", "ecasq_workspace_size_flags",
                  "ecasq_solve", "ecasq_solve_grid", "ecasq_workspace_size_grid", "ecasq_solve_timeshare",
-                 "ecasq_quantize_timeshare", "ecasq_workspace_size_opt", "ecasq_opt_dp", "ecasq_dp_pass",
+                 "ecasq_quantize_timeshare", "ecasq_workspace_size_opt", "ecasq_workspace_size_prep", "ecasq_opt_dp",
+                 "ecasq_dp_pass",
                  "ecasq_dp_tables", "ecasq_refine", "ecasq_evaluate", "ecasq_quantize", "ecasq_quantize_noalloc",
                  "ecasq_solve_batched",
                  "ecasq_prepare", "ecasq_kernel_launches"):
@@ -436,7 +438,7 @@ def ecasq_prepare(x, ws=None):
     x = _dev_f32(x)
     d = x.numel()
     if ws is None:
-        ws = workspace(d, 2)
+        ws = torch.empty(int(lib().ecasq_workspace_size_prep(d)), dtype=torch.uint8, device="cuda")
     v = torch.empty(d, dtype=torch.float32, device="cuda")
     w = torch.empty(d, dtype=torch.int64, device="cuda")
     N = torch.empty(d + 1, dtype=torch.int64, device="cuda")

@@ -47,6 +47,10 @@ def test_host_only_calls():
     assert native.ecasq_workspace_size_flags(4096, 8, 1, native.RESIDENT_COSTS) == base + 64 * 65 // 2 * 34816
     assert native.ecasq_workspace_size_flags(2 ** 31 - 1, 8, 1, native.RESIDENT_COSTS) == 0  # beyond size_t
     assert native.ecasq_workspace_size_flags(0, 8, 1, native.RESIDENT_COSTS) == 0
+    # preparation alone: the sort, histogram and sums (linear in d), far below a solve's
+    assert 80 * 2 ** 20 < native.lib().ecasq_workspace_size_prep(2 ** 20) < 100 * 2 ** 20
+    assert native.lib().ecasq_workspace_size_prep(0) == 0
+    assert native.lib().ecasq_workspace_size_prep(2 ** 20) < native.ecasq_workspace_size(2 ** 20, 2)
     # workspace grows with d and s
     assert native.ecasq_workspace_size(4096, 16) > native.ecasq_workspace_size(4096, 8)
     assert native.ecasq_workspace_size(8192, 8) > native.ecasq_workspace_size(4096, 8)
