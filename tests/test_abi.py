@@ -9,7 +9,8 @@ from conftest import ROOT
 
 
 def declared_symbols():
-    txt = open(os.path.join(ROOT, "include", "ecasq.h")).read()
+    with open(os.path.join(ROOT, "include", "ecasq.h")) as f:
+        txt = f.read()
     return sorted(set(re.findall(r"\b(ecasq_[a-z_]+)\s*\(", txt)))
 
 
@@ -93,6 +94,7 @@ def test_product_path_does_not_touch_the_oracle():
             continue
         for f in files:
             if f.endswith((".py", ".cu", ".cuh", ".h")):
-                txt = open(os.path.join(dirpath, f)).read()
+                with open(os.path.join(dirpath, f)) as fh:
+                    txt = fh.read()
                 assert "import oracle" not in txt and "from oracle" not in txt, f
                 assert "ecasq_oracle" not in txt and "liboracle" not in txt, f
