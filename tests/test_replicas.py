@@ -19,7 +19,7 @@ def _free_port():
         return s.getsockname()[1]
 
 
-def _rank(rank, world, port, out):
+def _rank(rank, world, port, outdir):
     import torch.distributed as dist
     os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
     dist.init_process_group("gloo", rank=rank, world_size=world)
@@ -27,16 +27,18 @@ def _rank(rank, world, port, out):
     import bench
     ms = bench.max_over_ranks(100.0 + 50.0 * rank, dist, "cpu")   # rank 1 is the slow replica
     dist.barrier()
-    out[rank] = (ms, bench.whole_job_rate(world, 3.0e12, ms))
+    with open(os.path.join(outdir, "rank%d.json" % rank), "w") as f:
+        json.dump([ms, bench.whole_job_rate(world, 3.0e12, ms)], f)
     dist.destroy_process_group()
 
 
-def test_two_gloo_ranks_take_the_slowest_replica():
+def test_two_gloo_ranks_take_the_slowest_replica(tmp_path):
     world = 2
-    with mp.Manager() as mgr:
-        out = mgr.dict()
-        mp.spawn(_rank, args=(world, _free_port(), out), nprocs=world, join=True)
-        res = dict(out)
+    mp.spawn(_rank, args=(world, _free_port(), str(tmp_path)), nprocs=world, join=True)  # spawn, not fork
+    res = {}
+    for r in range(world):
+        with open(tmp_path / ("rank%d.json" % r)) as f:
+            res[r] = tuple(json.load(f))
     assert res[0] == res[1]                       # every rank agrees
     ms, rate = res[0]
     assert ms == 150.0                            # the max over ranks
