@@ -753,13 +753,28 @@ __device__ __forceinline__ void cons_diag(const FastArgs &a, Smem &S, int b, int
     }
 }
 
-// Diagonal block when a.lgc == 2 (the usual s <= 16): lanes 0-15 of a warp take
-// k in [0, 32) of the block and lanes 16-31 k in [32, 64), for the same
-// multiplier and columns; the costs W = C + lambda' Phi of a lane's 4 x 32 pairs
-// stay in registers for all layers, so each layer reads only the previous
-// layer's 64 values from shared memory.  The band state is parked in `park`
+// Diagonal block when a.lgc == 2 (the usual s <= 16).  Only pairs k < j of the tile
+// count, so each lane takes two whole columns of its column group jq, balanced on the
+// triangle: lanes 0-15 column jq + 48 (k < 64) and column jq (k < 16), lanes 16-31
+// column jq + 32 (k < 48) and column jq + 16 (k < 32): 80 pairs each, in 20 groups of
+// four consecutive k (kdiag_group).  The costs W = C + lambda' Phi of those pairs stay
+// in registers for all layers, so each layer reads only the previous layer's 64 values
+// from shared memory, and every column's minimum is complete within one lane (pairs
+// k >= j carry C = +inf in the tile and never win).  The band state is parked in `park`
 // ([3][LPT][JPT][ncons] words: best, run 1, run 2) and folded there; the block
 // ends with its diagonal, so the registers are not restored.
+// Group g4 of a diagonal lane (half 0: lanes 0-15, half 1: lanes 16-31): its column
+// (q = 0: the long one, 1: the short one) and first k.  Groups 0-11 are k 0..47 of the
+// long column for both halves; groups 12-15 are k 48..63 of the long column (half 0)
+// or k 0..15 of the short one (half 1); groups 16-19 are k 0..15 (half 0) or 16..31
+// (half 1) of the short column.
+constexpr int kDiagGroups = 20;
+__device__ __forceinline__ void kdiag_group(int g4, int half, int &q, int &k) {
+    if (g4 < 12) { q = 0; k = 4 * g4; }
+    else if (g4 < 16) { q = half; k = half ? 4 * (g4 - 12) : 4 * g4; }
+    else { q = 1; k = half ? 4 * (g4 - 12) : 4 * (g4 - 16); }
+}
+
 __device__ __forceinline__ void cons_diag_pair(const FastArgs &a, Smem &S, uint32_t *park, int b, int J, int split,
                                                const ConsId &id, ConsState &cs) {
     const int L = a.s - 2;
@@ -767,7 +782,6 @@ __device__ __forceinline__ void cons_diag_pair(const FastArgs &a, Smem &S, uint3
     const int g = split * a.Gc + id.gl;
     const bool own = id.active && g < a.G;  // uniform over a warp (one multiplier per warp)
     const int64_t j0 = (int64_t)J * BJ;
-    const int kh = (ct & 16) ? BJ / 2 : 0;
     constexpr int NS = LPT * JPT;
 #pragma unroll
     for (int l = 0; l < LPT; l++)
@@ -786,21 +800,21 @@ __device__ __forceinline__ void cons_diag_pair(const FastArgs &a, Smem &S, uint3
         for (int o = 16; o > 0; o >>= 1) v = min(v, __shfl_xor_sync(0xffffffffu, v, o));
         if (lane == 0) a.mdp[((size_t)J * a.G + g) * a.mdp_stride + 2] = __int_as_float(v);
     }
-    float2 W[JPT][BJ / 4];  // W[q][p] = costs of k = kh + 2p, kh + 2p + 1 for column jq + 16 q
+    const int half = (ct >> 4) & 1;
+    const int qb = 3 - half, qs = half;  // the lane's long and short columns (q of jq + 16 q)
+    float2 W[2 * kDiagGroups];           // W[2 g4], W[2 g4 + 1]: costs of group g4's four pairs
     {
         const float lam = own ? S.lam32[g] : 0.f;
         const float2 lam2 = make_float2(lam, lam);
 #pragma unroll
-        for (int q = 0; q < JPT; q++) {
-            const int jl = id.jq + NJQ * q;
-#pragma unroll
-            for (int kk = 0; kk < BJ / 2; kk += 4) {
-                float4 c4 = *reinterpret_cast<const float4 *>(&S.C[b][jl][kh + kk]);
-                float4 f4 = *reinterpret_cast<const float4 *>(&S.Phi[b][jl][kh + kk]);
-                W[q][kk / 2] = fma2(lam2, make_float2(f4.x, f4.y), make_float2(c4.x, c4.y));
-                W[q][kk / 2 + 1] = fma2(lam2, make_float2(f4.z, f4.w), make_float2(c4.z, c4.w));
-            }
-            asm volatile("" ::: "memory");  // one column's loads in flight at a time (register pressure)
+        for (int g4 = 0; g4 < kDiagGroups; g4++) {
+            int q, k;
+            kdiag_group(g4, half, q, k);
+            const int jl = id.jq + NJQ * (q ? qs : qb);
+            float4 c4 = *reinterpret_cast<const float4 *>(&S.C[b][jl][k]);
+            float4 f4 = *reinterpret_cast<const float4 *>(&S.Phi[b][jl][k]);
+            W[2 * g4] = fma2(lam2, make_float2(f4.x, f4.y), make_float2(c4.x, c4.y));
+            W[2 * g4 + 1] = fma2(lam2, make_float2(f4.z, f4.w), make_float2(c4.z, c4.w));
         }
     }
     const uint32_t K = (uint32_t)J, KK = (K << 16) | K;
@@ -808,39 +822,40 @@ __device__ __forceinline__ void cons_diag_pair(const FastArgs &a, Smem &S, uint3
     for (int li = 0; li < L; li++) {
         const int i = 3 + li;
         const int olg = li / LPT, l = li - olg * LPT;
-        int m0[JPT], m1[JPT];
-#pragma unroll
-        for (int q = 0; q < JPT; q++) { m0[q] = 0x7f800000; m1[q] = 0x7f800000; }
+        // running minima (float bits; candidates are >= +0) of the long and the short
+        // column, two chains each
+        int b0 = 0x7f800000, b1 = 0x7f800000, s0 = 0x7f800000, s1 = 0x7f800000;
         if (own) {
-            const float *prow = &S.diag[cur][id.gl][kh];
+            const float *prow = &S.diag[cur][id.gl][0];
 #pragma unroll
-            for (int kk = 0; kk < BJ / 2; kk += 4) {
-                const float4 d4 = *reinterpret_cast<const float4 *>(prow + kk);
-                const float2 da = make_float2(d4.x, d4.y), db = make_float2(d4.z, d4.w);
-#pragma unroll
-                for (int q = 0; q < JPT; q++) {
-                    float2 t0 = add2(da, W[q][kk / 2]);
-                    float2 t1 = add2(db, W[q][kk / 2 + 1]);
-                    m0[q] = min(min(m0[q], __float_as_int(t0.x)), __float_as_int(t0.y));
-                    m1[q] = min(min(m1[q], __float_as_int(t1.x)), __float_as_int(t1.y));
+            for (int g4 = 0; g4 < kDiagGroups; g4++) {
+                int q, k;
+                kdiag_group(g4, half, q, k);
+                const float4 d4 = *reinterpret_cast<const float4 *>(prow + k);
+                const float2 t0 = add2(make_float2(d4.x, d4.y), W[2 * g4]);
+                const float2 t1 = add2(make_float2(d4.z, d4.w), W[2 * g4 + 1]);
+                if (g4 < 12) {
+                    b0 = min(min(b0, __float_as_int(t0.x)), __float_as_int(t0.y));
+                    b1 = min(min(b1, __float_as_int(t1.x)), __float_as_int(t1.y));
+                } else if (g4 < 16) {  // the long column for half 0, the short one for half 1
+                    const int m = min(min(__float_as_int(t0.x), __float_as_int(t0.y)),
+                                      min(__float_as_int(t1.x), __float_as_int(t1.y)));
+                    b0 = half ? b0 : min(b0, m);
+                    s0 = half ? min(s0, m) : s0;
+                } else {
+                    s0 = min(min(s0, __float_as_int(t0.x)), __float_as_int(t0.y));
+                    s1 = min(min(s1, __float_as_int(t1.x)), __float_as_int(t1.y));
                 }
             }
         }
-#pragma unroll
-        for (int q = 0; q < JPT; q++) {
-            m0[q] = min(m0[q], m1[q]);
-            m0[q] = min(m0[q], __shfl_xor_sync(0xffffffffu, m0[q], 16));
-        }
         if (own) {
-            // both halves of the warp fold: the owner half (layer group olg) columns
-            // q = 0, 1 into its own slots, the other half q = 2, 3 into the owner's
-            // slots (lane ^ 16 holds the same columns); m0 is complete in both halves
-            const bool mine = id.lg == olg;
-            const int cto = mine ? ct : (ct ^ 16);
+            // each lane folds its two columns into the owner's slots (layer group olg,
+            // same column group: lane jq + 16 olg of the warp)
+            const int cto = (ct & ~31) | (olg << 4) | id.jq;
 #pragma unroll
-            for (int qq = 0; qq < JPT / 2; qq++) {
-                const int q = mine ? qq : qq + JPT / 2;
-                const int mq = mine ? m0[qq] : m0[qq + JPT / 2];
+            for (int c = 0; c < 2; c++) {
+                const int q = c ? qs : qb;
+                const int mq = c ? min(s0, s1) : min(b0, b1);
                 const int jl = id.jq + NJQ * q;
                 const int x = (l * JPT + q) * nc + cto;
                 float bb = __uint_as_float(park[x]);
