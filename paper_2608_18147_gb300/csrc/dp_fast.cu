@@ -915,19 +915,21 @@ __device__ __forceinline__ void diag_pair_bands(const FastArgs &a, const uint32_
     }
 }
 
-// Bounded wait (one thread) until column block K of `split` is published.
-__device__ __forceinline__ void wait_block(const FastArgs &a, int split, int K) {
+// Bounded wait (one thread) until column block K of `split` is published; false
+// when the wait gave up (timeout or abort).
+__device__ __forceinline__ bool wait_block(const FastArgs &a, int split, int K) {
     const int *flag = a.done + (size_t)split * a.nJ + K;
     uint32_t spins = 0;
     while (ld_acquire(flag) == 0) {
-        if (*(volatile int *)a.abort_flag) break;
+        if (*(volatile int *)a.abort_flag) return false;
         if (++spins > kSpinLimit) {
             a.st->timeout = 1;
             atomicExch(a.abort_flag, 1);
-            break;
+            return false;
         }
         __nanosleep(64);
     }
+    return true;
 }
 
 // Publish column block J of `split` (after every thread's stores of the block).
@@ -1040,7 +1042,8 @@ __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
 // Warp 0 of the resident-cost kernel: expect the bytes of tile (K, J) on mbar[b]
 // and issue its bulk copies into buffer b -- the interval costs from the resident
 // table and, off the diagonal, the dp32 rows (g, layers 2..s-1) of the split's
-// real multipliers (rows of other slots are never read).
+// real multipliers (rows of other slots are never read).  The caller has made tile
+// K's rows visible to the copies (res_probe / res_wait).
 __device__ __forceinline__ void res_issue(const FastArgs &a, Smem &S, float *sDP, int b, int K, int J, int split,
                                           uint64_t policy, int lane) {
     const int L = a.s - 2, rowsDP = a.Gc * L;
@@ -1055,17 +1058,46 @@ __device__ __forceinline__ void res_issue(const FastArgs &a, Smem &S, float *sDP
         mbar_expect_tx(&S.mbar[b], 2 * kCostHalfBytes + (uint32_t)ngv * rows_bytes + mdp_bytes);
         bulk_g2s(&S.C[b][0][0], src, kCostHalfBytes, &S.mbar[b], policy);
         bulk_g2s(&S.Phi[b][0][0], src + kCostHalfFloats, kCostHalfBytes, &S.mbar[b], policy);
-        if (mdp_bytes) {
-            fence_proxy_async_global();
+        if (mdp_bytes)
             bulk_g2s_nohint(&S.mdp[b][0][0], a.mdp + ((size_t)K * a.G + gbase) * a.mdp_stride, mdp_bytes, &S.mbar[b]);
-        }
     }
     __syncwarp();
     if (lane < ngv) {
-        fence_proxy_async_global();  // rows other blocks wrote with generic stores
         float *dst = diag ? &S.diag[0][lane][0] : sDP + (size_t)b * rowsDP * BK + (size_t)lane * L * BK;
         bulk_g2s_nohint(dst, a.dp32 + d32(a, gbase + lane, 2, (int64_t)K * BK), rows_bytes, &S.mbar[b]);
     }
+}
+
+// Warp 0 of the resident-cost kernel tracks `frontier`: every column block <= frontier
+// of the current split is published.  A block publishes only after the block before
+// it (its last off-diagonal tile waits for that one), so one flag seen set vouches for
+// every block below it, and most tiles need no flag load at all.  When the frontier
+// advances, every lane of warp 0 fences the generic-proxy stores of the newly
+// published blocks (dp32 rows, block minima) against its later bulk copies, so the
+// copies themselves carry no fence.
+// res_probe: is block K published?  If K is past the frontier, the 32 lanes load the
+// flags of blocks K, K + st, K + 2 st, ... (below J) at once and the frontier moves to
+// the highest block seen published.
+__device__ __forceinline__ bool res_probe(const FastArgs &a, int split, int K, int J, int &frontier, int lane) {
+    if (K <= frontier) return true;
+    const int stride = (J - K + 31) / 32;
+    const int m = K + lane * stride;
+    const bool set = m < J && ld_acquire(a.done + (size_t)split * a.nJ + m) != 0;
+    const unsigned bal = __ballot_sync(0xffffffffu, set);
+    if (bal == 0u) return false;
+    frontier = K + (31 - __clz(bal)) * stride;
+    __syncwarp();
+    fence_proxy_async_global();
+    return true;
+}
+// res_wait: bounded wait until block K is published (after res_probe said no).
+__device__ __forceinline__ void res_wait(const FastArgs &a, int split, int K, int &frontier, int lane) {
+    int ok = 0;
+    if (lane == 0) ok = wait_block(a, split, K) ? 1 : 0;
+    ok = __shfl_sync(0xffffffffu, ok, 0);
+    if (ok) frontier = max(frontier, K);
+    __syncwarp();
+    fence_proxy_async_global();
 }
 
 // Resident interval costs: no producer warps.  Warp 0 claims the column blocks,
@@ -1092,6 +1124,7 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
     const uint64_t policy = policy_evict_first();
     uint32_t n = 0;  // tile sequence number: buffer n & 1, its fill number n >> 1
     unsigned long long n_run = 0, n_skip = 0;  // lane 0 of each warp: its (warp, tile) units
+    int frontier = -1, fsplit = -1;            // warp 0 (res_probe)
     for (;;) {
         if (ct == 0) S.ticket = atomicAdd(a.ticket, 1);
         __syncthreads();
@@ -1100,19 +1133,17 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
         const int J = t / a.nsplit, split = t % a.nsplit;
         const int g = split * a.Gc + id.gl;
         const bool own = id.active && g < a.G;
+        if (split != fsplit) { frontier = -1; fsplit = split; }
         cons_reset(cs);
         if (ct < 32) {
-            if (lane == 0 && J > 0) wait_block(a, split, 0);
-            __syncwarp();
+            if (J > 0 && !res_probe(a, split, 0, J, frontier, lane)) res_wait(a, split, 0, frontier, lane);
             res_issue(a, S, sDP, n & 1, 0, J, split, policy, lane);
         }
         for (int K = 0; K < J; K++) {  // off-diagonal tiles
             const int b = n & 1;
             bool pending = false;  // warp 0: tile K+1 still to be issued
             if (ct < 32) {
-                int ready = 1;
-                if (lane == 0 && K + 1 < J) ready = ld_acquire(a.done + (size_t)split * a.nJ + K + 1) != 0;
-                ready = __shfl_sync(0xffffffffu, ready, 0);
+                const bool ready = K + 1 >= J || res_probe(a, split, K + 1, J, frontier, lane);
                 if (ready) res_issue(a, S, sDP, b ^ 1, K + 1, J, split, policy, lane);
                 pending = !ready;
             }
@@ -1124,8 +1155,7 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
             }
             __syncthreads();  // buffer b free for tile K+2
             if (ct < 32 && pending) {
-                if (lane == 0) wait_block(a, split, K + 1);
-                __syncwarp();
+                res_wait(a, split, K + 1, frontier, lane);
                 res_issue(a, S, sDP, b ^ 1, K + 1, J, split, policy, lane);
             }
             n++;
