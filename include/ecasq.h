@@ -56,7 +56,7 @@ typedef struct CUstream_st *ecasq_stream_t; /* same type as cudaStream_t */
 #define ECASQ_EXACT_TABLES 16u    /* resolve every DP output exactly (default: only what eq. apx_final and the traceback read) */
 #define ECASQ_RESIDENT_COSTS 32u  /* fast DP: compute the lambda-independent interval costs C and Phi (Sec. 5, App. E)
                                      once per call into the workspace and stream them to every pass (workspace:
-                                     ecasq_workspace_size_flags with this flag; about 17 d^2 / 64 bytes extra) */
+                                     ecasq_workspace_size_flags with this flag; about 4.3 d^2 bytes extra) */
 
 typedef struct ecasq_params {
     int32_t s;                 /* codebook cap, 2..256 */
@@ -116,8 +116,9 @@ size_t ecasq_workspace_size(int64_t d, int32_t s, int64_t rows);
 
 /* Workspace bytes for calls made with `flags`: ecasq_workspace_size plus, with
  * ECASQ_RESIDENT_COSTS, the resident interval-cost tiles (fp32 C and Phi of
- * every pair k < j in 64 x 64 tiles: ceil(d/64)(ceil(d/64)+1)/2 tiles of
- * 34816 bytes, e.g. 73 GB at d = 2^17).  Returns 0 for invalid arguments or
+ * every pair k < j in 64 x 64 tiles, and per tile each column's minimum C and
+ * Phi: ceil(d/64)(ceil(d/64)+1)/2 tiles of 35328 bytes, e.g. 74 GB at
+ * d = 2^17).  Returns 0 for invalid arguments or
  * a size that does not fit in size_t. */
 size_t ecasq_workspace_size_flags(int64_t d, int32_t s, int64_t rows, uint32_t flags);
 

@@ -132,6 +132,7 @@ struct FastArgs {
     uint8_t *need;         // [G][s+1][ps] output resolved exactly
     float *corner;         // [nJ(nJ-1)/2][8]: state of pair (64K+63, 64J), K < J (N, E, Ec, A, Ac, C, Cc)
     const float *costs;    // resident interval costs (tile (K, J) at J(J+1)/2 + K), or null: computed per tile
+    float2 *tsum;          // with costs: per tile, {min_k C, min_k Phi} of its 64 columns (the rows' padding)
     int32_t *lists;        // [s+1][2][G ps]: needed outputs of layer i (g << 24 | j); 0: <= NMEM members, 1: more
     int *list_cnt;         // [s+1][2]
     float *mdp;            // [nJ][G][mdp_stride]: min over the block's 64 columns of dp32(g, i, .)
@@ -428,9 +429,11 @@ struct __align__(16) Smem {
     TileMeta meta[2];
     float wsum[2][2];                     // producer scan: per-warp totals
     int ticket;
-    int pad[3];
+    int sfront[2];                        // resident costs: frontier of the minima in stage buffer sb
+    int pad;
+    uint32_t needw[2][MAXCONS / 32];      // resident costs: per warp, the tiles of the batch it needs
     unsigned long long mbar[2];           // resident costs: bulk-copy completion of buffer b
-    unsigned long long pad2[2];
+    unsigned long long smbar[2];          // resident costs: completion of stage buffer sb
     float tau[kMaxS + 1];                 // FastParams::tau and lam32, read on every tile
     float lam32[kMaxG];
     __align__(16) float mdp[2][kMaxG][20];  // staged dp32 block minima (tile skipping, s <= 19)
@@ -545,6 +548,7 @@ __global__ void __launch_bounds__(NPROD) k_build_costs(FastArgs a, float *costs)
         tile_consts(a, K * BK, jl, S.kv, S.kw, S.kd);
         bar_sync(BAR_PROD, NPROD);
         tile_columns(a, K, J, jl, S.kv, S.kw, S.kd, S.wsum, S.C, S.Phi);
+        a.tsum[(size_t)t * BJ + jl] = make_float2(S.C[jl][BK], S.Phi[jl][BK]);  // this thread's own row
         fence_proxy_async_smem();
         bar_sync(BAR_PROD, NPROD);
         if (jl == 0) {
@@ -1039,33 +1043,48 @@ __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
     }
 }
 
-// Warp 0 of the resident-cost kernel: expect the bytes of tile (K, J) on mbar[b]
-// and issue its bulk copies into buffer b -- the interval costs from the resident
-// table and, off the diagonal, the dp32 rows (g, layers 2..s-1) of the split's
-// real multipliers (rows of other slots are never read).  The caller has made tile
-// K's rows visible to the copies (res_probe / res_wait).
-__device__ __forceinline__ void res_issue(const FastArgs &a, Smem &S, float *sDP, int b, int K, int J, int split,
-                                          uint64_t policy, int lane) {
-    const int L = a.s - 2, rowsDP = a.Gc * L;
+// Bulk copies of tile (K, J) into buffer b of the resident-cost kernel: the interval
+// costs from the resident table and, off the diagonal, the dp32 rows (g, layers
+// 2..s-1) of the split's real multipliers (rows of other slots are never read) and
+// their block minima; on the diagonal, row 2 of the block.  res_issue_costs (one
+// thread) expects every byte of the tile on mbar[b] and copies the costs, which no
+// block publishes; res_issue_rows(w) copies multiplier w's rows (w = 0 also the
+// minima) and needs block K made visible to the issuing thread's copies first
+// (res_probe / res_wait for warp 0, the fence after the stage wait for the others).
+// A copy may land before the expectation is posted: the phase cannot complete
+// before the single arrival, which carries the whole byte count.
+__device__ __forceinline__ void res_issue_costs(const FastArgs &a, Smem &S, int b, int K, int J, int split,
+                                                uint64_t policy) {
+    const int L = a.s - 2;
     const int gbase = split * a.Gc;
     const bool diag = K == J;
     const int ngv = std::min(a.G - gbase, a.Gc);  // real multipliers of the split
-    // off the diagonal: rows 2..s-1 of tile K; on it: row 2 of the block (S.diag[0])
     const uint32_t rows_bytes = (uint32_t)((diag ? 1 : L) * BK * sizeof(float));
-    if (lane == 0) {
-        const float *src = a.costs + cost_tile_idx(K, J) * kCostTileFloats;
-        const uint32_t mdp_bytes = (a.prune && !diag) ? (uint32_t)(ngv * a.mdp_stride * sizeof(float)) : 0u;
-        mbar_expect_tx(&S.mbar[b], 2 * kCostHalfBytes + (uint32_t)ngv * rows_bytes + mdp_bytes);
-        bulk_g2s(&S.C[b][0][0], src, kCostHalfBytes, &S.mbar[b], policy);
-        bulk_g2s(&S.Phi[b][0][0], src + kCostHalfFloats, kCostHalfBytes, &S.mbar[b], policy);
-        if (mdp_bytes)
-            bulk_g2s_nohint(&S.mdp[b][0][0], a.mdp + ((size_t)K * a.G + gbase) * a.mdp_stride, mdp_bytes, &S.mbar[b]);
-    }
+    const uint32_t mdp_bytes = (a.prune && !diag) ? (uint32_t)(ngv * a.mdp_stride * sizeof(float)) : 0u;
+    const float *src = a.costs + cost_tile_idx(K, J) * kCostTileFloats;
+    mbar_expect_tx(&S.mbar[b], 2 * kCostHalfBytes + (uint32_t)ngv * rows_bytes + mdp_bytes);
+    bulk_g2s(&S.C[b][0][0], src, kCostHalfBytes, &S.mbar[b], policy);
+    bulk_g2s(&S.Phi[b][0][0], src + kCostHalfFloats, kCostHalfBytes, &S.mbar[b], policy);
+}
+__device__ __forceinline__ void res_issue_rows(const FastArgs &a, Smem &S, float *sDP, int b, int K, int J, int split,
+                                               int w) {
+    const int L = a.s - 2, rowsDP = a.Gc * L;
+    const int gbase = split * a.Gc;
+    const bool diag = K == J;
+    const int ngv = std::min(a.G - gbase, a.Gc);
+    const uint32_t rows_bytes = (uint32_t)((diag ? 1 : L) * BK * sizeof(float));
+    if (w == 0 && a.prune && !diag)
+        bulk_g2s_nohint(&S.mdp[b][0][0], a.mdp + ((size_t)K * a.G + gbase) * a.mdp_stride,
+                        (uint32_t)(ngv * a.mdp_stride * sizeof(float)), &S.mbar[b]);
+    float *dst = diag ? &S.diag[0][w][0] : sDP + (size_t)b * rowsDP * BK + (size_t)w * L * BK;
+    bulk_g2s_nohint(dst, a.dp32 + d32(a, gbase + w, 2, (int64_t)K * BK), rows_bytes, &S.mbar[b]);
+}
+// Warp 0 alone issues the whole tile.
+__device__ __forceinline__ void res_issue(const FastArgs &a, Smem &S, float *sDP, int b, int K, int J, int split,
+                                          uint64_t policy, int lane) {
+    if (lane == 0) res_issue_costs(a, S, b, K, J, split, policy);
     __syncwarp();
-    if (lane < ngv) {
-        float *dst = diag ? &S.diag[0][lane][0] : sDP + (size_t)b * rowsDP * BK + (size_t)lane * L * BK;
-        bulk_g2s_nohint(dst, a.dp32 + d32(a, gbase + lane, 2, (int64_t)K * BK), rows_bytes, &S.mbar[b]);
-    }
+    if (lane < std::min(a.G - split * a.Gc, a.Gc)) res_issue_rows(a, S, sDP, b, K, J, split, lane);
 }
 
 // Warp 0 of the resident-cost kernel tracks `frontier`: every column block <= frontier
@@ -1100,9 +1119,88 @@ __device__ __forceinline__ void res_wait(const FastArgs &a, int split, int K, in
     fence_proxy_async_global();
 }
 
+// Tile skipping in batches (resident costs, two layer groups).  A batch is up to
+// kStageTiles consecutive off-diagonal tiles of block J; warp 0 stages their column
+// summaries (a.tsum) and the block minima of their column blocks (a.mdp, all G
+// multipliers) into a stage buffer with two bulk copies, one batch ahead.  The stage
+// buffers live where the diagonal parks its band state (free until the diagonal).
+constexpr int kStageTiles = 32;
+__host__ __device__ __forceinline__ size_t stage_floats(int G, int mdp_stride) {
+    return (size_t)kStageTiles * BJ * 2 + (size_t)kStageTiles * G * mdp_stride;
+}
+// The batch after the one ending at K1: 1, 1, 2, 4, ... kStageTiles tiles (the band
+// limits are +inf before the first tile and tighten fast).
+__device__ __forceinline__ int batch_end(int K1, int J) { return min(J, K1 + min(kStageTiles, max(1, K1))); }
+
+// Warp 0: stage tiles K0 <= K < K1 of block J into stage buffer sb.  Minima of blocks
+// past `frontier` may be incomplete in the copy; need_mask does not read them.
+__device__ __forceinline__ void res_stage(const FastArgs &a, Smem &S, float *stg, int sb, int K0, int K1, int J,
+                                          int frontier, uint64_t policy, int lane) {
+    if (lane == 0) {
+        const uint32_t tb = (uint32_t)((size_t)(K1 - K0) * BJ * sizeof(float2));
+        const uint32_t mb = (uint32_t)((size_t)(K1 - K0) * a.G * a.mdp_stride * sizeof(float));
+        S.sfront[sb] = frontier;  // ordered before the readers' wait by the arrive (release)
+        mbar_expect_tx(&S.smbar[sb], tb + mb);
+        bulk_g2s(stg, a.tsum + (cost_tile_idx(0, J) + (size_t)K0) * BJ, tb, &S.smbar[sb], policy);
+        bulk_g2s_nohint(stg + (size_t)kStageTiles * BJ * 2, a.mdp + (size_t)K0 * a.G * a.mdp_stride, mb, &S.smbar[sb]);
+    }
+}
+
+// Batch skip test of one warp over the staged tiles K0 <= K < K1: bit K - K0 of the
+// result is set when some output of the warp may take a candidate from tile K by the
+// test of cons_offdiag, here evaluated on the staged column minima and block minima
+// with the warp's band limits as they stand.  The limits only shrink as later tiles
+// fold, and rounding is monotone, so a tile this test rules out is ruled out by
+// cons_offdiag too: walking only the tiles some warp needs changes no result.  Blocks
+// past `fr` had no published minima when staged and are always needed.
+__device__ __forceinline__ uint32_t need_mask(const FastArgs &a, const Smem &S, const float *stg, int K0, int K1, int fr,
+                                              int g, const ConsId &id, const ConsState &cs) {
+    const int L = a.s - 2;
+    const float lam = S.lam32[g];
+    int rowl[LPT];
+    float lim[LPT][JPT];
+#pragma unroll
+    for (int l = 0; l < LPT; l++) {
+        rowl[l] = min(id.lg * LPT + l, L - 1);
+        const float tau = S.tau[3 + rowl[l]];
+#pragma unroll
+        for (int q = 0; q < JPT; q++) lim[l][q] = __fadd_rn(cs.best[l][q], __fmul_rn(cs.best[l][q], tau));
+    }
+    const float2 *ts = reinterpret_cast<const float2 *>(stg) + id.jq;
+    const float *md = stg + (size_t)kStageTiles * BJ * 2 + (size_t)g * a.mdp_stride + 2;
+    const int mstride = a.G * a.mdp_stride;
+    uint32_t mask = 0;
+#pragma unroll 2
+    for (int K = K0; K < K1; K++) {
+        bool need = true;
+        if (K <= fr) {
+            const int r = K - K0;
+            float lbq[JPT];
+#pragma unroll
+            for (int q = 0; q < JPT; q++) {
+                const float2 v = ts[r * BJ + NJQ * q];
+                lbq[q] = __fmaf_rn(lam, v.y, v.x);
+            }
+            need = false;
+#pragma unroll
+            for (int l = 0; l < LPT; l++) {
+                const float m = md[r * mstride + rowl[l]];
+#pragma unroll
+                for (int q = 0; q < JPT; q++) need |= __fadd_rn(m, lbq[q]) <= lim[l][q];
+            }
+        }
+        mask |= (__any_sync(0xffffffffu, need) ? 1u : 0u) << (K - K0);
+    }
+    return mask;
+}
+
 // Resident interval costs: no producer warps.  Warp 0 claims the column blocks,
-// waits for the flags and issues the bulk copies of tile K+1 while tile K is
-// evaluated (two buffers, one mbarrier each); all MAXCONS threads are consumers.
+// waits for the flags and issues the bulk copies of the next tile while the current
+// one is evaluated (two buffers, one mbarrier each); all MAXCONS threads are
+// consumers.  With tile skipping the off-diagonal tiles go in staged batches: every
+// warp runs need_mask over the batch and only the tiles some warp needs are copied
+// in and walked, so a tile every warp rules out costs neither HBM traffic nor a
+// barrier; the next batch is staged while this one is walked.
 __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     Smem &S = *reinterpret_cast<Smem *>(smem_raw);
@@ -1116,13 +1214,18 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
     if (ct == 0) {
         mbar_init(&S.mbar[0], 1);
         mbar_init(&S.mbar[1], 1);
+        mbar_init(&S.smbar[0], 1);
+        mbar_init(&S.smbar[1], 1);
         mbar_fence_init();
     }
     __syncthreads();
     const ConsId id = cons_id(a, ct);
     ConsState cs;
     const uint64_t policy = policy_evict_first();
-    uint32_t n = 0;  // tile sequence number: buffer n & 1, its fill number n >> 1
+    uint32_t n = 0;   // tile sequence number: buffer n & 1, its fill number n >> 1
+    uint32_t ns = 0;  // batch sequence number (tile skipping): stage buffer ns & 1, its fill ns >> 1
+    float *stage = sDP + (size_t)2 * rowsDP * BK;  // the park area, free off the diagonal
+    const size_t sfl = stage_floats(a.G, a.mdp_stride);
     unsigned long long n_run = 0, n_skip = 0;  // lane 0 of each warp: its (warp, tile) units
     int frontier = -1, fsplit = -1;            // warp 0 (res_probe)
     for (;;) {
@@ -1135,33 +1238,85 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
         const bool own = id.active && g < a.G;
         if (split != fsplit) { frontier = -1; fsplit = split; }
         cons_reset(cs);
-        if (ct < 32) {
-            if (J > 0 && !res_probe(a, split, 0, J, frontier, lane)) res_wait(a, split, 0, frontier, lane);
-            res_issue(a, S, sDP, n & 1, 0, J, split, policy, lane);
+        int issued = -1;  // the tile whose copies are in flight into buffer n & 1 (J: the diagonal), or -1
+        const int ngv = min(a.G - split * a.Gc, a.Gc);  // real multipliers of the split
+        if (a.prune && J > 0 && ct < 32) {  // stage the first batch
+            if (frontier < 0) res_probe(a, split, 0, J, frontier, lane);
+            res_stage(a, S, stage + (ns & 1) * sfl, ns & 1, 0, batch_end(0, J), J, frontier, policy, lane);
         }
-        for (int K = 0; K < J; K++) {  // off-diagonal tiles
-            const int b = n & 1;
-            bool pending = false;  // warp 0: tile K+1 still to be issued
-            if (ct < 32) {
-                const bool ready = K + 1 >= J || res_probe(a, split, K + 1, J, frontier, lane);
-                if (ready) res_issue(a, S, sDP, b ^ 1, K + 1, J, split, policy, lane);
-                pending = !ready;
+        for (int K0 = 0; K0 < J;) {
+            const int K1 = a.prune ? batch_end(K0, J) : min(J, K0 + 32);
+            uint32_t wm = 0xffffffffu;  // the warp's tiles of the batch
+            uint32_t U = 0xffffffffu;   // the tiles some warp needs
+            int frb = -1;               // tiles <= frb: every warp issues its own rows (res_issue_rows)
+            if (a.prune) {
+                const int sb = ns & 1;
+                mbar_wait_bounded(&S.smbar[sb], (ns >> 1) & 1u, a.st, a.abort_flag);
+                frb = S.sfront[sb];
+                if (lane == 0) fence_proxy_async_global();  // blocks <= frb, published, before this warp's copies
+                wm = own ? need_mask(a, S, stage + sb * sfl, K0, K1, frb, g, id, cs) : 0u;
+                if (lane == 0) S.needw[sb][ct >> 5] = wm;
+                __syncthreads();  // needw; every read of stage buffer sb is done
+                U = 0;
+                for (int w = 0; w < (int)(blockDim.x >> 5); w++) U |= S.needw[sb][w];
+                ns++;
+                if (K1 < J && ct < 32) {  // stage the next batch while this one is walked
+                    const int K2 = batch_end(K1, J);
+                    if (K2 - 1 > frontier) res_probe(a, split, frontier + 1, J, frontier, lane);
+                    res_stage(a, S, stage + (ns & 1) * sfl, ns & 1, K1, K2, J, frontier, policy, lane);
+                }
             }
-            mbar_wait_bounded(&S.mbar[b], (n >> 1) & 1u, a.st, a.abort_flag);
-            if (own) {
-                const bool ran = cons_offdiag(a, S, sDP + (size_t)b * rowsDP * BK, b, (uint32_t)K, g, id, cs);
-                n_run += ran ? 1 : 0;
-                n_skip += ran ? 0 : 1;
+            U &= (K1 - K0 == 32) ? 0xffffffffu : ((1u << (K1 - K0)) - 1u);
+            if (own) n_skip += (unsigned long long)(K1 - K0 - __popc(U));
+            if (U && issued < 0) {
+                const int Kf = K0 + __ffs(U) - 1;
+                if (Kf <= frb) {
+                    if (ct == 0) res_issue_costs(a, S, n & 1, Kf, J, split, policy);
+                    if (lane == 0 && (ct >> 5) < ngv) res_issue_rows(a, S, sDP, n & 1, Kf, J, split, ct >> 5);
+                } else if (ct < 32) {
+                    if (!res_probe(a, split, Kf, J, frontier, lane)) res_wait(a, split, Kf, frontier, lane);
+                    res_issue(a, S, sDP, n & 1, Kf, J, split, policy, lane);
+                }
             }
-            __syncthreads();  // buffer b free for tile K+2
-            if (ct < 32 && pending) {
-                res_wait(a, split, K + 1, frontier, lane);
-                res_issue(a, S, sDP, b ^ 1, K + 1, J, split, policy, lane);
+            while (U) {
+                const int K = K0 + __ffs(U) - 1;
+                U &= U - 1;
+                // the next tile to copy: the batch's next needed one, else the diagonal after
+                // the last batch, else (no skipping) the next batch's first tile
+                const int Kn = U ? K0 + __ffs(U) - 1 : (K1 == J ? J : (a.prune ? -1 : K1));
+                const int b = n & 1;
+                bool pending = false;  // warp 0: the rows of tile Kn still to be issued
+                if (Kn >= 0 && Kn < J && Kn <= frb) {
+                    if (ct == 0) res_issue_costs(a, S, b ^ 1, Kn, J, split, policy);
+                    if (lane == 0 && (ct >> 5) < ngv) res_issue_rows(a, S, sDP, b ^ 1, Kn, J, split, ct >> 5);
+                } else if (ct < 32 && Kn >= 0) {
+                    const bool ready = Kn >= J || res_probe(a, split, Kn, J, frontier, lane);
+                    if (ready)
+                        res_issue(a, S, sDP, b ^ 1, Kn, J, split, policy, lane);
+                    else if (lane == 0)
+                        res_issue_costs(a, S, b ^ 1, Kn, J, split, policy);  // the costs publish nothing
+                    pending = !ready;
+                }
+                issued = Kn;
+                mbar_wait_bounded(&S.mbar[b], (n >> 1) & 1u, a.st, a.abort_flag);
+                if (own) {
+                    const bool ran = ((wm >> (K - K0)) & 1u) &&
+                                     cons_offdiag(a, S, sDP + (size_t)b * rowsDP * BK, b, (uint32_t)K, g, id, cs);
+                    n_run += ran ? 1 : 0;
+                    n_skip += ran ? 0 : 1;
+                }
+                __syncthreads();  // buffer b free for the tile after Kn
+                if (ct < 32 && pending) {
+                    res_wait(a, split, Kn, frontier, lane);
+                    if (lane < ngv) res_issue_rows(a, S, sDP, b ^ 1, Kn, J, split, lane);
+                }
+                n++;
             }
-            n++;
+            K0 = K1;
         }
-        {  // the diagonal tile (issued with tile J-1, or at the block start when J = 0)
+        {  // the diagonal tile (issued with the last tile walked, else now)
             const int b = n & 1;
+            if (issued != J && ct < 32) res_issue(a, S, sDP, b, J, J, split, policy, lane);
             mbar_wait_bounded(&S.mbar[b], (n >> 1) & 1u, a.st, a.abort_flag);
             uint32_t *park = reinterpret_cast<uint32_t *>(sDP + (size_t)2 * rowsDP * BK);
             if (a.lgc == 2)
@@ -1520,13 +1675,15 @@ static void band_factors(int s, FastParams &fp) {
     }
 }
 
+// The resident table: every tile's C and Phi rows, then every tile's column summary
+// (BJ float2), both indexed by J(J+1)/2 + K with J < ceil(d / 64).
 size_t resident_costs_bytes(int64_t d) {
     if (d < 1) return 0;
     double nJ = (double)cdiv(d, BJ);
-    double bytes = nJ * (nJ + 1.0) * 0.5 * (double)kCostTileFloats * sizeof(float);
+    double bytes = nJ * (nJ + 1.0) * 0.5 * ((double)kCostTileFloats * sizeof(float) + BJ * sizeof(float2));
     if (!(bytes < 9.0e18)) return 0;
     size_t n = (size_t)cdiv(d, BJ);
-    return n * (n + 1) / 2 * kCostTileFloats * sizeof(float);
+    return n * (n + 1) / 2 * (kCostTileFloats * sizeof(float) + BJ * sizeof(float2));
 }
 
 int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, const Layout &Lw, cudaStream_t st,
@@ -1586,6 +1743,10 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     a.mdp_stride = mdp_stride(s);
     a.prune = (costs && a.lgc == 2 && a.mdp_stride <= 20) ? 1 : 0;
     a.costs = costs;
+    if (costs) {
+        const size_t nJd = (size_t)cdiv(Lw.d, BJ);
+        a.tsum = reinterpret_cast<float2 *>(costs + nJd * (nJd + 1) / 2 * kCostTileFloats);
+    }
     a.prm = dprm;
     a.done = flags;
     a.ticket = flags + (size_t)kMaxG * a.nJ;
@@ -1623,7 +1784,9 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
         ECASQ_LAUNCH_CHECK();
     }
     size_t smem = smem_bytes(a.Gc, s);
-    if (costs && a.lgc == 2) smem += (size_t)3 * LPT * JPT * a.ncons * sizeof(uint32_t);  // parked band state
+    if (costs && a.lgc == 2)  // parked band state; off the diagonal, the two stage buffers
+        smem += std::max((size_t)3 * LPT * JPT * a.ncons * sizeof(uint32_t),
+                         a.prune ? 2 * stage_floats(G, a.mdp_stride) * sizeof(float) : (size_t)0);
     auto wave = costs ? k_wavefront_res : k_wavefront;
     ECASQ_CUDA_TRY(cudaFuncSetAttribute(wave, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     int grid = std::min(nsm, a.nJ * a.nsplit);

@@ -42,10 +42,10 @@ def test_host_only_calls():
     assert native.ecasq_workspace_size(0, 8) == 0
     assert native.ecasq_workspace_size(100, 1) == 0
     assert native.ecasq_workspace_size(100, 257) == 0
-    # resident interval costs: 34816 bytes per 64 x 64 tile on top of the base size
+    # resident interval costs: 35328 bytes per 64 x 64 tile (C, Phi, column minima) on top of the base size
     base = native.ecasq_workspace_size(4096, 8)
     assert native.ecasq_workspace_size_flags(4096, 8, 1, 0) == base
-    assert native.ecasq_workspace_size_flags(4096, 8, 1, native.RESIDENT_COSTS) == base + 64 * 65 // 2 * 34816
+    assert native.ecasq_workspace_size_flags(4096, 8, 1, native.RESIDENT_COSTS) == base + 64 * 65 // 2 * 35328
     assert native.ecasq_workspace_size_flags(2 ** 31 - 1, 8, 1, native.RESIDENT_COSTS) == 0  # beyond size_t
     assert native.ecasq_workspace_size_flags(0, 8, 1, native.RESIDENT_COSTS) == 0
     # preparation alone: the sort, histogram and sums (linear in d), far below a solve's

@@ -119,7 +119,7 @@ def test_resident_costs_workspace_checks(E):
     base = E.ecasq_workspace_size(d, s)
     assert E.ecasq_workspace_size_flags(d, s, 1, 0) == base
     nJ = (d + 63) // 64
-    assert E.ecasq_workspace_size_flags(d, s, 1, E.RESIDENT_COSTS) >= base + nJ * (nJ + 1) // 2 * 34816
+    assert E.ecasq_workspace_size_flags(d, s, 1, E.RESIDENT_COSTS) >= base + nJ * (nJ + 1) // 2 * 35328
     x = workloads.normal(d, 2)
     small = E.workspace(d, s)  # no room for the resident tiles
     with pytest.raises(E.EcasqError) as ei:
