@@ -766,7 +766,9 @@ __device__ __forceinline__ void cons_diag(const FastArgs &a, Smem &S, int b, int
 // from shared memory, and every column's minimum is complete within one lane (pairs
 // k >= j carry C = +inf in the tile and never win).  The band state is parked in `park`
 // ([3][LPT][JPT][ncons] words: best, run 1, run 2) and folded there; the block
-// ends with its diagonal, so the registers are not restored.
+// ends with its diagonal, so the registers are not restored.  A warp holds one
+// multiplier, and the rows of S.diag and the parked slots it reads and writes are
+// that multiplier's alone, so the layers need only a warp barrier each.
 // Group g4 of a diagonal lane (half 0: lanes 0-15, half 1: lanes 16-31): its column
 // (q = 0: the long one, 1: the short one) and first k.  Groups 0-11 are k 0..47 of the
 // long column for both halves; groups 12-15 are k 48..63 of the long column (half 0)
@@ -826,11 +828,13 @@ __device__ __forceinline__ void cons_diag_pair(const FastArgs &a, Smem &S, uint3
     for (int li = 0; li < L; li++) {
         const int i = 3 + li;
         const int olg = li / LPT, l = li - olg * LPT;
-        // running minima (float bits; candidates are >= +0) of the long and the short
-        // column, two chains each
-        int b0 = 0x7f800000, b1 = 0x7f800000, s0 = 0x7f800000, s1 = 0x7f800000;
+        // minima (float bits; candidates are >= +0) of the long and the short column:
+        // each group of four k reduces on its own, then the groups by a tree, so the
+        // layer's dependency chain is a few mins deep
+        int lmin = 0x7f800000, smin = 0x7f800000;
         if (own) {
             const float *prow = &S.diag[cur][id.gl][0];
+            int m[kDiagGroups];
 #pragma unroll
             for (int g4 = 0; g4 < kDiagGroups; g4++) {
                 int q, k;
@@ -838,19 +842,15 @@ __device__ __forceinline__ void cons_diag_pair(const FastArgs &a, Smem &S, uint3
                 const float4 d4 = *reinterpret_cast<const float4 *>(prow + k);
                 const float2 t0 = add2(make_float2(d4.x, d4.y), W[2 * g4]);
                 const float2 t1 = add2(make_float2(d4.z, d4.w), W[2 * g4 + 1]);
-                if (g4 < 12) {
-                    b0 = min(min(b0, __float_as_int(t0.x)), __float_as_int(t0.y));
-                    b1 = min(min(b1, __float_as_int(t1.x)), __float_as_int(t1.y));
-                } else if (g4 < 16) {  // the long column for half 0, the short one for half 1
-                    const int m = min(min(__float_as_int(t0.x), __float_as_int(t0.y)),
-                                      min(__float_as_int(t1.x), __float_as_int(t1.y)));
-                    b0 = half ? b0 : min(b0, m);
-                    s0 = half ? min(s0, m) : s0;
-                } else {
-                    s0 = min(min(s0, __float_as_int(t0.x)), __float_as_int(t0.y));
-                    s1 = min(min(s1, __float_as_int(t1.x)), __float_as_int(t1.y));
-                }
+                m[g4] = min(min(__float_as_int(t0.x), __float_as_int(t0.y)), min(__float_as_int(t1.x), __float_as_int(t1.y)));
             }
+            // groups 0-11: the long column; 12-15: long (half 0) or short (half 1); 16-19: short
+            const int A = min(min(min(min(m[0], m[1]), min(m[2], m[3])), min(min(m[4], m[5]), min(m[6], m[7]))),
+                              min(min(m[8], m[9]), min(m[10], m[11])));
+            const int B = min(min(m[12], m[13]), min(m[14], m[15]));
+            const int C = min(min(m[16], m[17]), min(m[18], m[19]));
+            lmin = half ? A : min(A, B);
+            smin = half ? min(B, C) : C;
         }
         if (own) {
             // each lane folds its two columns into the owner's slots (layer group olg,
@@ -859,7 +859,7 @@ __device__ __forceinline__ void cons_diag_pair(const FastArgs &a, Smem &S, uint3
 #pragma unroll
             for (int c = 0; c < 2; c++) {
                 const int q = c ? qs : qb;
-                const int mq = c ? min(s0, s1) : min(b0, b1);
+                const int mq = c ? smin : lmin;
                 const int jl = id.jq + NJQ * q;
                 const int x = (l * JPT + q) * nc + cto;
                 float bb = __uint_as_float(park[x]);
@@ -871,7 +871,7 @@ __device__ __forceinline__ void cons_diag_pair(const FastArgs &a, Smem &S, uint3
                 S.diag[cur ^ 1][id.gl][jl] = bb;
             }
         }
-        bar_sync(BAR_CONS, nc);
+        __syncwarp();  // the layer's row and parked state belong to this warp alone
         cur ^= 1;
     }
     // the block's final values from the parked state, and the block minimum of
