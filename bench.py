@@ -42,10 +42,11 @@ SM_COUNT = 152
 FP32_LANES = 128          # FP32-pipe lanes per SM (adds and min/max share them)
 SM_MAX_MHZ = 2070.0
 OPS_PER_CANDIDATE = 2     # one add and one min per min-plus candidate
-# DRAM bytes of one k_wavefront_res launch per 64 x 64 tile, from the ncu capture in
-# profiles/k_wavefront_res_lognormal_d16384_s16.md (read 1.146089 GB + write 7.2 MB over
-# 32896 tiles); the benchmark launch is scaled by its own tile count.
-TRAFFIC_PER_TILE = (1.146089e9 + 7.165184e6) / 32896
+# DRAM bytes of k_wavefront_res per interval-cost tile it copies in (64 x 64 pairs,
+# 34 816 B of C and Phi, plus the dp32 rows and minima that miss L2), from the ncu
+# capture in profiles/k_wavefront_res_lognormal_d16384_s16.md; the benchmark launch is
+# scaled by the tiles it fetched (tile skipping leaves most tiles in HBM unread).
+TRAFFIC_PER_FETCHED_TILE = None
 ORACLE_SAMPLE = 16384     # entries of the CPU baseline's bounded sample
 
 
@@ -449,11 +450,15 @@ def main():
     # roofline of the min-plus kernel: FP32-pipe ops (one add + one min per candidate)
     achieved = OPS_PER_CANDIDATE * cand_total / (dp_ms / 1000.0) / 1e12 if dp_ms > 0 else None
     peak = SM_COUNT * FP32_LANES * SM_MAX_MHZ * 1e6 / 1e12
-    nJ = (last_p + 63) // 64
-    traffic = TRAFFIC_PER_TILE * nJ * (nJ + 1) // 2 if (flags & E.RESIDENT_COSTS) else None
+    last_launches = max(results[-1]["dp_kernel_launches"], 1)
+    fetched_per_launch = st["tiles_fetched"] / last_launches
+    traffic = (TRAFFIC_PER_FETCHED_TILE * fetched_per_launch
+               if (flags & E.RESIDENT_COSTS) and TRAFFIC_PER_FETCHED_TILE else None)
     roofline = {"bound": "alu", "achieved": achieved, "peak": peak, "unit": "TOP/s",
                 "frac": (achieved / peak) if achieved else None, "traffic": traffic,
-                "traffic_note": "DRAM bytes per launch, scaled from an ncu capture at d = 16384 by tiles",
+                "traffic_note": "DRAM bytes per launch: bytes per fetched cost tile from an ncu capture at "
+                                "d = 16384, times the tiles this launch fetched",
+                "tiles_fetched_per_launch": fetched_per_launch,
                 "kernel": "k_wavefront_res" if (flags & E.RESIDENT_COSTS) else "k_wavefront",
                 "peak_basis": "152 SMs x 128 FP32-pipe lanes (adds and mins share them) x 2070 MHz max clock",
                 "avg_launch_ms": dp_ms / max(dp_launches, 1), "launches": dp_launches,
@@ -507,6 +512,7 @@ def main():
                          "refine_rounds": last["refine_rounds"], "candidates_per_solve": last["candidates"],
                          "rescored_per_solve": last["rescored"], "dp_pass_ms": dp_ms / max(dp_launches, 1),
                          "tile_units_run": st["tiles_run"], "tile_units_skipped": st["tiles_skipped"],
+                         "cost_tiles_fetched": st["tiles_fetched"],
                          "solves_per_s": world * args.steps / (ms / 1000.0)},
                "roofline": roofline, "cpu_baseline": cb, "e2e": e2e, "gpu_launches": launches,
                "clocks": clocks}

@@ -49,6 +49,7 @@ struct DevStatus {
     int64_t tiles_skipped; // ... and skipped by the lower bound
     int64_t grid_nL;      // permissible set: |L| = #{p_a <= min x}, |R| = #{p_b >= max x} (Sec. 5)
     int64_t grid_nR;
+    int64_t tiles_fetched; // fast DP, resident costs: interval-cost tiles copied in from HBM
 };
 
 struct Layout {

@@ -1333,6 +1333,7 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
         atomicAdd((unsigned long long *)&a.st->tiles_run, n_run);
         atomicAdd((unsigned long long *)&a.st->tiles_skipped, n_skip);
     }
+    if (ct == 0 && n) atomicAdd((unsigned long long *)&a.st->tiles_fetched, (unsigned long long)n);  // one cost tile per buffer fill
 }
 
 // ------------------------------------------------------------ base layer

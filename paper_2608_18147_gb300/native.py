@@ -164,13 +164,13 @@ def _check(rc, where, ok=(OK,)):
 def ws_status(ws):
     """Counters the library leaves at the start of a workspace after a call
     (unique values, device-side flags, fast-DP statistics)."""
-    raw = ws[:112].cpu().numpy().tobytes()
+    raw = ws[:120].cpu().numpy().tobytes()
     (p, nonfinite, range_err, timeout, bound_viol, norm2, rescored, overflow, last_s, last_G, last_d, members,
-     big_bands, tiles_run, tiles_skipped, grid_nL, grid_nR) = __import__("struct").unpack("<qiiiidqqiiqqqqqqq", raw)
+     big_bands, tiles_run, tiles_skipped, grid_nL, grid_nR, tiles_fetched) = __import__("struct").unpack("<qiiiidqqiiqqqqqqqq", raw)
     return dict(p=p, nonfinite=nonfinite, range_err=range_err, timeout=timeout, bound_viol=bound_viol, norm2=norm2,
                 rescored=rescored, overflow=overflow, last_s=last_s, last_G=last_G, last_d=last_d, members=members,
                 big_bands=big_bands, tiles_run=tiles_run, tiles_skipped=tiles_skipped, grid_nL=grid_nL,
-                grid_nR=grid_nR)
+                grid_nR=grid_nR, tiles_fetched=tiles_fetched)
 
 
 def ecasq_workspace_size(d, s, rows=1) -> int:
