@@ -21,12 +21,9 @@ __device__ __forceinline__ uint64_t splitmix64(uint64_t z) {
 
 __device__ __forceinline__ int quant_one(float xv, int64_t i, const float *q, int m, uint64_t seed, bool &bad) {
     if (!(xv >= q[0] && xv <= q[m - 1])) { bad = true; return 0; }
-    int lo = 0, hi = m - 1;  // largest t with q[t] <= x
-    while (lo < hi) {
-        int mid = (lo + hi + 1) >> 1;
-        if (q[mid] <= xv) lo = mid; else hi = mid - 1;
-    }
-    int t = lo;
+    int t = 0;  // largest t with q[t] <= x: one step per bit of m - 1, the same count in every lane
+    for (int b = m > 1 ? 1 << (31 - __clz(m - 1)) : 0; b; b >>= 1)
+        if (t + b < m && q[t + b] <= xv) t += b;
     if (q[t] != xv) {
         uint64_t z = splitmix64(seed + (uint64_t)(i + 1) * 0x9E3779B97F4A7C15ull);
         float k = __fmul_rn((float)(uint32_t)(z >> 40), 0x1p-24f);
@@ -37,53 +34,128 @@ __device__ __forceinline__ int quant_one(float xv, int64_t i, const float *q, in
     return t;
 }
 
-__global__ void __launch_bounds__(256) k_quantize(const float *__restrict__ x, int64_t d, const float *__restrict__ Q,
-                                                  int m, uint64_t seed, uint8_t *__restrict__ idx,
-                                                  uint32_t *__restrict__ counts, DevStatus *st) {
+// Codebooks of at most kPrivBins values count their indices in per-thread
+// histograms: 16-bit counters packed in pairs, word w of thread t at
+// ph[w * 256 + t] (each thread its own bank column: no conflicts, no atomics).  A
+// thread folds its counters into the block's 32-bit totals after every
+// kFoldEntries of its entries, before any counter could pass 65535 (only inputs of
+// more than about 10^10 entries get that far).
+constexpr int kPrivBins = 32;
+constexpr int kQThreads = 256;
+constexpr int kFoldEntries = 32768;
+
+__device__ __forceinline__ void priv_count(uint32_t *ph, int t) {
+    ph[(t >> 1) * kQThreads + threadIdx.x] += 1u << ((t & 1) << 4);
+}
+__device__ __forceinline__ void priv_fold(uint32_t *ph, uint32_t *hcount, int m) {
+    for (int w = 0; w < (m + 1) >> 1; w++) {
+        const uint32_t v = ph[w * kQThreads + threadIdx.x];
+        if (v) {
+            if (v & 0xffffu) atomicAdd(&hcount[2 * w], v & 0xffffu);
+            if (v >> 16) atomicAdd(&hcount[2 * w + 1], v >> 16);
+            ph[w * kQThreads + threadIdx.x] = 0;
+        }
+    }
+}
+
+// Encode.  Vector path: each thread takes two groups of four entries per step (two
+// 16-byte loads in flight before any arithmetic), writes four indices per group.
+template <bool PRIV>
+__global__ void __launch_bounds__(kQThreads) k_quantize(const float *__restrict__ x, int64_t d,
+                                                        const float *__restrict__ Q, int m, uint64_t seed,
+                                                        uint8_t *__restrict__ idx, uint32_t *__restrict__ counts,
+                                                        DevStatus *st) {
     __shared__ float q[kMaxS];
     __shared__ uint32_t hcount[kMaxS];
+    __shared__ uint32_t ph[PRIV ? (kPrivBins / 2) * kQThreads : 1];
     for (int r = threadIdx.x; r < kMaxS; r += blockDim.x) {
         q[r] = r < m ? Q[r] : 0.0f;
         hcount[r] = 0;
     }
+    if (PRIV)
+        for (int w = 0; w < kPrivBins / 2; w++) ph[w * kQThreads + threadIdx.x] = 0;
     __syncthreads();
+    auto count = [&](int t) {
+        if (PRIV) priv_count(ph, t); else atomicAdd(&hcount[t], 1u);
+    };
     bool bad = false;
-    bool vec = ((reinterpret_cast<uintptr_t>(x) & 15) == 0) && ((reinterpret_cast<uintptr_t>(idx) & 3) == 0);
-    int64_t ngroups = d / 4;
-    int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    int64_t g0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (vec) {
-        for (int64_t g = g0; g < ngroups; g += stride) {
-            float4 xv = reinterpret_cast<const float4 *>(x)[g];
-            int64_t i = 4 * g;
-            int t0 = quant_one(xv.x, i, q, m, seed, bad);
-            int t1 = quant_one(xv.y, i + 1, q, m, seed, bad);
-            int t2 = quant_one(xv.z, i + 2, q, m, seed, bad);
-            int t3 = quant_one(xv.w, i + 3, q, m, seed, bad);
-            reinterpret_cast<uchar4 *>(idx)[g] = make_uchar4((uint8_t)t0, (uint8_t)t1, (uint8_t)t2, (uint8_t)t3);
-            atomicAdd(&hcount[t0], 1u); atomicAdd(&hcount[t1], 1u);
-            atomicAdd(&hcount[t2], 1u); atomicAdd(&hcount[t3], 1u);
+    const bool vec = ((reinterpret_cast<uintptr_t>(x) & 15) == 0) && ((reinterpret_cast<uintptr_t>(idx) & 3) == 0);
+    const int64_t ngroups = vec ? d / 4 : 0;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    const int64_t g0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const float4 *x4 = reinterpret_cast<const float4 *>(x);
+    uchar4 *i4 = reinterpret_cast<uchar4 *>(idx);
+    int since_fold = 0;  // entries counted since the last fold
+    for (int64_t g = g0; g < ngroups; g += 2 * stride) {
+        const int64_t h = g + stride;
+        const bool two = h < ngroups;
+        const float4 xa = x4[g];
+        const float4 xb = two ? x4[h] : make_float4(0.f, 0.f, 0.f, 0.f);
+        {
+            const int64_t i = 4 * g;
+            const int t0 = quant_one(xa.x, i, q, m, seed, bad), t1 = quant_one(xa.y, i + 1, q, m, seed, bad);
+            const int t2 = quant_one(xa.z, i + 2, q, m, seed, bad), t3 = quant_one(xa.w, i + 3, q, m, seed, bad);
+            i4[g] = make_uchar4((uint8_t)t0, (uint8_t)t1, (uint8_t)t2, (uint8_t)t3);
+            count(t0); count(t1); count(t2); count(t3);
+        }
+        if (two) {
+            const int64_t i = 4 * h;
+            const int t0 = quant_one(xb.x, i, q, m, seed, bad), t1 = quant_one(xb.y, i + 1, q, m, seed, bad);
+            const int t2 = quant_one(xb.z, i + 2, q, m, seed, bad), t3 = quant_one(xb.w, i + 3, q, m, seed, bad);
+            i4[h] = make_uchar4((uint8_t)t0, (uint8_t)t1, (uint8_t)t2, (uint8_t)t3);
+            count(t0); count(t1); count(t2); count(t3);
+        }
+        if (PRIV && (since_fold += 8) >= kFoldEntries) {
+            priv_fold(ph, hcount, m);
+            since_fold = 0;
         }
     }
-    int64_t start = vec ? 4 * ngroups : 0;
-    for (int64_t i = start + g0; i < d; i += stride) {
-        int t = quant_one(x[i], i, q, m, seed, bad);
+    for (int64_t i = 4 * ngroups + g0; i < d; i += stride) {
+        const int t = quant_one(x[i], i, q, m, seed, bad);
         idx[i] = (uint8_t)t;
-        atomicAdd(&hcount[t], 1u);
+        count(t);
+        if (PRIV && ++since_fold >= kFoldEntries) {
+            priv_fold(ph, hcount, m);
+            since_fold = 0;
+        }
     }
     if (bad) st->range_err = 1;
     __syncthreads();
+    if (PRIV) {
+        // bins of the per-thread counters, summed over the block: warp w takes words w, w + 8, ...
+        const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+        for (int w = wid; w < (m + 1) >> 1; w += kQThreads / 32) {
+            uint32_t lo = 0, hi = 0;
+            for (int c = lane; c < kQThreads; c += 32) {
+                const uint32_t v = ph[w * kQThreads + c];
+                lo += v & 0xffffu;
+                hi += v >> 16;
+            }
+            for (int o = 16; o; o >>= 1) {
+                lo += __shfl_xor_sync(0xffffffffu, lo, o);
+                hi += __shfl_xor_sync(0xffffffffu, hi, o);
+            }
+            if (lane == 0) {
+                hcount[2 * w] += lo;  // only warp wid writes these two bins after the barrier
+                if (2 * w + 1 < m) hcount[2 * w + 1] += hi;
+            }
+        }
+        __syncthreads();
+    }
     for (int r = threadIdx.x; r < m; r += blockDim.x)
         if (hcount[r]) atomicAdd(&counts[r], hcount[r]);
 }
 
 int launch_quantize(const float *x, int64_t d, const float *Q, int m, uint64_t seed, uint8_t *idx, uint32_t *counts,
                     DevStatus *st, int num_sms, cudaStream_t stream) {
-    int64_t groups = cdiv(d, 4);
-    int64_t blocks = std::min<int64_t>(cdiv(groups, 256), (int64_t)num_sms * 8);
+    const int64_t groups = cdiv(d, 4);
+    int64_t blocks = std::min<int64_t>(cdiv(groups, 2 * kQThreads), (int64_t)num_sms * 8);
     if (blocks < 1) blocks = 1;
     note_launch();
-    k_quantize<<<(unsigned)blocks, 256, 0, stream>>>(x, d, Q, m, seed, idx, counts, st);
+    if (m <= kPrivBins)
+        k_quantize<true><<<(unsigned)blocks, kQThreads, 0, stream>>>(x, d, Q, m, seed, idx, counts, st);
+    else
+        k_quantize<false><<<(unsigned)blocks, kQThreads, 0, stream>>>(x, d, Q, m, seed, idx, counts, st);
     ECASQ_LAUNCH_CHECK();
     return ECASQ_OK;
 }

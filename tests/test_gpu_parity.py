@@ -339,6 +339,27 @@ def test_quantize_bit_exact(E, oracle_mod, d, offset):
         assert he == pytest.approx(oh, rel=1e-12, abs=1e-15)
 
 
+@pytest.mark.parametrize("m", [2, 32, 33, 256])
+@pytest.mark.parametrize("offset", [0, 1])
+def test_quantize_bit_exact_codebook_sizes(E, oracle_mod, m, offset):
+    """Codebooks on both sides of the per-thread-histogram limit (32 values) and at the
+    cap, on an input long enough for several grid-stride steps per thread."""
+    import torch
+    d = 3_000_001
+    x = workloads.signed_lognormal(d + offset, 11)
+    xg = torch.as_tensor(x).cuda()[offset:]
+    xs = x[offset:]
+    Q = np.unique(np.quantile(xs, np.linspace(0.0, 1.0, m)).astype(np.float32))
+    Q[0], Q[-1] = xs.min(), xs.max()
+    assert Q.size == m
+    idx, counts, he = E.ecasq_quantize(xg, Q, 99)
+    oi, oc, oh = oracle_mod.quantize(xs, Q, 99)
+    np.testing.assert_array_equal(idx.cpu().numpy(), oi)
+    np.testing.assert_array_equal(counts.cpu().numpy().astype(np.uint32), oc)
+    assert int(oc.sum()) == d
+    assert he == pytest.approx(oh, rel=1e-12, abs=1e-15)
+
+
 def test_quantize_rejects_out_of_range(E):
     x = np.array([0.0, 2.0], np.float32)
     with pytest.raises(E.EcasqError) as ei:
