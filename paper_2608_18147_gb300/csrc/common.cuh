@@ -13,7 +13,9 @@ namespace ecasq {
 constexpr int kMaxS = 256;      // codebook cap
 constexpr int kMaxG = 8;        // multipliers per DP pass
 constexpr int kSortTile = 2048; // keys per radix-sort block
-constexpr int kScanTile = 1024; // elements per prefix-scan block
+constexpr int kScanTile = 1024; // longest row of the batched path (one block of 256 threads)
+constexpr int kHistPer = 16;    // sorted keys per thread in the histogram / prefix-sum blocks
+constexpr int kHistTile = 256 * kHistPer;  // keys per histogram block
 
 #define ECASQ_CUDA_TRY(expr)                          \
     do {                                              \
@@ -112,6 +114,13 @@ __device__ __forceinline__ dd dd_add(dd a, dd b) {
     s.lo = __dadd_rn(s.lo, t.hi);
     s = fast_two_sum(s.hi, s.lo);
     s.lo = __dadd_rn(s.lo, t.lo);
+    return fast_two_sum(s.hi, s.lo);
+}
+// a + b for a double b: the value dd_add(a, {b, 0}) gives (its second two_sum adds zero and
+// its last renormalisation leaves a normalised pair unchanged), in half the operations.
+__device__ __forceinline__ dd dd_add_d(dd a, double b) {
+    dd s = two_sum(a.hi, b);
+    s.lo = __dadd_rn(s.lo, a.lo);
     return fast_two_sum(s.hi, s.lo);
 }
 __device__ __forceinline__ dd dd_neg(dd a) { return {-a.hi, -a.lo}; }

@@ -48,19 +48,24 @@ __global__ void __launch_bounds__(256) k_radix_count(const uint32_t *__restrict_
     counts[(size_t)threadIdx.x * nb + blockIdx.x] = h[threadIdx.x];
 }
 
-// In-place exclusive scan of n uint32 values by one block of 1024 threads, in
-// coalesced tiles of 4096 (four consecutive values per thread) with a running carry.
-__global__ void __launch_bounds__(1024) k_scan_u32(uint32_t *a, int64_t n) {
+// In-place exclusive scan of uint32 values.  Block b scans a[b*chunk .. min(n, (b+1)*chunk))
+// by 1024 threads, in coalesced tiles of 4096 (four consecutive values per thread) with a
+// running carry that starts at carry_in[b] (0 when carry_in is null).  One block with
+// chunk = n scans the whole array; with several blocks, carry_in holds the exclusive
+// prefix of the chunks' totals (k_scan_chunk_sums, then a one-block scan of those).
+__global__ void __launch_bounds__(1024) k_scan_u32(uint32_t *a, int64_t n, int64_t chunk,
+                                                   const uint32_t *carry_in) {
     __shared__ uint32_t wsum[32];
     __shared__ uint32_t carry;
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-    if (threadIdx.x == 0) carry = 0;
+    const int64_t lo = (int64_t)blockIdx.x * chunk, hi = min(n, lo + chunk);
+    if (threadIdx.x == 0) carry = carry_in ? carry_in[blockIdx.x] : 0u;
     __syncthreads();
-    for (int64_t base = 0; base < n; base += 4 * 1024) {
+    for (int64_t base = lo; base < hi; base += 4 * 1024) {
         const int64_t i0 = base + 4 * (int64_t)threadIdx.x;
         uint32_t v[4];
 #pragma unroll
-        for (int e = 0; e < 4; e++) v[e] = i0 + e < n ? a[i0 + e] : 0u;
+        for (int e = 0; e < 4; e++) v[e] = i0 + e < hi ? a[i0 + e] : 0u;
         const uint32_t s = v[0] + v[1] + v[2] + v[3];
         uint32_t incl = s;
         for (int o = 1; o < 32; o <<= 1) {
@@ -81,13 +86,52 @@ __global__ void __launch_bounds__(1024) k_scan_u32(uint32_t *a, int64_t n) {
         uint32_t run = carry + wsum[wid] + incl - s;
 #pragma unroll
         for (int e = 0; e < 4; e++) {
-            if (i0 + e < n) a[i0 + e] = run;
+            if (i0 + e < hi) a[i0 + e] = run;
             run += v[e];
         }
         __syncthreads();  // every thread has read carry and wsum
         if (threadIdx.x == blockDim.x - 1) carry = run;  // the old carry plus this tile's total
         __syncthreads();
     }
+}
+
+// Totals of the chunks a[b*chunk .. min(n, (b+1)*chunk)), one block of 1024 per chunk.
+__global__ void __launch_bounds__(1024) k_scan_chunk_sums(const uint32_t *__restrict__ a, int64_t n, int64_t chunk,
+                                                          uint32_t *__restrict__ sums) {
+    __shared__ uint32_t wsum[32];
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    const int64_t lo = (int64_t)blockIdx.x * chunk, hi = min(n, lo + chunk);
+    uint32_t t = 0;
+    for (int64_t i = lo + threadIdx.x; i < hi; i += blockDim.x) t += a[i];
+    for (int o = 16; o; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    if (lane == 0) wsum[wid] = t;
+    __syncthreads();
+    if (wid == 0) {
+        t = wsum[lane];
+        for (int o = 16; o; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+        if (lane == 0) sums[blockIdx.x] = t;
+    }
+}
+
+// Exclusive scan of the n radix counts: one block while n is small, else the chunks'
+// totals, a one-block scan of them and a scan of every chunk from its offset
+// (sums: scratch of at least 1024 uint32 values).
+static void scan_counts(uint32_t *a, int64_t n, uint32_t *sums, cudaStream_t stream) {
+    constexpr int64_t kOneBlock = 1 << 16;
+    if (n <= kOneBlock) {
+        note_launch();
+        k_scan_u32<<<1, 1024, 0, stream>>>(a, n, n, nullptr);
+        return;
+    }
+    const int64_t nchunks = std::min<int64_t>(1024, cdiv(n, 16384));
+    const int64_t chunk = cdiv(cdiv(n, nchunks), 4096) * 4096;
+    const int64_t nc = cdiv(n, chunk);
+    note_launch();
+    k_scan_chunk_sums<<<(unsigned)nc, 1024, 0, stream>>>(a, n, chunk, sums);
+    note_launch();
+    k_scan_u32<<<1, 1024, 0, stream>>>(sums, nc, nc, nullptr);
+    note_launch();
+    k_scan_u32<<<(unsigned)nc, 1024, 0, stream>>>(a, n, chunk, sums);
 }
 
 // Stable scatter of one radix pass.  Positions inside a tile are visited in
@@ -132,7 +176,6 @@ __global__ void __launch_bounds__(256) k_radix_scatter(const uint32_t *__restric
 // of unique-value heads and the double-double sums of x and x^2.
 struct DDPart { double s_hi, s_lo, q_hi, q_lo; int64_t heads; int64_t pad; };
 
-__device__ __forceinline__ bool is_head(const uint32_t *keys, int64_t i) { return i == 0 || keys[i] != keys[i - 1]; }
 
 template <typename T>
 __device__ __forceinline__ T shfl_up(T v, int o) { return __shfl_up_sync(0xffffffffu, v, o); }
@@ -166,19 +209,68 @@ __device__ ScanVal block_scan_incl(ScanVal v, ScanVal *wtot, ScanVal &total) {
     return v;
 }
 
-__global__ void __launch_bounds__(256) k_hist_partials(const uint32_t *__restrict__ keys, int64_t d, DDPart *part) {
-    __shared__ ScanVal wtot[8];
-    int64_t base = (int64_t)blockIdx.x * kScanTile + threadIdx.x * 4;
+// The thread's kHistPer consecutive sorted keys starting at base (positions >= d are
+// left out): x as binary64, the sums of x and x^2 in double-double (x^2 of a binary32
+// value is exact in binary64) and the number of heads.  One fixed order per thread, so
+// the single-row and the batched paths, which both call it, give the same bits.
+__device__ __forceinline__ ScanVal hist_thread_sums(const uint32_t *keys, int64_t d, int64_t base) {
     ScanVal v{{0.0, 0.0}, {0.0, 0.0}, 0};
-    for (int e = 0; e < 4; e++) {
-        int64_t i = base + e;
+    uint32_t prev = base > 0 && base - 1 < d ? keys[base - 1] : 0u;
+#pragma unroll 4
+    for (int e = 0; e < kHistPer; e++) {
+        const int64_t i = base + e;
         if (i < d) {
-            double x = (double)key2f(keys[i]);
-            v.s = dd_add(v.s, dd{x, 0.0});
-            v.q = dd_add(v.q, dd{__dmul_rn(x, x), 0.0});
-            v.h += is_head(keys, i);
+            const uint32_t k = keys[i];
+            const double x = (double)key2f(k);
+            v.s = dd_add_d(v.s, x);
+            v.q = dd_add_d(v.q, __dmul_rn(x, x));
+            v.h += (i == 0 || k != prev) ? 1 : 0;
+            prev = k;
         }
     }
+    return v;
+}
+
+// Pass C for the thread's keys: from the exclusive prefix `run` before them, every head
+// i writes its unique index u = run.h, v[u], N[u] = i, S[u] and S2[u] (hi at [u], lo at
+// [lo_off + u]); the last position d - 1 also writes the totals at index p and returns
+// p and ||X||^2 through p_out and norm2_out.
+__device__ __forceinline__ void hist_thread_fill(const uint32_t *keys, int64_t d, int64_t base, ScanVal run,
+                                                 float *v, int64_t *N, double *S, double *S2, int64_t lo_off,
+                                                 int64_t *p_out, double *norm2_out) {
+    uint32_t prev = base > 0 && base - 1 < d ? keys[base - 1] : 0u;
+#pragma unroll 4
+    for (int e = 0; e < kHistPer; e++) {
+        const int64_t i = base + e;
+        if (i >= d) break;
+        const uint32_t k = keys[i];
+        const double x = (double)key2f(k);
+        const bool head = i == 0 || k != prev;
+        prev = k;
+        if (head) {
+            const int64_t u = run.h;
+            v[u] = (float)x;
+            N[u] = i;
+            S[u] = run.s.hi; S[lo_off + u] = run.s.lo;
+            S2[u] = run.q.hi; S2[lo_off + u] = run.q.lo;
+        }
+        run.s = dd_add_d(run.s, x);
+        run.q = dd_add_d(run.q, __dmul_rn(x, x));
+        run.h += head ? 1 : 0;
+        if (i == d - 1) {
+            const int64_t p = run.h;
+            N[p] = d;
+            S[p] = run.s.hi; S[lo_off + p] = run.s.lo;
+            S2[p] = run.q.hi; S2[lo_off + p] = run.q.lo;
+            *p_out = p;
+            *norm2_out = run.q.hi;
+        }
+    }
+}
+
+__global__ void __launch_bounds__(256) k_hist_partials(const uint32_t *__restrict__ keys, int64_t d, DDPart *part) {
+    __shared__ ScanVal wtot[8];
+    const ScanVal v = hist_thread_sums(keys, d, (int64_t)blockIdx.x * kHistTile + (int64_t)threadIdx.x * kHistPer);
     ScanVal tot;
     block_scan_incl(v, wtot, tot);
     if (threadIdx.x == 0) part[blockIdx.x] = {tot.s.hi, tot.s.lo, tot.q.hi, tot.q.lo, tot.h, 0};
@@ -216,50 +308,16 @@ __global__ void __launch_bounds__(256) k_hist_fill(const uint32_t *__restrict__ 
                                                    float *v, int64_t *N, double *S, double *S2, DevStatus *st,
                                                    int64_t pcap) {
     __shared__ ScanVal wtot[8];
-    int64_t base = (int64_t)blockIdx.x * kScanTile + threadIdx.x * 4;
-    ScanVal loc{{0.0, 0.0}, {0.0, 0.0}, 0};
-    double xs[4];
-    int hd[4];
-    for (int e = 0; e < 4; e++) {
-        int64_t i = base + e;
-        xs[e] = 0.0; hd[e] = 0;
-        if (i < d) {
-            xs[e] = (double)key2f(keys[i]);
-            hd[e] = is_head(keys, i);
-            loc.s = dd_add(loc.s, dd{xs[e], 0.0});
-            loc.q = dd_add(loc.q, dd{__dmul_rn(xs[e], xs[e]), 0.0});
-            loc.h += hd[e];
-        }
-    }
+    const int64_t base = (int64_t)blockIdx.x * kHistTile + (int64_t)threadIdx.x * kHistPer;
+    const ScanVal loc = hist_thread_sums(keys, d, base);
     ScanVal tot;
-    ScanVal incl = block_scan_incl(loc, wtot, tot);
+    const ScanVal incl = block_scan_incl(loc, wtot, tot);
     const DDPart &pb = part[blockIdx.x];
-    ScanVal off{{pb.s_hi, pb.s_lo}, {pb.q_hi, pb.q_lo}, pb.heads};
+    const ScanVal off{{pb.s_hi, pb.s_lo}, {pb.q_hi, pb.q_lo}, pb.heads};
     // exclusive prefix before this thread's first element
     ScanVal run{dd_sub(incl.s, loc.s), dd_sub(incl.q, loc.q), incl.h - loc.h};
     run = sv_add(off, run);
-    for (int e = 0; e < 4; e++) {
-        int64_t i = base + e;
-        if (i >= d) break;
-        if (hd[e]) {
-            int64_t u = run.h;
-            v[u] = (float)xs[e];
-            N[u] = i;
-            S[u] = run.s.hi; S[pcap + 1 + u] = run.s.lo;
-            S2[u] = run.q.hi; S2[pcap + 1 + u] = run.q.lo;
-        }
-        run.s = dd_add(run.s, dd{xs[e], 0.0});
-        run.q = dd_add(run.q, dd{__dmul_rn(xs[e], xs[e]), 0.0});
-        run.h += hd[e];
-        if (i == d - 1) {
-            int64_t p = run.h;
-            N[p] = d;
-            S[p] = run.s.hi; S[pcap + 1 + p] = run.s.lo;
-            S2[p] = run.q.hi; S2[pcap + 1 + p] = run.q.lo;
-            st->p = p;
-            st->norm2 = run.q.hi;
-        }
-    }
+    hist_thread_fill(keys, d, base, run, v, N, S, S2, pcap + 1, &st->p, &st->norm2);
 }
 
 // The arrays were written with lo parts at offset pcap+1 (pcap = d); repack
@@ -322,48 +380,15 @@ __global__ void __launch_bounds__(256) k_rows_prepare(const float *__restrict__ 
     int64_t *N = R.N + row * (dcap + 1), *w = R.w + row * dcap;
     double *S = R.S + row * 2 * (dcap + 1), *S2 = R.S2 + row * 2 * (dcap + 1);
     // k_hist_fill, one tile
-    const int base = threadIdx.x * 4;
-    ScanVal loc{{0.0, 0.0}, {0.0, 0.0}, 0};
-    double xs[4];
-    int hd[4];
-    for (int e = 0; e < 4; e++) {
-        int i = base + e;
-        xs[e] = 0.0; hd[e] = 0;
-        if (i < d) {
-            xs[e] = (double)key2f(keys[i]);
-            hd[e] = (i == 0 || keys[i] != keys[i - 1]);
-            loc.s = dd_add(loc.s, dd{xs[e], 0.0});
-            loc.q = dd_add(loc.q, dd{__dmul_rn(xs[e], xs[e]), 0.0});
-            loc.h += hd[e];
-        }
-    }
+    const int64_t base = (int64_t)threadIdx.x * kHistPer;
+    const ScanVal loc = hist_thread_sums(keys, d, base);
     ScanVal tot;
-    ScanVal incl = block_scan_incl(loc, wtot, tot);
+    const ScanVal incl = block_scan_incl(loc, wtot, tot);
     const int64_t p = tot.h;
-    ScanVal off{{0.0, 0.0}, {0.0, 0.0}, 0};
+    const ScanVal off{{0.0, 0.0}, {0.0, 0.0}, 0};
     ScanVal run{dd_sub(incl.s, loc.s), dd_sub(incl.q, loc.q), incl.h - loc.h};
     run = sv_add(off, run);
-    for (int e = 0; e < 4; e++) {
-        int i = base + e;
-        if (i >= d) break;
-        if (hd[e]) {
-            int64_t u = run.h;
-            v[u] = (float)xs[e];
-            N[u] = i;
-            S[u] = run.s.hi; S[p + 1 + u] = run.s.lo;
-            S2[u] = run.q.hi; S2[p + 1 + u] = run.q.lo;
-        }
-        run.s = dd_add(run.s, dd{xs[e], 0.0});
-        run.q = dd_add(run.q, dd{__dmul_rn(xs[e], xs[e]), 0.0});
-        run.h += hd[e];
-        if (i == d - 1) {
-            N[p] = d;
-            S[p] = run.s.hi; S[p + 1 + p] = run.s.lo;
-            S2[p] = run.q.hi; S2[p + 1 + p] = run.q.lo;
-            R.p[row] = p;
-            R.norm2[row] = run.q.hi;
-        }
-    }
+    hist_thread_fill(keys, d, base, run, v, N, S, S2, p + 1, R.p + row, R.norm2 + row);
     __syncthreads();
     for (int u = threadIdx.x; u < p; u += blockDim.x) w[u] = N[u + 1] - N[u];
     if (threadIdx.x == 0) R.nonfinite[row] = nonfin;
@@ -449,15 +474,14 @@ int prepare_device(const float *x, int64_t d, void *ws, const Layout &L, cudaStr
     for (int shift = 0; shift < 32; shift += 8) {
         note_launch();
         k_radix_count<<<nb, 256, 0, stream>>>(a, d, shift, cnt, nb);
-        note_launch();
-        k_scan_u32<<<1, 1024, 0, stream>>>(cnt, (int64_t)256 * nb);
+        scan_counts(cnt, (int64_t)256 * nb, wsp<uint32_t>(ws, L.v), stream);  // v is free until the histogram
         note_launch();
         k_radix_scatter<<<nb, 256, 0, stream>>>(a, b, d, shift, cnt, nb);
         ECASQ_LAUNCH_CHECK();
         uint32_t *t = a; a = b; b = t;
     }
     // a == k0 holds the sorted keys
-    int64_t nbs = cdiv(d, kScanTile);
+    int64_t nbs = cdiv(d, kHistTile);  // the layout holds cdiv(d, kScanTile) >= nbs partials
     DDPart *part = wsp<DDPart>(ws, L.part);
     // scratch copies of N/S/S2 with lo parts at offset d+1 live in keys1 / dp area
     double *Stmp = wsp<double>(ws, L.dp64);
