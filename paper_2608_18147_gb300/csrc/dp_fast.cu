@@ -449,47 +449,77 @@ __device__ __forceinline__ void tile_consts(const FastArgs &a, int64_t k0, int j
     kd[jl] = (k + 1 < a.p) ? __fsub_rn(a.v[k + 1], a.v[k]) : 0.f;
 }
 
+// Global inputs of column jl of tile (K, J), loaded by one of the 64 threads: the tile
+// constants of k = 64K + jl (v_k, w_{k+1}, v_{k+1} - v_k), the column's increment
+// (w_{jt+1}, v_{jt+1}, v_jt, jt = 64J + jl) and v_j, and off the diagonal the corner
+// state of (K, J).
+struct TileIn {
+    float kv, kw, kd;
+    float wn, vn, vt, vj;
+    float c[7];
+};
+__device__ __forceinline__ void tile_load_consts(const FastArgs &a, int64_t K, int jl, TileIn &q) {
+    const int64_t k = K * BK + jl;
+    q.kv = k < a.p ? a.v[k] : 0.f;
+    q.kw = (k + 1 < a.p) ? a.wf[k + 1] : 0.f;
+    q.kd = (k + 1 < a.p) ? __fsub_rn(a.v[k + 1], a.v[k]) : 0.f;
+}
+__device__ __forceinline__ void tile_load(const FastArgs &a, int64_t K, int64_t J, int jl, TileIn &q) {
+    const int64_t jt = J * BJ + jl;
+    const bool okc = jt + 1 < a.p;
+    q.wn = okc ? a.wf[jt + 1] : 0.f;
+    q.vn = okc ? a.v[jt + 1] : 0.f;
+    q.vt = okc ? a.v[jt] : 0.f;
+    q.vj = jt < a.p ? a.v[jt] : 0.f;
+#pragma unroll
+    for (int r = 0; r < 7; r++) q.c[r] = 0.f;
+    if (K != J) {
+        const float *cp = a.corner + 8 * corner_idx(K, J);
+#pragma unroll
+        for (int r = 0; r < 7; r++) q.c[r] = cp[r];
+    }
+}
+
+// Anchor of column jl at k = 64K + 63 (off the diagonal): the corner state of (K, J)
+// advanced along j with compensated exclusive scans of non-negative increments.
+// Threads 0..63 of the block all call it (the scans synchronise them on BAR_PROD);
+// vk = v at k = 64K + 63.
+__device__ Rec tile_anchor(const TileIn &q, int64_t J, int jl, float vk, const FastArgs &a, float (*wsum)[2]) {
+    const bool okc = J * BJ + jl + 1 < a.p;
+    const float wn = q.wn, vn = q.vn;
+    const float dj = okc ? __fsub_rn(vn, q.vt) : 0.f;
+    const float *cp = q.c;
+    float nx, nc, ax, ac, ex, ec, cx, cc;
+    scan64_excl(wn, nx, nc, wsum);                               // N (exact)
+    scan64_excl(okc ? __fmul_rn(wn, __fsub_rn(vn, vk)) : 0.f, ax, ac, wsum);  // A
+    float Nj = __fadd_rn(cp[0], __fadd_rn(nx, nc));
+    float Aj = __fadd_rn(__fadd_rn(cp[3], ax), __fadd_rn(cp[4], ac));
+    scan64_excl(__fmul_rn(dj, Nj), ex, ec, wsum);              // E
+    scan64_excl(__fmul_rn(dj, Aj), cx, cc, wsum);              // C
+    Rec anchor_r;
+    anchor_r.N = Nj;
+    anchor_r.E = cp[1]; anchor_r.Ec = cp[2];
+    pair_add(anchor_r.E, anchor_r.Ec, ex, ec);
+    anchor_r.A = cp[3]; anchor_r.Ac = cp[4];
+    pair_add(anchor_r.A, anchor_r.Ac, ax, ac);
+    anchor_r.C = cp[5]; anchor_r.Cc = cp[6];
+    pair_add(anchor_r.C, anchor_r.Cc, cx, cc);
+    return anchor_r;
+}
+
 // Interval costs C[k, j] and Phi[k, j] of column j = 64J + jl for the 64 k of tile K
 // (k descending) into Cr[jl][.] and Pr[jl][.]; +inf / 0 where k >= j or j >= p.
-// Threads 0..63 of the block all call it (the anchors' scans synchronise them on
-// BAR_PROD); kv, kw, kd hold tile_consts of tile K, visible to all 64.
-__device__ void tile_columns(const FastArgs &a, int64_t K, int64_t J, int jl, const float *kv, const float *kw,
-                             const float *kd, float (*wsum)[2], float (*Cr)[PSTR], float (*Pr)[PSTR]) {
+// anchor_r: the column's state at k = 64K + 63 (off the diagonal); vj = v_j.
+__device__ void tile_rows(const FastArgs &a, int64_t K, int64_t J, int jl, const Rec &anchor_r, float vj,
+                          const float *kv, const float *kw, const float *kd, float (*Cr)[PSTR], float (*Pr)[PSTR]) {
     const bool diag = (K == J);
     const int64_t j0 = J * BJ;
     const int64_t j = j0 + jl;
     const float d_f = (float)a.d;
-        // anchors of the 64 columns at k = 64K + 63: the corner state of (K, J) advanced
-        // along j with compensated exclusive scans of non-negative increments
-        Rec anchor_r = rec_empty();
-        if (!diag) {
-            const float *cp = a.corner + 8 * corner_idx(K, J);
-            float vk = kv[BK - 1];
-            int64_t jt = j0 + jl;  // increment of column jl: moving j from jt to jt + 1
-            bool okc = jt + 1 < a.p;
-            float wn = okc ? a.wf[jt + 1] : 0.f;
-            float vn = okc ? a.v[jt + 1] : 0.f;
-            float dj = okc ? __fsub_rn(vn, a.v[jt]) : 0.f;
-            float nx, nc, ax, ac, ex, ec, cx, cc;
-            scan64_excl(wn, nx, nc, wsum);                               // N (exact)
-            scan64_excl(okc ? __fmul_rn(wn, __fsub_rn(vn, vk)) : 0.f, ax, ac, wsum);  // A
-            float Nj = __fadd_rn(cp[0], __fadd_rn(nx, nc));
-            float Aj = __fadd_rn(__fadd_rn(cp[3], ax), __fadd_rn(cp[4], ac));
-            scan64_excl(__fmul_rn(dj, Nj), ex, ec, wsum);              // E
-            scan64_excl(__fmul_rn(dj, Aj), cx, cc, wsum);              // C
-            anchor_r.N = Nj;
-            anchor_r.E = cp[1]; anchor_r.Ec = cp[2];
-            pair_add(anchor_r.E, anchor_r.Ec, ex, ec);
-            anchor_r.A = cp[3]; anchor_r.Ac = cp[4];
-            pair_add(anchor_r.A, anchor_r.Ac, ax, ac);
-            anchor_r.C = cp[5]; anchor_r.Cc = cp[6];
-            pair_add(anchor_r.C, anchor_r.Cc, cx, cc);
-        }
         // interval costs of column j for k in the tile (descending k); the row's
         // padding slot BK receives min_k C and min_k Phi (lower bounds for tile skipping)
         float mc = CUDART_INF_F, mp = CUDART_INF_F;
         if (j < a.p) {
-            float vj = a.v[j];
             Rec r;
             int kl_hi;
             if (diag) {
@@ -525,9 +555,22 @@ __device__ void tile_columns(const FastArgs &a, int64_t K, int64_t J, int jl, co
         Pr[jl][BK] = mp;
 }
 
+// tile_anchor and tile_rows for one tile (threads 0..63 of the block; kv, kw, kd hold
+// the tile constants of tile K, visible to all 64).
+__device__ void tile_columns(const FastArgs &a, int64_t K, int64_t J, int jl, const float *kv, const float *kw,
+                             const float *kd, float (*wsum)[2], float (*Cr)[PSTR], float (*Pr)[PSTR]) {
+    TileIn q;
+    tile_load(a, K, J, jl, q);
+    const Rec anchor_r = K == J ? rec_empty() : tile_anchor(q, J, jl, kv[BK - 1], a, wsum);
+    tile_rows(a, K, J, jl, anchor_r, q.vj, kv, kw, kd, Cr, Pr);
+}
+
 // Resident interval costs: every tile (K <= J) computed once, exactly as the
-// wavefront's own producer computes it, staged in shared memory and written out
-// by a bulk copy.  64 threads per block; blocks stride over the tiles.
+// wavefront's own producer computes it (tile_anchor, tile_rows), staged in shared
+// memory and written out by a bulk copy.  64 threads per block; blocks stride over
+// the tiles.  A tile's global inputs are loaded while the previous tile's rows are
+// computed, and the wait for the previous bulk store to have read the staging rows
+// comes only just before they are overwritten.
 struct __align__(16) BuildSmem {
     float C[BJ][PSTR];
     float Phi[BJ][PSTR];
@@ -539,15 +582,32 @@ __global__ void __launch_bounds__(NPROD) k_build_costs(FastArgs a, float *costs)
     __shared__ BuildSmem S;
     const int jl = threadIdx.x;
     const int64_t ntiles = (int64_t)a.nJ * (a.nJ + 1) / 2;
-    for (int64_t t = blockIdx.x; t < ntiles; t += gridDim.x) {
-        // invert t = J(J+1)/2 + K, K <= J
-        int64_t J = (int64_t)((sqrt(8.0 * (double)t + 1.0) - 1.0) * 0.5);
-        while (J * (J + 1) / 2 > t) J--;
-        while ((J + 1) * (J + 2) / 2 <= t) J++;
-        int64_t K = t - J * (J + 1) / 2;
-        tile_consts(a, K * BK, jl, S.kv, S.kw, S.kd);
+    int64_t t = blockIdx.x;
+    if (t >= ntiles) return;
+    // invert t = J(J+1)/2 + K, K <= J
+    int64_t J = (int64_t)((sqrt(8.0 * (double)t + 1.0) - 1.0) * 0.5);
+    while (J * (J + 1) / 2 > t) J--;
+    while ((J + 1) * (J + 2) / 2 <= t) J++;
+    int64_t K = t - J * (J + 1) / 2;
+    TileIn cur;
+    tile_load_consts(a, K, jl, cur);
+    tile_load(a, K, J, jl, cur);
+    for (;;) {
+        S.kv[jl] = cur.kv; S.kw[jl] = cur.kw; S.kd[jl] = cur.kd;
         bar_sync(BAR_PROD, NPROD);
-        tile_columns(a, K, J, jl, S.kv, S.kw, S.kd, S.wsum, S.C, S.Phi);
+        const Rec anchor_r = K == J ? rec_empty() : tile_anchor(cur, J, jl, S.kv[BK - 1], a, S.wsum);
+        // the next tile of this block: t + gridDim.x, walking (J, K) along the rows
+        const int64_t tn = t + gridDim.x;
+        int64_t Jn = J, Kn = K + gridDim.x;
+        while (Kn > Jn) { Kn -= Jn + 1; Jn++; }
+        TileIn nxt;
+        if (tn < ntiles) {
+            tile_load_consts(a, Kn, jl, nxt);
+            tile_load(a, Kn, Jn, jl, nxt);
+        }
+        if (jl == 0) bulk_wait_read_all();  // the previous tile's bulk store has read the rows
+        bar_sync(BAR_PROD, NPROD);
+        tile_rows(a, K, J, jl, anchor_r, cur.vj, S.kv, S.kw, S.kd, S.C, S.Phi);
         a.tsum[(size_t)t * BJ + jl] = make_float2(S.C[jl][BK], S.Phi[jl][BK]);  // this thread's own row
         fence_proxy_async_smem();
         bar_sync(BAR_PROD, NPROD);
@@ -556,9 +616,10 @@ __global__ void __launch_bounds__(NPROD) k_build_costs(FastArgs a, float *costs)
             bulk_s2g(dst, &S.C[0][0], kCostHalfBytes);
             bulk_s2g(dst + kCostHalfFloats, &S.Phi[0][0], kCostHalfBytes);
             bulk_commit();
-            bulk_wait_read_all();  // shared buffers free again
         }
-        bar_sync(BAR_PROD, NPROD);
+        if (tn >= ntiles) break;
+        t = tn; J = Jn; K = Kn;
+        cur = nxt;
     }
     if (jl == 0) bulk_wait_all();
 }
