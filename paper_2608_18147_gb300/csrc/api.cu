@@ -31,8 +31,9 @@ int launch_eval_codebook(const Prefix &P, const int32_t *a, int m, double *out3,
 int launch_gather_q(const float *v, const int32_t *qidx, const int32_t *mcount, int G, int s, float *Q,
                     cudaStream_t st);
 int launch_locate_q(const float *v, int64_t p, const float *Q, int m, int32_t *a, DevStatus *ds, cudaStream_t st);
+size_t refine_ctx_bytes();
 int launch_refine_colour(const Prefix &P, const int32_t *a, int m, int colour, double lamp, int32_t *a_new,
-                         int32_t *moved, void *part_buf, cudaStream_t st, int *nblocks_out);
+                         int32_t *moved, void *part_buf, int32_t *ctx, cudaStream_t st, int *nblocks_out);
 size_t refine_scratch_bytes(int64_t d);
 int launch_quantize(const float *x, int64_t d, const float *Q, int m, uint64_t seed, uint8_t *idx, uint32_t *counts,
                     DevStatus *st, int num_sms, cudaStream_t stream);
@@ -101,7 +102,7 @@ size_t make_layout(int64_t d, int32_t s, int64_t rows, Layout *L) {
     L->mcount = take(4 * (size_t)kMaxG);
     L->metrics = take(8 * (size_t)kMaxG * 4);
     L->lam = take(8 * (size_t)kMaxG);
-    L->refine = take(4 * 2 * kMaxS + 256 + 8 * 8);
+    L->refine = take(4 * 2 * kMaxS + 256 + 8 * 8 + refine_ctx_bytes());
     L->refine_part = take(refine_scratch_bytes(d));
     L->band = take(fast_dp_band_bytes(d, s));
     L->costs = 0;
@@ -343,6 +344,9 @@ static int refine_device(void *ws, const Layout &L, const Prefix &P, std::vector
     int32_t *a = wsp<int32_t>(ws, L.refine);
     int32_t *an = a + kMaxS;
     int32_t *moved = an + kMaxS;
+    // records of scans that kept their value (refine.cu), after the evaluation output
+    int32_t *ctx = reinterpret_cast<int32_t *>(wsp<char>(ws, L.refine) + 4 * 2 * kMaxS + 256 + 8 * 8);
+    ECASQ_CUDA_TRY(cudaMemsetAsync(ctx, 0, refine_ctx_bytes(), st));
     ECASQ_CUDA_TRY(cudaMemcpyAsync(a, a_host.data(), sizeof(int32_t) * m, cudaMemcpyHostToDevice, st));
     double ev[3];
     int rc = eval_device(ws, L, P, a, m, st, ev);
@@ -354,7 +358,7 @@ static int refine_device(void *ws, const Layout &L, const Prefix &P, std::vector
             ECASQ_CUDA_TRY(cudaMemcpyAsync(an, a, sizeof(int32_t) * m, cudaMemcpyDeviceToDevice, st));
             ECASQ_CUDA_TRY(cudaMemsetAsync(moved, 0, sizeof(int32_t), st));
             int nblk = 0;
-            rc = launch_refine_colour(P, a, m, col, lamp, an, moved, wsp<void>(ws, L.refine_part), st, &nblk);
+            rc = launch_refine_colour(P, a, m, col, lamp, an, moved, wsp<void>(ws, L.refine_part), ctx, st, &nblk);
             if (rc != ECASQ_OK) return rc;
             if (nblk == 0) continue;
             int32_t mv = 0;

@@ -9,9 +9,32 @@
 // f_{l+1} = U[c, q_{l+1}] + D[q_{l+1}, q_{l+2}]   (U[c, q_{m-1}] when l+1 = m-1).
 // Values of one class never share a frequency term, so all of them move at
 // once (Sec. 6, Fig. 3).  Ties keep the current value, else the lowest index.
+//
+// The scan of q_l is a function of (q_{l-2}, q_{l-1}, q_l, q_{l+1}, q_{l+2}) alone (and of
+// lambda', fixed in a call).  ctx[l] records that context whenever a scan kept q_l
+// where it was; while the context is unchanged the scan would keep it again, so the
+// value is not scanned (same result, no candidate evaluated).  A value that moved has
+// no record (its move may still be undone by the caller).
 #include "common.cuh"
 
 namespace ecasq {
+
+constexpr int kCtx = 6;  // q_{l-2}, q_{l-1}, q_l, q_{l+1}, q_{l+2} (-1 past the ends), valid
+
+__device__ __forceinline__ void context_of(const int32_t *a, int m, int l, int32_t c[5]) {
+    c[0] = l >= 2 ? a[l - 2] : -1;
+    c[1] = a[l - 1];
+    c[2] = a[l];
+    c[3] = a[l + 1];
+    c[4] = l + 2 <= m - 1 ? a[l + 2] : -1;
+}
+__device__ __forceinline__ bool context_unchanged(const int32_t *a, int m, int l, const int32_t *ctx) {
+    const int32_t *r = ctx + kCtx * l;
+    if (!r[5]) return false;
+    int32_t c[5];
+    context_of(a, m, l, c);
+    return c[0] == r[0] && c[1] == r[1] && c[2] == r[2] && c[3] == r[3] && c[4] == r[4];
+}
 
 struct Nbr {
     int64_t L, R, cur, a0;
@@ -50,7 +73,7 @@ __device__ __forceinline__ Nbr make_nbr(const Prefix &P, const int32_t *a, int m
 struct RefPart { double v; int64_t i; };
 
 __global__ void __launch_bounds__(256) k_refine_chunks(Prefix P, const int32_t *a, int m, int colour, double lamp,
-                                                       RefPart *part, int nchunk) {
+                                                       RefPart *part, int nchunk, const int32_t *ctx) {
     __shared__ Nbr nb;
     __shared__ double rv[256];
     __shared__ int64_t ri[256];
@@ -59,6 +82,7 @@ __global__ void __launch_bounds__(256) k_refine_chunks(Prefix P, const int32_t *
     if (l > m - 2) return;
     int64_t lo = (int64_t)a[l - 1] + 1 + (int64_t)blockIdx.x * kRefineChunk;
     int64_t hi = min((int64_t)a[l + 1], lo + kRefineChunk);
+    if (lo >= hi || context_unchanged(a, m, l, ctx)) return;  // uniform over the block
     if (threadIdx.x == 0) nb = make_nbr(P, a, m, l);
     __syncthreads();
     Nbr n = nb;
@@ -87,10 +111,11 @@ __global__ void __launch_bounds__(256) k_refine_chunks(Prefix P, const int32_t *
 // One warp per moved value: best over the chunks (lowest index among equal
 // values), then keep the current position unless the best is strictly lower.
 __global__ void k_refine_pick(Prefix P, const int32_t *a, int m, int colour, double lamp, const RefPart *part,
-                              int nchunk, int32_t *a_new, int32_t *moved) {
+                              int nchunk, int32_t *a_new, int32_t *moved, int32_t *ctx) {
     int l0 = colour == 0 ? 3 : colour;
     int l = l0 + 3 * blockIdx.x;
     if (l > m - 2) return;
+    if (context_unchanged(a, m, l, ctx)) return;  // a_new[l] == a[l] already
     int64_t range = (int64_t)a[l + 1] - (int64_t)a[l - 1] - 1;
     int nc = (int)cdiv(range, kRefineChunk);
     double bv = CUDART_INF;
@@ -110,6 +135,15 @@ __global__ void k_refine_pick(Prefix P, const int32_t *a, int m, int colour, dou
         int64_t nw = (bi >= 0 && bv < vc) ? bi : n.cur;
         a_new[l] = (int32_t)nw;
         if (nw != n.cur) atomicExch(moved, 1);
+        int32_t *r = ctx + kCtx * l;
+        if (nw == n.cur) {
+            int32_t c[5];
+            context_of(a, m, l, c);
+            for (int q = 0; q < 5; q++) r[q] = c[q];
+            r[5] = 1;
+        } else {
+            r[5] = 0;
+        }
     }
 }
 
@@ -117,8 +151,10 @@ size_t refine_scratch_bytes(int64_t d) {
     return sizeof(RefPart) * (size_t)(kMaxS / 3 + 1) * (size_t)cdiv(d, kRefineChunk);
 }
 
+size_t refine_ctx_bytes() { return sizeof(int32_t) * kCtx * kMaxS; }
+
 int launch_refine_colour(const Prefix &P, const int32_t *a, int m, int colour, double lamp, int32_t *a_new,
-                         int32_t *moved, void *part_buf, cudaStream_t st, int *nblocks_out) {
+                         int32_t *moved, void *part_buf, int32_t *ctx, cudaStream_t st, int *nblocks_out) {
     int l0 = colour == 0 ? 3 : colour;
     int nblk = (m - 2 >= l0) ? (m - 2 - l0) / 3 + 1 : 0;
     *nblocks_out = nblk;
@@ -126,10 +162,10 @@ int launch_refine_colour(const Prefix &P, const int32_t *a, int m, int colour, d
     int nchunk = (int)cdiv(P.p, kRefineChunk);
     RefPart *part = reinterpret_cast<RefPart *>(part_buf);
     note_launch();
-    k_refine_chunks<<<dim3(nchunk, nblk), 256, 0, st>>>(P, a, m, colour, lamp, part, nchunk);
+    k_refine_chunks<<<dim3(nchunk, nblk), 256, 0, st>>>(P, a, m, colour, lamp, part, nchunk, ctx);
     ECASQ_LAUNCH_CHECK();
     note_launch();
-    k_refine_pick<<<nblk, 32, 0, st>>>(P, a, m, colour, lamp, part, nchunk, a_new, moved);
+    k_refine_pick<<<nblk, 32, 0, st>>>(P, a, m, colour, lamp, part, nchunk, a_new, moved, ctx);
     ECASQ_LAUNCH_CHECK();
     return ECASQ_OK;
 }
