@@ -27,7 +27,8 @@ int launch_rows_gather(const RowsData &R, const int32_t *a, const int32_t *m, in
                        cudaStream_t st);
 int launch_traceback_eval(const Prefix &P, int G, int s, int exact_s, const double *dp64, const int32_t *bp,
                           int32_t *qidx, int32_t *mcount, double *metrics, cudaStream_t st);
-int launch_eval_codebook(const Prefix &P, const int32_t *a, int m, double *out3, cudaStream_t st);
+int launch_eval_codebook(const Prefix &P, const int32_t *a, int m, double *out3, cudaStream_t st,
+                         const int32_t *gate = nullptr);
 int launch_gather_q(const float *v, const int32_t *qidx, const int32_t *mcount, int G, int s, float *Q,
                     cudaStream_t st);
 int launch_locate_q(const float *v, int64_t p, const float *Q, int m, int32_t *a, DevStatus *ds, cudaStream_t st);
@@ -325,10 +326,11 @@ static int64_t candidates_of(int64_t p, int s, int exact) {
 }
 
 // Upload a codebook (unique indices) and evaluate it: out3 = MSE, H(I,B), H(Xhat).
+// With gate (device), the kernel evaluates only if *gate != 0 (else out3 is stale).
 static int eval_device(void *ws, const Layout &L, const Prefix &P, const int32_t *a_dev, int m, cudaStream_t st,
-                       double *out3_host) {
+                       double *out3_host, const int32_t *gate = nullptr) {
     double *o = reinterpret_cast<double *>(wsp<char>(ws, L.refine) + 4 * 2 * kMaxS + 256);
-    int rc = launch_eval_codebook(P, a_dev, m, o, st);
+    int rc = launch_eval_codebook(P, a_dev, m, o, st, gate);
     if (rc != ECASQ_OK) return rc;
     ECASQ_CUDA_TRY(cudaMemcpyAsync(out3_host, o, 3 * sizeof(double), cudaMemcpyDeviceToHost, st));
     ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
@@ -363,7 +365,7 @@ static int refine_device(void *ws, const Layout &L, const Prefix &P, std::vector
             if (nblk == 0) continue;
             int32_t mv = 0;
             ECASQ_CUDA_TRY(cudaMemcpyAsync(&mv, moved, sizeof(int32_t), cudaMemcpyDeviceToHost, st));
-            rc = eval_device(ws, L, P, an, m, st, ev);
+            rc = eval_device(ws, L, P, an, m, st, ev, moved);  // only a step that moved a value is evaluated
             if (rc != ECASQ_OK) return rc;
             if (!mv) continue;
             if (guard && ev[2] > budget) continue;

@@ -239,19 +239,31 @@ static __device__ __noinline__ void eval_codebook_warp(const Prefix &P, const in
         scratch[3 * kMaxS + r] = D;
     }
     __syncwarp();
+    if (m < 2) {
+        if (lane == 0) { out3[0] = 0.0; out3[1] = 0.0; out3[2] = 0.0; }
+        __syncwarp();
+        return;
+    }
+    // output-entropy terms in parallel: f_r = U_{r-1} + D_r (w of the first value + D_0 for
+    // r = 0), term r = h(f_r / d), and term m-1 = h(U_{m-2} / d); each lane overwrites the
+    // D slots it alone reads
+    const double dd_ = (double)P.d;
+    for (int r = lane; r < m; r += 32) {
+        double f;
+        if (r == m - 1) f = scratch[2 * kMaxS + m - 2];
+        else f = (r == 0) ? __dadd_rn((double)P.w[a[0]], scratch[3 * kMaxS]) : __dadd_rn(scratch[2 * kMaxS + r - 1], scratch[3 * kMaxS + r]);
+        scratch[3 * kMaxS + r] = hfun(__ddiv_rn(f, dd_));
+    }
+    __syncwarp();
     if (lane == 0) {
-        double dd_ = (double)P.d;
-        if (m < 2) { out3[0] = 0.0; out3[1] = 0.0; out3[2] = 0.0; return; }
-        double mse = 0.0, hs = 0.0, hx = 0.0, prevU = 0.0;
+        // the sums in interval order, as a sequential evaluation adds them
+        double mse = 0.0, hs = 0.0, hx = 0.0;
         for (int r = 0; r + 1 < m; r++) {
             mse = __dadd_rn(mse, scratch[r]);
             hs = __dadd_rn(hs, scratch[kMaxS + r]);
-            double D = scratch[3 * kMaxS + r];
-            double f = (r == 0) ? __dadd_rn((double)P.w[a[0]], D) : __dadd_rn(prevU, D);
-            hx = __dadd_rn(hx, hfun(__ddiv_rn(f, dd_)));
-            prevU = scratch[2 * kMaxS + r];
+            hx = __dadd_rn(hx, scratch[3 * kMaxS + r]);
         }
-        hx = __dadd_rn(hx, hfun(__ddiv_rn(prevU, dd_)));
+        hx = __dadd_rn(hx, scratch[3 * kMaxS + m - 1]);
         out3[0] = mse; out3[1] = hs; out3[2] = hx;
     }
     __syncwarp();

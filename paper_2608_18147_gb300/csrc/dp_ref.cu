@@ -125,10 +125,12 @@ __global__ void k_traceback_eval(Prefix P, int G, int s, int exact_s, const doub
     if (m > 0) eval_codebook_warp(P, a, m, &metrics[4 * g + 1], scratch);
 }
 
-// Metrics of a caller-given codebook (unique indices on the device).
-__global__ void k_eval_codebook(Prefix P, const int32_t *a_in, int m, double *out3) {
+// Metrics of a caller-given codebook (unique indices on the device); nothing when
+// gate is given and holds 0 (the caller then reads no result).
+__global__ void k_eval_codebook(Prefix P, const int32_t *a_in, int m, double *out3, const int32_t *gate) {
     __shared__ double scratch[4 * kMaxS];
     __shared__ int32_t a[kMaxS];
+    if (gate && *gate == 0) return;
     for (int r = threadIdx.x; r < m; r += 32) a[r] = a_in[r];
     __syncwarp();
     eval_codebook_warp(P, a, m, out3, scratch);
@@ -355,9 +357,10 @@ int launch_traceback_eval(const Prefix &P, int G, int s, int exact_s, const doub
     return ECASQ_OK;
 }
 
-int launch_eval_codebook(const Prefix &P, const int32_t *a, int m, double *out3, cudaStream_t st) {
+int launch_eval_codebook(const Prefix &P, const int32_t *a, int m, double *out3, cudaStream_t st,
+                         const int32_t *gate) {
     note_launch();
-    k_eval_codebook<<<1, 32, 0, st>>>(P, a, m, out3);
+    k_eval_codebook<<<1, 32, 0, st>>>(P, a, m, out3, gate);
     ECASQ_LAUNCH_CHECK();
     return ECASQ_OK;
 }

@@ -69,11 +69,14 @@ __device__ __forceinline__ Nbr make_nbr(const Prefix &P, const int32_t *a, int m
 
 // Block (chunk, b): the b-th value of the colour class, candidates
 // L+1+chunk*kRefineChunk .. (excluding the current position); the best
-// (value, lowest index) of the chunk goes to part[b * nchunk + chunk].
+// (value, lowest index) of the chunk goes to part[b * nchunk + chunk], and the
+// objective at the current position to curval[b].
 struct RefPart { double v; int64_t i; };
+constexpr int kRefineValues = kMaxS / 3 + 1;  // values of one colour class, at most
 
 __global__ void __launch_bounds__(256) k_refine_chunks(Prefix P, const int32_t *a, int m, int colour, double lamp,
-                                                       RefPart *part, int nchunk, const int32_t *ctx) {
+                                                       RefPart *part, double *curval, int nchunk,
+                                                       const int32_t *ctx) {
     __shared__ Nbr nb;
     __shared__ double rv[256];
     __shared__ int64_t ri[256];
@@ -89,8 +92,8 @@ __global__ void __launch_bounds__(256) k_refine_chunks(Prefix P, const int32_t *
     double bv = CUDART_INF;
     int64_t bi = -1;
     for (int64_t c = lo + threadIdx.x; c < hi; c += blockDim.x) {
-        if (c == n.cur) continue;
         double v = local_obj(P, n, c, lamp);
+        if (c == n.cur) { curval[blockIdx.y] = v; continue; }
         if (v < bv) { bv = v; bi = c; }  // c ascends per thread: keeps the lowest
     }
     rv[threadIdx.x] = bv; ri[threadIdx.x] = bi;
@@ -110,7 +113,7 @@ __global__ void __launch_bounds__(256) k_refine_chunks(Prefix P, const int32_t *
 
 // One warp per moved value: best over the chunks (lowest index among equal
 // values), then keep the current position unless the best is strictly lower.
-__global__ void k_refine_pick(Prefix P, const int32_t *a, int m, int colour, double lamp, const RefPart *part,
+__global__ void k_refine_pick(const int32_t *a, int m, int colour, const RefPart *part, const double *curval,
                               int nchunk, int32_t *a_new, int32_t *moved, int32_t *ctx) {
     int l0 = colour == 0 ? 3 : colour;
     int l = l0 + 3 * blockIdx.x;
@@ -130,13 +133,13 @@ __global__ void k_refine_pick(Prefix P, const int32_t *a, int m, int colour, dou
         if (i2 >= 0 && (bi < 0 || v2 < bv || (v2 == bv && i2 < bi))) { bv = v2; bi = i2; }
     }
     if (threadIdx.x == 0) {
-        Nbr n = make_nbr(P, a, m, l);
-        double vc = local_obj(P, n, n.cur, lamp);
-        int64_t nw = (bi >= 0 && bv < vc) ? bi : n.cur;
+        const int64_t cur = a[l];
+        const double vc = curval[blockIdx.x];  // local_obj at the current position (k_refine_chunks)
+        int64_t nw = (bi >= 0 && bv < vc) ? bi : cur;
         a_new[l] = (int32_t)nw;
-        if (nw != n.cur) atomicExch(moved, 1);
+        if (nw != cur) atomicExch(moved, 1);
         int32_t *r = ctx + kCtx * l;
-        if (nw == n.cur) {
+        if (nw == cur) {
             int32_t c[5];
             context_of(a, m, l, c);
             for (int q = 0; q < 5; q++) r[q] = c[q];
@@ -148,7 +151,7 @@ __global__ void k_refine_pick(Prefix P, const int32_t *a, int m, int colour, dou
 }
 
 size_t refine_scratch_bytes(int64_t d) {
-    return sizeof(RefPart) * (size_t)(kMaxS / 3 + 1) * (size_t)cdiv(d, kRefineChunk);
+    return sizeof(double) * kRefineValues + sizeof(RefPart) * kRefineValues * (size_t)cdiv(d, kRefineChunk);
 }
 
 size_t refine_ctx_bytes() { return sizeof(int32_t) * kCtx * kMaxS; }
@@ -160,12 +163,13 @@ int launch_refine_colour(const Prefix &P, const int32_t *a, int m, int colour, d
     *nblocks_out = nblk;
     if (nblk == 0) return ECASQ_OK;
     int nchunk = (int)cdiv(P.p, kRefineChunk);
-    RefPart *part = reinterpret_cast<RefPart *>(part_buf);
+    double *curval = reinterpret_cast<double *>(part_buf);  // then the chunks' partial results
+    RefPart *part = reinterpret_cast<RefPart *>(curval + kRefineValues);
     note_launch();
-    k_refine_chunks<<<dim3(nchunk, nblk), 256, 0, st>>>(P, a, m, colour, lamp, part, nchunk, ctx);
+    k_refine_chunks<<<dim3(nchunk, nblk), 256, 0, st>>>(P, a, m, colour, lamp, part, curval, nchunk, ctx);
     ECASQ_LAUNCH_CHECK();
     note_launch();
-    k_refine_pick<<<nblk, 32, 0, st>>>(P, a, m, colour, lamp, part, nchunk, a_new, moved, ctx);
+    k_refine_pick<<<nblk, 32, 0, st>>>(a, m, colour, part, curval, nchunk, a_new, moved, ctx);
     ECASQ_LAUNCH_CHECK();
     return ECASQ_OK;
 }
