@@ -1575,11 +1575,14 @@ __global__ void k_fill_unneeded(FastArgs a, double *dp64, int32_t *bp) {
 }
 
 // ----------------------------------------------------------- exact layer
-__device__ __forceinline__ void exact_candidate(const Prefix &P, const double *prev, int64_t k, int64_t j,
-                                                double lam, double &best, int32_t &arg) {
+__device__ __forceinline__ double exact_value(const Prefix &P, const double *prev, int64_t k, int64_t j, double lam) {
     double C, U, D;
     pair_exact(P, k, j, C, U, D);
-    double c = __dadd_rn(prev[k], __dadd_rn(C, __dmul_rn(lam, phi_exact(P, U, D, false))));
+    return __dadd_rn(prev[k], __dadd_rn(C, __dmul_rn(lam, phi_exact(P, U, D, false))));
+}
+__device__ __forceinline__ void exact_candidate(const Prefix &P, const double *prev, int64_t k, int64_t j,
+                                                double lam, double &best, int32_t &arg) {
+    const double c = exact_value(P, prev, k, j, lam);
     if (c < best || (c == best && k < arg)) { best = c; arg = (int32_t)k; }
 }
 
@@ -1609,29 +1612,72 @@ __device__ __forceinline__ void count_exact(const FastArgs &a, unsigned long lon
 
 // Layer i, outputs with at most NMEM members: one thread each, binary64 re-scoring
 // with double-double interval costs; the lowest k among exact minima wins.
-__global__ void k_exact_small(Prefix P, FastArgs a, int i, double *dp64, int32_t *bp) {
+__global__ void __launch_bounds__(128) k_exact_small(Prefix P, FastArgs a, int i, double *dp64, int32_t *bp) {
+    // A warp takes 32 listed outputs at a time and evaluates their members flattened
+    // (member r of the 32 outputs' lists goes to lane r mod 32), so every lane of a
+    // binary64 sequence does useful work; then each output's lane takes the least value,
+    // lowest k on ties, over its own members (the per-output rule, which is order-free).
+    __shared__ double sval[4][32 * NMEM];
+    __shared__ int32_t sk[4][32 * NMEM];
     const int n = a.list_cnt[2 * i];
     const int32_t *list = layer_list(a, i, 0);
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
     unsigned long long nres = 0;
     int nviol = 0;
-    const int stride = gridDim.x * blockDim.x;
-    for (int base = blockIdx.x * blockDim.x; base < n; base += stride) {  // warp-uniform trip count
-        const int e = base + threadIdx.x;
+    const int wstride = gridDim.x * (blockDim.x >> 5) * 32;
+    for (int base = (blockIdx.x * (blockDim.x >> 5) + wid) * 32; base < n; base += wstride) {  // warp-uniform
+        const int e = base + lane;
+        int g = 0, cnt = 0;
+        int64_t j = 0;
+        long long o = 0;
         if (e < n) {
             const int32_t v = list[e];
-            const int g = v >> 24;
-            const int64_t j = v & 0xFFFFFF;
-            const size_t o = oidx(a, g, i, j);
-            const int cnt = a.mcnt[o];
-            const double lam = a.prm->lam64[g];
-            const double *prev = dp64 + oidx(a, g, i - 1, 0);
-            const int32_t *mem = a.members + o * NMEM;
+            g = v >> 24;
+            j = v & 0xFFFFFF;
+            o = (long long)oidx(a, g, i, j);
+            cnt = a.mcnt[o];
+        }
+        int off = cnt;  // inclusive, then exclusive prefix of the member counts
+#pragma unroll
+        for (int d = 1; d < 32; d <<= 1) {
+            const int t = __shfl_up_sync(0xffffffffu, off, d);
+            if (lane >= d) off += t;
+        }
+        const int total = __shfl_sync(0xffffffffu, off, 31);
+        off -= cnt;
+        for (int rb = 0; rb < total; rb += 32) {  // warp-uniform
+            const int r = rb + lane;
+            int ow = 0;  // the last lane whose offset is <= r: the owner of member r
+#pragma unroll
+            for (int st = 16; st > 0; st >>= 1) {
+                const int oc = __shfl_sync(0xffffffffu, off, ow + st);
+                if (oc <= r) ow += st;
+            }
+            const int og = __shfl_sync(0xffffffffu, g, ow);
+            const int64_t oj = __shfl_sync(0xffffffffu, j, ow);
+            const long long oo = __shfl_sync(0xffffffffu, o, ow);
+            const int q = r - __shfl_sync(0xffffffffu, off, ow);
+            if (r < total) {
+                const int32_t k = a.members[(size_t)oo * NMEM + q];
+                sk[wid][r] = k;
+                sval[wid][r] = exact_value(P, dp64 + oidx(a, og, i - 1, 0), k, oj, a.prm->lam64[og]);
+            }
+        }
+        __syncwarp();
+        if (cnt > 0) {
             double best = CUDART_INF;
             int32_t arg = INT32_MAX;
-            for (int q = 0; q < cnt; q++) exact_candidate(P, prev, mem[q], j, lam, best, arg);
+            for (int q = 0; q < cnt; q++) {
+                const double c = sval[wid][off + q];
+                const int32_t k = sk[wid][off + q];
+                if (c < best || (c == best && k < arg)) { best = c; arg = k; }
+            }
             nres += cnt;
             nviol += exact_store(a, g, i, j, best, arg, dp64, bp) ? 0 : 1;
+        } else if (e < n) {
+            nviol += exact_store(a, g, i, j, CUDART_INF, INT32_MAX, dp64, bp) ? 0 : 1;
         }
+        __syncwarp();  // the staging slots are free for the next 32 outputs
     }
     count_exact(a, nres, nviol);
 }
@@ -1641,7 +1687,8 @@ __global__ void k_exact_small(Prefix P, FastArgs a, int i, double *dp64, int32_t
 // then lowest k).  With resident costs the lanes split every tile's k (the table
 // gives any pair directly); otherwise they take whole tiles (the recurrence of
 // visit_tile runs along k).
-__global__ void k_exact_big(Prefix P, FastArgs a, int i, double *dp64, int32_t *bp) {
+__global__ void __launch_bounds__(128) k_exact_big(Prefix P, FastArgs a, int i, double *dp64, int32_t *bp) {
+    __shared__ int32_t queue[4][32];  // per warp: band members waiting for binary64 re-scoring
     const int n = a.list_cnt[2 * i + 1];
     const int32_t *list = layer_list(a, i, 1);
     const int lane = threadIdx.x & 31;
@@ -1664,6 +1711,12 @@ __global__ void k_exact_big(Prefix P, FastArgs a, int i, double *dp64, int32_t *
         double best = CUDART_INF;
         int32_t arg = INT32_MAX;
         if (a.costs) {
+            // the lanes test the tile's k in the fp32 band; the members met wait in the warp's
+            // queue, and each time it holds 32 every lane re-scores one of them in binary64
+            // (the result, least value then lowest k, does not depend on the order)
+            int32_t *qw = queue[threadIdx.x >> 5];
+            int qn = 0;  // warp-uniform queue length
+            const unsigned lt = (1u << lane) - 1u;
             const float lam32 = a.prm->lam32[g];
             const int64_t J = j / BJ, j0 = J * BJ;
             for (uint32_t t = 0; t < ntile; t++) {
@@ -1673,13 +1726,30 @@ __global__ void k_exact_big(Prefix P, FastArgs a, int i, double *dp64, int32_t *
                 const float *pr = cr + kCostHalfFloats;
                 const float *prev32 = a.dp32 + d32(a, g, i - 1, k0) - k0;
                 const int64_t khi = (K == J) ? j - 1 : k0 + BK - 1;
-                for (int64_t k = k0 + lane; k <= khi; k += 32) {
-                    if (cand32(prev32[k], lam32, cr[k - k0], pr[k - k0]) <= thr) {
-                        exact_candidate(P, prev, k, j, lam, best, arg);
+                for (int64_t kb = k0; kb <= khi; kb += 32) {  // warp-uniform
+                    const int64_t k = kb + lane;
+                    const bool in = k <= khi && cand32(prev32[k], lam32, cr[k - k0], pr[k - k0]) <= thr;
+                    const unsigned mask = __ballot_sync(0xffffffffu, in);
+                    const int cnt = __popc(mask), pos = qn + __popc(mask & lt);
+                    if (in && pos < 32) qw[pos] = (int32_t)k;
+                    __syncwarp();
+                    if (qn + cnt >= 32) {
+                        exact_candidate(P, prev, qw[lane], j, lam, best, arg);
                         nres++;
+                        __syncwarp();
+                        if (in && pos >= 32) qw[pos - 32] = (int32_t)k;
+                        __syncwarp();
+                        qn += cnt - 32;
+                    } else {
+                        qn += cnt;
                     }
                 }
             }
+            if (lane < qn) {
+                exact_candidate(P, prev, qw[lane], j, lam, best, arg);
+                nres++;
+            }
+            __syncwarp();  // the queue is free for the warp's next output
         } else {
             for (uint32_t t = lane; t < ntile; t += 32) {
                 const uint32_t K = t < n1 ? (w1 >> 16) + t : (w2 >> 16) + (t - n1);
