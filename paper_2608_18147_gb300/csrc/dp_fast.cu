@@ -986,20 +986,26 @@ __device__ __forceinline__ bool wait_block(const FastArgs &a, int split, int K) 
     const int *flag = a.done + (size_t)split * a.nJ + K;
     uint32_t spins = 0;
     while (ld_acquire(flag) == 0) {
-        if (*(volatile int *)a.abort_flag) return false;
-        if (++spins > kSpinLimit) {
-            a.st->timeout = 1;
-            atomicExch(a.abort_flag, 1);
-            return false;
+        // the abort flag and the spin limit are checked every 64 spins, so a spin costs
+        // one flag load and a short sleep
+        if ((++spins & 63u) == 0u) {
+            if (*(volatile int *)a.abort_flag) return false;
+            if (spins > kSpinLimit) {
+                a.st->timeout = 1;
+                atomicExch(a.abort_flag, 1);
+                return false;
+            }
         }
-        __nanosleep(64);
+        __nanosleep(32);
     }
     return true;
 }
 
-// Publish column block J of `split` (after every thread's stores of the block).
+// Publish column block J of `split` (one thread, after a barrier that follows every
+// thread's stores of the block).  The release store orders everything that happens
+// before it, the other threads' stores included through the barrier, before the flag
+// (the pattern of an acq_rel fence plus a relaxed store); readers acquire the flag.
 __device__ __forceinline__ void publish_block(const FastArgs &a, int split, int J) {
-    __threadfence();
     st_release(a.done + (size_t)split * a.nJ + J, 1);
 }
 
