@@ -46,7 +46,7 @@ OPS_PER_CANDIDATE = 2     # one add and one min per min-plus candidate
 # 34 816 B of C and Phi, plus the dp32 rows and minima that miss L2), from the ncu
 # capture in profiles/k_wavefront_res_lognormal_d16384_s16.md; the benchmark launch is
 # scaled by the tiles it fetched (tile skipping leaves most tiles in HBM unread).
-TRAFFIC_PER_FETCHED_TILE = (6114810880 + 36267008) / 172557  # 6 launches of one solve: read + write / tiles
+TRAFFIC_PER_FETCHED_TILE = (6112144640 + 36549120) / 172518  # 6 launches of one solve: read + write / tiles
 ORACLE_SAMPLE = 16384     # entries of the CPU baseline's bounded sample
 
 

@@ -19,13 +19,19 @@ __device__ __forceinline__ uint64_t splitmix64(uint64_t z) {
     return z ^ (z >> 31);
 }
 
-__device__ __forceinline__ int quant_one(float xv, int64_t i, const float *q, int m, uint64_t seed, bool &bad) {
+constexpr uint64_t kGamma = 0x9E3779B97F4A7C15ull;
+
+// half: the largest power of two <= m - 1 (0 when m = 1); q[m .. 2 half - 1] hold +inf, so
+// the search needs no bound test.  zc = seed + (i + 1) * gamma (mod 2^64) for entry i.
+__device__ __forceinline__ int search_half(int m) { return m > 1 ? 1 << (31 - __clz(m - 1)) : 0; }
+
+__device__ __forceinline__ int quant_one(float xv, uint64_t zc, const float *q, int m, int half, bool &bad) {
     if (!(xv >= q[0] && xv <= q[m - 1])) { bad = true; return 0; }
     int t = 0;  // largest t with q[t] <= x: one step per bit of m - 1, the same count in every lane
-    for (int b = m > 1 ? 1 << (31 - __clz(m - 1)) : 0; b; b >>= 1)
-        if (t + b < m && q[t + b] <= xv) t += b;
+    for (int b = half; b; b >>= 1)
+        if (q[t + b] <= xv) t += b;
     if (q[t] != xv) {
-        uint64_t z = splitmix64(seed + (uint64_t)(i + 1) * 0x9E3779B97F4A7C15ull);
+        uint64_t z = splitmix64(zc);
         float k = __fmul_rn((float)(uint32_t)(z >> 40), 0x1p-24f);
         float d1 = __fsub_rn(xv, q[t]);
         float d2 = __fsub_rn(q[t + 1], q[t]);
@@ -69,9 +75,10 @@ __global__ void __launch_bounds__(kQThreads) k_quantize(const float *__restrict_
     __shared__ uint32_t hcount[kMaxS];
     __shared__ uint32_t ph[PRIV ? (kPrivBins / 2) * kQThreads : 1];
     for (int r = threadIdx.x; r < kMaxS; r += blockDim.x) {
-        q[r] = r < m ? Q[r] : 0.0f;
+        q[r] = r < m ? Q[r] : CUDART_INF_F;
         hcount[r] = 0;
     }
+    const int half = search_half(m);
     if (PRIV)
         for (int w = 0; w < kPrivBins / 2; w++) ph[w * kQThreads + threadIdx.x] = 0;
     __syncthreads();
@@ -92,16 +99,18 @@ __global__ void __launch_bounds__(kQThreads) k_quantize(const float *__restrict_
         const float4 xa = x4[g];
         const float4 xb = two ? x4[h] : make_float4(0.f, 0.f, 0.f, 0.f);
         {
-            const int64_t i = 4 * g;
-            const int t0 = quant_one(xa.x, i, q, m, seed, bad), t1 = quant_one(xa.y, i + 1, q, m, seed, bad);
-            const int t2 = quant_one(xa.z, i + 2, q, m, seed, bad), t3 = quant_one(xa.w, i + 3, q, m, seed, bad);
+            const uint64_t z0 = seed + (uint64_t)(4 * g + 1) * kGamma;  // entries 4g .. 4g+3: z0 + r gamma
+            const int t0 = quant_one(xa.x, z0, q, m, half, bad), t1 = quant_one(xa.y, z0 + kGamma, q, m, half, bad);
+            const int t2 = quant_one(xa.z, z0 + 2 * kGamma, q, m, half, bad);
+            const int t3 = quant_one(xa.w, z0 + 3 * kGamma, q, m, half, bad);
             i4[g] = make_uchar4((uint8_t)t0, (uint8_t)t1, (uint8_t)t2, (uint8_t)t3);
             count(t0); count(t1); count(t2); count(t3);
         }
         if (two) {
-            const int64_t i = 4 * h;
-            const int t0 = quant_one(xb.x, i, q, m, seed, bad), t1 = quant_one(xb.y, i + 1, q, m, seed, bad);
-            const int t2 = quant_one(xb.z, i + 2, q, m, seed, bad), t3 = quant_one(xb.w, i + 3, q, m, seed, bad);
+            const uint64_t z0 = seed + (uint64_t)(4 * h + 1) * kGamma;
+            const int t0 = quant_one(xb.x, z0, q, m, half, bad), t1 = quant_one(xb.y, z0 + kGamma, q, m, half, bad);
+            const int t2 = quant_one(xb.z, z0 + 2 * kGamma, q, m, half, bad);
+            const int t3 = quant_one(xb.w, z0 + 3 * kGamma, q, m, half, bad);
             i4[h] = make_uchar4((uint8_t)t0, (uint8_t)t1, (uint8_t)t2, (uint8_t)t3);
             count(t0); count(t1); count(t2); count(t3);
         }
@@ -111,7 +120,7 @@ __global__ void __launch_bounds__(kQThreads) k_quantize(const float *__restrict_
         }
     }
     for (int64_t i = 4 * ngroups + g0; i < d; i += stride) {
-        const int t = quant_one(x[i], i, q, m, seed, bad);
+        const int t = quant_one(x[i], seed + (uint64_t)(i + 1) * kGamma, q, m, half, bad);
         idx[i] = (uint8_t)t;
         count(t);
         if (PRIV && ++since_fold >= kFoldEntries) {
@@ -173,8 +182,8 @@ __global__ void __launch_bounds__(256) k_quantize_timeshare(const float *__restr
     __shared__ float q[2][kMaxS];
     __shared__ uint32_t hcount[2 * kMaxS];
     for (int r = threadIdx.x; r < kMaxS; r += blockDim.x) {
-        q[0][r] = r < mm ? Qm[r] : 0.0f;
-        q[1][r] = r < mp ? Qp[r] : 0.0f;
+        q[0][r] = r < mm ? Qm[r] : CUDART_INF_F;
+        q[1][r] = r < mp ? Qp[r] : CUDART_INF_F;
         hcount[r] = 0;
         hcount[kMaxS + r] = 0;
     }
@@ -182,9 +191,10 @@ __global__ void __launch_bounds__(256) k_quantize_timeshare(const float *__restr
     bool bad = false;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < d; i += stride) {
-        uint64_t zs = splitmix64(seed_ts + (uint64_t)(i + 1) * 0x9E3779B97F4A7C15ull);
+        uint64_t zs = splitmix64(seed_ts + (uint64_t)(i + 1) * kGamma);
         int part = __dmul_rn((double)(uint32_t)(zs >> 40), 0x1p-24) < beta ? 1 : 0;
-        int t = quant_one(x[i], i, q[part], part ? mp : mm, seed, bad);
+        const int mq = part ? mp : mm;
+        int t = quant_one(x[i], seed + (uint64_t)(i + 1) * kGamma, q[part], mq, search_half(mq), bad);
         idx[i] = (uint8_t)t;
         if (sel) sel[i] = (uint8_t)part;
         atomicAdd(&hcount[part * kMaxS + t], 1u);
