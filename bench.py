@@ -22,6 +22,11 @@ Other rows of the path, each timed the same way on the chosen --config:
   --mode hbm        the HBM-bound rows on vectors far larger than L2: the encode (A10,
                     2^28 entries) and the sort + histogram + prefix sums (A1-A3, 2^26
                     entries); metric: GB/s of algorithmic traffic
+  --mode rows       the batched solve of many independent short rows (the KV-cache-like
+                    workload, 8192 rows of 128 entries); metric: rows/s
+  --mode pass       one DP pass (sort, histogram, interval costs, the min-plus layers, the
+                    exact stage, traceback) of the --config vector at the multipliers of
+                    --lambdas; metric: candidate evaluations/s
 """
 import argparse
 import json
@@ -59,7 +64,8 @@ def parse():
     ap.add_argument("--config", default="studentt_d131072_s16")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--mode", default="solve", choices=["solve", "grid", "timeshare", "opt", "hbm"])
+    ap.add_argument("--mode", default="solve", choices=["solve", "grid", "timeshare", "opt", "hbm", "rows", "pass"])
+    ap.add_argument("--lambdas", default="0.02", help="comma-separated multipliers (vNMSE scale) for --mode pass")
     ap.add_argument("--grid", type=int, default=256, help="grid size for --mode grid")
     return ap.parse_args()
 
@@ -203,6 +209,12 @@ def run_other_mode(args, cfg, x_np):
     if args.mode == "hbm":
         run_hbm_mode(args)
         return
+    if args.mode == "rows":
+        run_rows_mode(args)
+        return
+    if args.mode == "pass":
+        run_pass_mode(args, cfg, x_np)
+        return
     if args.mode == "grid":
         g = torch.as_tensor(E.uniform_grid(x_np, args.grid)).cuda()
         ws = torch.empty(int(E.lib().ecasq_workspace_size_grid(d, g.numel(), s, flags)), dtype=torch.uint8,
@@ -315,6 +327,79 @@ def run_hbm_mode(args):
                      "prepare": {"ms": ms_p, "bytes_per_entry": 32, "GBs": gbs_p, "frac": gbs_p / peak,
                                  "basis": "4 LSD radix passes x (4 B read + 4 B written); the histogram, "
                                           "prefix sums and count passes are extra"}})
+    print(json.dumps(out), flush=True)
+
+
+def _timed_steps(args, step):
+    """CUDA-event time (ms) of args.steps calls of step() after args.warmup untimed ones,
+    with the clocks sampled meanwhile."""
+    import torch
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    outs = []
+    with ClockSampler(int(os.environ.get("LOCAL_RANK", "0"))) as clk:
+        ev0.record(stream)
+        for _ in range(args.steps):
+            outs.append(step())
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    return ev0.elapsed_time(ev1), outs, clk.summary()
+
+
+def run_rows_mode(args):
+    """Batched budgeted solves of the KV-cache-like rows (8192 x 128, s = 8, b = 3):
+    rows per second, inputs in HBM."""
+    import torch
+    import paper_2608_18147_gb300 as E
+    from paper_2608_18147_gb300 import workloads
+    name = "kvrows_8192x128_s8"
+    cfg = workloads.CONFIGS[name]
+    X = torch.as_tensor(workloads.make(name)).cuda()
+    rows, d = X.shape
+    s, budget = cfg["s"], cfg["budgets"][0]
+    ws = E.workspace(d, s, rows)
+    launches0 = E.ecasq_kernel_launches()
+    ms, outs, clocks = _timed_steps(args, lambda: E.ecasq_solve_batched(X, s, budget_bits=budget, ws=ws))
+    Q, m, res = outs[-1]
+    ok = sum(1 for r in res if r["status"] == 0)
+    out = {"metric": "ECASQ batched solve: rows/s", "value": args.steps * rows / (ms / 1000.0), "unit": "rows/s",
+           "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
+           "higher_is_better": True, "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": {"workload": name, "mode": "rows", "rows": rows, "d": d, "s": s, "budget_bits": budget},
+           "rows_ok": ok, "mean_m": float(m.float().mean().item()),
+           "gpu_launches": E.ecasq_kernel_launches() - launches0, "clocks": clocks}
+    print(json.dumps(out), flush=True)
+
+
+def run_pass_mode(args, cfg, x_np):
+    """One DP pass of the configuration's vector at the --lambdas multipliers (resident
+    interval costs when they fit in 60 % of the free memory, else the fused kernel)."""
+    import torch
+    import paper_2608_18147_gb300 as E
+    s = cfg["s"]
+    lams = [float(t) for t in args.lambdas.split(",")]
+    x = torch.as_tensor(x_np).cuda()
+    d = x.numel()
+    flags = 0
+    need = E.ecasq_workspace_size_flags(d, s, 1, E.RESIDENT_COSTS)
+    if 0 < need <= 0.6 * torch.cuda.mem_get_info()[0]:
+        flags |= E.RESIDENT_COSTS
+    ws = E.workspace(d, s, flags=flags)
+    launches0 = E.ecasq_kernel_launches()
+    ms, outs, clocks = _timed_steps(args, lambda: E.ecasq_dp_pass(x, s, lams, flags=flags, ws=ws))
+    st = E.native.ws_status(ws)
+    p = st["p"]
+    cand = len(lams) * candidates_per_multiplier(p, s)
+    out = {"metric": "ECASQ DP pass: candidate evals/s", "value": args.steps * cand / (ms / 1000.0),
+           "unit": UNIT, "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
+           "higher_is_better": True, "vs_baseline": None, "dtype": "f32 (fp64 exact stage)", "data": "synthetic",
+           "config": {"workload": args.config, "mode": "pass", "d": d, "p": p, "s": s, "lambdas": lams,
+                      "resident_costs": bool(flags & E.RESIDENT_COSTS)},
+           "status": {"timeout": st["timeout"], "bound_viol": st["bound_viol"], "rescored": st["rescored"]},
+           "m": list(outs[-1][1]), "gpu_launches": E.ecasq_kernel_launches() - launches0, "clocks": clocks}
     print(json.dumps(out), flush=True)
 
 
