@@ -5,6 +5,9 @@
   the whole budgeted solve (multiplier search of Sec. 3 / Sec. 5 under reading R4,
   traceback, evaluation) in the benchmark's launch configuration (resident interval
   costs) against the oracle's full search;
+* the benchmark's pipeline (resident costs, search, refinement to 1e-9 relative in at most
+  50 rounds, encode) on its Student-t distribution at d = 16384, where the oracle's full
+  pipeline runs in seconds;
 * mixture 0.9 N(0,1) + 0.1 N(0,10^2), d = 2^20, s = 32 (too large for the oracle's
   full DP): one DP pass in the default mode, checked where the oracle can compute
   one output at a time -- eq. apx_rec at sampled outputs the traceback reads, from
@@ -92,5 +95,31 @@ def test_mixture_2p20_sampled_decisions(E, oracle_mod):
                 assert bp[i, j] == arg
         mse, hs, hx = H.eval_idx(idx)
         np.testing.assert_allclose(met[g][1:], [mse, hs, hx], rtol=MET_RTOL)
+    del ws
+    _free()
+
+
+def test_studentt_benchmark_pipeline_at_16k_matches_oracle(E, oracle_mod):
+    """The benchmark's pipeline (resident interval costs, budgeted search, refinement up to
+    50 rounds with the 1e-9 relative stop, then the encode) on the benchmark's distribution
+    (1e-3 Student-t(3), s = 16, b = 2.5) at d = 16384, against the oracle's full pipeline."""
+    x = workloads.student_t(16384, 0)
+    s, budget = 16, 2.5
+    ws = E.workspace(x.size, s, flags=E.RESIDENT_COSTS)
+    Q, res = E.ecasq_solve(x, s, budget_bits=budget, ws=ws, refine_max_rounds=50, refine_rel_tol=1e-9,
+                           flags=E.RESIDENT_COSTS)
+    st = E.native.ws_status(ws)
+    o = oracle_mod.solve_budget(x, s, budget, refine_rounds=50, refine_tol=1e-9)
+    assert res["status"] == o["status"] == 0
+    assert st["timeout"] == 0 and st["bound_viol"] == 0
+    assert res["lambda"] == o["lam"]
+    assert res["refine_rounds"] == o["refine_rounds"]
+    np.testing.assert_array_equal(Q.cpu().numpy(), o["Q"])
+    np.testing.assert_allclose([res["mse"], res["h_surrogate"], res["h_exact"]],
+                               [o["mse"], o["h_surrogate"], o["h_exact"]], rtol=MET_RTOL)
+    idx, counts, he = E.ecasq_quantize(x, Q, seed=12345)
+    oi, oc, oh = oracle_mod.quantize(x, Q.cpu().numpy(), 12345)
+    np.testing.assert_array_equal(idx.cpu().numpy(), oi)
+    np.testing.assert_array_equal(counts.cpu().numpy().astype(np.uint32), oc)
     del ws
     _free()
