@@ -50,6 +50,13 @@
  *     OOPSLA 2014) on seed + (i+1)*0x9E3779B97F4A7C15, k = top 24 bits;
  *     round up iff fl32(fl32(k*2^-24) * fl32(b-a)) < fl32(x-a).
  *
+ * Parity unpinned by the paper: the multiplier schedule of or_search, the scan
+ * and tie rules of or_refine and the random draw of or_quantize are the readings
+ * above, not values the paper fixes.  The tests pin them to those readings only
+ * (SplitMix64's published outputs, the exact rounding probability, refinement
+ * monotonicity and coordinate optimality, the search's feasibility and least-MSE
+ * choice among its evaluated points).
+ *
  * Build: gcc -O2 -fopenmp -ffp-contract=off -fPIC -shared (see build.py).
  */
 #include <math.h>
