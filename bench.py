@@ -43,14 +43,18 @@ if ROOT not in sys.path:
 
 METRIC = "ECASQ approx-DP solve ms & candidate evals/s at d=2^17,s=16; % of ALU peak"
 UNIT = "candidate evals/s"
-SM_COUNT = 152
 FP32_LANES = 128          # FP32-pipe lanes per SM (adds and min/max share them)
 SM_MAX_MHZ = 2070.0
-OPS_PER_CANDIDATE = 2     # one add and one min per min-plus candidate
+# Ops the min-plus kernel issues per candidate: one add (packed f32x2) and one min
+# (3-input integer min on the float bits).  W = C + lambda' Phi is formed once per
+# (pair, multiplier) and shared by every layer, so the FMA that a per-candidate count
+# (add + FMA + min = 3) includes is 1/(s-2) of an op per candidate here.
+OPS_PER_CANDIDATE = 2
+BK = BJ = 64              # the kernel's tile: 64 k by 64 columns
 # DRAM bytes of k_wavefront_res per interval-cost tile it copies in (64 x 64 pairs,
-# 34 816 B of C and Phi, plus the dp32 rows and minima that miss L2), from the ncu
-# capture in profiles/k_wavefront_res_lognormal_d16384_s16.md; the benchmark launch is
-# scaled by the tiles it fetched (tile skipping leaves most tiles in HBM unread).
+# 34 816 B of C and Phi, plus the dp32 rows and minima that miss L2), from the committed
+# ncu capture of every launch of one solve at d = 16384; the benchmark launch is scaled
+# by the tiles it fetched (tile skipping leaves most tiles in HBM unread).
 TRAFFIC_PER_FETCHED_TILE = (6112144640 + 36549120) / 172518  # 6 launches of one solve: read + write / tiles
 ORACLE_SAMPLE = 16384     # entries of the CPU baseline's bounded sample
 
@@ -95,6 +99,18 @@ def candidates_per_multiplier(p, s):
             break
         c += n * (n + 1) // 2
     return c
+
+
+def executed_candidates(st, p, s, multipliers):
+    """Candidates the min-plus kernel evaluated in one solve, from its own counters:
+    every off-diagonal (multiplier, tile) unit it ran is 64 x 64 pairs times the s - 2
+    layers; every diagonal block is evaluated for each multiplier of its pass, with its
+    pairs k < j (a 64-column triangle) over the s - 2 layers."""
+    L = max(s - 2, 0)
+    n_blocks = -(-p // BJ)
+    off = st["tiles_run"] * BK * BJ * L
+    diag = multipliers * n_blocks * (BJ * (BJ - 1) // 2) * L
+    return off + diag
 
 
 class ClockSampler:
@@ -532,10 +548,18 @@ def main():
     units = st["tiles_run"] + st["tiles_skipped"]
     run_frac = st["tiles_run"] / units if units else 1.0
 
-    # roofline of the min-plus kernel: FP32-pipe ops (one add + one min per candidate)
-    achieved = OPS_PER_CANDIDATE * cand_total / (dp_ms / 1000.0) / 1e12 if dp_ms > 0 else None
-    peak = SM_COUNT * FP32_LANES * SM_MAX_MHZ * 1e6 / 1e12
-    last_launches = max(results[-1]["dp_kernel_launches"], 1)
+    # roofline of the min-plus kernel against the FP32/ALU issue peak.  `achieved` counts
+    # the candidates the kernel executed (the tile units it ran and its diagonal blocks),
+    # not the algorithmic ones: the exact tile skip leaves most of eq. apx_rec unevaluated,
+    # and the algorithmic rate is reported beside it as `effective`.
+    last = results[-1]
+    n_sm = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
+    peak = n_sm * FP32_LANES * SM_MAX_MHZ * 1e6 / 1e12
+    last_launches = max(last["dp_kernel_launches"], 1)
+    last_ms = last["dp_kernel_ms"]
+    executed = executed_candidates(st, last_p, s, last["lambdas_evaluated"])
+    achieved = OPS_PER_CANDIDATE * executed / (last_ms / 1000.0) / 1e12 if last_ms > 0 else None
+    effective = OPS_PER_CANDIDATE * cand_total / (dp_ms / 1000.0) / 1e12 if dp_ms > 0 else None
     fetched_per_launch = st["tiles_fetched"] / last_launches
     traffic = (TRAFFIC_PER_FETCHED_TILE * fetched_per_launch
                if (flags & E.RESIDENT_COSTS) and TRAFFIC_PER_FETCHED_TILE else None)
@@ -545,14 +569,23 @@ def main():
                                 "d = 16384, times the tiles this launch fetched",
                 "tiles_fetched_per_launch": fetched_per_launch,
                 "kernel": "k_wavefront_res" if (flags & E.RESIDENT_COSTS) else "k_wavefront",
-                "peak_basis": "152 SMs x 128 FP32-pipe lanes (adds and mins share them) x 2070 MHz max clock",
+                "peak_basis": "%d SMs (device attribute) x 128 FP32-pipe lanes (adds and mins share the issue "
+                              "slots) x 2070 MHz max clock; of the 2-op count below" % n_sm,
                 "avg_launch_ms": dp_ms / max(dp_launches, 1), "launches": dp_launches,
-                "ops_basis": "algorithmic: 2 ops for every candidate of eq. apx_rec (all layers, multipliers, k < j)",
+                "ops_basis": "executed: 2 ops (add, min) per candidate the kernel evaluated -- %d-column x %d-k "
+                             "tile units it ran, times the s-2 layers, plus its diagonal blocks; "
+                             "C + lambda' Phi is formed once per pair and multiplier, so a 3-op count "
+                             "(add + FMA + min) would add 1/(s-2) op per candidate" % (BJ, BK),
+                "executed_candidates_per_launch": executed / last_launches,
+                "effective": effective,
+                "effective_frac": (effective / peak) if effective else None,
+                "effective_note": "algorithmic rate: 2 ops for every candidate of eq. apx_rec (all layers, "
+                                  "multipliers, k < j), including the ones the exact tile skip never evaluates",
                 "executed_unit_frac": run_frac,
                 "executed_note": "off-diagonal (warp, tile) units evaluated; the rest were skipped by an exact "
                                  "lower bound that proves they cannot change any minimum or band"}
     if achieved and clocks.get("sm_mhz"):
-        roofline["frac_at_measured_clock"] = achieved / (SM_COUNT * FP32_LANES * clocks["sm_mhz"] * 1e6 / 1e12)
+        roofline["frac_at_measured_clock"] = achieved / (n_sm * FP32_LANES * clocks["sm_mhz"] * 1e6 / 1e12)
 
     e2e = None
     if not args.no_e2e:

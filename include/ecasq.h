@@ -57,6 +57,10 @@ typedef struct CUstream_st *ecasq_stream_t; /* same type as cudaStream_t */
 #define ECASQ_RESIDENT_COSTS 32u  /* fast DP: compute the lambda-independent interval costs C and Phi (Sec. 5, App. E)
                                      once per call into the workspace and stream them to every pass (workspace:
                                      ecasq_workspace_size_flags with this flag; about 4.3 d^2 bytes extra) */
+#define ECASQ_TEST_STALL (1u << 30) /* test hook for the bounded device waits: column block 0 of the fast DP's
+                                     wavefront is never published and the flag waits give up after 2^14 spins, so
+                                     the call must return ECASQ_ETIMEOUT (nothing else) and leave the workspace
+                                     usable by the next call.  Not for production use. */
 
 typedef struct ecasq_params {
     int32_t s;                 /* codebook cap, 2..256 */
@@ -300,7 +304,10 @@ int ecasq_quantize(const float *x, int64_t d, const float *Q, int32_t m, uint64_
  * Set-up: the first call on each device looks up the scratch's device address
  * (cudaGetSymbolAddress, which may load this library's device code) and keeps
  * it; an error there returns ECASQ_ECUDA.  Make that first call on each device
- * before any stream capture begins.
+ * before any stream capture begins.  The kept address belongs to the device
+ * context of that first call: resetting the device (cudaDeviceReset) after it
+ * is not supported.  `stream` must belong to the current device (a stream of
+ * another device returns ECASQ_EINVAL).
  *
  * Concurrency: all calls on one device share the one scratch block.  Calls
  * that overlap in time on the same device -- from several host threads, or on

@@ -64,6 +64,7 @@ def _load():
             "or_pair": (None, [P, i64, i64, pd]),
             "or_phi": (dbl, [P, i64, i64, i32]),
             "or_apx_dp": (i32, [P, i32, dbl, i32, pd, pi32, pd, pi64, pi32, pd]),
+            "or_apx_dp_columns": (i32, [P, i32, dbl, i32, pd, pi32, pd, pi64, pi32, pd]),
             "or_dp_decision": (None, [P, pd, i32, i64, dbl, pd, pi64, pd]),
             "or_dp_candidate": (dbl, [P, dbl, i64, i64, dbl, i32]),
             "or_eval_idx": (i32, [P, pi64, i32, pd]),
@@ -165,8 +166,10 @@ class Hist:
     def phi(self, k, j, first=False):
         return float(_load().or_phi(self._h, int(k), int(j), int(bool(first))))
 
-    def apx_dp(self, s, lam_prime, exact_s=False, tables=True):
-        """Approximate DP of Sec. 5 at multiplier lambda' (eqs. apx_base/rec/final)."""
+    def apx_dp(self, s, lam_prime, exact_s=False, tables=True, columns=False):
+        """Approximate DP of Sec. 5 at multiplier lambda' (eqs. apx_base/rec/final).
+        columns: evaluate it column by column (or_apx_dp_columns: the same tables, each
+        pair's link cost computed once for all layers; for inputs too large to memoise)."""
         p = self.p
         rows = s + 1
         dp = np.empty(rows * p, np.float64) if tables else None
@@ -176,7 +179,8 @@ class Hist:
         m = C.c_int32()
         best = C.c_double()
         nul = lambda a, t: _ptr(a, t) if a is not None else None
-        st = _load().or_apx_dp(self._h, int(s), float(lam_prime), int(bool(exact_s)),
+        fn = _load().or_apx_dp_columns if columns else _load().or_apx_dp
+        st = fn(self._h, int(s), float(lam_prime), int(bool(exact_s)),
                                nul(dp, C.c_double), nul(bp, C.c_int32), nul(mg, C.c_double),
                                _ptr(Q, C.c_int64), C.byref(m), C.byref(best))
         if st != OK:

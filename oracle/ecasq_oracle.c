@@ -23,6 +23,10 @@
  *   pair_q           App. E: U_P, D_P, C_P from prefix differences
  *   h, or_phi        Sec. 4 (h), Sec. 5 (Phi, Phi^first)
  *   or_apx_dp        Sec. 5, eqs. apx_base / apx_rec / apx_final
+ *   or_apx_dp_columns the same DP evaluated column by column (each pair's link
+ *                    cost computed once for all layers), for full-size checks
+ *   or_dp_decision,  one output / one candidate of eq. apx_rec (eq. apx_base with
+ *   or_dp_candidate  `first`), for checking sampled outputs of large GPU runs
  *   or_eval_idx      Sec. 2 (MSE), Sec. 3 (H(Xhat)), Sec. 5 eq. apx_additive_entropy
  *   or_eval_direct   the per-entry definitions of Sec. 1-3 and Sec. 5 (no prefix sums)
  *   or_asq_dp        Sec. 2, eq. asqdp (ZipML/QUIVER recurrence, lambda = 0)
@@ -441,6 +445,98 @@ int32_t or_apx_dp(const or_hist *H, int32_t s, double lam_prime, int32_t exact_s
         }
     if (istar < 0) { free(dp); free(bp); free(mg); return OR_EINFEASIBLE; }
     /* traceback */
+    int64_t j = jstar;
+    Q_idx[istar - 1] = j;
+    for (int32_t i = istar; i >= 3; i--) {
+        j = bp[(size_t)i * (size_t)p + (size_t)j];
+        Q_idx[i - 2] = j;
+    }
+    Q_idx[0] = bp[2 * (size_t)p + (size_t)j];
+    *m_out = istar;
+    *best_out = best;
+    if (dp_out) memcpy(dp_out, dp, sizeof(double) * rows * (size_t)p);
+    if (bp_out) memcpy(bp_out, bp, sizeof(int32_t) * rows * (size_t)p);
+    if (margin_out) memcpy(margin_out, mg, sizeof(double) * rows * (size_t)p);
+    free(dp); free(bp); free(mg);
+    return OR_OK;
+}
+
+/* The same DP as or_apx_dp (same tables, same codebook), evaluated column by
+ * column so that inputs far too large for the pair memo stay practical: for
+ * each j, in increasing order, the link costs C[k, j] + lambda' Phi[k, j] of
+ * every k < j are computed once (in parallel over k) and every layer
+ * i = 3..s then takes its minimum over k in [i-2, j-1] of
+ * dp(i-1, k) + (C + lambda' Phi) -- the binary64 candidate of or_apx_dp,
+ * lowest k among exact minima, the same second-best margin.  dp(i-1, k) for
+ * k < j is final when column j is reached, because every k < j was visited
+ * earlier.  Memory: the (s+1) x p tables plus one column.
+ * Used by the one-off full-size checks, where or_apx_dp would recompute each
+ * pair once per layer. */
+int32_t or_apx_dp_columns(const or_hist *H, int32_t s, double lam_prime, int32_t exact_s,
+                          double *dp_out, int32_t *bp_out, double *margin_out,
+                          int64_t *Q_idx, int32_t *m_out, double *best_out) {
+    int64_t p = H->p;
+    if (s < 2) return OR_EINVAL;
+    if (p == 1) {
+        Q_idx[0] = 0; *m_out = 1; *best_out = 0.0;
+        return OR_OK;
+    }
+    size_t rows = (size_t)s + 1;
+    double *dp = (double *)malloc(sizeof(double) * rows * (size_t)p);
+    int32_t *bp = (int32_t *)malloc(sizeof(int32_t) * rows * (size_t)p);
+    double *mg = (double *)malloc(sizeof(double) * rows * (size_t)p);
+    double *W = (double *)malloc(sizeof(double) * (size_t)p);
+    if (!dp || !bp || !mg || !W) { free(dp); free(bp); free(mg); free(W); return OR_ENOMEM; }
+    for (size_t t = 0; t < rows * (size_t)p; t++) { dp[t] = INFINITY; bp[t] = -1; mg[t] = INFINITY; }
+    /* base layer: as or_apx_dp */
+    for (int64_t j = 1; j < p; j++) {
+        double best = INFINITY;
+        int64_t arg = -1;
+        for (int64_t a = 0; a < H->nL && a < j; a++) {
+            double C, U, D;
+            pair_q(H, a, j, &C, &U, &D);
+            double c = C + lam_prime * phi_of(H, U, D, a);
+            if (c < best) { best = c; arg = a; }
+        }
+        dp[2 * (size_t)p + (size_t)j] = best;
+        bp[2 * (size_t)p + (size_t)j] = (int32_t)arg;
+    }
+    for (int64_t j = 1; j < p; j++) {
+        if (s < 3) break;
+#pragma omp parallel for schedule(static)
+        for (int64_t k = 0; k < j; k++) {
+            double C, Phi;
+            cphi(H, k, j, &C, &Phi);
+            W[k] = C + lam_prime * Phi;
+        }
+        int32_t itop = s < (int32_t)(j + 1) ? s : (int32_t)(j + 1);  /* layers with j >= i - 1 */
+#pragma omp parallel for schedule(dynamic, 1)
+        for (int32_t i = 3; i <= itop; i++) {
+            const double *prev = dp + (size_t)(i - 1) * (size_t)p;
+            double best = INFINITY, second = INFINITY;
+            int64_t arg = -1;
+            for (int64_t k = i - 2; k < j; k++) {
+                double cand = prev[k] + W[k];
+                if (cand < best) { second = best; best = cand; arg = k; }
+                else if (cand < second) second = cand;
+            }
+            size_t o = (size_t)i * (size_t)p + (size_t)j;
+            dp[o] = best;
+            bp[o] = (int32_t)arg;
+            mg[o] = (best > 0.0) ? (second - best) / best : (second > best ? INFINITY : 0.0);
+        }
+    }
+    free(W);
+    int32_t istar = -1;
+    int64_t jstar = -1;
+    double best = INFINITY;
+    int32_t ilo = exact_s ? s : 2;
+    for (int32_t i = ilo; i <= s; i++)
+        for (int64_t jr = p - H->nR; jr < p; jr++) {
+            double v = dp[(size_t)i * (size_t)p + (size_t)jr];
+            if (v < best) { best = v; istar = i; jstar = jr; }
+        }
+    if (istar < 0) { free(dp); free(bp); free(mg); return OR_EINFEASIBLE; }
     int64_t j = jstar;
     Q_idx[istar - 1] = j;
     for (int32_t i = istar; i >= 3; i--) {

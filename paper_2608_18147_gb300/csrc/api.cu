@@ -16,7 +16,7 @@ namespace ecasq {
 int launch_dp_reference(const Prefix &P, const double *lamp, int G, int s, double *dp64, int32_t *bp,
                         cudaStream_t st);
 int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, const Layout &L, cudaStream_t st,
-                   bool exact_s, bool exact_tables, float *costs, bool build_costs);
+                   bool exact_s, bool exact_tables, float *costs, bool build_costs, bool test_stall);
 size_t resident_costs_bytes(int64_t d);
 int launch_rows_prepare(const float *X, int64_t rows, const RowsData &R, cudaStream_t st);
 int launch_grid_prefix(const float *P, int64_t n, const float *vX, const int64_t *NX, const double *SX,
@@ -164,10 +164,12 @@ static std::mutex g_noalloc_mu;
 static void *g_noalloc_addr[kNoAllocMaxDevices];
 
 // Device address of the scratch block on the current device, looked up once
-// per device (cudaGetSymbolAddress) and kept.
-static int noalloc_scratch(void **out) {
-    int dev = -1;
+// per device (cudaGetSymbolAddress) and kept.  `st` must belong to that device.
+static int noalloc_scratch(cudaStream_t st, void **out) {
+    int dev = -1, sdev = -1;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kNoAllocMaxDevices) return ECASQ_ECUDA;
+    if (cudaStreamGetDevice(st, &sdev) != cudaSuccess) return ECASQ_ECUDA;
+    if (sdev != dev) return ECASQ_EINVAL;
     std::lock_guard<std::mutex> lock(g_noalloc_mu);
     if (!g_noalloc_addr[dev]) {
         void *p = nullptr;
@@ -282,7 +284,7 @@ static int dp_pass_prepared(void *ws, const Layout &L, const Prefix &P, int s, c
     } else {
         float *costs = L.costs_bytes ? wsp<float>(ws, L.costs) : nullptr;
         rc = launch_dp_fast(P, lamp, G, s, ws, L, st, (flags & ECASQ_EXACT_S) != 0, (flags & ECASQ_EXACT_TABLES) != 0,
-                            costs, costs && !*costs_built);
+                            costs, costs && !*costs_built, (flags & ECASQ_TEST_STALL) != 0);
         if (costs && rc == ECASQ_OK) *costs_built = true;
     }
     if (rc != ECASQ_OK) return rc;
@@ -984,10 +986,10 @@ int ecasq_quantize(const float *x, int64_t d, const float *Q, int32_t m, uint64_
 int ecasq_quantize_noalloc(const float *x, int64_t d, const float *Q, int32_t m, uint64_t seed, uint8_t *idx,
                            uint32_t *counts, double *h_emp, ecasq_stream_t stream) {
     if (!x || !Q || !idx || !counts || d < 1 || d >= ((int64_t)1 << 31) || m < 1 || m > kMaxS) return ECASQ_EINVAL;
-    void *scratch = nullptr;
-    int rc = noalloc_scratch(&scratch);
-    if (rc) return rc;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    void *scratch = nullptr;
+    int rc = noalloc_scratch(st, &scratch);
+    if (rc) return rc;
     DevStatus *ds = reinterpret_cast<DevStatus *>(scratch);
     float qh[kMaxS];
     ECASQ_CUDA_TRY(cudaMemcpyAsync(qh, Q, 4 * (size_t)m, cudaMemcpyDeviceToHost, st));

@@ -67,6 +67,7 @@ constexpr int MAXCONS = 256;
 constexpr int NMEM = 8;        // members kept inline per output
 constexpr int64_t kMaxFastP = (int64_t)1 << 20;
 constexpr uint32_t kSpinLimit = 1u << 26;
+constexpr uint32_t kTestSpinLimit = 1u << 14;  // the ECASQ_TEST_STALL hook: about 10-20 ms of spinning
 constexpr uint32_t kCopySpinLimit = 1u << 22;  // waits on bulk copies (microseconds when healthy)
 // Resident interval costs: per tile, C[64][PSTR] then Phi[64][PSTR] (the shared-memory layout).
 constexpr int kCostHalfFloats = BJ * PSTR;
@@ -138,6 +139,8 @@ struct FastArgs {
     float *mdp;            // [nJ][G][mdp_stride]: min over the block's 64 columns of dp32(g, i, .)
     int mdp_stride;        // s + 1 rounded up to a multiple of 4 (16-byte rows)
     int prune;             // skip tiles by the lower bound (resident costs, two layer groups)
+    uint32_t spin_limit;   // flag waits give up after this many spins (kSpinLimit; lower in the test hook)
+    int hold0;             // test hook: column block 0 is never published (its waiters time out)
     int *done;             // [nsplit][nJ]
     int *ticket;
     int *abort_flag;
@@ -990,7 +993,7 @@ __device__ __forceinline__ bool wait_block(const FastArgs &a, int split, int K) 
         // one flag load and a short sleep
         if ((++spins & 63u) == 0u) {
             if (*(volatile int *)a.abort_flag) return false;
-            if (spins > kSpinLimit) {
+            if (spins > a.spin_limit) {
                 a.st->timeout = 1;
                 atomicExch(a.abort_flag, 1);
                 return false;
@@ -1006,6 +1009,7 @@ __device__ __forceinline__ bool wait_block(const FastArgs &a, int split, int K) 
 // before it, the other threads' stores included through the barrier, before the flag
 // (the pattern of an acq_rel fence plus a relaxed store); readers acquire the flag.
 __device__ __forceinline__ void publish_block(const FastArgs &a, int split, int J) {
+    if (a.hold0 && J == 0) return;  // test hook: the waiters on block 0 must give up
     st_release(a.done + (size_t)split * a.nJ + J, 1);
 }
 
@@ -1521,6 +1525,7 @@ __device__ __forceinline__ int32_t *layer_list(const FastArgs &a, int i, int kin
 // Backward closure, layer i: members of every needed output; mark (i-1, k) needed;
 // list the needed outputs for the exact stage (inline members / big bands).
 __global__ void k_need_layer(FastArgs a, int i) {
+    if (*(volatile const int *)a.abort_flag) return;  // a wait gave up: the tables are not valid
     const int64_t tot = (int64_t)a.G * a.p;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     unsigned long long nmem = 0, nbig = 0, nover = 0;
@@ -1568,6 +1573,7 @@ __global__ void k_need_layer(FastArgs a, int i) {
 
 // Outputs the answer does not read keep their fp32 minimum: dp64 = m32, bp = -2.
 __global__ void k_fill_unneeded(FastArgs a, double *dp64, int32_t *bp) {
+    if (*(volatile const int *)a.abort_flag) return;  // a wait gave up: the tables are not valid
     const int64_t tot = (int64_t)a.G * (a.s + 1) * a.ps;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t o = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; o < tot; o += stride) {
@@ -1619,6 +1625,7 @@ __device__ __forceinline__ void count_exact(const FastArgs &a, unsigned long lon
 // Layer i, outputs with at most NMEM members: one thread each, binary64 re-scoring
 // with double-double interval costs; the lowest k among exact minima wins.
 __global__ void __launch_bounds__(128) k_exact_small(Prefix P, FastArgs a, int i, double *dp64, int32_t *bp) {
+    if (*(volatile const int *)a.abort_flag) return;  // a wait gave up: the tables are not valid
     // A warp takes 32 listed outputs at a time and evaluates their members flattened
     // (member r of the 32 outputs' lists goes to lane r mod 32), so every lane of a
     // binary64 sequence does useful work; then each output's lane takes the least value,
@@ -1694,6 +1701,7 @@ __global__ void __launch_bounds__(128) k_exact_small(Prefix P, FastArgs a, int i
 // gives any pair directly); otherwise they take whole tiles (the recurrence of
 // visit_tile runs along k).
 __global__ void __launch_bounds__(128) k_exact_big(Prefix P, FastArgs a, int i, double *dp64, int32_t *bp) {
+    if (*(volatile const int *)a.abort_flag) return;  // a wait gave up: the tables are not valid
     __shared__ int32_t queue[4][32];  // per warp: band members waiting for binary64 re-scoring
     const int n = a.list_cnt[2 * i + 1];
     const int32_t *list = layer_list(a, i, 1);
@@ -1825,7 +1833,7 @@ size_t resident_costs_bytes(int64_t d) {
 }
 
 int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, const Layout &Lw, cudaStream_t st,
-                   bool exact_s, bool exact_tables, float *costs, bool build_costs) {
+                   bool exact_s, bool exact_tables, float *costs, bool build_costs, bool test_stall) {
     double *dp64 = wsp<double>(ws, Lw.dp64);
     int32_t *bp = wsp<int32_t>(ws, Lw.bp);
     // small inputs, very large ones and huge counts take the reference kernel
@@ -1879,6 +1887,8 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
         a.list_cnt = reinterpret_cast<int *>(q);
     }
     a.mdp_stride = mdp_stride(s);
+    a.spin_limit = test_stall ? kTestSpinLimit : kSpinLimit;
+    a.hold0 = test_stall ? 1 : 0;
     a.prune = (costs && a.lgc == 2 && a.mdp_stride <= 20) ? 1 : 0;
     a.costs = costs;
     if (costs) {

@@ -109,12 +109,14 @@ __global__ void k_traceback_eval(Prefix P, int G, int s, int exact_s, const doub
         } else {
             int64_t j = jstar;
             a[istar - 1] = (int32_t)j;
-            for (int i = istar; i >= 3; i--) {
+            bool ok = true;  // every output on the path carries a backpointer (not so after a timed-out wait)
+            for (int i = istar; i >= 3 && ok; i--) {
                 j = bp[dp_at(g, i, j, s, P.ps)];
+                ok = j >= 0;
                 a[i - 2] = (int32_t)j;
             }
-            a[0] = bp[dp_at(g, 2, j, s, P.ps)];
-            sm_m = istar;
+            if (ok) a[0] = bp[dp_at(g, 2, j, s, P.ps)];
+            sm_m = (ok && a[0] >= 0) ? istar : 0;
         }
         metrics[4 * g + 0] = best;
         mcount[g] = sm_m;

@@ -18,6 +18,7 @@ from . import build as _build
 
 OK, EINVAL, ENONFINITE, EINFEASIBLE, EWORKSPACE, ECUDA, ETIMEOUT, ERANGE = 0, -1, -2, -3, -4, -5, -6, -7
 EXACT_S, NO_REFINE_GUARD, DP_REFERENCE, TIME_KERNELS, EXACT_TABLES, RESIDENT_COSTS = 1, 2, 4, 8, 16, 32
+TEST_STALL = 1 << 30  # test hook of the bounded waits (include/ecasq.h)
 
 _lock = threading.Lock()
 _lib = None
@@ -392,9 +393,13 @@ def ecasq_quantize(x, Q, seed, ws=None, idx=None, counts=None):
     if ws is None:
         ws = torch.empty(256, dtype=torch.uint8, device="cuda")
     if idx is None:
-        idx = torch.empty(d, dtype=torch.uint8, device="cuda")
+        idx = torch.empty(d, dtype=torch.uint8, device=x.device)
     if counts is None:
-        counts = torch.empty(m, dtype=torch.int32, device="cuda")
+        counts = torch.empty(m, dtype=torch.int32, device=x.device)
+    _out_tensor(idx, d, (torch.uint8,), "ecasq_quantize", "idx")
+    _out_tensor(counts, m, _count_dtypes(), "ecasq_quantize", "counts")
+    if not (idx.device == x.device == counts.device == ws.device):
+        raise EcasqError(EINVAL, "ecasq_quantize: x, idx, counts and ws must be on one device")
     he = C.c_double()
     rc = lib().ecasq_quantize(_ptr(x), d, _ptr(Q), m, C.c_uint64(int(seed) & 0xFFFFFFFFFFFFFFFF), _ptr(idx),
                               _ptr(counts), _ptr(ws), ws.numel(), C.byref(he), _stream())
@@ -402,11 +407,37 @@ def ecasq_quantize(x, Q, seed, ws=None, idx=None, counts=None):
     return idx, counts, he.value
 
 
+def _out_tensor(t, n, dtypes, where, name):
+    """An output buffer the kernel writes through a raw pointer: a contiguous CUDA tensor
+    of one of `dtypes` with at least n elements (else EINVAL before any device work)."""
+    torch = _torch()
+    ok = (isinstance(t, torch.Tensor) and t.is_cuda and t.dtype in dtypes and t.is_contiguous()
+          and t.numel() >= n)
+    if not ok:
+        raise EcasqError(EINVAL, "%s: %s must be a contiguous CUDA tensor of %s with at least %d elements"
+                         % (where, name, "/".join(str(d) for d in dtypes), n))
+    return t
+
+
+def _count_dtypes():
+    torch = _torch()
+    u32 = getattr(torch, "uint32", None)
+    return (torch.int32,) + ((u32,) if u32 is not None else ())
+
+
 def ecasq_quantize_noalloc(x, Q, seed, idx, counts):
     """ecasq_quantize without a workspace; idx (uint8 [d]) and counts (int32 [m])
-    are the caller's device tensors.  Returns the empirical entropy."""
+    are the caller's device tensors, on the device of x.  Returns the empirical entropy."""
+    torch = _torch()
+    where = "ecasq_quantize_noalloc"
+    _out_tensor(idx, 0, (torch.uint8,), where, "idx")
+    _out_tensor(counts, 0, _count_dtypes(), where, "counts")
     x = _dev_f32(x)
     Q = _dev_f32(Q)
+    _out_tensor(idx, x.numel(), (torch.uint8,), where, "idx")
+    _out_tensor(counts, Q.numel(), _count_dtypes(), where, "counts")
+    if not (idx.device == x.device == Q.device == counts.device):
+        raise EcasqError(EINVAL, "%s: x, Q, idx and counts must be on one device" % where)
     he = C.c_double()
     rc = lib().ecasq_quantize_noalloc(_ptr(x), x.numel(), _ptr(Q), Q.numel(),
                                       C.c_uint64(int(seed) & 0xFFFFFFFFFFFFFFFF), _ptr(idx), _ptr(counts),

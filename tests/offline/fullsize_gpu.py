@@ -1,0 +1,108 @@
+"""Full-size check, GPU half: the budgeted solve of a workload at its full size, then one
+pass at the multiplier it selected with every DP output resolved exactly, written out for
+the oracle half (fullsize_oracle.py) to compare with the oracle's own DP.
+
+    python tests/offline/fullsize_gpu.py studentt_d131072_s16 mixture_d1048576_s32 --out gpurun_out/fullsize
+
+For each workload it writes <name>.json (the solve: multiplier, codebook, metrics, timings)
+and <name>.npz (the exactly resolved dp / bp tables of that pass: every output when they fit
+in --max-mb, else every output of the layers' rows j = 0 (mod stride), of column p - 1 and of
+the traced path).  Nothing here reads the oracle.
+"""
+import argparse
+import json
+import os
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+
+def run(name, out_dir, max_mb):
+    import torch
+    import paper_2608_18147_gb300 as E
+    from paper_2608_18147_gb300 import workloads
+    cfg = workloads.CONFIGS[name]
+    x_np = workloads.make(name, 0)
+    s, budget = cfg["s"], cfg["budgets"][0]
+    x = torch.as_tensor(x_np).cuda()
+    d = x.numel()
+    flags = E.TIME_KERNELS
+    need = E.ecasq_workspace_size_flags(d, s, 1, E.RESIDENT_COSTS)
+    if 0 < need <= 0.6 * torch.cuda.mem_get_info()[0]:
+        flags |= E.RESIDENT_COSTS
+    ws = E.workspace(d, s, flags=flags)
+    stream = torch.cuda.current_stream()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    ev0.record(stream)
+    Q, res = E.ecasq_solve(x, s, budget_bits=budget, ws=ws, flags=flags)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - t0
+    solve_ms = ev0.elapsed_time(ev1)
+    st = E.native.ws_status(ws)
+    lam = res["lambda"]
+    # the selected multiplier once more, every output resolved exactly
+    ev0.record(stream)
+    Q2, m2, met2 = E.ecasq_dp_pass(x, s, [lam], flags=flags | E.EXACT_TABLES, ws=ws)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    pass_ms = ev0.elapsed_time(ev1)
+    st2 = E.native.ws_status(ws)
+    p = st2["p"]
+    dp, bp = E.ecasq_dp_tables(ws, 0, s, d)
+    dp = dp.cpu().numpy()
+    bp = bp.cpu().numpy()
+    m = int(res["m"])
+    q_solve = Q.cpu().numpy()
+    q_pass = Q2[0, :m2[0]].cpu().numpy()
+    v = E.ecasq_prepare(x)["v"].cpu().numpy()
+    a = np.searchsorted(v, q_pass)
+    full_mb = dp.nbytes / 2 ** 20 + bp.nbytes / 2 ** 20
+    if full_mb <= max_mb:
+        sel = None
+        np.savez_compressed(os.path.join(out_dir, name + ".npz"), dp=dp, bp=bp)
+    else:
+        stride = int(np.ceil(full_mb / max_mb))
+        cols = np.unique(np.concatenate([np.arange(0, p, stride), [p - 1], a]))
+        sel = stride
+        np.savez_compressed(os.path.join(out_dir, name + ".npz"), cols=cols, dp=dp[:, cols], bp=bp[:, cols])
+    meta = dict(workload=name, d=d, p=p, s=s, budget_bits=budget, flags=flags, lam=lam,
+                lam_prime=res["lambda_prime"], norm2=res["norm2"], m=m, Q=[float(t) for t in q_solve],
+                pass_Q=[float(t) for t in q_pass], pass_m=int(m2[0]), pass_metrics=[float(t) for t in met2[0]],
+                mse=res["mse"], h_surrogate=res["h_surrogate"], h_exact=res["h_exact"], passes=res["passes"],
+                lambdas_evaluated=res["lambdas_evaluated"], candidates=res["candidates"],
+                solve_ms=solve_ms, solve_wall_s=wall, dp_kernel_ms=res["dp_kernel_ms"],
+                dp_kernel_launches=res["dp_kernel_launches"], exact_pass_ms=pass_ms,
+                cand_per_s=res["candidates"] / (res["dp_kernel_ms"] / 1000.0) if res["dp_kernel_ms"] else None,
+                status_solve=dict(timeout=st["timeout"], bound_viol=st["bound_viol"], rescored=st["rescored"]),
+                status_exact=dict(timeout=st2["timeout"], bound_viol=st2["bound_viol"], rescored=st2["rescored"]),
+                column_stride=sel, gpu=torch.cuda.get_device_name())
+    with open(os.path.join(out_dir, name + ".json"), "w") as f:
+        json.dump(meta, f, indent=1)
+    print(json.dumps({k: meta[k] for k in ("workload", "lam", "m", "mse", "h_surrogate", "solve_ms", "passes",
+                                            "lambdas_evaluated", "dp_kernel_ms", "cand_per_s", "exact_pass_ms")}),
+          flush=True)
+    del ws
+    torch.cuda.empty_cache()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("workloads", nargs="+")
+    ap.add_argument("--out", default="gpurun_out/fullsize")
+    ap.add_argument("--max-mb", type=float, default=24.0)
+    args = ap.parse_args()
+    os.makedirs(args.out, exist_ok=True)
+    for name in args.workloads:
+        run(name, args.out, args.max_mb)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,115 @@
+"""Full-size check, oracle half: the CPU oracle's approximate DP (Sec. 5, eqs. apx_base,
+apx_rec, apx_final) at the multiplier the GPU's budgeted solve selected, over the whole
+input, compared with what fullsize_gpu.py wrote.
+
+    python tests/offline/fullsize_oracle.py gpurun_out/fullsize/studentt_d131072_s16.json
+
+The oracle runs or_apx_dp_columns (each pair's link cost computed once for all layers;
+the same tables as or_apx_dp) on this host's OpenMP threads.  Checks, with the parity
+bar of the GPU tests:
+  * every exactly resolved GPU output the file holds: dp within 1e-12 relative of the
+    oracle's, the same backpointer unless the oracle's best two candidates are within
+    1e-9 relative (then the GPU's choice, re-scored by the oracle, is within 1e-9 of the
+    minimum);
+  * the codebook and m equal the oracle's, unless a decision on the oracle's traced path
+    had a margin under 1e-9 (then the two objectives agree within 1e-9);
+  * MSE, H(I,B) and H(Xhat) of the GPU's codebook, evaluated by the oracle, within 1e-9
+    relative of the GPU's own figures, and H(I,B) within the budget.
+Writes <name>.report.json next to the input (or to --out) and prints it.
+"""
+import argparse
+import json
+import os
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
+for p in (ROOT, os.path.join(ROOT, "tests")):
+    if p not in sys.path:
+        sys.path.insert(0, p)
+
+TIE = 1e-9
+DP_RTOL = 1e-12
+MET_RTOL = 1e-9
+
+
+def check(meta_path, out_dir=None):
+    import oracle
+    from paper_2608_18147_gb300 import workloads
+    meta = json.load(open(meta_path))
+    tables = np.load(meta_path[:-len(".json")] + ".npz")
+    name, s = meta["workload"], meta["s"]
+    x = workloads.make(name, 0)
+    oracle.build()
+    t0 = time.perf_counter()
+    H = oracle.Hist(x)
+    assert H.p == meta["p"], (H.p, meta["p"])
+    lp = meta["lam"] * H.norm2
+    r = H.apx_dp(s, lp, columns=True)
+    wall = time.perf_counter() - t0
+    dp_o, bp_o, mg_o = r["dp"], r["bp"], r["margin"]
+    cols = tables["cols"] if "cols" in tables.files else np.arange(H.p)
+    dp_g, bp_g = tables["dp"], tables["bp"]
+    rep = dict(workload=name, d=int(x.size), p=int(H.p), s=s, lam=meta["lam"], oracle_wall_s=wall,
+               oracle_threads=oracle.num_threads(), oracle_host=os.uname().machine,
+               outputs_compared=0, dp_max_rel=0.0, bp_mismatch=0, bp_mismatch_near_tie=0, bp_invalid=0)
+    for i in range(2, s + 1):
+        o, g = dp_o[i, cols], dp_g[i]
+        fin = np.isfinite(o)
+        assert np.array_equal(fin, np.isfinite(g)), "finite pattern differs at layer %d" % i
+        rel = np.abs(g[fin] - o[fin]) / np.maximum(np.abs(o[fin]), 1e-300)
+        rep["dp_max_rel"] = max(rep["dp_max_rel"], float(rel.max()) if rel.size else 0.0)
+        rep["outputs_compared"] += int(fin.sum())
+        diff = np.nonzero(fin & (bp_o[i, cols] != bp_g[i]))[0]
+        for t in diff:
+            j = int(cols[t])
+            rep["bp_mismatch"] += 1
+            if mg_o[i, j] < TIE:
+                rep["bp_mismatch_near_tie"] += 1
+                k = int(bp_g[i][t])
+                v = H.dp_candidate(dp_o[i - 1, k], k, j, lp)
+                if not (0 <= k < j and v <= dp_o[i, j] * (1 + TIE)):
+                    rep["bp_invalid"] += 1
+            else:
+                rep["bp_invalid"] += 1
+    v = H.arrays()["v"]
+    a_gpu = np.searchsorted(v, np.float32(meta["Q"]))
+    a_pass = np.searchsorted(v, np.float32(meta["pass_Q"]))
+    rep["codebook_equal"] = bool(np.array_equal(a_gpu, r["Q_idx"]))
+    rep["pass_codebook_equal_solve"] = bool(np.array_equal(a_gpu, a_pass))
+    rep["m_gpu"], rep["m_oracle"] = int(meta["m"]), int(r["m"])
+    # margins of the decisions on the oracle's traced path
+    path = r["Q_idx"]
+    rep["path_min_margin"] = float(min([mg_o[i, path[i - 1]] for i in range(3, r["m"] + 1)] or [np.inf]))
+    mse, hs, hx = H.eval_idx(a_gpu)
+    rep["metrics_oracle_of_gpu_codebook"] = [mse, hs, hx]
+    rep["metrics_gpu"] = [meta["mse"], meta["h_surrogate"], meta["h_exact"]]
+    rep["metrics_max_rel"] = max(abs(a - b) / abs(b) for a, b in zip(rep["metrics_gpu"], [mse, hs, hx]) if b)
+    rep["objective_oracle"] = r["best"]
+    rep["objective_of_gpu_codebook"] = mse + lp * hs
+    rep["objective_rel"] = abs(rep["objective_of_gpu_codebook"] - r["best"]) / abs(r["best"])
+    rep["feasible"] = bool(hs <= meta["budget_bits"])
+    ok = (rep["dp_max_rel"] <= DP_RTOL and rep["bp_invalid"] == 0 and rep["metrics_max_rel"] <= MET_RTOL
+          and rep["feasible"] and rep["pass_codebook_equal_solve"]
+          and (rep["codebook_equal"] or (rep["path_min_margin"] < TIE and rep["objective_rel"] <= TIE)))
+    rep["pass"] = bool(ok)
+    out = os.path.join(out_dir or os.path.dirname(meta_path), name + ".report.json")
+    with open(out, "w") as f:
+        json.dump(rep, f, indent=1)
+    print(json.dumps(rep), flush=True)
+    return ok
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("meta", nargs="+")
+    ap.add_argument("--out", default=None)
+    args = ap.parse_args()
+    ok = all([check(m, args.out) for m in args.meta])
+    sys.exit(0 if ok else 1)
+
+
+if __name__ == "__main__":
+    main()

@@ -98,3 +98,22 @@ def test_product_path_does_not_touch_the_oracle():
                     txt = fh.read()
                 assert "import oracle" not in txt and "from oracle" not in txt, f
                 assert "ecasq_oracle" not in txt and "liboracle" not in txt, f
+
+
+def test_quantize_wrappers_refuse_host_output_buffers():
+    """The bindings pass idx and counts to the kernel as raw device pointers, so they
+    refuse anything that is not a CUDA tensor of the right type (EINVAL) before any call
+    into the library or any device work."""
+    import numpy as np
+    import torch
+    from paper_2608_18147_gb300 import native
+    x = np.linspace(-1.0, 1.0, 64, dtype=np.float32)
+    Q = np.float32([-1.0, 0.0, 1.0])
+    cases = [(np.zeros(64, np.uint8), np.zeros(3, np.int32)),
+             (torch.zeros(64, dtype=torch.uint8), torch.zeros(3, dtype=torch.int32)),
+             (torch.zeros(64, dtype=torch.int64), torch.zeros(3, dtype=torch.int32)),
+             (None, None)]
+    for idx, cnt in cases:
+        with pytest.raises(native.EcasqError) as ei:
+            native.ecasq_quantize_noalloc(x, Q, 0, idx, cnt)
+        assert ei.value.code == native.EINVAL

@@ -38,3 +38,17 @@ def test_opt_candidates_is_the_recurrence_count(n, s, nL):
     import bench
     assert bench.opt_candidates(n, s, 1, nL) == _opt_candidates(n, s, nL)
     assert bench.opt_candidates(n, s, 3, nL) == 3 * _opt_candidates(n, s, nL)
+
+
+@pytest.mark.parametrize("p,s,G", [(64, 16, 8), (130, 5, 7), (131072, 16, 43)])
+def test_executed_candidates_counts_tile_units_and_diagonal_triangles(p, s, G):
+    """bench.py's executed count: every 64 x 64 off-diagonal tile unit the kernel ran,
+    over the s - 2 layers, plus one 64-column triangle (pairs k < j) per column block
+    and multiplier."""
+    import bench
+    L = s - 2
+    blocks = -(-p // 64)
+    tri = sum(1 for j in range(64) for k in range(j))
+    assert bench.executed_candidates({"tiles_run": 0}, p, s, G) == G * blocks * tri * L
+    assert (bench.executed_candidates({"tiles_run": 5}, p, s, G)
+            - bench.executed_candidates({"tiles_run": 0}, p, s, G)) == 5 * 64 * 64 * L

@@ -193,3 +193,36 @@ def test_decision_ties_take_lowest_k(oracle_mod):
             assert (b, a) == (best, min(winners))
             assert (r["dp"][i, j], r["bp"][i, j]) == (best, min(winners))
     assert ties > 0
+
+
+@pytest.mark.parametrize("name,x", _inputs() + [("tiny", np.float32([0.5, -1.0, 2.0])),
+                                                ("single", np.float32([1.0, 1.0]))])
+@pytest.mark.parametrize("s", [2, 3, 8, 16])
+def test_column_order_equals_layer_order(oracle_mod, name, x, s):
+    """or_apx_dp_columns (each pair's link cost computed once for all layers) returns
+    or_apx_dp's tables, codebook and optimum bit for bit: the recurrence of eq. apx_rec
+    does not depend on the order its outputs are visited in."""
+    for grid in (None, "grid"):
+        g = None
+        if grid:
+            lo, hi = float(x.min()), float(x.max())
+            g = np.unique(np.concatenate([np.linspace(lo - 0.5, hi + 0.5, 40).astype(np.float32),
+                                          np.float32([lo, hi])]))
+        H = oracle_mod.Hist(x, g)
+        for lam in (0.0, 0.01, 1.5):
+            lp = lam * H.norm2
+            for exact_s in (False, True):
+                if exact_s and s > H.p > 1:  # exactly s values do not exist: both report it
+                    for cols in (False, True):
+                        with pytest.raises(oracle_mod.OracleError) as e:
+                            H.apx_dp(s, lp, exact_s=True, columns=cols)
+                        assert e.value.code == oracle_mod.EINFEASIBLE
+                    continue
+                a = H.apx_dp(s, lp, exact_s=exact_s)
+                b = H.apx_dp(s, lp, exact_s=exact_s, columns=True)
+                assert a["m"] == b["m"] and a["best"] == b["best"]
+                assert np.array_equal(a["Q_idx"], b["Q_idx"])
+                if H.p > 1:
+                    assert np.array_equal(a["dp"], b["dp"])
+                    assert np.array_equal(a["bp"], b["bp"])
+                    assert np.array_equal(a["margin"], b["margin"])

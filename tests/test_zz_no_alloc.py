@@ -66,8 +66,10 @@ def test_noalloc_error_flag_starts_at_zero_on_every_call(E):
 
 
 def test_noalloc_takes_no_device_memory(E):
-    """After the first call on the device (set-up), further calls leave the
-    device's free memory unchanged."""
+    """After the first call on the device (set-up), further calls make no allocation
+    through torch's allocator and take no device memory of their own: a cudaMalloc
+    reserves at least a 2 MiB page, so the device's free memory may move by less than
+    that (other users of the GPU) but must not drop by a page."""
     import torch
     x, Q = _case(1 << 16, 13)
     xg = torch.as_tensor(x).cuda()
@@ -76,11 +78,42 @@ def test_noalloc_takes_no_device_memory(E):
     cnt = torch.empty(Qg.numel(), dtype=torch.int32, device="cuda")
     E.ecasq_quantize_noalloc(xg, Qg, 0, idx, cnt)
     torch.cuda.synchronize()
+    n_alloc0 = torch.cuda.memory_stats().get("allocation.all.allocated", 0)
+    reserved0 = torch.cuda.memory_reserved()
     free0 = torch.cuda.mem_get_info()[0]
     for seed in (1, 2):
         E.ecasq_quantize_noalloc(xg, Qg, seed, idx, cnt)
     torch.cuda.synchronize()
-    assert torch.cuda.mem_get_info()[0] == free0
+    assert torch.cuda.memory_stats().get("allocation.all.allocated", 0) == n_alloc0
+    assert torch.cuda.memory_reserved() == reserved0
+    assert free0 - torch.cuda.mem_get_info()[0] < 2 * 2 ** 20
+
+
+def test_noalloc_rejects_bad_output_buffers_before_launch(E):
+    """idx and counts are written through raw pointers: a buffer that is too short, of
+    the wrong type, not contiguous or on the host is refused (EINVAL) and left untouched."""
+    import torch
+    x, Q = _case(4096, 21)
+    xg = torch.as_tensor(x).cuda()
+    Qg = torch.as_tensor(Q).cuda()
+    m = Qg.numel()
+    good_idx = torch.full((x.size,), 7, dtype=torch.uint8, device="cuda")
+    good_cnt = torch.full((m,), 7, dtype=torch.int32, device="cuda")
+    bad = [
+        (torch.empty(x.size - 1, dtype=torch.uint8, device="cuda"), good_cnt),           # idx too short
+        (good_idx, torch.empty(m - 1, dtype=torch.int32, device="cuda")),                # counts too short
+        (torch.empty(x.size, dtype=torch.int32, device="cuda"), good_cnt),               # idx not uint8
+        (good_idx, torch.empty(m, dtype=torch.float32, device="cuda")),                  # counts not int32
+        (torch.empty(2 * x.size, dtype=torch.uint8, device="cuda")[::2], good_cnt),      # idx strided
+        (torch.empty(x.size, dtype=torch.uint8), good_cnt),                              # idx on the host
+        (good_idx, torch.empty(m, dtype=torch.int32)),                                   # counts on the host
+    ]
+    for idx, cnt in bad:
+        with pytest.raises(E.EcasqError) as ei:
+            E.ecasq_quantize_noalloc(xg, Qg, 1, idx, cnt)
+        assert ei.value.code == E.native.EINVAL
+    torch.cuda.synchronize()
+    assert bool((good_idx == 7).all()) and bool((good_cnt == 7).all())
 
 
 def test_noalloc_rejects_sizes_beyond_its_limits(E):
