@@ -71,6 +71,8 @@ def parse():
     ap.add_argument("--mode", default="solve", choices=["solve", "grid", "timeshare", "opt", "hbm", "rows", "pass"])
     ap.add_argument("--lambdas", default="0.02", help="comma-separated multipliers (vNMSE scale) for --mode pass")
     ap.add_argument("--grid", type=int, default=256, help="grid size for --mode grid")
+    ap.add_argument("--prefix", type=int, default=0,
+                    help="--mode pass: use only the first N entries of the configuration's vector")
     return ap.parse_args()
 
 
@@ -397,6 +399,8 @@ def run_pass_mode(args, cfg, x_np):
     import paper_2608_18147_gb300 as E
     s = cfg["s"]
     lams = [float(t) for t in args.lambdas.split(",")]
+    if args.prefix > 0:
+        x_np = x_np[:args.prefix]
     x = torch.as_tensor(x_np).cuda()
     d = x.numel()
     flags = 0
@@ -412,9 +416,13 @@ def run_pass_mode(args, cfg, x_np):
     out = {"metric": "ECASQ DP pass: candidate evals/s", "value": args.steps * cand / (ms / 1000.0),
            "unit": UNIT, "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
            "higher_is_better": True, "vs_baseline": None, "dtype": "f32 (fp64 exact stage)", "data": "synthetic",
-           "config": {"workload": args.config, "mode": "pass", "d": d, "p": p, "s": s, "lambdas": lams,
+           "config": {"workload": args.config + (" (first %d entries)" % d if args.prefix > 0 else ""),
+                      "mode": "pass", "d": d, "p": p, "s": s, "lambdas": lams,
                       "resident_costs": bool(flags & E.RESIDENT_COSTS)},
-           "status": {"timeout": st["timeout"], "bound_viol": st["bound_viol"], "rescored": st["rescored"]},
+           "status": {"timeout": st["timeout"], "bound_viol": st["bound_viol"], "rescored": st["rescored"],
+                      "tile_units_run": st["tiles_run"], "tile_units_skipped": st["tiles_skipped"],
+                      "cost_tiles_fetched": st["tiles_fetched"],
+                      "executed_candidates": executed_candidates(st, p, s, len(lams))},
            "m": list(outs[-1][1]), "gpu_launches": E.ecasq_kernel_launches() - launches0, "clocks": clocks}
     print(json.dumps(out), flush=True)
 
@@ -499,7 +507,9 @@ def main():
         torch.cuda.synchronize()
 
     s, budget = cfg["s"], cfg["budgets"][0]
-    refine_rounds = 50 if cfg.get("refine") else 0
+    # the stop rule of Sec. 6 (a round lowering J by at most refine_tol relative) ends the
+    # refinement; the cap is only a safeguard (Student-t d = 2^17 stops after about 90 rounds)
+    refine_rounds = 500 if cfg.get("refine") else 0
     refine_tol = cfg.get("refine_tol", 0.0)
     d = x_np.size
     x = torch.as_tensor(x_np).cuda()
@@ -627,7 +637,9 @@ def main():
                "solve": {"m": last["m"], "lambda": last["lambda"], "vnmse": last["vnmse"],
                          "h_surrogate": last["h_surrogate"], "h_exact": last["h_exact"],
                          "passes": last["passes"], "lambdas_evaluated": last["lambdas_evaluated"],
-                         "refine_rounds": last["refine_rounds"], "candidates_per_solve": last["candidates"],
+                         "refine_rounds": last["refine_rounds"], "refine_last_rel": last["refine_last_rel"],
+                         "refine_stopped_by_rule": last["refine_rounds"] < refine_rounds,
+                         "candidates_per_solve": last["candidates"],
                          "rescored_per_solve": last["rescored"], "dp_pass_ms": dp_ms / max(dp_launches, 1),
                          "tile_units_run": st["tiles_run"], "tile_units_skipped": st["tiles_skipped"],
                          "cost_tiles_fetched": st["tiles_fetched"],

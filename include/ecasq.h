@@ -57,6 +57,11 @@ typedef struct CUstream_st *ecasq_stream_t; /* same type as cudaStream_t */
 #define ECASQ_RESIDENT_COSTS 32u  /* fast DP: compute the lambda-independent interval costs C and Phi (Sec. 5, App. E)
                                      once per call into the workspace and stream them to every pass (workspace:
                                      ecasq_workspace_size_flags with this flag; about 4.3 d^2 bytes extra) */
+#define ECASQ_STREAMED_COSTS 64u  /* fast DP, for inputs whose full table does not fit: the interval-cost tiles of a
+                                     band of column blocks at a time are built into a bounded buffer (about 64 columns
+                                     of tiles, 2.3 MB x ceil(d / 64); ecasq_workspace_size_flags with this flag) and
+                                     the wavefront runs band by band; rebuilt in every pass.  RESIDENT_COSTS wins
+                                     when both are given.  Results are the same as with either other mode. */
 #define ECASQ_TEST_STALL (1u << 30) /* test hook for the bounded device waits: column block 0 of the fast DP's
                                      wavefront is never published and the flag waits give up after 2^14 spins, so
                                      the call must return ECASQ_ETIMEOUT (nothing else) and leave the workspace
@@ -96,6 +101,8 @@ typedef struct ecasq_result {
     double dp_kernel_ms;       /* with ECASQ_TIME_KERNELS: summed duration of the min-plus kernel launches */
     int32_t dp_kernel_launches;/* with ECASQ_TIME_KERNELS: number of those launches */
     int32_t reserved2;
+    double refine_last_rel;    /* (J_before - J_after) / |J_before| of the last refinement round (Sec. 6), 0 without
+                                  refinement: at most refine_rel_tol when the stop rule ended it */
 } ecasq_result_t;
 
 /* Two-way time-sharing (Sec. 7): the mixture of the budgeted solution Q- (rate

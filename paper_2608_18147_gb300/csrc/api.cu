@@ -16,8 +16,10 @@ namespace ecasq {
 int launch_dp_reference(const Prefix &P, const double *lamp, int G, int s, double *dp64, int32_t *bp,
                         cudaStream_t st);
 int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, const Layout &L, cudaStream_t st,
-                   bool exact_s, bool exact_tables, float *costs, bool build_costs, bool test_stall);
+                   bool exact_s, bool exact_tables, float *costs, bool build_costs, bool test_stall,
+                   size_t chunk_bytes);
 size_t resident_costs_bytes(int64_t d);
+size_t streamed_costs_bytes(int64_t d);
 int launch_rows_prepare(const float *X, int64_t rows, const RowsData &R, cudaStream_t st);
 int launch_grid_prefix(const float *P, int64_t n, const float *vX, const int64_t *NX, const double *SX,
                        const double *S2X, int64_t pX, float *v, int64_t *w, int64_t *N, double *S, double *S2,
@@ -108,6 +110,7 @@ size_t make_layout(int64_t d, int32_t s, int64_t rows, Layout *L) {
     L->band = take(fast_dp_band_bytes(d, s));
     L->costs = 0;
     L->costs_bytes = 0;
+    L->costs_streamed = false;
     L->gpairs = 0;
     L->gpairs_bytes = 0;
     L->total = off;
@@ -219,13 +222,16 @@ static size_t rows_region_bytes(int64_t d, int32_t s, int64_t rows) {
     return rows_layout(d, s, rows, &R);
 }
 
-// ECASQ_RESIDENT_COSTS: the interval-cost tiles follow the common layout.
+// ECASQ_RESIDENT_COSTS: the interval-cost tiles follow the common layout;
+// ECASQ_STREAMED_COSTS (without RESIDENT): a buffer for one band of tiles there instead.
 static int add_resident_costs(uint32_t flags, Layout *L) {
-    if (!(flags & ECASQ_RESIDENT_COSTS)) return ECASQ_OK;
-    size_t cb = resident_costs_bytes(L->d);
+    if (!(flags & (ECASQ_RESIDENT_COSTS | ECASQ_STREAMED_COSTS))) return ECASQ_OK;
+    const bool streamed = !(flags & ECASQ_RESIDENT_COSTS);
+    size_t cb = streamed ? streamed_costs_bytes(L->d) : resident_costs_bytes(L->d);
     if (!cb || L->total > SIZE_MAX - align256(cb)) return ECASQ_EINVAL;
     L->costs = L->total;
     L->costs_bytes = cb;
+    L->costs_streamed = streamed;
     L->total += align256(cb);
     return ECASQ_OK;
 }
@@ -283,8 +289,10 @@ static int dp_pass_prepared(void *ws, const Layout &L, const Prefix &P, int s, c
         if (rc == ECASQ_OK) *costs_built = true;
     } else {
         float *costs = L.costs_bytes ? wsp<float>(ws, L.costs) : nullptr;
+        // streamed costs are rebuilt band by band in every pass
         rc = launch_dp_fast(P, lamp, G, s, ws, L, st, (flags & ECASQ_EXACT_S) != 0, (flags & ECASQ_EXACT_TABLES) != 0,
-                            costs, costs && !*costs_built, (flags & ECASQ_TEST_STALL) != 0);
+                            costs, costs && (L.costs_streamed || !*costs_built), (flags & ECASQ_TEST_STALL) != 0,
+                            L.costs_streamed ? L.costs_bytes : 0);
         if (costs && rc == ECASQ_OK) *costs_built = true;
     }
     if (rc != ECASQ_OK) return rc;
@@ -341,9 +349,11 @@ static int eval_device(void *ws, const Layout &L, const Prefix &P, const int32_t
 
 // Three-colour refinement loop (Sec. 6) on the host; a_host in/out.
 static int refine_device(void *ws, const Layout &L, const Prefix &P, std::vector<int32_t> &a_host, double lamp,
-                         double budget, bool guard, int max_rounds, double tol, cudaStream_t st, int *rounds_used) {
+                         double budget, bool guard, int max_rounds, double tol, cudaStream_t st, int *rounds_used,
+                         double *last_rel = nullptr) {
     int m = (int)a_host.size();
     *rounds_used = 0;
+    if (last_rel) *last_rel = 0.0;
     if (m < 3 || max_rounds <= 0) return ECASQ_OK;
     int32_t *a = wsp<int32_t>(ws, L.refine);
     int32_t *an = a + kMaxS;
@@ -377,6 +387,7 @@ static int refine_device(void *ws, const Layout &L, const Prefix &P, std::vector
         if (rc != ECASQ_OK) return rc;
         J = ev[0] + lamp * ev[2];
         *rounds_used = r + 1;
+        if (last_rel) *last_rel = J0 != 0.0 ? (J0 - J) / fabs(J0) : 0.0;
         if (!(J0 - J > tol * fabs(J0))) break;
     }
     ECASQ_CUDA_TRY(cudaMemcpyAsync(a_host.data(), a, sizeof(int32_t) * m, cudaMemcpyDeviceToHost, st));
@@ -439,8 +450,8 @@ size_t ecasq_workspace_size(int64_t d, int32_t s, int64_t rows) {
 
 size_t ecasq_workspace_size_flags(int64_t d, int32_t s, int64_t rows, uint32_t flags) {
     size_t base = ecasq_workspace_size(d, s, rows);
-    if (!base || !(flags & ECASQ_RESIDENT_COSTS)) return base;
-    size_t cb = resident_costs_bytes(d);
+    if (!base || !(flags & (ECASQ_RESIDENT_COSTS | ECASQ_STREAMED_COSTS))) return base;
+    size_t cb = (flags & ECASQ_RESIDENT_COSTS) ? resident_costs_bytes(d) : streamed_costs_bytes(d);
     if (!cb || base > SIZE_MAX - align256(cb)) return 0;
     return base + align256(cb);
 }
@@ -682,10 +693,11 @@ static int solve_prepared(void *ws, const Layout &L, const Prefix &P, int64_t d,
     double lam = sel->lam;
     double lamp = lam * n2;
     int rr = 0;
+    double last_rel = 0.0;
     if (status == ECASQ_OK && prm->refine_max_rounds > 0 && (int)a.size() >= 3) {
         bool guard = prm->lambda < 0.0 && !(prm->flags & ECASQ_NO_REFINE_GUARD);
         rc = refine_device(ws, L, P, a, lamp, prm->budget_bits, guard, prm->refine_max_rounds, prm->refine_rel_tol,
-                           st, &rr);
+                           st, &rr, &last_rel);
         if (rc) return rc;
     }
     rc = write_codebook(ws, L, a, Q, st);
@@ -695,7 +707,11 @@ static int solve_prepared(void *ws, const Layout &L, const Prefix &P, int64_t d,
     if (rc) return rc;
     double obj = prm->refine_max_rounds > 0 ? ev[0] + lamp * ev[2] : ev[0] + lamp * ev[1];
     fill_result(res, status, (int)a.size(), d, p, lam, n2, ev, obj, passes, nlam, rr, cand, read_rescored(ws, st));
-    if (res) { res->dp_kernel_ms = g_timer.ms; res->dp_kernel_launches = g_timer.launches; }
+    if (res) {
+        res->dp_kernel_ms = g_timer.ms;
+        res->dp_kernel_launches = g_timer.launches;
+        res->refine_last_rel = last_rel;
+    }
     g_timer.on = false;
     return status;
 }
@@ -910,7 +926,8 @@ int ecasq_refine(const float *x, int64_t d, float *Q, int32_t m, double lambda, 
     double lamp = lambda * n2;
     bool guard = budget_bits >= 0.0 && !(flags & ECASQ_NO_REFINE_GUARD);
     int rr = 0;
-    rc = refine_device(ws, L, P, a, lamp, budget_bits, guard, max_rounds, rel_tol, st, &rr);
+    double last_rel = 0.0;
+    rc = refine_device(ws, L, P, a, lamp, budget_bits, guard, max_rounds, rel_tol, st, &rr, &last_rel);
     if (rc) return rc;
     rc = write_codebook(ws, L, a, Q, st);
     if (rc) return rc;
@@ -918,6 +935,7 @@ int ecasq_refine(const float *x, int64_t d, float *Q, int32_t m, double lambda, 
     rc = eval_device(ws, L, P, wsp<int32_t>(ws, L.qidx), m, st, ev);
     if (rc) return rc;
     fill_result(res, ECASQ_OK, m, d, p, lambda, n2, ev, ev[0] + lamp * ev[2], 0, 0, rr, 0, 0);
+    if (res) res->refine_last_rel = last_rel;
     return ECASQ_OK;
 }
 

@@ -76,6 +76,7 @@ struct Layout {
     size_t band;           // fast DP band lists
     size_t costs;          // resident interval-cost tiles (ECASQ_RESIDENT_COSTS), after everything else
     size_t costs_bytes;    // 0 when absent
+    bool costs_streamed;   // ECASQ_STREAMED_COSTS: the costs region holds one band of tiles at a time
     size_t gpairs;         // grid DP pair cache (permissible sets up to kGridPairsMax values)
     size_t gpairs_bytes;   // 0 when absent
     size_t total;

@@ -132,8 +132,10 @@ struct FastArgs {
     int32_t *members;      // [G][s+1][ps][NMEM]
     uint8_t *need;         // [G][s+1][ps] output resolved exactly
     float *corner;         // [nJ(nJ-1)/2][8]: state of pair (64K+63, 64J), K < J (N, E, Ec, A, Ac, C, Cc)
-    const float *costs;    // resident interval costs (tile (K, J) at J(J+1)/2 + K), or null: computed per tile
+    const float *costs;    // resident interval costs (tile (K, J) at J(J+1)/2 + K - tile_base), or null
     float2 *tsum;          // with costs: per tile, {min_k C, min_k Phi} of its 64 columns (the rows' padding)
+    size_t tile_base;      // index of the first tile the costs hold: 0, or J0(J0+1)/2 for a band of blocks
+    int J0, J1;            // the wavefront's column blocks [J0, J1): all of them, or one band (streamed costs)
     int32_t *lists;        // [s+1][2][G ps]: needed outputs of layer i (g << 24 | j); 0: <= NMEM members, 1: more
     int *list_cnt;         // [s+1][2]
     float *mdp;            // [nJ][G][mdp_stride]: min over the block's 64 columns of dp32(g, i, .)
@@ -584,8 +586,9 @@ struct __align__(16) BuildSmem {
 __global__ void __launch_bounds__(NPROD) k_build_costs(FastArgs a, float *costs) {
     __shared__ BuildSmem S;
     const int jl = threadIdx.x;
-    const int64_t ntiles = (int64_t)a.nJ * (a.nJ + 1) / 2;
-    int64_t t = blockIdx.x;
+    // the tiles of column blocks [J0, J1): indices J0(J0+1)/2 .. J1(J1+1)/2 - 1, stored from tile_base
+    const int64_t ntiles = (int64_t)a.J1 * (a.J1 + 1) / 2;
+    int64_t t = (int64_t)a.tile_base + blockIdx.x;
     if (t >= ntiles) return;
     // invert t = J(J+1)/2 + K, K <= J
     int64_t J = (int64_t)((sqrt(8.0 * (double)t + 1.0) - 1.0) * 0.5);
@@ -611,11 +614,11 @@ __global__ void __launch_bounds__(NPROD) k_build_costs(FastArgs a, float *costs)
         if (jl == 0) bulk_wait_read_all();  // the previous tile's bulk store has read the rows
         bar_sync(BAR_PROD, NPROD);
         tile_rows(a, K, J, jl, anchor_r, cur.vj, S.kv, S.kw, S.kd, S.C, S.Phi);
-        a.tsum[(size_t)t * BJ + jl] = make_float2(S.C[jl][BK], S.Phi[jl][BK]);  // this thread's own row
+        a.tsum[((size_t)t - a.tile_base) * BJ + jl] = make_float2(S.C[jl][BK], S.Phi[jl][BK]);  // this thread's own row
         fence_proxy_async_smem();
         bar_sync(BAR_PROD, NPROD);
         if (jl == 0) {
-            float *dst = costs + (size_t)t * kCostTileFloats;
+            float *dst = costs + ((size_t)t - a.tile_base) * kCostTileFloats;
             bulk_s2g(dst, &S.C[0][0], kCostHalfBytes);
             bulk_s2g(dst + kCostHalfFloats, &S.Phi[0][0], kCostHalfBytes);
             bulk_commit();
@@ -1132,7 +1135,7 @@ __device__ __forceinline__ void res_issue_costs(const FastArgs &a, Smem &S, int 
     const int ngv = std::min(a.G - gbase, a.Gc);  // real multipliers of the split
     const uint32_t rows_bytes = (uint32_t)((diag ? 1 : L) * BK * sizeof(float));
     const uint32_t mdp_bytes = (a.prune && !diag) ? (uint32_t)(ngv * a.mdp_stride * sizeof(float)) : 0u;
-    const float *src = a.costs + cost_tile_idx(K, J) * kCostTileFloats;
+    const float *src = a.costs + (cost_tile_idx(K, J) - a.tile_base) * kCostTileFloats;
     mbar_expect_tx(&S.mbar[b], 2 * kCostHalfBytes + (uint32_t)ngv * rows_bytes + mdp_bytes);
     bulk_g2s(&S.C[b][0][0], src, kCostHalfBytes, &S.mbar[b], policy);
     bulk_g2s(&S.Phi[b][0][0], src + kCostHalfFloats, kCostHalfBytes, &S.mbar[b], policy);
@@ -1212,7 +1215,7 @@ __device__ __forceinline__ void res_stage(const FastArgs &a, Smem &S, float *stg
         const uint32_t mb = (uint32_t)((size_t)(K1 - K0) * a.G * a.mdp_stride * sizeof(float));
         S.sfront[sb] = frontier;  // ordered before the readers' wait by the arrive (release)
         mbar_expect_tx(&S.smbar[sb], tb + mb);
-        bulk_g2s(stg, a.tsum + (cost_tile_idx(0, J) + (size_t)K0) * BJ, tb, &S.smbar[sb], policy);
+        bulk_g2s(stg, a.tsum + (cost_tile_idx(0, J) - a.tile_base + (size_t)K0) * BJ, tb, &S.smbar[sb], policy);
         bulk_g2s_nohint(stg + (size_t)kStageTiles * BJ * 2, a.mdp + (size_t)K0 * a.G * a.mdp_stride, mb, &S.smbar[sb]);
     }
 }
@@ -1303,8 +1306,8 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
         if (ct == 0) S.ticket = atomicAdd(a.ticket, 1);
         __syncthreads();
         const int t = S.ticket;
-        if (t >= a.nJ * a.nsplit) break;
-        const int J = t / a.nsplit, split = t % a.nsplit;
+        if (t >= (a.J1 - a.J0) * a.nsplit) break;
+        const int J = a.J0 + t / a.nsplit, split = t % a.nsplit;
         const int g = split * a.Gc + id.gl;
         const bool own = id.active && g < a.G;
         if (split != fsplit) { frontier = -1; fsplit = split; }
@@ -1445,7 +1448,7 @@ __device__ void visit_tile(const FastArgs &a, int g, int i, int64_t j, int64_t K
     const float *prev = a.dp32 + d32(a, g, i - 1, k0) - k0;  // prev[k] for k in tile K
     if (a.costs) {
         // the wavefront's own interval costs, read back from the resident table
-        const float *cr = a.costs + cost_tile_idx(K, J) * kCostTileFloats + (size_t)(j - j0) * PSTR;
+        const float *cr = a.costs + (cost_tile_idx(K, J) - a.tile_base) * kCostTileFloats + (size_t)(j - j0) * PSTR;
         const float *pr = cr + kCostHalfFloats;
         int64_t khi = (K == J) ? j - 1 : k0 + BK - 1;
         for (int64_t k = khi; k >= k0; k--)
@@ -1736,7 +1739,7 @@ __global__ void __launch_bounds__(128) k_exact_big(Prefix P, FastArgs a, int i, 
             for (uint32_t t = 0; t < ntile; t++) {
                 const int64_t K = t < n1 ? (w1 >> 16) + t : (w2 >> 16) + (t - n1);
                 const int64_t k0 = K * BK;
-                const float *cr = a.costs + cost_tile_idx(K, J) * kCostTileFloats + (size_t)(j - j0) * PSTR;
+                const float *cr = a.costs + (cost_tile_idx(K, J) - a.tile_base) * kCostTileFloats + (size_t)(j - j0) * PSTR;
                 const float *pr = cr + kCostHalfFloats;
                 const float *prev32 = a.dp32 + d32(a, g, i - 1, k0) - k0;
                 const int64_t khi = (K == J) ? j - 1 : k0 + BK - 1;
@@ -1832,8 +1835,21 @@ size_t resident_costs_bytes(int64_t d) {
     return n * (n + 1) / 2 * (kCostTileFloats * sizeof(float) + BJ * sizeof(float2));
 }
 
+// Streamed interval costs: the cost tiles of a band of column blocks at a time, in a
+// buffer of streamed_costs_bytes(d) (tiles, then their column summaries).  The band
+// holds up to 64 full columns of tiles, so a band near the end of the triangle still
+// has 64 blocks (times the multiplier splits) to spread over the SMs.
+static size_t tile_bytes_with_summary() { return kCostTileFloats * sizeof(float) + BJ * sizeof(float2); }
+size_t streamed_costs_bytes(int64_t d) {
+    if (d < 1) return 0;
+    const size_t nJ = (size_t)cdiv(d, BJ);
+    const size_t full = nJ * (nJ + 1) / 2, band = std::min(full, (size_t)64 * nJ);
+    return band * tile_bytes_with_summary();
+}
+
 int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, const Layout &Lw, cudaStream_t st,
-                   bool exact_s, bool exact_tables, float *costs, bool build_costs, bool test_stall) {
+                   bool exact_s, bool exact_tables, float *costs, bool build_costs, bool test_stall,
+                   size_t chunk_bytes) {
     double *dp64 = wsp<double>(ws, Lw.dp64);
     int32_t *bp = wsp<int32_t>(ws, Lw.bp);
     // small inputs, very large ones and huge counts take the reference kernel
@@ -1891,10 +1907,14 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     a.hold0 = test_stall ? 1 : 0;
     a.prune = (costs && a.lgc == 2 && a.mdp_stride <= 20) ? 1 : 0;
     a.costs = costs;
-    if (costs) {
-        const size_t nJd = (size_t)cdiv(Lw.d, BJ);
-        a.tsum = reinterpret_cast<float2 *>(costs + nJd * (nJd + 1) / 2 * kCostTileFloats);
-    }
+    a.tile_base = 0;
+    a.J0 = 0;
+    a.J1 = a.nJ;
+    // tiles the costs buffer holds at once: the whole triangle, or (streamed) one band
+    const size_t cap_tiles = chunk_bytes ? chunk_bytes / tile_bytes_with_summary()
+                                         : (size_t)cdiv(Lw.d, BJ) * (size_t)(cdiv(Lw.d, BJ) + 1) / 2;
+    if (costs) a.tsum = reinterpret_cast<float2 *>(costs + cap_tiles * kCostTileFloats);
+    if (chunk_bytes && cap_tiles < (size_t)a.nJ) return ECASQ_EWORKSPACE;  // one column of tiles must fit
     a.prm = dprm;
     a.done = flags;
     a.ticket = flags + (size_t)kMaxG * a.nJ;
@@ -1923,26 +1943,54 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
         k_corners<<<(unsigned)std::min<int64_t>(cdiv((int64_t)a.nJ * (a.nJ - 1) / 2, 128), 152 * 64), 128, 0, st>>>(a);
         ECASQ_LAUNCH_CHECK();
     }
-    if (costs && build_costs) {
-        int per_sm = 0;
-        ECASQ_CUDA_TRY(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_build_costs, NPROD, 0));
-        int64_t ntiles = (int64_t)a.nJ * (a.nJ + 1) / 2;
-        note_launch();
-        k_build_costs<<<(unsigned)std::min<int64_t>(ntiles, (int64_t)nsm * std::max(per_sm, 1)), NPROD, 0, st>>>(a, costs);
-        ECASQ_LAUNCH_CHECK();
-    }
     size_t smem = smem_bytes(a.Gc, s);
     if (costs && a.lgc == 2)  // parked band state; off the diagonal, the two stage buffers
         smem += std::max((size_t)3 * LPT * JPT * a.ncons * sizeof(uint32_t),
                          a.prune ? 2 * stage_floats(G, a.mdp_stride) * sizeof(float) : (size_t)0);
     auto wave = costs ? k_wavefront_res : k_wavefront;
     ECASQ_CUDA_TRY(cudaFuncSetAttribute(wave, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-    int grid = std::min(nsm, a.nJ * a.nsplit);
-    timer_begin(st);
-    note_launch();
-    wave<<<grid, (costs ? 0 : NPROD) + a.ncons, smem, st>>>(a);
-    timer_end(st);
-    ECASQ_LAUNCH_CHECK();
+    int per_sm = 0;
+    if (costs && build_costs)
+        ECASQ_CUDA_TRY(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_build_costs, NPROD, 0));
+    // one band of column blocks per round: [J0, J1) whose tiles fit the buffer (all of them
+    // when the buffer holds the whole triangle); with streamed costs every band's tiles are
+    // built just before its wavefront, else the table is built once per call.  The
+    // timer covers the min-plus kernel; with streamed costs, every band's build and
+    // wavefront together (the builds are then part of every pass)
+    if (chunk_bytes) timer_begin(st);
+    for (int J0 = 0; J0 < a.nJ;) {
+        int J1 = a.nJ;
+        if (chunk_bytes) {
+            J1 = J0 + 1;
+            const size_t T0 = (size_t)J0 * (J0 + 1) / 2;
+            while (J1 < a.nJ && (size_t)(J1 + 1) * (J1 + 2) / 2 - T0 <= cap_tiles) J1++;
+        }
+        a.J0 = J0;
+        a.J1 = J1;
+        a.tile_base = chunk_bytes ? (size_t)J0 * (J0 + 1) / 2 : 0;
+        if (costs && build_costs) {
+            const int64_t ntiles = (int64_t)J1 * (J1 + 1) / 2 - (int64_t)a.tile_base;
+            note_launch();
+            k_build_costs<<<(unsigned)std::min<int64_t>(ntiles, (int64_t)nsm * std::max(per_sm, 1)), NPROD, 0, st>>>(
+                a, costs);
+            ECASQ_LAUNCH_CHECK();
+        }
+        if (J0 > 0) ECASQ_CUDA_TRY(cudaMemsetAsync(a.ticket, 0, sizeof(int), st));
+        int grid = std::min(nsm, (J1 - J0) * a.nsplit);
+        if (!chunk_bytes) timer_begin(st);
+        note_launch();
+        wave<<<grid, (costs ? 0 : NPROD) + a.ncons, smem, st>>>(a);
+        if (!chunk_bytes) timer_end(st);
+        ECASQ_LAUNCH_CHECK();
+        J0 = J1;
+    }
+    if (chunk_bytes) timer_end(st);
+    // a streamed band holds only the last band's tiles: the need and exact stages re-derive
+    // the costs they read (any evaluation within the certified bound will do)
+    if (chunk_bytes) {
+        a.costs = nullptr;
+        a.tile_base = 0;
+    }
     const int ilo = exact_s ? s : 2;
     note_launch();
     k_need_init<<<(unsigned)std::min<int64_t>(cdiv((int64_t)G * (s + 1) * P.ps, 256), (int64_t)nsm * 32), 256, 0, st>>>(

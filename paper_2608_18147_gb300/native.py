@@ -17,7 +17,7 @@ import numpy as np
 from . import build as _build
 
 OK, EINVAL, ENONFINITE, EINFEASIBLE, EWORKSPACE, ECUDA, ETIMEOUT, ERANGE = 0, -1, -2, -3, -4, -5, -6, -7
-EXACT_S, NO_REFINE_GUARD, DP_REFERENCE, TIME_KERNELS, EXACT_TABLES, RESIDENT_COSTS = 1, 2, 4, 8, 16, 32
+EXACT_S, NO_REFINE_GUARD, DP_REFERENCE, TIME_KERNELS, EXACT_TABLES, RESIDENT_COSTS, STREAMED_COSTS = 1, 2, 4, 8, 16, 32, 64
 TEST_STALL = 1 << 30  # test hook of the bounded waits (include/ecasq.h)
 
 _lock = threading.Lock()
@@ -36,7 +36,8 @@ class Result(C.Structure):
                 ("lambda_", C.c_double), ("lambda_prime", C.c_double), ("norm2", C.c_double), ("mse", C.c_double),
                 ("vnmse", C.c_double), ("h_surrogate", C.c_double), ("h_exact", C.c_double), ("r_tot", C.c_double),
                 ("objective", C.c_double), ("candidates", C.c_int64), ("rescored", C.c_int64),
-                ("dp_kernel_ms", C.c_double), ("dp_kernel_launches", C.c_int32), ("reserved2", C.c_int32)]
+                ("dp_kernel_ms", C.c_double), ("dp_kernel_launches", C.c_int32), ("reserved2", C.c_int32),
+                ("refine_last_rel", C.c_double)]
 
     def as_dict(self):
         out = {}

@@ -91,7 +91,26 @@ def check(meta_path, out_dir=None):
     rep["objective_of_gpu_codebook"] = mse + lp * hs
     rep["objective_rel"] = abs(rep["objective_of_gpu_codebook"] - r["best"]) / abs(r["best"])
     rep["feasible"] = bool(hs <= meta["budget_bits"])
-    ok = (rep["dp_max_rel"] <= DP_RTOL and rep["bp_invalid"] == 0 and rep["metrics_max_rel"] <= MET_RTOL
+    ref_ok = True
+    if "refined" in meta:
+        # Sec. 6 refinement of the oracle's own DP codebook at the same multiplier, the same
+        # budget guard and stop rule, against the GPU's refined solve
+        g = meta["refined"]
+        t1 = time.perf_counter()
+        rf = H.refine(r["Q_idx"], lp, budget=meta["budget_bits"], guard=True, max_rounds=g["max_rounds"],
+                      tol=g["tol"])
+        a_ref = np.searchsorted(v, np.float32(g["Q"]))
+        mo = H.eval_idx(rf["Q_idx"])
+        rep["refine"] = dict(rounds_gpu=g["rounds"], rounds_oracle=rf["rounds"],
+                             codebook_equal=bool(np.array_equal(a_ref, rf["Q_idx"])),
+                             last_rel_gpu=g["last_rel"],
+                             last_rel_oracle=float((rf["J"][-2] - rf["J"][-1]) / abs(rf["J"][-2])),
+                             metrics_max_rel=max(abs(a - b) / abs(b) for a, b in
+                                                 zip([g["mse"], g["h_surrogate"], g["h_exact"]], mo) if b),
+                             stopped_by_rule=rf["rounds"] < g["max_rounds"], oracle_wall_s=time.perf_counter() - t1)
+        ref_ok = (rep["refine"]["codebook_equal"] and rep["refine"]["rounds_gpu"] == rep["refine"]["rounds_oracle"]
+                  and rep["refine"]["metrics_max_rel"] <= MET_RTOL)
+    ok = ref_ok and (rep["dp_max_rel"] <= DP_RTOL and rep["bp_invalid"] == 0 and rep["metrics_max_rel"] <= MET_RTOL
           and rep["feasible"] and rep["pass_codebook_equal_solve"]
           and (rep["codebook_equal"] or (rep["path_min_margin"] < TIE and rep["objective_rel"] <= TIE)))
     rep["pass"] = bool(ok)

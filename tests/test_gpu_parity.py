@@ -340,16 +340,20 @@ def test_quantize_bit_exact(E, oracle_mod, d, offset):
         assert he == pytest.approx(oh, rel=1e-12, abs=1e-15)
 
 
-@pytest.mark.parametrize("m", [2, 32, 33, 256])
+@pytest.mark.parametrize("m", [1, 2, 3, 5, 8, 9, 16, 17, 32, 33, 256])
 @pytest.mark.parametrize("offset", [0, 1])
 def test_quantize_bit_exact_codebook_sizes(E, oracle_mod, m, offset):
-    """Codebooks on both sides of the per-thread-histogram limit (32 values) and at the
-    cap, on an input long enough for several grid-stride steps per thread."""
+    """Every search depth of the short-codebook kernel (m <= 16: 0 to 4 unrolled steps),
+    both sides of the per-thread-histogram limits (16 and 32 values) and the cap, on an
+    input long enough for several grid-stride steps per thread."""
     import torch
     d = 3_000_001
     x = workloads.signed_lognormal(d + offset, 11)
     xg = torch.as_tensor(x).cuda()[offset:]
     xs = x[offset:]
+    if m == 1:  # a constant input: every entry equals the single value
+        xs = np.full_like(xs, np.float32(2.5))
+        xg = torch.as_tensor(xs).cuda()
     Q = np.unique(np.quantile(xs, np.linspace(0.0, 1.0, m)).astype(np.float32))
     Q[0], Q[-1] = xs.min(), xs.max()
     assert Q.size == m

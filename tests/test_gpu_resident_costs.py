@@ -176,3 +176,53 @@ def test_full_size_sampled_decisions(E, oracle_mod):
         np.testing.assert_allclose(met[g][1:], [mse, hs, hx], rtol=MET_RTOL)
     del ws
     _free()
+
+
+@pytest.mark.parametrize("flags_name", ["DEFAULT", "EXACT_TABLES"])
+@pytest.mark.parametrize("name,s", [("lognormal16k", 16), ("ragged20001", 9), ("mixture12k", 32)])
+def test_streamed_costs_bit_identical_to_fused(E, name, s, flags_name):
+    """ECASQ_STREAMED_COSTS builds the cost tiles band by band into a bounded buffer and runs
+    the wavefront over each band: the same fp32 values as the fused producer's, so the same
+    tables (resolved and unresolved outputs alike), codebooks and metrics, over several bands."""
+    if name == "lognormal16k":
+        x = workloads.signed_lognormal(16384, 0)
+    elif name == "ragged20001":
+        x = workloads.student_t(20001, 4, scale=1.0)
+    else:
+        x = workloads.mixture(12288, 2)
+    flags = getattr(E, flags_name, 0)
+    lams = [0.0, 1e-5, 1e-3, 0.01, 0.05, 0.2, 1.0, 10.0]
+    wsf = E.workspace(x.size, s)
+    wss = E.workspace(x.size, s, flags=E.STREAMED_COSTS)
+    full = E.ecasq_workspace_size_flags(x.size, s, 1, E.RESIDENT_COSTS)
+    assert wsf.numel() < wss.numel() < full
+    Qf, mf, metf = E.ecasq_dp_pass(x, s, lams, flags=flags, ws=wsf)
+    n0 = E.ecasq_kernel_launches()
+    Qs, ms, mets = E.ecasq_dp_pass(x, s, lams, flags=flags | E.STREAMED_COSTS, ws=wss)
+    n1 = E.ecasq_kernel_launches()
+    Qf2, _, _ = E.ecasq_dp_pass(x, s, lams, flags=flags, ws=wsf)
+    n2 = E.ecasq_kernel_launches()
+    assert (n1 - n0) - (n2 - n1) >= 3  # at least two bands: a build and a wavefront launch each
+    for ws in (wsf, wss):
+        st = E.native.ws_status(ws)
+        assert st["timeout"] == 0 and st["bound_viol"] == 0
+    assert mf == ms
+    np.testing.assert_array_equal(Qf.cpu().numpy(), Qs.cpu().numpy())
+    np.testing.assert_array_equal(metf, mets)
+    for (dpf, bpf), (dps, bps) in zip(_tables(E, wsf, len(lams), s, x.size), _tables(E, wss, len(lams), s, x.size)):
+        np.testing.assert_array_equal(dpf, dps)
+        np.testing.assert_array_equal(bpf, bps)
+    del wsf, wss
+    _free()
+
+
+def test_streamed_costs_budgeted_solve_matches_oracle(E, oracle_mod):
+    """The budgeted solve (multiplier search, refinement) with streamed costs against the oracle."""
+    x = workloads.mixture(9000, 5)
+    Q, res = E.ecasq_solve(x, 12, budget_bits=3.0, refine_max_rounds=5, refine_rel_tol=1e-9,
+                           flags=E.STREAMED_COSTS)
+    o = oracle_mod.solve_budget(x, 12, 3.0, refine_rounds=5, refine_tol=1e-9)
+    assert res["lambda"] == o["lam"]
+    np.testing.assert_array_equal(Q.cpu().numpy(), o["Q"])
+    np.testing.assert_allclose([res["mse"], res["h_surrogate"], res["h_exact"]],
+                               [o["mse"], o["h_surrogate"], o["h_exact"]], rtol=MET_RTOL)
