@@ -115,6 +115,21 @@ def executed_candidates(st, p, s, multipliers):
     return off + diag
 
 
+def cost_mode_flags(E, d, s, free_bytes, share=0.6):
+    """Interval-cost mode of the fast DP: the whole table resident when it fits in `share` of
+    the free device memory, else band by band through a bounded buffer when that fits, else
+    the fused kernel (costs rebuilt by producer warps in every pass)."""
+    for flag in (E.RESIDENT_COSTS, E.STREAMED_COSTS):
+        need = E.ecasq_workspace_size_flags(d, s, 1, flag)
+        if 0 < need <= share * free_bytes:
+            return flag
+    return 0
+
+
+def cost_mode_name(E, flags):
+    return "resident" if flags & E.RESIDENT_COSTS else ("streamed" if flags & E.STREAMED_COSTS else "fused")
+
+
 class ClockSampler:
     """nvidia-smi clocks and throttle reasons sampled during the timed region."""
     REASONS = {0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap", 0x8: "hw_slowdown",
@@ -243,9 +258,7 @@ def run_other_mode(args, cfg, x_np):
             _, _, he = E.ecasq_quantize(x, Q, seed=12345, ws=qws, idx=idx, counts=counts[:Q.numel()])
             return res, {}
     else:
-        need = E.ecasq_workspace_size_flags(d, s, 1, E.RESIDENT_COSTS)
-        if 0 < need <= 0.6 * torch.cuda.mem_get_info()[0]:
-            flags |= E.RESIDENT_COSTS
+        flags |= cost_mode_flags(E, d, s, torch.cuda.mem_get_info()[0])
         ws = E.workspace(d, s, flags=flags)
 
         def step():
@@ -276,7 +289,7 @@ def run_other_mode(args, cfg, x_np):
            "dtype": "f64" if args.mode == "grid" else "f32 (fp64 exact stage)", "data": "synthetic",
            "config": {"workload": args.config, "mode": args.mode, "d": d, "s": s, "budget_bits": budget,
                       "grid": args.grid if args.mode == "grid" else None,
-                      "resident_costs": bool(flags & E.RESIDENT_COSTS)},
+                      "cost_mode": cost_mode_name(E, flags)},
            "solve": {"m": res["m"], "p": res["p"], "lambda": res["lambda"], "vnmse": res["vnmse"],
                      "h_surrogate": res["h_surrogate"], "h_exact": res["h_exact"], "passes": res["passes"],
                      "candidates_per_solve": res["candidates"], "dp_ms_per_solve": dp_ms / args.steps,
@@ -403,10 +416,7 @@ def run_pass_mode(args, cfg, x_np):
         x_np = x_np[:args.prefix]
     x = torch.as_tensor(x_np).cuda()
     d = x.numel()
-    flags = 0
-    need = E.ecasq_workspace_size_flags(d, s, 1, E.RESIDENT_COSTS)
-    if 0 < need <= 0.6 * torch.cuda.mem_get_info()[0]:
-        flags |= E.RESIDENT_COSTS
+    flags = cost_mode_flags(E, d, s, torch.cuda.mem_get_info()[0])
     ws = E.workspace(d, s, flags=flags)
     launches0 = E.ecasq_kernel_launches()
     ms, outs, clocks = _timed_steps(args, lambda: E.ecasq_dp_pass(x, s, lams, flags=flags, ws=ws))
@@ -418,7 +428,7 @@ def run_pass_mode(args, cfg, x_np):
            "higher_is_better": True, "vs_baseline": None, "dtype": "f32 (fp64 exact stage)", "data": "synthetic",
            "config": {"workload": args.config + (" (first %d entries)" % d if args.prefix > 0 else ""),
                       "mode": "pass", "d": d, "p": p, "s": s, "lambdas": lams,
-                      "resident_costs": bool(flags & E.RESIDENT_COSTS)},
+                      "cost_mode": cost_mode_name(E, flags)},
            "status": {"timeout": st["timeout"], "bound_viol": st["bound_viol"], "rescored": st["rescored"],
                       "tile_units_run": st["tiles_run"], "tile_units_skipped": st["tiles_skipped"],
                       "cost_tiles_fetched": st["tiles_fetched"],
@@ -515,10 +525,7 @@ def main():
     x = torch.as_tensor(x_np).cuda()
     # resident interval costs when they fit in 60% of the free device memory
     flags = E.TIME_KERNELS
-    free_b = torch.cuda.mem_get_info()[0]
-    need = E.ecasq_workspace_size_flags(d, s, 1, E.RESIDENT_COSTS)
-    if 0 < need <= 0.6 * free_b:
-        flags |= E.RESIDENT_COSTS
+    flags |= cost_mode_flags(E, d, s, torch.cuda.mem_get_info()[0])
     ws = E.workspace(d, s, flags=flags)
     idx = torch.empty(d, dtype=torch.uint8, device="cuda")
     counts = torch.empty(s, dtype=torch.int32, device="cuda")
@@ -578,7 +585,7 @@ def main():
                 "traffic_note": "DRAM bytes per launch: bytes per fetched cost tile from an ncu capture at "
                                 "d = 16384, times the tiles this launch fetched",
                 "tiles_fetched_per_launch": fetched_per_launch,
-                "kernel": "k_wavefront_res" if (flags & E.RESIDENT_COSTS) else "k_wavefront",
+                "kernel": "k_wavefront" if cost_mode_name(E, flags) == "fused" else "k_wavefront_res",
                 "peak_basis": "%d SMs (device attribute) x 128 FP32-pipe lanes (adds and mins share the issue "
                               "slots) x 2070 MHz max clock; of the 2-op count below" % n_sm,
                 "avg_launch_ms": dp_ms / max(dp_launches, 1), "launches": dp_launches,
@@ -629,7 +636,7 @@ def main():
                "scaling": "weak", "vs_baseline": None, "dtype": "f32 (fp64 exact stage)", "data": "synthetic",
                "config": {"workload": args.config, "d": d, "s": s, "budget_bits": budget,
                           "refine": {"max_rounds": refine_rounds, "rel_tol": refine_tol},
-                          "resident_costs": bool(flags & E.RESIDENT_COSTS),
+                          "cost_mode": cost_mode_name(E, flags),
                           "workspace_gb": round(ws.numel() / 1e9, 2),
                           "l2": "working set larger than the 129 MB L2 (DP tables ~0.9 GB; resident costs "
                                 "streamed once per pass); no flush",

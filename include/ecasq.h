@@ -62,6 +62,9 @@ typedef struct CUstream_st *ecasq_stream_t; /* same type as cudaStream_t */
                                      of tiles, 2.3 MB x ceil(d / 64); ecasq_workspace_size_flags with this flag) and
                                      the wavefront runs band by band; rebuilt in every pass.  RESIDENT_COSTS wins
                                      when both are given.  Results are the same as with either other mode. */
+#define ECASQ_ONE_PART_PUBLISH 128u /* fast DP with resident or streamed costs and s <= 16: publish each column block
+                                     of the wavefront once, after all its layers, instead of in two parts (rows 2..8
+                                     after layer 8, then the rest); same results, for comparison */
 #define ECASQ_TEST_STALL (1u << 30) /* test hook for the bounded device waits: column block 0 of the fast DP's
                                      wavefront is never published and the flag waits give up after 2^14 spins, so
                                      the call must return ECASQ_ETIMEOUT (nothing else) and leave the workspace

@@ -17,7 +17,7 @@ int launch_dp_reference(const Prefix &P, const double *lamp, int G, int s, doubl
                         cudaStream_t st);
 int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, const Layout &L, cudaStream_t st,
                    bool exact_s, bool exact_tables, float *costs, bool build_costs, bool test_stall,
-                   size_t chunk_bytes);
+                   size_t chunk_bytes, bool split_off);
 size_t resident_costs_bytes(int64_t d);
 size_t streamed_costs_bytes(int64_t d);
 int launch_rows_prepare(const float *X, int64_t rows, const RowsData &R, cudaStream_t st);
@@ -292,7 +292,7 @@ static int dp_pass_prepared(void *ws, const Layout &L, const Prefix &P, int s, c
         // streamed costs are rebuilt band by band in every pass
         rc = launch_dp_fast(P, lamp, G, s, ws, L, st, (flags & ECASQ_EXACT_S) != 0, (flags & ECASQ_EXACT_TABLES) != 0,
                             costs, costs && (L.costs_streamed || !*costs_built), (flags & ECASQ_TEST_STALL) != 0,
-                            L.costs_streamed ? L.costs_bytes : 0);
+                            L.costs_streamed ? L.costs_bytes : 0, (flags & ECASQ_ONE_PART_PUBLISH) != 0);
         if (costs && rc == ECASQ_OK) *costs_built = true;
     }
     if (rc != ECASQ_OK) return rc;

@@ -143,7 +143,9 @@ struct FastArgs {
     int prune;             // skip tiles by the lower bound (resident costs, two layer groups)
     uint32_t spin_limit;   // flag waits give up after this many spins (kSpinLimit; lower in the test hook)
     int hold0;             // test hook: column block 0 is never published (its waiters time out)
-    int *done;             // [nsplit][nJ]
+    int split_pub;         // resident costs, two layer groups: blocks are published in two parts (below)
+    int *done;             // [nsplit][nJ]: every row of the block is stored
+    int *half;             // [nsplit][nJ]: rows 2..8 of the block are stored (split_pub)
     int *ticket;
     int *abort_flag;
     DevStatus *st;
@@ -848,13 +850,15 @@ __device__ __forceinline__ void kdiag_group(int g4, int half, int &q, int &k) {
     else { q = 1; k = half ? 4 * (g4 - 12) : 4 * (g4 - 16); }
 }
 
-__device__ __forceinline__ void cons_diag_pair(const FastArgs &a, Smem &S, uint32_t *park, int b, int J, int split,
-                                               const ConsId &id, ConsState &cs) {
-    const int L = a.s - 2;
+// cons_diag_pair in three steps, so that the block can be published in two parts
+// (diag_prepare; diag_layers over a range of layers; diag_store over a range of rows).
+// diag_prepare: park the band state, store the block minimum of layer 2, and build the
+// lane's costs W = C + lambda' Phi of its 80 pairs (kept in registers for all layers).
+__device__ __forceinline__ void diag_prepare(const FastArgs &a, Smem &S, uint32_t *park, int b, int J, int split,
+                                             const ConsId &id, const ConsState &cs, float2 (&W)[2 * kDiagGroups]) {
     const int ct = id.ct, nc = a.ncons;
     const int g = split * a.Gc + id.gl;
     const bool own = id.active && g < a.G;  // uniform over a warp (one multiplier per warp)
-    const int64_t j0 = (int64_t)J * BJ;
     constexpr int NS = LPT * JPT;
 #pragma unroll
     for (int l = 0; l < LPT; l++)
@@ -875,24 +879,33 @@ __device__ __forceinline__ void cons_diag_pair(const FastArgs &a, Smem &S, uint3
     }
     const int half = (ct >> 4) & 1;
     const int qb = 3 - half, qs = half;  // the lane's long and short columns (q of jq + 16 q)
-    float2 W[2 * kDiagGroups];           // W[2 g4], W[2 g4 + 1]: costs of group g4's four pairs
-    {
-        const float lam = own ? S.lam32[g] : 0.f;
-        const float2 lam2 = make_float2(lam, lam);
+    const float lam = own ? S.lam32[g] : 0.f;
+    const float2 lam2 = make_float2(lam, lam);
 #pragma unroll
-        for (int g4 = 0; g4 < kDiagGroups; g4++) {
-            int q, k;
-            kdiag_group(g4, half, q, k);
-            const int jl = id.jq + NJQ * (q ? qs : qb);
-            float4 c4 = *reinterpret_cast<const float4 *>(&S.C[b][jl][k]);
-            float4 f4 = *reinterpret_cast<const float4 *>(&S.Phi[b][jl][k]);
-            W[2 * g4] = fma2(lam2, make_float2(f4.x, f4.y), make_float2(c4.x, c4.y));
-            W[2 * g4 + 1] = fma2(lam2, make_float2(f4.z, f4.w), make_float2(c4.z, c4.w));
-        }
+    for (int g4 = 0; g4 < kDiagGroups; g4++) {  // W[2 g4], W[2 g4 + 1]: costs of group g4's four pairs
+        int q, k;
+        kdiag_group(g4, half, q, k);
+        const int jl = id.jq + NJQ * (q ? qs : qb);
+        float4 c4 = *reinterpret_cast<const float4 *>(&S.C[b][jl][k]);
+        float4 f4 = *reinterpret_cast<const float4 *>(&S.Phi[b][jl][k]);
+        W[2 * g4] = fma2(lam2, make_float2(f4.x, f4.y), make_float2(c4.x, c4.y));
+        W[2 * g4 + 1] = fma2(lam2, make_float2(f4.z, f4.w), make_float2(c4.z, c4.w));
     }
+}
+
+// Layers li0 <= li < li1 (i = 3 + li) of the diagonal block; cur: the S.diag row
+// holding layer i - 1 (in/out).
+__device__ __forceinline__ void diag_layers(const FastArgs &a, Smem &S, uint32_t *park, int J, int split,
+                                            const ConsId &id, const float2 (&W)[2 * kDiagGroups], int li0, int li1,
+                                            int &cur) {
+    const int ct = id.ct, nc = a.ncons;
+    const int g = split * a.Gc + id.gl;
+    const bool own = id.active && g < a.G;
+    constexpr int NS = LPT * JPT;
+    const int half = (ct >> 4) & 1;
+    const int qb = 3 - half, qs = half;
     const uint32_t K = (uint32_t)J, KK = (K << 16) | K;
-    int cur = 0;
-    for (int li = 0; li < L; li++) {
+    for (int li = li0; li < li1; li++) {
         const int i = 3 + li;
         const int olg = li / LPT, l = li - olg * LPT;
         // minima (float bits; candidates are >= +0) of the long and the short column:
@@ -941,14 +954,21 @@ __device__ __forceinline__ void cons_diag_pair(const FastArgs &a, Smem &S, uint3
         __syncwarp();  // the layer's row and parked state belong to this warp alone
         cur ^= 1;
     }
-    // the block's final values from the parked state, and the block minimum of
-    // every layer (over the 64 columns a half-warp holds); the band words follow
-    // after the block is published (diag_pair_bands: only the exact stage reads them)
+}
+
+// The block's final values of layers ilo <= i <= ihi from the parked state, and the
+// block minimum of each of those layers (over the 64 columns a half-warp holds).
+__device__ __forceinline__ void diag_store(const FastArgs &a, const uint32_t *park, int J, int split,
+                                           const ConsId &id, int ilo, int ihi) {
+    const int ct = id.ct, nc = a.ncons;
+    const int g = split * a.Gc + id.gl;
+    const bool own = id.active && g < a.G;
+    const int64_t j0 = (int64_t)J * BJ;
     if (own) {
 #pragma unroll
         for (int l = 0; l < LPT; l++) {
             const int i = 3 + id.lg * LPT + l;
-            const bool real = i <= a.s;
+            const bool real = i <= a.s && i >= ilo && i <= ihi;
             int v = 0x7f800000;
 #pragma unroll
             for (int q = 0; q < JPT; q++) {
@@ -961,6 +981,89 @@ __device__ __forceinline__ void cons_diag_pair(const FastArgs &a, Smem &S, uint3
 #pragma unroll
                 for (int o = 8; o > 0; o >>= 1) v = min(v, __shfl_xor_sync(0xffffffffu, v, o));
                 if (real && id.jq == 0) a.mdp[((size_t)J * a.G + g) * a.mdp_stride + i] = __int_as_float(v);
+            }
+        }
+    }
+}
+
+// The whole diagonal block at once (the block is then published in one part).
+__device__ __forceinline__ void cons_diag_pair(const FastArgs &a, Smem &S, uint32_t *park, int b, int J, int split,
+                                               const ConsId &id, ConsState &cs) {
+    float2 W[2 * kDiagGroups];
+    diag_prepare(a, S, park, b, J, split, id, cs, W);
+    int cur = 0;
+    diag_layers(a, S, park, J, split, id, W, 0, a.s - 2, cur);
+    diag_store(a, park, J, split, id, 3, a.s);
+}
+
+// Split publish (resident costs, two layer groups).  The chain of blocks runs through the
+// last off-diagonal tile (J-1, J) and the diagonal block J.  Block J-1 is published in
+// two parts -- rows 2..8 (layer group 0's inputs) after its layer 8, every row at the
+// end -- and block J takes tile (J-1, J) in the same two parts, so its layers 3..9
+// start as soon as block J-1 has finished layer 8.
+// cons_lasttile_grp: tile (J-1, J) for layer group grp (0: layers 3..9 from rows 2..8;
+// 1: layers 10..s from rows 9..s-1) by all 32 lanes of the warp -- lane 16 h + jq takes
+// columns jq + 16 q, q in {2h, 2h+1}, over the group's seven layers -- after which the
+// owners (the lanes of layer group grp) fold the tile minima of their four columns
+// into their parked band state.  There is no skip test: this tile is on the chain.
+__device__ __forceinline__ void cons_lasttile_grp(const FastArgs &a, const Smem &S, const float *sDPb, int b,
+                                                  uint32_t *park, uint32_t K, int g, const ConsId &id, int grp) {
+    const int L = a.s - 2;
+    const int ct = id.ct, nc = a.ncons;
+    const int h = (ct >> 4) & 1;
+    constexpr int NS = LPT * JPT;
+    int cm[LPT][2];
+#pragma unroll
+    for (int l = 0; l < LPT; l++) { cm[l][0] = 0x7f800000; cm[l][1] = 0x7f800000; }
+    const float *dpb = sDPb + (size_t)id.gl * L * BK;
+    const float lam = S.lam32[g];
+    const float2 lam2 = make_float2(lam, lam);
+    int rowl[LPT];
+#pragma unroll
+    for (int l = 0; l < LPT; l++) rowl[l] = min(grp * LPT + l, L - 1);
+#pragma unroll 1
+    for (int kk = 0; kk < BK; kk += 4) {
+        float2 W[2][2];
+#pragma unroll
+        for (int c = 0; c < 2; c++) {
+            const int jl = id.jq + NJQ * (2 * h + c);
+            const float4 c4 = *reinterpret_cast<const float4 *>(&S.C[b][jl][kk]);
+            const float4 f4 = *reinterpret_cast<const float4 *>(&S.Phi[b][jl][kk]);
+            W[c][0] = fma2(lam2, make_float2(f4.x, f4.y), make_float2(c4.x, c4.y));
+            W[c][1] = fma2(lam2, make_float2(f4.z, f4.w), make_float2(c4.z, c4.w));
+        }
+#pragma unroll
+        for (int l = 0; l < LPT; l++) {
+            const float4 d4 = *reinterpret_cast<const float4 *>(dpb + (size_t)rowl[l] * BK + kk);
+            const float2 da = make_float2(d4.x, d4.y), db = make_float2(d4.z, d4.w);
+#pragma unroll
+            for (int c = 0; c < 2; c++) {
+                const float2 t0 = add2(da, W[c][0]);
+                const float2 t1 = add2(db, W[c][1]);
+                const int m = min(min(cm[l][c], __float_as_int(t0.x)), __float_as_int(t0.y));
+                cm[l][c] = min(min(m, __float_as_int(t1.x)), __float_as_int(t1.y));
+            }
+        }
+    }
+    const uint32_t KK = (K << 16) | K;
+#pragma unroll
+    for (int l = 0; l < LPT; l++) {
+        const float tau = S.tau[3 + rowl[l]];
+#pragma unroll
+        for (int c = 0; c < 2; c++) {
+            const int other = __shfl_xor_sync(0xffffffffu, cm[l][c], 16);  // the partner's column q ^ 2
+            if (h == grp) {  // the owner of layer group grp (id.lg == h when there are two groups)
+#pragma unroll
+                for (int e = 0; e < 2; e++) {
+                    const int q = e ? 2 * (1 - h) + c : 2 * h + c;
+                    const int x = (l * JPT + q) * nc + ct;
+                    float bb = __uint_as_float(park[x]);
+                    uint32_t w1 = park[NS * nc + x], w2 = park[2 * NS * nc + x];
+                    band_fold(__int_as_float(e ? other : cm[l][c]), bb, tau, w1, w2, K, KK);
+                    park[x] = __float_as_uint(bb);
+                    park[NS * nc + x] = w1;
+                    park[2 * NS * nc + x] = w2;
+                }
             }
         }
     }
@@ -986,10 +1089,9 @@ __device__ __forceinline__ void diag_pair_bands(const FastArgs &a, const uint32_
     }
 }
 
-// Bounded wait (one thread) until column block K of `split` is published; false
-// when the wait gave up (timeout or abort).
-__device__ __forceinline__ bool wait_block(const FastArgs &a, int split, int K) {
-    const int *flag = a.done + (size_t)split * a.nJ + K;
+// Bounded wait (one thread) until `flag` is set; false when the wait gave up
+// (timeout or abort).
+__device__ __forceinline__ bool wait_flag(const FastArgs &a, const int *flag) {
     uint32_t spins = 0;
     while (ld_acquire(flag) == 0) {
         // the abort flag and the spin limit are checked every 64 spins, so a spin costs
@@ -1006,6 +1108,13 @@ __device__ __forceinline__ bool wait_block(const FastArgs &a, int split, int K) 
     }
     return true;
 }
+// ... until column block K of `split` is published (every row), or its rows 2..8 are.
+__device__ __forceinline__ bool wait_block(const FastArgs &a, int split, int K) {
+    return wait_flag(a, a.done + (size_t)split * a.nJ + K);
+}
+__device__ __forceinline__ bool wait_lower(const FastArgs &a, int split, int K) {
+    return wait_flag(a, a.half + (size_t)split * a.nJ + K);
+}
 
 // Publish column block J of `split` (one thread, after a barrier that follows every
 // thread's stores of the block).  The release store orders everything that happens
@@ -1014,6 +1123,11 @@ __device__ __forceinline__ bool wait_block(const FastArgs &a, int split, int K) 
 __device__ __forceinline__ void publish_block(const FastArgs &a, int split, int J) {
     if (a.hold0 && J == 0) return;  // test hook: the waiters on block 0 must give up
     st_release(a.done + (size_t)split * a.nJ + J, 1);
+}
+// The first part of a split publish: rows 2..8 of block J (and their block minima).
+__device__ __forceinline__ void publish_lower(const FastArgs &a, int split, int J) {
+    if (a.hold0 && J == 0) return;
+    st_release(a.half + (size_t)split * a.nJ + J, 1);
 }
 
 // ------------------------------------------------------------------ kernels
@@ -1296,7 +1410,8 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
     const ConsId id = cons_id(a, ct);
     ConsState cs;
     const uint64_t policy = policy_evict_first();
-    uint32_t n = 0;   // tile sequence number: buffer n & 1, its fill number n >> 1
+    uint32_t n = 0;   // tile sequence number: buffer n & 1
+    uint32_t mph[2] = {0u, 0u};  // completed phases of mbar[0], mbar[1] (one per fill; two for a split last tile)
     uint32_t ns = 0;  // batch sequence number (tile skipping): stage buffer ns & 1, its fill ns >> 1
     float *stage = sDP + (size_t)2 * rowsDP * BK;  // the park area, free off the diagonal
     const size_t sfl = stage_floats(a.G, a.mdp_stride);
@@ -1314,12 +1429,14 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
         cons_reset(cs);
         int issued = -1;  // the tile whose copies are in flight into buffer n & 1 (J: the diagonal), or -1
         const int ngv = min(a.G - split * a.Gc, a.Gc);  // real multipliers of the split
-        if (a.prune && J > 0 && ct < 32) {  // stage the first batch
+        // the tiles walked here: K < Kend (with a split publish the last one, J - 1, is the chain's)
+        const int Kend = a.split_pub ? max(J - 1, 0) : J;
+        if (a.prune && Kend > 0 && ct < 32) {  // stage the first batch
             if (frontier < 0) res_probe(a, split, 0, J, frontier, lane);
-            res_stage(a, S, stage + (ns & 1) * sfl, ns & 1, 0, batch_end(0, J), J, frontier, policy, lane);
+            res_stage(a, S, stage + (ns & 1) * sfl, ns & 1, 0, batch_end(0, Kend), J, frontier, policy, lane);
         }
-        for (int K0 = 0; K0 < J;) {
-            const int K1 = a.prune ? batch_end(K0, J) : min(J, K0 + 32);
+        for (int K0 = 0; K0 < Kend;) {
+            const int K1 = a.prune ? batch_end(K0, Kend) : min(Kend, K0 + 32);
             uint32_t wm = 0xffffffffu;  // the warp's tiles of the batch
             uint32_t U = 0xffffffffu;   // the tiles some warp needs
             int frb = -1;               // tiles <= frb: every warp issues its own rows (res_issue_rows)
@@ -1334,8 +1451,8 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
                 U = 0;
                 for (int w = 0; w < (int)(blockDim.x >> 5); w++) U |= S.needw[sb][w];
                 ns++;
-                if (K1 < J && ct < 32) {  // stage the next batch while this one is walked
-                    const int K2 = batch_end(K1, J);
+                if (K1 < Kend && ct < 32) {  // stage the next batch while this one is walked
+                    const int K2 = batch_end(K1, Kend);
                     if (K2 - 1 > frontier) res_probe(a, split, frontier + 1, J, frontier, lane);
                     res_stage(a, S, stage + (ns & 1) * sfl, ns & 1, K1, K2, J, frontier, policy, lane);
                 }
@@ -1356,8 +1473,9 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
                 const int K = K0 + __ffs(U) - 1;
                 U &= U - 1;
                 // the next tile to copy: the batch's next needed one, else the diagonal after
-                // the last batch, else (no skipping) the next batch's first tile
-                const int Kn = U ? K0 + __ffs(U) - 1 : (K1 == J ? J : (a.prune ? -1 : K1));
+                // the last batch (with a split publish the tail copies its own tiles), else (no
+                // skipping) the next batch's first tile
+                const int Kn = U ? K0 + __ffs(U) - 1 : (K1 == Kend ? (a.split_pub ? -1 : J) : (a.prune ? -1 : K1));
                 const int b = n & 1;
                 bool pending = false;  // warp 0: the rows of tile Kn still to be issued
                 if (Kn >= 0 && Kn < J && Kn <= frb) {
@@ -1372,7 +1490,8 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
                     pending = !ready;
                 }
                 issued = Kn;
-                mbar_wait_bounded(&S.mbar[b], (n >> 1) & 1u, a.st, a.abort_flag);
+                mbar_wait_bounded(&S.mbar[b], mph[b] & 1u, a.st, a.abort_flag);
+                mph[b]++;
                 if (own) {
                     const bool ran = ((wm >> (K - K0)) & 1u) &&
                                      cons_offdiag(a, S, sDP + (size_t)b * rowsDP * BK, b, (uint32_t)K, g, id, cs);
@@ -1388,10 +1507,82 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
             }
             K0 = K1;
         }
-        {  // the diagonal tile (issued with the last tile walked, else now)
+        if (a.split_pub) {
+            // the chain's part: tile (J-1, J) in buffer bA, the diagonal in bD (the cost copies
+            // depend on nothing published; the diagonal also copies row 2 of block J)
+            uint32_t *park = reinterpret_cast<uint32_t *>(sDP + (size_t)2 * rowsDP * BK);
+            const int bA = n & 1, bD = bA ^ 1;
+            const int gbase = split * a.Gc;
+            const uint32_t lo_bytes = (uint32_t)(LPT * BK * sizeof(float));        // rows 2..8
+            const uint32_t hi_bytes = (uint32_t)((L - LPT) * BK * sizeof(float));  // rows 9..s-1
+            float *rowsA = sDP + (size_t)bA * rowsDP * BK;
+            if (ct < 32) {
+                if (lane == 0) {
+                    if (J > 0) {
+                        mbar_expect_tx(&S.mbar[bA], 2 * kCostHalfBytes + (uint32_t)ngv * lo_bytes);
+                        const float *src = a.costs + (cost_tile_idx(J - 1, J) - a.tile_base) * kCostTileFloats;
+                        bulk_g2s(&S.C[bA][0][0], src, kCostHalfBytes, &S.mbar[bA], policy);
+                        bulk_g2s(&S.Phi[bA][0][0], src + kCostHalfFloats, kCostHalfBytes, &S.mbar[bA], policy);
+                    }
+                    res_issue_costs(a, S, bD, J, J, split, policy);
+                }
+                __syncwarp();
+                if (lane < ngv) res_issue_rows(a, S, sDP, bD, J, J, split, lane);
+            }
+            mbar_wait_bounded(&S.mbar[bD], mph[bD] & 1u, a.st, a.abort_flag);
+            mph[bD]++;
+            float2 W[2 * kDiagGroups];
+            diag_prepare(a, S, park, bD, J, split, id, cs, W);
+            int cur = 0;
+            if (J > 0) {  // layer group 0 of tile (J-1, J): rows 2..8 of block J-1
+                if (ct < 32) {
+                    if (lane == 0) wait_lower(a, split, J - 1);
+                    __syncwarp();
+                    fence_proxy_async_global();
+                    if (lane < ngv)
+                        bulk_g2s_nohint(rowsA + (size_t)lane * L * BK, a.dp32 + d32(a, gbase + lane, 2, (int64_t)(J - 1) * BK),
+                                        lo_bytes, &S.mbar[bA]);
+                }
+                mbar_wait_bounded(&S.mbar[bA], mph[bA] & 1u, a.st, a.abort_flag);
+                mph[bA]++;
+                if (own) cons_lasttile_grp(a, S, rowsA, bA, park, (uint32_t)(J - 1), g, id, 0);
+                __syncwarp();
+            }
+            diag_layers(a, S, park, J, split, id, W, 0, LPT - 1, cur);  // layers 3..8
+            diag_store(a, park, J, split, id, 3, 2 + LPT - 1);
+            __syncthreads();  // rows 3..8 and their block minima are stored
+            if (ct == 0) publish_lower(a, split, J);
+            diag_layers(a, S, park, J, split, id, W, LPT - 1, LPT, cur);  // layer 9
+            if (J > 0) {  // layer group 1: rows 9..s-1 of block J-1, after its full publish
+                if (ct < 32) {
+                    if (lane == 0) {
+                        mbar_expect_tx(&S.mbar[bA], (uint32_t)ngv * hi_bytes);
+                        wait_block(a, split, J - 1);
+                    }
+                    __syncwarp();
+                    fence_proxy_async_global();
+                    if (lane < ngv)
+                        bulk_g2s_nohint(rowsA + (size_t)lane * L * BK + LPT * BK,
+                                        a.dp32 + d32(a, gbase + lane, 2 + LPT, (int64_t)(J - 1) * BK), hi_bytes,
+                                        &S.mbar[bA]);
+                }
+                mbar_wait_bounded(&S.mbar[bA], mph[bA] & 1u, a.st, a.abort_flag);
+                mph[bA]++;
+                if (own) cons_lasttile_grp(a, S, rowsA, bA, park, (uint32_t)(J - 1), g, id, 1);
+                __syncwarp();
+                if (own) n_run++;
+            }
+            diag_layers(a, S, park, J, split, id, W, LPT, L, cur);  // layers 10..s
+            diag_store(a, park, J, split, id, 2 + LPT, a.s);
+            __syncthreads();  // every row and block minimum of block J is stored
+            if (ct == 0) publish_block(a, split, J);
+            diag_pair_bands(a, park, J, split, id);
+            n += 2;
+        } else {  // the diagonal tile (issued with the last tile walked, else now)
             const int b = n & 1;
             if (issued != J && ct < 32) res_issue(a, S, sDP, b, J, J, split, policy, lane);
-            mbar_wait_bounded(&S.mbar[b], (n >> 1) & 1u, a.st, a.abort_flag);
+            mbar_wait_bounded(&S.mbar[b], mph[b] & 1u, a.st, a.abort_flag);
+            mph[b]++;
             uint32_t *park = reinterpret_cast<uint32_t *>(sDP + (size_t)2 * rowsDP * BK);
             if (a.lgc == 2)
                 cons_diag_pair(a, S, park, b, J, split, id, cs);
@@ -1803,7 +1994,7 @@ size_t fast_dp_band_bytes(int64_t d, int32_t s) {
     size_t rows = (size_t)kMaxG * (size_t)(s + 1) * (size_t)table_stride(d);
     size_t nJ = (size_t)cdiv(d, BJ);
     return align256(8 * rows) + align256(4 * rows) + align256(4 * NMEM * rows) + align256(rows) +
-           align256(4 * (size_t)kMaxG * nJ + 64) + align256(sizeof(FastParams)) + align256(32 * nJ * (nJ + 1) / 2) +
+           align256(8 * (size_t)kMaxG * nJ + 64) + align256(sizeof(FastParams)) + align256(32 * nJ * (nJ + 1) / 2) +
            align256(4 * (size_t)kMaxG * (size_t)mdp_stride(s) * nJ) +
            align256(2 * 4 * (size_t)kMaxG * (size_t)(s + 1) * (size_t)table_stride(d)) +
            align256(4 * 2 * (size_t)(s + 1));
@@ -1849,7 +2040,7 @@ size_t streamed_costs_bytes(int64_t d) {
 
 int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, const Layout &Lw, cudaStream_t st,
                    bool exact_s, bool exact_tables, float *costs, bool build_costs, bool test_stall,
-                   size_t chunk_bytes) {
+                   size_t chunk_bytes, bool split_off) {
     double *dp64 = wsp<double>(ws, Lw.dp64);
     int32_t *bp = wsp<int32_t>(ws, Lw.bp);
     // small inputs, very large ones and huge counts take the reference kernel
@@ -1888,8 +2079,8 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     base += align256(4 * NMEM * rows);
     a.need = reinterpret_cast<uint8_t *>(base);
     base += align256(rows);
-    int *flags = reinterpret_cast<int *>(base);
-    base += align256(4 * (size_t)kMaxG * (size_t)cdiv(Lw.d, BJ) + 64);
+    int *flags = reinterpret_cast<int *>(base);  // done [kMaxG][nJ], half [kMaxG][nJ], ticket, abort
+    base += align256(8 * (size_t)kMaxG * (size_t)cdiv(Lw.d, BJ) + 64);
     FastParams *dprm = reinterpret_cast<FastParams *>(base);
     base += align256(sizeof(FastParams));
     a.corner = reinterpret_cast<float *>(base);
@@ -1904,6 +2095,8 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     }
     a.mdp_stride = mdp_stride(s);
     a.spin_limit = test_stall ? kTestSpinLimit : kSpinLimit;
+    // two-part publishing of each block (the chain's last tile in two layer groups)
+    a.split_pub = (costs && a.lgc == 2 && !split_off) ? 1 : 0;
     a.hold0 = test_stall ? 1 : 0;
     a.prune = (costs && a.lgc == 2 && a.mdp_stride <= 20) ? 1 : 0;
     a.costs = costs;
@@ -1917,7 +2110,8 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     if (chunk_bytes && cap_tiles < (size_t)a.nJ) return ECASQ_EWORKSPACE;  // one column of tiles must fit
     a.prm = dprm;
     a.done = flags;
-    a.ticket = flags + (size_t)kMaxG * a.nJ;
+    a.half = flags + (size_t)kMaxG * a.nJ;
+    a.ticket = a.half + (size_t)kMaxG * a.nJ;
     a.abort_flag = a.ticket + 1;
     a.st = wsp<DevStatus>(ws, Lw.status);
     float *wf = wsp<float>(ws, Lw.keys1);  // the sort's ping-pong buffer is free now
@@ -1930,7 +2124,7 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     note_launch();
     k_weights_f32<<<(unsigned)cdiv(P.p, 256), 256, 0, st>>>(P.w, wf, P.p);
     ECASQ_LAUNCH_CHECK();
-    ECASQ_CUDA_TRY(cudaMemsetAsync(flags, 0, sizeof(int) * ((size_t)kMaxG * a.nJ + 2), st));
+    ECASQ_CUDA_TRY(cudaMemsetAsync(flags, 0, sizeof(int) * (2 * (size_t)kMaxG * a.nJ + 2), st));
     note_launch();
     k_fast_base<<<(unsigned)cdiv(P.p - 1, 128), 128, 0, st>>>(P, a, dp64, bp);
     ECASQ_LAUNCH_CHECK();

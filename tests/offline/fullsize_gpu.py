@@ -32,9 +32,11 @@ def run(name, out_dir, max_mb):
     x = torch.as_tensor(x_np).cuda()
     d = x.numel()
     flags = E.TIME_KERNELS
-    need = E.ecasq_workspace_size_flags(d, s, 1, E.RESIDENT_COSTS)
-    if 0 < need <= 0.6 * torch.cuda.mem_get_info()[0]:
-        flags |= E.RESIDENT_COSTS
+    for flag in (E.RESIDENT_COSTS, E.STREAMED_COSTS):  # the benchmark's choice of cost mode
+        need = E.ecasq_workspace_size_flags(d, s, 1, flag)
+        if 0 < need <= 0.6 * torch.cuda.mem_get_info()[0]:
+            flags |= flag
+            break
     ws = E.workspace(d, s, flags=flags)
     stream = torch.cuda.current_stream()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)

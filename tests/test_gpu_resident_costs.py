@@ -226,3 +226,33 @@ def test_streamed_costs_budgeted_solve_matches_oracle(E, oracle_mod):
     np.testing.assert_array_equal(Q.cpu().numpy(), o["Q"])
     np.testing.assert_allclose([res["mse"], res["h_surrogate"], res["h_exact"]],
                                [o["mse"], o["h_surrogate"], o["h_exact"]], rtol=MET_RTOL)
+
+
+@pytest.mark.parametrize("name,s", [("lognormal16k", 16), ("studentt9000", 12), ("normal5000", 10)])
+def test_two_part_publish_bit_identical_to_one_part(E, name, s):
+    """Publishing each column block in two parts (rows 2..8 after layer 8, then the rest) lets the
+    next block start its last tile and first layers early; the results are those of the one-part
+    publish: the same tables, resolved and unresolved outputs alike."""
+    if name == "lognormal16k":
+        x = workloads.signed_lognormal(16384, 0)
+    elif name == "studentt9000":
+        x = workloads.student_t(9000, 6)
+    else:
+        x = workloads.normal(5000, 7)
+    lams = [0.0, 1e-4, 0.01, 0.1, 0.4, 1.0, 3.0, 30.0]
+    for costs_flag in (E.RESIDENT_COSTS, E.STREAMED_COSTS):
+        ws1 = E.workspace(x.size, s, flags=costs_flag)
+        ws2 = E.workspace(x.size, s, flags=costs_flag)
+        Q1, m1, met1 = E.ecasq_dp_pass(x, s, lams, flags=costs_flag | E.ONE_PART_PUBLISH, ws=ws1)
+        Q2, m2, met2 = E.ecasq_dp_pass(x, s, lams, flags=costs_flag, ws=ws2)
+        for ws in (ws1, ws2):
+            st = E.native.ws_status(ws)
+            assert st["timeout"] == 0 and st["bound_viol"] == 0
+        assert m1 == m2
+        np.testing.assert_array_equal(Q1.cpu().numpy(), Q2.cpu().numpy())
+        np.testing.assert_array_equal(met1, met2)
+        for (dp1, bp1), (dp2, bp2) in zip(_tables(E, ws1, len(lams), s, x.size), _tables(E, ws2, len(lams), s, x.size)):
+            np.testing.assert_array_equal(dp1, dp2)
+            np.testing.assert_array_equal(bp1, bp2)
+        del ws1, ws2
+        _free()
