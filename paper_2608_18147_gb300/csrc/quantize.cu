@@ -156,74 +156,57 @@ __global__ void __launch_bounds__(kQThreads) k_quantize(const float *__restrict_
 }
 
 // ------------------------------------------------ short codebooks (m <= 16)
-// The same decisions as k_quantize with fewer integer-pipe instructions per entry (the
-// kernel is bound by the integer ALU pipe, not by HBM):
-//  * the search takes STEPS = ceil(log2 m) unrolled steps (a template argument) walking a
-//    pointer into the codebook, so every probe is a load with an immediate offset;
-//  * the draw computes only bits 32..63 of SplitMix64's second product, the bits the rule
-//    reads (k = bits 40..63 of the output, and the final xor-shift by 31 leaves bits 40..63
-//    unchanged), on 32-bit limbs: each 64-bit multiply modulo 2^64 is a wide 32 x 32 product
-//    plus two 32-bit multiply-adds, the top word of the second one a high product plus two;
-//    each right shift is a high product with 2^(32 - shift) and each left shift a product
-//    with 2^shift, both with the power of two passed at run time (FMA-pipe multiplies in
-//    place of ALU-pipe shifts), and a three-way xor joins the two halves of a shifted word;
-//  * the counter state seed + (i + 1) gamma is one wide multiply-add with the seed as addend
-//    plus one multiply-add for the high word;
+// The same decisions as k_quantize with fewer instructions per entry:
+//  * the search takes STEPS = ceil(log2 m) unrolled steps (a template argument), and the
+//    range test compares with q[0] and q[m-1] held in registers;
+//  * the draw computes only bits 32..63 of SplitMix64's second product, the bits the
+//    rule reads (k = bits 40..63 of the output, and the final xor-shift by 31 leaves
+//    bits 40..63 unchanged), with 32-bit limbs: each 64-bit multiply modulo 2^64 is a
+//    wide 32 x 32 product plus two 32-bit multiply-adds, and the top word of the second
+//    one a high product plus two;
 //  * the index counts are per-thread 32-bit counters in shared memory (one column per
 //    thread, no packing and no folding).
-// An entry outside [q_0, q_{m-1}] raises the range error (the call then returns
-// ECASQ_ERANGE; its indices are not meaningful).
 constexpr int kFastBins = 16;
 constexpr uint32_t kC1lo = 0x1CE4E5B9u, kC1hi = 0xBF58476Du;  // SplitMix64 multipliers (Steele, Lea, Flood 2014)
 constexpr uint32_t kC2lo = 0x133111EBu, kC2hi = 0x94D049BBu;
-constexpr uint32_t kGammaLo = 0x7F4A7C15u, kGammaHi = 0x9E3779B9u;
-
-// Powers of two for the shifts, read from kernel arguments at run time.
-struct ShiftPows { uint32_t p2, p4, p5, p32, p24; };  // 2^2 = 4, 2^(32-30) = 4, 2^5, 2^(32-27) = 32, 2^(32-8)
-
-__device__ __forceinline__ uint32_t mulhi(uint32_t a, uint32_t b) { return __umulhi(a, b); }
 
 // Bits 32..63 of the SplitMix64 output for state z = (zh:zl).
-__device__ __forceinline__ uint32_t splitmix64_hi(uint32_t zl, uint32_t zh, const ShiftPows &P) {
-    // x = z ^ (z >> 30): (z >> 30).lo = (zl >> 30) | (zh << 2), (z >> 30).hi = zh >> 30
-    const uint32_t xl = zl ^ mulhi(zl, P.p4) ^ (zh * P.p2), xh = zh ^ mulhi(zh, P.p4);
-    const uint64_t w = (uint64_t)xl * kC1lo;  // a = x * C1 mod 2^64
+__device__ __forceinline__ uint32_t splitmix64_hi(uint32_t zl, uint32_t zh) {
+    const uint32_t xl = zl ^ __funnelshift_r(zl, zh, 30), xh = zh ^ (zh >> 30);  // z ^ (z >> 30)
+    const uint64_t w = (uint64_t)xl * kC1lo;                                       // (xh:xl) * C1 mod 2^64
     const uint32_t al = (uint32_t)w;
     const uint32_t ah = (uint32_t)(w >> 32) + xl * kC1hi + xh * kC1lo;
-    // y = a ^ (a >> 27): (a >> 27).lo = (al >> 27) | (ah << 5), (a >> 27).hi = ah >> 27
-    const uint32_t yl = al ^ mulhi(al, P.p32) ^ (ah * P.p5), yh = ah ^ mulhi(ah, P.p32);
-    return __umulhi(yl, kC2lo) + yl * kC2hi + yh * kC2lo;  // top word of y * C2
-}
-
-// Counter state of entry i: seed + (i + 1) gamma mod 2^64, i + 1 < 2^32.
-__device__ __forceinline__ void counter_state(uint64_t seed, uint32_t n, uint32_t &zl, uint32_t &zh) {
-    const uint64_t z = (uint64_t)n * kGammaLo + seed;  // one wide multiply-add
-    zl = (uint32_t)z;
-    zh = (uint32_t)(z >> 32) + n * kGammaHi;
+    const uint32_t yl = al ^ __funnelshift_r(al, ah, 27), yh = ah ^ (ah >> 27);   // a ^ (a >> 27)
+    return __umulhi(yl, kC2lo) + yl * kC2hi + yh * kC2lo;                         // top word of y * C2
 }
 
 template <int STEPS>
-__device__ __forceinline__ int quant_fast(float xv, uint32_t n, uint64_t seed, const float *q, float q0, float qm,
-                                          const ShiftPows &P, bool &bad) {
-    bad |= !(xv >= q0 && xv <= qm);
-    const float *qp = q;  // largest t with q[t] <= x: qp = q + t
+__device__ __forceinline__ int quant_fast(float xv, uint32_t zl, uint32_t zh, const float *q, float q0, float qm,
+                                          bool &bad) {
+    const bool in = xv >= q0 && xv <= qm;  // outside the codebook's range: index 0 and the error flag
+    bad |= !in;
+    int t = 0;
 #pragma unroll
     for (int s = STEPS - 1; s >= 0; s--)
-        if (qp[1 << s] <= xv) qp += 1 << s;
-    const float a = qp[0], b = qp[1];
-    uint32_t zl, zh;
-    counter_state(seed, n, zl, zh);
-    const float k = __fmul_rn((float)mulhi(splitmix64_hi(zl, zh, P), P.p24), 0x1p-24f);
-    const bool up = a != xv && __fmul_rn(k, __fsub_rn(b, a)) < __fsub_rn(xv, a);
-    return (int)(qp - q) + (up ? 1 : 0);
+        if (q[t + (1 << s)] <= xv) t += 1 << s;
+    const float a = q[t];
+    const float k = __fmul_rn((float)(splitmix64_hi(zl, zh) >> 8), 0x1p-24f);
+    const bool up = a != xv && __fmul_rn(k, __fsub_rn(q[t + 1], a)) < __fsub_rn(xv, a);
+    return in ? t + (up ? 1 : 0) : 0;
+}
+
+// 64-bit counter state (zh:zl) advanced by gamma.
+__device__ __forceinline__ void add_gamma(uint32_t &zl, uint32_t &zh) {
+    const uint64_t z = (((uint64_t)zh << 32) | zl) + kGamma;
+    zl = (uint32_t)z;
+    zh = (uint32_t)(z >> 32);
 }
 
 template <int STEPS>
 __global__ void __launch_bounds__(kQThreads) k_quantize_short(const float *__restrict__ x, int64_t d,
                                                               const float *__restrict__ Q, int m, uint64_t seed,
                                                               uint8_t *__restrict__ idx,
-                                                              uint32_t *__restrict__ counts, DevStatus *st,
-                                                              ShiftPows P) {
+                                                              uint32_t *__restrict__ counts, DevStatus *st) {
     __shared__ float q[2 * kFastBins + 1];
     __shared__ uint32_t ph[kFastBins * kQThreads];  // ph[t * kQThreads + thread]
     for (int r = threadIdx.x; r < 2 * kFastBins + 1; r += blockDim.x) q[r] = r < m ? Q[r] : CUDART_INF_F;
@@ -238,31 +221,36 @@ __global__ void __launch_bounds__(kQThreads) k_quantize_short(const float *__res
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     const int64_t g0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const float4 *x4 = reinterpret_cast<const float4 *>(x);
-    uint32_t *i4 = reinterpret_cast<uint32_t *>(idx);
+    uchar4 *i4 = reinterpret_cast<uchar4 *>(idx);
     for (int64_t g = g0; g < ngroups; g += 2 * stride) {
         const int64_t h = g + stride;
         const bool two = h < ngroups;
         const float4 xa = x4[g];
         const float4 xb = two ? x4[h] : make_float4(q0, q0, q0, q0);
         const float xs[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
-        const uint32_t na = (uint32_t)(4 * g + 1), nb = (uint32_t)(4 * h + 1);  // i + 1 of the first entries
-        uint32_t ts[8];
+        int ts[8];
+        uint64_t za = seed + (uint64_t)(4 * g + 1) * kGamma;  // entry 4g: seed + (4g + 1) gamma
+        uint64_t zb = seed + (uint64_t)(4 * h + 1) * kGamma;
+        uint32_t al = (uint32_t)za, ah = (uint32_t)(za >> 32), bl = (uint32_t)zb, bh = (uint32_t)(zb >> 32);
 #pragma unroll
         for (int r = 0; r < 4; r++) {
-            ts[r] = (uint32_t)quant_fast<STEPS>(xs[r], na + r, seed, q, q0, qm, P, bad);
-            ts[4 + r] = (uint32_t)quant_fast<STEPS>(xs[4 + r], nb + r, seed, q, q0, qm, P, bad);
+            ts[r] = quant_fast<STEPS>(xs[r], al, ah, q, q0, qm, bad);
+            ts[4 + r] = quant_fast<STEPS>(xs[4 + r], bl, bh, q, q0, qm, bad);
+            add_gamma(al, ah);
+            add_gamma(bl, bh);
         }
-        i4[g] = ts[0] + ts[1] * 0x100u + ts[2] * 0x10000u + ts[3] * 0x1000000u;  // four indices, little-endian
+        i4[g] = make_uchar4((uint8_t)ts[0], (uint8_t)ts[1], (uint8_t)ts[2], (uint8_t)ts[3]);
 #pragma unroll
         for (int r = 0; r < 4; r++) myc[ts[r] * kQThreads] += 1u;
         if (two) {
-            i4[h] = ts[4] + ts[5] * 0x100u + ts[6] * 0x10000u + ts[7] * 0x1000000u;
+            i4[h] = make_uchar4((uint8_t)ts[4], (uint8_t)ts[5], (uint8_t)ts[6], (uint8_t)ts[7]);
 #pragma unroll
             for (int r = 4; r < 8; r++) myc[ts[r] * kQThreads] += 1u;
         }
     }
     for (int64_t i = 4 * ngroups + g0; i < d; i += stride) {
-        const int t = quant_fast<STEPS>(x[i], (uint32_t)(i + 1), seed, q, q0, qm, P, bad);
+        const uint64_t z = seed + (uint64_t)(i + 1) * kGamma;
+        const int t = quant_fast<STEPS>(x[i], (uint32_t)z, (uint32_t)(z >> 32), q, q0, qm, bad);
         idx[i] = (uint8_t)t;
         myc[t * kQThreads] += 1u;
     }
@@ -287,13 +275,12 @@ int launch_quantize(const float *x, int64_t d, const float *Q, int m, uint64_t s
     if (m <= kFastBins) {
         // STEPS = ceil(log2 m): the search visits q[t + 2^s] for s < STEPS
         const int steps = m > 1 ? 32 - __builtin_clz((unsigned)(m - 1)) : 0;
-        const ShiftPows P{4u, 4u, 32u, 32u, 1u << 24};
         switch (steps) {
-            case 0: k_quantize_short<0><<<(unsigned)blocks, kQThreads, 0, stream>>>(x, d, Q, m, seed, idx, counts, st, P); break;
-            case 1: k_quantize_short<1><<<(unsigned)blocks, kQThreads, 0, stream>>>(x, d, Q, m, seed, idx, counts, st, P); break;
-            case 2: k_quantize_short<2><<<(unsigned)blocks, kQThreads, 0, stream>>>(x, d, Q, m, seed, idx, counts, st, P); break;
-            case 3: k_quantize_short<3><<<(unsigned)blocks, kQThreads, 0, stream>>>(x, d, Q, m, seed, idx, counts, st, P); break;
-            default: k_quantize_short<4><<<(unsigned)blocks, kQThreads, 0, stream>>>(x, d, Q, m, seed, idx, counts, st, P); break;
+            case 0: k_quantize_short<0><<<(unsigned)blocks, kQThreads, 0, stream>>>(x, d, Q, m, seed, idx, counts, st); break;
+            case 1: k_quantize_short<1><<<(unsigned)blocks, kQThreads, 0, stream>>>(x, d, Q, m, seed, idx, counts, st); break;
+            case 2: k_quantize_short<2><<<(unsigned)blocks, kQThreads, 0, stream>>>(x, d, Q, m, seed, idx, counts, st); break;
+            case 3: k_quantize_short<3><<<(unsigned)blocks, kQThreads, 0, stream>>>(x, d, Q, m, seed, idx, counts, st); break;
+            default: k_quantize_short<4><<<(unsigned)blocks, kQThreads, 0, stream>>>(x, d, Q, m, seed, idx, counts, st); break;
         }
     } else if (m <= kPrivBins)
         k_quantize<true><<<(unsigned)blocks, kQThreads, 0, stream>>>(x, d, Q, m, seed, idx, counts, st);
