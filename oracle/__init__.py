@@ -65,6 +65,7 @@ def _load():
             "or_phi": (dbl, [P, i64, i64, i32]),
             "or_apx_dp": (i32, [P, i32, dbl, i32, pd, pi32, pd, pi64, pi32, pd]),
             "or_apx_dp_columns": (i32, [P, i32, dbl, i32, pd, pi32, pd, pi64, pi32, pd]),
+            "or_apx_dp_linear": (i32, [P, i32, dbl, i32, pi64, pi32, pd]),
             "or_dp_decision": (None, [P, pd, i32, i64, dbl, pd, pi64, pd]),
             "or_dp_candidate": (dbl, [P, dbl, i64, i64, dbl, i32]),
             "or_eval_idx": (i32, [P, pi64, i32, pd]),
@@ -189,6 +190,18 @@ class Hist:
         if tables:
             out.update(dp=dp.reshape(rows, p), bp=bp.reshape(rows, p), margin=mg.reshape(rows, p))
         return out
+
+    def apx_dp_linear(self, s, lam_prime, exact_s=False):
+        """Linear-space traceback of the approximate DP (Sec. 5, Hirschberg's method):
+        (codebook indices, m, dp(m, p-1)); O(p) memory."""
+        Q = np.empty(s + 1, np.int64)
+        m = C.c_int32()
+        best = C.c_double()
+        st = _load().or_apx_dp_linear(self._h, int(s), float(lam_prime), int(bool(exact_s)), _ptr(Q, C.c_int64),
+                                      C.byref(m), C.byref(best))
+        if st != OK:
+            raise OracleError(st, "or_apx_dp_linear")
+        return Q[:m.value].copy(), m.value, best.value
 
     def dp_decision(self, prev, i, j, lam_prime):
         """min over k of prev[k] + C[k,j] + lambda' Phi[k,j] (eq. apx_rec), one output."""

@@ -25,6 +25,8 @@
  *   or_apx_dp        Sec. 5, eqs. apx_base / apx_rec / apx_final
  *   or_apx_dp_columns the same DP evaluated column by column (each pair's link
  *                    cost computed once for all layers), for full-size checks
+ *   or_apx_dp_linear Sec. 5 (last paragraph): the codebook of the same DP in linear
+ *                    space (forward and backward passes, split at a middle value)
  *   or_dp_decision,  one output / one candidate of eq. apx_rec (eq. apx_base with
  *   or_dp_candidate  `first`), for checking sampled outputs of large GPU runs
  *   or_eval_idx      Sec. 2 (MSE), Sec. 3 (H(Xhat)), Sec. 5 eq. apx_additive_entropy
@@ -550,6 +552,127 @@ int32_t or_apx_dp_columns(const or_hist *H, int32_t s, double lam_prime, int32_t
     if (bp_out) memcpy(bp_out, bp, sizeof(int32_t) * rows * (size_t)p);
     if (margin_out) memcpy(margin_out, mg, sizeof(double) * rows * (size_t)p);
     free(dp); free(bp); free(mg);
+    return OR_OK;
+}
+
+/* Linear-space traceback of the approximate DP (Sec. 5, last paragraph: Hirschberg's
+ * method specialised to eq. apx_rec).  Link cost of consecutive values k < j:
+ * C[k, j] + lambda' Phi[k, j], with Phi^first when k is the first value (index 0, P = X).
+ *   1. A forward pass over the layers of eq. apx_rec keeping two rows finds the answer of
+ *      eq. apx_final: m = the smallest i with the least dp(i, p-1).
+ *   2. Subproblem (u, v, n): the n values of the chain with u and v fixed at its ends.
+ *      For n >= 3 the middle position is t = (n + 1) / 2.  The forward pass from u gives
+ *      G(c), the least cost of a chain of t values from u to c; the backward pass to v
+ *      gives B(c), the least cost of a chain of n - t + 1 values from c to v (suffix
+ *      costs, links taken from the right).  The middle value is the lowest c, u < c < v,
+ *      among the exact binary64 minima of G(c) + B(c); recurse on (u, c, t) and
+ *      (c, v, n - t + 1).  Each pass keeps two rows of p values.
+ * Reading (the paper gives none): ties of G + B go to the lowest c.  The sums G + B add
+ * a prefix and a suffix cost, in a different order from the forward recurrence, so at
+ * exact or near ties the codebook may differ from or_apx_dp's (whose traceback takes
+ * the lowest k at every step from the end); its objective is the same optimum.
+ * Q_idx receives the codebook, m its size, best = dp(m, p-1) of the forward pass. */
+static double link_cost(const or_hist *H, int64_t k, int64_t j, double lam_prime) {
+    double C, U, D;
+    pair_q(H, k, j, &C, &U, &D);
+    return C + lam_prime * phi_of(H, U, D, k == 0 ? 0 : -1);
+}
+
+int32_t or_apx_dp_linear(const or_hist *H, int32_t s, double lam_prime, int32_t exact_s, int64_t *Q_idx,
+                         int32_t *m_out, double *best_out) {
+    int64_t p = H->p;
+    if (s < 2 || H->nL != 1 || H->nR != 1) return OR_EINVAL;
+    if (p == 1) { Q_idx[0] = 0; *m_out = 1; *best_out = 0.0; return OR_OK; }
+    double *r0 = (double *)malloc(sizeof(double) * (size_t)p);
+    double *r1 = (double *)malloc(sizeof(double) * (size_t)p);
+    double *r2 = (double *)malloc(sizeof(double) * (size_t)p);
+    double *r3 = (double *)malloc(sizeof(double) * (size_t)p);
+    int64_t *stk = (int64_t *)malloc(sizeof(int64_t) * 3 * (size_t)(s + 2));
+    if (!r0 || !r1 || !r2 || !r3 || !stk) { free(r0); free(r1); free(r2); free(r3); free(stk); return OR_ENOMEM; }
+    /* 1. forward pass: dp(i, p-1) for every i */
+    double best = INFINITY;
+    int32_t m = -1;
+    double *prev = r0, *cur = r1;
+    for (int64_t j = 0; j < p; j++) prev[j] = INFINITY;
+    for (int64_t j = 1; j < p; j++) prev[j] = link_cost(H, 0, j, lam_prime);  /* layer 2 */
+    for (int32_t i = 2; i <= s; i++) {
+        if (i > 2) {
+            for (int64_t j = 0; j < p; j++) cur[j] = INFINITY;
+#pragma omp parallel for schedule(dynamic, 8)
+            for (int64_t j = i - 1; j < p; j++) {
+                double b = INFINITY;
+                for (int64_t k = i - 2; k < j; k++) {
+                    double c = prev[k] + link_cost(H, k, j, lam_prime);
+                    if (c < b) b = c;
+                }
+                cur[j] = b;
+            }
+            double *t = prev; prev = cur; cur = t;
+        }
+        if ((!exact_s || i == s) && prev[p - 1] < best) { best = prev[p - 1]; m = i; }
+    }
+    if (m < 0) { free(r0); free(r1); free(r2); free(r3); free(stk); return OR_EINFEASIBLE; }
+    /* 2. the chain, by splitting at middle values */
+    Q_idx[0] = 0;
+    Q_idx[m - 1] = p - 1;
+    int32_t top = 0;
+    stk[0] = 0; stk[1] = p - 1; stk[2] = m;  /* (u, v, n); Q_idx position of u = pos below */
+    int64_t *pos = (int64_t *)malloc(sizeof(int64_t) * (size_t)(s + 2));
+    pos[0] = 0;
+    top = 1;
+    while (top > 0) {
+        top--;
+        int64_t u = stk[3 * top], v = stk[3 * top + 1], n = stk[3 * top + 2], pu = pos[top];
+        if (n <= 2) continue;
+        int64_t t = (n + 1) / 2;
+        /* forward from u: G_r(c) for c in (u, v), r = 2..t */
+        double *G = r0, *Gn = r1;
+        for (int64_t c = u; c <= v; c++) G[c] = INFINITY;
+        for (int64_t c = u + 1; c < v; c++) G[c] = link_cost(H, u, c, lam_prime);
+        for (int64_t r = 3; r <= t; r++) {
+            for (int64_t c = u; c <= v; c++) Gn[c] = INFINITY;
+#pragma omp parallel for schedule(dynamic, 8)
+            for (int64_t c = u + r - 1; c < v; c++) {
+                double b = INFINITY;
+                for (int64_t k = u + r - 2; k < c; k++) {
+                    double x = G[k] + link_cost(H, k, c, lam_prime);
+                    if (x < b) b = x;
+                }
+                Gn[c] = b;
+            }
+            double *tt = G; G = Gn; Gn = tt;
+        }
+        /* backward to v: B_r(c) for c in (u, v), r = 2..n-t+1 */
+        double *B = r2, *Bn = r3;
+        for (int64_t c = u; c <= v; c++) B[c] = INFINITY;
+        for (int64_t c = u + 1; c < v; c++) B[c] = link_cost(H, c, v, lam_prime);
+        for (int64_t r = 3; r <= n - t + 1; r++) {
+            for (int64_t c = u; c <= v; c++) Bn[c] = INFINITY;
+#pragma omp parallel for schedule(dynamic, 8)
+            for (int64_t c = u + 1; c <= v - (r - 1); c++) {
+                double b = INFINITY;
+                for (int64_t j = c + 1; j <= v - (r - 2); j++) {
+                    double x = link_cost(H, c, j, lam_prime) + B[j];
+                    if (x < b) b = x;
+                }
+                Bn[c] = b;
+            }
+            double *tt = B; B = Bn; Bn = tt;
+        }
+        int64_t cs = -1;
+        double sb = INFINITY;
+        for (int64_t c = u + 1; c < v; c++) {
+            double x = G[c] + B[c];
+            if (x < sb) { sb = x; cs = c; }
+        }
+        if (cs < 0) { free(r0); free(r1); free(r2); free(r3); free(stk); free(pos); return OR_EINFEASIBLE; }
+        Q_idx[pu + t - 1] = cs;
+        stk[3 * top] = u; stk[3 * top + 1] = cs; stk[3 * top + 2] = t; pos[top] = pu; top++;
+        stk[3 * top] = cs; stk[3 * top + 1] = v; stk[3 * top + 2] = n - t + 1; pos[top] = pu + t - 1; top++;
+    }
+    *m_out = m;
+    *best_out = best;
+    free(r0); free(r1); free(r2); free(r3); free(stk); free(pos);
     return OR_OK;
 }
 
