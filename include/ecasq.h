@@ -262,6 +262,29 @@ int ecasq_dp_pass(const float *x, int64_t d, int32_t s, const double *lambdas, i
 int ecasq_dp_tables(void *ws, size_t ws_bytes, int32_t g, double *dp_out, int32_t *bp_out, int64_t *p_out,
                     ecasq_stream_t stream);
 
+/* Linear-space traceback of the approximate DP (Sec. 5, last paragraph: Hirschberg's
+ * method on eq. apx_rec), one multiplier `lambda` (vNMSE scale, lambda' = lambda ||X||^2),
+ * P = X.  Memory O(d): the workspace holds the histogram and prefix sums, four DP rows and
+ * a few scalars (ecasq_workspace_size_linear(d), about 124 d bytes) -- no table of
+ * backpointers.  A forward pass over the layers of eq. apx_rec (two rows) gives dp(i, p-1)
+ * and the answer of eq. apx_final (m = the smallest i with the least value; ECASQ_EXACT_S:
+ * i = s).  The chain of m values is then rebuilt by splitting subproblems (u, v, n) -- n
+ * values with u and v fixed at the ends -- at the middle position t = (n + 1) / 2: the
+ * middle value is the lowest c among the exact binary64 minima of G(c) + B(c), G the least
+ * cost of a chain of t values from u to c (forward pass), B of n - t + 1 values from c to v
+ * (backward pass over suffix costs).  All costs are binary64 with the reference interval
+ * quantities (the values of ECASQ_DP_REFERENCE).  The optimum is the one of eq. apx_final;
+ * at exact ties of G + B the codebook may differ from the backpointer traceback's (which
+ * takes the lowest k at every step from the end).  Time O(s d^2) pair evaluations.
+ * Q_out [s] device (first m entries), m_out host, metrics host [4]: dp(m, p-1) (the
+ * surrogate Lagrangian of eq. apx_final), MSE, H(I,B), H(Xhat) of the codebook.
+ * ECASQ_EINVAL for d < 1, s outside [2, 256] or a negative / non-finite lambda;
+ * ECASQ_EINFEASIBLE when no codebook of the required size exists (ECASQ_EXACT_S with
+ * s above the number of unique values).  Synchronises `stream`. */
+size_t ecasq_workspace_size_linear(int64_t d);
+int ecasq_dp_linear(const float *x, int64_t d, int32_t s, double lambda, uint32_t flags, void *ws, size_t ws_bytes,
+                    float *Q_out, int32_t *m_out, double *metrics, ecasq_stream_t stream);
+
 /* Three-colour refinement (Sec. 6) of a codebook Q subset of X at a fixed
  * multiplier, minimising MSE + lambda' H(Xhat): colours 0, 1, 2 in turn move
  * each interior value with index % 3 == colour to the best unique input value

@@ -52,6 +52,9 @@ size_t opt_tables_bytes(int64_t n, int s, int G);
 int launch_opt_dp(const Prefix &P, const double *lamp, int G, int s, int exact_s, void *pairs, bool build_pairs,
                   void *tables, int32_t *qidx, int32_t *mcount, double *metrics, int num_sms, cudaStream_t st);
 
+int launch_dp_linear(const Prefix &P, double lam, int s, int exact_s, double *rows, double *col, void *small,
+                     std::vector<int32_t> &qidx_host, int *m_out, double *best, cudaStream_t st);
+
 static std::atomic<long long> g_launches{0};
 void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
@@ -1032,6 +1035,70 @@ int ecasq_quantize_noalloc(const float *x, int64_t d, const float *Q, int32_t m,
         }
         *h_emp = he;
     }
+    return ECASQ_OK;
+}
+
+// Linear-space traceback (Sec. 5, last paragraph): the preparation layout, then four DP
+// rows of d + 1 doubles, the column dp(i, p-1), the codebook and a little scratch.
+struct LinearLayout { Layout prep; size_t rows, col, qidx, mcount, small, total; };
+static bool linear_layout(int64_t d, LinearLayout *LL) {
+    if (d < 1 || d >= ((int64_t)1 << 31)) return false;
+    size_t off = make_prep_layout(d, &LL->prep);
+    auto take = [&](size_t bytes) { size_t o = off; off += align256(bytes); return o; };
+    LL->rows = take(4 * 8 * (size_t)(d + 1));
+    LL->col = take(8 * (size_t)(kMaxS + 1));
+    LL->qidx = take(4 * (size_t)kMaxS);
+    LL->mcount = take(4);
+    LL->small = take(64);
+    LL->total = off;
+    return true;
+}
+
+size_t ecasq_workspace_size_linear(int64_t d) {
+    LinearLayout LL;
+    return linear_layout(d, &LL) ? LL.total : 0;
+}
+
+int ecasq_dp_linear(const float *x, int64_t d, int32_t s, double lambda, uint32_t flags, void *ws, size_t ws_bytes,
+                    float *Q_out, int32_t *m_out, double *metrics, ecasq_stream_t stream) {
+    if (!x || !Q_out || !m_out || !metrics || s < 2 || s > kMaxS || !(lambda >= 0.0) || !isfinite(lambda))
+        return ECASQ_EINVAL;
+    LinearLayout LL;
+    if (!linear_layout(d, &LL)) return ECASQ_EINVAL;
+    int rc = check_ws(ws, ws_bytes, LL.prep);
+    if (rc) return rc;
+    if (ws_bytes < LL.total) return ECASQ_EWORKSPACE;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    int64_t p;
+    double n2;
+    rc = prepare_device(x, d, ws, LL.prep, st, &p, &n2);
+    if (rc) return rc;
+    Prefix P = make_prefix(ws, LL.prep, p, d);
+    std::vector<int32_t> a;
+    int m = 0;
+    double best = 0.0;
+    rc = launch_dp_linear(P, lambda * n2, s, (flags & ECASQ_EXACT_S) ? 1 : 0, wsp<double>(ws, LL.rows),
+                          wsp<double>(ws, LL.col), wsp<void>(ws, LL.small), a, &m, &best, st);
+    if (rc) return rc;
+    int32_t *qi = wsp<int32_t>(ws, LL.qidx);
+    int32_t *mc = wsp<int32_t>(ws, LL.mcount);
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(qi, a.data(), sizeof(int32_t) * m, cudaMemcpyHostToDevice, st));
+    ECASQ_CUDA_TRY(cudaMemcpyAsync(mc, &m, sizeof(int32_t), cudaMemcpyHostToDevice, st));
+    rc = launch_gather_q(P.v, qi, mc, 1, kMaxS, Q_out, st);
+    if (rc) return rc;
+    double ev[3] = {0.0, 0.0, 0.0};
+    if (m >= 2) {
+        double *o = wsp<double>(ws, LL.small) + 4;
+        rc = launch_eval_codebook(P, qi, m, o, st);
+        if (rc) return rc;
+        ECASQ_CUDA_TRY(cudaMemcpyAsync(ev, o, 3 * sizeof(double), cudaMemcpyDeviceToHost, st));
+    }
+    ECASQ_CUDA_TRY(cudaStreamSynchronize(st));
+    *m_out = m;
+    metrics[0] = best;
+    metrics[1] = ev[0];
+    metrics[2] = ev[1];
+    metrics[3] = ev[2];
     return ECASQ_OK;
 }
 

@@ -99,6 +99,8 @@ def lib():
                                                    vp]),
             "ecasq_dp_pass": (C.c_int, [vp, i64, i32, pd, i32, u32, vp, sz, vp, pi32, pd, vp]),
             "ecasq_dp_tables": (C.c_int, [vp, sz, i32, vp, vp, pi64, vp]),
+            "ecasq_workspace_size_linear": (sz, [i64]),
+            "ecasq_dp_linear": (C.c_int, [vp, i64, i32, dbl, u32, vp, sz, vp, pi32, pd, vp]),
             "ecasq_refine": (C.c_int, [vp, i64, vp, i32, dbl, dbl, i32, dbl, u32, vp, sz, PR, vp]),
             "ecasq_evaluate": (C.c_int, [vp, i64, vp, i32, vp, sz, pd, vp]),
             "ecasq_quantize": (C.c_int, [vp, i64, vp, i32, u64, vp, vp, vp, sz, pd, vp]),
@@ -123,7 +125,7 @@ def exported_symbols():
                  "ecasq_solve", "ecasq_solve_grid", "ecasq_workspace_size_grid", "ecasq_solve_timeshare",
                  "ecasq_quantize_timeshare", "ecasq_workspace_size_opt", "ecasq_workspace_size_prep", "ecasq_opt_dp",
                  "ecasq_dp_pass",
-                 "ecasq_dp_tables", "ecasq_refine", "ecasq_evaluate", "ecasq_quantize", "ecasq_quantize_noalloc",
+                 "ecasq_dp_tables", "ecasq_workspace_size_linear", "ecasq_dp_linear", "ecasq_refine", "ecasq_evaluate", "ecasq_quantize", "ecasq_quantize_noalloc",
                  "ecasq_solve_batched",
                  "ecasq_prepare", "ecasq_kernel_launches"):
         if hasattr(L, name):
@@ -341,6 +343,26 @@ def ecasq_dp_pass(x, s, lambdas, flags=0, ws=None):
                              _ptr(ws), ws.numel(), _ptr(Q), m, met.ctypes.data_as(C.POINTER(C.c_double)), _stream())
     _check(rc, "ecasq_dp_pass")
     return Q, list(m), met.reshape(G, 4)
+
+
+def ecasq_dp_linear(x, s, lambda_, flags=0, ws=None):
+    """Linear-space traceback of the approximate DP at one multiplier (vNMSE scale):
+    (Q tensor [m], metrics [4] = dp(m, p-1), MSE, H(I,B), H(Xhat))."""
+    torch = _torch()
+    x = _dev_f32(x)
+    d = x.numel()
+    if ws is None:
+        nb = int(lib().ecasq_workspace_size_linear(d))
+        if nb == 0:
+            raise EcasqError(EINVAL, "ecasq_workspace_size_linear")
+        ws = torch.empty(nb, dtype=torch.uint8, device=x.device)
+    Q = torch.zeros(s, dtype=torch.float32, device=x.device)
+    m = C.c_int32()
+    met = np.zeros(4, np.float64)
+    rc = lib().ecasq_dp_linear(_ptr(x), d, int(s), float(lambda_), int(flags), _ptr(ws), ws.numel(), _ptr(Q),
+                               C.byref(m), met.ctypes.data_as(C.POINTER(C.c_double)), _stream())
+    _check(rc, "ecasq_dp_linear")
+    return Q[:m.value].clone(), met
 
 
 def ecasq_dp_tables(ws, g, s, p_max):
