@@ -68,7 +68,8 @@ def parse():
     ap.add_argument("--config", default="studentt_d131072_s16")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--mode", default="solve", choices=["solve", "grid", "timeshare", "opt", "hbm", "rows", "pass"])
+    ap.add_argument("--mode", default="solve",
+                    choices=["solve", "grid", "timeshare", "opt", "hbm", "rows", "pass", "linear"])
     ap.add_argument("--lambdas", default="0.02", help="comma-separated multipliers (vNMSE scale) for --mode pass")
     ap.add_argument("--grid", type=int, default=256, help="grid size for --mode grid")
     ap.add_argument("--prefix", type=int, default=0,
@@ -247,6 +248,9 @@ def run_other_mode(args, cfg, x_np):
         return
     if args.mode == "pass":
         run_pass_mode(args, cfg, x_np)
+        return
+    if args.mode == "linear":
+        run_linear_mode(args, cfg, x_np)
         return
     if args.mode == "grid":
         g = torch.as_tensor(E.uniform_grid(x_np, args.grid)).cuda()
@@ -434,6 +438,37 @@ def run_pass_mode(args, cfg, x_np):
                       "cost_tiles_fetched": st["tiles_fetched"],
                       "executed_candidates": executed_candidates(st, p, s, len(lams))},
            "m": list(outs[-1][1]), "gpu_launches": E.ecasq_kernel_launches() - launches0, "clocks": clocks}
+    print(json.dumps(out), flush=True)
+
+
+def run_linear_mode(args, cfg, x_np):
+    """The linear-space traceback (Sec. 5, last paragraph) of the configuration's vector (or
+    its first --prefix entries) at the first multiplier of --lambdas: ms per call.  The
+    throughput unit is the forward recurrence's candidate count (the splits' forward and
+    backward passes roughly double the work)."""
+    import torch
+    import paper_2608_18147_gb300 as E
+    s = cfg["s"]
+    lam = float(args.lambdas.split(",")[0])
+    if args.prefix > 0:
+        x_np = x_np[:args.prefix]
+    x = torch.as_tensor(x_np).cuda()
+    d = x.numel()
+    ws = torch.empty(int(E.lib().ecasq_workspace_size_linear(d)), dtype=torch.uint8, device="cuda")
+    launches0 = E.ecasq_kernel_launches()
+    ms, outs, clocks = _timed_steps(args, lambda: E.ecasq_dp_linear(x, s, lam, ws=ws))
+    Q, met = outs[-1]
+    p = E.native.ws_status(ws)["p"]
+    cand = candidates_per_multiplier(p, s)
+    out = {"metric": "ECASQ linear-space traceback: candidate evals/s of the forward recurrence", "unit": UNIT,
+           "value": args.steps * cand / (ms / 1000.0), "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": ms / args.steps, "higher_is_better": True, "vs_baseline": None,
+           "dtype": "f64", "data": "synthetic",
+           "config": {"workload": args.config + (" (first %d entries)" % d if args.prefix > 0 else ""),
+                      "mode": "linear", "d": d, "p": p, "s": s, "lambda": lam,
+                      "workspace_mb": round(ws.numel() / 2 ** 20, 2)},
+           "m": int(Q.numel()), "objective": float(met[0]),
+           "gpu_launches": E.ecasq_kernel_launches() - launches0, "clocks": clocks}
     print(json.dumps(out), flush=True)
 
 
