@@ -214,7 +214,8 @@ static size_t rows_layout(int64_t d, int32_t s, int64_t rows, RowsLayout *R) {
     R->sel = take(4 * n * (size_t)s);
     R->m = take(4 * n);
     const int64_t pm = std::min<int64_t>(d, kRowsMaxP);
-    R->pstride = pm * (pm - 1) + pm;
+    // binary64 {C, Phi} by pair, Phi^first, fp32 {C, Phi} by pair; even, so rows start on 16 bytes
+    R->pstride = (3 * (pm * (pm - 1) / 2) + pm + 1) & ~(int64_t)1;
     R->pairs = take(8 * n * (size_t)R->pstride);
     R->total = off;
     return off;

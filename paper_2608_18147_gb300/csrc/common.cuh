@@ -165,9 +165,11 @@ struct RowsPass {
     int32_t *qidx;        // [nact][G][s]
     int32_t *mcount;      // [nact][G]
     double *metrics;      // [nact][G][4]
-    double *pairs;        // [rows][pstride]: the row's C, Phi (pair order) and Phi^first, kept across rounds
-    int64_t pstride;      // doubles per row: 2 npair(pmax) + pmax
+    double *pairs;        // [rows][pstride]: the row's binary64 {C, Phi} by pair, Phi^first and fp32
+                          // {C scale, Phi} by pair, kept across rounds
+    int64_t pstride;      // doubles per row: 3 npair(pmax) + pmax
     int pairs_ready;      // the rows' interval costs are already in `pairs`
+    int bp_smem;          // backpointers in shared memory (set by the launcher)
 };
 
 // Prefix-sum view (App. E) used by every exact pair evaluation.

@@ -189,20 +189,40 @@ __global__ void __launch_bounds__(256) k_rows_pass(RowsPass A) {
     P.d = R.d;
     P.ps = p;
     const int npair = p * (p - 1) / 2;
-    double *Cs = rsm;                    // [npair]
-    double *Ph = Cs + npair;             // [npair]
-    double *PhF = Ph + npair;            // [p]   Phi^first[0, j]
-    double *dpb = PhF + p;               // [2][G][p]
-    double *last = dpb + 2 * G * p;      // [G][s+1] dp(i, p-1)
+    double *PhF = rsm;                    // [p]   Phi^first[0, j]
+    double *dpb = PhF + p;                // [2][G][p] binary64 layers
+    double *last = dpb + 2 * G * p;       // [G][s+1] dp(i, p-1)
     double *scratch = last + G * (s + 1);  // [4 kMaxS] evaluation scratch
+    // [npair] {C scale, Phi}, k-major: pair (k, j) at koff(k) + j - k - 1, koff(k) = k p - k (k + 1) / 2,
+    // so the lanes of a warp (consecutive j, one k) read consecutive words
+    float2 *pc32 = reinterpret_cast<float2 *>(scratch + 4 * kMaxS);
+    float *d32 = reinterpret_cast<float *>(pc32 + npair);            // [2][G][p] dp scale, fp32
+    // backpointers: read only by this block's traceback, so they stay in shared memory
+    // (int8: a row has at most kRowsMaxP = 128 unique values) unless that does not fit
+    int8_t *bps = reinterpret_cast<int8_t *>(d32 + 2 * (size_t)G * p);  // [G][s+1][p]
     __shared__ int32_t a_sm[kMaxS];
     __shared__ int sm_m;
-    double lam[kMaxG];
-#pragma unroll
-    for (int g = 0; g < kMaxG; g++) lam[g] = g < G ? A.lam[(size_t)b * G + g] : 0.0;
-    double *gp = A.pairs + row * A.pstride;  // the same three arrays, kept across rounds
+    // the row's scale 2^-e (2^e <= ||X_row||^2 < 2^(e+1)) keeps the fp32 copies near 1
+    const double n2 = R.norm2[row];
+    const double scale = (n2 > 0.0 && isfinite(n2)) ? ldexp(1.0, -ilogb(n2)) : 1.0;
+    __shared__ double lam[kMaxG], slack[kMaxG];
+    __shared__ float lam32[kMaxG];
+    if (threadIdx.x < kMaxG) {
+        const int g = threadIdx.x;
+        lam[g] = g < G ? A.lam[(size_t)b * G + g] : 0.0;
+        lam32[g] = __double2float_rn(__dmul_rn(lam[g], scale));
+        slack[g] = 3.0 * (70.0 + (double)lam32[g]) * 0x1p-150;
+    }
+    // the row's interval costs, kept across rounds in `pairs`: binary64 {C, Phi} by pair,
+    // Phi^first, and the fp32 copies
+    // (plain 8-byte accesses: a row's cache starts on a multiple of 8 bytes, not of 16)
+    double *gp = A.pairs + row * A.pstride;
+    double *gpc64 = gp;  // {C, Phi} of pair t at gpc64[2 t], gpc64[2 t + 1]
+    double *gphf = gp + 2 * (size_t)npair;
+    float2 *gpc32 = reinterpret_cast<float2 *>(gphf + p);
     if (A.pairs_ready) {
-        for (int t = threadIdx.x; t < 2 * npair + p; t += blockDim.x) Cs[t] = gp[t];
+        for (int t = threadIdx.x; t < npair; t += blockDim.x) pc32[t] = gpc32[t];
+        for (int t = threadIdx.x; t < p; t += blockDim.x) PhF[t] = gphf[t];
     } else {
         for (int t = threadIdx.x; t < npair; t += blockDim.x) {
             int j = (int)((1.0 + sqrt(1.0 + 8.0 * (double)t)) * 0.5);
@@ -211,42 +231,72 @@ __global__ void __launch_bounds__(256) k_rows_pass(RowsPass A) {
             int k = t - j * (j - 1) / 2;
             double C, U, D;
             pair_exact(P, k, j, C, U, D);
-            Cs[t] = C;
-            Ph[t] = phi_exact(P, U, D, false);
-            if (k == 0) PhF[j] = phi_exact(P, U, D, true);
+            const double F = phi_exact(P, U, D, false);
+            gpc64[2 * (size_t)t] = C;
+            gpc64[2 * (size_t)t + 1] = F;
+            const float2 c32 = make_float2(__double2float_rn(__dmul_rn(C, scale)), __double2float_rn(F));
+            const int r = k * p - k * (k + 1) / 2 + (j - k - 1);
+            pc32[r] = c32;
+            gpc32[r] = c32;
+            if (k == 0) { PhF[j] = phi_exact(P, U, D, true); gphf[j] = PhF[j]; }
         }
-        __syncthreads();
-        for (int t = threadIdx.x; t < 2 * npair + p; t += blockDim.x) gp[t] = Cs[t];
     }
     for (int q = threadIdx.x; q < G * (s + 1); q += blockDim.x) last[q] = CUDART_INF;
     int32_t *bp = A.bp + (size_t)b * G * (s + 1) * dcap;
+    const bool bp_sm = A.bp_smem != 0;
+    auto set_bp = [&](int g, int i, int j, int32_t v) {
+        if (bp_sm) bps[((size_t)g * (s + 1) + i) * p + j] = (int8_t)v;
+        else bp[((size_t)g * (s + 1) + i) * dcap + j] = v;
+    };
     __syncthreads();
     // eq. apx_base: dp(2, j) = C[0, j] + lambda' Phi^first[0, j]
     for (int q = threadIdx.x; q < G * p; q += blockDim.x) {
         int g = q / p, j = q % p;
         double v = CUDART_INF;
         int32_t arg = -1;
-        if (j >= 1) { v = __dadd_rn(Cs[tri(0, j)], __dmul_rn(lam[g], PhF[j])); arg = 0; }
+        if (j >= 1) { v = __dadd_rn(gpc64[2 * (size_t)tri(0, j)], __dmul_rn(lam[g], PhF[j])); arg = 0; }
         dpb[g * p + j] = v;
-        bp[((size_t)g * (s + 1) + 2) * dcap + j] = arg;
+        d32[g * p + j] = __double2float_rn(__dmul_rn(v, scale));
+        set_bp(g, 2, j, arg);
         if (j == p - 1) last[g * (s + 1) + 2] = v;
     }
     __syncthreads();
-    // eq. apx_rec, layers 3..s
+    // eq. apx_rec, layers 3..s: an fp32 pass over k finds the fp32 minimum m32; every k whose
+    // fp32 candidate is within the certified band of m32 is re-scored with the binary64
+    // candidate, and the lowest k among the exact minima wins (the result of the binary64
+    // recurrence, bit for bit).  The band, as in the grid DP: all terms are >= 0, each fp32
+    // input is within u = 2^-24 (relative) of its binary64 value or 2^-150 (absolute) when
+    // subnormal, the fma and the add round once each, so an exact minimiser has
+    // val32 <= (m32 + A)(1 + 8.0001u) + A < m32 (1 + 10u) + 3A, A = (70 + lam32) 2^-150.
     int cur = 0;
     for (int i = 3; i <= s; i++) {
         const double *prev = dpb + (size_t)cur * G * p;
+        const float *prev32 = d32 + (size_t)cur * G * p;
         double *nxt = dpb + (size_t)(cur ^ 1) * G * p;
+        float *nxt32 = d32 + (size_t)(cur ^ 1) * G * p;
         for (int q = threadIdx.x; q < G * p; q += blockDim.x) {
-            int g = q / p, j = q % p;
+            const int g = q / p, j = q % p;
+            const int tb = j * (j - 1) / 2;
+            const int koff0 = (i - 2) * p - (i - 2) * (i - 1) / 2 - 1;  // koff(i - 2) - 1: pair (k, j) at koff + j - k
+            float m32 = CUDART_INF_F;
+            for (int k = i - 2, ko = koff0; k < j; ko += p - k - 1, k++) {
+                const float2 cf = pc32[ko + j - k];
+                m32 = fminf(m32, __fadd_rn(prev32[g * p + k], __fmaf_rn(lam32[g], cf.y, cf.x)));
+            }
+            const float T = __double2float_rd(__dadd_rn(__dmul_rn((double)m32, 1.0 + 10.0 * 0x1p-24), slack[g]));
             double best = CUDART_INF;
             int32_t arg = -1;
-            for (int k = i - 2; k < j; k++) {
-                double c = __dadd_rn(prev[g * p + k], __dadd_rn(Cs[tri(k, j)], __dmul_rn(lam[g], Ph[tri(k, j)])));
-                if (c < best) { best = c; arg = k; }
+            for (int k = i - 2, ko = koff0; k < j; ko += p - k - 1, k++) {
+                const float2 cf = pc32[ko + j - k];
+                if (__fadd_rn(prev32[g * p + k], __fmaf_rn(lam32[g], cf.y, cf.x)) <= T) {
+                    const double *e = gpc64 + 2 * (size_t)(tb + k);
+                    const double c = __dadd_rn(prev[g * p + k], __dadd_rn(e[0], __dmul_rn(lam[g], e[1])));
+                    if (c < best) { best = c; arg = k; }
+                }
             }
             nxt[g * p + j] = best;
-            bp[((size_t)g * (s + 1) + i) * dcap + j] = arg;
+            nxt32[g * p + j] = __double2float_rn(__dmul_rn(best, scale));
+            set_bp(g, i, j, arg);
             if (j == p - 1) last[g * (s + 1) + i] = best;
         }
         __syncthreads();
@@ -268,7 +318,8 @@ __global__ void __launch_bounds__(256) k_rows_pass(RowsPass A) {
                     int64_t j = p - 1;
                     a_sm[istar - 1] = (int32_t)j;
                     for (int i = istar; i >= 3; i--) {
-                        j = bp[((size_t)g * (s + 1) + i) * dcap + j];
+                        j = bp_sm ? (int64_t)bps[((size_t)g * (s + 1) + i) * p + j]
+                                  : (int64_t)bp[((size_t)g * (s + 1) + i) * dcap + j];
                         a_sm[i - 2] = (int32_t)j;
                     }
                     a_sm[0] = 0;
@@ -286,18 +337,24 @@ __global__ void __launch_bounds__(256) k_rows_pass(RowsPass A) {
     }
 }
 
-size_t rows_pass_smem(int p, int G, int s) {
+size_t rows_pass_smem(int p, int G, int s, bool bp_smem) {
     size_t npair = (size_t)p * (p - 1) / 2;
-    return sizeof(double) * (2 * npair + (size_t)p + 2 * (size_t)G * p + (size_t)G * (s + 1) + 4 * (size_t)kMaxS);
+    return sizeof(double) * ((size_t)p + 2 * (size_t)G * p + (size_t)G * (s + 1) + 4 * (size_t)kMaxS) +
+           sizeof(float2) * npair + sizeof(float) * 2 * (size_t)G * p +
+           (bp_smem ? (size_t)G * (s + 1) * p : 0);
 }
+// Backpointers in shared memory when that still leaves room for two blocks per SM.
+static bool rows_bp_in_smem(int p, int G, int s) { return rows_pass_smem(p, G, s, true) <= 110 * 1024; }
 
 int launch_rows_pass(const RowsPass &A, int nact, int pmax, cudaStream_t st) {
     if (nact == 0) return ECASQ_OK;
     if (pmax > kRowsMaxP) return ECASQ_EINVAL;
-    size_t smem = rows_pass_smem(pmax, A.G, A.s);
+    RowsPass B = A;
+    B.bp_smem = rows_bp_in_smem(pmax, A.G, A.s) ? 1 : 0;
+    size_t smem = rows_pass_smem(pmax, A.G, A.s, B.bp_smem != 0);
     ECASQ_CUDA_TRY(cudaFuncSetAttribute(k_rows_pass, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     note_launch();
-    k_rows_pass<<<(unsigned)nact, 256, smem, st>>>(A);
+    k_rows_pass<<<(unsigned)nact, 256, smem, st>>>(B);
     ECASQ_LAUNCH_CHECK();
     return ECASQ_OK;
 }
