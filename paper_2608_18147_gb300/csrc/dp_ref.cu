@@ -284,14 +284,30 @@ __global__ void __launch_bounds__(256) k_rows_pass(RowsPass A) {
                 m32 = fminf(m32, __fadd_rn(prev32[g * p + k], __fmaf_rn(lam32[g], cf.y, cf.x)));
             }
             const float T = __double2float_rd(__dadd_rn(__dmul_rn((double)m32, 1.0 + 10.0 * 0x1p-24), slack[g]));
-            double best = CUDART_INF;
-            int32_t arg = -1;
+            // the band's members as a 128-bit mask (k < p <= kRowsMaxP), re-scored after the scan in
+            // increasing k, so a warp runs the binary64 step once per member of its busiest lane
+            // rather than once per k at which any lane has a member
+            uint32_t mk0 = 0u, mk1 = 0u, mk2 = 0u, mk3 = 0u;
             for (int k = i - 2, ko = koff0; k < j; ko += p - k - 1, k++) {
                 const float2 cf = pc32[ko + j - k];
-                if (__fadd_rn(prev32[g * p + k], __fmaf_rn(lam32[g], cf.y, cf.x)) <= T) {
+                const bool in = __fadd_rn(prev32[g * p + k], __fmaf_rn(lam32[g], cf.y, cf.x)) <= T;
+                const uint32_t bit = in ? 1u << (k & 31) : 0u, w = (uint32_t)k >> 5;
+                mk0 |= w == 0u ? bit : 0u;
+                mk1 |= w == 1u ? bit : 0u;
+                mk2 |= w == 2u ? bit : 0u;
+                mk3 |= w == 3u ? bit : 0u;
+            }
+            double best = CUDART_INF;
+            int32_t arg = -1;
+#pragma unroll
+            for (int w = 0; w < 4; w++) {
+                uint32_t mk = w == 0 ? mk0 : (w == 1 ? mk1 : (w == 2 ? mk2 : mk3));
+                while (mk) {
+                    const int k = 32 * w + __ffs(mk) - 1;
+                    mk &= mk - 1u;
                     const double *e = gpc64 + 2 * (size_t)(tb + k);
                     const double c = __dadd_rn(prev[g * p + k], __dadd_rn(e[0], __dmul_rn(lam[g], e[1])));
-                    if (c < best) { best = c; arg = k; }
+                    if (c < best) { best = c; arg = k; }  // increasing k: the lowest k among exact minima
                 }
             }
             nxt[g * p + j] = best;
