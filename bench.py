@@ -435,7 +435,8 @@ def run_pass_mode(args, cfg, x_np):
                       "cost_mode": cost_mode_name(E, flags)},
            "status": {"timeout": st["timeout"], "bound_viol": st["bound_viol"], "rescored": st["rescored"],
                       "tile_units_run": st["tiles_run"], "tile_units_skipped": st["tiles_skipped"],
-                      "cost_tiles_fetched": st["tiles_fetched"],
+                      "cost_tiles_fetched": st["tiles_fetched"], "band_members": st["members"],
+                      "big_bands": st["big_bands"], "wide_bands": st["overflow"],
                       "executed_candidates": executed_candidates(st, p, s, len(lams))},
            "m": list(outs[-1][1]), "gpu_launches": E.ecasq_kernel_launches() - launches0, "clocks": clocks}
     print(json.dumps(out), flush=True)

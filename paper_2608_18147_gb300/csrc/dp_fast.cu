@@ -1892,14 +1892,20 @@ __global__ void __launch_bounds__(128) k_exact_small(Prefix P, FastArgs a, int i
 // Layer i, outputs with more members: one warp each (fp32 re-evaluation within the
 // band, exact re-scoring of the members met), then the lanes' results meet (value,
 // then lowest k).  With resident costs the lanes split every tile's k (the table
-// gives any pair directly); otherwise they take whole tiles (the recurrence of
-// visit_tile runs along k).
+// gives any pair directly); otherwise they take whole tiles and walk them in step
+// (the recurrence of visit_tile runs along k, so its values, and the members, are
+// the ones the closure stage found).  Either way the members met wait in the warp's
+// queue, and each time it holds 32 every lane re-scores one of them in binary64, so
+// the binary64 sequence runs with all lanes busy (the result, least value then lowest
+// k, does not depend on the order).
 __global__ void __launch_bounds__(128) k_exact_big(Prefix P, FastArgs a, int i, double *dp64, int32_t *bp) {
     if (*(volatile const int *)a.abort_flag) return;  // a wait gave up: the tables are not valid
     __shared__ int32_t queue[4][32];  // per warp: band members waiting for binary64 re-scoring
     const int n = a.list_cnt[2 * i + 1];
     const int32_t *list = layer_list(a, i, 1);
     const int lane = threadIdx.x & 31;
+    const unsigned lt = (1u << lane) - 1u;
+    int32_t *qw = queue[threadIdx.x >> 5];
     const int warps = gridDim.x * (blockDim.x >> 5);
     unsigned long long nres = 0;
     int nviol = 0;
@@ -1915,18 +1921,31 @@ __global__ void __launch_bounds__(128) k_exact_big(Prefix P, FastArgs a, int i, 
         const uint32_t n1 = (w1 & 0xFFFFu) - (w1 >> 16) + 1u;
         const uint32_t ntile = n1 + (w2 ? (w2 & 0xFFFFu) - (w2 >> 16) + 1u : 0u);
         const double lam = a.prm->lam64[g];
+        const float lam32 = a.prm->lam32[g];
         const double *prev = dp64 + oidx(a, g, i - 1, 0);
+        const int64_t J = j / BJ, j0 = J * BJ;
         double best = CUDART_INF;
         int32_t arg = INT32_MAX;
+        int qn = 0;  // warp-uniform queue length
+        // every lane calls this with its verdict on candidate k (warp-uniform call)
+        auto push = [&](bool in, int64_t k) {
+            const unsigned mask = __ballot_sync(0xffffffffu, in);
+            if (!mask) return;
+            const int cnt = __popc(mask), pos = qn + __popc(mask & lt);
+            if (in && pos < 32) qw[pos] = (int32_t)k;
+            __syncwarp();
+            if (qn + cnt >= 32) {
+                exact_candidate(P, prev, qw[lane], j, lam, best, arg);
+                nres++;
+                __syncwarp();
+                if (in && pos >= 32) qw[pos - 32] = (int32_t)k;
+                __syncwarp();
+                qn += cnt - 32;
+            } else {
+                qn += cnt;
+            }
+        };
         if (a.costs) {
-            // the lanes test the tile's k in the fp32 band; the members met wait in the warp's
-            // queue, and each time it holds 32 every lane re-scores one of them in binary64
-            // (the result, least value then lowest k, does not depend on the order)
-            int32_t *qw = queue[threadIdx.x >> 5];
-            int qn = 0;  // warp-uniform queue length
-            const unsigned lt = (1u << lane) - 1u;
-            const float lam32 = a.prm->lam32[g];
-            const int64_t J = j / BJ, j0 = J * BJ;
             for (uint32_t t = 0; t < ntile; t++) {
                 const int64_t K = t < n1 ? (w1 >> 16) + t : (w2 >> 16) + (t - n1);
                 const int64_t k0 = K * BK;
@@ -1936,37 +1955,49 @@ __global__ void __launch_bounds__(128) k_exact_big(Prefix P, FastArgs a, int i, 
                 const int64_t khi = (K == J) ? j - 1 : k0 + BK - 1;
                 for (int64_t kb = k0; kb <= khi; kb += 32) {  // warp-uniform
                     const int64_t k = kb + lane;
-                    const bool in = k <= khi && cand32(prev32[k], lam32, cr[k - k0], pr[k - k0]) <= thr;
-                    const unsigned mask = __ballot_sync(0xffffffffu, in);
-                    const int cnt = __popc(mask), pos = qn + __popc(mask & lt);
-                    if (in && pos < 32) qw[pos] = (int32_t)k;
-                    __syncwarp();
-                    if (qn + cnt >= 32) {
-                        exact_candidate(P, prev, qw[lane], j, lam, best, arg);
-                        nres++;
-                        __syncwarp();
-                        if (in && pos >= 32) qw[pos - 32] = (int32_t)k;
-                        __syncwarp();
-                        qn += cnt - 32;
-                    } else {
-                        qn += cnt;
-                    }
+                    push(k <= khi && cand32(prev32[k], lam32, cr[k - k0], pr[k - k0]) <= thr, k);
                 }
             }
-            if (lane < qn) {
-                exact_candidate(P, prev, qw[lane], j, lam, best, arg);
-                nres++;
-            }
-            __syncwarp();  // the queue is free for the warp's next output
         } else {
-            for (uint32_t t = lane; t < ntile; t += 32) {
-                const uint32_t K = t < n1 ? (w1 >> 16) + t : (w2 >> 16) + (t - n1);
-                visit_tile(a, g, i, j, (int64_t)K, thr, [&](int64_t k) {
-                    exact_candidate(P, prev, k, j, lam, best, arg);
-                    nres++;
-                });
+            const float vj = a.v[j], d_f = (float)a.d;
+            for (uint32_t tb = 0; tb < ntile; tb += 32) {  // warp-uniform
+                const uint32_t t = tb + lane;
+                // tile K of the band (lanes past the band's end take tile 0 and no candidate)
+                const int64_t K = t >= ntile ? 0 : (int64_t)(t < n1 ? (w1 >> 16) + t : (w2 >> 16) + (t - n1));
+                const int64_t k0 = K * BK;
+                const float *prev32 = a.dp32 + d32(a, g, i - 1, k0) - k0;
+                // the state visit_tile starts from: the anchor at the tile's top pair, or the
+                // empty interval (j, j] on the diagonal tile (which steps before its first value)
+                Rec r = rec_empty();
+                int64_t kfirst = k0 + BK - 1;
+                int nk = 0;  // candidates of the lane's tile: k = kfirst, kfirst - 1, ..., kfirst - nk + 1
+                if (t < ntile) {
+                    if (K == J) {
+                        kfirst = j - 1;
+                        nk = (int)(j - k0);
+                    } else {
+                        nk = BK;
+                        rec_anchor(a, kfirst, j, r);
+                    }
+                }
+                for (int it = 0; it < BK; it++) {  // warp-uniform
+                    const int64_t k = kfirst - it;
+                    bool in = false;
+                    if (it < nk) {
+                        if (it > 0 || K == J) rec_step(r, vj, a.v[k + 1], a.wf[k + 1], __fsub_rn(a.v[k + 1], a.v[k]));
+                        float c, ph;
+                        rec_emit(r, vj, a.v[k], d_f, a.invd, c, ph);
+                        in = cand32(prev32[k], lam32, c, ph) <= thr;
+                    }
+                    push(in, k);
+                }
             }
         }
+        if (lane < qn) {
+            exact_candidate(P, prev, qw[lane], j, lam, best, arg);
+            nres++;
+        }
+        __syncwarp();  // the queue is free for the warp's next output
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) {
             const double b2 = __shfl_xor_sync(0xffffffffu, best, off);
