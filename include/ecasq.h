@@ -65,6 +65,11 @@ typedef struct CUstream_st *ecasq_stream_t; /* same type as cudaStream_t */
 #define ECASQ_ONE_PART_PUBLISH 128u /* fast DP with resident or streamed costs and s <= 16: publish each column block
                                      of the wavefront once, after all its layers, instead of in two parts (rows 2..8
                                      after layer 8, then the rest); same results, for comparison */
+#define ECASQ_UNSEEDED_SEARCH 256u /* fast DP with resident or streamed costs and tile skipping (s <= 16): in the
+                                     multiplier search, start every pass's tile skipping from scratch instead of from
+                                     the fp32 minima of the bracket's evaluated upper end (an upper bound of every
+                                     later pass's minima, Sec. 5's candidates being non-decreasing in lambda); same
+                                     results, for comparison */
 #define ECASQ_TEST_STALL (1u << 30) /* test hook for the bounded device waits: column block 0 of the fast DP's
                                      wavefront is never published and the flag waits give up after 2^14 spins, so
                                      the call must return ECASQ_ETIMEOUT (nothing else) and leave the workspace

@@ -17,7 +17,8 @@ int launch_dp_reference(const Prefix &P, const double *lamp, int G, int s, doubl
                         cudaStream_t st);
 int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, const Layout &L, cudaStream_t st,
                    bool exact_s, bool exact_tables, float *costs, bool build_costs, bool test_stall,
-                   size_t chunk_bytes, bool split_off);
+                   size_t chunk_bytes, bool split_off, bool seeded);
+int save_dp_seed(void *ws, const Layout &Lw, int64_t p, int G, int s, int g, cudaStream_t st);
 size_t resident_costs_bytes(int64_t d);
 size_t streamed_costs_bytes(int64_t d);
 int launch_rows_prepare(const float *X, int64_t rows, const RowsData &R, cudaStream_t st);
@@ -280,8 +281,11 @@ struct PassOut {
 // evaluation, results to the host.
 // costs_built: in/out, whether the resident interval costs (if the layout has
 // them) already hold this call's prefix data.
+// seeded: the workspace's seed rows hold an earlier pass's fp32 minima at a multiplier
+// >= every multiplier of this pass (save_dp_seed); the fast kernel's tile skipping
+// starts from them.
 static int dp_pass_prepared(void *ws, const Layout &L, const Prefix &P, int s, const double *lamp, int G,
-                            uint32_t flags, cudaStream_t st, PassOut &out, bool *costs_built) {
+                            uint32_t flags, cudaStream_t st, PassOut &out, bool *costs_built, bool seeded = false) {
     double *dp64 = wsp<double>(ws, L.dp64);
     int32_t *bp = wsp<int32_t>(ws, L.bp);
     int rc;
@@ -296,7 +300,8 @@ static int dp_pass_prepared(void *ws, const Layout &L, const Prefix &P, int s, c
         // streamed costs are rebuilt band by band in every pass
         rc = launch_dp_fast(P, lamp, G, s, ws, L, st, (flags & ECASQ_EXACT_S) != 0, (flags & ECASQ_EXACT_TABLES) != 0,
                             costs, costs && (L.costs_streamed || !*costs_built), (flags & ECASQ_TEST_STALL) != 0,
-                            L.costs_streamed ? L.costs_bytes : 0, (flags & ECASQ_ONE_PART_PUBLISH) != 0);
+                            L.costs_streamed ? L.costs_bytes : 0, (flags & ECASQ_ONE_PART_PUBLISH) != 0,
+                            seeded && !(flags & ECASQ_UNSEEDED_SEARCH));
         if (costs && rc == ECASQ_OK) *costs_built = true;
     }
     if (rc != ECASQ_OK) return rc;
@@ -611,13 +616,23 @@ static int solve_prepared(void *ws, const Layout &L, const Prefix &P, int64_t d,
     int64_t cand_per = candidates_of(p, s, 0);
     int64_t cand = 0;
     std::vector<Eval> evals;
+    // Seed rows (tile skipping of the fast kernel): the fp32 minima of the last pass at
+    // seed_lam, kept while every later multiplier stays below it.  The search's upper
+    // bracket end is such a multiplier once it has been evaluated.
+    double seed_lam = -1.0;
+    int last_G = 0;
     auto run = [&](const std::vector<double> &lams) -> int {
         double lamp[kMaxG];
         int G = (int)lams.size();
-        for (int g = 0; g < G; g++) lamp[g] = lams[g] * n2;
+        bool seeded = seed_lam >= 0.0;
+        for (int g = 0; g < G; g++) {
+            lamp[g] = lams[g] * n2;
+            seeded = seeded && lams[g] <= seed_lam;
+        }
         PassOut po;
-        int r = dp_pass_prepared(ws, L, P, s, lamp, G, prm->flags, st, po, &costs_built);
+        int r = dp_pass_prepared(ws, L, P, s, lamp, G, prm->flags, st, po, &costs_built, seeded);
         if (r) return r;
+        last_G = G;
         passes++;
         nlam += G;
         cand += cand_per * G;
@@ -668,6 +683,12 @@ static int solve_prepared(void *ws, const Layout &L, const Prefix &P, int64_t d,
                     double nlo = f > 0 ? pts[f - 1].lam : lo;
                     hi = pts[f].lam;
                     lo = nlo;
+                    // the next passes lie below hi: its fp32 minima bound theirs
+                    if (L.costs_bytes && !L.gpairs_bytes && !(prm->flags & (ECASQ_DP_REFERENCE | ECASQ_UNSEEDED_SEARCH))) {
+                        rc = save_dp_seed(ws, L, p, last_G, s, last_G - 7 + f, st);
+                        if (rc) return rc;
+                        seed_lam = hi;
+                    }
                 } else {
                     lo = pts[6].lam;
                 }

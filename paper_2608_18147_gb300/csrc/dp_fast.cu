@@ -141,6 +141,8 @@ struct FastArgs {
     float *mdp;            // [nJ][G][mdp_stride]: min over the block's 64 columns of dp32(g, i, .)
     int mdp_stride;        // s + 1 rounded up to a multiple of 4 (16-byte rows)
     int prune;             // skip tiles by the lower bound (resident costs, two layer groups)
+    const float *seed;     // with prune: fp32 dp rows [nJ][s+1][64] of an earlier pass at a multiplier >= every
+                           // multiplier of this one (upper bounds of this pass's fp32 minima), or null
     uint32_t spin_limit;   // flag waits give up after this many spins (kSpinLimit; lower in the test hook)
     int hold0;             // test hook: column block 0 is never published (its waiters time out)
     int split_pub;         // resident costs, two layer groups: blocks are published in two parts (below)
@@ -661,6 +663,36 @@ __device__ __forceinline__ void cons_reset(ConsState &cs) {
         for (int q = 0; q < JPT; q++) { cs.best[l][q] = CUDART_INF_F; cs.w1[l][q] = 0u; cs.w2[l][q] = 0u; }
 }
 
+// A band word with no run yet (a seeded running minimum, below): the first tile that
+// joins the band opens run 2 (run 1 cannot extend: its end + 1 is 2^16, above every K),
+// and diag_pair_bands moves run 2 into run 1 when run 1 was never set.
+constexpr uint32_t kNoRun = 0xFFFFFFFFu;
+
+// Seeded running minima of block J.  Every fp32 candidate is monotone in lambda' (C and
+// Phi are >= 0 and the roundings are monotone), so by induction over the layers an
+// earlier pass's fp32 minimum at a multiplier >= this one's bounds this pass's minimum
+// m from above.  Starting the running minimum at that bound changes no result: the
+// tile holding m is never skipped (its lower bound is <= m <= the limit), so the final
+// minimum is m itself; a tile the tighter limit skips has every candidate above
+// m (1 + tau), outside the band; and band_fold keeps the band a superset of the tiles
+// with a candidate within m (1 + tau) from any starting bb >= m (a reset drops only
+// tiles whose candidates all lie above the band).  Only the skip tests see the seed:
+// more tiles are skipped, the tables are unchanged.
+__device__ __forceinline__ void cons_seed(const FastArgs &a, ConsState &cs, int J, const ConsId &id) {
+    const float *sr = a.seed + (size_t)J * (size_t)(a.s + 1) * BJ;
+#pragma unroll
+    for (int l = 0; l < LPT; l++) {
+        // rows past the last layer repeat the last one (cons_offdiag): so does their seed
+        const int i = 3 + min(id.lg * LPT + l, a.s - 3);
+#pragma unroll
+        for (int q = 0; q < JPT; q++) {
+            const int jl = id.jq + NJQ * q;
+            const float v = ((int64_t)J * BJ + jl < a.p) ? sr[(size_t)i * BJ + jl] : CUDART_INF_F;
+            if (v < CUDART_INF_F) { cs.best[l][q] = v; cs.w1[l][q] = kNoRun; }
+        }
+    }
+}
+
 // Off-diagonal tile K: the fp32 minimum over the tile's 64 k of every output the
 // thread owns (g must be a real multiplier), folded into its band state.
 // Candidate values are >= +0, so their bit patterns order like the floats: the
@@ -1084,7 +1116,9 @@ __device__ __forceinline__ void diag_pair_bands(const FastArgs &a, const uint32_
         for (int q = 0; q < JPT; q++) {
             const int64_t j = j0 + id.jq + NJQ * q;
             const int x = (l * JPT + q) * nc + ct;
-            if (i <= a.s && j < a.p) a.band[oidx(a, g, i, j)] = band_pack(park[NS * nc + x], park[2 * NS * nc + x]);
+            uint32_t w1 = park[NS * nc + x], w2 = park[2 * NS * nc + x];
+            if (w1 == kNoRun) { w1 = w2; w2 = 0u; }  // seeded: the band's only run was opened as run 2
+            if (i <= a.s && j < a.p) a.band[oidx(a, g, i, j)] = band_pack(w1, w2);
         }
     }
 }
@@ -1427,6 +1461,7 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
         const bool own = id.active && g < a.G;
         if (split != fsplit) { frontier = -1; fsplit = split; }
         cons_reset(cs);
+        if (a.seed && own) cons_seed(a, cs, J, id);
         int issued = -1;  // the tile whose copies are in flight into buffer n & 1 (J: the diagonal), or -1
         const int ngv = min(a.G - split * a.Gc, a.Gc);  // real multipliers of the split
         // the tiles walked here: K < Kend (with a split publish the last one, J - 1, is the chain's)
@@ -2021,7 +2056,9 @@ __global__ void k_store_params(FastParams prm, FastParams *dst) {
 
 static int mdp_stride(int s) { return (s + 1 + 3) & ~3; }
 
-size_t fast_dp_band_bytes(int64_t d, int32_t s) {
+// The band region: band words, member lists, need marks, flags, constants, corner
+// states, block minima, the exact stage's lists; then the seed rows (cons_seed).
+static size_t band_core_bytes(int64_t d, int32_t s) {
     size_t rows = (size_t)kMaxG * (size_t)(s + 1) * (size_t)table_stride(d);
     size_t nJ = (size_t)cdiv(d, BJ);
     return align256(8 * rows) + align256(4 * rows) + align256(4 * NMEM * rows) + align256(rows) +
@@ -2029,6 +2066,22 @@ size_t fast_dp_band_bytes(int64_t d, int32_t s) {
            align256(4 * (size_t)kMaxG * (size_t)mdp_stride(s) * nJ) +
            align256(2 * 4 * (size_t)kMaxG * (size_t)(s + 1) * (size_t)table_stride(d)) +
            align256(4 * 2 * (size_t)(s + 1));
+}
+static size_t seed_rows_bytes(int64_t d, int32_t s) { return align256(4 * (size_t)cdiv(d, BJ) * BJ * (size_t)(s + 1)); }
+size_t fast_dp_band_bytes(int64_t d, int32_t s) { return band_core_bytes(d, s) + seed_rows_bytes(d, s); }
+static float *seed_rows(void *ws, const Layout &Lw) {
+    return reinterpret_cast<float *>(wsp<char>(ws, Lw.band) + band_core_bytes(Lw.d, Lw.s));
+}
+
+// Keep the fp32 dp rows of multiplier g of the last pass (G multipliers over p values) as
+// the seed rows of a later pass at multipliers <= this one's (cons_seed).
+int save_dp_seed(void *ws, const Layout &Lw, int64_t p, int G, int s, int g, cudaStream_t st) {
+    if (g < 0 || g >= G || s != Lw.s) return ECASQ_EINVAL;
+    const size_t row = (size_t)(s + 1) * BJ * sizeof(float);
+    const float *src = wsp<float>(ws, Lw.dp32) + (size_t)g * (s + 1) * BJ;
+    ECASQ_CUDA_TRY(cudaMemcpy2DAsync(seed_rows(ws, Lw), row, src, row * (size_t)G, row, (size_t)cdiv(p, BJ),
+                                     cudaMemcpyDeviceToDevice, st));
+    return ECASQ_OK;
 }
 
 static size_t smem_bytes(int Gc, int s) { return sizeof(Smem) + (size_t)2 * Gc * (s - 2) * BK * sizeof(float); }
@@ -2071,7 +2124,7 @@ size_t streamed_costs_bytes(int64_t d) {
 
 int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, const Layout &Lw, cudaStream_t st,
                    bool exact_s, bool exact_tables, float *costs, bool build_costs, bool test_stall,
-                   size_t chunk_bytes, bool split_off) {
+                   size_t chunk_bytes, bool split_off, bool seeded) {
     double *dp64 = wsp<double>(ws, Lw.dp64);
     int32_t *bp = wsp<int32_t>(ws, Lw.bp);
     // small inputs, very large ones and huge counts take the reference kernel
@@ -2130,6 +2183,7 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     a.split_pub = (costs && a.lgc == 2 && !split_off) ? 1 : 0;
     a.hold0 = test_stall ? 1 : 0;
     a.prune = (costs && a.lgc == 2 && a.mdp_stride <= 20) ? 1 : 0;
+    a.seed = (seeded && a.prune && s == Lw.s) ? seed_rows(ws, Lw) : nullptr;
     a.costs = costs;
     a.tile_base = 0;
     a.J0 = 0;

@@ -19,6 +19,7 @@ from . import build as _build
 OK, EINVAL, ENONFINITE, EINFEASIBLE, EWORKSPACE, ECUDA, ETIMEOUT, ERANGE = 0, -1, -2, -3, -4, -5, -6, -7
 EXACT_S, NO_REFINE_GUARD, DP_REFERENCE, TIME_KERNELS, EXACT_TABLES, RESIDENT_COSTS, STREAMED_COSTS = 1, 2, 4, 8, 16, 32, 64
 ONE_PART_PUBLISH = 128  # fast DP: publish every column block once (no two-part publish)
+UNSEEDED_SEARCH = 256  # fast DP search: no seeded tile skipping (same results)
 TEST_STALL = 1 << 30  # test hook of the bounded waits (include/ecasq.h)
 
 _lock = threading.Lock()

@@ -258,3 +258,37 @@ def test_two_part_publish_bit_identical_to_one_part(E, name, s):
             np.testing.assert_array_equal(bp1, bp2)
         del ws1, ws2
         _free()
+
+
+@pytest.mark.parametrize("name,s,b", [("studentt16k", 16, 2.5), ("lognormal16k", 16, 1.0), ("studentt20001", 12, 2.5),
+                                      ("normal8192", 10, 2.0)])
+def test_seeded_search_bit_identical_to_unseeded(E, name, s, b):
+    """Later passes of the search start their tile skipping from the fp32 minima of the
+    bracket's evaluated upper end (an upper bound of theirs: candidates are non-decreasing
+    in lambda').  Same multiplier, codebook and metrics as without; with every output
+    resolved exactly, the same last-pass tables; fewer tiles walked."""
+    x = {"studentt16k": lambda: workloads.student_t(16384, 0),
+         "lognormal16k": lambda: workloads.signed_lognormal(16384, 0),
+         "studentt20001": lambda: workloads.student_t(20001, 5, scale=1.0),
+         "normal8192": lambda: workloads.normal(8192, 7)}[name]()
+    out = {}
+    for extra in (0, E.UNSEEDED_SEARCH):
+        ws = E.workspace(x.size, s, flags=E.RESIDENT_COSTS)
+        Q, res = E.ecasq_solve(x, s, budget_bits=b, refine_max_rounds=0,
+                               flags=E.RESIDENT_COSTS | E.EXACT_TABLES | extra, ws=ws)
+        st = E.native.ws_status(ws)
+        assert st["timeout"] == 0 and st["bound_viol"] == 0
+        out[extra] = (Q.cpu().numpy(), res, st, _tables(E, ws, st["last_G"], s, x.size))
+        del ws
+        _free()
+    (Qs, rs, sts, ts), (Qu, ru, stu, tu) = out[0], out[E.UNSEEDED_SEARCH]
+    assert rs["passes"] == ru["passes"] >= 3
+    np.testing.assert_array_equal(Qs, Qu)
+    for k in ("lambda", "m", "mse", "h_exact", "h_surrogate", "status"):
+        assert rs[k] == ru[k], k
+    for (dps, bps), (dpu, bpu) in zip(ts, tu):
+        np.testing.assert_array_equal(dps, dpu)
+        np.testing.assert_array_equal(bps, bpu)
+    assert sts["tiles_run"] <= stu["tiles_run"]
+    if name == "studentt16k":  # five seeded passes at multipliers where most tiles are skipped
+        assert sts["tiles_run"] < 0.95 * stu["tiles_run"]
