@@ -8,7 +8,7 @@
 // keeps the fp32 values near 1 (the DP is invariant under scaling X by a power of
 // two when lambda' scales with ||X||^2, Sec. 3).
 //
-// Layer i >= 3 (eq. apx_rec) runs one warp per output j for all G multipliers:
+// Layer i >= 3 (eq. apx_rec) runs one block per output j for all G multipliers:
 //  1. fp32 pass over k in [i-2, j-1]: val32 = fl(dp32(i-1,k) + fl(fma(lam32, Phi32, C32)))
 //     gives the fp32 minimum m32 of each multiplier;
 //  2. every k with val32 <= T = m32 (1 + 10u) + 3A is re-scored with the binary64
@@ -35,6 +35,7 @@ struct GridArgs {
     double *dp64;          // [G][s+1][ps]
     int32_t *bp;
     float *dp32;           // [G][s+1][ps], dp64 * scale rounded to fp32
+    const int64_t *N;      // [n+1]: N[t+1] = #{x <= P_t}
     int64_t n, ps;
     int G, s;
     double scale;
@@ -73,47 +74,83 @@ __global__ void k_grid_round(GridArgs A, int i) {
     }
 }
 
-__global__ void __launch_bounds__(256) k_grid_layer(GridArgs A, int i) {
-    const int lane = threadIdx.x & 31;
-    const int64_t wid = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
-    const int64_t j = A.n - 1 - wid;  // heavy outputs first
-    if (j < i - 1) return;
+// One block per output j (heavy outputs first), its threads splitting the k range, so
+// that no output's scan is a long serial walk of one warp (the last outputs have n - 1
+// candidates per multiplier, and each step of a walk waits on its loads from L2).
+constexpr int kGridThreads = 256;
+__global__ void __launch_bounds__(kGridThreads, 3) k_grid_layer(GridArgs A, int i) {
+    __shared__ float sm[kGridThreads / 32][kMaxG];
+    __shared__ double sb[kGridThreads / 32][kMaxG];
+    __shared__ int32_t sa[kGridThreads / 32][kMaxG];
+    __shared__ float sT[kMaxG];
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    const int64_t j = A.n - 1 - (int64_t)blockIdx.x;
+    if (j < i - 1) return;  // block-uniform
     const size_t tb = (size_t)j * (size_t)(j - 1) / 2;
     const int G = A.G;
     float m[kMaxG];
 #pragma unroll
     for (int g = 0; g < kMaxG; g++) m[g] = CUDART_INF_F;
-    for (int64_t k = i - 2 + lane; k < j; k += 32) {
+    for (int64_t k = i - 2 + threadIdx.x; k < j; k += kGridThreads) {
         float2 cf = A.pc32[tb + k];
 #pragma unroll
         for (int g = 0; g < kMaxG; g++)
             if (g < G) m[g] = fminf(m[g], __fadd_rn(A.dp32[g_at(A, g, i - 1, k)], __fmaf_rn(A.lam32[g], cf.y, cf.x)));
     }
-    float T[kMaxG];  // rounded down to fp32: for an fp32 candidate c, c <= T32 exactly when c <= T
 #pragma unroll
     for (int g = 0; g < kMaxG; g++) {
         float v = m[g];
         for (int o = 16; o > 0; o >>= 1) v = fminf(v, __shfl_xor_sync(0xffffffffu, v, o));
-        T[g] = __double2float_rd(__dadd_rn(__dmul_rn((double)v, 1.0 + 10.0 * 0x1p-24), A.slack[g]));
+        if (lane == 0) sm[wid][g] = v;
     }
+    __syncthreads();
+    // the band limits, once per block (binary64 runs at 1/64 of the fp32 rate): rounded down
+    // to fp32, so that for an fp32 candidate c, c <= T32 exactly when c <= T
+    if (threadIdx.x < kMaxG) {
+        const int g = threadIdx.x;
+        float v = sm[0][g];
+        for (int w = 1; w < kGridThreads / 32; w++) v = fminf(v, sm[w][g]);
+        sT[g] = __double2float_rd(__dadd_rn(__dmul_rn((double)v, 1.0 + 10.0 * 0x1p-24), A.slack[g]));
+    }
+    __syncthreads();
+    float T[kMaxG];
+#pragma unroll
+    for (int g = 0; g < kMaxG; g++) T[g] = sT[g];
     double best[kMaxG];
     int32_t arg[kMaxG];
 #pragma unroll
     for (int g = 0; g < kMaxG; g++) { best[g] = CUDART_INF; arg[g] = -1; }
-    for (int64_t k = i - 2 + lane; k < j; k += 32) {
+    const int64_t Nj = A.N[j + 1];
+    for (int64_t k = i - 2 + threadIdx.x; k < j; k += kGridThreads) {
         float2 cf = A.pc32[tb + k];
+        // no data in (P_k, P_j]: then App. E's sums are differences of equal prefix values,
+        // so C = U = D = 0 and Phi = 0 exactly, and the candidate is dp(i-1, k) itself
+        // (x + 0 = x for x >= +0, lambda' 0 = +0): no pair load, no binary64 arithmetic.
+        // Grids with many empty intervals (heavy tails) have long runs of such candidates
+        // in their bands.
+        const bool empty = A.N[k + 1] == Nj;
 #pragma unroll
         for (int g = 0; g < kMaxG; g++) {
             if (g < G) {
                 float v = __fadd_rn(A.dp32[g_at(A, g, i - 1, k)], __fmaf_rn(A.lam32[g], cf.y, cf.x));
                 if (v <= T[g]) {
-                    double2 e = A.pc64[tb + k];
-                    double c = __dadd_rn(A.dp64[g_at(A, g, i - 1, k)], __dadd_rn(e.x, __dmul_rn(A.lam64[g], e.y)));
-                    if (c < best[g]) { best[g] = c; arg[g] = (int32_t)k; }  // k ascends per lane
+                    const double dprev = A.dp64[g_at(A, g, i - 1, k)];
+                    double c = dprev;
+                    if (!empty) {
+                        const double2 e = A.pc64[tb + k];
+                        c = __dadd_rn(dprev, __dadd_rn(e.x, __dmul_rn(A.lam64[g], e.y)));
+                    }
+                    // integer compares of the bit patterns (binary64 compares run on the
+                    // binary64 pipe)
+                    const long long cb = __double_as_longlong(c), bb = __double_as_longlong(best[g]);
+                    // non-negative doubles (+inf included) order like their bit patterns
+                    const bool lt = (cb >= 0 && bb >= 0) ? cb < bb : c < best[g];
+                    if (lt) { best[g] = c; arg[g] = (int32_t)k; }  // k ascends per thread
                 }
             }
         }
     }
+    // least value, then lowest k: over the lanes, then over the warps
 #pragma unroll
     for (int g = 0; g < kMaxG; g++) {
         double b = best[g];
@@ -123,11 +160,21 @@ __global__ void __launch_bounds__(256) k_grid_layer(GridArgs A, int i) {
             int32_t a2 = __shfl_xor_sync(0xffffffffu, a, o);
             if (a2 >= 0 && (a < 0 || b2 < b || (b2 == b && a2 < a))) { b = b2; a = a2; }
         }
-        if (lane == g && g < G) {
-            A.dp64[g_at(A, g, i, j)] = b;
-            A.bp[g_at(A, g, i, j)] = a;
-            A.dp32[g_at(A, g, i, j)] = __double2float_rn(__dmul_rn(b, A.scale));
+        if (lane == 0) { sb[wid][g] = b; sa[wid][g] = a; }
+    }
+    __syncthreads();
+    if (threadIdx.x < G) {
+        const int g = threadIdx.x;
+        double b = sb[0][g];
+        int32_t a = sa[0][g];
+        for (int w = 1; w < kGridThreads / 32; w++) {
+            const double b2 = sb[w][g];
+            const int32_t a2 = sa[w][g];
+            if (a2 >= 0 && (a < 0 || b2 < b || (b2 == b && a2 < a))) { b = b2; a = a2; }
         }
+        A.dp64[g_at(A, g, i, j)] = b;
+        A.bp[g_at(A, g, i, j)] = a;
+        A.dp32[g_at(A, g, i, j)] = __double2float_rn(__dmul_rn(b, A.scale));
     }
 }
 
@@ -149,6 +196,7 @@ int launch_dp_grid(const Prefix &P, const double *lamp, int G, int s, double *dp
     A.pc64 = reinterpret_cast<const double2 *>(pairs);
     A.pc32 = reinterpret_cast<const float2 *>(static_cast<char *>(pairs) + align256(16 * np));
     A.dp64 = dp64; A.bp = bp; A.dp32 = dp32;
+    A.N = P.N;
     A.n = n; A.ps = P.ps; A.G = G; A.s = s;
     A.scale = P.scale32;
     for (int g = 0; g < kMaxG; g++) {
@@ -174,7 +222,7 @@ int launch_dp_grid(const Prefix &P, const double *lamp, int G, int s, double *dp
     for (int i = 3; i <= s; i++) {
         if (n < i) break;
         note_launch();
-        k_grid_layer<<<(unsigned)cdiv(n, 8), 256, 0, st>>>(A, i);
+        k_grid_layer<<<(unsigned)n, kGridThreads, 0, st>>>(A, i);
         ECASQ_LAUNCH_CHECK();
     }
     timer_end(st);
