@@ -210,12 +210,13 @@ __device__ __forceinline__ float h32_small(float y) {
     float r = __fmul_rn(y, -__log2f(fmaxf(y, 1e-37f)));
     return (y > 0.0f) ? fmaxf(r, 0.0f) : 0.0f;
 }
-// h(y) for y in [0, 1], `comp` = 1 - y computed from the complementary mass;
-// both branches are evaluated and one is selected.
+// h(y) for y in [0, 1], `comp` = 1 - y computed from the complementary mass.  The
+// series for y > 1/2 is a branch: only intervals holding more than half of all entries
+// reach it, and a warp whose lanes have none skips it.
 __device__ __forceinline__ float h32_any(float y, float comp) {
-    float lsm = -__log2f(fmaxf(y, 1e-37f));
-    float lbig = neg_log2_1m(fminf(fmaxf(comp, 0.0f), 0.5f));
-    float r = __fmul_rn(y, (y <= 0.5f) ? lsm : lbig);
+    float l = -__log2f(fmaxf(y, 1e-37f));
+    if (y > 0.5f) l = neg_log2_1m(fminf(fmaxf(comp, 0.0f), 0.5f));
+    float r = __fmul_rn(y, l);
     return (y > 0.0f) ? fmaxf(r, 0.0f) : 0.0f;
 }
 
