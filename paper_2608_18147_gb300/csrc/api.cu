@@ -39,6 +39,8 @@ size_t refine_ctx_bytes();
 int launch_refine_colour(const Prefix &P, const int32_t *a, int m, int colour, double lamp, int32_t *a_new,
                          int32_t *moved, void *part_buf, int32_t *ctx, cudaStream_t st, int *nblocks_out);
 size_t refine_scratch_bytes(int64_t d);
+int launch_refine_commit(int32_t *a, const int32_t *a_new, const int32_t *moved, const double *ev, int m, bool guard,
+                         double budget, cudaStream_t st);
 int launch_quantize(const float *x, int64_t d, const float *Q, int m, uint64_t seed, uint8_t *idx, uint32_t *counts,
                     DevStatus *st, int num_sms, cudaStream_t stream);
 int launch_quantize_timeshare(const float *x, int64_t d, const float *Qm, int mm, const float *Qp, int mp,
@@ -375,6 +377,7 @@ static int refine_device(void *ws, const Layout &L, const Prefix &P, std::vector
     int rc = eval_device(ws, L, P, a, m, st, ev);
     if (rc != ECASQ_OK) return rc;
     double J = ev[0] + lamp * ev[2];
+    double *evd = reinterpret_cast<double *>(wsp<char>(ws, L.refine) + 4 * 2 * kMaxS + 256);  // eval_device's output
     for (int r = 0; r < max_rounds; r++) {
         double J0 = J;
         for (int col = 0; col < 3; col++) {
@@ -384,13 +387,11 @@ static int refine_device(void *ws, const Layout &L, const Prefix &P, std::vector
             rc = launch_refine_colour(P, a, m, col, lamp, an, moved, wsp<void>(ws, L.refine_part), ctx, st, &nblk);
             if (rc != ECASQ_OK) return rc;
             if (nblk == 0) continue;
-            int32_t mv = 0;
-            ECASQ_CUDA_TRY(cudaMemcpyAsync(&mv, moved, sizeof(int32_t), cudaMemcpyDeviceToHost, st));
-            rc = eval_device(ws, L, P, an, m, st, ev, moved);  // only a step that moved a value is evaluated
+            // only a step that moved a value is evaluated; the step is kept or dropped on the device
+            rc = launch_eval_codebook(P, an, m, evd, st, moved);
             if (rc != ECASQ_OK) return rc;
-            if (!mv) continue;
-            if (guard && ev[2] > budget) continue;
-            ECASQ_CUDA_TRY(cudaMemcpyAsync(a, an, sizeof(int32_t) * m, cudaMemcpyDeviceToDevice, st));
+            rc = launch_refine_commit(a, an, moved, evd, m, guard, budget, st);
+            if (rc != ECASQ_OK) return rc;
         }
         rc = eval_device(ws, L, P, a, m, st, ev);
         if (rc != ECASQ_OK) return rc;

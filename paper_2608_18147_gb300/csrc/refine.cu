@@ -150,6 +150,25 @@ __global__ void k_refine_pick(const int32_t *a, int m, int colour, const RefPart
     }
 }
 
+// After a colour step: the step's codebook replaces the current one unless no value moved,
+// or (with the guard) its H(Xhat), ev[2] from the gated evaluation, exceeds the budget
+// (Sec. 6).  On the device, so that a refinement round needs no host round trip until
+// its stop test.
+__global__ void k_refine_commit(int32_t *a, const int32_t *a_new, const int32_t *moved, const double *ev, int m,
+                                int guard, double budget) {
+    if (!*moved) return;
+    if (guard && ev[2] > budget) return;
+    for (int t = threadIdx.x; t < m; t += blockDim.x) a[t] = a_new[t];
+}
+
+int launch_refine_commit(int32_t *a, const int32_t *a_new, const int32_t *moved, const double *ev, int m, bool guard,
+                         double budget, cudaStream_t st) {
+    note_launch();
+    k_refine_commit<<<1, 32, 0, st>>>(a, a_new, moved, ev, m, guard ? 1 : 0, budget);
+    ECASQ_LAUNCH_CHECK();
+    return ECASQ_OK;
+}
+
 size_t refine_scratch_bytes(int64_t d) {
     return sizeof(double) * kRefineValues + sizeof(RefPart) * kRefineValues * (size_t)cdiv(d, kRefineChunk);
 }
