@@ -138,6 +138,9 @@ struct FastArgs {
     int J0, J1;            // the wavefront's column blocks [J0, J1): all of them, or one band (streamed costs)
     int32_t *lists;        // [s+1][2][G ps]: needed outputs of layer i (g << 24 | j); 0: <= NMEM members, 1: more
     int *list_cnt;         // [s+1][2]
+    int32_t *wide;         // [G ps]: needed outputs of the layer being closed whose bands span more than
+                           // kThreadTiles tiles (g << 24 | j), walked by a warp each (k_need_wide)
+    int *wide_cnt;         // [s+1]
     float *mdp;            // [nJ][G][mdp_stride]: min over the block's 64 columns of dp32(g, i, .)
     int mdp_stride;        // s + 1 rounded up to a multiple of 4 (16-byte rows)
     int prune;             // skip tiles by the lower bound (resident costs, two layer groups)
@@ -1722,6 +1725,70 @@ __device__ __forceinline__ float band_threshold(const FastArgs &a, int i, float 
     return __fadd_rn(m32, __fmul_rn(m32, a.prm->tau[i]));
 }
 
+// The candidates of output (g, i, j)'s band, by the 32 lanes of a warp together, with
+// visit_tile's verdicts (fp32 value <= thr): f(in, k) is called by every lane at once
+// (a warp-uniform call; `in` is false for a lane without a candidate in that step).
+// With resident costs the lanes split every tile's k (the table gives any pair
+// directly); otherwise they take whole tiles and walk them in step along visit_tile's
+// recurrence (k descending from the anchor at the tile's top pair, or from the empty
+// interval (j, j] on the diagonal tile), so the values, and the verdicts, are visit_tile's.
+template <typename F>
+__device__ __forceinline__ void warp_visit_band(const FastArgs &a, int g, int i, int64_t j, uint64_t w, float thr,
+                                                F &&f) {
+    const int lane = threadIdx.x & 31;
+    const uint32_t w1 = (uint32_t)w, w2 = (uint32_t)(w >> 32);
+    const uint32_t n1 = (w1 & 0xFFFFu) - (w1 >> 16) + 1u;
+    const uint32_t ntile = n1 + (w2 ? (w2 & 0xFFFFu) - (w2 >> 16) + 1u : 0u);
+    const float lam32 = a.prm->lam32[g];
+    const int64_t J = j / BJ, j0 = J * BJ;
+    if (a.costs) {
+        for (uint32_t t = 0; t < ntile; t++) {
+            const int64_t K = t < n1 ? (w1 >> 16) + t : (w2 >> 16) + (t - n1);
+            const int64_t k0 = K * BK;
+            const float *cr = a.costs + (cost_tile_idx(K, J) - a.tile_base) * kCostTileFloats + (size_t)(j - j0) * PSTR;
+            const float *pr = cr + kCostHalfFloats;
+            const float *prev32 = a.dp32 + d32(a, g, i - 1, k0) - k0;
+            const int64_t khi = (K == J) ? j - 1 : k0 + BK - 1;
+            for (int64_t kb = k0; kb <= khi; kb += 32) {  // warp-uniform
+                const int64_t k = kb + lane;
+                f(k <= khi && cand32(prev32[k], lam32, cr[k - k0], pr[k - k0]) <= thr, k);
+            }
+        }
+        return;
+    }
+    const float vj = a.v[j], d_f = (float)a.d;
+    for (uint32_t tb = 0; tb < ntile; tb += 32) {  // warp-uniform
+        const uint32_t t = tb + lane;
+        // tile K of the band (lanes past the band's end take tile 0 and no candidate)
+        const int64_t K = t >= ntile ? 0 : (int64_t)(t < n1 ? (w1 >> 16) + t : (w2 >> 16) + (t - n1));
+        const int64_t k0 = K * BK;
+        const float *prev32 = a.dp32 + d32(a, g, i - 1, k0) - k0;
+        Rec r = rec_empty();
+        int64_t kfirst = k0 + BK - 1;
+        int nk = 0;  // candidates of the lane's tile: k = kfirst, kfirst - 1, ..., kfirst - nk + 1
+        if (t < ntile) {
+            if (K == J) {
+                kfirst = j - 1;
+                nk = (int)(j - k0);
+            } else {
+                nk = BK;
+                rec_anchor(a, kfirst, j, r);
+            }
+        }
+        for (int it = 0; it < BK; it++) {  // warp-uniform
+            const int64_t k = kfirst - it;
+            bool in = false;
+            if (it < nk) {
+                if (it > 0 || K == J) rec_step(r, vj, a.v[k + 1], a.wf[k + 1], __fsub_rn(a.v[k + 1], a.v[k]));
+                float c, ph;
+                rec_emit(r, vj, a.v[k], d_f, a.invd, c, ph);
+                in = cand32(prev32[k], lam32, c, ph) <= thr;
+            }
+            f(in, k);
+        }
+    }
+}
+
 // Outputs eq. apx_final reads: dp(i, p-1) for i in [ilo, s] (or every output).
 __global__ void k_need_init(FastArgs a, int ilo, int all) {
     int64_t tot = (int64_t)a.G * (a.s + 1) * a.ps;
@@ -1753,17 +1820,21 @@ __device__ __forceinline__ int32_t *layer_list(const FastArgs &a, int i, int kin
 }
 
 // Backward closure, layer i: members of every needed output; mark (i-1, k) needed;
-// list the needed outputs for the exact stage (inline members / big bands).
+// list the needed outputs for the exact stage (inline members / big bands).  A thread
+// walks an output's band when it spans at most kThreadTiles tiles; wider bands go to
+// k_need_wide, a warp each (threads of one warp walking bands of very different widths
+// would wait on the widest).
+constexpr uint32_t kThreadTiles = 4;
 __global__ void k_need_layer(FastArgs a, int i) {
     if (*(volatile const int *)a.abort_flag) return;  // a wait gave up: the tables are not valid
     const int64_t tot = (int64_t)a.G * a.p;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    unsigned long long nmem = 0, nbig = 0, nover = 0;
+    unsigned long long nmem = 0, nbig = 0;
     int32_t *lsmall = layer_list(a, i, 0), *lbig = layer_list(a, i, 1);
     int *csmall = a.list_cnt + 2 * i, *cbig = csmall + 1;
     for (int64_t base = (int64_t)blockIdx.x * blockDim.x; base < tot; base += stride) {  // warp-uniform trip count
         const int64_t id = base + threadIdx.x;
-        bool listed = false;
+        bool listed = false, wide = false;
         int cnt = 0;
         int32_t packed = 0;
         if (id < tot) {
@@ -1776,29 +1847,80 @@ __global__ void k_need_layer(FastArgs a, int i) {
                     a.mcnt[o] = 0;
                 } else {
                     const uint64_t w = a.band[o];
-                    int32_t *mem = a.members + o * NMEM;
-                    uint8_t *below = a.need + oidx(a, g, i - 1, 0);
-                    const bool mark = i - 1 >= 3;
-                    visit_band(a, g, i, j, w, band_threshold(a, i, m32), [&](int64_t k) {
-                        if (cnt < NMEM) mem[cnt] = (int32_t)k;
-                        cnt++;
-                        if (mark) below[k] = 1;
-                    });
-                    a.mcnt[o] = cnt;
-                    nmem += cnt;
-                    nbig += cnt > NMEM;
-                    nover += band_tiles(w) > 32u ? 1 : 0;  // wide bands (diagnostic)
-                    listed = true;
                     packed = (int32_t)((g << 24) | (int32_t)j);
+                    if (band_tiles(w) > kThreadTiles) {
+                        wide = true;  // a warp walks it (k_need_wide): lanes' walks would diverge
+                    } else {
+                        int32_t *mem = a.members + o * NMEM;
+                        uint8_t *below = a.need + oidx(a, g, i - 1, 0);
+                        const bool mark = i - 1 >= 3;
+                        visit_band(a, g, i, j, w, band_threshold(a, i, m32), [&](int64_t k) {
+                            if (cnt < NMEM) mem[cnt] = (int32_t)k;
+                            cnt++;
+                            if (mark) below[k] = 1;
+                        });
+                        a.mcnt[o] = cnt;
+                        nmem += cnt;
+                        nbig += cnt > NMEM;
+                        listed = true;
+                    }
                 }
             }
         }
         warp_append(0xffffffffu, listed && cnt <= NMEM, packed, lsmall, csmall);
         warp_append(0xffffffffu, listed && cnt > NMEM, packed, lbig, cbig);
+        warp_append(0xffffffffu, wide, packed, a.wide, a.wide_cnt + i);
     }
     if (nmem) atomicAdd((unsigned long long *)&a.st->members, nmem);
     if (nbig) atomicAdd((unsigned long long *)&a.st->big_bands, nbig);
-    if (nover) atomicAdd((unsigned long long *)&a.st->overflow, nover);
+}
+
+// The closure of layer i for the outputs k_need_layer deferred: a warp per output walks
+// its band (warp_visit_band), marks (i-1, k) needed for every member, keeps the first
+// NMEM members it meets (the exact stage's rule is order-free) and lists the output.
+__global__ void __launch_bounds__(128) k_need_wide(FastArgs a, int i) {
+    if (*(volatile const int *)a.abort_flag) return;  // a wait gave up: the tables are not valid
+    const int n = a.wide_cnt[i];
+    const int lane = threadIdx.x & 31;
+    const unsigned lt = (1u << lane) - 1u;
+    const int warps = gridDim.x * (blockDim.x >> 5);
+    const bool mark = i - 1 >= 3;
+    int32_t *lsmall = layer_list(a, i, 0), *lbig = layer_list(a, i, 1);
+    int *csmall = a.list_cnt + 2 * i, *cbig = csmall + 1;
+    unsigned long long nmem = 0, nbig = 0, nover = 0;  // lane 0
+    for (int e = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); e < n; e += warps) {
+        const int32_t v = a.wide[e];
+        const int g = v >> 24;
+        const int64_t j = v & 0xFFFFFF;
+        const size_t o = oidx(a, g, i, j);
+        const uint64_t w = a.band[o];
+        int32_t *mem = a.members + o * NMEM;
+        uint8_t *below = a.need + oidx(a, g, i - 1, 0);
+        int cnt = 0;  // warp-uniform
+        warp_visit_band(a, g, i, j, w, band_threshold(a, i, a.dp32[d32(a, g, i, j)]), [&](bool in, int64_t k) {
+            const unsigned mask = __ballot_sync(0xffffffffu, in);
+            if (in) {
+                const int pos = cnt + __popc(mask & lt);
+                if (pos < NMEM) mem[pos] = (int32_t)k;
+                if (mark) below[k] = 1;
+            }
+            cnt += __popc(mask);
+        });
+        if (lane == 0) {
+            a.mcnt[o] = cnt;
+            nmem += cnt;
+            nbig += cnt > NMEM;
+            nover += band_tiles(w) > 32u ? 1 : 0;  // wide bands (diagnostic)
+            if (cnt <= NMEM) lsmall[atomicAdd(csmall, 1)] = v;
+            else lbig[atomicAdd(cbig, 1)] = v;
+        }
+        __syncwarp();
+    }
+    if (lane == 0) {
+        if (nmem) atomicAdd((unsigned long long *)&a.st->members, nmem);
+        if (nbig) atomicAdd((unsigned long long *)&a.st->big_bands, nbig);
+        if (nover) atomicAdd((unsigned long long *)&a.st->overflow, nover);
+    }
 }
 
 // Outputs the answer does not read keep their fp32 minimum: dp64 = m32, bp = -2.
@@ -1926,14 +2048,11 @@ __global__ void __launch_bounds__(128) k_exact_small(Prefix P, FastArgs a, int i
 }
 
 // Layer i, outputs with more members: one warp each (fp32 re-evaluation within the
-// band, exact re-scoring of the members met), then the lanes' results meet (value,
-// then lowest k).  With resident costs the lanes split every tile's k (the table
-// gives any pair directly); otherwise they take whole tiles and walk them in step
-// (the recurrence of visit_tile runs along k, so its values, and the members, are
-// the ones the closure stage found).  Either way the members met wait in the warp's
-// queue, and each time it holds 32 every lane re-scores one of them in binary64, so
-// the binary64 sequence runs with all lanes busy (the result, least value then lowest
-// k, does not depend on the order).
+// band by warp_visit_band, whose verdicts are the closure stage's; exact re-scoring of
+// the members met), then the lanes' results meet (value, then lowest k).  The members
+// met wait in the warp's queue, and each time it holds 32 every lane re-scores one of
+// them in binary64, so the binary64 sequence runs with all lanes busy (the result,
+// least value then lowest k, does not depend on the order).
 __global__ void __launch_bounds__(128) k_exact_big(Prefix P, FastArgs a, int i, double *dp64, int32_t *bp) {
     if (*(volatile const int *)a.abort_flag) return;  // a wait gave up: the tables are not valid
     __shared__ int32_t queue[4][32];  // per warp: band members waiting for binary64 re-scoring
@@ -1953,18 +2072,12 @@ __global__ void __launch_bounds__(128) k_exact_big(Prefix P, FastArgs a, int i, 
         const float m32 = a.dp32[d32(a, g, i, j)];
         const float thr = band_threshold(a, i, m32);
         const uint64_t w = a.band[o];
-        const uint32_t w1 = (uint32_t)w, w2 = (uint32_t)(w >> 32);
-        const uint32_t n1 = (w1 & 0xFFFFu) - (w1 >> 16) + 1u;
-        const uint32_t ntile = n1 + (w2 ? (w2 & 0xFFFFu) - (w2 >> 16) + 1u : 0u);
         const double lam = a.prm->lam64[g];
-        const float lam32 = a.prm->lam32[g];
         const double *prev = dp64 + oidx(a, g, i - 1, 0);
-        const int64_t J = j / BJ, j0 = J * BJ;
         double best = CUDART_INF;
         int32_t arg = INT32_MAX;
         int qn = 0;  // warp-uniform queue length
-        // every lane calls this with its verdict on candidate k (warp-uniform call)
-        auto push = [&](bool in, int64_t k) {
+        warp_visit_band(a, g, i, j, w, thr, [&](bool in, int64_t k) {
             const unsigned mask = __ballot_sync(0xffffffffu, in);
             if (!mask) return;
             const int cnt = __popc(mask), pos = qn + __popc(mask & lt);
@@ -1980,55 +2093,7 @@ __global__ void __launch_bounds__(128) k_exact_big(Prefix P, FastArgs a, int i, 
             } else {
                 qn += cnt;
             }
-        };
-        if (a.costs) {
-            for (uint32_t t = 0; t < ntile; t++) {
-                const int64_t K = t < n1 ? (w1 >> 16) + t : (w2 >> 16) + (t - n1);
-                const int64_t k0 = K * BK;
-                const float *cr = a.costs + (cost_tile_idx(K, J) - a.tile_base) * kCostTileFloats + (size_t)(j - j0) * PSTR;
-                const float *pr = cr + kCostHalfFloats;
-                const float *prev32 = a.dp32 + d32(a, g, i - 1, k0) - k0;
-                const int64_t khi = (K == J) ? j - 1 : k0 + BK - 1;
-                for (int64_t kb = k0; kb <= khi; kb += 32) {  // warp-uniform
-                    const int64_t k = kb + lane;
-                    push(k <= khi && cand32(prev32[k], lam32, cr[k - k0], pr[k - k0]) <= thr, k);
-                }
-            }
-        } else {
-            const float vj = a.v[j], d_f = (float)a.d;
-            for (uint32_t tb = 0; tb < ntile; tb += 32) {  // warp-uniform
-                const uint32_t t = tb + lane;
-                // tile K of the band (lanes past the band's end take tile 0 and no candidate)
-                const int64_t K = t >= ntile ? 0 : (int64_t)(t < n1 ? (w1 >> 16) + t : (w2 >> 16) + (t - n1));
-                const int64_t k0 = K * BK;
-                const float *prev32 = a.dp32 + d32(a, g, i - 1, k0) - k0;
-                // the state visit_tile starts from: the anchor at the tile's top pair, or the
-                // empty interval (j, j] on the diagonal tile (which steps before its first value)
-                Rec r = rec_empty();
-                int64_t kfirst = k0 + BK - 1;
-                int nk = 0;  // candidates of the lane's tile: k = kfirst, kfirst - 1, ..., kfirst - nk + 1
-                if (t < ntile) {
-                    if (K == J) {
-                        kfirst = j - 1;
-                        nk = (int)(j - k0);
-                    } else {
-                        nk = BK;
-                        rec_anchor(a, kfirst, j, r);
-                    }
-                }
-                for (int it = 0; it < BK; it++) {  // warp-uniform
-                    const int64_t k = kfirst - it;
-                    bool in = false;
-                    if (it < nk) {
-                        if (it > 0 || K == J) rec_step(r, vj, a.v[k + 1], a.wf[k + 1], __fsub_rn(a.v[k + 1], a.v[k]));
-                        float c, ph;
-                        rec_emit(r, vj, a.v[k], d_f, a.invd, c, ph);
-                        in = cand32(prev32[k], lam32, c, ph) <= thr;
-                    }
-                    push(in, k);
-                }
-            }
-        }
+        });
         if (lane < qn) {
             exact_candidate(P, prev, qw[lane], j, lam, best, arg);
             nres++;
@@ -2066,7 +2131,8 @@ static size_t band_core_bytes(int64_t d, int32_t s) {
            align256(8 * (size_t)kMaxG * nJ + 64) + align256(sizeof(FastParams)) + align256(32 * nJ * (nJ + 1) / 2) +
            align256(4 * (size_t)kMaxG * (size_t)mdp_stride(s) * nJ) +
            align256(2 * 4 * (size_t)kMaxG * (size_t)(s + 1) * (size_t)table_stride(d)) +
-           align256(4 * 2 * (size_t)(s + 1));
+           align256(4 * 2 * (size_t)(s + 1)) + align256(4 * (size_t)kMaxG * (size_t)table_stride(d)) +
+           align256(4 * (size_t)(s + 1));
 }
 static size_t seed_rows_bytes(int64_t d, int32_t s) { return align256(4 * (size_t)cdiv(d, BJ) * BJ * (size_t)(s + 1)); }
 size_t fast_dp_band_bytes(int64_t d, int32_t s) { return band_core_bytes(d, s) + seed_rows_bytes(d, s); }
@@ -2177,6 +2243,10 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
         a.lists = reinterpret_cast<int32_t *>(q);
         q += align256(2 * 4 * (size_t)kMaxG * (size_t)(s + 1) * (size_t)table_stride(Lw.d));
         a.list_cnt = reinterpret_cast<int *>(q);
+        q += align256(4 * 2 * (size_t)(s + 1));
+        a.wide = reinterpret_cast<int32_t *>(q);
+        q += align256(4 * (size_t)kMaxG * (size_t)table_stride(Lw.d));
+        a.wide_cnt = reinterpret_cast<int *>(q);
     }
     a.mdp_stride = mdp_stride(s);
     a.spin_limit = test_stall ? kTestSpinLimit : kSpinLimit;
@@ -2277,10 +2347,14 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
         a, ilo, exact_tables ? 1 : 0);
     ECASQ_LAUNCH_CHECK();
     ECASQ_CUDA_TRY(cudaMemsetAsync(a.list_cnt, 0, sizeof(int) * 2 * (size_t)(s + 1), st));
+    ECASQ_CUDA_TRY(cudaMemsetAsync(a.wide_cnt, 0, sizeof(int) * (size_t)(s + 1), st));
     const unsigned gl = (unsigned)std::min<int64_t>(cdiv((int64_t)G * P.p, 128), (int64_t)nsm * 64);
     for (int i = s; i >= 3; i--) {
         note_launch();
         k_need_layer<<<gl, 128, 0, st>>>(a, i);
+        ECASQ_LAUNCH_CHECK();
+        note_launch();
+        k_need_wide<<<(unsigned)nsm * 16, 128, 0, st>>>(a, i);
         ECASQ_LAUNCH_CHECK();
     }
     note_launch();

@@ -260,9 +260,12 @@ def test_two_part_publish_bit_identical_to_one_part(E, name, s):
         _free()
 
 
-@pytest.mark.parametrize("name,s,b", [("studentt16k", 16, 2.5), ("lognormal16k", 16, 1.0), ("studentt20001", 12, 2.5),
-                                      ("normal8192", 10, 2.0)])
-def test_seeded_search_bit_identical_to_unseeded(E, name, s, b):
+@pytest.mark.parametrize("name,s,b,mode", [("studentt16k", 16, 2.5, "RESIDENT_COSTS"),
+                                           ("lognormal16k", 16, 1.0, "RESIDENT_COSTS"),
+                                           ("studentt20001", 12, 2.5, "RESIDENT_COSTS"),
+                                           ("normal8192", 10, 2.0, "RESIDENT_COSTS"),
+                                           ("studentt16k", 16, 2.5, "STREAMED_COSTS")])
+def test_seeded_search_bit_identical_to_unseeded(E, name, s, b, mode):
     """Later passes of the search start their tile skipping from the fp32 minima of the
     bracket's evaluated upper end (an upper bound of theirs: candidates are non-decreasing
     in lambda').  Same multiplier, codebook and metrics as without; with every output
@@ -271,11 +274,12 @@ def test_seeded_search_bit_identical_to_unseeded(E, name, s, b):
          "lognormal16k": lambda: workloads.signed_lognormal(16384, 0),
          "studentt20001": lambda: workloads.student_t(20001, 5, scale=1.0),
          "normal8192": lambda: workloads.normal(8192, 7)}[name]()
+    cost = getattr(E, mode)  # streamed costs: bands of column blocks, tile skipping and seeds as resident
     out = {}
     for extra in (0, E.UNSEEDED_SEARCH):
-        ws = E.workspace(x.size, s, flags=E.RESIDENT_COSTS)
+        ws = E.workspace(x.size, s, flags=cost)
         Q, res = E.ecasq_solve(x, s, budget_bits=b, refine_max_rounds=0,
-                               flags=E.RESIDENT_COSTS | E.EXACT_TABLES | extra, ws=ws)
+                               flags=cost | E.EXACT_TABLES | extra, ws=ws)
         st = E.native.ws_status(ws)
         assert st["timeout"] == 0 and st["bound_viol"] == 0
         out[extra] = (Q.cpu().numpy(), res, st, _tables(E, ws, st["last_G"], s, x.size))
