@@ -656,13 +656,18 @@ __device__ __forceinline__ ConsId cons_id(const FastArgs &a, int ct) {
     return id;
 }
 
-struct ConsState {
-    float best[LPT][JPT];
-    uint32_t w1[LPT][JPT], w2[LPT][JPT];  // band runs (band_update)
+// The outputs a consumer thread owns: LP layers x JPT columns (LP = LPT, or 8 for the
+// generic path of the resident kernel at larger s: see launch_dp_fast).
+template <int LP>
+struct ConsStateT {
+    float best[LP][JPT];
+    uint32_t w1[LP][JPT], w2[LP][JPT];  // band runs (band_update)
 };
-__device__ __forceinline__ void cons_reset(ConsState &cs) {
+using ConsState = ConsStateT<LPT>;
+template <int LP>
+__device__ __forceinline__ void cons_reset(ConsStateT<LP> &cs) {
 #pragma unroll
-    for (int l = 0; l < LPT; l++)
+    for (int l = 0; l < LP; l++)
 #pragma unroll
         for (int q = 0; q < JPT; q++) { cs.best[l][q] = CUDART_INF_F; cs.w1[l][q] = 0u; cs.w2[l][q] = 0u; }
 }
@@ -703,20 +708,21 @@ __device__ __forceinline__ void cons_seed(const FastArgs &a, ConsState &cs, int 
 // running minimum is kept as int bits and updated with integer min (ALU pipe)
 // next to the packed adds (FMA pipe).
 // Returns false when the warp skipped the tile (see below).
+template <int LP>
 __device__ __forceinline__ bool cons_offdiag(const FastArgs &a, const Smem &S, const float *sDPb, int b, uint32_t K,
-                                             int g, const ConsId &id, ConsState &cs) {
+                                             int g, const ConsId &id, ConsStateT<LP> &cs) {
     const int L = a.s - 2;
-    int cm[LPT][JPT];
+    int cm[LP][JPT];
 #pragma unroll
-    for (int l = 0; l < LPT; l++)
+    for (int l = 0; l < LP; l++)
 #pragma unroll
         for (int q = 0; q < JPT; q++) cm[l][q] = 0x7f800000;  // +inf
     const float *dpb = sDPb + (size_t)id.gl * L * BK;
     const float lam = S.lam32[g];
     const float2 lam2 = make_float2(lam, lam);
-    int rowl[LPT];
+    int rowl[LP];
 #pragma unroll
-    for (int l = 0; l < LPT; l++) rowl[l] = min(id.lg * LPT + l, L - 1);
+    for (int l = 0; l < LP; l++) rowl[l] = min(id.lg * LP + l, L - 1);
     if (a.prune) {
         // Exact tile skipping.  Every candidate of the tile for output (l, q) is
         // >= lb = fl(min dp(i-1, .) + fl(fma(lam, min Phi, min C))) (rounding is monotone);
@@ -731,7 +737,7 @@ __device__ __forceinline__ bool cons_offdiag(const FastArgs &a, const Smem &S, c
         }
         bool need = false;
 #pragma unroll
-        for (int l = 0; l < LPT; l++) {
+        for (int l = 0; l < LP; l++) {
             const float m = md[rowl[l]], tau = S.tau[3 + rowl[l]];
 #pragma unroll
             for (int q = 0; q < JPT; q++) {
@@ -752,7 +758,7 @@ __device__ __forceinline__ bool cons_offdiag(const FastArgs &a, const Smem &S, c
             W[q][1] = fma2(lam2, make_float2(f4.z, f4.w), make_float2(c4.z, c4.w));
         }
 #pragma unroll
-        for (int l = 0; l < LPT; l++) {
+        for (int l = 0; l < LP; l++) {
             // layer i = 3 + li uses dp row 2 + li; rows past the last layer are
             // clamped (their results are never used)
             const float4 d4 = *reinterpret_cast<const float4 *>(dpb + (size_t)rowl[l] * BK + kk);
@@ -769,7 +775,7 @@ __device__ __forceinline__ bool cons_offdiag(const FastArgs &a, const Smem &S, c
     // band bookkeeping (branch-free; layers past the last one carry state that is never read)
     const uint32_t KK = (K << 16) | K;
 #pragma unroll
-    for (int l = 0; l < LPT; l++) {
+    for (int l = 0; l < LP; l++) {
         const float tau = S.tau[3 + rowl[l]];
 #pragma unroll
         for (int q = 0; q < JPT; q++) band_fold(__int_as_float(cm[l][q]), cs.best[l][q], tau, cs.w1[l][q], cs.w2[l][q], K, KK);
@@ -785,8 +791,9 @@ __device__ __forceinline__ bool cons_offdiag(const FastArgs &a, const Smem &S, c
 // by a shuffle.  All `a.ncons` consumer threads take part (BAR_CONS).
 // staged: S.diag[0] already holds layer 2 of the block (bulk copy), else it is
 // loaded here.
+template <int LP>
 __device__ __forceinline__ void cons_diag(const FastArgs &a, Smem &S, int b, int J, int split, const ConsId &id,
-                                          ConsState &cs, bool staged) {
+                                          ConsStateT<LP> &cs, bool staged) {
     const int L = a.s - 2;
     const int ct = id.ct;
     const int g = split * a.Gc + id.gl;
@@ -808,7 +815,7 @@ __device__ __forceinline__ void cons_diag(const FastArgs &a, Smem &S, int b, int
     int cur = 0;
     for (int li = 0; li < L; li++) {
         const int i = 3 + li;
-        const int olg = li / LPT, l = li - olg * LPT;
+        const int olg = li / LP, l = li - olg * LP;
         const bool owner = own && id.lg == olg;
         const int kbeg = (pair && !owner) ? BJ / 2 : 0;
         const int kend = (pair && owner) ? BJ / 2 : BJ;
@@ -841,7 +848,7 @@ __device__ __forceinline__ void cons_diag(const FastArgs &a, Smem &S, int b, int
         }
         if (owner) {
 #pragma unroll
-            for (int lx = 0; lx < LPT; lx++) {
+            for (int lx = 0; lx < LP; lx++) {
                 if (lx != l) continue;
 #pragma unroll
                 for (int q = 0; q < JPT; q++) {
@@ -1427,6 +1434,7 @@ __device__ __forceinline__ uint32_t need_mask(const FastArgs &a, const Smem &S, 
 // warp runs need_mask over the batch and only the tiles some warp needs are copied
 // in and walked, so a tile every warp rules out costs neither HBM traffic nor a
 // barrier; the next batch is staged while this one is walked.
+template <int LP>
 __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     Smem &S = *reinterpret_cast<Smem *>(smem_raw);
@@ -1446,7 +1454,7 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
     }
     __syncthreads();
     const ConsId id = cons_id(a, ct);
-    ConsState cs;
+    ConsStateT<LP> cs;
     const uint64_t policy = policy_evict_first();
     uint32_t n = 0;   // tile sequence number: buffer n & 1
     uint32_t mph[2] = {0u, 0u};  // completed phases of mbar[0], mbar[1] (one per fill; two for a split last tile)
@@ -1465,7 +1473,9 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
         const bool own = id.active && g < a.G;
         if (split != fsplit) { frontier = -1; fsplit = split; }
         cons_reset(cs);
-        if (a.seed && own) cons_seed(a, cs, J, id);
+        if constexpr (LP == LPT) {  // seeds, tile skipping and the split publish: LPT only
+            if (a.seed && own) cons_seed(a, cs, J, id);
+        }
         int issued = -1;  // the tile whose copies are in flight into buffer n & 1 (J: the diagonal), or -1
         const int ngv = min(a.G - split * a.Gc, a.Gc);  // real multipliers of the split
         // the tiles walked here: K < Kend (with a split publish the last one, J - 1, is the chain's)
@@ -1484,7 +1494,7 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
                 mbar_wait_bounded(&S.smbar[sb], (ns >> 1) & 1u, a.st, a.abort_flag);
                 frb = S.sfront[sb];
                 if (lane == 0) fence_proxy_async_global();  // blocks <= frb, published, before this warp's copies
-                wm = own ? need_mask(a, S, stage + sb * sfl, K0, K1, frb, g, id, cs) : 0u;
+                if constexpr (LP == LPT) wm = own ? need_mask(a, S, stage + sb * sfl, K0, K1, frb, g, id, cs) : 0u;
                 if (lane == 0) S.needw[sb][ct >> 5] = wm;
                 __syncthreads();  // needw; every read of stage buffer sb is done
                 U = 0;
@@ -1546,7 +1556,16 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
             }
             K0 = K1;
         }
-        if (a.split_pub) {
+        if constexpr (LP != LPT) {  // the generic diagonal (no split publish, no parked state)
+            const int b = n & 1;
+            if (issued != J && ct < 32) res_issue(a, S, sDP, b, J, J, split, policy, lane);
+            mbar_wait_bounded(&S.mbar[b], mph[b] & 1u, a.st, a.abort_flag);
+            mph[b]++;
+            cons_diag(a, S, b, J, split, id, cs, true);
+            __syncthreads();  // every thread's dp32 and layer minima of block J are stored
+            if (ct == 0) publish_block(a, split, J);
+            n++;
+        } else if (a.split_pub) {
             // the chain's part: tile (J-1, J) in buffer bA, the diagonal in bD (the cost copies
             // depend on nothing published; the diagonal also copies row 2 of block J)
             uint32_t *park = reinterpret_cast<uint32_t *>(sDP + (size_t)2 * rowsDP * BK);
@@ -2208,7 +2227,19 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     a.invd = 1.0f / (float)P.d;  // IEEE division on the host: correctly rounded
     a.G = G;
     a.s = s;
-    a.lgc = (int)cdiv(s - 2, LPT);
+    // Layers per consumer thread: LPT, or 8 on the resident kernel's generic path (no tile
+    // skipping) when that costs fewer layer slots times multiplier splits; at s = 32, 4
+    // groups of 8 layers (64 threads per multiplier, 4 multipliers per split) against 5
+    // of 7 (80 threads, 3 per split): 2 splits of 8 slots per pass instead of 3 of 7.
+    int lp = LPT;
+    if (costs && !(cdiv(s - 2, LPT) == 2 && mdp_stride(s) <= 20)) {
+        auto slots = [&](int l) {
+            const int lgc = (int)cdiv(s - 2, l), gc = std::max(1, std::min(G, MAXCONS / (lgc * NJQ)));
+            return (int64_t)cdiv(G, gc) * l;
+        };
+        if (cdiv(s - 2, 8) * NJQ <= MAXCONS && slots(8) < slots(LPT)) lp = 8;
+    }
+    a.lgc = (int)cdiv(s - 2, lp);
     a.Gc = std::max(1, std::min(G, MAXCONS / (a.lgc * NJQ)));
     a.nsplit = (int)cdiv(G, a.Gc);
     a.nJ = (int)cdiv(P.p, BJ);
@@ -2251,9 +2282,9 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     a.mdp_stride = mdp_stride(s);
     a.spin_limit = test_stall ? kTestSpinLimit : kSpinLimit;
     // two-part publishing of each block (the chain's last tile in two layer groups)
-    a.split_pub = (costs && a.lgc == 2 && !split_off) ? 1 : 0;
+    a.split_pub = (costs && lp == LPT && a.lgc == 2 && !split_off) ? 1 : 0;
     a.hold0 = test_stall ? 1 : 0;
-    a.prune = (costs && a.lgc == 2 && a.mdp_stride <= 20) ? 1 : 0;
+    a.prune = (costs && lp == LPT && a.lgc == 2 && a.mdp_stride <= 20) ? 1 : 0;
     a.seed = (seeded && a.prune && s == Lw.s) ? seed_rows(ws, Lw) : nullptr;
     a.costs = costs;
     a.tile_base = 0;
@@ -2294,10 +2325,10 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
         ECASQ_LAUNCH_CHECK();
     }
     size_t smem = smem_bytes(a.Gc, s);
-    if (costs && a.lgc == 2)  // parked band state; off the diagonal, the two stage buffers
+    if (costs && lp == LPT && a.lgc == 2)  // parked band state; off the diagonal, the two stage buffers
         smem += std::max((size_t)3 * LPT * JPT * a.ncons * sizeof(uint32_t),
                          a.prune ? 2 * stage_floats(G, a.mdp_stride) * sizeof(float) : (size_t)0);
-    auto wave = costs ? k_wavefront_res : k_wavefront;
+    auto wave = costs ? (lp == 8 ? k_wavefront_res<8> : k_wavefront_res<LPT>) : k_wavefront;
     ECASQ_CUDA_TRY(cudaFuncSetAttribute(wave, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     int per_sm = 0;
     if (costs && build_costs)

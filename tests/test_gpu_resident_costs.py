@@ -39,11 +39,16 @@ def _tables(E, ws, G, s, d):
 
 
 @pytest.mark.parametrize("flags_name", ["DEFAULT", "EXACT_TABLES"])
-@pytest.mark.parametrize("name,s", [("lognormal16k", 16), ("ragged2049", 9)])
+@pytest.mark.parametrize("name,s", [("lognormal16k", 16), ("ragged2049", 9), ("mixture12k", 32), ("ragged5000", 18)])
 def test_resident_costs_bit_identical_to_fused(E, name, s, flags_name):
     """Same codebooks and metrics with and without resident costs; the same
-    exact tables; the same fp32 minima where the closure left outputs unresolved."""
-    x = workloads.signed_lognormal(16384, 0) if name == "lognormal16k" else workloads.student_t(2049, 3, scale=1.0)
+    exact tables; the same fp32 minima where the closure left outputs unresolved.
+    At s = 32 and s = 18 the resident kernel runs eight layers per thread (the fused
+    kernel seven)."""
+    x = {"lognormal16k": lambda: workloads.signed_lognormal(16384, 0),
+         "ragged2049": lambda: workloads.student_t(2049, 3, scale=1.0),
+         "mixture12k": lambda: workloads.mixture(12288, 2),
+         "ragged5000": lambda: workloads.student_t(5000, 6, scale=1.0)}[name]()
     flags = getattr(E, flags_name, 0)
     lams = [0.0, 1e-5, 1e-3, 0.01, 0.05, 0.2, 1.0, 10.0]
     wsf = E.workspace(x.size, s)
