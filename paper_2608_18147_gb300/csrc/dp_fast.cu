@@ -1179,6 +1179,7 @@ __device__ __forceinline__ void publish_lower(const FastArgs &a, int split, int 
 // Fused producer: two producer warps compute each tile's interval costs
 // (tile_columns) and stage the dp32 rows with cp.async while the consumer warps
 // evaluate the previous tile (named barriers FULL / EMPTY per buffer).
+template <int LP>
 __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     Smem &S = *reinterpret_cast<Smem *>(smem_raw);
@@ -1255,7 +1256,7 @@ __global__ void __launch_bounds__(NPROD + MAXCONS, 1) k_wavefront(FastArgs a) {
 
     // ============================= consumer warps =============================
     const ConsId id = cons_id(a, tid - NPROD);
-    ConsState cs;
+    ConsStateT<LP> cs;
     uint32_t n = 0;
     for (;;) {
         int b = n & 1;
@@ -2227,12 +2228,13 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     a.invd = 1.0f / (float)P.d;  // IEEE division on the host: correctly rounded
     a.G = G;
     a.s = s;
-    // Layers per consumer thread: LPT, or 8 on the resident kernel's generic path (no tile
-    // skipping) when that costs fewer layer slots times multiplier splits; at s = 32, 4
-    // groups of 8 layers (64 threads per multiplier, 4 multipliers per split) against 5
-    // of 7 (80 threads, 3 per split): 2 splits of 8 slots per pass instead of 3 of 7.
+    // Layers per consumer thread: LPT, or 8 on the generic path (the fused kernel, or the
+    // resident one without tile skipping) when that costs fewer layer slots times
+    // multiplier splits; at s = 32, 4 groups of 8 layers (64 threads per multiplier, 4
+    // multipliers per split) against 5 of 7 (80 threads, 3 per split): 2 splits of 8
+    // slots per pass instead of 3 of 7.
     int lp = LPT;
-    if (costs && !(cdiv(s - 2, LPT) == 2 && mdp_stride(s) <= 20)) {
+    if (!(costs && cdiv(s - 2, LPT) == 2 && mdp_stride(s) <= 20)) {
         auto slots = [&](int l) {
             const int lgc = (int)cdiv(s - 2, l), gc = std::max(1, std::min(G, MAXCONS / (lgc * NJQ)));
             return (int64_t)cdiv(G, gc) * l;
@@ -2328,7 +2330,8 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     if (costs && lp == LPT && a.lgc == 2)  // parked band state; off the diagonal, the two stage buffers
         smem += std::max((size_t)3 * LPT * JPT * a.ncons * sizeof(uint32_t),
                          a.prune ? 2 * stage_floats(G, a.mdp_stride) * sizeof(float) : (size_t)0);
-    auto wave = costs ? (lp == 8 ? k_wavefront_res<8> : k_wavefront_res<LPT>) : k_wavefront;
+    auto wave = costs ? (lp == 8 ? k_wavefront_res<8> : k_wavefront_res<LPT>)
+                      : (lp == 8 ? k_wavefront<8> : k_wavefront<LPT>);
     ECASQ_CUDA_TRY(cudaFuncSetAttribute(wave, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     int per_sm = 0;
     if (costs && build_costs)

@@ -110,6 +110,8 @@ def test_dp_parity_normal1024(E, oracle_mod, lams, flags_name):
     ("tiny_offset", 9, [0.0, 0.02, 0.5]),
     ("normal1024", 3, [0.0, 0.3]),
     ("normal1024", 23, [0.0, 0.01, 0.2, 1.0, 5.0, 20.0, 100.0]),
+    ("ragged2049", 32, [0.0, 1e-3, 0.02, 0.3, 2.0, 9.0, 30.0, 100.0]),  # 8 layers per thread, 2 splits
+    ("normal1024", 18, [0.0, 0.05, 0.4]),                                # 8 layers per thread, 2 groups
 ])
 def test_dp_fast_parity(E, oracle_mod, name, s, lams):
     """The fast kernel (fp32 filter + certified band + exact re-scoring) against the oracle."""
