@@ -399,7 +399,7 @@ def run_rows_mode(args):
     launches0 = E.ecasq_kernel_launches()
     ms, outs, clocks = _timed_steps(args, lambda: E.ecasq_solve_batched(X, s, budget_bits=budget, ws=ws))
     Q, m, res = outs[-1]
-    ok = sum(1 for r in res if r["status"] == 0)
+    ok = int((res.field("status") == 0).sum())
     out = {"metric": "ECASQ batched solve: rows/s", "value": args.steps * rows / (ms / 1000.0), "unit": "rows/s",
            "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
            "higher_is_better": True, "vs_baseline": None, "dtype": "f64", "data": "synthetic",

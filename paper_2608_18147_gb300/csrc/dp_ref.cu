@@ -202,6 +202,7 @@ __global__ void __launch_bounds__(256) k_rows_pass(RowsPass A) {
     int8_t *bps = reinterpret_cast<int8_t *>(d32 + 2 * (size_t)G * p);  // [G][s+1][p]
     __shared__ int32_t a_sm[kMaxS];
     __shared__ int sm_m;
+    __shared__ int next_out[2];  // per layer parity: outputs handed out so far
     // the row's scale 2^-e (2^e <= ||X_row||^2 < 2^(e+1)) keeps the fp32 copies near 1
     const double n2 = R.norm2[row];
     const double scale = (n2 > 0.0 && isfinite(n2)) ? ldexp(1.0, -ilogb(n2)) : 1.0;
@@ -242,6 +243,7 @@ __global__ void __launch_bounds__(256) k_rows_pass(RowsPass A) {
         }
     }
     for (int q = threadIdx.x; q < G * (s + 1); q += blockDim.x) last[q] = CUDART_INF;
+    if (threadIdx.x < 2) next_out[threadIdx.x] = 0;
     int32_t *bp = A.bp + (size_t)b * G * (s + 1) * dcap;
     const bool bp_sm = A.bp_smem != 0;
     auto set_bp = [&](int g, int i, int j, int32_t v) {
@@ -268,46 +270,69 @@ __global__ void __launch_bounds__(256) k_rows_pass(RowsPass A) {
     // input is within u = 2^-24 (relative) of its binary64 value or 2^-150 (absolute) when
     // subnormal, the fma and the add round once each, so an exact minimiser has
     // val32 <= (m32 + A)(1 + 8.0001u) + A < m32 (1 + 10u) + 3A, A = (70 + lam32) 2^-150.
+    // The outputs of a layer go to the warps in order of decreasing work (j descending, all
+    // multipliers of one j together), 32 at a time from a shared counter, so no thread
+    // waits on one that drew the longest scans.  Each output takes one fp32 pass over k:
+    // the running minimum m32 and, for every k, whether its value is within a conservative
+    // band of the running minimum, Tr(x) = ru(ru(x (1 + 2^-20)) + ru(2 slack)) >= T(x) for
+    // x >= 0, non-decreasing in x; the running minimum only falls, so every k within the
+    // final band T(m32) was within Tr of the minimum at its visit, and the bits marked hold
+    // every member (the re-scoring re-checks each against T(m32)).
+    const int lane = threadIdx.x & 31;
+    const int nout = G * p;
     int cur = 0;
     for (int i = 3; i <= s; i++) {
         const double *prev = dpb + (size_t)cur * G * p;
         const float *prev32 = d32 + (size_t)cur * G * p;
         double *nxt = dpb + (size_t)(cur ^ 1) * G * p;
         float *nxt32 = d32 + (size_t)(cur ^ 1) * G * p;
-        for (int q = threadIdx.x; q < G * p; q += blockDim.x) {
-            const int g = q / p, j = q % p;
+        int *ctr = &next_out[i & 1];
+        if (threadIdx.x == 0) next_out[(i + 1) & 1] = 0;  // the next layer's counter (unused until the barrier)
+        for (;;) {
+            int base = 0;
+            if (lane == 0) base = atomicAdd(ctr, 32);
+            base = __shfl_sync(0xffffffffu, base, 0);
+            if (base >= nout) break;  // warp-uniform
+            const int q = base + lane;
+            if (q >= nout) continue;
+            const int g = q % G, j = p - 1 - q / G;
             const int tb = j * (j - 1) / 2;
-            const int koff0 = (i - 2) * p - (i - 2) * (i - 1) / 2 - 1;  // koff(i - 2) - 1: pair (k, j) at koff + j - k
-            float m32 = CUDART_INF_F;
-            for (int k = i - 2, ko = koff0; k < j; ko += p - k - 1, k++) {
-                const float2 cf = pc32[ko + j - k];
-                m32 = fminf(m32, __fadd_rn(prev32[g * p + k], __fmaf_rn(lam32[g], cf.y, cf.x)));
+            const float l32 = lam32[g];
+            const float sl = __double2float_ru(__dmul_rn(2.0, slack[g]));
+            const float *pv = prev32 + g * p;
+            float m32 = CUDART_INF_F, Tr = CUDART_INF_F;
+            uint32_t mkw[4];
+#pragma unroll
+            for (int w = 0; w < 4; w++) {
+                const int k0 = max(i - 2, 32 * w), k1 = min(j, 32 * w + 32);
+                uint32_t mk = 0u;
+                int ko = k0 * p - k0 * (k0 + 1) / 2 - 1;  // koff(k0) - 1: pair (k, j) at ko + j - k
+                for (int k = k0; k < k1; ko += p - k - 1, k++) {
+                    const float2 cf = pc32[ko + j - k];
+                    const float v = __fadd_rn(pv[k], __fmaf_rn(l32, cf.y, cf.x));
+                    if (v < m32) {
+                        m32 = v;
+                        Tr = __fadd_ru(__fmul_ru(v, 1.0f + 0x1p-20f), sl);
+                    }
+                    mk |= (v <= Tr ? 1u : 0u) << (k & 31);
+                }
+                mkw[w] = mk;
             }
             const float T = __double2float_rd(__dadd_rn(__dmul_rn((double)m32, 1.0 + 10.0 * 0x1p-24), slack[g]));
-            // the band's members as a 128-bit mask (k < p <= kRowsMaxP), re-scored after the scan in
-            // increasing k, so a warp runs the binary64 step once per member of its busiest lane
-            // rather than once per k at which any lane has a member
-            uint32_t mk0 = 0u, mk1 = 0u, mk2 = 0u, mk3 = 0u;
-            for (int k = i - 2, ko = koff0; k < j; ko += p - k - 1, k++) {
-                const float2 cf = pc32[ko + j - k];
-                const bool in = __fadd_rn(prev32[g * p + k], __fmaf_rn(lam32[g], cf.y, cf.x)) <= T;
-                const uint32_t bit = in ? 1u << (k & 31) : 0u, w = (uint32_t)k >> 5;
-                mk0 |= w == 0u ? bit : 0u;
-                mk1 |= w == 1u ? bit : 0u;
-                mk2 |= w == 2u ? bit : 0u;
-                mk3 |= w == 3u ? bit : 0u;
-            }
+            // members re-scored in binary64 in increasing k (the lowest k among exact minima)
             double best = CUDART_INF;
             int32_t arg = -1;
 #pragma unroll
             for (int w = 0; w < 4; w++) {
-                uint32_t mk = w == 0 ? mk0 : (w == 1 ? mk1 : (w == 2 ? mk2 : mk3));
+                uint32_t mk = mkw[w];
                 while (mk) {
                     const int k = 32 * w + __ffs(mk) - 1;
                     mk &= mk - 1u;
+                    const float2 cf = pc32[k * p - k * (k + 1) / 2 + j - k - 1];
+                    if (!(__fadd_rn(pv[k], __fmaf_rn(l32, cf.y, cf.x)) <= T)) continue;
                     const double *e = gpc64 + 2 * (size_t)(tb + k);
                     const double c = __dadd_rn(prev[g * p + k], __dadd_rn(e[0], __dmul_rn(lam[g], e[1])));
-                    if (c < best) { best = c; arg = k; }  // increasing k: the lowest k among exact minima
+                    if (c < best) { best = c; arg = k; }
                 }
             }
             nxt[g * p + j] = best;

@@ -471,8 +471,34 @@ def ecasq_quantize_noalloc(x, Q, seed, idx, counts):
     return he.value
 
 
+class BatchResults:
+    """The per-row results of ecasq_solve_batched as a read-only sequence of dicts, each
+    built from the C records when it is read (building 10^4 dicts up front costs more
+    than the solve of short rows)."""
+
+    def __init__(self, records):
+        self._records = records
+
+    def __len__(self):
+        return len(self._records)
+
+    def __getitem__(self, i):
+        if isinstance(i, slice):
+            return [self._records[t].as_dict() for t in range(*i.indices(len(self._records)))]
+        return self._records[i].as_dict()
+
+    def __iter__(self):
+        for r in self._records:
+            yield r.as_dict()
+
+    def field(self, name):
+        """One field of every row, as a numpy array."""
+        return np.array([getattr(r, "lambda_" if name == "lambda" else name) for r in self._records])
+
+
 def ecasq_solve_batched(X, s, budget_bits=0.0, lambda_=-1.0, ws=None, **kw):
-    """Independent budgeted solves of the rows of X [rows, d]: (Q [rows, s], m [rows], results)."""
+    """Independent budgeted solves of the rows of X [rows, d]: (Q [rows, s], m [rows], results);
+    results is a BatchResults sequence (one dict per row, built when read)."""
     torch = _torch()
     X = _dev_f32(X)
     rows, d = X.shape
@@ -485,7 +511,7 @@ def ecasq_solve_batched(X, s, budget_bits=0.0, lambda_=-1.0, ws=None, **kw):
     rc = lib().ecasq_solve_batched(_ptr(X), rows, d, C.byref(prm), _ptr(ws), ws.numel(), _ptr(Q), _ptr(m), res,
                                    _stream())
     _check(rc, "ecasq_solve_batched", ok=(OK, EINFEASIBLE))
-    return Q, m, [r.as_dict() for r in res]
+    return Q, m, BatchResults(res)
 
 
 def ecasq_prepare(x, ws=None):
