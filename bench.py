@@ -400,11 +400,25 @@ def run_rows_mode(args):
     ms, outs, clocks = _timed_steps(args, lambda: E.ecasq_solve_batched(X, s, budget_bits=budget, ws=ws))
     Q, m, res = outs[-1]
     ok = int((res.field("status") == 0).sum())
+    # candidates of eq. apx_rec over all rows and their evaluated multipliers, against the
+    # same FP32 issue peak as the single-vector kernel (2 ops per candidate), over the whole
+    # step (host search logic and copies included, so a lower bound for the kernel)
+    cand = sum(int(l) * candidates_per_multiplier(int(pr), s)
+               for pr, l in zip(res.field("p"), res.field("lambdas_evaluated")))
+    sm_count = torch.cuda.get_device_properties(0).multi_processor_count
+    peak = sm_count * 128 * 2.07e9 / 1e12
+    achieved = 2.0 * cand / (ms / args.steps / 1000.0) / 1e12
     out = {"metric": "ECASQ batched solve: rows/s", "value": args.steps * rows / (ms / 1000.0), "unit": "rows/s",
            "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
            "higher_is_better": True, "vs_baseline": None, "dtype": "f64", "data": "synthetic",
            "config": {"workload": name, "mode": "rows", "rows": rows, "d": d, "s": s, "budget_bits": budget},
            "rows_ok": ok, "mean_m": float(m.float().mean().item()),
+           "roofline": {"bound": "alu", "achieved": achieved, "peak": peak, "unit": "TOP/s", "frac": achieved / peak,
+                        "traffic": None, "kernel": "k_rows_pass",
+                        "candidates_per_step": cand,
+                        "note": "2 ops per candidate of eq. apx_rec over the whole step; the first search round "
+                                "builds each row's binary64 pair costs (binary64 pipe), the later rounds are "
+                                "latency-bound at two 8-warp blocks per SM (shared memory per row)"},
            "gpu_launches": E.ecasq_kernel_launches() - launches0, "clocks": clocks}
     print(json.dumps(out), flush=True)
 

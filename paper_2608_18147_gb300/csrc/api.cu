@@ -1289,6 +1289,7 @@ static int solve_rows_batched(const float *X, int64_t rows, int64_t d, const eca
         double lo, hi;
         bool done = false, failed = false;
         int sel = -1, status = ECASQ_OK, passes = 0, nlam = 0;
+        int best = -1;  // the feasible evaluation the selection rule prefers so far
     };
     std::vector<Row> st_rows(rows);
     const bool fixed = prm->lambda >= 0.0;
@@ -1302,6 +1303,7 @@ static int solve_rows_batched(const float *X, int64_t rows, int64_t d, const eca
         st_rows[r].hi = hi0;
         if (ph[r] > kRowsMaxP) { slow.push_back(r); st_rows[r].done = true; }
         else if (ph[r] == 1) st_rows[r].done = true;
+        else st_rows[r].evals.reserve(fixed ? 1 : 8 + 7 * (size_t)Rn + 1);
     }
     int32_t *actd = reinterpret_cast<int32_t *>(rb + RL.act);
     double *lamd = reinterpret_cast<double *>(rb + RL.lam);
@@ -1358,7 +1360,14 @@ static int solve_rows_batched(const float *X, int64_t rows, int64_t d, const eca
                 e.hs = meth[4 * q + 2];
                 e.hx = meth[4 * q + 3];
                 e.feas = fixed ? true : (e.hs <= prm->budget_bits);
-                e.a.assign(qh.begin() + q * s, qh.begin() + q * s + std::max(e.m, 0));
+                // the codebook is kept only where it can be selected: a fixed multiplier, the
+                // closing pass at the bracket's upper end, or the best feasible point so far
+                // (least MSE, then the smaller multiplier: the final selection's rule)
+                const bool lead = e.feas && (w.best < 0 || e.mse < w.evals[w.best].mse ||
+                                             (e.mse == w.evals[w.best].mse && e.lam < w.evals[w.best].lam));
+                if (lead) w.best = (int)w.evals.size();
+                if (lead || fixed || G == 1)
+                    e.a.assign(qh.begin() + q * s, qh.begin() + q * s + std::max(e.m, 0));
                 w.evals.push_back(e);
                 if (e.m < 1) bad = true;
             }
