@@ -171,7 +171,8 @@ __global__ void k_locate_q(const float *v, int64_t p, const float *Q, int m, int
 // eval_codebook_warp.  Backpointers go to the caller's scratch.
 __host__ __device__ __forceinline__ int tri(int k, int j) { return j * (j - 1) / 2 + k; }
 
-__global__ void __launch_bounds__(256) k_rows_pass(RowsPass A) {
+constexpr int kRowsThreads = 512;  // 16 warps: two blocks per SM fit the shared-memory pair caches
+__global__ void __launch_bounds__(kRowsThreads) k_rows_pass(RowsPass A) {
     extern __shared__ __align__(16) double rsm[];
     const int b = blockIdx.x;
     const int64_t row = A.rows[b];
@@ -395,7 +396,7 @@ int launch_rows_pass(const RowsPass &A, int nact, int pmax, cudaStream_t st) {
     size_t smem = rows_pass_smem(pmax, A.G, A.s, B.bp_smem != 0);
     ECASQ_CUDA_TRY(cudaFuncSetAttribute(k_rows_pass, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     note_launch();
-    k_rows_pass<<<(unsigned)nact, 256, smem, st>>>(B);
+    k_rows_pass<<<(unsigned)nact, kRowsThreads, smem, st>>>(B);
     ECASQ_LAUNCH_CHECK();
     return ECASQ_OK;
 }
