@@ -272,6 +272,34 @@ static __device__ __noinline__ void eval_codebook_warp(const Prefix &P, const in
     __syncwarp();
 }
 
+// eval_codebook_warp for m <= 32 with no shared scratch: lane r holds interval r's C,
+// Phi (Phi^first for r = 0), U and D, and term r of the output entropy (the neighbour's U
+// by a shuffle); the three sums run in interval order from shuffled values, as there.
+static __device__ __noinline__ void eval_codebook_lanes(const Prefix &P, const int32_t *a, int m, double *out3) {
+    const int lane = threadIdx.x & 31;
+    double C = 0.0, F = 0.0, U = 0.0, D = 0.0;
+    if (lane + 1 < m) {
+        pair_exact(P, a[lane], a[lane + 1], C, U, D);
+        F = lane == 0 ? phi_first_at(P, a[0], U, D) : phi_exact(P, U, D, false);
+    }
+    const double Uprev = __shfl_up_sync(0xffffffffu, U, 1);
+    const double Ulast = __shfl_sync(0xffffffffu, U, m >= 2 ? m - 2 : 0);
+    double ht = 0.0;
+    if (m >= 2 && lane < m) {
+        const double f = lane == m - 1 ? Ulast : (lane == 0 ? __dadd_rn((double)P.w[a[0]], D) : __dadd_rn(Uprev, D));
+        ht = hfun(__ddiv_rn(f, (double)P.d));
+    }
+    double mse = 0.0, hs = 0.0, hx = 0.0;
+    for (int r = 0; r + 1 < m; r++) {
+        mse = __dadd_rn(mse, __shfl_sync(0xffffffffu, C, r));
+        hs = __dadd_rn(hs, __shfl_sync(0xffffffffu, F, r));
+        hx = __dadd_rn(hx, __shfl_sync(0xffffffffu, ht, r));
+    }
+    if (m >= 2) hx = __dadd_rn(hx, __shfl_sync(0xffffffffu, ht, m - 1));
+    if (lane == 0) { out3[0] = mse; out3[1] = hs; out3[2] = hx; }
+    __syncwarp();
+}
+
 // -------------------------------------------------------------- host helpers
 // Kernels launched by this library in this process (all threads).
 void note_launch();

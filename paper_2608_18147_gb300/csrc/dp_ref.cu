@@ -344,32 +344,46 @@ __global__ void __launch_bounds__(kRowsThreads) k_rows_pass(RowsPass A) {
         __syncthreads();
         cur ^= 1;
     }
-    // eq. apx_final and the traceback, then the metrics (one warp, multiplier by multiplier)
-    if (threadIdx.x < 32) {
-        for (int g = 0; g < G; g++) {
-            if (threadIdx.x == 0) {
-                int istar = -1;
-                double best = CUDART_INF;
-                for (int i = A.exact_s ? s : 2; i <= s; i++) {
-                    double v = last[g * (s + 1) + i];
-                    if (v < best) { best = v; istar = i; }
-                }
-                if (istar < 0) {
-                    sm_m = 0;
-                } else {
-                    int64_t j = p - 1;
-                    a_sm[istar - 1] = (int32_t)j;
-                    for (int i = istar; i >= 3; i--) {
-                        j = bp_sm ? (int64_t)bps[((size_t)g * (s + 1) + i) * p + j]
-                                  : (int64_t)bp[((size_t)g * (s + 1) + i) * dcap + j];
-                        a_sm[i - 2] = (int32_t)j;
-                    }
-                    a_sm[0] = 0;
-                    sm_m = istar;
-                }
-                A.metrics[((size_t)b * G + g) * 4 + 0] = best;
-                A.mcount[(size_t)b * G + g] = sm_m;
+    // eq. apx_final and the traceback of multiplier g into a[0..m-1] (lane 0); returns m
+    auto trace = [&](int g, int32_t *a) -> int {
+        int istar = -1;
+        double best = CUDART_INF;
+        for (int i = A.exact_s ? s : 2; i <= s; i++) {
+            double v = last[g * (s + 1) + i];
+            if (v < best) { best = v; istar = i; }
+        }
+        int m = 0;
+        if (istar >= 0) {
+            int64_t j = p - 1;
+            a[istar - 1] = (int32_t)j;
+            for (int i = istar; i >= 3; i--) {
+                j = bp_sm ? (int64_t)bps[((size_t)g * (s + 1) + i) * p + j]
+                          : (int64_t)bp[((size_t)g * (s + 1) + i) * dcap + j];
+                a[i - 2] = (int32_t)j;
             }
+            a[0] = 0;
+            m = istar;
+        }
+        A.metrics[((size_t)b * G + g) * 4 + 0] = best;
+        A.mcount[(size_t)b * G + g] = m;
+        return m;
+    };
+    if (s <= 32) {
+        // codebooks of at most 32 values: warp g takes multiplier g, its lanes holding one
+        // interval each (eval_codebook_lanes), so no warp of the block waits on a serial tail
+        __shared__ int32_t a_w[kMaxG][32];
+        __shared__ int m_w[kMaxG];
+        const int g = threadIdx.x >> 5;
+        if (g < G) {
+            if (lane == 0) m_w[g] = trace(g, a_w[g]);
+            __syncwarp();
+            const int m = m_w[g];
+            if (lane < m) A.qidx[((size_t)b * G + g) * s + lane] = a_w[g][lane];
+            if (m > 0) eval_codebook_lanes(P, a_w[g], m, &A.metrics[((size_t)b * G + g) * 4 + 1]);
+        }
+    } else if (threadIdx.x < 32) {  // one warp, multiplier by multiplier
+        for (int g = 0; g < G; g++) {
+            if (threadIdx.x == 0) sm_m = trace(g, a_sm);
             __syncwarp();
             const int m = sm_m;
             for (int r = threadIdx.x; r < m; r += 32) A.qidx[((size_t)b * G + g) * s + r] = a_sm[r];
