@@ -69,6 +69,7 @@ constexpr int64_t kMaxFastP = (int64_t)1 << 20;
 constexpr uint32_t kSpinLimit = 1u << 26;
 constexpr uint32_t kTestSpinLimit = 1u << 14;  // the ECASQ_TEST_STALL hook: about 10-20 ms of spinning
 constexpr uint32_t kCopySpinLimit = 1u << 22;  // waits on bulk copies (microseconds when healthy)
+constexpr int kMdpMax = 36;  // block-minimum row stride bound (s + 1 rounded up to 4): tile skipping for s <= 35
 // Resident interval costs: per tile, C[64][PSTR] then Phi[64][PSTR] (the shared-memory layout).
 constexpr int kCostHalfFloats = BJ * PSTR;
 constexpr uint32_t kCostHalfBytes = (uint32_t)(kCostHalfFloats * sizeof(float));  // 17408, a multiple of 16
@@ -143,7 +144,8 @@ struct FastArgs {
     int *wide_cnt;         // [s+1]
     float *mdp;            // [nJ][G][mdp_stride]: min over the block's 64 columns of dp32(g, i, .)
     int mdp_stride;        // s + 1 rounded up to a multiple of 4 (16-byte rows)
-    int prune;             // skip tiles by the lower bound (resident costs, two layer groups)
+    int prune;             // skip tiles by the lower bound (resident or streamed costs)
+    int stage_tiles;       // with prune: tiles per staged batch (32, or 16 off the parked diagonal)
     const float *seed;     // with prune: fp32 dp rows [nJ][s+1][64] of an earlier pass at a multiplier >= every
                            // multiplier of this one (upper bounds of this pass's fp32 minima), or null
     uint32_t spin_limit;   // flag waits give up after this many spins (kSpinLimit; lower in the test hook)
@@ -449,7 +451,9 @@ struct __align__(16) Smem {
     unsigned long long smbar[2];          // resident costs: completion of stage buffer sb
     float tau[kMaxS + 1];                 // FastParams::tau and lam32, read on every tile
     float lam32[kMaxG];
-    __align__(16) float mdp[2][kMaxG][20];  // staged dp32 block minima (tile skipping, s <= 19)
+    // staged dp32 block minima of a tile's column block (tile skipping): the split's
+    // multipliers' rows of a.mdp_stride floats each, flat (up to kMaxG x 20 floats)
+    __align__(16) float mdp[2][kMaxG][20];
     // followed by dp32 slices [2][Gc * (s-2)][BK] (dynamic)
 };
 
@@ -687,12 +691,13 @@ constexpr uint32_t kNoRun = 0xFFFFFFFFu;
 // with a candidate within m (1 + tau) from any starting bb >= m (a reset drops only
 // tiles whose candidates all lie above the band).  Only the skip tests see the seed:
 // more tiles are skipped, the tables are unchanged.
-__device__ __forceinline__ void cons_seed(const FastArgs &a, ConsState &cs, int J, const ConsId &id) {
+template <int LP>
+__device__ __forceinline__ void cons_seed(const FastArgs &a, ConsStateT<LP> &cs, int J, const ConsId &id) {
     const float *sr = a.seed + (size_t)J * (size_t)(a.s + 1) * BJ;
 #pragma unroll
-    for (int l = 0; l < LPT; l++) {
+    for (int l = 0; l < LP; l++) {
         // rows past the last layer repeat the last one (cons_offdiag): so does their seed
-        const int i = 3 + min(id.lg * LPT + l, a.s - 3);
+        const int i = 3 + min(id.lg * LP + l, a.s - 3);
 #pragma unroll
         for (int q = 0; q < JPT; q++) {
             const int jl = id.jq + NJQ * q;
@@ -814,6 +819,18 @@ __device__ __forceinline__ void cons_diag(const FastArgs &a, Smem &S, int b, int
     const uint32_t K = (uint32_t)J, KK = (K << 16) | K;
     int cur = 0;
     for (int li = 0; li < L; li++) {
+        if (LP != LPT && a.prune) {
+            // block minimum of the layer below (row 2 + li) for later blocks' skip tests, by the
+            // warp of that index (values >= +0: integer min on the bits); with LPT layers per
+            // thread, skipping runs on the paired diagonal only, which writes its own minima
+            const int w = ct >> 5, wl = ct & 31;
+            const int gw = split * a.Gc + w;
+            if (w < a.Gc && gw < a.G) {
+                const int v = min(__float_as_int(S.diag[cur][w][wl]), __float_as_int(S.diag[cur][w][wl + 32]));
+                const int mn = __reduce_min_sync(0xffffffffu, v);
+                if (wl == 0) a.mdp[((size_t)J * a.G + gw) * a.mdp_stride + 2 + li] = __int_as_float(mn);
+            }
+        }
         const int i = 3 + li;
         const int olg = li / LP, l = li - olg * LP;
         const bool owner = own && id.lg == olg;
@@ -859,7 +876,13 @@ __device__ __forceinline__ void cons_diag(const FastArgs &a, Smem &S, int b, int
                     S.diag[cur ^ 1][id.gl][jl] = bb;
                     if (j < a.p) {
                         a.dp32[d32(a, g, i, j)] = bb;
-                        a.band[oidx(a, g, i, j)] = band_pack(cs.w1[lx][q], cs.w2[lx][q]);
+                        // kNoRun: seeded, run 2 only (seeds come with tile skipping, which with LPT
+                        // layers per thread runs on the paired diagonal, not here)
+                        const uint32_t w1 = cs.w1[lx][q], w2 = cs.w2[lx][q];
+                        if constexpr (LP != LPT)
+                            a.band[oidx(a, g, i, j)] = w1 == kNoRun ? band_pack(w2, 0u) : band_pack(w1, w2);
+                        else
+                            a.band[oidx(a, g, i, j)] = band_pack(w1, w2);
                     }
                 }
             }
@@ -1353,21 +1376,23 @@ __device__ __forceinline__ void res_wait(const FastArgs &a, int split, int K, in
     fence_proxy_async_global();
 }
 
-// Tile skipping in batches (resident costs, two layer groups).  A batch is up to
-// kStageTiles consecutive off-diagonal tiles of block J; warp 0 stages their column
+// Tile skipping in batches (resident or streamed costs).  A batch is up to a.stage_tiles
+// (at most 32) consecutive off-diagonal tiles of block J; warp 0 stages their column
 // summaries (a.tsum) and the block minima of their column blocks (a.mdp, all G
 // multipliers) into a stage buffer with two bulk copies, one batch ahead.  The stage
-// buffers live where the diagonal parks its band state (free until the diagonal).
-constexpr int kStageTiles = 32;
-__host__ __device__ __forceinline__ size_t stage_floats(int G, int mdp_stride) {
-    return (size_t)kStageTiles * BJ * 2 + (size_t)kStageTiles * G * mdp_stride;
+// buffers follow the dp32 rows in shared memory: where the paired diagonal parks its
+// band state (free until the diagonal; 32 tiles per batch), else in space of their own
+// (16 tiles per batch, for the larger rows of more layers).
+__host__ __device__ __forceinline__ size_t stage_floats(int G, int mdp_stride, int ntiles) {
+    return (size_t)ntiles * BJ * 2 + (size_t)ntiles * G * mdp_stride;
 }
-// The batch after the one ending at K1: 1, 1, 2, 4, ... kStageTiles tiles (the band
-// limits are +inf before the first tile and tighten fast).
-__device__ __forceinline__ int batch_end(int K1, int J) { return min(J, K1 + min(kStageTiles, max(1, K1))); }
+// The batch after the one ending at K1: 1, 1, 2, 4, ... nt tiles (the band limits are
+// +inf before the first tile and tighten fast).
+__device__ __forceinline__ int batch_end(int K1, int J, int nt) { return min(J, K1 + min(nt, max(1, K1))); }
 
 // Warp 0: stage tiles K0 <= K < K1 of block J into stage buffer sb.  Minima of blocks
 // past `frontier` may be incomplete in the copy; need_mask does not read them.
+template <int NT>
 __device__ __forceinline__ void res_stage(const FastArgs &a, Smem &S, float *stg, int sb, int K0, int K1, int J,
                                           int frontier, uint64_t policy, int lane) {
     if (lane == 0) {
@@ -1376,7 +1401,7 @@ __device__ __forceinline__ void res_stage(const FastArgs &a, Smem &S, float *stg
         S.sfront[sb] = frontier;  // ordered before the readers' wait by the arrive (release)
         mbar_expect_tx(&S.smbar[sb], tb + mb);
         bulk_g2s(stg, a.tsum + (cost_tile_idx(0, J) - a.tile_base + (size_t)K0) * BJ, tb, &S.smbar[sb], policy);
-        bulk_g2s_nohint(stg + (size_t)kStageTiles * BJ * 2, a.mdp + (size_t)K0 * a.G * a.mdp_stride, mb, &S.smbar[sb]);
+        bulk_g2s_nohint(stg + (size_t)NT * BJ * 2, a.mdp + (size_t)K0 * a.G * a.mdp_stride, mb, &S.smbar[sb]);
     }
 }
 
@@ -1387,21 +1412,22 @@ __device__ __forceinline__ void res_stage(const FastArgs &a, Smem &S, float *stg
 // fold, and rounding is monotone, so a tile this test rules out is ruled out by
 // cons_offdiag too: walking only the tiles some warp needs changes no result.  Blocks
 // past `fr` had no published minima when staged and are always needed.
+template <int NT, int LP>
 __device__ __forceinline__ uint32_t need_mask(const FastArgs &a, const Smem &S, const float *stg, int K0, int K1, int fr,
-                                              int g, const ConsId &id, const ConsState &cs) {
+                                              int g, const ConsId &id, const ConsStateT<LP> &cs) {
     const int L = a.s - 2;
     const float lam = S.lam32[g];
-    int rowl[LPT];
-    float lim[LPT][JPT];
+    int rowl[LP];
+    float lim[LP][JPT];
 #pragma unroll
-    for (int l = 0; l < LPT; l++) {
-        rowl[l] = min(id.lg * LPT + l, L - 1);
+    for (int l = 0; l < LP; l++) {
+        rowl[l] = min(id.lg * LP + l, L - 1);
         const float tau = S.tau[3 + rowl[l]];
 #pragma unroll
         for (int q = 0; q < JPT; q++) lim[l][q] = __fadd_rn(cs.best[l][q], __fmul_rn(cs.best[l][q], tau));
     }
     const float2 *ts = reinterpret_cast<const float2 *>(stg) + id.jq;
-    const float *md = stg + (size_t)kStageTiles * BJ * 2 + (size_t)g * a.mdp_stride + 2;
+    const float *md = stg + (size_t)NT * BJ * 2 + (size_t)g * a.mdp_stride + 2;
     const int mstride = a.G * a.mdp_stride;
     uint32_t mask = 0;
 #pragma unroll 2
@@ -1417,7 +1443,7 @@ __device__ __forceinline__ uint32_t need_mask(const FastArgs &a, const Smem &S, 
             }
             need = false;
 #pragma unroll
-            for (int l = 0; l < LPT; l++) {
+            for (int l = 0; l < LP; l++) {
                 const float m = md[r * mstride + rowl[l]];
 #pragma unroll
                 for (int q = 0; q < JPT; q++) need |= __fadd_rn(m, lbq[q]) <= lim[l][q];
@@ -1461,7 +1487,8 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
     uint32_t mph[2] = {0u, 0u};  // completed phases of mbar[0], mbar[1] (one per fill; two for a split last tile)
     uint32_t ns = 0;  // batch sequence number (tile skipping): stage buffer ns & 1, its fill ns >> 1
     float *stage = sDP + (size_t)2 * rowsDP * BK;  // the park area, free off the diagonal
-    const size_t sfl = stage_floats(a.G, a.mdp_stride);
+    constexpr int NT = LP == LPT ? 32 : 16;  // tiles per staged batch (a.stage_tiles, set to match)
+    const size_t sfl = stage_floats(a.G, a.mdp_stride, NT);
     unsigned long long n_run = 0, n_skip = 0;  // lane 0 of each warp: its (warp, tile) units
     int frontier = -1, fsplit = -1;            // warp 0 (res_probe)
     for (;;) {
@@ -1474,19 +1501,17 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
         const bool own = id.active && g < a.G;
         if (split != fsplit) { frontier = -1; fsplit = split; }
         cons_reset(cs);
-        if constexpr (LP == LPT) {  // seeds, tile skipping and the split publish: LPT only
-            if (a.seed && own) cons_seed(a, cs, J, id);
-        }
+        if (a.seed && own) cons_seed(a, cs, J, id);
         int issued = -1;  // the tile whose copies are in flight into buffer n & 1 (J: the diagonal), or -1
         const int ngv = min(a.G - split * a.Gc, a.Gc);  // real multipliers of the split
         // the tiles walked here: K < Kend (with a split publish the last one, J - 1, is the chain's)
         const int Kend = a.split_pub ? max(J - 1, 0) : J;
         if (a.prune && Kend > 0 && ct < 32) {  // stage the first batch
             if (frontier < 0) res_probe(a, split, 0, J, frontier, lane);
-            res_stage(a, S, stage + (ns & 1) * sfl, ns & 1, 0, batch_end(0, Kend), J, frontier, policy, lane);
+            res_stage<NT>(a, S, stage + (ns & 1) * sfl, ns & 1, 0, batch_end(0, Kend, NT), J, frontier, policy, lane);
         }
         for (int K0 = 0; K0 < Kend;) {
-            const int K1 = a.prune ? batch_end(K0, Kend) : min(Kend, K0 + 32);
+            const int K1 = a.prune ? batch_end(K0, Kend, NT) : min(Kend, K0 + 32);
             uint32_t wm = 0xffffffffu;  // the warp's tiles of the batch
             uint32_t U = 0xffffffffu;   // the tiles some warp needs
             int frb = -1;               // tiles <= frb: every warp issues its own rows (res_issue_rows)
@@ -1495,16 +1520,16 @@ __global__ void __launch_bounds__(MAXCONS, 1) k_wavefront_res(FastArgs a) {
                 mbar_wait_bounded(&S.smbar[sb], (ns >> 1) & 1u, a.st, a.abort_flag);
                 frb = S.sfront[sb];
                 if (lane == 0) fence_proxy_async_global();  // blocks <= frb, published, before this warp's copies
-                if constexpr (LP == LPT) wm = own ? need_mask(a, S, stage + sb * sfl, K0, K1, frb, g, id, cs) : 0u;
+                wm = own ? need_mask<NT>(a, S, stage + sb * sfl, K0, K1, frb, g, id, cs) : 0u;
                 if (lane == 0) S.needw[sb][ct >> 5] = wm;
                 __syncthreads();  // needw; every read of stage buffer sb is done
                 U = 0;
                 for (int w = 0; w < (int)(blockDim.x >> 5); w++) U |= S.needw[sb][w];
                 ns++;
                 if (K1 < Kend && ct < 32) {  // stage the next batch while this one is walked
-                    const int K2 = batch_end(K1, Kend);
+                    const int K2 = batch_end(K1, Kend, NT);
                     if (K2 - 1 > frontier) res_probe(a, split, frontier + 1, J, frontier, lane);
-                    res_stage(a, S, stage + (ns & 1) * sfl, ns & 1, K1, K2, J, frontier, policy, lane);
+                    res_stage<NT>(a, S, stage + (ns & 1) * sfl, ns & 1, K1, K2, J, frontier, policy, lane);
                 }
             }
             U &= (K1 - K0 == 32) ? 0xffffffffu : ((1u << (K1 - K0)) - 1u);
@@ -2286,7 +2311,14 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     // two-part publishing of each block (the chain's last tile in two layer groups)
     a.split_pub = (costs && lp == LPT && a.lgc == 2 && !split_off) ? 1 : 0;
     a.hold0 = test_stall ? 1 : 0;
-    a.prune = (costs && lp == LPT && a.lgc == 2 && a.mdp_stride <= 20) ? 1 : 0;
+    // Tile skipping needs every warp to hold whole multipliers (its batch test is a warp
+    // vote), so an even number of layer groups (16-thread groups, 32-lane warps), and a
+    // diagonal that writes the blocks' minima: the paired one (LPT layers per thread, two
+    // groups) or the generic one with 8 layers per thread.
+    a.prune = (costs && (lp == LPT ? a.lgc == 2 : a.lgc % 2 == 0) && a.mdp_stride <= kMdpMax &&
+               a.Gc * a.mdp_stride <= kMaxG * 20) ? 1 : 0;
+    const bool parked = costs && lp == LPT && a.lgc == 2;  // the paired diagonal and its parked state
+    a.stage_tiles = lp == LPT ? 32 : 16;  // k_wavefront_res<LP>'s batch size
     a.seed = (seeded && a.prune && s == Lw.s) ? seed_rows(ws, Lw) : nullptr;
     a.costs = costs;
     a.tile_base = 0;
@@ -2327,9 +2359,11 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
         ECASQ_LAUNCH_CHECK();
     }
     size_t smem = smem_bytes(a.Gc, s);
-    if (costs && lp == LPT && a.lgc == 2)  // parked band state; off the diagonal, the two stage buffers
-        smem += std::max((size_t)3 * LPT * JPT * a.ncons * sizeof(uint32_t),
-                         a.prune ? 2 * stage_floats(G, a.mdp_stride) * sizeof(float) : (size_t)0);
+    const size_t stage_bytes = a.prune ? 2 * stage_floats(G, a.mdp_stride, a.stage_tiles) * sizeof(float) : 0;
+    if (parked)  // parked band state; off the diagonal, the two stage buffers
+        smem += std::max((size_t)3 * LPT * JPT * a.ncons * sizeof(uint32_t), stage_bytes);
+    else
+        smem += stage_bytes;
     auto wave = costs ? (lp == 8 ? k_wavefront_res<8> : k_wavefront_res<LPT>)
                       : (lp == 8 ? k_wavefront<8> : k_wavefront<LPT>);
     ECASQ_CUDA_TRY(cudaFuncSetAttribute(wave, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));

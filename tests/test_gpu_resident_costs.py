@@ -269,7 +269,9 @@ def test_two_part_publish_bit_identical_to_one_part(E, name, s):
                                            ("lognormal16k", 16, 1.0, "RESIDENT_COSTS"),
                                            ("studentt20001", 12, 2.5, "RESIDENT_COSTS"),
                                            ("normal8192", 10, 2.0, "RESIDENT_COSTS"),
-                                           ("studentt16k", 16, 2.5, "STREAMED_COSTS")])
+                                           ("studentt16k", 16, 2.5, "STREAMED_COSTS"),
+                                           ("mixture12k", 32, 4.0, "RESIDENT_COSTS"),   # 8 layers per thread
+                                           ("ragged5000", 18, 2.5, "STREAMED_COSTS")])
 def test_seeded_search_bit_identical_to_unseeded(E, name, s, b, mode):
     """Later passes of the search start their tile skipping from the fp32 minima of the
     bracket's evaluated upper end (an upper bound of theirs: candidates are non-decreasing
@@ -278,7 +280,9 @@ def test_seeded_search_bit_identical_to_unseeded(E, name, s, b, mode):
     x = {"studentt16k": lambda: workloads.student_t(16384, 0),
          "lognormal16k": lambda: workloads.signed_lognormal(16384, 0),
          "studentt20001": lambda: workloads.student_t(20001, 5, scale=1.0),
-         "normal8192": lambda: workloads.normal(8192, 7)}[name]()
+         "normal8192": lambda: workloads.normal(8192, 7),
+         "mixture12k": lambda: workloads.mixture(12288, 2),
+         "ragged5000": lambda: workloads.student_t(5000, 6, scale=1.0)}[name]()
     cost = getattr(E, mode)  # streamed costs: bands of column blocks, tile skipping and seeds as resident
     out = {}
     for extra in (0, E.UNSEEDED_SEARCH):
@@ -299,5 +303,6 @@ def test_seeded_search_bit_identical_to_unseeded(E, name, s, b, mode):
         np.testing.assert_array_equal(dps, dpu)
         np.testing.assert_array_equal(bps, bpu)
     assert sts["tiles_run"] <= stu["tiles_run"]
+    assert stu["tiles_skipped"] > 0  # tile skipping runs at every s here (even layer groups)
     if name == "studentt16k":  # five seeded passes at multipliers where most tiles are skipped
         assert sts["tiles_run"] < 0.95 * stu["tiles_run"]
