@@ -1715,7 +1715,7 @@ __device__ __forceinline__ float cand32(float dprev, float lam, float C, float P
 }
 
 // Visit the candidates k of tile K for output (g, i, j) in the wavefront's fp32
-// arithmetic (k descending) and call f(k) for every k with value <= thr.
+// arithmetic (k descending) and call f(k, value) for every k with value <= thr.
 template <typename F>
 __device__ void visit_tile(const FastArgs &a, int g, int i, int64_t j, int64_t K, float thr, F &&f) {
     int64_t J = j / BJ, j0 = J * BJ, k0 = K * BK;
@@ -1726,8 +1726,10 @@ __device__ void visit_tile(const FastArgs &a, int g, int i, int64_t j, int64_t K
         const float *cr = a.costs + (cost_tile_idx(K, J) - a.tile_base) * kCostTileFloats + (size_t)(j - j0) * PSTR;
         const float *pr = cr + kCostHalfFloats;
         int64_t khi = (K == J) ? j - 1 : k0 + BK - 1;
-        for (int64_t k = khi; k >= k0; k--)
-            if (cand32(prev[k], lam, cr[k - k0], pr[k - k0]) <= thr) f(k);
+        for (int64_t k = khi; k >= k0; k--) {
+            const float v = cand32(prev[k], lam, cr[k - k0], pr[k - k0]);
+            if (v <= thr) f(k, v);
+        }
         return;
     }
     float vj = a.v[j];
@@ -1742,12 +1744,14 @@ __device__ void visit_tile(const FastArgs &a, int g, int i, int64_t j, int64_t K
         khi = k0 + BK - 1;
         rec_anchor(a, khi, j, r);  // any evaluation within the certified bound will do
         rec_emit(r, vj, a.v[khi], d_f, a.invd, c, ph);
-        if (cand32(prev[khi], lam, c, ph) <= thr) f(khi);
+        const float v = cand32(prev[khi], lam, c, ph);
+        if (v <= thr) f(khi, v);
     }
     for (int64_t k = khi - 1; k >= k0; k--) {
         rec_step(r, vj, a.v[k + 1], a.wf[k + 1], __fsub_rn(a.v[k + 1], a.v[k]));
         rec_emit(r, vj, a.v[k], d_f, a.invd, c, ph);
-        if (cand32(prev[k], lam, c, ph) <= thr) f(k);
+        const float v = cand32(prev[k], lam, c, ph);
+        if (v <= thr) f(k, v);
     }
 }
 
@@ -1772,7 +1776,8 @@ __device__ __forceinline__ float band_threshold(const FastArgs &a, int i, float 
 
 // The candidates of output (g, i, j)'s band, by the 32 lanes of a warp together, with
 // visit_tile's verdicts (fp32 value <= thr): f(in, k) is called by every lane at once
-// (a warp-uniform call; `in` is false for a lane without a candidate in that step).
+// (a warp-uniform call; `in` is false for a lane without a candidate in that step;
+// `v` is the candidate's fp32 value, +inf for a lane without one).
 // With resident costs the lanes split every tile's k (the table gives any pair
 // directly); otherwise they take whole tiles and walk them in step along visit_tile's
 // recurrence (k descending from the anchor at the tile's top pair, or from the empty
@@ -1796,7 +1801,8 @@ __device__ __forceinline__ void warp_visit_band(const FastArgs &a, int g, int i,
             const int64_t khi = (K == J) ? j - 1 : k0 + BK - 1;
             for (int64_t kb = k0; kb <= khi; kb += 32) {  // warp-uniform
                 const int64_t k = kb + lane;
-                f(k <= khi && cand32(prev32[k], lam32, cr[k - k0], pr[k - k0]) <= thr, k);
+                const float v = k <= khi ? cand32(prev32[k], lam32, cr[k - k0], pr[k - k0]) : CUDART_INF_F;
+                f(v <= thr, k, v);
             }
         }
         return;
@@ -1822,14 +1828,14 @@ __device__ __forceinline__ void warp_visit_band(const FastArgs &a, int g, int i,
         }
         for (int it = 0; it < BK; it++) {  // warp-uniform
             const int64_t k = kfirst - it;
-            bool in = false;
+            float v = CUDART_INF_F;
             if (it < nk) {
                 if (it > 0 || K == J) rec_step(r, vj, a.v[k + 1], a.wf[k + 1], __fsub_rn(a.v[k + 1], a.v[k]));
                 float c, ph;
                 rec_emit(r, vj, a.v[k], d_f, a.invd, c, ph);
-                in = cand32(prev32[k], lam32, c, ph) <= thr;
+                v = cand32(prev32[k], lam32, c, ph);
             }
-            f(in, k);
+            f(it < nk && v <= thr, k, v);
         }
     }
 }
@@ -1899,11 +1905,15 @@ __global__ void k_need_layer(FastArgs a, int i) {
                         int32_t *mem = a.members + o * NMEM;
                         uint8_t *below = a.need + oidx(a, g, i - 1, 0);
                         const bool mark = i - 1 >= 3;
-                        visit_band(a, g, i, j, w, band_threshold(a, i, m32), [&](int64_t k) {
+                        float vmin = CUDART_INF_F;
+                        int32_t kmin = -1;
+                        visit_band(a, g, i, j, w, band_threshold(a, i, m32), [&](int64_t k, float v) {
                             if (cnt < NMEM) mem[cnt] = (int32_t)k;
                             cnt++;
                             if (mark) below[k] = 1;
+                            if (v < vmin || (v == vmin && (int32_t)k < kmin)) { vmin = v; kmin = (int32_t)k; }
                         });
+                        if (cnt > NMEM) mem[0] = kmin;  // a big output keeps its fp32 argmin (k_exact_big)
                         a.mcnt[o] = cnt;
                         nmem += cnt;
                         nbig += cnt > NMEM;
@@ -1942,16 +1952,27 @@ __global__ void __launch_bounds__(128) k_need_wide(FastArgs a, int i) {
         int32_t *mem = a.members + o * NMEM;
         uint8_t *below = a.need + oidx(a, g, i - 1, 0);
         int cnt = 0;  // warp-uniform
-        warp_visit_band(a, g, i, j, w, band_threshold(a, i, a.dp32[d32(a, g, i, j)]), [&](bool in, int64_t k) {
+        float vmin = CUDART_INF_F;  // per lane: its least member value, lowest k on ties
+        int32_t kmin = INT32_MAX;
+        warp_visit_band(a, g, i, j, w, band_threshold(a, i, a.dp32[d32(a, g, i, j)]), [&](bool in, int64_t k, float v) {
             const unsigned mask = __ballot_sync(0xffffffffu, in);
             if (in) {
                 const int pos = cnt + __popc(mask & lt);
                 if (pos < NMEM) mem[pos] = (int32_t)k;
                 if (mark) below[k] = 1;
+                if (v < vmin || (v == vmin && (int32_t)k < kmin)) { vmin = v; kmin = (int32_t)k; }
             }
             cnt += __popc(mask);
         });
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+            const float v2 = __shfl_xor_sync(0xffffffffu, vmin, off);
+            const int32_t k2 = __shfl_xor_sync(0xffffffffu, kmin, off);
+            if (v2 < vmin || (v2 == vmin && k2 < kmin)) { vmin = v2; kmin = k2; }
+        }
+        __syncwarp();  // every lane's member stores are done before lane 0 overwrites slot 0
         if (lane == 0) {
+            if (cnt > NMEM) mem[0] = kmin;  // a big output keeps its fp32 argmin (k_exact_big)
             a.mcnt[o] = cnt;
             nmem += cnt;
             nbig += cnt > NMEM;
@@ -2122,7 +2143,23 @@ __global__ void __launch_bounds__(128) k_exact_big(Prefix P, FastArgs a, int i, 
         double best = CUDART_INF;
         int32_t arg = INT32_MAX;
         int qn = 0;  // warp-uniform queue length
-        warp_visit_band(a, g, i, j, w, thr, [&](bool in, int64_t k) {
+        // The closure stage kept the band's fp32 argmin kb in the member slot 0; its binary64
+        // value b0 bounds the binary64 minimum from above.  Every fp32 candidate value is within
+        // eps_i (relative) of the candidate's exact (real) value V, so V >= val32 / (1 + eps_i);
+        // a binary64 candidate is within far less than 2^-40 of V (a few correctly rounded
+        // operations per layer on non-negative terms, s <= 256 layers).  So a member with
+        // val32 > b0 (1 + eps_i + 2^-30) has V > b0 (1 + 2^-31) and a binary64 value above b0:
+        // it can neither be the minimum nor tie it, and is not re-scored.
+        const int32_t kb = a.members[o * NMEM];
+        double b0 = CUDART_INF;
+        if (lane == 0 && kb >= 0) b0 = exact_value(P, prev, kb, j, lam);
+        b0 = __shfl_sync(0xffffffffu, b0, 0);
+        if (lane == 0 && kb >= 0) { best = b0; arg = kb; nres++; }
+        const float thr2 = b0 < CUDART_INF
+                               ? __double2float_ru(__dmul_ru(b0, __dadd_ru(1.0 + 0x1p-30, (double)a.prm->eps[i])))
+                               : CUDART_INF_F;
+        warp_visit_band(a, g, i, j, w, thr, [&](bool in0, int64_t k, float v) {
+            const bool in = in0 && v <= thr2 && (int32_t)k != kb;
             const unsigned mask = __ballot_sync(0xffffffffu, in);
             if (!mask) return;
             const int cnt = __popc(mask), pos = qn + __popc(mask & lt);
