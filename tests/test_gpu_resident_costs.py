@@ -62,6 +62,8 @@ def test_resident_costs_bit_identical_to_fused(E, name, s, flags_name):
         assert st["timeout"] == 0 and st["bound_viol"] == 0
         if name == "lognormal16k":
             assert st["big_bands"] > 0  # both branches of the many-member exact stage run
+            # the exact stage's bound (the band's fp32 argmin in binary64) spares some members
+            assert st["rescored"] < st["members"]
     assert mf == mr
     np.testing.assert_array_equal(Qf.cpu().numpy(), Qr.cpu().numpy())
     np.testing.assert_array_equal(metf, metr)
