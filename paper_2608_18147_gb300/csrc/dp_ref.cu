@@ -124,7 +124,10 @@ __global__ void k_traceback_eval(Prefix P, int G, int s, int exact_s, const doub
     __syncwarp();
     int m = sm_m;
     for (int r = threadIdx.x; r < m; r += 32) qidx[g * s + r] = a[r];
-    if (m > 0) eval_codebook_warp(P, a, m, &metrics[4 * g + 1], scratch);
+    if (m > 0 && m <= 32)
+        eval_codebook_lanes(P, a, m, &metrics[4 * g + 1]);  // the same values, one interval per lane
+    else if (m > 0)
+        eval_codebook_warp(P, a, m, &metrics[4 * g + 1], scratch);
 }
 
 // Metrics of a caller-given codebook (unique indices on the device); nothing when
@@ -135,7 +138,10 @@ __global__ void k_eval_codebook(Prefix P, const int32_t *a_in, int m, double *ou
     if (gate && *gate == 0) return;
     for (int r = threadIdx.x; r < m; r += 32) a[r] = a_in[r];
     __syncwarp();
-    eval_codebook_warp(P, a, m, out3, scratch);
+    if (m <= 32)
+        eval_codebook_lanes(P, a, m, out3);  // the same values, one interval per lane
+    else
+        eval_codebook_warp(P, a, m, out3, scratch);
 }
 
 // Q[r] = v[a[r]] for every multiplier row g.
