@@ -1775,13 +1775,13 @@ __device__ __forceinline__ float band_threshold(const FastArgs &a, int i, float 
 }
 
 // The candidates of output (g, i, j)'s band, by the 32 lanes of a warp together, with
-// visit_tile's verdicts (fp32 value <= thr): f(in, k) is called by every lane at once
+// visit_tile's decisions (fp32 value <= thr): f(in, k, v) is called by every lane at once
 // (a warp-uniform call; `in` is false for a lane without a candidate in that step;
 // `v` is the candidate's fp32 value, +inf for a lane without one).
 // With resident costs the lanes split every tile's k (the table gives any pair
 // directly); otherwise they take whole tiles and walk them in step along visit_tile's
 // recurrence (k descending from the anchor at the tile's top pair, or from the empty
-// interval (j, j] on the diagonal tile), so the values, and the verdicts, are visit_tile's.
+// interval (j, j] on the diagonal tile), so the values, and the decisions, are visit_tile's.
 template <typename F>
 __device__ __forceinline__ void warp_visit_band(const FastArgs &a, int g, int i, int64_t j, uint64_t w, float thr,
                                                 F &&f) {
@@ -2114,7 +2114,7 @@ __global__ void __launch_bounds__(128) k_exact_small(Prefix P, FastArgs a, int i
 }
 
 // Layer i, outputs with more members: one warp each (fp32 re-evaluation within the
-// band by warp_visit_band, whose verdicts are the closure stage's; exact re-scoring of
+// band by warp_visit_band, whose decisions are the closure stage's; exact re-scoring of
 // the members met), then the lanes' results meet (value, then lowest k).  The members
 // met wait in the warp's queue, and each time it holds 32 every lane re-scores one of
 // them in binary64, so the binary64 sequence runs with all lanes busy (the result,
