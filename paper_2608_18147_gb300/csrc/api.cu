@@ -40,7 +40,7 @@ int launch_refine_colour(const Prefix &P, const int32_t *a, int m, int colour, d
                          int32_t *moved, void *part_buf, int32_t *ctx, cudaStream_t st, int *nblocks_out);
 size_t refine_scratch_bytes(int64_t d);
 int launch_refine_commit(int32_t *a, const int32_t *a_new, const int32_t *moved, const double *ev, int m, bool guard,
-                         double budget, cudaStream_t st);
+                         double budget, int32_t *ctx, cudaStream_t st);
 int launch_quantize(const float *x, int64_t d, const float *Q, int m, uint64_t seed, uint8_t *idx, uint32_t *counts,
                     DevStatus *st, int num_sms, cudaStream_t stream);
 int launch_quantize_timeshare(const float *x, int64_t d, const float *Qm, int mm, const float *Qp, int mp,
@@ -390,7 +390,7 @@ static int refine_device(void *ws, const Layout &L, const Prefix &P, std::vector
             // only a step that moved a value is evaluated; the step is kept or dropped on the device
             rc = launch_eval_codebook(P, an, m, evd, st, moved);
             if (rc != ECASQ_OK) return rc;
-            rc = launch_refine_commit(a, an, moved, evd, m, guard, budget, st);
+            rc = launch_refine_commit(a, an, moved, evd, m, guard, budget, ctx, st);
             if (rc != ECASQ_OK) return rc;
         }
         rc = eval_device(ws, L, P, a, m, st, ev);

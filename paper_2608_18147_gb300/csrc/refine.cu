@@ -154,17 +154,31 @@ __global__ void k_refine_pick(const int32_t *a, int m, int colour, const RefPart
 // or (with the guard) its H(Xhat), ev[2] from the gated evaluation, exceeds the budget
 // (Sec. 6).  On the device, so that a refinement round needs no host round trip until
 // its stop test.
+// A value that moved went to the lowest-index minimiser of its local objective, which does
+// not depend on the value itself, only on its four neighbours (other colours: they did not
+// move in this step); a scan in its new context would keep it there, so a kept step gives
+// it the record such a scan writes, and the next round does not scan it again unless a
+// neighbour moves.
 __global__ void k_refine_commit(int32_t *a, const int32_t *a_new, const int32_t *moved, const double *ev, int m,
-                                int guard, double budget) {
+                                int guard, double budget, int32_t *ctx) {
     if (!*moved) return;
     if (guard && ev[2] > budget) return;
+    for (int l = threadIdx.x; l < m; l += blockDim.x) {
+        if (a_new[l] == a[l]) continue;
+        int32_t c[5];
+        context_of(a_new, m, l, c);
+        int32_t *r = ctx + kCtx * l;
+        for (int q = 0; q < 5; q++) r[q] = c[q];
+        r[5] = 1;
+    }
+    __syncwarp();  // every comparison with the old codebook is done
     for (int t = threadIdx.x; t < m; t += blockDim.x) a[t] = a_new[t];
 }
 
 int launch_refine_commit(int32_t *a, const int32_t *a_new, const int32_t *moved, const double *ev, int m, bool guard,
-                         double budget, cudaStream_t st) {
+                         double budget, int32_t *ctx, cudaStream_t st) {
     note_launch();
-    k_refine_commit<<<1, 32, 0, st>>>(a, a_new, moved, ev, m, guard ? 1 : 0, budget);
+    k_refine_commit<<<1, 32, 0, st>>>(a, a_new, moved, ev, m, guard ? 1 : 0, budget, ctx);
     ECASQ_LAUNCH_CHECK();
     return ECASQ_OK;
 }
