@@ -65,11 +65,16 @@ typedef struct CUstream_st *ecasq_stream_t; /* same type as cudaStream_t */
 #define ECASQ_ONE_PART_PUBLISH 128u /* fast DP with resident or streamed costs and s <= 16: publish each column block
                                      of the wavefront once, after all its layers, instead of in two parts (rows 2..8
                                      after layer 8, then the rest); same results, for comparison */
-#define ECASQ_UNSEEDED_SEARCH 256u /* fast DP with resident or streamed costs and tile skipping (s <= 16): in the
+#define ECASQ_UNSEEDED_SEARCH 256u /* fast DP with resident or streamed costs and tile skipping (10 <= s <= 18, 27 <= s <= 34): in the
                                      multiplier search, start every pass's tile skipping from scratch instead of from
                                      the fp32 minima of the bracket's evaluated upper end (an upper bound of every
                                      later pass's minima, Sec. 5's candidates being non-decreasing in lambda); same
                                      results, for comparison */
+#define ECASQ_TEST_SELF_SEED (1u << 29) /* test hook for the seeded tile skipping: with a fixed multiplier and resident
+                                     or streamed costs, the pass runs twice, the second time seeded with the first
+                                     one's fp32 minima (the seed then equals every output's minimum, the tightest
+                                     start the seeding allows); results must equal those without the flag.
+                                     ecasq_result_t.passes counts both.  Not for production use. */
 #define ECASQ_TEST_STALL (1u << 30) /* test hook for the bounded device waits: column block 0 of the fast DP's
                                      wavefront is never published and the flag waits give up after 2^14 spins, so
                                      the call must return ECASQ_ETIMEOUT (nothing else) and leave the workspace

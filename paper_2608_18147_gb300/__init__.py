@@ -8,7 +8,7 @@ There is no CPU fallback: without libecasq.so and a GPU every call raises.
 """
 from . import workloads
 from .native import (DP_REFERENCE, EXACT_S, EXACT_TABLES, NO_REFINE_GUARD, ONE_PART_PUBLISH, RESIDENT_COSTS,
-                     STREAMED_COSTS, TEST_STALL, UNSEEDED_SEARCH,
+                     STREAMED_COSTS, TEST_SELF_SEED, TEST_STALL, UNSEEDED_SEARCH,
                      TIME_KERNELS,
                      EcasqError,
                      ecasq_dp_linear, ecasq_dp_pass, ecasq_dp_tables, ecasq_evaluate, ecasq_kernel_launches, ecasq_opt_dp, ecasq_prepare,
@@ -21,4 +21,4 @@ __all__ = ["workloads", "ecasq_solve", "ecasq_solve_grid", "ecasq_solve_timeshar
            "ecasq_quantize_noalloc", "ecasq_quantize_timeshare", "ecasq_prepare", "ecasq_workspace_size",
            "ecasq_workspace_size_flags", "ecasq_kernel_launches", "workspace", "uniform_grid", "lib", "EcasqError",
            "EXACT_S", "EXACT_TABLES", "RESIDENT_COSTS", "NO_REFINE_GUARD", "DP_REFERENCE", "TIME_KERNELS", "TEST_STALL", "STREAMED_COSTS", "ONE_PART_PUBLISH",
-           "UNSEEDED_SEARCH"]
+           "UNSEEDED_SEARCH", "TEST_SELF_SEED"]

@@ -653,9 +653,17 @@ static int solve_prepared(void *ws, const Layout &L, const Prefix &P, int64_t d,
     int status = ECASQ_OK;
     const Eval *sel = nullptr;
     if (prm->lambda >= 0.0) {
+        if ((prm->flags & ECASQ_TEST_SELF_SEED) && L.costs_bytes && !L.gpairs_bytes &&
+            !(prm->flags & (ECASQ_DP_REFERENCE | ECASQ_UNSEEDED_SEARCH))) {
+            rc = run({prm->lambda});
+            if (rc) return rc;
+            rc = save_dp_seed(ws, L, p, 1, s, 0, st);
+            if (rc) return rc;
+            seed_lam = prm->lambda;
+        }
         rc = run({prm->lambda});
         if (rc) return rc;
-        sel = &evals[0];
+        sel = &evals.back();
     } else {
         double lo = prm->lambda_lo > 0.0 ? prm->lambda_lo : 1e-8;
         double hi = prm->lambda_hi > 0.0 ? prm->lambda_hi : 1e3;

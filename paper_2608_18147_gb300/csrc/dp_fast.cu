@@ -676,11 +676,6 @@ __device__ __forceinline__ void cons_reset(ConsStateT<LP> &cs) {
         for (int q = 0; q < JPT; q++) { cs.best[l][q] = CUDART_INF_F; cs.w1[l][q] = 0u; cs.w2[l][q] = 0u; }
 }
 
-// A band word with no run yet (a seeded running minimum, below): the first tile that
-// joins the band opens run 2 (run 1 cannot extend: its end + 1 is 2^16, above every K),
-// and diag_pair_bands moves run 2 into run 1 when run 1 was never set.
-constexpr uint32_t kNoRun = 0xFFFFFFFFu;
-
 // Seeded running minima of block J.  Every fp32 candidate is monotone in lambda' (C and
 // Phi are >= 0 and the roundings are monotone), so by induction over the layers an
 // earlier pass's fp32 minimum at a multiplier >= this one's bounds this pass's minimum
@@ -689,8 +684,10 @@ constexpr uint32_t kNoRun = 0xFFFFFFFFu;
 // minimum is m itself; a tile the tighter limit skips has every candidate above
 // m (1 + tau), outside the band; and band_fold keeps the band a superset of the tiles
 // with a candidate within m (1 + tau) from any starting bb >= m (a reset drops only
-// tiles whose candidates all lie above the band).  Only the skip tests see the seed:
-// more tiles are skipped, the tables are unchanged.
+// tiles whose candidates all lie above the band).  The band words keep their reset
+// state, run 1 = tile 0: a seeded output whose walk never resets its band keeps tile 0
+// in it (a superset again; a run opened at tile 0 could not be told from no run).
+// Only the skip tests see the seed: more tiles are skipped, the tables are unchanged.
 template <int LP>
 __device__ __forceinline__ void cons_seed(const FastArgs &a, ConsStateT<LP> &cs, int J, const ConsId &id) {
     const float *sr = a.seed + (size_t)J * (size_t)(a.s + 1) * BJ;
@@ -702,7 +699,7 @@ __device__ __forceinline__ void cons_seed(const FastArgs &a, ConsStateT<LP> &cs,
         for (int q = 0; q < JPT; q++) {
             const int jl = id.jq + NJQ * q;
             const float v = ((int64_t)J * BJ + jl < a.p) ? sr[(size_t)i * BJ + jl] : CUDART_INF_F;
-            if (v < CUDART_INF_F) { cs.best[l][q] = v; cs.w1[l][q] = kNoRun; }
+            if (v < CUDART_INF_F) cs.best[l][q] = v;
         }
     }
 }
@@ -876,13 +873,7 @@ __device__ __forceinline__ void cons_diag(const FastArgs &a, Smem &S, int b, int
                     S.diag[cur ^ 1][id.gl][jl] = bb;
                     if (j < a.p) {
                         a.dp32[d32(a, g, i, j)] = bb;
-                        // kNoRun: seeded, run 2 only (seeds come with tile skipping, which with LPT
-                        // layers per thread runs on the paired diagonal, not here)
-                        const uint32_t w1 = cs.w1[lx][q], w2 = cs.w2[lx][q];
-                        if constexpr (LP != LPT)
-                            a.band[oidx(a, g, i, j)] = w1 == kNoRun ? band_pack(w2, 0u) : band_pack(w1, w2);
-                        else
-                            a.band[oidx(a, g, i, j)] = band_pack(w1, w2);
+                        a.band[oidx(a, g, i, j)] = band_pack(cs.w1[lx][q], cs.w2[lx][q]);
                     }
                 }
             }
@@ -1150,8 +1141,7 @@ __device__ __forceinline__ void diag_pair_bands(const FastArgs &a, const uint32_
         for (int q = 0; q < JPT; q++) {
             const int64_t j = j0 + id.jq + NJQ * q;
             const int x = (l * JPT + q) * nc + ct;
-            uint32_t w1 = park[NS * nc + x], w2 = park[2 * NS * nc + x];
-            if (w1 == kNoRun) { w1 = w2; w2 = 0u; }  // seeded: the band's only run was opened as run 2
+            const uint32_t w1 = park[NS * nc + x], w2 = park[2 * NS * nc + x];
             if (i <= a.s && j < a.p) a.band[oidx(a, g, i, j)] = band_pack(w1, w2);
         }
     }
@@ -2235,7 +2225,7 @@ int save_dp_seed(void *ws, const Layout &Lw, int64_t p, int G, int s, int g, cud
 
 static size_t smem_bytes(int Gc, int s) { return sizeof(Smem) + (size_t)2 * Gc * (s - 2) * BK * sizeof(float); }
 
-// Certified band factors (see the file header): eps_2 = 1.0001u, eps_i = max(eps_{i-1}, 20u) + 1.0001u.
+// Certified band factors (see the file header): eps_2 = 1.0001u, eps_i = max(eps_{i-1}, 24u) + 1.0001u.
 static void band_factors(int s, FastParams &fp) {
     const double u = 1.0 / 16777216.0;
     for (int i = 0; i <= kMaxS; i++) { fp.tau[i] = 0.f; fp.eps[i] = 0.f; }
@@ -2291,17 +2281,23 @@ int launch_dp_fast(const Prefix &P, const double *lamp, int G, int s, void *ws, 
     a.G = G;
     a.s = s;
     // Layers per consumer thread: LPT, or 8 on the generic path (the fused kernel, or the
-    // resident one without tile skipping) when that costs fewer layer slots times
+    // resident one without the paired diagonal) when that costs fewer layer slots times
     // multiplier splits; at s = 32, 4 groups of 8 layers (64 threads per multiplier, 4
     // multipliers per split) against 5 of 7 (80 threads, 3 per split): 2 splits of 8
-    // slots per pass instead of 3 of 7.
+    // slots per pass instead of 3 of 7.  With resident or streamed costs, also when 8
+    // layers give an even number of layer groups and LPT an odd one or more than two:
+    // only then can the generic path skip tiles (s = 17, 18; s = 27..30 with several
+    // multipliers, where the slots favour LPT).  A single multiplier at s = 27..34 keeps
+    // LPT: with one warp pair per block the skipping did not pay for the eighth layer.
     int lp = LPT;
     if (!(costs && cdiv(s - 2, LPT) == 2 && mdp_stride(s) <= 20)) {
         auto slots = [&](int l) {
             const int lgc = (int)cdiv(s - 2, l), gc = std::max(1, std::min(G, MAXCONS / (lgc * NJQ)));
             return (int64_t)cdiv(G, gc) * l;
         };
-        if (cdiv(s - 2, 8) * NJQ <= MAXCONS && slots(8) < slots(LPT)) lp = 8;
+        const int lg8 = (int)cdiv(s - 2, 8);
+        const bool skip8 = costs && lg8 % 2 == 0 && mdp_stride(s) <= kMdpMax && (lg8 == 2 || G > 1);
+        if (cdiv(s - 2, 8) * NJQ <= MAXCONS && (skip8 || slots(8) < slots(LPT))) lp = 8;
     }
     a.lgc = (int)cdiv(s - 2, lp);
     a.Gc = std::max(1, std::min(G, MAXCONS / (a.lgc * NJQ)));

@@ -21,6 +21,7 @@ EXACT_S, NO_REFINE_GUARD, DP_REFERENCE, TIME_KERNELS, EXACT_TABLES, RESIDENT_COS
 ONE_PART_PUBLISH = 128  # fast DP: publish every column block once (no two-part publish)
 UNSEEDED_SEARCH = 256  # fast DP search: no seeded tile skipping (same results)
 TEST_STALL = 1 << 30  # test hook of the bounded waits (include/ecasq.h)
+TEST_SELF_SEED = 1 << 29  # test hook: a fixed-multiplier pass seeded with its own fp32 minima (same results)
 
 _lock = threading.Lock()
 _lib = None

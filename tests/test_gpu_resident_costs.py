@@ -308,3 +308,43 @@ def test_seeded_search_bit_identical_to_unseeded(E, name, s, b, mode):
     assert stu["tiles_skipped"] > 0  # tile skipping runs at every s here (even layer groups)
     if name == "studentt16k":  # five seeded passes at multipliers where most tiles are skipped
         assert sts["tiles_run"] < 0.95 * stu["tiles_run"]
+
+
+@pytest.mark.parametrize("lam", [0.0, 0.05])
+@pytest.mark.parametrize("name,s,mode", [("studentt16k", 16, "RESIDENT_COSTS"),
+                                         ("lognormal16k", 16, "RESIDENT_COSTS"),
+                                         ("mixture12k", 17, "RESIDENT_COSTS"),  # 8 layers per thread
+                                         ("ragged5000", 18, "STREAMED_COSTS")])  # 8 layers per thread
+def test_self_seeded_pass_bit_identical(E, name, s, mode, lam):
+    """A fixed-multiplier pass seeded with its own fp32 minima: every running minimum
+    starts at the output's final value, the tightest seed that the monotonicity of the
+    candidates in lambda' (Sec. 5) allows, so the seeded band starts with no run and
+    tiles within the band join it without a reset (a walk whose band started empty
+    once dropped a tile 0 that joined it first).  Same codebook, metrics and exact
+    tables as the plain pass, no certificate violation, and fewer tiles walked."""
+    x = {"studentt16k": lambda: workloads.student_t(16384, 0),
+         "lognormal16k": lambda: workloads.signed_lognormal(16384, 0),
+         "mixture12k": lambda: workloads.mixture(12288, 2),
+         "ragged5000": lambda: workloads.student_t(5000, 6, scale=1.0)}[name]()
+    cost = getattr(E, mode)
+    out = {}
+    for extra in (0, E.TEST_SELF_SEED):
+        ws = E.workspace(x.size, s, flags=cost)
+        Q, res = E.ecasq_solve(x, s, lambda_=lam, refine_max_rounds=0, flags=cost | E.EXACT_TABLES | extra, ws=ws)
+        st = E.native.ws_status(ws)
+        assert st["timeout"] == 0 and st["bound_viol"] == 0
+        out[extra] = (Q.cpu().numpy(), res, st, _tables(E, ws, 1, s, x.size))
+        del ws
+        _free()
+    (Q0, r0, st0, t0), (Q1, r1, st1, t1) = out[0], out[E.TEST_SELF_SEED]
+    assert r1["passes"] == r0["passes"] + 1
+    np.testing.assert_array_equal(Q0, Q1)
+    for k in ("lambda", "m", "mse", "h_exact", "h_surrogate", "status"):
+        assert r0[k] == r1[k], k
+    (dp0, bp0), (dp1, bp1) = t0[0], t1[0]
+    np.testing.assert_array_equal(dp0, dp1)
+    np.testing.assert_array_equal(bp0, bp1)
+    # the counters add up over a call's passes: the seeded pass is the second one
+    assert st1["tiles_run"] <= 2 * st0["tiles_run"]
+    assert st0["tiles_skipped"] > 0  # 8 layers per thread at s = 17 and 18: tile skipping with one multiplier
+    assert st1["tiles_run"] - st0["tiles_run"] < st0["tiles_run"]
