@@ -55,7 +55,7 @@ BK = BJ = 64              # the kernel's tile: 64 k by 64 columns
 # 34 816 B of C and Phi, plus the dp32 rows and minima that miss L2), from the committed
 # ncu capture of every launch of one solve at d = 16384; the benchmark launch is scaled
 # by the tiles it fetched (tile skipping leaves most tiles in HBM unread).
-TRAFFIC_PER_FETCHED_TILE = (6113806592 + 34871552) / 172536  # 6 launches of one solve: read + write / tiles
+TRAFFIC_PER_FETCHED_TILE = (6115167744 + 34815232) / 172545  # 6 launches of one solve: read + write / tiles
 ORACLE_SAMPLE = 16384     # entries of the CPU baseline's bounded sample
 
 
