@@ -213,7 +213,7 @@ def ecasq_solve(x, s, budget_bits=0.0, lambda_=-1.0, ws=None, **kw):
     if ws is None:
         ws = workspace(d, s, flags=kw.get("flags", 0))
     prm = make_params(s, budget_bits, lambda_, **kw)
-    Q = torch.empty(s, dtype=torch.float32, device="cuda")  # the call writes Q[:m]
+    Q = torch.zeros(s, dtype=torch.float32, device="cuda")
     res = Result()
     rc = lib().ecasq_solve(_ptr(x), d, C.byref(prm), _ptr(ws), ws.numel(), _ptr(Q), C.byref(res), _stream())
     _check(rc, "ecasq_solve", ok=(OK, EINFEASIBLE))
