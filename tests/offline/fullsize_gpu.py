@@ -2,7 +2,7 @@
 pass at the multiplier it selected with every DP output resolved exactly, written out for
 the oracle half (fullsize_oracle.py) to compare with the oracle's own DP.
 
-    python tests/offline/fullsize_gpu.py studentt_d131072_s16 mixture_d1048576_s32 --out gpurun_out/fullsize
+    python tests/offline/fullsize_gpu.py studentt_d131072_s16 mixture_d1048576_s32 --out fullsize_out
 
 For each workload it writes <name>.json (the solve: multiplier, codebook, metrics, timings)
 and <name>.npz (the exactly resolved dp / bp tables of that pass: every output when they fit
@@ -110,7 +110,7 @@ def run(name, out_dir, max_mb):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("workloads", nargs="+")
-    ap.add_argument("--out", default="gpurun_out/fullsize")
+    ap.add_argument("--out", default="fullsize_out")
     ap.add_argument("--max-mb", type=float, default=24.0)
     args = ap.parse_args()
     os.makedirs(args.out, exist_ok=True)

@@ -2,7 +2,7 @@
 apx_rec, apx_final) at the multiplier the GPU's budgeted solve selected, over the whole
 input, compared with what fullsize_gpu.py wrote.
 
-    python tests/offline/fullsize_oracle.py gpurun_out/fullsize/studentt_d131072_s16.json
+    python tests/offline/fullsize_oracle.py fullsize_out/studentt_d131072_s16.json
 
 The oracle runs or_apx_dp_columns (each pair's link cost computed once for all layers;
 the same tables as or_apx_dp) on this host's OpenMP threads.  Checks, with the parity
