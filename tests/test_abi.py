@@ -117,3 +117,24 @@ def test_quantize_wrappers_refuse_host_output_buffers():
         with pytest.raises(native.EcasqError) as ei:
             native.ecasq_quantize_noalloc(x, Q, 0, idx, cnt)
         assert ei.value.code == native.EINVAL
+
+
+def test_binding_constants_match_the_header():
+    """Every ECASQ_* flag and status code the header defines has the same value in the
+    binding (native.py restates them for ctypes callers)."""
+    from paper_2608_18147_gb300 import native
+    with open(os.path.join(ROOT, "include", "ecasq.h")) as f:
+        txt = f.read()
+    defs = {}
+    for name, val in re.findall(r"^#define\s+ECASQ_([A-Z0-9_]+)\s+([-()0-9u <]+?)\s*(?:/\*|$)", txt, re.M):
+        expr = re.sub(r"(\d)u\b", r"\1", val)  # 1u << 30, (-1), 256u
+        assert re.fullmatch(r"[-()0-9 <]+", expr), (name, val)
+        defs[name] = eval(expr, {"__builtins__": {}})
+    codes = {"OK", "EINVAL", "ENONFINITE", "EINFEASIBLE", "EWORKSPACE", "ECUDA", "ETIMEOUT", "ERANGE"}
+    flags = {"EXACT_S", "NO_REFINE_GUARD", "DP_REFERENCE", "TIME_KERNELS", "EXACT_TABLES", "RESIDENT_COSTS",
+             "STREAMED_COSTS", "ONE_PART_PUBLISH", "UNSEEDED_SEARCH", "TEST_STALL", "TEST_SELF_SEED"}
+    for name in codes | flags:
+        assert name in defs, name
+        assert getattr(native, name) == defs[name], (name, getattr(native, name), defs[name])
+    assert len({defs[n] for n in flags}) == len(flags)  # distinct bits
+    assert all(bin(defs[n]).count("1") == 1 for n in flags)
