@@ -62,7 +62,7 @@ typedef struct CUstream_st *ecasq_stream_t; /* same type as cudaStream_t */
                                      of tiles, 2.3 MB x ceil(d / 64); ecasq_workspace_size_flags with this flag) and
                                      the wavefront runs band by band; rebuilt in every pass.  RESIDENT_COSTS wins
                                      when both are given.  Results are the same as with either other mode. */
-#define ECASQ_ONE_PART_PUBLISH 128u /* fast DP with resident or streamed costs and s <= 16: publish each column block
+#define ECASQ_ONE_PART_PUBLISH 128u /* fast DP with resident or streamed costs and 10 <= s <= 16: publish each column block
                                      of the wavefront once, after all its layers, instead of in two parts (rows 2..8
                                      after layer 8, then the rest); same results, for comparison */
 #define ECASQ_UNSEEDED_SEARCH 256u /* fast DP with resident or streamed costs and tile skipping (10 <= s <= 18, 27 <= s <= 34): in the
