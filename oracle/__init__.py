@@ -65,6 +65,7 @@ def _load():
             "or_phi": (dbl, [P, i64, i64, i32]),
             "or_apx_dp": (i32, [P, i32, dbl, i32, pd, pi32, pd, pi64, pi32, pd]),
             "or_apx_dp_columns": (i32, [P, i32, dbl, i32, pd, pi32, pd, pi64, pi32, pd]),
+            "or_apx_dp_columns_prefix": (i32, [P, i32, dbl, i64, pd, pi32, pd]),
             "or_apx_dp_linear": (i32, [P, i32, dbl, i32, pi64, pi32, pd]),
             "or_dp_decision": (None, [P, pd, i32, i64, dbl, pd, pi64, pd]),
             "or_dp_candidate": (dbl, [P, dbl, i64, i64, dbl, i32]),
@@ -190,6 +191,20 @@ class Hist:
         if tables:
             out.update(dp=dp.reshape(rows, p), bp=bp.reshape(rows, p), margin=mg.reshape(rows, p))
         return out
+
+    def apx_dp_columns_prefix(self, s, lam_prime, jend):
+        """The approximate DP's tables (dp, bp, margin; (s+1) x p) for the columns j < jend
+        only, evaluated column by column as apx_dp(columns=True) does; later columns are
+        left at +inf / -1 / +inf and no codebook is formed."""
+        p, rows = self.p, s + 1
+        dp = np.empty(rows * p, np.float64)
+        bp = np.empty(rows * p, np.int32)
+        mg = np.empty(rows * p, np.float64)
+        st = _load().or_apx_dp_columns_prefix(self._h, int(s), float(lam_prime), int(jend), _ptr(dp, C.c_double),
+                                              _ptr(bp, C.c_int32), _ptr(mg, C.c_double))
+        if st != OK:
+            raise OracleError(st, "or_apx_dp_columns_prefix")
+        return dict(dp=dp.reshape(rows, p), bp=bp.reshape(rows, p), margin=mg.reshape(rows, p))
 
     def apx_dp_linear(self, s, lam_prime, exact_s=False):
         """Linear-space traceback of the approximate DP (Sec. 5, Hirschberg's method):

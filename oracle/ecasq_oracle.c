@@ -24,7 +24,8 @@
  *   h, or_phi        Sec. 4 (h), Sec. 5 (Phi, Phi^first)
  *   or_apx_dp        Sec. 5, eqs. apx_base / apx_rec / apx_final
  *   or_apx_dp_columns the same DP evaluated column by column (each pair's link
- *                    cost computed once for all layers), for full-size checks
+ *                    cost computed once for all layers), for full-size checks;
+ *                    or_apx_dp_columns_prefix its tables for the first columns alone
  *   or_apx_dp_linear Sec. 5 (last paragraph): the codebook of the same DP in linear
  *                    space (forward and backward passes, split at a middle value)
  *   or_dp_decision,  one output / one candidate of eq. apx_rec (eq. apx_base with
@@ -463,6 +464,52 @@ int32_t or_apx_dp(const or_hist *H, int32_t s, double lam_prime, int32_t exact_s
     return OR_OK;
 }
 
+/* Columns 1 <= j < jend of the column-by-column DP into dp, bp, mg ((s+1) x p,
+ * preset to +inf / -1 / +inf): the base layer, then layers 3..s of each column in
+ * increasing j; W holds one column's link costs. */
+static void apx_columns_fill(const or_hist *H, int32_t s, double lam_prime, int64_t jend, double *dp, int32_t *bp,
+                             double *mg, double *W) {
+    int64_t p = H->p;
+    /* base layer: as or_apx_dp */
+    for (int64_t j = 1; j < jend; j++) {
+        double best = INFINITY;
+        int64_t arg = -1;
+        for (int64_t a = 0; a < H->nL && a < j; a++) {
+            double C, U, D;
+            pair_q(H, a, j, &C, &U, &D);
+            double c = C + lam_prime * phi_of(H, U, D, a);
+            if (c < best) { best = c; arg = a; }
+        }
+        dp[2 * (size_t)p + (size_t)j] = best;
+        bp[2 * (size_t)p + (size_t)j] = (int32_t)arg;
+    }
+    for (int64_t j = 1; j < jend; j++) {
+        if (s < 3) break;
+#pragma omp parallel for schedule(static)
+        for (int64_t k = 0; k < j; k++) {
+            double C, Phi;
+            cphi(H, k, j, &C, &Phi);
+            W[k] = C + lam_prime * Phi;
+        }
+        int32_t itop = s < (int32_t)(j + 1) ? s : (int32_t)(j + 1);  /* layers with j >= i - 1 */
+#pragma omp parallel for schedule(dynamic, 1)
+        for (int32_t i = 3; i <= itop; i++) {
+            const double *prev = dp + (size_t)(i - 1) * (size_t)p;
+            double best = INFINITY, second = INFINITY;
+            int64_t arg = -1;
+            for (int64_t k = i - 2; k < j; k++) {
+                double cand = prev[k] + W[k];
+                if (cand < best) { second = best; best = cand; arg = k; }
+                else if (cand < second) second = cand;
+            }
+            size_t o = (size_t)i * (size_t)p + (size_t)j;
+            dp[o] = best;
+            bp[o] = (int32_t)arg;
+            mg[o] = (best > 0.0) ? (second - best) / best : (second > best ? INFINITY : 0.0);
+        }
+    }
+}
+
 /* The same DP as or_apx_dp (same tables, same codebook), evaluated column by
  * column so that inputs far too large for the pair memo stay practical: for
  * each j, in increasing order, the link costs C[k, j] + lambda' Phi[k, j] of
@@ -490,44 +537,7 @@ int32_t or_apx_dp_columns(const or_hist *H, int32_t s, double lam_prime, int32_t
     double *W = (double *)malloc(sizeof(double) * (size_t)p);
     if (!dp || !bp || !mg || !W) { free(dp); free(bp); free(mg); free(W); return OR_ENOMEM; }
     for (size_t t = 0; t < rows * (size_t)p; t++) { dp[t] = INFINITY; bp[t] = -1; mg[t] = INFINITY; }
-    /* base layer: as or_apx_dp */
-    for (int64_t j = 1; j < p; j++) {
-        double best = INFINITY;
-        int64_t arg = -1;
-        for (int64_t a = 0; a < H->nL && a < j; a++) {
-            double C, U, D;
-            pair_q(H, a, j, &C, &U, &D);
-            double c = C + lam_prime * phi_of(H, U, D, a);
-            if (c < best) { best = c; arg = a; }
-        }
-        dp[2 * (size_t)p + (size_t)j] = best;
-        bp[2 * (size_t)p + (size_t)j] = (int32_t)arg;
-    }
-    for (int64_t j = 1; j < p; j++) {
-        if (s < 3) break;
-#pragma omp parallel for schedule(static)
-        for (int64_t k = 0; k < j; k++) {
-            double C, Phi;
-            cphi(H, k, j, &C, &Phi);
-            W[k] = C + lam_prime * Phi;
-        }
-        int32_t itop = s < (int32_t)(j + 1) ? s : (int32_t)(j + 1);  /* layers with j >= i - 1 */
-#pragma omp parallel for schedule(dynamic, 1)
-        for (int32_t i = 3; i <= itop; i++) {
-            const double *prev = dp + (size_t)(i - 1) * (size_t)p;
-            double best = INFINITY, second = INFINITY;
-            int64_t arg = -1;
-            for (int64_t k = i - 2; k < j; k++) {
-                double cand = prev[k] + W[k];
-                if (cand < best) { second = best; best = cand; arg = k; }
-                else if (cand < second) second = cand;
-            }
-            size_t o = (size_t)i * (size_t)p + (size_t)j;
-            dp[o] = best;
-            bp[o] = (int32_t)arg;
-            mg[o] = (best > 0.0) ? (second - best) / best : (second > best ? INFINITY : 0.0);
-        }
-    }
+    apx_columns_fill(H, s, lam_prime, p, dp, bp, mg, W);
     free(W);
     int32_t istar = -1;
     int64_t jstar = -1;
@@ -552,6 +562,23 @@ int32_t or_apx_dp_columns(const or_hist *H, int32_t s, double lam_prime, int32_t
     if (bp_out) memcpy(bp_out, bp, sizeof(int32_t) * rows * (size_t)p);
     if (margin_out) memcpy(margin_out, mg, sizeof(double) * rows * (size_t)p);
     free(dp); free(bp); free(mg);
+    return OR_OK;
+}
+
+/* The tables of or_apx_dp_columns for the columns j < jend alone (0 < jend <= p):
+ * dp(i, j) reads only columns k < j, so these entries are the whole DP's.  For
+ * full-size checks whose whole DP would take too long; the codebook (eq. apx_final)
+ * needs every column and is not formed.  Entries of columns >= jend: +inf, -1, +inf. */
+int32_t or_apx_dp_columns_prefix(const or_hist *H, int32_t s, double lam_prime, int64_t jend, double *dp_out,
+                                 int32_t *bp_out, double *margin_out) {
+    int64_t p = H->p;
+    if (s < 2 || jend < 1 || jend > p || !dp_out || !bp_out || !margin_out) return OR_EINVAL;
+    size_t rows = (size_t)s + 1;
+    double *W = (double *)malloc(sizeof(double) * (size_t)p);
+    if (!W) return OR_ENOMEM;
+    for (size_t t = 0; t < rows * (size_t)p; t++) { dp_out[t] = INFINITY; bp_out[t] = -1; margin_out[t] = INFINITY; }
+    apx_columns_fill(H, s, lam_prime, jend, dp_out, bp_out, margin_out, W);
+    free(W);
     return OR_OK;
 }
 

@@ -226,3 +226,22 @@ def test_column_order_equals_layer_order(oracle_mod, name, x, s):
                     assert np.array_equal(a["dp"], b["dp"])
                     assert np.array_equal(a["bp"], b["bp"])
                     assert np.array_equal(a["margin"], b["margin"])
+
+
+@pytest.mark.parametrize("name,x", _inputs())
+@pytest.mark.parametrize("s", [3, 9, 16])
+def test_column_prefix_equals_the_whole_dp_on_its_columns(oracle_mod, name, x, s):
+    """or_apx_dp_columns_prefix (the column-by-column DP stopped before column jend) gives
+    or_apx_dp's tables bit for bit on every column j < jend, since dp(i, j) reads only
+    columns k < j (eq. apx_rec), and leaves the later columns unset."""
+    H = oracle_mod.Hist(x)
+    for lam in (0.0, 0.05):
+        lp = lam * H.norm2
+        full = H.apx_dp(s, lp)
+        for jend in sorted({1, 2, max(1, H.p // 3), H.p}):
+            pr = H.apx_dp_columns_prefix(s, lp, jend)
+            for key in ("dp", "bp", "margin"):
+                assert np.array_equal(pr[key][:, :jend], full[key][:, :jend]), (key, jend)
+            assert np.isinf(pr["dp"][:, jend:]).all() and (pr["bp"][:, jend:] == -1).all()
+    with pytest.raises(oracle_mod.OracleError):
+        H.apx_dp_columns_prefix(s, 0.0, H.p + 1)
